@@ -1,0 +1,374 @@
+"""fp64 CPU oracle of the FL-GLM server block stack under client-batching.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path may import or run this
+module: only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` use it.  It shares no code with the CUDA
+library; the only shared module is ``synthetic`` (seeded inputs, no arithmetic of
+the method).
+
+What it computes (plain definitions, in the paper's order, float64 throughout):
+
+* §3.1 (Model Split): the server holds blocks 1..N-2 and maps the smashed data
+  h_0 of each client to h_{N-2} = Block_(1,N-2)(h_0); the client sends back the
+  gradient of its loss w.r.t. h_{N-2} and the server back-propagates it and updates
+  its own parameters (the split-learning protocol the introduction describes for
+  FedBERT, which FL-GLM keeps).
+* §3.3 (Parallel Acceleration, client-batch): the M clients' {seqlength, batch,
+  hidden} tensors are stacked into one server batch.  Stacking is not averaging,
+  so each client row is an independent causal segment: packed results equal the
+  per-client results (the batching invariant tested on this module).
+* The block internals are not printed in the paper (§3.1 only says each block is
+  a transformer layer of multi-head self-attention and an FFN; §4.1.4 gives 28
+  layers, hidden 4096, 32 heads).  The reading taken is the ChatGLM-6B block:
+      a = LN1(x); qkv = a Wqkv^T + bqkv; q,k <- RoPE; o = causal softmax(q k^T/sqrt(d_h)) v
+      h = alpha * a + (o Wd^T + bd)        (residual_from_ln = 1; alpha*x with 0)
+      m = LN2(h); y = alpha * m + (gelu(m W1^T + b1) W2^T + b2)   (alpha*h with 0)
+  with the softmax scale 1/sqrt(d_h) of App. A (P-tuning v2 equations).
+* The optimizer of §4.1.4 (Adam, without weight decay) in the decoupled AdamW form
+  with bias correction; the decay rate is a parameter that defaults to 0.
+
+The backward is the exact chain rule of the forward, written out by hand.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass
+from typing import List, Optional, Sequence, Tuple
+
+import numpy as np
+
+import synthetic as syn
+
+F64 = np.float64
+
+# ----------------------------------------------------------------------------- packing
+# §3.3 client-batch: each client sends {seqlength, batch, hidden}; the server stacks them.
+
+
+@dataclass
+class Packing:
+    cu_seqlens: np.ndarray   # int32 [S + 1], segment s = tokens [cu[s], cu[s+1])
+    pos: np.ndarray          # int32 [T], position of each token inside its own segment
+    seg_client: np.ndarray   # int32 [S], client that owns segment s
+    seg_row: np.ndarray      # int32 [S], row of that client's batch
+
+    @property
+    def T(self) -> int:
+        return int(self.cu_seqlens[-1])
+
+    @property
+    def S(self) -> int:
+        return len(self.cu_seqlens) - 1
+
+
+def make_packing(seq_lens: Sequence[int], client_batch: int) -> Packing:
+    """Segments in client-major, then row-major order: client k row r is segment k*b + r."""
+    cu = [0]
+    pos, segc, segr = [], [], []
+    for k, L in enumerate(seq_lens):
+        for r in range(client_batch):
+            cu.append(cu[-1] + L)
+            pos.extend(range(L))
+            segc.append(k)
+            segr.append(r)
+    return Packing(np.array(cu, np.int32), np.array(pos, np.int32),
+                   np.array(segc, np.int32), np.array(segr, np.int32))
+
+
+def pack(client_tensors: Sequence[np.ndarray]) -> np.ndarray:
+    """Concatenate K tensors [b, L_k, H] into X[T, H] (segment = one client row)."""
+    H = client_tensors[0].shape[-1]
+    return np.concatenate([t.reshape(-1, H) for t in client_tensors], axis=0)
+
+
+def unpack(X: np.ndarray, seq_lens: Sequence[int], client_batch: int) -> List[np.ndarray]:
+    out, t0 = [], 0
+    H = X.shape[-1]
+    for L in seq_lens:
+        n = client_batch * L
+        out.append(X[t0:t0 + n].reshape(client_batch, L, H))
+        t0 += n
+    return out
+
+
+# ----------------------------------------------------------------------------- LayerNorm
+
+
+def layer_norm_fwd(x: np.ndarray, gamma: np.ndarray, beta: np.ndarray, eps: float):
+    """Row LayerNorm with the biased variance over the hidden dim."""
+    mu = x.mean(axis=-1)
+    xc = x - mu[:, None]
+    var = (xc * xc).mean(axis=-1)
+    rstd = 1.0 / np.sqrt(var + eps)
+    xhat = xc * rstd[:, None]
+    return xhat * gamma[None, :] + beta[None, :], mu, rstd
+
+
+def layer_norm_bwd(dy: np.ndarray, x: np.ndarray, mu: np.ndarray, rstd: np.ndarray, gamma: np.ndarray):
+    """dx = rstd * (g - mean(g) - xhat * mean(g * xhat)), g = gamma * dy; dgamma, dbeta summed over rows."""
+    xhat = (x - mu[:, None]) * rstd[:, None]
+    g = dy * gamma[None, :]
+    dx = rstd[:, None] * (g - g.mean(axis=-1, keepdims=True) - xhat * (g * xhat).mean(axis=-1, keepdims=True))
+    dgamma = (dy * xhat).sum(axis=0)
+    dbeta = dy.sum(axis=0)
+    return dx, dgamma, dbeta
+
+
+# ----------------------------------------------------------------------------- RoPE
+
+
+def rope_cos_sin(pos: np.ndarray, rotary_dim: int, base: float):
+    """Angles p * base^(-2i/rotary_dim), i < rotary_dim/2, one per rotated pair."""
+    half = rotary_dim // 2
+    inv_freq = base ** (-(2.0 * np.arange(half, dtype=F64)) / rotary_dim)
+    ang = pos.astype(F64)[:, None] * inv_freq[None, :]
+    return np.cos(ang), np.sin(ang)
+
+
+def rope_rotate(x: np.ndarray, cos: np.ndarray, sin: np.ndarray, rotary_dim: int, inverse: bool = False):
+    """Rotate-half pairing (i, i + rotary_dim/2) inside dims [0, rotary_dim) of every head;
+    dims [rotary_dim, head_dim) pass through.  x: [T, nh, hd]."""
+    half = rotary_dim // 2
+    s = -sin if inverse else sin
+    c = cos[:, None, :]
+    s = s[:, None, :]
+    out = x.copy()
+    x1 = x[..., :half]
+    x2 = x[..., half:rotary_dim]
+    out[..., :half] = x1 * c - x2 * s
+    out[..., half:rotary_dim] = x2 * c + x1 * s
+    return out
+
+
+# ----------------------------------------------------------------------------- attention
+
+
+def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray):
+    """Per segment, per head: O = softmax(Q K^T / sqrt(d_h) + causal) V (App. A scale).
+    Returns O [T, nh, hd] and the row log-sum-exp LSE [nh, T] of the scaled scores."""
+    T, nh, hd = q.shape
+    scale = 1.0 / math.sqrt(hd)
+    o = np.zeros_like(q)
+    lse = np.zeros((nh, T), F64)
+    for s in range(len(cu_seqlens) - 1):
+        a, b = int(cu_seqlens[s]), int(cu_seqlens[s + 1])
+        L = b - a
+        if L == 0:
+            continue
+        causal = np.tril(np.ones((L, L), bool))
+        for h in range(nh):
+            S = (q[a:b, h] @ k[a:b, h].T) * scale
+            S = np.where(causal, S, -np.inf)
+            m = S.max(axis=-1)
+            P = np.exp(S - m[:, None])
+            l = P.sum(axis=-1)
+            P /= l[:, None]
+            o[a:b, h] = P @ v[a:b, h]
+            lse[h, a:b] = m + np.log(l)
+    return o, lse
+
+
+def attention_bwd(do: np.ndarray, q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray):
+    """Chain rule of attention_fwd: dV = P^T dO, dP = dO V^T, dS = P (dP - rowsum(dP P)),
+    dQ = dS K / sqrt(d_h), dK = dS^T Q / sqrt(d_h)."""
+    T, nh, hd = q.shape
+    scale = 1.0 / math.sqrt(hd)
+    dq = np.zeros_like(q)
+    dk = np.zeros_like(k)
+    dv = np.zeros_like(v)
+    for s in range(len(cu_seqlens) - 1):
+        a, b = int(cu_seqlens[s]), int(cu_seqlens[s + 1])
+        L = b - a
+        if L == 0:
+            continue
+        causal = np.tril(np.ones((L, L), bool))
+        for h in range(nh):
+            S = (q[a:b, h] @ k[a:b, h].T) * scale
+            S = np.where(causal, S, -np.inf)
+            P = np.exp(S - S.max(axis=-1, keepdims=True))
+            P /= P.sum(axis=-1, keepdims=True)
+            dP = do[a:b, h] @ v[a:b, h].T
+            dS = P * (dP - (dP * P).sum(axis=-1, keepdims=True))
+            dv[a:b, h] = P.T @ do[a:b, h]
+            dq[a:b, h] = (dS @ k[a:b, h]) * scale
+            dk[a:b, h] = (dS.T @ q[a:b, h]) * scale
+    return dq, dk, dv
+
+
+# ----------------------------------------------------------------------------- GeLU (tanh form)
+
+_C = math.sqrt(2.0 / math.pi)
+_A = 0.044715
+
+
+def gelu(u: np.ndarray) -> np.ndarray:
+    return 0.5 * u * (1.0 + np.tanh(_C * (u + _A * u ** 3)))
+
+
+def gelu_grad(u: np.ndarray) -> np.ndarray:
+    t = np.tanh(_C * (u + _A * u ** 3))
+    return 0.5 * (1.0 + t) + 0.5 * u * (1.0 - t * t) * _C * (1.0 + 3.0 * _A * u * u)
+
+
+# ----------------------------------------------------------------------------- one block
+
+
+@dataclass
+class BlockShape:
+    hidden: int
+    n_heads: int
+    head_dim: int
+    ffn_hidden: int
+    rotary_dim: int
+    rope_base: float
+    ln_eps: float
+    alpha: float
+    residual_from_ln: int
+
+    @staticmethod
+    def of(cfg: syn.ServerConfig) -> "BlockShape":
+        return BlockShape(cfg.hidden, cfg.n_heads, cfg.head_dim, cfg.ffn_hidden, cfg.rdim,
+                          cfg.rope_base, cfg.ln_eps, cfg.residual_alpha, cfg.residual_from_ln)
+
+
+def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShape):
+    """One server block over the packed tokens x [T, H]; returns y and the saved values."""
+    Wqkv, bqkv, Wd, bd, W1, b1, W2, b2, g1, be1, g2, be2 = P
+    T, H = x.shape
+    nh, hd = sh.n_heads, sh.head_dim
+    a, mu1, rs1 = layer_norm_fwd(x, g1, be1, sh.ln_eps)
+    qkv = a @ Wqkv.T + bqkv[None, :]                         # [T, 3H]: q | k | v, each [nh, hd]
+    q = qkv[:, 0:H].reshape(T, nh, hd)
+    k = qkv[:, H:2 * H].reshape(T, nh, hd)
+    v = qkv[:, 2 * H:3 * H].reshape(T, nh, hd)
+    cos, sin = rope_cos_sin(pk.pos, sh.rotary_dim, sh.rope_base)
+    qr = rope_rotate(q, cos, sin, sh.rotary_dim)
+    kr = rope_rotate(k, cos, sin, sh.rotary_dim)
+    o, lse = attention_fwd(qr, kr, v, pk.cu_seqlens)
+    o = o.reshape(T, H)
+    res1 = a if sh.residual_from_ln else x
+    h = sh.alpha * res1 + (o @ Wd.T + bd[None, :])
+    m, mu2, rs2 = layer_norm_fwd(h, g2, be2, sh.ln_eps)
+    u = m @ W1.T + b1[None, :]
+    g = gelu(u)
+    res2 = m if sh.residual_from_ln else h
+    y = sh.alpha * res2 + (g @ W2.T + b2[None, :])
+    saved = dict(x=x, a=a, mu1=mu1, rs1=rs1, qr=qr, kr=kr, v=v, o=o, lse=lse, h=h, m=m,
+                 mu2=mu2, rs2=rs2, u=u, g=g, cos=cos, sin=sin)
+    return y, saved
+
+
+def block_bwd(P: Sequence[np.ndarray], sv: dict, dy: np.ndarray, pk: Packing, sh: BlockShape):
+    """Exact chain rule of block_fwd.  Returns dx and the 12 parameter gradients (summed over T)."""
+    Wqkv, bqkv, Wd, bd, W1, b1, W2, b2, g1, be1, g2, be2 = P
+    T, H = dy.shape
+    nh, hd = sh.n_heads, sh.head_dim
+    al = sh.alpha
+    # FFN down: y = alpha*res2 + g W2^T + b2
+    dW2 = dy.T @ sv["g"]
+    db2 = dy.sum(axis=0)
+    dg = dy @ W2
+    du = dg * gelu_grad(sv["u"])
+    dW1 = du.T @ sv["m"]
+    db1 = du.sum(axis=0)
+    dm = du @ W1
+    if sh.residual_from_ln:
+        dm = dm + al * dy
+    dh, dg2, dbe2 = layer_norm_bwd(dm, sv["h"], sv["mu2"], sv["rs2"], g2)
+    if not sh.residual_from_ln:
+        dh = dh + al * dy
+    # attention output projection: h = alpha*res1 + o Wd^T + bd
+    dWd = dh.T @ sv["o"]
+    dbd = dh.sum(axis=0)
+    do = (dh @ Wd).reshape(T, nh, hd)
+    dqr, dkr, dv = attention_bwd(do, sv["qr"], sv["kr"], sv["v"], pk.cu_seqlens)
+    dq = rope_rotate(dqr, sv["cos"], sv["sin"], sh.rotary_dim, inverse=True)
+    dk = rope_rotate(dkr, sv["cos"], sv["sin"], sh.rotary_dim, inverse=True)
+    dqkv = np.concatenate([dq.reshape(T, H), dk.reshape(T, H), dv.reshape(T, H)], axis=1)
+    dWqkv = dqkv.T @ sv["a"]
+    dbqkv = dqkv.sum(axis=0)
+    da = dqkv @ Wqkv
+    if sh.residual_from_ln:
+        da = da + al * dh
+    dx, dg1, dbe1 = layer_norm_bwd(da, sv["x"], sv["mu1"], sv["rs1"], g1)
+    if not sh.residual_from_ln:
+        dx = dx + al * dh
+    return dx, [dWqkv, dbqkv, dWd, dbd, dW1, db1, dW2, db2, dg1, dbe1, dg2, dbe2]
+
+
+# ----------------------------------------------------------------------------- stack + server
+
+
+def stack_fwd(params: Sequence[Sequence[np.ndarray]], x: np.ndarray, pk: Packing, sh: BlockShape):
+    saved = []
+    for P in params:
+        x, sv = block_fwd(P, x, pk, sh)
+        saved.append(sv)
+    return x, saved
+
+
+def stack_bwd(params, saved, dy, pk: Packing, sh: BlockShape):
+    grads = [None] * len(params)
+    for b in range(len(params) - 1, -1, -1):
+        dy, grads[b] = block_bwd(params[b], saved[b], dy, pk, sh)
+    return dy, grads
+
+
+def adamw_update(w, g, m, v, t: int, lr: float, beta1: float, beta2: float, eps: float, wd: float):
+    """Decoupled-weight-decay Adam with bias correction (step t >= 1).  Returns new w, m, v."""
+    m = beta1 * m + (1.0 - beta1) * g
+    v = beta2 * v + (1.0 - beta2) * g * g
+    mhat = m / (1.0 - beta1 ** t)
+    vhat = v / (1.0 - beta2 ** t)
+    w = w - lr * (mhat / (np.sqrt(vhat) + eps) + wd * w)
+    return w, m, v
+
+
+class OracleServer:
+    """The server's protocol on the oracle: forward(client states) -> output states,
+    backward(output-state grads) -> input-state grads (+ accumulated weight grads),
+    step(lr) -> AdamW update that clears the grads."""
+
+    def __init__(self, cfg: syn.ServerConfig, params: Optional[List[List[np.ndarray]]] = None):
+        self.cfg = cfg
+        self.sh = BlockShape.of(cfg)
+        if params is None:
+            params = syn.init_params(cfg)
+        self.params = [[np.asarray(p, F64).copy() for p in blk] for blk in params]
+        self.grads = [[np.zeros_like(p) for p in blk] for blk in self.params]
+        self.m = [[np.zeros_like(p) for p in blk] for blk in self.params]
+        self.v = [[np.zeros_like(p) for p in blk] for blk in self.params]
+        self.t = 0
+        self._pending = None
+
+    def forward(self, client_states: Sequence[np.ndarray]) -> List[np.ndarray]:
+        seq_lens = [s.shape[1] for s in client_states]
+        b = client_states[0].shape[0]
+        pk = make_packing(seq_lens, b)
+        X = pack([np.asarray(s, F64) for s in client_states])
+        Y, saved = stack_fwd(self.params, X, pk, self.sh)
+        self._pending = (seq_lens, b, pk, saved)
+        return unpack(Y, seq_lens, b)
+
+    def backward(self, grad_out: Sequence[np.ndarray]) -> List[np.ndarray]:
+        if self._pending is None:
+            raise RuntimeError("backward without a pending forward")
+        seq_lens, b, pk, saved = self._pending
+        dY = pack([np.asarray(g, F64) for g in grad_out])
+        dX, grads = stack_bwd(self.params, saved, dY, pk, self.sh)
+        for gb, acc in zip(grads, self.grads):
+            for i in range(12):
+                acc[i] += gb[i]
+        self._pending = None
+        return unpack(dX, seq_lens, b)
+
+    def step(self, lr: float):
+        c = self.cfg
+        self.t += 1
+        for bi in range(len(self.params)):
+            for i in range(12):
+                w, m, v = adamw_update(self.params[bi][i], self.grads[bi][i], self.m[bi][i], self.v[bi][i],
+                                       self.t, lr, c.adam_beta1, c.adam_beta2, c.adam_eps, c.weight_decay)
+                self.params[bi][i], self.m[bi][i], self.v[bi][i] = w, m, v
+                self.grads[bi][i] = np.zeros_like(w)
+

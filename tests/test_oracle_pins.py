@@ -1,0 +1,392 @@
+"""Pins of the fp64 oracle to facts other than itself (CPU only).
+
+Each pin is chosen so that a plausible slip in the oracle (a dropped term, a sign,
+a wrong index or operand order) fails at least one of them:
+
+* finite differences pin every backward formula against the forward;
+* library routines that special cases reduce to (torch's LayerNorm, causal SDPA,
+  tanh-GeLU and AdamW, all in float64) pin the forward primitives;
+* closed forms (zero-weight block, first AdamW step, single-token attention,
+  constant keys) and invariants (client-batching, causality, segment isolation,
+  RoPE norm and relative-position properties, LayerNorm row statistics) pin the
+  composition the paper fixes: §3.3 stacks clients without mixing them.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import synthetic as syn
+from oracle import flglm_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def tiny_cfg(residual_from_ln=1, n_blocks=2, seq_lens=(3, 5), b=1, alpha=2.0):
+    return syn.ServerConfig(name="fd", n_blocks=n_blocks, hidden=16, n_heads=2, head_dim=8,
+                            ffn_hidden=32, residual_alpha=alpha, client_batch=b, seq_lens=tuple(seq_lens),
+                            residual_from_ln=residual_from_ln)
+
+
+def random_params(cfg, rng, std=0.3):
+    """Large random weights and non-trivial LayerNorm affine parameters so that every
+    term of the block contributes measurably to the finite differences."""
+    out = []
+    for _ in range(cfg.n_blocks):
+        blk = []
+        for t, shp in enumerate(syn.param_shapes(cfg)):
+            if t in (syn.T_G1, syn.T_G2):
+                blk.append(1.0 + 0.3 * rng.standard_normal(shp))
+            elif t in (syn.T_BE1, syn.T_BE2):
+                blk.append(0.3 * rng.standard_normal(shp))
+            else:
+                blk.append(std * rng.standard_normal(shp))
+        out.append(blk)
+    return out
+
+
+def run_stack(cfg, params, X, pk):
+    sh = O.BlockShape.of(cfg)
+    return O.stack_fwd(params, X, pk, sh)
+
+
+def loss_and_grads(cfg, params, X, pk, dY):
+    sh = O.BlockShape.of(cfg)
+    Y, saved = O.stack_fwd(params, X, pk, sh)
+    dX, grads = O.stack_bwd(params, saved, dY, pk, sh)
+    return float((Y * dY).sum()), dX, grads
+
+
+# ----------------------------------------------------------------------------- generator pins
+
+def test_splitmix64_published_vector():
+    vals = [int(l) for l in open(os.path.join(GOLDEN, "splitmix64_seed1234567.txt")) if l.strip() and not l.startswith("#")]
+    got = [int(v) for v in syn.raw_u64(1234567, 0, 5)]
+    assert got == vals
+
+
+def test_normal_stream_statistics_and_offsets():
+    key = syn.stream_key(0, syn.P_WEIGHTS, 3, 2)
+    z = syn.normal_f64(key, 200001, 0.0, 1.0)
+    assert abs(z.mean()) < 0.01 and abs(z.std() - 1.0) < 0.01
+    # counter-based: any window equals the slice of the full stream
+    for start, n in [(0, 7), (1, 6), (13, 100), (99999, 3)]:
+        np.testing.assert_array_equal(syn.normal_f64(key, n, 0.0, 1.0, start), z[start:start + n])
+
+
+def test_bf16_rounding_is_rne():
+    x = np.array([1.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -2.5, 1.0 + 2 ** -9, 3.0e38], np.float32)
+    got = syn.bf16_bits_to_f32(syn.f32_to_bf16_bits(x))
+    want = torch.tensor(x).to(torch.bfloat16).float().numpy()
+    np.testing.assert_array_equal(got, want)
+
+
+def test_ragged_lengths_range_and_seed():
+    L = syn.ragged_lengths(7, 16)
+    assert len(L) == 16 and all(64 <= l <= 1024 for l in L)
+    assert syn.CONFIGS["ragged26"].seq_lens == L
+    assert len(set(L)) > 8
+
+
+# ----------------------------------------------------------------------------- packing
+
+def test_pack_unpack_roundtrip_and_metadata():
+    rng = np.random.default_rng(1)
+    seq = (3, 1, 4)
+    b = 2
+    ts = [rng.standard_normal((b, L, 5)) for L in seq]
+    pk = O.make_packing(seq, b)
+    assert list(pk.cu_seqlens) == [0, 3, 6, 7, 8, 12, 16]
+    assert list(pk.pos) == [0, 1, 2, 0, 1, 2, 0, 0, 0, 1, 2, 3, 0, 1, 2, 3]
+    assert list(pk.seg_client) == [0, 0, 1, 1, 2, 2]
+    X = O.pack(ts)
+    np.testing.assert_array_equal(X[6], ts[1][0, 0])
+    np.testing.assert_array_equal(X[12:16], ts[2][1])
+    for a, c in zip(O.unpack(X, seq, b), ts):
+        np.testing.assert_array_equal(a, c)
+
+
+# ----------------------------------------------------------------------------- forward primitives vs library routines
+
+def test_layer_norm_matches_torch_and_row_stats():
+    rng = np.random.default_rng(2)
+    x = 3.0 * rng.standard_normal((7, 33)) + 1.5
+    g = rng.standard_normal(33)
+    be = rng.standard_normal(33)
+    y, mu, rs = O.layer_norm_fwd(x, g, be, 1e-5)
+    ref = torch.nn.functional.layer_norm(torch.tensor(x), (33,), torch.tensor(g), torch.tensor(be), 1e-5).numpy()
+    np.testing.assert_allclose(y, ref, rtol=0, atol=1e-12)
+    # gamma = 1, beta = 0: zero row mean, variance sigma^2 / (sigma^2 + eps)
+    y1, _, _ = O.layer_norm_fwd(x, np.ones(33), np.zeros(33), 1e-5)
+    assert np.abs(y1.mean(axis=1)).max() < 1e-12
+    var = x.var(axis=1)
+    np.testing.assert_allclose(y1.var(axis=1), var / (var + 1e-5), rtol=1e-12)
+
+
+def test_gelu_matches_torch_tanh_form():
+    u = np.linspace(-8, 8, 1001)
+    ref = torch.nn.functional.gelu(torch.tensor(u), approximate="tanh").numpy()
+    np.testing.assert_allclose(O.gelu(u), ref, rtol=0, atol=1e-14)
+    # derivative against torch autograd
+    tu = torch.tensor(u, requires_grad=True)
+    torch.nn.functional.gelu(tu, approximate="tanh").sum().backward()
+    np.testing.assert_allclose(O.gelu_grad(u), tu.grad.numpy(), rtol=0, atol=1e-13)
+
+
+def test_attention_matches_torch_sdpa_per_segment():
+    rng = np.random.default_rng(3)
+    seq = [5, 1, 9]
+    cu = np.cumsum([0] + seq).astype(np.int32)
+    T, nh, hd = cu[-1], 3, 8
+    q, k, v = (rng.standard_normal((T, nh, hd)) for _ in range(3))
+    o, lse = O.attention_fwd(q, k, v, cu)
+    for s in range(len(seq)):
+        a, b = cu[s], cu[s + 1]
+        tq = torch.tensor(q[a:b]).transpose(0, 1)
+        tk = torch.tensor(k[a:b]).transpose(0, 1)
+        tv = torch.tensor(v[a:b]).transpose(0, 1)
+        ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, is_causal=True).transpose(0, 1).numpy()
+        np.testing.assert_allclose(o[a:b], ref, rtol=0, atol=1e-12)
+        # LSE against torch.logsumexp of the masked, scaled scores
+        S = torch.einsum("hid,hjd->hij", tq, tk) / math.sqrt(hd)
+        S = S.masked_fill(~torch.ones(b - a, b - a, dtype=torch.bool).tril(), float("-inf"))
+        np.testing.assert_allclose(lse[:, a:b], torch.logsumexp(S, -1).numpy(), rtol=0, atol=1e-12)
+
+
+def test_attention_brute_force_global_mask():
+    """The packed form equals one dense softmax over all T keys with a block-diagonal
+    causal mask (brute force over the whole packed batch)."""
+    rng = np.random.default_rng(4)
+    seq = [4, 6, 2]
+    cu = np.cumsum([0] + seq).astype(np.int32)
+    T, nh, hd = cu[-1], 2, 4
+    q, k, v = (rng.standard_normal((T, nh, hd)) for _ in range(3))
+    o, _ = O.attention_fwd(q, k, v, cu)
+    seg = np.repeat(np.arange(len(seq)), seq)
+    for h in range(nh):
+        for t in range(T):
+            w = np.array([math.exp(float(q[t, h] @ k[u, h]) / math.sqrt(hd)) if (seg[u] == seg[t] and u <= t) else 0.0
+                          for u in range(T)])
+            np.testing.assert_allclose(o[t, h], (w[:, None] * v[:, h]).sum(0) / w.sum(), rtol=0, atol=1e-12)
+
+
+def test_attention_special_cases():
+    rng = np.random.default_rng(5)
+    # L = 1: output equals v exactly
+    q, k, v = (rng.standard_normal((1, 2, 8)) for _ in range(3))
+    o, lse = O.attention_fwd(q, k, v, np.array([0, 1], np.int32))
+    np.testing.assert_array_equal(o, v)
+    # all keys equal: every row is the running mean of v
+    L = 6
+    q = rng.standard_normal((L, 1, 4))
+    k = np.tile(rng.standard_normal((1, 1, 4)), (L, 1, 1))
+    v = rng.standard_normal((L, 1, 4))
+    o, _ = O.attention_fwd(q, k, v, np.array([0, L], np.int32))
+    want = np.cumsum(v[:, 0], axis=0) / np.arange(1, L + 1)[:, None]
+    np.testing.assert_allclose(o[:, 0], want, rtol=0, atol=1e-13)
+
+
+def test_rope_properties():
+    rng = np.random.default_rng(6)
+    hd, rd, base = 16, 8, 10000.0
+    pos = np.arange(12, dtype=np.int32)
+    cos, sin = O.rope_cos_sin(pos, rd, base)
+    x = rng.standard_normal((12, 2, hd))
+    xr = O.rope_rotate(x, cos, sin, rd)
+    # p = 0 is the identity; dims beyond the rotary dims pass through
+    np.testing.assert_array_equal(xr[0], x[0])
+    np.testing.assert_array_equal(xr[..., rd:], x[..., rd:])
+    # norm preserved; inverse undoes the rotation
+    np.testing.assert_allclose(np.linalg.norm(xr, axis=-1), np.linalg.norm(x, axis=-1), rtol=1e-13)
+    np.testing.assert_allclose(O.rope_rotate(xr, cos, sin, rd, inverse=True), x, atol=1e-13)
+    # complex-number form: pair (i, i + rd/2) is z = x_i + j x_{i+rd/2}, rotated by e^{j p theta_i}
+    theta = base ** (-2.0 * np.arange(rd // 2) / rd)
+    z = (x[..., :rd // 2] + 1j * x[..., rd // 2:rd]) * np.exp(1j * pos[:, None, None] * theta[None, None, :])
+    np.testing.assert_allclose(xr[..., :rd // 2], z.real, atol=1e-13)
+    np.testing.assert_allclose(xr[..., rd // 2:rd], z.imag, atol=1e-13)
+    # q . k depends only on the position difference
+    q = rng.standard_normal((1, 1, hd))
+    kk = rng.standard_normal((1, 1, hd))
+    def dot(p, pp):
+        c1, s1 = O.rope_cos_sin(np.array([p]), rd, base)
+        c2, s2 = O.rope_cos_sin(np.array([pp]), rd, base)
+        return float((O.rope_rotate(q, c1, s1, rd) * O.rope_rotate(kk, c2, s2, rd)).sum())
+    assert abs(dot(7, 3) - dot(11, 7)) < 1e-12
+    assert abs(dot(5, 0) - dot(9, 4)) < 1e-12
+
+
+# ----------------------------------------------------------------------------- block closed form
+
+@pytest.mark.parametrize("rfl", [1, 0])
+def test_zero_weight_block_closed_form(rfl):
+    cfg = tiny_cfg(residual_from_ln=rfl, n_blocks=1, seq_lens=(4, 3))
+    rng = np.random.default_rng(7)
+    P = [np.zeros(s) for s in syn.param_shapes(cfg)]
+    P[syn.T_G1][:] = 1.0
+    P[syn.T_G2][:] = 1.0
+    pk = O.make_packing(cfg.seq_lens, 1)
+    x = 2.0 * rng.standard_normal((pk.T, cfg.hidden)) + 0.5
+    y, _ = run_stack(cfg, [P], x, pk)
+    al, eps = cfg.residual_alpha, cfg.ln_eps
+
+    def ln(z):
+        zc = z - z.mean(1, keepdims=True)
+        return zc / np.sqrt((zc * zc).mean(1, keepdims=True) + eps)
+    if rfl:
+        want = al * ln(al * ln(x))
+    else:
+        want = al * al * x   # attention and FFN branches are exactly zero
+    np.testing.assert_allclose(y, want, rtol=1e-12, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------- finite differences
+
+@pytest.mark.parametrize("rfl", [1, 0])
+def test_finite_difference_gradients(rfl):
+    cfg = tiny_cfg(residual_from_ln=rfl, n_blocks=2, seq_lens=(3, 5), b=1)
+    rng = np.random.default_rng(10 + rfl)
+    params = random_params(cfg, rng)
+    pk = O.make_packing(cfg.seq_lens, cfg.client_batch)
+    X = rng.standard_normal((pk.T, cfg.hidden))
+    dY = rng.standard_normal((pk.T, cfg.hidden))
+    _, dX, grads = loss_and_grads(cfg, params, X, pk, dY)
+
+    def f(params_, X_):
+        Y, _ = run_stack(cfg, params_, X_, pk)
+        return float((Y * dY).sum())
+
+    h = 1e-5
+
+    def check(an, perturb, n_samples, idx_rng):
+        flat = an.reshape(-1)
+        scale = max(np.abs(flat).max(), 1e-8)
+        idx = idx_rng.choice(flat.size, size=min(n_samples, flat.size), replace=False)
+        for i in idx:
+            fp = perturb(i, +h)
+            fm = perturb(i, -h)
+            fd = (fp - fm) / (2 * h)
+            assert abs(fd - flat[i]) <= 1e-6 * scale, (i, fd, flat[i], scale)
+
+    irng = np.random.default_rng(99)
+
+    def pert_x(i, d):
+        Xp = X.copy()
+        Xp.reshape(-1)[i] += d
+        return f(params, Xp)
+    check(dX, pert_x, 60, irng)
+
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            def pert_p(i, d, b=b, t=t):
+                pp = [[p.copy() if (bb == b and tt == t) else p for tt, p in enumerate(blk)]
+                      for bb, blk in enumerate(params)]
+                pp[b][t].reshape(-1)[i] += d
+                return f(pp, X)
+            check(grads[b][t], pert_p, 25, irng)
+
+
+# ----------------------------------------------------------------------------- client-batching invariant
+
+@pytest.mark.parametrize("rfl", [1, 0])
+def test_client_batching_invariant(rfl):
+    """§3.3 stacks clients: packed results equal each client run alone; weight
+    gradients equal the sum of the per-client runs."""
+    cfg = tiny_cfg(residual_from_ln=rfl, n_blocks=2, seq_lens=(3, 7, 1), b=2)
+    rng = np.random.default_rng(20)
+    params = random_params(cfg, rng, std=0.2)
+    states = [rng.standard_normal((cfg.client_batch, L, cfg.hidden)) for L in cfg.seq_lens]
+    gouts = [rng.standard_normal((cfg.client_batch, L, cfg.hidden)) for L in cfg.seq_lens]
+    srv = O.OracleServer(cfg, params)
+    outs = srv.forward(states)
+    gins = srv.backward(gouts)
+    gsum = [[np.zeros_like(p) for p in blk] for blk in srv.params]
+    for k in range(cfg.K):
+        for r in range(cfg.client_batch):
+            c1 = cfg.with_(seq_lens=(cfg.seq_lens[k],), client_batch=1)
+            s1 = O.OracleServer(c1, params)
+            o1 = s1.forward([states[k][r:r + 1]])
+            g1 = s1.backward([gouts[k][r:r + 1]])
+            np.testing.assert_allclose(o1[0][0], outs[k][r], rtol=0, atol=1e-12)
+            np.testing.assert_allclose(g1[0][0], gins[k][r], rtol=0, atol=1e-12)
+            for b in range(cfg.n_blocks):
+                for t in range(12):
+                    gsum[b][t] += s1.grads[b][t]
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            np.testing.assert_allclose(srv.grads[b][t], gsum[b][t], rtol=1e-10, atol=1e-12)
+
+
+def test_causality_and_segment_isolation():
+    cfg = tiny_cfg(n_blocks=2, seq_lens=(6, 5), b=1)
+    rng = np.random.default_rng(21)
+    params = random_params(cfg, rng)
+    pk = O.make_packing(cfg.seq_lens, 1)
+    X = rng.standard_normal((pk.T, cfg.hidden))
+    Y, _ = run_stack(cfg, params, X, pk)
+    # a later token of the same segment
+    Xp = X.copy()
+    Xp[4] += 3.0 * rng.standard_normal(cfg.hidden)   # not a constant shift: LN would remove that
+    Yp, _ = run_stack(cfg, params, Xp, pk)
+    np.testing.assert_array_equal(Yp[:4], Y[:4])
+    assert np.abs(Yp[4:6] - Y[4:6]).max() > 1e-3
+    np.testing.assert_array_equal(Yp[6:], Y[6:])
+    # any token of the other segment
+    Xq = X.copy()
+    Xq[7] -= 2.0 * rng.standard_normal(cfg.hidden)
+    Yq, _ = run_stack(cfg, params, Xq, pk)
+    np.testing.assert_array_equal(Yq[:6], Y[:6])
+
+
+# ----------------------------------------------------------------------------- AdamW
+
+def test_adamw_first_step_closed_form():
+    rng = np.random.default_rng(30)
+    w = rng.standard_normal(1000)
+    g = rng.standard_normal(1000) * 1e-3
+    for wd in (0.0, 0.01):
+        w1, m1, v1 = O.adamw_update(w, g, np.zeros_like(w), np.zeros_like(w), 1, 1e-4, 0.9, 0.999, 1e-8, wd)
+        np.testing.assert_allclose(w1, w - 1e-4 * (g / (np.abs(g) + 1e-8) + wd * w), rtol=0, atol=1e-15)
+        np.testing.assert_allclose(m1, 0.1 * g, rtol=1e-14)
+        np.testing.assert_allclose(v1, 0.001 * g * g, rtol=1e-14)
+
+
+def test_adamw_matches_torch_over_steps():
+    rng = np.random.default_rng(31)
+    w0 = rng.standard_normal(257)
+    tw = torch.tensor(w0.copy(), requires_grad=True)
+    opt = torch.optim.AdamW([tw], lr=3e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=0.05)
+    w, m, v = w0.copy(), np.zeros(257), np.zeros(257)
+    for t in range(1, 6):
+        g = rng.standard_normal(257)
+        tw.grad = torch.tensor(g)
+        opt.step()
+        w, m, v = O.adamw_update(w, g, m, v, t, 3e-3, 0.9, 0.999, 1e-8, 0.05)
+        np.testing.assert_allclose(w, tw.detach().numpy(), rtol=0, atol=1e-13)
+
+
+def test_server_protocol_state_and_accumulation():
+    """forward/backward pairs without a step accumulate (serial mode, §3.3); step clears."""
+    cfg = tiny_cfg(n_blocks=1, seq_lens=(3, 2), b=1)
+    rng = np.random.default_rng(40)
+    params = random_params(cfg, rng, std=0.2)
+    st = [rng.standard_normal((1, L, cfg.hidden)) for L in cfg.seq_lens]
+    gr = [rng.standard_normal((1, L, cfg.hidden)) for L in cfg.seq_lens]
+    srv = O.OracleServer(cfg, params)
+    with pytest.raises(RuntimeError):
+        srv.backward(gr)
+    # serial: one client at a time, then one step
+    ser = O.OracleServer(cfg, params)
+    for k in range(cfg.K):
+        ser.forward([st[k]])
+        ser.backward([gr[k]])
+    srv.forward(st)
+    srv.backward(gr)
+    for t in range(12):
+        np.testing.assert_allclose(ser.grads[0][t], srv.grads[0][t], rtol=1e-10, atol=1e-12)
+    srv.step(1e-3)
+    assert all(not g.any() for g in srv.grads[0])
+    assert srv.t == 1
