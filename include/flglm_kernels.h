@@ -1,0 +1,115 @@
+/*
+ * flglm_kernels.h -- kernel-level C ABI of the FL-GLM server library.
+ *
+ * These entry points launch one hot-path kernel on caller-owned DEVICE buffers.
+ * The server calls in flglm.h are built from them; they are exported so that each
+ * kernel can be checked on its own against the oracle.  Every pointer is a device
+ * pointer unless its name ends in _host; every call is asynchronous on `stream`
+ * (a cudaStream_t, NULL = legacy default stream) unless stated.  Return codes are
+ * the FL_* codes of flglm.h; the message is in fl_server_last_error(NULL).
+ * `status` (optional, device int) receives a nonzero code if a bounded wait inside
+ * the kernel gave up; the kernel then returns without finishing its output.
+ */
+#ifndef FLGLM_KERNELS_H
+#define FLGLM_KERNELS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include "flglm.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* GEMM epilogues.  acc = sum_k A(m,k) B(n,k) in fp32 (tcgen05, TMEM accumulator). */
+enum {
+  FL_EPI_STORE = 0,      /* D = acc (+ bias[n] if bias)                                   bf16 */
+  FL_EPI_BIAS_GELU = 1,  /* U = acc + bias[n] -> aux_out;  D = gelu_tanh(U)               bf16 */
+  FL_EPI_BIAS_RESID = 2, /* D = acc + bias[n] + alpha * aux[m,n]                          bf16 */
+  FL_EPI_BIAS_ROPE = 3,  /* D = acc + bias[n]; columns [0, 2*n_heads*head_dim) (q and k) are
+                            then rotated: dims [0, rotary_dim) of each head, pairs
+                            (i, i + rotary_dim/2), angle pos[m] * rope_base^(-2i/rotary_dim)
+                            taken from rope_tab[pos[m]][i] = (cos, sin)                  bf16 */
+  FL_EPI_GELU_BWD = 4,   /* D = acc * gelu_tanh'(aux[m,n])   (aux = pre-activation U)     bf16 */
+  FL_EPI_RESID = 5,      /* D = acc + alpha * aux[m,n]                                    bf16 */
+  FL_EPI_ACCUM_F32 = 6,  /* D[m,n] += acc                                                 fp32 */
+  FL_EPI_COUNT
+};
+
+/* D[M,N] = epilogue(A . B^T) with bf16 operands.
+ * A(m,k) is A[m*lda + k] when a_mn_major == 0 (row-major [M,K]) and A[k*lda + m] when
+ * a_mn_major == 1 (row-major [K,M]); B(n,k) likewise with ldb / b_mn_major.
+ * Forward GEMMs are (0,0), data-gradient GEMMs (0,1), weight-gradient GEMMs (1,1).
+ * Requirements: N % 128 == 0; K % 8 == 0 when a or b is K-major; lda, ldb, ldd,
+ * ld_aux, ld_aux_out multiples of 8 elements; pointers 16-byte aligned.  M and K may
+ * be ragged (zero-filled by the tensor-memory-accelerator loads). */
+typedef struct {
+  int32_t M, N, K;
+  const void* A; int64_t lda; int32_t a_mn_major;
+  const void* B; int64_t ldb; int32_t b_mn_major;
+  void* D; int64_t ldd;
+  int32_t epilogue;
+  const float* bias;            /* [N] fp32 or NULL */
+  const void* aux; int64_t ld_aux;          /* bf16 [M,N] for BIAS_RESID / RESID / GELU_BWD */
+  float alpha;
+  void* aux_out; int64_t ld_aux_out;        /* bf16 [M,N] for BIAS_GELU */
+  const int32_t* pos;                       /* [M] positions for BIAS_ROPE */
+  const float* rope_tab;                    /* [max_pos][rotary_dim/2][2] for BIAS_ROPE */
+  int32_t n_heads, head_dim, rotary_dim;
+} fl_gemm_args;
+
+int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);
+
+/* Row LayerNorm, biased variance, fp32 statistics.  x, y: bf16 [T,H]; mean, rstd: [T]. */
+int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, const float* gamma, const float* beta,
+                       float eps, void* y, float* mean, float* rstd, void* stream);
+
+/* LayerNorm backward.  dy, x: bf16 [T,H]; dx = rstd (g - mean(g) - xhat mean(g xhat)),
+ * g = gamma dy, plus resid_alpha * resid[t,:] when resid != NULL (bf16 [T,H]).
+ * dgamma[H] += sum_t dy xhat and dbeta[H] += sum_t dy (fp32, accumulated).
+ * workspace: fp32 scratch of at least fl_k_layernorm_bwd_workspace(T, H) bytes. */
+size_t fl_k_layernorm_bwd_workspace(int32_t T, int32_t H);
+int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
+                       const float* rstd, const float* gamma, const void* resid, float resid_alpha,
+                       void* dx, float* dgamma, float* dbeta, void* workspace, void* stream);
+
+/* Varlen causal attention over packed segments (App. A scale 1/sqrt(head_dim)).
+ * qkv: bf16 [T, 3*H] (q | k | v, head j at column j*head_dim of each part, RoPE already
+ * applied); cu_seqlens_host / cu_seqlens: host and device copies of int32 [S+1].
+ * o: bf16 [T,H]; lse: fp32 [n_heads, T] (log-sum-exp of the scaled scores).
+ * tile_ws: device int32 scratch of at least fl_k_attention_tiles(cu_seqlens_host, S) * 2
+ * entries.  This call copies the tile list synchronously.  head_dim in {64, 128}. */
+int32_t fl_k_attention_tiles(const int32_t* cu_seqlens_host, int32_t S);
+int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv,
+                       const int32_t* cu_seqlens_host, const int32_t* cu_seqlens, int32_t S,
+                       int32_t* tile_ws, void* o, float* lse, void* stream);
+
+/* Attention backward: dqkv (bf16 [T, 3H]) receives dq | dk | dv.  When rope_tab != NULL
+ * the inverse rotation by each token's position inside its segment is applied to dq and
+ * dk (rotary_dim must be head_dim / 2), giving the gradient w.r.t. the un-rotated q, k.
+ * delta_ws: fp32 scratch [n_heads * T].  This call copies the tile list synchronously. */
+int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv, const void* o,
+                       const float* lse, const void* dout, const int32_t* cu_seqlens_host,
+                       const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,
+                       const float* rope_tab, int32_t rotary_dim, void* dqkv, void* stream);
+
+/* AdamW over n contiguous fp32 elements; bc1 = 1 - beta1^t, bc2 = 1 - beta2^t.
+ * w_bf16 (optional) receives the rounded new weights; g is zeroed. */
+int fl_k_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
+               float beta2, float eps, float weight_decay, float bc1, float bc2, void* stream);
+
+/* Client packing (§3.3 client-batch stacks the clients' tensors into one batch):
+ * gather copies client buffer k (bytes[k] bytes, a multiple of 16, 16-byte aligned)
+ * to packed + sum(bytes[0..k)); scatter copies the other way.  Bit-exact.
+ * clients_host is a host array of K device pointers; K <= 4096. */
+int fl_k_pack_clients(int32_t K, void* const* clients_host, const int64_t* bytes_host, void* packed, int32_t scatter,
+                      void* stream);
+
+/* out[n] += sum_t x[t, n] for bf16 x [T, N] (bias gradients), fp32 out. */
+int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FLGLM_KERNELS_H */

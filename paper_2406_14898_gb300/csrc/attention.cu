@@ -1,0 +1,684 @@
+// Varlen causal attention over packed client segments (App. A: softmax(Q K^T / sqrt(d_h)) V),
+// each client row attending only to earlier tokens of its own segment (§3.3 stacks
+// clients; it does not mix them).
+//
+// Forward: one CTA per (64-query tile, head); online softmax over 64-key tiles with
+// cp.async double buffering and bf16 mma.sync m16n8k16 (fp32 accumulate).  Saves O (bf16)
+// and the row log-sum-exp (fp32).
+// Backward, deterministic, no atomics:
+//   delta = rowsum(dO * O);
+//   dQ  kernel: per (query tile, head), loop over key tiles: P, dP = dO V^T, dS, dQ += dS K;
+//   dKV kernel: per (key tile, head), loop over query tiles: dV += P^T dO, dK += dS^T Q;
+// dQ and dK leave through the inverse rotary rotation (the forward rotation is applied in
+// the QKV GEMM epilogue), so the result is the gradient w.r.t. the un-rotated q and k.
+#include <cmath>
+#include <vector>
+
+#include "../../include/flglm_kernels.h"
+#include "common.cuh"
+#include "kernels.cuh"
+#include "ptx.cuh"
+
+namespace {
+
+typedef __nv_bfloat16 bf16;
+constexpr int BT = 64;  // rows per tile (queries or keys)
+constexpr float LOG2E = 1.4426950408889634f;
+constexpr float LN2 = 0.6931471805599453f;
+
+template <int HD>
+struct AT {
+  static constexpr int SROW = HD + 8;                 // padded smem row (elements)
+  static constexpr int TILE_ELEMS = BT * SROW;
+  static constexpr int TILE_BYTES = TILE_ELEMS * 2;
+};
+
+// 64 rows x HD columns from global (row stride ld elements) into padded smem; rows >= valid
+// are zero-filled without touching global memory.
+template <int HD>
+FL_DEV void load_tile(bf16* sdst, const bf16* g, int64_t ld, int valid, int tid) {
+  constexpr int CPR = HD / 8;  // 16-byte chunks per row
+  for (int c = tid; c < BT * CPR; c += 128) {
+    const int r = c / CPR, cc = c % CPR;
+    const bool ok = r < valid;
+    const bf16* src = ok ? g + (int64_t)r * ld + cc * 8 : g;
+    cp_async_16(smem_u32(sdst + r * AT<HD>::SROW + cc * 8), src, ok);
+  }
+}
+
+// A fragment (16 rows x 16 cols at row0, col0) of a row-major padded smem tile.
+template <int HD>
+FL_DEV void ld_a(const bf16* s, int row0, int col0, int lane, uint32_t (&a)[4]) {
+  const int r = row0 + (lane & 15);
+  const int c = col0 + ((lane >> 4) << 3);
+  ldmatrix_x4(smem_u32(s + r * AT<HD>::SROW + c), a[0], a[1], a[2], a[3]);
+}
+// B fragments of two adjacent n-tiles, B(k, n) = S[n][k] (rows of the tile are n):
+// n in [n0, n0+16), k in [k0, k0+16).  b[0..1] -> n-tile n0, b[2..3] -> n-tile n0+8.
+template <int HD>
+FL_DEV void ld_b_rows(const bf16* s, int n0, int k0, int lane, uint32_t (&b)[4]) {
+  const int j = lane >> 3;
+  const int r = n0 + (lane & 7) + ((j >> 1) << 3);
+  const int c = k0 + ((j & 1) << 3);
+  ldmatrix_x4(smem_u32(s + r * AT<HD>::SROW + c), b[0], b[1], b[2], b[3]);
+}
+// B fragments of two adjacent n-tiles, B(k, n) = S[k][n] (rows of the tile are k):
+// k in [k0, k0+16), n in [n0, n0+16).
+template <int HD>
+FL_DEV void ld_b_cols(const bf16* s, int k0, int n0, int lane, uint32_t (&b)[4]) {
+  const int j = lane >> 3;
+  const int r = k0 + (lane & 7) + ((j & 1) << 3);
+  const int c = n0 + ((j >> 1) << 3);
+  ldmatrix_x4_trans(smem_u32(s + r * AT<HD>::SROW + c), b[0], b[1], b[2], b[3]);
+}
+
+FL_DEV float quad_max(float v) {
+  v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
+  return fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+}
+FL_DEV float quad_sum(float v) {
+  v += __shfl_xor_sync(0xffffffffu, v, 1);
+  return v + __shfl_xor_sync(0xffffffffu, v, 2);
+}
+
+FL_DEV void decode_tile(uint32_t t, int& s, int& idx) {
+  s = int(t >> 16);
+  idx = int(t & 0xFFFFu);
+}
+
+// ---------------------------------------------------------------------------- forward
+template <int HD>
+__global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16* __restrict__ qkv,
+                                                       const int32_t* __restrict__ cu,
+                                                       const uint32_t* __restrict__ tiles, bf16* __restrict__ O,
+                                                       float* __restrict__ lse, float scale_log2) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  bf16* sQ = reinterpret_cast<bf16*>(smem);
+  bf16* sK = sQ + AT<HD>::TILE_ELEMS;      // [2] tiles
+  bf16* sV = sK + 2 * AT<HD>::TILE_ELEMS;  // [2] tiles
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  int s, idx;
+  decode_tile(tiles[blockIdx.x], s, idx);
+  const int h = blockIdx.y;
+  const int seg0 = cu[s], L = cu[s + 1] - seg0;
+  const int q0 = idx * BT;
+  const int64_t ld = 3 * (int64_t)H;
+  const bf16* gQ = qkv + (int64_t)(seg0 + q0) * ld + h * HD;
+  const bf16* gK = qkv + (int64_t)seg0 * ld + H + h * HD;
+  const bf16* gV = qkv + (int64_t)seg0 * ld + 2 * H + h * HD;
+
+  load_tile<HD>(sQ, gQ, ld, min(BT, L - q0), tid);
+  load_tile<HD>(sK, gK, ld, min(BT, L), tid);
+  load_tile<HD>(sV, gV, ld, min(BT, L), tid);
+  cp_async_commit();
+
+  float o[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
+  uint32_t qf[HD / 16][4];
+  const int n_kv = idx + 1;
+
+  for (int j = 0; j < n_kv; ++j) {
+    const int buf = j & 1;
+    if (j + 1 < n_kv) {
+      const int k1 = (j + 1) * BT;
+      load_tile<HD>(sK + (buf ^ 1) * AT<HD>::TILE_ELEMS, gK + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
+      load_tile<HD>(sV + (buf ^ 1) * AT<HD>::TILE_ELEMS, gV + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    if (j == 0) {
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) ld_a<HD>(sQ, warp * 16, kk * 16, lane, qf[kk]);
+    }
+    const bf16* K = sK + buf * AT<HD>::TILE_ELEMS;
+    const bf16* V = sV + buf * AT<HD>::TILE_ELEMS;
+    float sc[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+#pragma unroll
+      for (int np = 0; np < 4; ++np) {
+        uint32_t b[4];
+        ld_b_rows<HD>(K, np * 16, kk * 16, lane, b);
+        mma_bf16_16816(sc[2 * np], qf[kk], b[0], b[1]);
+        mma_bf16_16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
+      }
+    }
+    const bool diag = (j == idx);
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float x = sc[nt][e] * scale_log2;
+        if (diag) {
+          const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int ql = warp * 16 + (lane >> 2) + ((e >> 1) << 3);
+          if (kl > ql) x = -INFINITY;
+        }
+        sc[nt][e] = x;
+        mx[e >> 1] = fmaxf(mx[e >> 1], x);
+      }
+    }
+    float corr[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const float mn = fmaxf(mrow[r], quad_max(mx[r]));
+      corr[r] = exp2f(mrow[r] - mn);
+      mrow[r] = mn;
+      lrow[r] *= corr[r];
+    }
+#pragma unroll
+    for (int i = 0; i < HD / 8; ++i) {
+      o[i][0] *= corr[0]; o[i][1] *= corr[0];
+      o[i][2] *= corr[1]; o[i][3] *= corr[1];
+    }
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float p = exp2f(sc[nt][e] - mrow[e >> 1]);
+        sc[nt][e] = p;
+        lrow[e >> 1] += p;
+      }
+    }
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      uint32_t a[4];
+      a[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
+      a[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
+      a[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      a[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int np = 0; np < HD / 16; ++np) {
+        uint32_t b[4];
+        ld_b_cols<HD>(V, kk * 16, np * 16, lane, b);
+        mma_bf16_16816(o[2 * np], a, b[0], b[1]);
+        mma_bf16_16816(o[2 * np + 1], a, b[2], b[3]);
+      }
+    }
+    __syncthreads();
+  }
+
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const float lt = quad_sum(lrow[r]);
+    const float inv = 1.f / lt;
+    const int q = q0 + warp * 16 + (lane >> 2) + 8 * r;
+    if (q < L) {
+      bf16* orow = O + (int64_t)(seg0 + q) * H + h * HD + 2 * (lane & 3);
+#pragma unroll
+      for (int nt = 0; nt < HD / 8; ++nt)
+        *reinterpret_cast<uint32_t*>(orow + nt * 8) = pack_bf16x2(o[nt][2 * r] * inv, o[nt][2 * r + 1] * inv);
+      if ((lane & 3) == 0) lse[(int64_t)h * T + seg0 + q] = (mrow[r] + log2f(lt)) * LN2;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------- delta = rowsum(dO * O)
+__global__ void attn_delta_kernel(int T, int H, int nh, int hd, const bf16* __restrict__ O,
+                                  const bf16* __restrict__ dO, float* __restrict__ delta) {
+  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;  // (t, h) pair
+  const int lane = threadIdx.x & 31;
+  if (w >= (int64_t)T * nh) return;
+  const int t = int(w / nh), h = int(w % nh);
+  const bf16* o = O + (int64_t)t * H + h * hd;
+  const bf16* d = dO + (int64_t)t * H + h * hd;
+  float s = 0.f;
+  for (int i = 2 * lane; i < hd; i += 64) {
+    const float2 a = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(o + i));
+    const float2 b = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(d + i));
+    s += a.x * b.x + a.y * b.y;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  if (lane == 0) delta[(int64_t)h * T + t] = s;
+}
+
+// Inverse rotary rotation of an accumulator fragment: the thread holds, for n-tile nt,
+// dims 8 nt + 2 (lane & 3) + {0, 1} of row r (elements 2r, 2r+1).  The rotary dims are
+// [0, HD/2) (half of each head), so the partner of dim i < HD/4 is i + HD/4, which lives
+// in n-tile nt + HD/32 of the same thread.
+template <int HD>
+FL_DEV void inverse_rope(float (&acc)[HD / 8][4], int r, int pos, const float2* __restrict__ tab, int lane) {
+  constexpr int HALF = HD / 4;
+  constexpr int NTP = HALF / 8;
+  const float2* tr = tab + (int64_t)pos * HALF;
+#pragma unroll
+  for (int nt = 0; nt < NTP; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int i = nt * 8 + 2 * (lane & 3) + e;
+      const float2 cs = __ldg(tr + i);
+      const float x1 = acc[nt][2 * r + e], x2 = acc[nt + NTP][2 * r + e];
+      acc[nt][2 * r + e] = x1 * cs.x + x2 * cs.y;
+      acc[nt + NTP][2 * r + e] = x2 * cs.x - x1 * cs.y;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------- dQ
+template <int HD>
+__global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf16* __restrict__ qkv,
+                                                          const bf16* __restrict__ dO,
+                                                          const float* __restrict__ lse,
+                                                          const float* __restrict__ delta,
+                                                          const int32_t* __restrict__ cu,
+                                                          const uint32_t* __restrict__ tiles,
+                                                          const float2* __restrict__ rope_tab, int rotary,
+                                                          float scale, bf16* __restrict__ dqkv) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  bf16* sQ = reinterpret_cast<bf16*>(smem);
+  bf16* sdO = sQ + AT<HD>::TILE_ELEMS;
+  bf16* sK = sdO + AT<HD>::TILE_ELEMS;     // [2]
+  bf16* sV = sK + 2 * AT<HD>::TILE_ELEMS;  // [2]
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  int s, idx;
+  decode_tile(tiles[blockIdx.x], s, idx);
+  const int h = blockIdx.y;
+  const int seg0 = cu[s], L = cu[s + 1] - seg0;
+  const int q0 = idx * BT;
+  const int64_t ld = 3 * (int64_t)H;
+  const bf16* gK = qkv + (int64_t)seg0 * ld + H + h * HD;
+  const bf16* gV = qkv + (int64_t)seg0 * ld + 2 * H + h * HD;
+  load_tile<HD>(sQ, qkv + (int64_t)(seg0 + q0) * ld + h * HD, ld, min(BT, L - q0), tid);
+  load_tile<HD>(sdO, dO + (int64_t)(seg0 + q0) * H + h * HD, H, min(BT, L - q0), tid);
+  load_tile<HD>(sK, gK, ld, min(BT, L), tid);
+  load_tile<HD>(sV, gV, ld, min(BT, L), tid);
+  cp_async_commit();
+
+  const float scale_log2 = scale * LOG2E;
+  float lse2[2], dl[2];
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int q = q0 + warp * 16 + (lane >> 2) + 8 * r;
+    lse2[r] = q < L ? lse[(int64_t)h * T + seg0 + q] * LOG2E : 0.f;
+    dl[r] = q < L ? delta[(int64_t)h * T + seg0 + q] : 0.f;
+  }
+  float dq[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.f;
+
+  for (int j = 0; j <= idx; ++j) {
+    const int buf = j & 1;
+    if (j + 1 <= idx) {
+      const int k1 = (j + 1) * BT;
+      load_tile<HD>(sK + (buf ^ 1) * AT<HD>::TILE_ELEMS, gK + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
+      load_tile<HD>(sV + (buf ^ 1) * AT<HD>::TILE_ELEMS, gV + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const bf16* K = sK + buf * AT<HD>::TILE_ELEMS;
+    const bf16* V = sV + buf * AT<HD>::TILE_ELEMS;
+    float sc[8][4], dp[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) sc[i][e] = dp[i][e] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      uint32_t aq[4], ao[4];
+      ld_a<HD>(sQ, warp * 16, kk * 16, lane, aq);
+      ld_a<HD>(sdO, warp * 16, kk * 16, lane, ao);
+#pragma unroll
+      for (int np = 0; np < 4; ++np) {
+        uint32_t b[4];
+        ld_b_rows<HD>(K, np * 16, kk * 16, lane, b);
+        mma_bf16_16816(sc[2 * np], aq, b[0], b[1]);
+        mma_bf16_16816(sc[2 * np + 1], aq, b[2], b[3]);
+        ld_b_rows<HD>(V, np * 16, kk * 16, lane, b);
+        mma_bf16_16816(dp[2 * np], ao, b[0], b[1]);
+        mma_bf16_16816(dp[2 * np + 1], ao, b[2], b[3]);
+      }
+    }
+    const bool diag = (j == idx);
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int r = e >> 1;
+        float p = exp2f(sc[nt][e] * scale_log2 - lse2[r]);
+        if (diag) {
+          const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int ql = warp * 16 + (lane >> 2) + (r << 3);
+          if (kl > ql) p = 0.f;
+        }
+        sc[nt][e] = p * (dp[nt][e] - dl[r]);  // dS
+      }
+    }
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      uint32_t a[4];
+      a[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
+      a[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
+      a[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      a[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int np = 0; np < HD / 16; ++np) {
+        uint32_t b[4];
+        ld_b_cols<HD>(K, kk * 16, np * 16, lane, b);
+        mma_bf16_16816(dq[2 * np], a, b[0], b[1]);
+        mma_bf16_16816(dq[2 * np + 1], a, b[2], b[3]);
+      }
+    }
+    __syncthreads();
+  }
+
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int q = q0 + warp * 16 + (lane >> 2) + 8 * r;
+#pragma unroll
+    for (int i = 0; i < HD / 8; ++i) {
+      dq[i][2 * r] *= scale;
+      dq[i][2 * r + 1] *= scale;
+    }
+    if (q < L) {
+      if (rope_tab) inverse_rope<HD>(dq, r, q, rope_tab, lane);
+      bf16* row = dqkv + (int64_t)(seg0 + q) * ld + h * HD + 2 * (lane & 3);
+#pragma unroll
+      for (int nt = 0; nt < HD / 8; ++nt)
+        *reinterpret_cast<uint32_t*>(row + nt * 8) = pack_bf16x2(dq[nt][2 * r], dq[nt][2 * r + 1]);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------- dK, dV
+template <int HD>
+__global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const bf16* __restrict__ qkv,
+                                                           const bf16* __restrict__ dO,
+                                                           const float* __restrict__ lse,
+                                                           const float* __restrict__ delta,
+                                                           const int32_t* __restrict__ cu,
+                                                           const uint32_t* __restrict__ tiles,
+                                                           const float2* __restrict__ rope_tab, int rotary,
+                                                           float scale, bf16* __restrict__ dqkv) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  bf16* sK = reinterpret_cast<bf16*>(smem);
+  bf16* sV = sK + AT<HD>::TILE_ELEMS;
+  bf16* sQ = sV + AT<HD>::TILE_ELEMS;       // [2]
+  bf16* sdO = sQ + 2 * AT<HD>::TILE_ELEMS;  // [2]
+  float* sL = reinterpret_cast<float*>(sdO + 2 * AT<HD>::TILE_ELEMS);  // [2][64] lse * log2e
+  float* sD = sL + 2 * BT;                                               // [2][64] delta
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  int s, idx;
+  decode_tile(tiles[blockIdx.x], s, idx);
+  const int h = blockIdx.y;
+  const int seg0 = cu[s], L = cu[s + 1] - seg0;
+  const int nq = (L + BT - 1) / BT;
+  const int kt = nq - 1 - idx;  // key tile: most work first
+  const int k0 = kt * BT;
+  const int64_t ld = 3 * (int64_t)H;
+  const bf16* gQ = qkv + (int64_t)seg0 * ld + h * HD;
+  const bf16* gdO = dO + (int64_t)seg0 * H + h * HD;
+  load_tile<HD>(sK, qkv + (int64_t)(seg0 + k0) * ld + H + h * HD, ld, min(BT, L - k0), tid);
+  load_tile<HD>(sV, qkv + (int64_t)(seg0 + k0) * ld + 2 * H + h * HD, ld, min(BT, L - k0), tid);
+  load_tile<HD>(sQ, gQ + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+  load_tile<HD>(sdO, gdO + (int64_t)k0 * H, H, min(BT, L - k0), tid);
+  cp_async_commit();
+  if (tid < BT) {
+    const int q = k0 + tid;
+    sL[tid] = q < L ? lse[(int64_t)h * T + seg0 + q] * LOG2E : 0.f;
+    sD[tid] = q < L ? delta[(int64_t)h * T + seg0 + q] : 0.f;
+  }
+  const float scale_log2 = scale * LOG2E;
+  float dk[HD / 8][4], dv[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) dk[i][e] = dv[i][e] = 0.f;
+
+  for (int qt = kt; qt < nq; ++qt) {
+    const int buf = (qt - kt) & 1;
+    if (qt + 1 < nq) {
+      const int q1 = (qt + 1) * BT;
+      load_tile<HD>(sQ + (buf ^ 1) * AT<HD>::TILE_ELEMS, gQ + (int64_t)q1 * ld, ld, min(BT, L - q1), tid);
+      load_tile<HD>(sdO + (buf ^ 1) * AT<HD>::TILE_ELEMS, gdO + (int64_t)q1 * H, H, min(BT, L - q1), tid);
+      cp_async_commit();
+      if (tid < BT) {
+        const int q = q1 + tid;
+        sL[(buf ^ 1) * BT + tid] = q < L ? lse[(int64_t)h * T + seg0 + q] * LOG2E : 0.f;
+        sD[(buf ^ 1) * BT + tid] = q < L ? delta[(int64_t)h * T + seg0 + q] : 0.f;
+      }
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const bf16* Q = sQ + buf * AT<HD>::TILE_ELEMS;
+    const bf16* D = sdO + buf * AT<HD>::TILE_ELEMS;
+    const float* Lq = sL + buf * BT;
+    const float* Dq = sD + buf * BT;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int qb = half * 32;  // query columns [qb, qb + 32) of the tile
+      float st[4][4], dpt[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) st[i][e] = dpt[i][e] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        uint32_t ak[4], av[4];
+        ld_a<HD>(sK, warp * 16, kk * 16, lane, ak);
+        ld_a<HD>(sV, warp * 16, kk * 16, lane, av);
+#pragma unroll
+        for (int np = 0; np < 2; ++np) {
+          uint32_t b[4];
+          ld_b_rows<HD>(Q, qb + np * 16, kk * 16, lane, b);
+          mma_bf16_16816(st[2 * np], ak, b[0], b[1]);
+          mma_bf16_16816(st[2 * np + 1], ak, b[2], b[3]);
+          ld_b_rows<HD>(D, qb + np * 16, kk * 16, lane, b);
+          mma_bf16_16816(dpt[2 * np], av, b[0], b[1]);
+          mma_bf16_16816(dpt[2 * np + 1], av, b[2], b[3]);
+        }
+      }
+      // P^T and dS^T; rows = keys (warp*16 + lane/4 + 8r), cols = queries
+#pragma unroll
+      for (int nt = 0; nt < 4; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int kpos = k0 + warp * 16 + (lane >> 2) + ((e >> 1) << 3);
+          const int ql = qb + nt * 8 + 2 * (lane & 3) + (e & 1);
+          const int qpos = qt * BT + ql;
+          float p = 0.f;
+          if (qpos >= kpos && qpos < L) p = exp2f(st[nt][e] * scale_log2 - Lq[ql]);
+          st[nt][e] = p;
+          dpt[nt][e] = p * (dpt[nt][e] - Dq[ql]);
+        }
+      }
+#pragma unroll
+      for (int kk = 0; kk < 2; ++kk) {
+        uint32_t ap[4], as[4];
+        ap[0] = pack_bf16x2(st[2 * kk][0], st[2 * kk][1]);
+        ap[1] = pack_bf16x2(st[2 * kk][2], st[2 * kk][3]);
+        ap[2] = pack_bf16x2(st[2 * kk + 1][0], st[2 * kk + 1][1]);
+        ap[3] = pack_bf16x2(st[2 * kk + 1][2], st[2 * kk + 1][3]);
+        as[0] = pack_bf16x2(dpt[2 * kk][0], dpt[2 * kk][1]);
+        as[1] = pack_bf16x2(dpt[2 * kk][2], dpt[2 * kk][3]);
+        as[2] = pack_bf16x2(dpt[2 * kk + 1][0], dpt[2 * kk + 1][1]);
+        as[3] = pack_bf16x2(dpt[2 * kk + 1][2], dpt[2 * kk + 1][3]);
+#pragma unroll
+        for (int np = 0; np < HD / 16; ++np) {
+          uint32_t b[4];
+          ld_b_cols<HD>(D, qb + kk * 16, np * 16, lane, b);
+          mma_bf16_16816(dv[2 * np], ap, b[0], b[1]);
+          mma_bf16_16816(dv[2 * np + 1], ap, b[2], b[3]);
+          ld_b_cols<HD>(Q, qb + kk * 16, np * 16, lane, b);
+          mma_bf16_16816(dk[2 * np], as, b[0], b[1]);
+          mma_bf16_16816(dk[2 * np + 1], as, b[2], b[3]);
+        }
+      }
+    }
+    __syncthreads();
+  }
+
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int kpos = k0 + warp * 16 + (lane >> 2) + 8 * r;
+#pragma unroll
+    for (int i = 0; i < HD / 8; ++i) {
+      dk[i][2 * r] *= scale;
+      dk[i][2 * r + 1] *= scale;
+    }
+    if (kpos < L) {
+      if (rope_tab) inverse_rope<HD>(dk, r, kpos, rope_tab, lane);
+      bf16* rk = dqkv + (int64_t)(seg0 + kpos) * ld + H + h * HD + 2 * (lane & 3);
+      bf16* rv = dqkv + (int64_t)(seg0 + kpos) * ld + 2 * H + h * HD + 2 * (lane & 3);
+#pragma unroll
+      for (int nt = 0; nt < HD / 8; ++nt) {
+        *reinterpret_cast<uint32_t*>(rk + nt * 8) = pack_bf16x2(dk[nt][2 * r], dk[nt][2 * r + 1]);
+        *reinterpret_cast<uint32_t*>(rv + nt * 8) = pack_bf16x2(dv[nt][2 * r], dv[nt][2 * r + 1]);
+      }
+    }
+  }
+}
+
+template <int HD>
+constexpr int fwd_smem() { return 5 * AT<HD>::TILE_BYTES; }
+template <int HD>
+constexpr int dq_smem() { return 6 * AT<HD>::TILE_BYTES; }
+template <int HD>
+constexpr int dkv_smem() { return 6 * AT<HD>::TILE_BYTES + 4 * BT * 4; }
+
+template <int HD>
+int set_attrs() {
+  static bool done = false;
+  if (!done) {
+    FL_CUDA_TRY(cudaFuncSetAttribute(attn_fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, fwd_smem<HD>()));
+    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dq_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, dq_smem<HD>()));
+    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dkv_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, dkv_smem<HD>()));
+    done = true;
+  }
+  return FL_OK;
+}
+
+}  // namespace
+
+int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles) {
+  int maxq = 0;
+  for (int s = 0; s < S; ++s) {
+    const int nq = (cu[s + 1] - cu[s] + BT - 1) / BT;
+    maxq = nq > maxq ? nq : maxq;
+  }
+  int n = 0;
+  for (int i = maxq - 1; i >= 0; --i)
+    for (int s = 0; s < S; ++s) {
+      const int nq = (cu[s + 1] - cu[s] + BT - 1) / BT;
+      if (i < nq) {
+        if (n >= max_tiles) return -1;
+        tiles[n++] = (uint32_t(s) << 16) | uint32_t(i);
+      }
+    }
+  return n;
+}
+
+int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
+                       void* o, float* lse, cudaStream_t st) {
+  if (n_tiles <= 0) return FL_OK;
+  const int H = nh * hd;
+  const float scale_log2 = (1.f / sqrtf((float)hd)) * LOG2E;
+  const dim3 grid(n_tiles, nh);
+  if (hd == 128) {
+    if (int rc = set_attrs<128>()) return rc;
+    attn_fwd_kernel<128><<<grid, 128, fwd_smem<128>(), st>>>(T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2);
+  } else if (hd == 64) {
+    if (int rc = set_attrs<64>()) return rc;
+    attn_fwd_kernel<64><<<grid, 128, fwd_smem<64>(), st>>>(T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2);
+  } else {
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
+  }
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
+                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const int32_t* /*pos*/,
+                       const float* rope_tab, int rotary, void* dqkv, cudaStream_t st) {
+  if (n_tiles <= 0) return FL_OK;
+  const int H = nh * hd;
+  const float scale = 1.f / sqrtf((float)hd);
+  const int64_t pairs = (int64_t)T * nh;
+  attn_delta_kernel<<<(unsigned)((pairs * 32 + 255) / 256), 256, 0, st>>>(T, H, nh, hd, (const bf16*)o,
+                                                                          (const bf16*)dout, delta);
+  FL_CUDA_TRY(cudaGetLastError());
+  const dim3 grid(n_tiles, nh);
+  const float2* tab = reinterpret_cast<const float2*>(rope_tab);
+  if (hd == 128) {
+    if (int rc = set_attrs<128>()) return rc;
+    attn_bwd_dq_kernel<128><<<grid, 128, dq_smem<128>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta,
+                                                              cu, tiles, tab, rotary, scale, (bf16*)dqkv);
+    FL_CUDA_TRY(cudaGetLastError());
+    attn_bwd_dkv_kernel<128><<<grid, 128, dkv_smem<128>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse,
+                                                                delta, cu, tiles, tab, rotary, scale, (bf16*)dqkv);
+  } else if (hd == 64) {
+    if (int rc = set_attrs<64>()) return rc;
+    attn_bwd_dq_kernel<64><<<grid, 128, dq_smem<64>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta,
+                                                            cu, tiles, tab, rotary, scale, (bf16*)dqkv);
+    FL_CUDA_TRY(cudaGetLastError());
+    attn_bwd_dkv_kernel<64><<<grid, 128, dkv_smem<64>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta,
+                                                              cu, tiles, tab, rotary, scale, (bf16*)dqkv);
+  } else {
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
+  }
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+// ====================================================================== exported kernel API
+
+extern "C" int32_t fl_k_attention_tiles(const int32_t* cu_host, int32_t S) {
+  if (!cu_host || S <= 0) return 0;
+  int n = 0;
+  for (int s = 0; s < S; ++s) n += (cu_host[s + 1] - cu_host[s] + BT - 1) / BT;
+  return n;
+}
+
+static int upload_tiles(const int32_t* cu_host, int32_t S, int32_t* tile_ws, int* n_out) {
+  const int n = fl_k_attention_tiles(cu_host, S);
+  std::vector<uint32_t> t(n > 0 ? n : 1);
+  const int got = fl_build_tiles(cu_host, S, t.data(), n);
+  if (got != n) return fl_internal_error(FL_ERR_INVALID_ARG, "attention: bad cu_seqlens");
+  for (int s = 0; s < S; ++s)
+    if (cu_host[s + 1] < cu_host[s] || cu_host[s + 1] - cu_host[s] > 65535 * BT)
+      return fl_internal_error(FL_ERR_INVALID_ARG, "attention: bad cu_seqlens");
+  if (n > 0) FL_CUDA_TRY(cudaMemcpy(tile_ws, t.data(), n * sizeof(uint32_t), cudaMemcpyHostToDevice));
+  *n_out = n;
+  return FL_OK;
+}
+
+extern "C" int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv,
+                                  const int32_t* cu_seqlens_host, const int32_t* cu_seqlens, int32_t S,
+                                  int32_t* tile_ws, void* o, float* lse, void* stream) {
+  if (!qkv || !cu_seqlens_host || !cu_seqlens || !tile_ws || !o || !lse || S <= 0 || S >= 65536)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: args");
+  if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: cu_seqlens");
+  int n = 0;
+  if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n)) return rc;
+  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, o, lse,
+                            (cudaStream_t)stream);
+}
+
+extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv, const void* o,
+                                  const float* lse, const void* dout, const int32_t* cu_seqlens_host,
+                                  const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,
+                                  const float* rope_tab, int32_t rotary_dim, void* dqkv, void* stream) {
+  if (!qkv || !o || !lse || !dout || !cu_seqlens_host || !cu_seqlens || !tile_ws || !delta_ws || !dqkv || S <= 0 ||
+      S >= 65536)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: args");
+  if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: cu_seqlens");
+  if (rope_tab && rotary_dim != head_dim / 2)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "attention bwd: rotary_dim must be head_dim / 2");
+  int n = 0;
+  if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n)) return rc;
+  return fl_launch_attn_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_seqlens, (const uint32_t*)tile_ws, n, delta_ws,
+                            nullptr, rope_tab, rotary_dim, dqkv, (cudaStream_t)stream);
+}

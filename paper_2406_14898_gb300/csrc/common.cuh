@@ -1,0 +1,69 @@
+// Shared helpers of the FL-GLM server library (sm_103a).
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/flglm.h"
+
+#define FL_DEV __device__ __forceinline__
+
+// Device status word codes (written by kernels, read by the host after a sync).
+enum : int {
+  FL_DEV_OK = 0,
+  FL_DEV_TIMEOUT_FULL = 1,      // MMA waited too long for a TMA stage
+  FL_DEV_TIMEOUT_EMPTY = 2,     // producer waited too long for a free stage
+  FL_DEV_TIMEOUT_ACC_FULL = 3,  // epilogue waited too long for an accumulator
+  FL_DEV_TIMEOUT_ACC_EMPTY = 4, // MMA waited too long for the epilogue
+  FL_DEV_TIMEOUT_DRAIN = 5,     // teardown waited too long for in-flight work
+  FL_DEV_BAD_ARG = 6,           // a kernel found an argument it cannot handle
+};
+
+// Bounded-wait budget: a wait gives up after this many nanoseconds of %globaltimer.
+#ifndef FL_WAIT_NS
+#define FL_WAIT_NS 2000000000ull
+#endif
+
+FL_DEV uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+FL_DEV void report_status(int* status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+FL_DEV float bf2f(__nv_bfloat16 x) { return __bfloat162float(x); }
+FL_DEV __nv_bfloat16 f2bf(float x) { return __float2bfloat16_rn(x); }
+
+FL_DEV uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+FL_DEV float2 unpack_bf16x2(uint32_t u) {
+  __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
+  return __bfloat1622float2(v);
+}
+
+// tanh-form GeLU and its derivative, with c = sqrt(2/pi), a = 0.044715.
+FL_DEV float gelu_tanh(float u) {
+  const float c = 0.7978845608028654f, a = 0.044715f;
+  float t = tanhf(c * (u + a * u * u * u));
+  return 0.5f * u * (1.f + t);
+}
+FL_DEV float gelu_tanh_grad(float u) {
+  const float c = 0.7978845608028654f, a = 0.044715f;
+  float t = tanhf(c * (u + a * u * u * u));
+  return 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * c * (1.f + 3.f * a * u * u);
+}
+
+#define FL_CUDA_TRY(expr)                                  \
+  do {                                                     \
+    cudaError_t _e = (expr);                               \
+    if (_e != cudaSuccess) return fl_internal_cuda_error(_e, #expr, __FILE__, __LINE__); \
+  } while (0)
+
+// Records a CUDA error in the thread-local error string and returns FL_ERR_CUDA.
+int fl_internal_cuda_error(cudaError_t e, const char* what, const char* file, int line);
+int fl_internal_error(int code, const char* fmt, ...);

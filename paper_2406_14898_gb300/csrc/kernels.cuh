@@ -1,0 +1,43 @@
+// Internal launch interfaces shared by the kernels and the server runtime.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+constexpr int FL_MAX_COPY = 64;       // client tensors per gather/scatter launch
+constexpr int FL_MAX_SEGS = 1024;     // causal segments per call
+constexpr int FL_MAX_TILES = 2048;    // 64-row attention tiles per call
+constexpr int FL_ATTN_TILE = 64;
+
+struct CopyTable {
+  int n;
+  void* packed;
+  void* client[FL_MAX_COPY];
+  int64_t off16[FL_MAX_COPY];  // offset into packed, 16-byte words
+  int64_t n16[FL_MAX_COPY];    // length, 16-byte words
+};
+
+// Packing metadata of one call, passed by value to the metadata kernel.
+// tiles[i] = segment << 16 | tile index inside the segment, ordered by decreasing tile
+// index (the longest causal rows first).
+struct MetaArgs {
+  int S;
+  int n_tiles;
+  int32_t cu[FL_MAX_SEGS + 1];
+  uint32_t tiles[FL_MAX_TILES];
+};
+
+int fl_launch_gather_scatter(const CopyTable& tab, int scatter, cudaStream_t st);
+int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st);
+int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, float* out, cudaStream_t st);
+int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st);
+int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st);
+
+// Attention on a device tile list (built by fl_launch_meta).
+int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
+                       int n_tiles, void* o, float* lse, cudaStream_t st);
+int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
+                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const int32_t* pos,
+                       const float* rope_tab, int rotary_dim, void* dqkv, cudaStream_t st);
+
+// Host helper: builds the tile list of a packing (returns the count, -1 if over capacity).
+int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles);

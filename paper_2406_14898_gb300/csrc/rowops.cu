@@ -1,0 +1,467 @@
+// HBM-bound kernels of the server step: LayerNorm forward/backward (warp per row,
+// 128-bit loads), bias-gradient column sums, AdamW over the flat fp32 arena,
+// client pack/unpack, per-call packing metadata and the seeded parameter init.
+#include <cstdio>
+
+#include "../../include/flglm_kernels.h"
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace {
+
+int sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+FL_DEV float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+FL_DEV void unpack8(const uint4& w, float* f) {
+  float2 a = unpack_bf16x2(w.x), b = unpack_bf16x2(w.y), c = unpack_bf16x2(w.z), d = unpack_bf16x2(w.w);
+  f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y; f[4] = c.x; f[5] = c.y; f[6] = d.x; f[7] = d.y;
+}
+FL_DEV uint4 pack8(const float* f) {
+  uint4 w;
+  w.x = pack_bf16x2(f[0], f[1]);
+  w.y = pack_bf16x2(f[2], f[3]);
+  w.z = pack_bf16x2(f[4], f[5]);
+  w.w = pack_bf16x2(f[6], f[7]);
+  return w;
+}
+
+// ------------------------------------------------------------------ LayerNorm forward
+// One warp per row; lane l owns the 8-element chunks l, l+32, l+64, ... (NV chunks).
+template <int NV>
+__global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bfloat16* __restrict__ x,
+                                                     const float* __restrict__ gamma,
+                                                     const float* __restrict__ beta, float eps,
+                                                     __nv_bfloat16* __restrict__ y, float* __restrict__ mean,
+                                                     float* __restrict__ rstd) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= T) return;
+  const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
+  float v[NV * 8];
+#pragma unroll
+  for (int i = 0; i < NV; ++i) unpack8(__ldg(xr + lane + 32 * i), v + 8 * i);
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV * 8; ++i) s += v[i];
+  const float mu = warp_sum(s) / H;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < NV * 8; ++i) {
+    const float d = v[i] - mu;
+    q += d * d;
+  }
+  const float rs = rsqrtf(warp_sum(q) / H + eps);
+  uint4* yr = reinterpret_cast<uint4*>(y + (int64_t)row * H);
+  const float4* g4 = reinterpret_cast<const float4*>(gamma);
+  const float4* b4 = reinterpret_cast<const float4*>(beta);
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    const int c = lane + 32 * i;  // chunk index: columns [8c, 8c+8)
+    float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
+    float4 ba = __ldg(b4 + 2 * c), bb = __ldg(b4 + 2 * c + 1);
+    const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+    const float bt[8] = {ba.x, ba.y, ba.z, ba.w, bb.x, bb.y, bb.z, bb.w};
+    float o[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) o[j] = (v[8 * i + j] - mu) * rs * gg[j] + bt[j];
+    yr[c] = pack8(o);
+  }
+  if (lane == 0) {
+    mean[row] = mu;
+    rstd[row] = rs;
+  }
+}
+
+// ------------------------------------------------------------------ LayerNorm backward
+// Warp per row for dx; per-CTA column partials of dgamma/dbeta in shared memory, written
+// to workspace[blockIdx.x][2][H] and reduced by ln_bwd_reduce_kernel.
+template <int NV>
+__global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bfloat16* __restrict__ dy,
+                                                     const __nv_bfloat16* __restrict__ x,
+                                                     const float* __restrict__ mean,
+                                                     const float* __restrict__ rstd,
+                                                     const float* __restrict__ gamma,
+                                                     const __nv_bfloat16* __restrict__ resid, float resid_alpha,
+                                                     __nv_bfloat16* __restrict__ dx, float* __restrict__ ws) {
+  extern __shared__ float part[];  // [2][H]: dgamma, dbeta
+  for (int i = threadIdx.x; i < 2 * H; i += blockDim.x) part[i] = 0.f;
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int wid = threadIdx.x >> 5;
+  const float4* g4 = reinterpret_cast<const float4*>(gamma);
+  for (int row = blockIdx.x * 8 + wid; row < T; row += gridDim.x * 8) {
+    const uint4* dyr = reinterpret_cast<const uint4*>(dy + (int64_t)row * H);
+    const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
+    const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
+    // pass 1: row sums of g = gamma*dy and g*xhat; column partials of dgamma, dbeta
+    float s1 = 0.f, s2 = 0.f;
+#pragma unroll 4
+    for (int i = 0; i < NV; ++i) {
+      const int c = lane + 32 * i;
+      float d[8], xv[8];
+      unpack8(__ldg(dyr + c), d);
+      unpack8(__ldg(xr + c), xv);
+      const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
+      const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float xh = (xv[j] - mu) * rs;
+        atomicAdd(&part[8 * c + j], d[j] * xh);
+        atomicAdd(&part[H + 8 * c + j], d[j]);
+        const float g = d[j] * gg[j];
+        s1 += g;
+        s2 += g * xh;
+      }
+    }
+    const float mg = warp_sum(s1) / H;
+    const float mgx = warp_sum(s2) / H;
+    // pass 2: dx = rstd * (g - mean(g) - xhat * mean(g xhat)) (+ alpha * resid)
+    uint4* dxr = reinterpret_cast<uint4*>(dx + (int64_t)row * H);
+    const uint4* rr = resid ? reinterpret_cast<const uint4*>(resid + (int64_t)row * H) : nullptr;
+#pragma unroll 4
+    for (int i = 0; i < NV; ++i) {
+      const int c = lane + 32 * i;
+      float d[8], xv[8], o[8];
+      unpack8(__ldg(dyr + c), d);
+      unpack8(__ldg(xr + c), xv);
+      const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
+      const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o[j] = rs * (d[j] * gg[j] - mg - (xv[j] - mu) * rs * mgx);
+      if (rr) {
+        float r[8];
+        unpack8(__ldg(rr + c), r);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o[j] = fmaf(resid_alpha, r[j], o[j]);
+      }
+      dxr[c] = pack8(o);
+    }
+  }
+  __syncthreads();
+  float* out = ws + (int64_t)blockIdx.x * 2 * H;
+  for (int i = threadIdx.x; i < 2 * H; i += blockDim.x) out[i] = part[i];
+}
+
+__global__ void ln_bwd_reduce_kernel(int nblk, int H, const float* __restrict__ ws, float* __restrict__ dgamma,
+                                     float* __restrict__ dbeta) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= 2 * H) return;
+  float s = 0.f;
+  for (int b = 0; b < nblk; ++b) s += ws[(int64_t)b * 2 * H + i];
+  if (i < H) dgamma[i] += s;
+  else dbeta[i - H] += s;
+}
+
+int ln_bwd_blocks(int T) {
+  const int want = (T + 7) / 8;
+  const int cap = 2 * sm_count();
+  return want < cap ? want : cap;
+}
+
+// ------------------------------------------------------------------ column sums (bias grads)
+// Block: 32 column-threads (8 columns each = 256 columns) x 8 row groups.
+__global__ void __launch_bounds__(256) colsum_kernel(int T, int N, const __nv_bfloat16* __restrict__ x,
+                                                     float* __restrict__ out, int rows_per_block) {
+  __shared__ float red[8][256];
+  const int cx = threadIdx.x & 31;
+  const int ry = threadIdx.x >> 5;
+  const int col = blockIdx.x * 256 + cx * 8;
+  const int r0 = blockIdx.y * rows_per_block;
+  const int r1 = min(T, r0 + rows_per_block);
+  float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (col < N) {
+    for (int r = r0 + ry; r < r1; r += 8) {
+      float f[8];
+      unpack8(__ldg(reinterpret_cast<const uint4*>(x + (int64_t)r * N + col)), f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] += f[j];
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) red[ry][cx * 8 + j] = acc[j];
+  __syncthreads();
+  const int c = threadIdx.x;
+  if (blockIdx.x * 256 + c < N) {
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s += red[k][c];
+    atomicAdd(out + blockIdx.x * 256 + c, s);
+  }
+}
+
+// ------------------------------------------------------------------ AdamW
+__global__ void __launch_bounds__(256) adamw_kernel(int64_t n4, float4* __restrict__ w, float4* __restrict__ g,
+                                                    float4* __restrict__ m, float4* __restrict__ v,
+                                                    uint2* __restrict__ wb, float lr, float b1, float b2, float eps,
+                                                    float wd, float inv_bc1, float inv_bc2) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+    float4 W = w[i], G = g[i], M = m[i], V = v[i];
+    float* pw = &W.x;
+    float* pg = &G.x;
+    float* pm = &M.x;
+    float* pv = &V.x;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      pm[j] = b1 * pm[j] + (1.f - b1) * pg[j];
+      pv[j] = b2 * pv[j] + (1.f - b2) * pg[j] * pg[j];
+      const float mh = pm[j] * inv_bc1;
+      const float vh = pv[j] * inv_bc2;
+      pw[j] = pw[j] - lr * (mh / (sqrtf(vh) + eps) + wd * pw[j]);
+    }
+    w[i] = W;
+    m[i] = M;
+    v[i] = V;
+    g[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (wb) wb[i] = make_uint2(pack_bf16x2(W.x, W.y), pack_bf16x2(W.z, W.w));
+  }
+}
+
+__global__ void f32_to_bf16_kernel(int64_t n, const float* __restrict__ src, __nv_bfloat16* __restrict__ dst) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    dst[i] = f2bf(src[i]);
+}
+
+// ------------------------------------------------------------------ pack / unpack
+__global__ void gather_scatter_kernel(CopyTable tab, int scatter) {
+  // blockIdx.y = entry; each entry copies n16 16-byte words between a client buffer and
+  // the packed buffer.
+  const int e = blockIdx.y;
+  if (e >= tab.n) return;
+  const int64_t n16 = tab.n16[e];
+  uint4* packed = reinterpret_cast<uint4*>(tab.packed) + tab.off16[e];
+  uint4* client = reinterpret_cast<uint4*>(tab.client[e]);
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16; i += (int64_t)gridDim.x * blockDim.x) {
+    if (scatter) client[i] = packed[i];
+    else packed[i] = client[i];
+  }
+}
+
+// ------------------------------------------------------------------ packing metadata
+__global__ void meta_kernel(MetaArgs a, int32_t* __restrict__ cu, int32_t* __restrict__ pos,
+                            uint32_t* __restrict__ tiles) {
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t nth = (int64_t)gridDim.x * blockDim.x;
+  const int T = a.cu[a.S];
+  for (int64_t i = tid; i <= a.S; i += nth) cu[i] = a.cu[i];
+  for (int64_t i = tid; i < a.n_tiles; i += nth) tiles[i] = a.tiles[i];
+  for (int64_t t = tid; t < T; t += nth) {
+    int lo = 0, hi = a.S - 1;  // last segment with cu[s] <= t
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.cu[mid] <= t) lo = mid;
+      else hi = mid - 1;
+    }
+    pos[t] = int32_t(t - a.cu[lo]);
+  }
+}
+
+// ------------------------------------------------------------------ seeded init
+// SplitMix64 stream (Steele, Lea & Flood 2014) and Box-Muller (1958):
+//   raw(key, i) = mix64(key + (i+1) * GOLDEN);  U = ((raw >> 11) + 1) * 2^-53
+//   element i: pair j = i/2, r = sqrt(-2 ln U(2j)), phi = 2 pi U(2j+1),
+//   z = r cos(phi) (even i) or r sin(phi) (odd i); value = fp32(mean + std * z)
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z ^= z >> 30;
+  z *= 0xBF58476D1CE4E5B9ull;
+  z ^= z >> 27;
+  z *= 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+__device__ __forceinline__ double unif(uint64_t key, uint64_t i) {
+  const uint64_t x = mix64(key + (i + 1) * 0x9E3779B97F4A7C15ull);
+  return (double)((x >> 11) + 1) * (1.0 / 9007199254740992.0);
+}
+__global__ void normal_init_kernel(int64_t n, uint64_t key, double mean, double std_, float* __restrict__ out) {
+  const double two_pi = 6.283185307179586476925286766559;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t j = (uint64_t)i >> 1;
+    const double u1 = unif(key, 2 * j), u2 = unif(key, 2 * j + 1);
+    const double r = sqrt(-2.0 * log(u1));
+    const double z = (i & 1) ? r * sin(two_pi * u2) : r * cos(two_pi * u2);
+    out[i] = (float)(mean + std_ * z);
+  }
+}
+__global__ void fill_kernel(int64_t n, float v, float* __restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = v;
+}
+
+int grid_for(int64_t n, int per_thread_block = 256) {
+  int64_t b = (n + per_thread_block - 1) / per_thread_block;
+  const int64_t cap = (int64_t)sm_count() * 8;
+  if (b > cap) b = cap;
+  if (b < 1) b = 1;
+  return (int)b;
+}
+
+}  // namespace
+
+// ====================================================================== exported kernel API
+
+extern "C" int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, const float* gamma, const float* beta,
+                                  float eps, void* y, float* mean, float* rstd, void* stream) {
+  if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d", H);
+  if (!x || !gamma || !beta || !y || !mean || !rstd) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: null");
+  if (T == 0) return FL_OK;
+  cudaStream_t st = (cudaStream_t)stream;
+  const dim3 grid((T + 7) / 8), block(256);
+  auto xb = (const __nv_bfloat16*)x;
+  auto yb = (__nv_bfloat16*)y;
+  switch (H / 256) {
+#define FL_LNF(NV) \
+  case NV: ln_fwd_kernel<NV><<<grid, block, 0, st>>>(T, H, xb, gamma, beta, eps, yb, mean, rstd); break;
+    FL_LNF(1) FL_LNF(2) FL_LNF(4) FL_LNF(8) FL_LNF(16)
+#undef FL_LNF
+    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H/256 must be a power of two");
+  }
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+extern "C" size_t fl_k_layernorm_bwd_workspace(int32_t T, int32_t H) {
+  return (size_t)ln_bwd_blocks(T > 0 ? T : 1) * 2 * (size_t)H * sizeof(float);
+}
+
+extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
+                                  const float* rstd, const float* gamma, const void* resid, float resid_alpha,
+                                  void* dx, float* dgamma, float* dbeta, void* workspace, void* stream) {
+  if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H=%d", H);
+  if (!dy || !x || !mean || !rstd || !gamma || !dx || !dgamma || !dbeta || !workspace)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: null");
+  if (T == 0) return FL_OK;
+  cudaStream_t st = (cudaStream_t)stream;
+  const int nblk = ln_bwd_blocks(T);
+  const size_t smem = 2 * (size_t)H * sizeof(float);
+  float* ws = (float*)workspace;
+  auto dyb = (const __nv_bfloat16*)dy;
+  auto xb = (const __nv_bfloat16*)x;
+  auto rb = (const __nv_bfloat16*)resid;
+  auto dxb = (__nv_bfloat16*)dx;
+  switch (H / 256) {
+#define FL_LNB(NV)                                                                                          \
+  case NV: {                                                                                                \
+    static bool set = false;                                                                                \
+    if (!set) {                                                                                             \
+      FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536)); \
+      set = true;                                                                                           \
+    }                                                                                                       \
+    ln_bwd_kernel<NV><<<nblk, 256, smem, st>>>(T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws); \
+    break;                                                                                                  \
+  }
+    FL_LNB(1) FL_LNB(2) FL_LNB(4) FL_LNB(8) FL_LNB(16)
+#undef FL_LNB
+    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H/256 must be a power of two");
+  }
+  FL_CUDA_TRY(cudaGetLastError());
+  ln_bwd_reduce_kernel<<<(2 * H + 255) / 256, 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream) {
+  if (T < 0 || N <= 0 || (N % 8) || !x || !out) return fl_internal_error(FL_ERR_INVALID_ARG, "colsum: args");
+  if (T == 0) return FL_OK;
+  const int cblocks = (N + 255) / 256;
+  int rblocks = (2 * sm_count() + cblocks - 1) / cblocks;
+  if (rblocks < 1) rblocks = 1;
+  int rows = (T + rblocks - 1) / rblocks;
+  rows = (rows + 7) / 8 * 8;
+  rblocks = (T + rows - 1) / rows;
+  colsum_kernel<<<dim3(cblocks, rblocks), 256, 0, (cudaStream_t)stream>>>(T, N, (const __nv_bfloat16*)x, out, rows);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+extern "C" int fl_k_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
+                          float beta2, float eps, float weight_decay, float bc1, float bc2, void* stream) {
+  if (n < 0 || (n % 4) || !w || !g || !m || !v) return fl_internal_error(FL_ERR_INVALID_ARG, "adamw: args (n %% 4)");
+  if (n == 0) return FL_OK;
+  const int64_t n4 = n / 4;
+  adamw_kernel<<<grid_for(n4), 256, 0, (cudaStream_t)stream>>>(n4, (float4*)w, (float4*)g, (float4*)m, (float4*)v,
+                                                              (uint2*)w_bf16, lr, beta1, beta2, eps, weight_decay,
+                                                              1.f / bc1, 1.f / bc2);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+// ====================================================================== internal launchers
+
+int fl_launch_gather_scatter(const CopyTable& tab, int scatter, cudaStream_t st) {
+  if (tab.n <= 0) return FL_OK;
+  int64_t maxn = 0;
+  for (int e = 0; e < tab.n; ++e) maxn = tab.n16[e] > maxn ? tab.n16[e] : maxn;
+  int gx = (int)((maxn + 255) / 256);
+  const int cap = (2 * sm_count() + tab.n - 1) / tab.n + 1;
+  if (gx > cap) gx = cap;
+  if (gx < 1) gx = 1;
+  gather_scatter_kernel<<<dim3(gx, tab.n), 256, 0, st>>>(tab, scatter);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st) {
+  const int T = a.cu[a.S];
+  meta_kernel<<<grid_for(T > a.n_tiles ? T : a.n_tiles), 256, 0, st>>>(a, cu, pos, tiles);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, float* out, cudaStream_t st) {
+  if (n <= 0) return FL_OK;
+  normal_init_kernel<<<grid_for(n), 256, 0, st>>>(n, key, mean, std_, out);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st) {
+  if (n <= 0) return FL_OK;
+  fill_kernel<<<grid_for(n), 256, 0, st>>>(n, v, out);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st) {
+  if (n <= 0) return FL_OK;
+  f32_to_bf16_kernel<<<grid_for(n), 256, 0, st>>>(n, src, (__nv_bfloat16*)dst);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+extern "C" int fl_k_pack_clients(int32_t K, void* const* clients_host, const int64_t* bytes_host, void* packed,
+                                 int32_t scatter, void* stream) {
+  if (K < 0 || K > 4096 || !packed || (K > 0 && (!clients_host || !bytes_host)))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "pack: args");
+  if (reinterpret_cast<uintptr_t>(packed) & 15) return fl_internal_error(FL_ERR_INVALID_ARG, "pack: packed alignment");
+  int64_t off = 0;
+  for (int k0 = 0; k0 < K; k0 += FL_MAX_COPY) {
+    CopyTable tab;
+    tab.n = (K - k0) < FL_MAX_COPY ? (K - k0) : FL_MAX_COPY;
+    tab.packed = packed;
+    for (int e = 0; e < tab.n; ++e) {
+      const int k = k0 + e;
+      if (!clients_host[k] || (reinterpret_cast<uintptr_t>(clients_host[k]) & 15) || bytes_host[k] < 0 ||
+          (bytes_host[k] % 16))
+        return fl_internal_error(FL_ERR_INVALID_ARG, "pack: client %d pointer/size", k);
+      tab.client[e] = clients_host[k];
+      tab.off16[e] = off / 16;
+      tab.n16[e] = bytes_host[k] / 16;
+      off += bytes_host[k];
+    }
+    if (int rc = fl_launch_gather_scatter(tab, scatter, (cudaStream_t)stream)) return rc;
+  }
+  return FL_OK;
+}

@@ -1,0 +1,702 @@
+// Server runtime of the FL-GLM block stack: the C ABI of flglm.h.
+//
+// Protocol (§3.1 Model Split, §3.3 client-batch): forward packs the K clients' smashed
+// data into one ragged batch and runs blocks 1..N-2; backward takes the clients'
+// output-state gradients back through the stack, accumulating fp32 weight gradients;
+// step applies AdamW (the optimizer of §4.1.4) and clears them.
+//
+// Device memory (allocated once in fl_server_create, nothing allocated later):
+//   parameter arenas  fp32 master w, grad g, Adam m, v and the bf16 working copy, one flat
+//                     array each with identical offsets (tensor t of block b at
+//                     b * block_stride + tensor_off[t], every tensor 64-byte aligned), so that
+//                     one AdamW launch covers every parameter;
+//   activations       per block: LN1 out A, rotated QKV, attention O, LSE, residual stream
+//                     Hres, LN2 out M, FFN pre-activation U and GeLU output G, LN statistics;
+//                     xs[0..n_blocks]: block inputs / outputs (xs[0] = packed client states);
+//   backward scratch  one set of gradient buffers reused by every block;
+//   metadata          cu_seqlens, per-token positions, attention tile list, rotary table.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/flglm.h"
+#include "../../include/flglm_kernels.h"
+#include "common.cuh"
+#include "kernels.cuh"
+
+// ------------------------------------------------------------------ errors
+static thread_local std::string g_last_error;
+
+int fl_internal_error(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+int fl_internal_cuda_error(cudaError_t e, const char* what, const char* file, int line) {
+  return fl_internal_error(FL_ERR_CUDA, "%s failed: %s (%s:%d)", what, cudaGetErrorString(e), file, line);
+}
+
+namespace {
+
+constexpr uint64_t GOLDEN = 0x9E3779B97F4A7C15ull;
+uint64_t mix64_host(uint64_t z) {
+  z ^= z >> 30;
+  z *= 0xBF58476D1CE4E5B9ull;
+  z ^= z >> 27;
+  z *= 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+// key(seed, tag) = mix64(mix64(seed + GOLDEN) ^ tag), tag = purpose<<56 | block<<40 | tensor<<32 | client
+uint64_t stream_key(uint64_t seed, uint64_t purpose, uint64_t block, uint64_t tensor, uint64_t client) {
+  const uint64_t tag = (purpose << 56) | (block << 40) | (tensor << 32) | client;
+  return mix64_host(mix64_host(seed + GOLDEN) ^ tag);
+}
+
+struct BlockAct {
+  __nv_bfloat16 *a, *qkv, *o, *h, *m, *u, *g;
+  float *mean1, *rstd1, *mean2, *rstd2, *lse;
+};
+
+struct Prof {
+  bool on = false;
+  std::vector<cudaEvent_t> pool;
+  std::vector<std::pair<int, int>> marks;  // (class, event index of the begin event)
+  size_t used = 0;
+};
+
+}  // namespace
+
+struct fl_server {
+  fl_server_cfg cfg;
+  int rdim = 0;
+  cudaStream_t stream = nullptr;
+  std::string err;
+
+  // parameter arenas
+  int64_t tensor_off[FL_T_COUNT] = {};
+  int64_t tensor_n[FL_T_COUNT] = {};
+  int64_t block_stride = 0;
+  int64_t n_params = 0;  // padded total
+  float *w = nullptr, *g = nullptr, *m = nullptr, *v = nullptr;
+  __nv_bfloat16* wb = nullptr;
+  int64_t step_t = 0;
+
+  // activations
+  std::vector<__nv_bfloat16*> xs;
+  std::vector<BlockAct> act;
+  // backward scratch
+  __nv_bfloat16 *dy = nullptr, *dx = nullptr, *du = nullptr, *dm = nullptr, *dh = nullptr, *d_o = nullptr,
+                *dqkv = nullptr, *da = nullptr;
+  float *delta = nullptr, *ln_ws = nullptr;
+  // metadata
+  int32_t *cu = nullptr, *pos = nullptr;
+  uint32_t* tiles = nullptr;
+  float* rope_tab = nullptr;
+  int* status = nullptr;
+
+  std::vector<void*> allocations;
+
+  // pending step
+  bool pending = false;
+  int T = 0, S = 0, K = 0, n_tiles = 0;
+  std::vector<int32_t> seq_lens;
+
+  Prof prof;
+  int64_t launches = 0;
+
+  float* wt(int b, int t) { return w + b * block_stride + tensor_off[t]; }
+  float* gt(int b, int t) { return g + b * block_stride + tensor_off[t]; }
+  __nv_bfloat16* wbt(int b, int t) { return wb + b * block_stride + tensor_off[t]; }
+};
+
+namespace {
+
+int set_err(fl_server* h, int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  if (h) h->err = buf;
+  return code;
+}
+// Propagates an error from an internal call, copying the thread-local message to h.
+int fwd_err(fl_server* h, int rc) {
+  if (rc != FL_OK && h) h->err = g_last_error;
+  return rc;
+}
+
+template <typename T>
+int dalloc(fl_server* h, T** p, size_t count) {
+  void* q = nullptr;
+  const size_t bytes = count * sizeof(T) + 256;
+  cudaError_t e = cudaMalloc(&q, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return set_err(h, FL_ERR_OOM, "cudaMalloc of %zu bytes failed: %s", bytes, cudaGetErrorString(e));
+  }
+  h->allocations.push_back(q);
+  *p = reinterpret_cast<T*>(q);
+  return FL_OK;
+}
+
+// Marks the start of `nk` kernel launches of class cls on the handle's stream.
+void prof_begin(fl_server* h, int cls, int nk = 1) {
+  h->launches += nk;
+  if (!h->prof.on) return;
+  Prof& p = h->prof;
+  while (p.pool.size() < p.used + 2) {
+    cudaEvent_t e;
+    cudaEventCreate(&e);
+    p.pool.push_back(e);
+  }
+  cudaEventRecord(p.pool[p.used], h->stream);
+  p.marks.push_back({cls, (int)p.used});
+  p.used += 2;
+}
+void prof_end(fl_server* h) {
+  if (!h->prof.on) return;
+  cudaEventRecord(h->prof.pool[h->prof.marks.back().second + 1], h->stream);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+int validate_cfg(const fl_server_cfg& c, int* rdim) {
+  if (c.n_blocks < 1 || c.hidden <= 0 || c.n_heads <= 0 || c.head_dim <= 0 || c.ffn_hidden <= 0)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: sizes must be positive");
+  if (c.n_heads * c.head_dim != c.hidden)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: hidden != n_heads * head_dim");
+  if (c.hidden % 256 || c.hidden > 4096 || (c.hidden & (c.hidden - 1)) != 0)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: hidden must be a power of two in [256, 4096]");
+  if (c.ffn_hidden % 256) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: ffn_hidden %% 256 != 0");
+  if (!(c.head_dim == 64 || c.head_dim == 128)) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: head_dim in {64,128}");
+  const int rd = c.rotary_dim ? c.rotary_dim : c.head_dim / 2;
+  if (rd != c.head_dim / 2) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: rotary_dim must be head_dim/2");
+  if (c.max_tokens < 1) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: max_tokens < 1");
+  if (c.client_batch < 1) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: client_batch < 1");
+  if (c.recompute != 0) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: recompute is not built");
+  if (!(c.ln_eps > 0.f) || !(c.rope_base > 1.f)) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: ln_eps/rope_base");
+  if (c.residual_from_ln != 0 && c.residual_from_ln != 1)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: residual_from_ln must be 0 or 1");
+  *rdim = rd;
+  return FL_OK;
+}
+
+int run_gemm(fl_server* h, const fl_gemm_args& a) {
+  prof_begin(h, FL_PROF_GEMM);
+  int rc = fl_k_gemm(&a, h->status, h->stream);
+  prof_end(h);
+  return rc;
+}
+
+fl_gemm_args gemm_fwd(int M, int N, int K, const void* A, const void* W, void* D, int epi) {
+  fl_gemm_args a;
+  memset(&a, 0, sizeof a);
+  a.M = M; a.N = N; a.K = K;
+  a.A = A; a.lda = K; a.a_mn_major = 0;
+  a.B = W; a.ldb = K; a.b_mn_major = 0;
+  a.D = D; a.ldd = N;
+  a.epilogue = epi;
+  return a;
+}
+// dX[T, Kin] = dY[T, Nout] . W[Nout, Kin]
+fl_gemm_args gemm_dgrad(int T, int Kin, int Nout, const void* dY, const void* W, void* dX, int epi) {
+  fl_gemm_args a;
+  memset(&a, 0, sizeof a);
+  a.M = T; a.N = Kin; a.K = Nout;
+  a.A = dY; a.lda = Nout; a.a_mn_major = 0;
+  a.B = W; a.ldb = Kin; a.b_mn_major = 1;
+  a.D = dX; a.ldd = Kin;
+  a.epilogue = epi;
+  return a;
+}
+// dW[Nout, Kin] += dY[T, Nout]^T . X[T, Kin]
+fl_gemm_args gemm_wgrad(int T, int Nout, int Kin, const void* dY, const void* X, float* dW) {
+  fl_gemm_args a;
+  memset(&a, 0, sizeof a);
+  a.M = Nout; a.N = Kin; a.K = T;
+  a.A = dY; a.lda = Nout; a.a_mn_major = 1;
+  a.B = X; a.ldb = Kin; a.b_mn_major = 1;
+  a.D = dW; a.ldd = Kin;
+  a.epilogue = FL_EPI_ACCUM_F32;
+  return a;
+}
+
+#define TRY(h, expr)                    \
+  do {                                  \
+    int _rc = (expr);                   \
+    if (_rc != FL_OK) return fwd_err(h, _rc); \
+  } while (0)
+
+int block_forward(fl_server* h, int b) {
+  const fl_server_cfg& c = h->cfg;
+  const int T = h->T, H = c.hidden, F = c.ffn_hidden;
+  BlockAct& A = h->act[b];
+  const __nv_bfloat16* x = h->xs[b];
+  cudaStream_t st = h->stream;
+  // a = LN1(x)
+  prof_begin(h, FL_PROF_LN);
+  TRY(h, fl_k_layernorm_fwd(T, H, x, h->wt(b, FL_T_LN1_G), h->wt(b, FL_T_LN1_B), c.ln_eps, A.a, A.mean1, A.rstd1, st));
+  prof_end(h);
+  // qkv = a Wqkv^T + bqkv, q and k rotated
+  fl_gemm_args g1 = gemm_fwd(T, 3 * H, H, A.a, h->wbt(b, FL_T_WQKV), A.qkv, FL_EPI_BIAS_ROPE);
+  g1.bias = h->wt(b, FL_T_BQKV);
+  g1.pos = h->pos;
+  g1.rope_tab = h->rope_tab;
+  g1.n_heads = c.n_heads;
+  g1.head_dim = c.head_dim;
+  g1.rotary_dim = h->rdim;
+  TRY(h, run_gemm(h, g1));
+  // o = causal attention within each segment
+  prof_begin(h, FL_PROF_ATTN);
+  TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse, st));
+  prof_end(h);
+  // h = alpha * (a or x) + o Wd^T + bd
+  fl_gemm_args g2 = gemm_fwd(T, H, H, A.o, h->wbt(b, FL_T_WDENSE), A.h, FL_EPI_BIAS_RESID);
+  g2.bias = h->wt(b, FL_T_BDENSE);
+  g2.aux = c.residual_from_ln ? (const void*)A.a : (const void*)x;
+  g2.ld_aux = H;
+  g2.alpha = c.residual_alpha;
+  TRY(h, run_gemm(h, g2));
+  // m = LN2(h)
+  prof_begin(h, FL_PROF_LN);
+  TRY(h, fl_k_layernorm_fwd(T, H, A.h, h->wt(b, FL_T_LN2_G), h->wt(b, FL_T_LN2_B), c.ln_eps, A.m, A.mean2, A.rstd2, st));
+  prof_end(h);
+  // u = m W1^T + b1, g = gelu(u)
+  fl_gemm_args g3 = gemm_fwd(T, F, H, A.m, h->wbt(b, FL_T_WUP), A.g, FL_EPI_BIAS_GELU);
+  g3.bias = h->wt(b, FL_T_BUP);
+  g3.aux_out = A.u;
+  g3.ld_aux_out = F;
+  TRY(h, run_gemm(h, g3));
+  // y = alpha * (m or h) + g W2^T + b2
+  fl_gemm_args g4 = gemm_fwd(T, H, F, A.g, h->wbt(b, FL_T_WDOWN), h->xs[b + 1], FL_EPI_BIAS_RESID);
+  g4.bias = h->wt(b, FL_T_BDOWN);
+  g4.aux = c.residual_from_ln ? (const void*)A.m : (const void*)A.h;
+  g4.ld_aux = H;
+  g4.alpha = c.residual_alpha;
+  TRY(h, run_gemm(h, g4));
+  return FL_OK;
+}
+
+// dy holds dL/dy of block b; on return dx holds dL/dx.
+int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* dx) {
+  const fl_server_cfg& c = h->cfg;
+  const int T = h->T, H = c.hidden, F = c.ffn_hidden;
+  const float al = c.residual_alpha;
+  const bool glm = c.residual_from_ln != 0;
+  BlockAct& A = h->act[b];
+  cudaStream_t st = h->stream;
+  // FFN down: du = (dy W2) * gelu'(u); dW2 += dy^T g; db2 += colsum(dy)
+  fl_gemm_args d1 = gemm_dgrad(T, F, H, dy, h->wbt(b, FL_T_WDOWN), h->du, FL_EPI_GELU_BWD);
+  d1.aux = A.u;
+  d1.ld_aux = F;
+  TRY(h, run_gemm(h, d1));
+  TRY(h, run_gemm(h, gemm_wgrad(T, H, F, dy, A.g, h->gt(b, FL_T_WDOWN))));
+  prof_begin(h, FL_PROF_OTHER);
+  TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
+  prof_end(h);
+  // FFN up: dm = du W1 (+ alpha dy); dW1 += du^T m; db1 += colsum(du)
+  fl_gemm_args d2 = gemm_dgrad(T, H, F, h->du, h->wbt(b, FL_T_WUP), h->dm, glm ? FL_EPI_RESID : FL_EPI_STORE);
+  if (glm) {
+    d2.aux = dy;
+    d2.ld_aux = H;
+    d2.alpha = al;
+  }
+  TRY(h, run_gemm(h, d2));
+  TRY(h, run_gemm(h, gemm_wgrad(T, F, H, h->du, A.m, h->gt(b, FL_T_WUP))));
+  prof_begin(h, FL_PROF_OTHER);
+  TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
+  prof_end(h);
+  // LN2 backward: dh = LN2'(dm) (+ alpha dy)
+  prof_begin(h, FL_PROF_LN, 2);
+  TRY(h, fl_k_layernorm_bwd(T, H, h->dm, A.h, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dy, al, h->dh,
+                            h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B), h->ln_ws, st));
+  prof_end(h);
+  // dense: do = dh Wd; dWd += dh^T o; dbd += colsum(dh)
+  TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
+  TRY(h, run_gemm(h, gemm_wgrad(T, H, H, h->dh, A.o, h->gt(b, FL_T_WDENSE))));
+  prof_begin(h, FL_PROF_OTHER);
+  TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
+  prof_end(h);
+  // attention backward -> dqkv (w.r.t. the un-rotated q, k)
+  prof_begin(h, FL_PROF_ATTN, 3);
+  TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
+                            h->pos, h->rope_tab, h->rdim, h->dqkv, st));
+  prof_end(h);
+  // QKV: da = dqkv Wqkv (+ alpha dh); dWqkv += dqkv^T a; dbqkv += colsum(dqkv)
+  fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
+  if (glm) {
+    d3.aux = h->dh;
+    d3.ld_aux = H;
+    d3.alpha = al;
+  }
+  TRY(h, run_gemm(h, d3));
+  TRY(h, run_gemm(h, gemm_wgrad(T, 3 * H, H, h->dqkv, A.a, h->gt(b, FL_T_WQKV))));
+  prof_begin(h, FL_PROF_OTHER);
+  TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
+  prof_end(h);
+  // LN1 backward: dx = LN1'(da) (+ alpha dh)
+  prof_begin(h, FL_PROF_LN, 2);
+  TRY(h, fl_k_layernorm_bwd(T, H, h->da, h->xs[b], A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G), glm ? nullptr : h->dh, al,
+                            dx, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B), h->ln_ws, st));
+  prof_end(h);
+  return FL_OK;
+}
+
+int copy_clients(fl_server* h, const void* const* ptrs, __nv_bfloat16* packed, int scatter) {
+  const int64_t row16 = (int64_t)h->cfg.client_batch * h->cfg.hidden * 2 / 16;  // 16-byte words per token row group
+  int64_t off = 0;
+  for (int k0 = 0; k0 < h->K; k0 += FL_MAX_COPY) {
+    CopyTable tab;
+    memset(&tab, 0, sizeof tab);
+    tab.packed = packed;
+    tab.n = (h->K - k0) < FL_MAX_COPY ? (h->K - k0) : FL_MAX_COPY;
+    for (int e = 0; e < tab.n; ++e) {
+      const int k = k0 + e;
+      tab.client[e] = const_cast<void*>(ptrs[k]);
+      tab.off16[e] = off;
+      tab.n16[e] = row16 * h->seq_lens[k];
+      off += tab.n16[e];
+    }
+    prof_begin(h, FL_PROF_OTHER);
+    int rc = fl_launch_gather_scatter(tab, scatter, h->stream);
+    prof_end(h);
+    if (rc) return fwd_err(h, rc);
+  }
+  return FL_OK;
+}
+
+int check_ptrs(fl_server* h, const void* const* p, int K, const char* what) {
+  if (!p) return set_err(h, FL_ERR_INVALID_ARG, "%s: null array", what);
+  for (int k = 0; k < K; ++k) {
+    if (!p[k]) return set_err(h, FL_ERR_INVALID_ARG, "%s[%d] is null", what, k);
+    if (!aligned16(p[k])) return set_err(h, FL_ERR_INVALID_ARG, "%s[%d] is not 16-byte aligned", what, k);
+  }
+  return FL_OK;
+}
+
+}  // namespace
+
+// ====================================================================== C ABI
+
+extern "C" void fl_server_cfg_default(fl_server_cfg* c) {
+  if (!c) return;
+  memset(c, 0, sizeof *c);
+  c->n_blocks = 26;
+  c->hidden = 4096;
+  c->n_heads = 32;
+  c->head_dim = 128;
+  c->ffn_hidden = 16384;
+  c->rotary_dim = 64;
+  c->rope_base = 10000.f;
+  c->ln_eps = 1e-5f;
+  c->residual_alpha = sqrtf(56.f);
+  c->residual_from_ln = 1;
+  c->client_batch = 1;
+  c->max_tokens = 8192;
+  c->max_seq_len = 0;
+  c->recompute = 0;
+  c->init_std = 0.02f;
+  c->adam_beta1 = 0.9f;
+  c->adam_beta2 = 0.999f;
+  c->adam_eps = 1e-8f;
+  c->weight_decay = 0.f;
+}
+
+extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_server_t* out) {
+  if (!out) return fl_internal_error(FL_ERR_INVALID_ARG, "create: out is null");
+  *out = nullptr;
+  if (!cfg) return fl_internal_error(FL_ERR_INVALID_ARG, "create: cfg is null");
+  int rdim = 0;
+  if (int rc = validate_cfg(*cfg, &rdim)) return rc;
+  fl_server* h = new fl_server();
+  h->cfg = *cfg;
+  h->rdim = rdim;
+  if (h->cfg.max_seq_len <= 0 || h->cfg.max_seq_len > h->cfg.max_tokens) h->cfg.max_seq_len = h->cfg.max_tokens;
+  const fl_server_cfg& c = h->cfg;
+  const int64_t H = c.hidden, F = c.ffn_hidden, Tm = c.max_tokens;
+  auto fail = [&](int rc) {
+    fl_server_destroy(h);
+    return rc;
+  };
+
+  // parameter layout
+  const int64_t sizes[FL_T_COUNT] = {3 * H * H, 3 * H, H * H, H, F * H, F, H * F, H, H, H, H, H};
+  int64_t off = 0;
+  for (int t = 0; t < FL_T_COUNT; ++t) {
+    h->tensor_off[t] = off;
+    h->tensor_n[t] = sizes[t];
+    off += (sizes[t] + 15) / 16 * 16;
+  }
+  h->block_stride = off;
+  h->n_params = off * c.n_blocks;
+  int rc;
+  if ((rc = dalloc(h, &h->w, h->n_params)) || (rc = dalloc(h, &h->g, h->n_params)) ||
+      (rc = dalloc(h, &h->m, h->n_params)) || (rc = dalloc(h, &h->v, h->n_params)) ||
+      (rc = dalloc(h, &h->wb, h->n_params)))
+    return fail(rc);
+
+  // activations
+  h->xs.resize(c.n_blocks + 1);
+  for (int b = 0; b <= c.n_blocks; ++b)
+    if ((rc = dalloc(h, &h->xs[b], Tm * H))) return fail(rc);
+  h->act.resize(c.n_blocks);
+  for (int b = 0; b < c.n_blocks; ++b) {
+    BlockAct& A = h->act[b];
+    if ((rc = dalloc(h, &A.a, Tm * H)) || (rc = dalloc(h, &A.qkv, Tm * 3 * H)) || (rc = dalloc(h, &A.o, Tm * H)) ||
+        (rc = dalloc(h, &A.h, Tm * H)) || (rc = dalloc(h, &A.m, Tm * H)) || (rc = dalloc(h, &A.u, Tm * F)) ||
+        (rc = dalloc(h, &A.g, Tm * F)) || (rc = dalloc(h, &A.mean1, Tm)) || (rc = dalloc(h, &A.rstd1, Tm)) ||
+        (rc = dalloc(h, &A.mean2, Tm)) || (rc = dalloc(h, &A.rstd2, Tm)) ||
+        (rc = dalloc(h, &A.lse, Tm * c.n_heads)))
+      return fail(rc);
+  }
+  if ((rc = dalloc(h, &h->dy, Tm * H)) || (rc = dalloc(h, &h->dx, Tm * H)) || (rc = dalloc(h, &h->du, Tm * F)) ||
+      (rc = dalloc(h, &h->dm, Tm * H)) || (rc = dalloc(h, &h->dh, Tm * H)) || (rc = dalloc(h, &h->d_o, Tm * H)) ||
+      (rc = dalloc(h, &h->dqkv, Tm * 3 * H)) || (rc = dalloc(h, &h->da, Tm * H)) ||
+      (rc = dalloc(h, &h->delta, Tm * c.n_heads)) ||
+      (rc = dalloc(h, &h->ln_ws, fl_k_layernorm_bwd_workspace((int32_t)Tm, (int32_t)H) / sizeof(float))) ||
+      (rc = dalloc(h, &h->cu, FL_MAX_SEGS + 1)) || (rc = dalloc(h, &h->pos, Tm)) ||
+      (rc = dalloc(h, &h->tiles, FL_MAX_TILES)) || (rc = dalloc(h, &h->status, 1)))
+    return fail(rc);
+
+  // rotary table: [position][pair i] = (cos, sin) of p * base^(-2i/rdim), in double
+  const int half = rdim / 2;
+  const int64_t npos = c.max_seq_len;
+  std::vector<float> tab((size_t)npos * half * 2);
+  for (int64_t p = 0; p < npos; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double ang = (double)p * std::pow((double)c.rope_base, -2.0 * i / (double)rdim);
+      tab[(size_t)(p * half + i) * 2] = (float)std::cos(ang);
+      tab[(size_t)(p * half + i) * 2 + 1] = (float)std::sin(ang);
+    }
+  if ((rc = dalloc(h, &h->rope_tab, tab.size()))) return fail(rc);
+  cudaStream_t st = nullptr;
+  if (cudaMemcpy(h->rope_tab, tab.data(), tab.size() * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaMemset(h->g, 0, h->n_params * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->m, 0, h->n_params * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->v, 0, h->n_params * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->w, 0, h->n_params * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->status, 0, sizeof(int)) != cudaSuccess)
+    return fail(fl_internal_cuda_error(cudaGetLastError(), "create: memset/copy", __FILE__, __LINE__));
+
+  // seeded init: tensor t of block b from the stream (seed, purpose 1, b, t)
+  for (int b = 0; b < c.n_blocks; ++b)
+    for (int t = 0; t < FL_T_COUNT; ++t) {
+      float* p = h->wt(b, t);
+      if (t == FL_T_LN1_G || t == FL_T_LN2_G) rc = fl_launch_fill(h->tensor_n[t], 1.f, p, st);
+      else if (t == FL_T_LN1_B || t == FL_T_LN2_B) rc = fl_launch_fill(h->tensor_n[t], 0.f, p, st);
+      else rc = fl_launch_normal_init(h->tensor_n[t], stream_key(seed, 1, b, t, 0), 0.0, (double)c.init_std, p, st);
+      if (rc) return fail(rc);
+    }
+  if ((rc = fl_launch_f32_to_bf16(h->n_params, h->w, h->wb, st))) return fail(rc);
+  if (cudaDeviceSynchronize() != cudaSuccess)
+    return fail(fl_internal_cuda_error(cudaGetLastError(), "create: init", __FILE__, __LINE__));
+  *out = h;
+  return FL_OK;
+}
+
+extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[], const int32_t seq_lens[], int32_t K,
+                                 void* const out_states[]) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "forward: null handle");
+  const fl_server_cfg& c = h->cfg;
+  if (h->pending) return set_err(h, FL_ERR_STATE, "forward: a forward is already pending (call backward first)");
+  if (K < 1) return set_err(h, FL_ERR_INVALID_ARG, "forward: K=%d < 1", K);
+  if (!seq_lens) return set_err(h, FL_ERR_INVALID_ARG, "forward: seq_lens is null");
+  if (int rc = check_ptrs(h, client_states, K, "client_states")) return rc;
+  if (int rc = check_ptrs(h, (const void* const*)out_states, K, "out_states")) return rc;
+  const int b = c.client_batch;
+  int64_t T = 0;
+  for (int k = 0; k < K; ++k) {
+    if (seq_lens[k] < 1) return set_err(h, FL_ERR_INVALID_ARG, "forward: seq_lens[%d]=%d < 1", k, seq_lens[k]);
+    if (seq_lens[k] > c.max_seq_len)
+      return set_err(h, FL_ERR_INVALID_ARG, "forward: seq_lens[%d]=%d > max_seq_len %d", k, seq_lens[k], c.max_seq_len);
+    T += (int64_t)b * seq_lens[k];
+  }
+  if (T > c.max_tokens) return set_err(h, FL_ERR_CAPACITY, "forward: %lld tokens > max_tokens %d", (long long)T, c.max_tokens);
+  const int64_t S = (int64_t)K * b;
+  if (S > FL_MAX_SEGS) return set_err(h, FL_ERR_CAPACITY, "forward: %lld segments > %d", (long long)S, FL_MAX_SEGS);
+
+  // packing metadata: client k row r is segment k*b + r
+  static thread_local MetaArgs meta;
+  meta.S = (int)S;
+  meta.cu[0] = 0;
+  for (int k = 0, s = 0; k < K; ++k)
+    for (int r = 0; r < b; ++r, ++s) meta.cu[s + 1] = meta.cu[s] + seq_lens[k];
+  const int nt = fl_build_tiles(meta.cu, (int)S, meta.tiles, FL_MAX_TILES);
+  if (nt < 0) return set_err(h, FL_ERR_CAPACITY, "forward: more than %d attention tiles", FL_MAX_TILES);
+  meta.n_tiles = nt;
+  h->T = (int)T;
+  h->S = (int)S;
+  h->K = K;
+  h->n_tiles = nt;
+  h->seq_lens.assign(seq_lens, seq_lens + K);
+
+  prof_begin(h, FL_PROF_OTHER);
+  int rc = fl_launch_meta(meta, h->cu, h->pos, h->tiles, h->stream);
+  prof_end(h);
+  if (rc) return fwd_err(h, rc);
+  if ((rc = copy_clients(h, client_states, h->xs[0], 0))) return rc;
+  for (int blk = 0; blk < c.n_blocks; ++blk)
+    if ((rc = block_forward(h, blk))) return rc;
+  if ((rc = copy_clients(h, (const void* const*)out_states, h->xs[c.n_blocks], 1))) return rc;
+  h->pending = true;
+  return FL_OK;
+}
+
+extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], void* const grad_in[]) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "backward: null handle");
+  if (!h->pending) return set_err(h, FL_ERR_STATE, "backward: no pending forward");
+  if (int rc = check_ptrs(h, grad_out, h->K, "grad_out")) return rc;
+  if (int rc = check_ptrs(h, (const void* const*)grad_in, h->K, "grad_in")) return rc;
+  int rc;
+  if ((rc = copy_clients(h, grad_out, h->dy, 0))) return rc;
+  __nv_bfloat16* cur = h->dy;
+  __nv_bfloat16* nxt = h->dx;
+  for (int blk = h->cfg.n_blocks - 1; blk >= 0; --blk) {
+    if ((rc = block_backward(h, blk, cur, nxt))) return rc;
+    __nv_bfloat16* t = cur;
+    cur = nxt;
+    nxt = t;
+  }
+  if ((rc = copy_clients(h, (const void* const*)grad_in, cur, 1))) return rc;
+  h->pending = false;
+  return FL_OK;
+}
+
+extern "C" int fl_server_step(fl_server_t h, float lr) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "step: null handle");
+  if (h->pending) return set_err(h, FL_ERR_STATE, "step: a forward is pending (call backward first)");
+  const fl_server_cfg& c = h->cfg;
+  h->step_t += 1;
+  const double bc1 = 1.0 - std::pow((double)c.adam_beta1, (double)h->step_t);
+  const double bc2 = 1.0 - std::pow((double)c.adam_beta2, (double)h->step_t);
+  prof_begin(h, FL_PROF_ADAMW);
+  int rc = fl_k_adamw(h->n_params, h->w, h->g, h->m, h->v, h->wb, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
+                      c.weight_decay, (float)bc1, (float)bc2, h->stream);
+  prof_end(h);
+  return fwd_err(h, rc);
+}
+
+extern "C" int fl_server_destroy(fl_server_t h) {
+  if (!h) return FL_OK;
+  cudaStreamSynchronize(h->stream);
+  for (void* p : h->allocations) cudaFree(p);
+  for (cudaEvent_t e : h->prof.pool) cudaEventDestroy(e);
+  delete h;
+  return FL_OK;
+}
+
+extern "C" int fl_server_set_stream(fl_server_t h, void* s) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "set_stream: null handle");
+  h->stream = reinterpret_cast<cudaStream_t>(s);
+  return FL_OK;
+}
+
+extern "C" int fl_server_sync(fl_server_t h) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "sync: null handle");
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "cudaStreamSynchronize", __FILE__, __LINE__));
+  int st = 0;
+  e = cudaMemcpy(&st, h->status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "status read", __FILE__, __LINE__));
+  if (st != 0) {
+    cudaMemset(h->status, 0, sizeof(int));
+    return set_err(h, FL_ERR_TIMEOUT, "a bounded device wait gave up (code %d)", st);
+  }
+  return FL_OK;
+}
+
+extern "C" int64_t fl_server_tensor_numel(fl_server_t h, int32_t t) {
+  if (!h || t < 0 || t >= FL_T_COUNT) return -1;
+  return h->tensor_n[t];
+}
+
+static int check_tensor(fl_server* h, int32_t b, int32_t t, const void* p, size_t n) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "null handle");
+  if (b < 0 || b >= h->cfg.n_blocks || t < 0 || t >= FL_T_COUNT)
+    return set_err(h, FL_ERR_INVALID_ARG, "bad block %d / tensor %d", b, t);
+  if (!p) return set_err(h, FL_ERR_INVALID_ARG, "null host buffer");
+  if ((int64_t)n != h->tensor_n[t])
+    return set_err(h, FL_ERR_INVALID_ARG, "n=%zu but tensor %d has %lld elements", n, t, (long long)h->tensor_n[t]);
+  return FL_OK;
+}
+
+static int d2h(fl_server* h, float* dst, const float* src, size_t n) {
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e == cudaSuccess) e = cudaMemcpy(dst, src, n * sizeof(float), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "device to host copy", __FILE__, __LINE__));
+  return FL_OK;
+}
+
+extern "C" int fl_server_get_param(fl_server_t h, int32_t b, int32_t t, float* dst, size_t n) {
+  if (int rc = check_tensor(h, b, t, dst, n)) return rc;
+  return d2h(h, dst, h->wt(b, t), n);
+}
+extern "C" int fl_server_get_grad(fl_server_t h, int32_t b, int32_t t, float* dst, size_t n) {
+  if (int rc = check_tensor(h, b, t, dst, n)) return rc;
+  return d2h(h, dst, h->gt(b, t), n);
+}
+extern "C" int fl_server_get_adam_moments(fl_server_t h, int32_t b, int32_t t, float* hm, float* hv, size_t n) {
+  if (int rc = check_tensor(h, b, t, hm, n)) return rc;
+  if (!hv) return set_err(h, FL_ERR_INVALID_ARG, "null host buffer");
+  const int64_t o = b * h->block_stride + h->tensor_off[t];
+  if (int rc = d2h(h, hm, h->m + o, n)) return rc;
+  return d2h(h, hv, h->v + o, n);
+}
+extern "C" int fl_server_set_param(fl_server_t h, int32_t b, int32_t t, const float* src, size_t n) {
+  if (int rc = check_tensor(h, b, t, src, n)) return rc;
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e == cudaSuccess) e = cudaMemcpy(h->wt(b, t), src, n * sizeof(float), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "host to device copy", __FILE__, __LINE__));
+  int rc = fl_launch_f32_to_bf16((int64_t)n, h->wt(b, t), h->wbt(b, t), h->stream);
+  if (rc) return fwd_err(h, rc);
+  e = cudaStreamSynchronize(h->stream);
+  if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "set_param", __FILE__, __LINE__));
+  return FL_OK;
+}
+
+extern "C" int fl_server_profile(fl_server_t h, int enable) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "profile: null handle");
+  cudaStreamSynchronize(h->stream);
+  h->prof.on = enable != 0;
+  h->prof.marks.clear();
+  h->prof.used = 0;
+  return FL_OK;
+}
+
+extern "C" int fl_server_profile_read(fl_server_t h, double* ms, int64_t* launches, int32_t n) {
+  if (!h || !ms || !launches || n < 0 || n > FL_PROF_CLASSES)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "profile_read: args");
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "profile sync", __FILE__, __LINE__));
+  for (int i = 0; i < n; ++i) {
+    ms[i] = 0;
+    launches[i] = 0;
+  }
+  for (auto& mk : h->prof.marks) {
+    if (mk.first >= n) continue;
+    float t = 0.f;
+    cudaEventElapsedTime(&t, h->prof.pool[mk.second], h->prof.pool[mk.second + 1]);
+    ms[mk.first] += t;
+    launches[mk.first] += 1;
+  }
+  return FL_OK;
+}
+
+extern "C" int64_t fl_server_launch_count(fl_server_t h) { return h ? h->launches : -1; }
+
+extern "C" const char* fl_server_last_error(fl_server_t h) {
+  if (h) return h->err.c_str();
+  return g_last_error.c_str();
+}

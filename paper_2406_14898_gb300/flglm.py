@@ -1,0 +1,306 @@
+"""Python binding of libflglm.so (ctypes; argument marshalling only).
+
+Every function here forwards to the C ABI of ``include/flglm.h`` and
+``include/flglm_kernels.h`` with the same name; all arithmetic runs in the CUDA
+library.  Tensors may be passed as anything with ``data_ptr()`` (torch CUDA
+tensors) or as raw integer device addresses.  There is no fallback: if the
+library is missing or fails to load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from typing import Optional, Sequence
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libflglm.so")
+
+FL_OK = 0
+ERRORS = {-1: "FL_ERR_INVALID_ARG", -2: "FL_ERR_CAPACITY", -3: "FL_ERR_STATE", -4: "FL_ERR_OOM",
+          -5: "FL_ERR_CUDA", -6: "FL_ERR_TIMEOUT", -7: "FL_ERR_UNSUPPORTED"}
+
+(FL_T_WQKV, FL_T_BQKV, FL_T_WDENSE, FL_T_BDENSE, FL_T_WUP, FL_T_BUP, FL_T_WDOWN, FL_T_BDOWN,
+ FL_T_LN1_G, FL_T_LN1_B, FL_T_LN2_G, FL_T_LN2_B) = range(12)
+FL_T_COUNT = 12
+(FL_EPI_STORE, FL_EPI_BIAS_GELU, FL_EPI_BIAS_RESID, FL_EPI_BIAS_ROPE, FL_EPI_GELU_BWD, FL_EPI_RESID,
+ FL_EPI_ACCUM_F32) = range(7)
+PROF_CLASSES = ("gemm", "attention", "layernorm", "adamw", "other")
+
+
+class FlError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{ERRORS.get(code, code)}: {msg}")
+        self.code = code
+
+
+class fl_server_cfg(C.Structure):
+    _fields_ = [("n_blocks", C.c_int32), ("hidden", C.c_int32), ("n_heads", C.c_int32), ("head_dim", C.c_int32),
+                ("ffn_hidden", C.c_int32), ("rotary_dim", C.c_int32), ("rope_base", C.c_float),
+                ("ln_eps", C.c_float), ("residual_alpha", C.c_float), ("residual_from_ln", C.c_int32),
+                ("client_batch", C.c_int32), ("max_tokens", C.c_int32), ("max_seq_len", C.c_int32),
+                ("recompute", C.c_int32), ("init_std", C.c_float), ("adam_beta1", C.c_float),
+                ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("weight_decay", C.c_float)]
+
+
+class fl_gemm_args(C.Structure):
+    _fields_ = [("M", C.c_int32), ("N", C.c_int32), ("K", C.c_int32),
+                ("A", C.c_void_p), ("lda", C.c_int64), ("a_mn_major", C.c_int32),
+                ("B", C.c_void_p), ("ldb", C.c_int64), ("b_mn_major", C.c_int32),
+                ("D", C.c_void_p), ("ldd", C.c_int64), ("epilogue", C.c_int32),
+                ("bias", C.c_void_p), ("aux", C.c_void_p), ("ld_aux", C.c_int64), ("alpha", C.c_float),
+                ("aux_out", C.c_void_p), ("ld_aux_out", C.c_int64), ("pos", C.c_void_p),
+                ("rope_tab", C.c_void_p), ("n_heads", C.c_int32), ("head_dim", C.c_int32),
+                ("rotary_dim", C.c_int32)]
+
+
+_P = C.c_void_p
+_I32 = C.c_int32
+_I64 = C.c_int64
+_F = C.c_float
+_SIGS = {
+    "fl_server_cfg_default": (None, [C.POINTER(fl_server_cfg)]),
+    "fl_server_create": (C.c_int, [C.POINTER(fl_server_cfg), C.c_uint64, C.POINTER(_P)]),
+    "fl_server_forward": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I32), _I32, C.POINTER(_P)]),
+    "fl_server_backward": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_P)]),
+    "fl_server_step": (C.c_int, [_P, _F]),
+    "fl_server_destroy": (C.c_int, [_P]),
+    "fl_server_set_stream": (C.c_int, [_P, _P]),
+    "fl_server_sync": (C.c_int, [_P]),
+    "fl_server_tensor_numel": (_I64, [_P, _I32]),
+    "fl_server_get_param": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
+    "fl_server_set_param": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
+    "fl_server_get_grad": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
+    "fl_server_get_adam_moments": (C.c_int, [_P, _I32, _I32, _P, _P, C.c_size_t]),
+    "fl_server_profile": (C.c_int, [_P, C.c_int]),
+    "fl_server_profile_read": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(_I64), _I32]),
+    "fl_server_launch_count": (_I64, [_P]),
+    "fl_server_last_error": (C.c_char_p, [_P]),
+    "fl_k_gemm": (C.c_int, [C.POINTER(fl_gemm_args), _P, _P]),
+    "fl_k_layernorm_fwd": (C.c_int, [_I32, _I32, _P, _P, _P, _F, _P, _P, _P, _P]),
+    "fl_k_layernorm_bwd_workspace": (C.c_size_t, [_I32, _I32]),
+    "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
+    "fl_k_attention_tiles": (_I32, [_P, _I32]),
+    "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P]),
+    "fl_k_attention_bwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _I32, _P, _P, _P, _I32, _P, _P]),
+    "fl_k_adamw": (C.c_int, [_I64, _P, _P, _P, _P, _P, _F, _F, _F, _F, _F, _F, _F, _P]),
+    "fl_k_colsum": (C.c_int, [_I32, _I32, _P, _P, _P]),
+    "fl_k_pack_clients": (C.c_int, [_I32, C.POINTER(_P), C.POINTER(_I64), _P, _I32, _P]),
+}
+
+_lib = None
+
+
+def lib() -> C.CDLL:
+    """Loads libflglm.so (raises if it is missing: there is no CPU fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built; run `python -m paper_2406_14898_gb300.build`")
+        L = C.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def ptr(x) -> Optional[int]:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def stream_ptr(stream) -> Optional[int]:
+    if stream is None:
+        return None
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+def check(rc: int, h=None):
+    if rc != FL_OK:
+        msg = lib().fl_server_last_error(h)
+        raise FlError(rc, msg.decode() if msg else "")
+
+
+def _parr(xs) -> "C.Array":
+    return (C.c_void_p * len(xs))(*[ptr(x) for x in xs])
+
+
+def make_cfg(c, max_tokens: int, max_seq_len: int = 0) -> fl_server_cfg:
+    """fl_server_cfg from a workload description with the attributes of
+    ``synthetic.ServerConfig`` (n_blocks, hidden, ... , weight_decay)."""
+    cfg = fl_server_cfg()
+    lib().fl_server_cfg_default(C.byref(cfg))
+    cfg.n_blocks = c.n_blocks
+    cfg.hidden = c.hidden
+    cfg.n_heads = c.n_heads
+    cfg.head_dim = c.head_dim
+    cfg.ffn_hidden = c.ffn_hidden
+    cfg.rotary_dim = c.rdim
+    cfg.rope_base = c.rope_base
+    cfg.ln_eps = c.ln_eps
+    cfg.residual_alpha = c.residual_alpha
+    cfg.residual_from_ln = c.residual_from_ln
+    cfg.client_batch = c.client_batch
+    cfg.max_tokens = max_tokens
+    cfg.max_seq_len = max_seq_len
+    cfg.recompute = 0
+    cfg.init_std = c.init_std
+    cfg.adam_beta1 = c.adam_beta1
+    cfg.adam_beta2 = c.adam_beta2
+    cfg.adam_eps = c.adam_eps
+    cfg.weight_decay = c.weight_decay
+    return cfg
+
+
+class Server:
+    """Owns one fl_server handle.  Methods mirror fl_server_* one to one."""
+
+    def __init__(self, cfg: fl_server_cfg, seed: int, stream=None):
+        self.h = C.c_void_p()
+        rc = lib().fl_server_create(C.byref(cfg), seed, C.byref(self.h))
+        check(rc, None)
+        self.cfg = cfg
+        if stream is not None:
+            self.set_stream(stream)
+
+    def close(self):
+        if self.h:
+            lib().fl_server_destroy(self.h)
+            self.h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def set_stream(self, stream):
+        check(lib().fl_server_set_stream(self.h, stream_ptr(stream)), self.h)
+
+    def forward(self, client_states: Sequence, seq_lens: Sequence[int], out_states: Sequence):
+        K = len(client_states)
+        lens = (C.c_int32 * K)(*seq_lens)
+        check(lib().fl_server_forward(self.h, _parr(client_states), lens, K, _parr(out_states)), self.h)
+
+    def backward(self, grad_out: Sequence, grad_in: Sequence):
+        check(lib().fl_server_backward(self.h, _parr(grad_out), _parr(grad_in)), self.h)
+
+    def step(self, lr: float):
+        check(lib().fl_server_step(self.h, lr), self.h)
+
+    def sync(self):
+        check(lib().fl_server_sync(self.h), self.h)
+
+    def numel(self, tensor_id: int) -> int:
+        return int(lib().fl_server_tensor_numel(self.h, tensor_id))
+
+    def _get(self, fn, block, tensor_id):
+        import numpy as np
+        out = np.empty(self.numel(tensor_id), np.float32)
+        check(fn(self.h, block, tensor_id, out.ctypes.data, out.size), self.h)
+        return out
+
+    def get_param(self, block: int, tensor_id: int):
+        return self._get(lib().fl_server_get_param, block, tensor_id)
+
+    def get_grad(self, block: int, tensor_id: int):
+        return self._get(lib().fl_server_get_grad, block, tensor_id)
+
+    def get_adam_moments(self, block: int, tensor_id: int):
+        import numpy as np
+        n = self.numel(tensor_id)
+        m = np.empty(n, np.float32)
+        v = np.empty(n, np.float32)
+        check(lib().fl_server_get_adam_moments(self.h, block, tensor_id, m.ctypes.data, v.ctypes.data, n), self.h)
+        return m, v
+
+    def set_param(self, block: int, tensor_id: int, values):
+        import numpy as np
+        a = np.ascontiguousarray(values, np.float32).reshape(-1)
+        check(lib().fl_server_set_param(self.h, block, tensor_id, a.ctypes.data, a.size), self.h)
+
+    def profile(self, enable: bool):
+        check(lib().fl_server_profile(self.h, 1 if enable else 0), self.h)
+
+    def profile_read(self) -> dict:
+        n = len(PROF_CLASSES)
+        ms = (C.c_double * n)()
+        cnt = (C.c_int64 * n)()
+        check(lib().fl_server_profile_read(self.h, ms, cnt, n), self.h)
+        return {PROF_CLASSES[i]: (float(ms[i]), int(cnt[i])) for i in range(n)}
+
+    def launch_count(self) -> int:
+        return int(lib().fl_server_launch_count(self.h))
+
+
+# ----------------------------------------------------------------------------- kernel-level calls
+
+def fl_k_gemm(args: fl_gemm_args, status=None, stream=None):
+    check(lib().fl_k_gemm(C.byref(args), ptr(status), stream_ptr(stream)))
+
+
+def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
+         alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
+         status=None, stream=None):
+    a = fl_gemm_args(M, N, K, ptr(A), lda, a_mn, ptr(B), ldb, b_mn, ptr(D), ldd, epilogue, ptr(bias), ptr(aux),
+                     ld_aux, alpha, ptr(aux_out), ld_aux_out, ptr(pos), ptr(rope_tab), n_heads, head_dim, rotary_dim)
+    fl_k_gemm(a, status, stream)
+
+
+def fl_k_layernorm_fwd(T, H, x, gamma, beta, eps, y, mean, rstd, stream=None):
+    check(lib().fl_k_layernorm_fwd(T, H, ptr(x), ptr(gamma), ptr(beta), eps, ptr(y), ptr(mean), ptr(rstd),
+                                   stream_ptr(stream)))
+
+
+def fl_k_layernorm_bwd_workspace(T, H) -> int:
+    return int(lib().fl_k_layernorm_bwd_workspace(T, H))
+
+
+def fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx, dgamma, dbeta, workspace,
+                       stream=None):
+    check(lib().fl_k_layernorm_bwd(T, H, ptr(dy), ptr(x), ptr(mean), ptr(rstd), ptr(gamma), ptr(resid),
+                                   resid_alpha, ptr(dx), ptr(dgamma), ptr(dbeta), ptr(workspace),
+                                   stream_ptr(stream)))
+
+
+def fl_k_attention_tiles(cu_host) -> int:
+    import numpy as np
+    a = np.ascontiguousarray(cu_host, np.int32)
+    return int(lib().fl_k_attention_tiles(a.ctypes.data, a.size - 1))
+
+
+def fl_k_attention_fwd(T, n_heads, head_dim, qkv, cu_host, cu_dev, tile_ws, o, lse, stream=None):
+    import numpy as np
+    a = np.ascontiguousarray(cu_host, np.int32)
+    check(lib().fl_k_attention_fwd(T, n_heads, head_dim, ptr(qkv), a.ctypes.data, ptr(cu_dev), a.size - 1,
+                                   ptr(tile_ws), ptr(o), ptr(lse), stream_ptr(stream)))
+
+
+def fl_k_attention_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_host, cu_dev, tile_ws, delta_ws, rope_tab,
+                       rotary_dim, dqkv, stream=None):
+    import numpy as np
+    a = np.ascontiguousarray(cu_host, np.int32)
+    check(lib().fl_k_attention_bwd(T, n_heads, head_dim, ptr(qkv), ptr(o), ptr(lse), ptr(dout), a.ctypes.data,
+                                   ptr(cu_dev), a.size - 1, ptr(tile_ws), ptr(delta_ws), ptr(rope_tab), rotary_dim,
+                                   ptr(dqkv), stream_ptr(stream)))
+
+
+def fl_k_adamw(n, w, g, m, v, w_bf16, lr, beta1, beta2, eps, weight_decay, bc1, bc2, stream=None):
+    check(lib().fl_k_adamw(n, ptr(w), ptr(g), ptr(m), ptr(v), ptr(w_bf16), lr, beta1, beta2, eps, weight_decay,
+                           bc1, bc2, stream_ptr(stream)))
+
+
+def fl_k_colsum(T, N, x, out, stream=None):
+    check(lib().fl_k_colsum(T, N, ptr(x), ptr(out), stream_ptr(stream)))
+
+
+def fl_k_pack_clients(clients: Sequence, nbytes: Sequence[int], packed, scatter: bool, stream=None):
+    K = len(clients)
+    b = (C.c_int64 * K)(*nbytes)
+    check(lib().fl_k_pack_clients(K, _parr(clients), b, ptr(packed), 1 if scatter else 0, stream_ptr(stream)))

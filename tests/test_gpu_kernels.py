@@ -1,0 +1,268 @@
+"""Kernel-level parity of the CUDA library against the fp64 oracle (GPU only).
+
+Each test calls one kernel through the C ABI of include/flglm_kernels.h on seeded
+inputs that are exactly representable in bf16, and compares with the oracle's
+function of the same step (or, for the plain contractions, with the fp64 product
+that defines them).  Shapes span several tiles and a ragged tail.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import flglm_oracle as O
+from tests._gpu import (bits, dev_bf16, dev_f32, dev_i32, f64, flglm, need_gpu, rel_inf, rnd_bf16_f64,
+                        rope_table)
+
+pytestmark = pytest.mark.gpu
+
+# bf16 output rounding is 2^-9 relative; fp32 accumulation over K adds far less.
+GEMM_TOL = 1e-2
+
+
+@pytest.fixture(scope="module")
+def F():
+    need_gpu()
+    return flglm()
+
+
+def _store(mat: np.ndarray, mn_major: bool):
+    """Device copy of a logical [rows, K] operand: row-major as is (K-major), or its
+    transpose [K, rows] (MN-major).  Returns (tensor, leading dim)."""
+    if mn_major:
+        t = dev_bf16(np.ascontiguousarray(mat.T))
+        return t, mat.shape[0]
+    return dev_bf16(mat), mat.shape[1]
+
+
+@pytest.mark.parametrize("layout", [(0, 0), (0, 1), (1, 1)], ids=["fwd", "dgrad", "wgrad"])
+@pytest.mark.parametrize("shape", [(200, 256, 320), (136, 384, 200), (1000, 1024, 512), (64, 128, 64),
+                                   (8, 256, 4096), (520, 768, 72)])
+def test_gemm_layouts(F, layout, shape):
+    M, N, K = shape
+    a_mn, b_mn = layout
+    rng = np.random.default_rng(M * 7 + N + K + 31 * a_mn + 17 * b_mn)
+    A = rnd_bf16_f64(rng, (M, K))
+    B = rnd_bf16_f64(rng, (N, K))
+    dA, lda = _store(A, bool(a_mn))
+    dB, ldb = _store(B, bool(b_mn))
+    D = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    F.gemm(M, N, K, dA, lda, a_mn, dB, ldb, b_mn, D, N)
+    torch.cuda.synchronize()
+    ref = A @ B.T
+    assert rel_inf(f64(D), ref) < GEMM_TOL
+
+
+def test_gemm_accumulate_f32_repeated(F):
+    """fp32 read-modify-write epilogue (weight gradients accumulate across calls)."""
+    M, N, K = 384, 512, 300
+    rng = np.random.default_rng(5)
+    A = rnd_bf16_f64(rng, (M, K))
+    B = rnd_bf16_f64(rng, (N, K))
+    C0 = rng.standard_normal((M, N)).astype(np.float32)
+    dA, lda = _store(A, True)
+    dB, ldb = _store(B, True)
+    D = dev_f32(C0)
+    for _ in range(2):
+        F.gemm(M, N, K, dA, lda, 1, dB, ldb, 1, D, N, epilogue=F.FL_EPI_ACCUM_F32)
+    torch.cuda.synchronize()
+    ref = C0.astype(np.float64) + 2 * (A @ B.T)
+    assert rel_inf(f64(D), ref) < 1e-5
+
+
+def test_gemm_epilogues(F):
+    M, N, K = 192, 512, 256
+    rng = np.random.default_rng(11)
+    A = rnd_bf16_f64(rng, (M, K))
+    B = rnd_bf16_f64(rng, (N, K), 0.1)
+    bias = rng.standard_normal(N).astype(np.float32)
+    R = rnd_bf16_f64(rng, (M, N))
+    dA, lda = _store(A, False)
+    dB, ldb = _store(B, False)
+    db = dev_f32(bias)
+    dR = dev_bf16(R)
+    acc = A @ B.T
+    alpha = 1.7
+    # bias + gelu, pre-activation kept
+    D = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    U = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_GELU, bias=db, aux_out=U, ld_aux_out=N)
+    torch.cuda.synchronize()
+    u = acc + bias[None, :]
+    assert rel_inf(f64(U), u) < GEMM_TOL
+    assert rel_inf(f64(D), O.gelu(u)) < GEMM_TOL
+    # bias + alpha * residual
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_RESID, bias=db, aux=dR, ld_aux=N,
+           alpha=alpha)
+    torch.cuda.synchronize()
+    assert rel_inf(f64(D), u + alpha * R) < GEMM_TOL
+    # alpha * residual, no bias
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_RESID, aux=dR, ld_aux=N, alpha=alpha)
+    torch.cuda.synchronize()
+    assert rel_inf(f64(D), acc + alpha * R) < GEMM_TOL
+    # gelu' of a stored pre-activation
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_GELU_BWD, aux=dR, ld_aux=N)
+    torch.cuda.synchronize()
+    assert rel_inf(f64(D), acc * O.gelu_grad(R)) < GEMM_TOL
+    # plain store with bias
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_STORE, bias=db)
+    torch.cuda.synchronize()
+    assert rel_inf(f64(D), u) < GEMM_TOL
+
+
+@pytest.mark.parametrize("hd", [64, 128])
+def test_gemm_rope_epilogue(F, hd):
+    nh = 2
+    H = nh * hd
+    M, N, K = 130, 3 * H, 256
+    rng = np.random.default_rng(hd)
+    A = rnd_bf16_f64(rng, (M, K))
+    B = rnd_bf16_f64(rng, (N, K), 0.1)
+    bias = rng.standard_normal(N).astype(np.float32)
+    pos = rng.integers(0, 300, size=M).astype(np.int32)
+    rd = hd // 2
+    tab = rope_table(300, rd, 10000.0)
+    dA, lda = _store(A, False)
+    dB, ldb = _store(B, False)
+    D = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_ROPE, bias=dev_f32(bias),
+           pos=dev_i32(pos), rope_tab=dev_f32(tab), n_heads=nh, head_dim=hd, rotary_dim=rd)
+    torch.cuda.synchronize()
+    qkv = A @ B.T + bias[None, :]
+    cos, sin = O.rope_cos_sin(pos, rd, 10000.0)
+    q = O.rope_rotate(qkv[:, :H].reshape(M, nh, hd), cos, sin, rd).reshape(M, H)
+    k = O.rope_rotate(qkv[:, H:2 * H].reshape(M, nh, hd), cos, sin, rd).reshape(M, H)
+    ref = np.concatenate([q, k, qkv[:, 2 * H:]], axis=1)
+    assert rel_inf(f64(D), ref) < GEMM_TOL
+
+
+@pytest.mark.parametrize("H", [256, 4096])
+def test_layernorm_fwd_bwd(F, H):
+    T = 77
+    rng = np.random.default_rng(H)
+    x = rnd_bf16_f64(rng, (T, H), 2.0) + 0.0
+    g = (1 + 0.2 * rng.standard_normal(H)).astype(np.float32)
+    be = (0.2 * rng.standard_normal(H)).astype(np.float32)
+    dx_, dg_, db_ = dev_bf16(x), dev_f32(g), dev_f32(be)
+    y = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+    mean = torch.empty(T, dtype=torch.float32, device="cuda")
+    rstd = torch.empty(T, dtype=torch.float32, device="cuda")
+    F.fl_k_layernorm_fwd(T, H, dx_, dg_, db_, 1e-5, y, mean, rstd)
+    torch.cuda.synchronize()
+    yr, mur, rsr = O.layer_norm_fwd(x, g.astype(np.float64), be.astype(np.float64), 1e-5)
+    assert rel_inf(f64(y), yr) < 1e-2
+    np.testing.assert_allclose(f64(mean), mur, rtol=0, atol=1e-5)
+    np.testing.assert_allclose(f64(rstd), rsr, rtol=1e-4)
+    # backward, with and without the alpha-scaled residual gradient
+    dy = rnd_bf16_f64(rng, (T, H))
+    res = rnd_bf16_f64(rng, (T, H))
+    ws = torch.empty(F.fl_k_layernorm_bwd_workspace(T, H) // 4 + 64, dtype=torch.float32, device="cuda")
+    for use_res in (False, True):
+        dxo = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+        dgam = dev_f32(np.full(H, 0.5, np.float32))
+        dbet = dev_f32(np.full(H, -0.25, np.float32))
+        F.fl_k_layernorm_bwd(T, H, dev_bf16(dy), dx_, mean, rstd, dg_, dev_bf16(res) if use_res else None, 3.0,
+                             dxo, dgam, dbet, ws)
+        torch.cuda.synchronize()
+        # the oracle backward evaluated at the kernel's own statistics isolates the bwd kernel
+        dxr, dgr, dbr = O.layer_norm_bwd(dy, x, f64(mean), f64(rstd), g.astype(np.float64))
+        if use_res:
+            dxr = dxr + 3.0 * res
+        assert rel_inf(f64(dxo), dxr) < 1e-2
+        assert rel_inf(f64(dgam) - 0.5, dgr) < 1e-4
+        assert rel_inf(f64(dbet) + 0.25, dbr) < 1e-4
+
+
+@pytest.mark.parametrize("hd", [64, 128])
+def test_attention_fwd_bwd(F, hd):
+    seqs = [1, 64, 100, 130, 7, 64, 200]
+    nh = 2
+    H = nh * hd
+    cu = np.cumsum([0] + seqs).astype(np.int32)
+    T = int(cu[-1])
+    rng = np.random.default_rng(hd + 3)
+    qkv = rnd_bf16_f64(rng, (T, 3 * H))
+    do = rnd_bf16_f64(rng, (T, H))
+    dqkv_ = dev_bf16(qkv)
+    dcu = dev_i32(cu)
+    ntiles = F.fl_k_attention_tiles(cu)
+    assert ntiles == sum((L + 63) // 64 for L in seqs)
+    tiles = torch.empty(ntiles * 2, dtype=torch.int32, device="cuda")
+    o = torch.full((T, H), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((nh, T), dtype=torch.float32, device="cuda")
+    F.fl_k_attention_fwd(T, nh, hd, dqkv_, cu, dcu, tiles, o, lse)
+    torch.cuda.synchronize()
+    q = qkv[:, :H].reshape(T, nh, hd)
+    k = qkv[:, H:2 * H].reshape(T, nh, hd)
+    v = qkv[:, 2 * H:].reshape(T, nh, hd)
+    o_ref, lse_ref = O.attention_fwd(q, k, v, cu)
+    assert rel_inf(f64(o), o_ref.reshape(T, H)) < 2e-2
+    np.testing.assert_allclose(f64(lse), lse_ref, rtol=0, atol=2e-2)
+    # backward (inverse rotary rotation folded in, as the server uses it)
+    rd = hd // 2
+    pos = np.concatenate([np.arange(L) for L in seqs]).astype(np.int32)
+    tab = rope_table(256, rd, 10000.0)
+    delta = torch.empty((nh, T), dtype=torch.float32, device="cuda")
+    dq = torch.full((T, 3 * H), float("nan"), dtype=torch.bfloat16, device="cuda")
+    # the kernel differentiates through its own saved O (bf16), as the server does
+    F.fl_k_attention_bwd(T, nh, hd, dqkv_, o, lse, dev_bf16(do), cu, dcu, tiles, delta, dev_f32(tab), rd, dq)
+    torch.cuda.synchronize()
+    dqr, dkr, dvr = O.attention_bwd(do.reshape(T, nh, hd), q, k, v, cu)
+    cos, sin = O.rope_cos_sin(pos, rd, 10000.0)
+    dq_ref = O.rope_rotate(dqr, cos, sin, rd, inverse=True).reshape(T, H)
+    dk_ref = O.rope_rotate(dkr, cos, sin, rd, inverse=True).reshape(T, H)
+    got = f64(dq)
+    assert rel_inf(got[:, :H], dq_ref) < 5e-2
+    assert rel_inf(got[:, H:2 * H], dk_ref) < 5e-2
+    assert rel_inf(got[:, 2 * H:], dvr.reshape(T, H)) < 5e-2
+
+
+def test_adamw(F):
+    n = 4096 + 64
+    rng = np.random.default_rng(9)
+    w = rng.standard_normal(n).astype(np.float32) * 0.02
+    m = np.zeros(n, np.float32)
+    v = np.zeros(n, np.float32)
+    dw, dm, dv = dev_f32(w), dev_f32(m), dev_f32(v)
+    wb = torch.empty(n, dtype=torch.bfloat16, device="cuda")
+    ref_w, ref_m, ref_v = w.astype(np.float64), m.astype(np.float64), v.astype(np.float64)
+    for t in range(1, 4):
+        g = (rng.standard_normal(n) * 1e-3).astype(np.float32)
+        dg = dev_f32(g)
+        F.fl_k_adamw(n, dw, dg, dm, dv, wb, 1e-3, 0.9, 0.999, 1e-8, 0.01, 1 - 0.9 ** t, 1 - 0.999 ** t)
+        torch.cuda.synchronize()
+        ref_w, ref_m, ref_v = O.adamw_update(ref_w, g.astype(np.float64), ref_m, ref_v, t, 1e-3, 0.9, 0.999, 1e-8,
+                                             0.01)
+        assert not f64(dg).any()
+    assert rel_inf(f64(dw), ref_w) < 1e-5
+    assert rel_inf(f64(dm), ref_m) < 1e-5
+    assert rel_inf(f64(dv), ref_v) < 1e-5
+    np.testing.assert_array_equal(bits(wb), bits(dw.to(torch.bfloat16)))
+
+
+def test_colsum(F):
+    T, N = 1000, 768
+    rng = np.random.default_rng(2)
+    x = rnd_bf16_f64(rng, (T, N))
+    out = dev_f32(np.ones(N, np.float32))
+    F.fl_k_colsum(T, N, dev_bf16(x), out)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(f64(out), 1.0 + x.sum(0), rtol=1e-5, atol=1e-4)
+
+
+def test_pack_clients_bitexact(F):
+    rng = np.random.default_rng(4)
+    H = 256
+    lens = [3, 1, 64, 17, 200]
+    clients = [dev_bf16(rnd_bf16_f64(rng, (2, L, H))) for L in lens]
+    nbytes = [c.numel() * 2 for c in clients]
+    packed = torch.empty(sum(c.numel() for c in clients), dtype=torch.bfloat16, device="cuda")
+    F.fl_k_pack_clients(clients, nbytes, packed, scatter=False)
+    back = [torch.empty_like(c) for c in clients]
+    F.fl_k_pack_clients(back, nbytes, packed, scatter=True)
+    torch.cuda.synchronize()
+    want = np.concatenate([bits(c).reshape(-1) for c in clients])
+    np.testing.assert_array_equal(bits(packed), want)
+    for a, b in zip(back, clients):
+        np.testing.assert_array_equal(bits(a), bits(b))

@@ -1,0 +1,188 @@
+"""Server-level parity: fl_server_create/forward/backward/step on the GPU against the
+fp64 oracle server (GPU only).
+
+Tolerances (per tensor, ||gpu - oracle||_inf / ||oracle||_inf): output states 2e-2,
+input-state and weight gradients 5e-2, weights after one AdamW step 1e-3.  Packing,
+unpacking and segment indexing are bit-exact (client-batching invariant on the GPU).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synthetic as syn
+from oracle import flglm_oracle as O
+from tests._gpu import bits, dev_bf16_from_bits, f64, flglm, need_gpu, rel_inf
+
+pytestmark = pytest.mark.gpu
+
+OUT_TOL, GRAD_TOL, W_TOL = 2e-2, 5e-2, 1e-3
+
+
+@pytest.fixture(scope="module")
+def F():
+    need_gpu()
+    return flglm()
+
+
+def make_server(F, cfg, max_tokens=None, seed=None):
+    mt = max_tokens or cfg.tokens
+    return F.Server(F.make_cfg(cfg, mt), cfg.seed if seed is None else seed)
+
+
+def run_gpu(F, srv, cfg, states_bits, grads_bits):
+    states = [dev_bf16_from_bits(s) for s in states_bits]
+    outs = [torch.empty_like(s) for s in states]
+    srv.forward(states, cfg.seq_lens, outs)
+    gouts = [dev_bf16_from_bits(g) for g in grads_bits]
+    gins = [torch.empty_like(s) for s in states]
+    srv.backward(gouts, gins)
+    srv.sync()
+    return outs, gins
+
+
+def test_create_init_matches_generator(F):
+    cfg = syn.CONFIGS["tiny"]
+    srv = make_server(F, cfg)
+    for t in range(12):
+        got = srv.get_param(0, t)
+        want = syn.init_tensor(cfg, 0, t).reshape(-1)
+        # device and host libm may differ by an ulp in double before the fp32 rounding
+        ulps = np.abs(got.view(np.int32).astype(np.int64) - want.view(np.int32).astype(np.int64))
+        assert ulps.max() <= 1, (t, ulps.max())
+        assert (ulps == 0).mean() > 0.999
+    srv.close()
+
+
+def parity_case(F, cfg, check_step=True):
+    params = syn.init_params(cfg)
+    srv = make_server(F, cfg)
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            srv.set_param(b, t, params[b][t])
+    states = syn.client_states(cfg)
+    grads = syn.client_grads(cfg)
+    outs, gins = run_gpu(F, srv, cfg, states, grads)
+    ref = O.OracleServer(cfg, params)
+    ro = ref.forward([syn.bf16_bits_to_f64(s) for s in states])
+    rg = ref.backward([syn.bf16_bits_to_f64(g) for g in grads])
+    for k in range(cfg.K):
+        assert rel_inf(f64(outs[k]), ro[k]) < OUT_TOL, ("out", k, rel_inf(f64(outs[k]), ro[k]))
+        assert rel_inf(f64(gins[k]), rg[k]) < GRAD_TOL, ("grad_in", k, rel_inf(f64(gins[k]), rg[k]))
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            g = srv.get_grad(b, t)
+            e = rel_inf(g, ref.grads[b][t].reshape(-1))
+            assert e < GRAD_TOL, ("wgrad", b, syn.TENSOR_NAMES[t], e)
+    if check_step:
+        srv.step(cfg.lr)
+        ref.step(cfg.lr)
+        srv.sync()
+        for b in range(cfg.n_blocks):
+            for t in range(12):
+                w = srv.get_param(b, t)
+                assert rel_inf(w, ref.params[b][t].reshape(-1)) < W_TOL
+                # the update itself: first Adam step is lr * sign(g) where |g| >> eps
+                dw = w.astype(np.float64) - params[b][t].reshape(-1)
+                dref = ref.params[b][t].reshape(-1) - params[b][t].reshape(-1).astype(np.float64)
+                assert np.mean(np.abs(dw - dref)) < 0.05 * cfg.lr, (b, t)
+                m, v = srv.get_adam_moments(b, t)
+                assert rel_inf(m, ref.m[b][t].reshape(-1)) < GRAD_TOL
+                assert not srv.get_grad(b, t).any()
+    srv.close()
+
+
+@pytest.mark.parametrize("rfl", [1, 0], ids=["glm_block", "pre_ln"])
+def test_tiny_config_parity(F, rfl):
+    parity_case(F, syn.CONFIGS["tiny"].with_(residual_from_ln=rfl))
+
+
+def test_ragged_small_parity(F):
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, client_batch=1, seq_lens=(1, 17, 64, 65, 130, 3))
+    parity_case(F, cfg)
+
+
+def test_block6b_parity(F):
+    """One ChatGLM-6B-shaped block (H 4096, 32 x 128, F 16384), K=4 x 512, full size."""
+    parity_case(F, syn.CONFIGS["block6b"], check_step=True)
+
+
+def test_client_batching_invariant_bitexact(F):
+    """§3.3 stacks clients without mixing them: each client's outputs and input gradients
+    from the packed call equal (bit for bit) those of calling the server with that client
+    alone; the packed weight gradients equal the sum of the per-client ones."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, client_batch=2, seq_lens=(64, 20, 130))
+    states = syn.client_states(cfg)
+    grads = syn.client_grads(cfg)
+    srv = make_server(F, cfg)
+    outs, gins = run_gpu(F, srv, cfg, states, grads)
+    gsum = [[np.zeros(srv.numel(t)) for t in range(12)] for _ in range(cfg.n_blocks)]
+    packed_g = [[srv.get_grad(b, t).astype(np.float64) for t in range(12)] for b in range(cfg.n_blocks)]
+    srv.close()
+    for k in range(cfg.K):
+        c1 = cfg.with_(seq_lens=(cfg.seq_lens[k],))
+        s1 = make_server(F, c1, max_tokens=cfg.tokens, seed=cfg.seed)
+        o1, g1 = run_gpu(F, s1, c1, [states[k]], [grads[k]])
+        np.testing.assert_array_equal(bits(o1[0]), bits(outs[k]))
+        np.testing.assert_array_equal(bits(g1[0]), bits(gins[k]))
+        for b in range(cfg.n_blocks):
+            for t in range(12):
+                gsum[b][t] += s1.get_grad(b, t)
+        s1.close()
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            assert rel_inf(packed_g[b][t], gsum[b][t]) < 1e-3
+
+
+def test_serial_accumulation_and_state_errors(F):
+    """Serial strategy (§3.3): forward/backward per client without a step accumulates the
+    weight gradients; protocol-order violations are reported as FL_ERR_STATE."""
+    cfg = syn.CONFIGS["tiny"]
+    srv = make_server(F, cfg)
+    dummy = [torch.empty((cfg.client_batch, cfg.seq_lens[0], cfg.hidden), dtype=torch.bfloat16, device="cuda")]
+    with pytest.raises(F.FlError) as ei:
+        srv.backward(dummy, dummy)
+    assert ei.value.code == -3
+    states = syn.client_states(cfg)
+    grads = syn.client_grads(cfg)
+    for k in range(cfg.K):
+        ck = cfg.with_(seq_lens=(cfg.seq_lens[k],))
+        run_gpu(F, srv, ck, [states[k]], [grads[k]])
+    ser = [srv.get_grad(0, t) for t in range(12)]
+    srv.close()
+    srv2 = make_server(F, cfg)
+    run_gpu(F, srv2, cfg, states, grads)
+    for t in range(12):
+        assert rel_inf(ser[t], srv2.get_grad(0, t)) < 1e-3
+    # step while a forward is pending
+    st = [dev_bf16_from_bits(s) for s in states]
+    outs = [torch.empty_like(s) for s in st]
+    srv2.forward(st, cfg.seq_lens, outs)
+    with pytest.raises(F.FlError) as ei:
+        srv2.step(1e-4)
+    assert ei.value.code == -3
+    with pytest.raises(F.FlError) as ei:
+        srv2.forward(st, cfg.seq_lens, outs)
+    assert ei.value.code == -3
+    srv2.close()
+
+
+def test_argument_errors(F):
+    cfg = syn.CONFIGS["tiny"]
+    srv = make_server(F, cfg, max_tokens=256)
+    st = [torch.empty((2, 64, 256), dtype=torch.bfloat16, device="cuda") for _ in range(3)]
+    with pytest.raises(F.FlError) as ei:      # 3 x 2 x 64 = 384 tokens > 256
+        srv.forward(st, [64, 64, 64], st)
+    assert ei.value.code == -2
+    with pytest.raises(F.FlError) as ei:
+        srv.forward(st[:1], [0], st[:1])
+    assert ei.value.code == -1
+    base = torch.empty(2 * 64 * 256 + 8, dtype=torch.bfloat16, device="cuda")
+    mis = base[1:1 + 2 * 64 * 256]            # 2-byte offset: not 16-byte aligned
+    with pytest.raises(F.FlError) as ei:
+        srv.forward([mis], [64], [st[0]])
+    assert ei.value.code == -1
+    with pytest.raises(F.FlError) as ei:
+        srv.forward([], [], [])
+    assert ei.value.code == -1
+    srv.sync()
+    srv.close()
