@@ -26,6 +26,8 @@ from this text):
         r = sqrt(-2 ln U(key, 2j));  phi = 2 pi U(key, 2j + 1)
         z = r cos(phi) if i is even else r sin(phi)
         value = float32(mean + std * z)   (bf16 inputs: then narrowed RNE to bf16)
+    (the weight init uses std = the fp32 value of init_std, which is what the C ABI's
+    float field carries)
     ragged length k (seed 7 in the ragged workload):
         L_k = 64 + raw(key(seed, LENGTHS), k) mod 961        in [64, 1024]
 """
@@ -208,7 +210,7 @@ def init_tensor(cfg: ServerConfig, block: int, tensor: int, seed: Optional[int] 
     if tensor in (T_BE1, T_BE2):
         return np.zeros(shape, np.float32)
     key = stream_key(seed, P_WEIGHTS, block, tensor)
-    return normal_f32(key, n, 0.0, cfg.init_std).reshape(shape)
+    return normal_f32(key, n, 0.0, float(np.float32(cfg.init_std))).reshape(shape)
 
 
 def init_params(cfg: ServerConfig, seed: Optional[int] = None) -> List[List[np.ndarray]]:

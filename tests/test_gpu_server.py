@@ -53,6 +53,28 @@ def test_create_init_matches_generator(F):
     srv.close()
 
 
+def check_updated_weights(w, w_ref, w0, g_ref, lr, where):
+    """Weights after one AdamW step.  The first Adam step moves each weight by about
+    lr * sign(g), a jump at g = 0, so an element whose reference gradient is below the
+    gradient precision may legitimately move the other way.  Some gradients are zero in
+    exact arithmetic (the key bias on the un-rotated dims only shifts every score of a
+    row by the same amount, which softmax ignores), so their sign is rounding noise.
+    The 1e-3 bound applies to elements whose gradient is resolved (>= the gradient
+    tolerance x max); elements with a significant gradient (>= 1e-2 x max) must move the
+    same way (under 2% flipped, mean update error under 5% of lr)."""
+    w = w.astype(np.float64)
+    den = np.abs(w_ref).max()
+    gmax = max(np.abs(g_ref).max(), 1e-30)
+    resolved = np.abs(g_ref) >= GRAD_TOL * gmax
+    if resolved.any():
+        assert np.abs(w - w_ref)[resolved].max() / den < W_TOL, where
+    significant = np.abs(g_ref) >= 1e-2 * gmax
+    if significant.any():
+        err = np.abs((w - w0) - (w_ref - w0.astype(np.float64)))[significant]
+        assert np.mean(err) < 0.05 * lr, (where, np.mean(err) / lr)
+        assert np.mean(err > lr) < 0.02, (where, np.mean(err > lr))
+
+
 def parity_case(F, cfg, check_step=True):
     params = syn.init_params(cfg)
     srv = make_server(F, cfg)
@@ -74,17 +96,14 @@ def parity_case(F, cfg, check_step=True):
             e = rel_inf(g, ref.grads[b][t].reshape(-1))
             assert e < GRAD_TOL, ("wgrad", b, syn.TENSOR_NAMES[t], e)
     if check_step:
+        gref = [[ref.grads[b][t].reshape(-1).copy() for t in range(12)] for b in range(cfg.n_blocks)]
         srv.step(cfg.lr)
         ref.step(cfg.lr)
         srv.sync()
         for b in range(cfg.n_blocks):
             for t in range(12):
-                w = srv.get_param(b, t)
-                assert rel_inf(w, ref.params[b][t].reshape(-1)) < W_TOL
-                # the update itself: first Adam step is lr * sign(g) where |g| >> eps
-                dw = w.astype(np.float64) - params[b][t].reshape(-1)
-                dref = ref.params[b][t].reshape(-1) - params[b][t].reshape(-1).astype(np.float64)
-                assert np.mean(np.abs(dw - dref)) < 0.05 * cfg.lr, (b, t)
+                check_updated_weights(srv.get_param(b, t), ref.params[b][t].reshape(-1),
+                                      params[b][t].reshape(-1), gref[b][t], cfg.lr, (b, t))
                 m, v = srv.get_adam_moments(b, t)
                 assert rel_inf(m, ref.m[b][t].reshape(-1)) < GRAD_TOL
                 assert not srv.get_grad(b, t).any()
