@@ -1,0 +1,421 @@
+"""Throughput of the client-batched FL-GLM server step on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload stack26] [--impl reference]
+
+A step is one pass of the whole server hot path for one call: pack the K clients'
+hidden states, forward through the block stack, unpack; pack the output-state
+gradients, backward through the stack (input-state and weight gradients), unpack;
+one AdamW update.  `value` is tokens/s of the whole job with the inputs resident in
+HBM; `e2e` repeats the measurement through host (pinned) buffers with the
+host<->device copies of every step inside the timed region.  The default workload is
+the 26-block ChatGLM-6B-shaped server stack with K=8 clients x 4 rows x 256 tokens.
+
+Under torchrun (N > 1) each rank runs an independent replica of the server (the path
+is one GPU; there is no collective on the data path) and `value` counts every rank's
+tokens over the slowest rank's time.
+
+--impl reference times the fp64 CPU oracle on a bounded sample of the same workload
+(the repository's reference arm; rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synthetic as syn  # noqa: E402
+
+METRIC = "server fwd+bwd tokens/s, client-batched GLM stack bf16; % of BF16 peak"
+
+
+def workload(name: str) -> syn.ServerConfig:
+    if name.startswith("sweep26_K"):
+        return syn.sweep_config(int(name[len("sweep26_K"):]))
+    return syn.CONFIGS[name]
+
+
+def describe(cfg: syn.ServerConfig) -> str:
+    lens = sorted(set(cfg.seq_lens))
+    L = f"{lens[0]}" if len(lens) == 1 else f"{min(lens)}..{max(lens)} (ragged)"
+    return (f"{cfg.name}: {cfg.n_blocks} GLM blocks, hidden {cfg.hidden}, {cfg.n_heads} heads x {cfg.head_dim}, "
+            f"FFN {cfg.ffn_hidden}, K={cfg.K} clients x {cfg.client_batch} rows x {L} tokens, T={cfg.tokens}")
+
+
+def gemm_flops(cfg: syn.ServerConfig) -> float:
+    """Dense contractions of one fwd+bwd: forward 2T(3H^2 + H^2 + 2HF) per block, data
+    and weight gradients the same again each."""
+    H, F, T = cfg.hidden, cfg.ffn_hidden, cfg.tokens
+    return float(cfg.n_blocks * 3 * 2 * T * (4 * H * H + 2 * H * F))
+
+
+def attn_flops(cfg: syn.ServerConfig) -> float:
+    """Causal attention: 2 H L (L+1) forward and 2.5x that backward, per segment per block."""
+    return float(cfg.n_blocks * sum(7 * cfg.hidden * L * (L + 1) for L in cfg.segment_lengths))
+
+
+def peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16": d["bf16_tflops"], "bf16_sustained": d["bf16_tflops_sustained"],
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+    Q = ("index,pci.bus_id,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, bus_id: str | None):
+        self.bus_id = bus_id
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            cmd = ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.bus_id:
+                cmd += ["-i", self.bus_id]
+            self.proc = subprocess.Popen(cmd, stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = [l.split(", ") for l in open(self.path).read().strip().splitlines() if l.strip()]
+        os.unlink(self.path)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            if len(r) < 10:
+                continue
+            try:
+                sm.append(float(r[2]))
+                mx.append(float(r[3]))
+            except ValueError:
+                continue
+            for i, n in enumerate(names):
+                if r[6 + i].strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- oracle CPU sample
+
+class OracleSample:
+    """Times the fp64 oracle on a bounded sample of `cfg`'s step: forward + backward of one
+    block at the workload's shapes over `tokens` tokens (segments of the workload's first
+    length), and one AdamW update over 1/ADAM_FRACTION of that block's parameters.  The
+    full step is estimated as n_blocks x (t_fwd_bwd x T / tokens + t_adamw x ADAM_FRACTION)."""
+    ADAM_FRACTION = 16
+
+    def __init__(self, cfg: syn.ServerConfig, tokens: int, seed: int = 0):
+        from oracle import flglm_oracle as O
+        self.O = O
+        self.cfg = cfg
+        rng = np.random.default_rng(seed)
+        L = cfg.segment_lengths[0]
+        self.nseg = max(1, tokens // L)
+        self.L = L
+        self.one = cfg.with_(n_blocks=1, client_batch=1, seq_lens=(L,) * self.nseg)
+        params = [[cfg.init_std * rng.standard_normal(s) for s in syn.param_shapes(self.one)]]
+        for t, v in ((syn.T_G1, 1.0), (syn.T_G2, 1.0), (syn.T_BE1, 0.0), (syn.T_BE2, 0.0)):
+            params[0][t][:] = v
+        self.params = params
+        self.states = [rng.standard_normal((1, L, cfg.hidden)) for _ in range(self.nseg)]
+        self.grads = [1e-3 * rng.standard_normal((1, L, cfg.hidden)) for _ in range(self.nseg)]
+        n = sum(p.size for p in params[0]) // self.ADAM_FRACTION
+        self.adam = [rng.standard_normal(n) * 0.02, rng.standard_normal(n) * 1e-3, np.zeros(n), np.zeros(n)]
+
+    def run(self) -> dict:
+        cfg, O = self.cfg, self.O
+        srv = O.OracleServer(self.one, self.params)
+        t0 = time.perf_counter()
+        srv.forward(self.states)
+        srv.backward(self.grads)
+        t1 = time.perf_counter()
+        w, g, m, v = self.adam
+        O.adamw_update(w, g, m, v, 1, cfg.lr, cfg.adam_beta1, cfg.adam_beta2, cfg.adam_eps, cfg.weight_decay)
+        t2 = time.perf_counter()
+        sample_tokens = self.nseg * self.L
+        t_step = cfg.n_blocks * ((t1 - t0) * cfg.tokens / sample_tokens + (t2 - t1) * self.ADAM_FRACTION)
+        return {"t_fwd_bwd_s": t1 - t0, "t_adamw_s": t2 - t1, "sample_tokens": sample_tokens,
+                "t_step_s": t_step, "tokens_per_s": cfg.tokens / t_step,
+                "sample": (f"1 of {cfg.n_blocks} blocks at the workload's shapes, {self.nseg} segment(s) x {self.L} "
+                           f"tokens fwd+bwd, plus AdamW over 1/{self.ADAM_FRACTION} of that block's parameters; "
+                           f"fp64 numpy; full step estimated as n_blocks x (t_fwd_bwd x {cfg.tokens}/"
+                           f"{sample_tokens} + t_adamw x {self.ADAM_FRACTION})")}
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args, cfg: syn.ServerConfig):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    sample = OracleSample(cfg, min(cfg.tokens, args.ref_tokens))
+    for _ in range(args.warmup):
+        sample.run()
+    ts, last = [], None
+    for _ in range(args.steps):
+        last = sample.run()
+        ts.append(last["t_step_s"])
+    t = statistics.mean(ts)
+    value = cfg.tokens / t
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": describe(cfg), "global_batch": cfg.tokens,
+                       "seq_len": max(cfg.seq_lens), "parallelism": "cpu"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+                             "sample": last["sample"]},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="stack26")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the oracle sample")
+    ap.add_argument("--ref-tokens", type=int, default=256, help="tokens of the reference-arm sample")
+    ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_dram_traffic.json"))
+    args = ap.parse_args()
+    cfg = workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, cfg)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+
+    # oracle CPU sample first (rank 0, one GPU): no CUDA context exists yet
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        sample = OracleSample(cfg, min(cfg.tokens, args.cpu_tokens))
+        sample.run()
+        cpu = sample.run()
+        del sample
+
+    import torch
+    import torch.distributed as dist
+    from paper_2406_14898_gb300 import flglm as F
+
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    dev = torch.device("cuda", local_rank)
+    F.lib()
+    stream = torch.cuda.Stream(device=dev)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens)), cfg.seed, stream=stream)
+
+    states_bits = syn.client_states(cfg)
+    grads_bits = syn.client_grads(cfg)
+
+    def to_dev(b):
+        return torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev)
+
+    states = [to_dev(s) for s in states_bits]
+    gouts = [to_dev(g) for g in grads_bits]
+    outs = [torch.empty_like(s) for s in states]
+    gins = [torch.empty_like(s) for s in states]
+    torch.cuda.synchronize()
+
+    def step():
+        srv.forward(states, cfg.seq_lens, outs)
+        srv.backward(gouts, gins)
+        srv.step(cfg.lr)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(x: float) -> float:
+        if world == 1:
+            return x
+        t = torch.tensor([x], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    for _ in range(args.warmup):
+        step()
+    srv.sync()
+
+    # ---- device-resident timed region
+    clocks = ClockSampler(pci_bus_id(torch, dev))
+    clocks.start()
+    srv.profile(True)
+    l0 = srv.launch_count()
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    srv.sync()
+    torch.cuda.synchronize()
+    barrier()
+    ms = e0.elapsed_time(e1)
+    launches = srv.launch_count() - l0
+    prof = srv.profile_read()
+    srv.profile(False)
+    clk = clocks.stop()
+    ms = max_over_ranks(ms)
+    ms_step = ms / args.steps
+    value = world * cfg.tokens * args.steps / (ms / 1e3)
+
+    # fwd+bwd only (AdamW excluded) from the per-class event totals
+    adam_ms = prof["adamw"][0] / args.steps
+    fb_ms = ms_step - adam_ms
+    pk = peaks()
+    flops = gemm_flops(cfg) + attn_flops(cfg)
+    gemm_ms, gemm_n = prof["gemm"]
+    gemm_per_launch_flops = gemm_flops(cfg) * args.steps / max(gemm_n, 1)
+    achieved = gemm_per_launch_flops / (gemm_ms / max(gemm_n, 1) / 1e3) / 1e12
+    traffic = None
+    if os.path.exists(args.ncu_traffic):
+        try:
+            tr = json.load(open(args.ncu_traffic))
+            if tr.get("workload") == cfg.name and tr.get("kernel_version") == kernel_version():
+                traffic = tr.get("bytes_per_launch")
+        except Exception:
+            traffic = None
+
+    # ---- end to end through host buffers (pinned), copies inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        h_states = [torch.from_numpy(s.view(np.int16)).view(torch.bfloat16).pin_memory() for s in states_bits]
+        h_gouts = [torch.from_numpy(g.view(np.int16)).view(torch.bfloat16).pin_memory() for g in grads_bits]
+        h_outs = [torch.empty(s.shape, dtype=torch.bfloat16).pin_memory() for s in states_bits]
+        h_gins = [torch.empty(s.shape, dtype=torch.bfloat16).pin_memory() for s in states_bits]
+
+        def e2e_step():
+            with torch.cuda.stream(stream):
+                for d, h in zip(states, h_states):
+                    d.copy_(h, non_blocking=True)
+                srv.forward(states, cfg.seq_lens, outs)
+                for h, d in zip(h_outs, outs):
+                    h.copy_(d, non_blocking=True)
+                for d, h in zip(gouts, h_gouts):
+                    d.copy_(h, non_blocking=True)
+                srv.backward(gouts, gins)
+                for h, d in zip(h_gins, gins):
+                    h.copy_(d, non_blocking=True)
+                srv.step(cfg.lr)
+
+        for _ in range(2):
+            e2e_step()
+        srv.sync()
+        barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        e0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        e1.record(stream)
+        srv.sync()
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        barrier()
+        ems = max_over_ranks(max(e0.elapsed_time(e1), 1e3 * wall))
+        nbytes = sum(s.nbytes for s in states_bits)
+        e2e = {"value": world * cfg.tokens * args.steps / (ems / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": 2 * nbytes, "d2h_bytes_per_step": 2 * nbytes,
+               "ms_per_step": ems / args.steps}
+
+    srv.close()
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,0.02) weights, N(0,1) states, "
+                                                       "N(0,1e-3) output-state grads)",
+            "config": {"workload": describe(cfg), "global_batch": world * cfg.tokens, "seq_len": max(cfg.seq_lens),
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "l2": "working set (~125 GB of weights, optimizer state and activations) is far larger "
+                             "than L2; no flush needed",
+                       "step": "pack + forward + unpack + backward + AdamW"},
+            "pct_bf16_peak": 100.0 * flops / (ms_step / 1e3) / (pk["bf16_sustained"] * 1e12),
+            "pct_bf16_peak_basis": f"algorithmic FLOPs (GEMM + causal attention) of the whole step over the "
+                                   f"{pk['source']} sustained bf16 peak {pk['bf16_sustained']} TFLOP/s",
+            "fwd_bwd_tokens_per_s": world * cfg.tokens / (fb_ms / 1e3),
+            "fwd_bwd_ms": fb_ms, "adamw_ms": adam_ms,
+            "kernel_ms_per_step": {k: v[0] / args.steps for k, v in prof.items()},
+            "roofline": {"kernel": "gemm_tc_kernel (tcgen05)", "bound": "tensor", "achieved": achieved,
+                         "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
+                         "peak_basis": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
+                         "traffic": traffic, "launches_per_step": gemm_n / args.steps,
+                         "share_of_step": gemm_ms / ms},
+            "gpu_launches": launches,
+            "clocks": clk,
+        }
+        if cpu is not None:
+            line["cpu_baseline"] = {"value": cpu["tokens_per_s"], "unit": "tokens/s", "cores": cpu_cores(),
+                                    "kind": "oracle", "sample": cpu["sample"]}
+        if e2e is not None:
+            line["e2e"] = e2e
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def pci_bus_id(torch, dev):
+    """nvidia-smi id (domain:bus:device.function) of the CUDA device, or None."""
+    try:
+        p = torch.cuda.get_device_properties(dev)
+        return f"{p.pci_domain_id:08X}:{p.pci_bus_id:02X}:{p.pci_device_id:02X}.0"
+    except Exception:
+        return None
+
+
+def kernel_version() -> str:
+    """Fingerprint of the GEMM source, so that stored ncu traffic is used only for the
+    kernel it was measured on."""
+    import hashlib
+    src = open(os.path.join(ROOT, "paper_2406_14898_gb300", "csrc", "gemm_tc.cu"), "rb").read()
+    return hashlib.sha256(src).hexdigest()[:16]
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,157 @@
+"""Per-kernel timing of the server's hot-path kernels at a workload's shapes.
+
+    python -m paper_2406_14898_gb300.kernel_bench [--workload stack26] [--kernel all|<name>] [--reps 5]
+
+Each kernel runs on random device buffers (uninitialised values are never read: every
+input is filled first) with CUDA events around `reps` launches on one stream, after one
+warm-up launch.  Prints one JSON line per kernel with its algorithmic work (FLOPs for
+the contractions, bytes for the row kernels), mean time and achieved rate.  The inputs
+of every GEMM here are larger than L2 at the ChatGLM-6B shapes.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def gemm_cases(cfg):
+    """(name, M, N, K, a_mn, b_mn, epilogue) of the 12 GEMMs of one block, T tokens."""
+    from paper_2406_14898_gb300 import flglm as F
+    T, H, Fh = cfg.tokens, cfg.hidden, cfg.ffn_hidden
+    return [
+        ("qkv_fwd", T, 3 * H, H, 0, 0, F.FL_EPI_BIAS_ROPE),
+        ("dense_fwd", T, H, H, 0, 0, F.FL_EPI_BIAS_RESID),
+        ("up_fwd", T, Fh, H, 0, 0, F.FL_EPI_BIAS_GELU),
+        ("down_fwd", T, H, Fh, 0, 0, F.FL_EPI_BIAS_RESID),
+        ("down_dgrad", T, Fh, H, 0, 1, F.FL_EPI_GELU_BWD),
+        ("down_wgrad", H, Fh, T, 1, 1, F.FL_EPI_ACCUM_F32),
+        ("up_dgrad", T, H, Fh, 0, 1, F.FL_EPI_RESID),
+        ("up_wgrad", Fh, H, T, 1, 1, F.FL_EPI_ACCUM_F32),
+        ("dense_dgrad", T, H, H, 0, 1, F.FL_EPI_STORE),
+        ("dense_wgrad", H, H, T, 1, 1, F.FL_EPI_ACCUM_F32),
+        ("qkv_dgrad", T, H, 3 * H, 0, 1, F.FL_EPI_RESID),
+        ("qkv_wgrad", 3 * H, H, T, 1, 1, F.FL_EPI_ACCUM_F32),
+    ]
+
+
+def main():
+    import numpy as np
+    import torch
+
+    import synthetic as syn
+    from paper_2406_14898_gb300 import flglm as F
+
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--workload", default="stack26")
+    ap.add_argument("--kernel", default="all")
+    ap.add_argument("--reps", type=int, default=5)
+    args = ap.parse_args()
+    cfg = syn.CONFIGS[args.workload]
+    F.lib()
+    dev = torch.device("cuda", 0)
+    st = torch.cuda.Stream(device=dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g = torch.Generator(device=dev)
+    g.manual_seed(0)
+
+    def rnd(*shape, scale=1.0, dtype=torch.bfloat16):
+        return (torch.randn(*shape, device=dev, generator=g) * scale).to(dtype)
+
+    def timed(fn):
+        with torch.cuda.stream(st):
+            fn()
+            torch.cuda.synchronize()
+            ev0.record(st)
+            for _ in range(args.reps):
+                fn()
+            ev1.record(st)
+        torch.cuda.synchronize()
+        return ev0.elapsed_time(ev1) / args.reps
+
+    T, H, Fh, nh, hd = cfg.tokens, cfg.hidden, cfg.ffn_hidden, cfg.n_heads, cfg.head_dim
+    out = []
+    for (name, M, N, K, amn, bmn, epi) in gemm_cases(cfg):
+        if args.kernel not in ("all", "gemm", name):
+            continue
+        A = rnd(K, M, scale=0.1) if amn else rnd(M, K, scale=0.1)
+        B = rnd(K, N, scale=0.1) if bmn else rnd(N, K, scale=0.1)
+        D = torch.zeros(M, N, device=dev, dtype=torch.float32 if epi == F.FL_EPI_ACCUM_F32 else torch.bfloat16)
+        kw = {}
+        if epi in (F.FL_EPI_BIAS_ROPE, F.FL_EPI_BIAS_RESID, F.FL_EPI_BIAS_GELU):
+            kw["bias"] = rnd(N, dtype=torch.float32)
+        if epi in (F.FL_EPI_BIAS_RESID, F.FL_EPI_RESID, F.FL_EPI_GELU_BWD):
+            kw["aux"] = rnd(M, N)
+            kw["ld_aux"] = N
+            kw["alpha"] = 1.5
+        if epi == F.FL_EPI_BIAS_GELU:
+            kw["aux_out"] = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+            kw["ld_aux_out"] = N
+        if epi == F.FL_EPI_BIAS_ROPE:
+            L = max(cfg.seq_lens)
+            kw["pos"] = (torch.arange(M, device=dev, dtype=torch.int32) % L)
+            kw["rope_tab"] = rnd(L, hd // 4, 2, dtype=torch.float32)
+            kw.update(n_heads=nh, head_dim=hd, rotary_dim=hd // 2)
+        lda = M if amn else K
+        ldb = N if bmn else K
+        ms = timed(lambda: F.gemm(M, N, K, A, lda, amn, B, ldb, bmn, D, N, epilogue=epi, stream=st, **kw))
+        flops = 2.0 * M * N * K
+        out.append({"kernel": f"gemm_{name}", "M": M, "N": N, "K": K, "ms": ms, "tflops": flops / ms / 1e9})
+        del A, B, D, kw
+    if args.kernel in ("all", "attention"):
+        seqs = cfg.segment_lengths
+        cu = np.cumsum([0] + list(seqs)).astype(np.int32)
+        qkv = rnd(T, 3 * H)
+        o = torch.empty(T, H, device=dev, dtype=torch.bfloat16)
+        lse = torch.empty(nh, T, device=dev, dtype=torch.float32)
+        tiles = torch.empty(2 * F.fl_k_attention_tiles(cu), device=dev, dtype=torch.int32)
+        dcu = torch.from_numpy(cu).to(dev)
+        fl = float(sum(2 * H * L * (L + 1) for L in seqs))
+        ms = timed(lambda: F.fl_k_attention_fwd(T, nh, hd, qkv, cu, dcu, tiles, o, lse, stream=st))
+        out.append({"kernel": "attention_fwd", "T": T, "ms": ms, "tflops": fl / ms / 1e9})
+        do = rnd(T, H)
+        delta = torch.empty(nh, T, device=dev, dtype=torch.float32)
+        dqkv = torch.empty(T, 3 * H, device=dev, dtype=torch.bfloat16)
+        tab = rnd(max(seqs), hd // 4, 2, dtype=torch.float32)
+        ms = timed(lambda: F.fl_k_attention_bwd(T, nh, hd, qkv, o, lse, do, cu, dcu, tiles, delta, tab, hd // 2, dqkv,
+                                                stream=st))
+        out.append({"kernel": "attention_bwd", "T": T, "ms": ms, "tflops": 2.5 * fl / ms / 1e9})
+    if args.kernel in ("all", "layernorm"):
+        x = rnd(T, H)
+        gm = rnd(H, dtype=torch.float32)
+        bt = rnd(H, dtype=torch.float32)
+        y = torch.empty_like(x)
+        mean = torch.empty(T, device=dev, dtype=torch.float32)
+        rstd = torch.empty(T, device=dev, dtype=torch.float32)
+        ms = timed(lambda: F.fl_k_layernorm_fwd(T, H, x, gm, bt, 1e-5, y, mean, rstd, stream=st))
+        nbytes = 2 * T * H * 2 + 8 * T
+        out.append({"kernel": "layernorm_fwd", "ms": ms, "gbs": nbytes / ms / 1e6})
+        dy = rnd(T, H)
+        dx = torch.empty_like(x)
+        ws = torch.empty(F.fl_k_layernorm_bwd_workspace(T, H) // 4 + 64, device=dev, dtype=torch.float32)
+        dg = torch.zeros(H, device=dev, dtype=torch.float32)
+        db = torch.zeros(H, device=dev, dtype=torch.float32)
+        ms = timed(lambda: F.fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gm, None, 0.0, dx, dg, db, ws, stream=st))
+        nbytes = 3 * T * H * 2 + 8 * T
+        out.append({"kernel": "layernorm_bwd", "ms": ms, "gbs": nbytes / ms / 1e6})
+    if args.kernel in ("all", "adamw"):
+        n = syn.params_per_block(cfg) // 4 * 4
+        w = rnd(n, dtype=torch.float32)
+        gr = rnd(n, dtype=torch.float32)
+        m = torch.zeros(n, device=dev, dtype=torch.float32)
+        v = torch.zeros(n, device=dev, dtype=torch.float32)
+        wb = torch.empty(n, device=dev, dtype=torch.bfloat16)
+        ms = timed(lambda: F.fl_k_adamw(n, w, gr, m, v, wb, 1e-4, 0.9, 0.999, 1e-8, 0.0, 0.1, 0.001, stream=st))
+        nbytes = n * (16 + 16 + 2)  # read w g m v, write w g m v, write bf16 copy
+        out.append({"kernel": "adamw_one_block", "n": n, "ms": ms, "gbs": nbytes / ms / 1e6})
+    for r in out:
+        print(json.dumps(r), flush=True)
+
+
+if __name__ == "__main__":
+    main()
