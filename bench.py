@@ -215,7 +215,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the oracle sample")
     ap.add_argument("--ref-tokens", type=int, default=256, help="tokens of the reference-arm sample")
-    ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_dram_traffic.json"))
+    ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
     if args.impl == "reference":
@@ -313,14 +313,7 @@ def main():
     gemm_ms, gemm_n = prof["gemm"]
     gemm_per_launch_flops = gemm_flops(cfg) * args.steps / max(gemm_n, 1)
     achieved = gemm_per_launch_flops / (gemm_ms / max(gemm_n, 1) / 1e3) / 1e12
-    traffic = None
-    if os.path.exists(args.ncu_traffic):
-        try:
-            tr = json.load(open(args.ncu_traffic))
-            if tr.get("workload") == cfg.name and tr.get("kernel_version") == kernel_version():
-                traffic = tr.get("bytes_per_launch")
-        except Exception:
-            traffic = None
+    traffic = ncu_traffic(args.ncu_traffic, cfg.name)
 
     # ---- end to end through host buffers (pinned), copies inside the timed region
     e2e = None
@@ -385,7 +378,10 @@ def main():
             "roofline": {"kernel": "gemm_tc_kernel (tcgen05)", "bound": "tensor", "achieved": achieved,
                          "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
                          "peak_basis": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
-                         "traffic": traffic, "launches_per_step": gemm_n / args.steps,
+                         "traffic": traffic["bytes_per_launch"] if traffic else None,
+                         "traffic_basis": (f"{traffic['launch']}, one ncu capture ({traffic['source']}); achieved is "
+                                           f"the mean over all GEMM launches of the step") if traffic else None,
+                         "launches_per_step": gemm_n / args.steps,
                          "share_of_step": gemm_ms / ms},
             "gpu_launches": launches,
             "clocks": clk,
@@ -407,6 +403,21 @@ def pci_bus_id(torch, dev):
         return f"{p.pci_domain_id:08X}:{p.pci_bus_id:02X}:{p.pci_device_id:02X}.0"
     except Exception:
         return None
+
+
+def ncu_traffic(path: str, workload_name: str):
+    """DRAM bytes per launch of the GEMM from the committed ncu summary, if it was taken on
+    this workload and on the current GEMM source; else None."""
+    if not os.path.exists(path) or workload_name not in os.path.basename(path):
+        return None
+    txt = open(path).read()
+    if kernel_version() not in txt:
+        return None
+    for line in txt.splitlines():
+        if line.startswith("traffic_bytes_per_launch:"):
+            return {"bytes_per_launch": int(line.split(":")[1]), "source": os.path.relpath(path, ROOT),
+                    "launch": "FFN up-projection forward GEMM (M=8192, N=16384, K=4096)"}
+    return None
 
 
 def kernel_version() -> str:
