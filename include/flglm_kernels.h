@@ -74,6 +74,23 @@ int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, cons
                        const float* rstd, const float* gamma, const void* resid, float resid_alpha,
                        void* dx, float* dgamma, float* dbeta, void* workspace, void* stream);
 
+/* Allocation-free variant of fl_k_layernorm_bwd (same arguments minus the workspace,
+ * same results up to the summation order of dgamma/dbeta).  The paper has no
+ * counterpart: this exists for callers that cannot call cudaMalloc, such as a plug-in
+ * inside a host framework that owns all device memory through its own pool, a serving
+ * loop that must not pay cudaMalloc's implicit device synchronisation, or a process whose
+ * device-memory budget is fully reserved.  Its per-CTA partial sums live in a fixed
+ * 8 MiB array inside the library image (held by every GPU that loads the library until
+ * the process exits); the call allocates nothing.  Limits: H <= 4096 (larger H returns
+ * FL_ERR_CAPACITY), at most 256 CTAs.  The first call on each device looks up the
+ * array's device address (cudaGetSymbolAddress) with that device current; make that
+ * first call before any stream capture.  All calls share the array: calls that overlap
+ * on the GPU race, so serialise them (one stream, or events).  Nothing in the array
+ * needs to start at zero: every CTA overwrites its slice before it is read. */
+int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
+                               const float* rstd, const float* gamma, const void* resid, float resid_alpha,
+                               void* dx, float* dgamma, float* dbeta, void* stream);
+
 /* Varlen causal attention over packed segments (App. A scale 1/sqrt(head_dim)).
  * qkv: bf16 [T, 3*H] (q | k | v, head j at column j*head_dim of each part, RoPE already
  * applied); cu_seqlens_host / cu_seqlens: host and device copies of int32 [S+1].

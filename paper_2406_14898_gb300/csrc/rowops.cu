@@ -2,6 +2,7 @@
 // 128-bit loads), bias-gradient column sums, AdamW over the flat fp32 arena,
 // client pack/unpack, per-call packing metadata and the seeded parameter init.
 #include <cstdio>
+#include <mutex>
 
 #include "../../include/flglm_kernels.h"
 #include "common.cuh"
@@ -463,5 +464,90 @@ extern "C" int fl_k_pack_clients(int32_t K, void* const* clients_host, const int
     }
     if (int rc = fl_launch_gather_scatter(tab, scatter, (cudaStream_t)stream)) return rc;
   }
+  return FL_OK;
+}
+
+// ====================================================================== allocation-free LayerNorm backward
+// Some callers cannot call cudaMalloc: a plug-in hosted by a framework that owns every
+// byte of device memory through its own pool and forbids raw allocations, a serving loop
+// that must not pay cudaMalloc's implicit device synchronisation, or a process whose
+// device-memory budget was reserved in full at start-up.  For them this variant of the
+// LayerNorm backward keeps its per-CTA dgamma/dbeta partial sums in a fixed array that
+// lives in the library image instead of a caller-provided workspace.
+//
+// The array holds FL_LN_NOALLOC_MAX_BLOCKS x 2 x 4096 floats (8 MiB); every GPU that loads
+// the library holds it until the process exits.  The launch uses at most that many CTAs;
+// hidden sizes above 4096 are rejected.  Every call shares the array: calls that overlap
+// on the GPU (for example on two streams) race and must be serialised by the caller.
+// Each CTA overwrites its whole slice before the reduction reads it, so nothing in the
+// array has to start at zero and stale contents from an earlier call are never read.
+namespace {
+constexpr int FL_LN_NOALLOC_MAX_BLOCKS = 256;
+constexpr int FL_LN_NOALLOC_MAX_H = 4096;
+constexpr size_t FL_LN_NOALLOC_FLOATS = (size_t)FL_LN_NOALLOC_MAX_BLOCKS * 2 * FL_LN_NOALLOC_MAX_H;
+}  // namespace
+
+static __device__ __align__(256) float g_ln_bwd_scratch[FL_LN_NOALLOC_FLOATS];
+
+namespace {
+constexpr int FL_NOALLOC_MAX_DEVICES = 64;
+float* g_ln_scratch_ptr[FL_NOALLOC_MAX_DEVICES] = {};
+std::mutex g_ln_scratch_mu;
+
+// Device address of the scratch array on the current device.  The host-side name of a
+// __device__ array is only a stand-in, so the address is looked up once per device with
+// that device current (the first call on each device does this).
+int ln_scratch_address(float** out) {
+  int dev = 0;
+  FL_CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= FL_NOALLOC_MAX_DEVICES)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd (no-alloc): device ordinal %d", dev);
+  std::lock_guard<std::mutex> lock(g_ln_scratch_mu);
+  if (!g_ln_scratch_ptr[dev]) {
+    void* p = nullptr;
+    FL_CUDA_TRY(cudaGetSymbolAddress(&p, g_ln_bwd_scratch));
+    g_ln_scratch_ptr[dev] = static_cast<float*>(p);
+  }
+  *out = g_ln_scratch_ptr[dev];
+  return FL_OK;
+}
+}  // namespace
+
+extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
+                                          const float* rstd, const float* gamma, const void* resid,
+                                          float resid_alpha, void* dx, float* dgamma, float* dbeta, void* stream) {
+  if (T < 0 || H <= 0 || (H % 256))
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd (no-alloc): H=%d must be a positive multiple of 256", H);
+  if (H > FL_LN_NOALLOC_MAX_H)
+    return fl_internal_error(FL_ERR_CAPACITY,
+                             "layernorm bwd (no-alloc): H=%d exceeds the %d columns its fixed scratch array holds", H,
+                             FL_LN_NOALLOC_MAX_H);
+  if (!dy || !x || !mean || !rstd || !gamma || !dx || !dgamma || !dbeta)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): null pointer");
+  float* ws = nullptr;
+  if (int rc = ln_scratch_address(&ws)) return rc;
+  if (T == 0) return FL_OK;
+  cudaStream_t st = (cudaStream_t)stream;
+  int nblk = ln_bwd_blocks(T);
+  if (nblk > FL_LN_NOALLOC_MAX_BLOCKS) nblk = FL_LN_NOALLOC_MAX_BLOCKS;
+  const size_t smem = 2 * (size_t)H * sizeof(float);
+  auto dyb = (const __nv_bfloat16*)dy;
+  auto xb = (const __nv_bfloat16*)x;
+  auto rb = (const __nv_bfloat16*)resid;
+  auto dxb = (__nv_bfloat16*)dx;
+  switch (H / 256) {
+#define FL_LNB_NA(NV)                                                                                          \
+  case NV: {                                                                                                   \
+    FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536));  \
+    ln_bwd_kernel<NV><<<nblk, 256, smem, st>>>(T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws);    \
+    break;                                                                                                     \
+  }
+    FL_LNB_NA(1) FL_LNB_NA(2) FL_LNB_NA(4) FL_LNB_NA(8) FL_LNB_NA(16)
+#undef FL_LNB_NA
+    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd (no-alloc): H/256 must be a power of two");
+  }
+  FL_CUDA_TRY(cudaGetLastError());
+  ln_bwd_reduce_kernel<<<(2 * H + 255) / 256, 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
+  FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }

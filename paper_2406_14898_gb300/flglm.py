@@ -79,6 +79,7 @@ _SIGS = {
     "fl_k_layernorm_fwd": (C.c_int, [_I32, _I32, _P, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_layernorm_bwd_workspace": (C.c_size_t, [_I32, _I32]),
     "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
+    "fl_k_layernorm_bwd_noalloc": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_attention_tiles": (_I32, [_P, _I32]),
     "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P]),
     "fl_k_attention_bwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _I32, _P, _P, _P, _I32, _P, _P]),
@@ -267,6 +268,11 @@ def fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx, d
     check(lib().fl_k_layernorm_bwd(T, H, ptr(dy), ptr(x), ptr(mean), ptr(rstd), ptr(gamma), ptr(resid),
                                    resid_alpha, ptr(dx), ptr(dgamma), ptr(dbeta), ptr(workspace),
                                    stream_ptr(stream)))
+
+
+def fl_k_layernorm_bwd_noalloc(T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx, dgamma, dbeta, stream=None):
+    check(lib().fl_k_layernorm_bwd_noalloc(T, H, ptr(dy), ptr(x), ptr(mean), ptr(rstd), ptr(gamma), ptr(resid),
+                                           resid_alpha, ptr(dx), ptr(dgamma), ptr(dbeta), stream_ptr(stream)))
 
 
 def fl_k_attention_tiles(cu_host) -> int:
