@@ -105,8 +105,10 @@ int fl_server_backward(fl_server_t h, const void* const grad_out[], void* const 
 
 /* One AdamW step over every parameter (Adam of §4.1.4 with decoupled weight decay and
  * bias correction): t += 1; m = b1 m + (1-b1) g; v = b2 v + (1-b2) g^2;
- * w -= lr (m/(1-b1^t) / (sqrt(v/(1-b2^t)) + eps) + wd w); refreshes the bf16 copy and
- * zeroes the gradients.  Errors: STATE (a forward is pending), CUDA. */
+ * w -= lr (m/(1-b1^t) / (sqrt(v/(1-b2^t)) + eps) + wd w); refreshes the bf16 copy.
+ * Afterwards the gradients are zero (fl_server_get_grad returns zeros): the next
+ * backward stores its weight gradients instead of adding them, so the step never has to
+ * write the gradient arena.  Errors: STATE (a forward is pending), CUDA. */
 int fl_server_step(fl_server_t h, float lr);
 
 /* Frees every device buffer of h after synchronising its stream.  NULL is accepted. */

@@ -34,6 +34,7 @@ enum {
   FL_EPI_GELU_BWD = 4,   /* D = acc * gelu_tanh'(aux[m,n])   (aux = pre-activation U)     bf16 */
   FL_EPI_RESID = 5,      /* D = acc + alpha * aux[m,n]                                    bf16 */
   FL_EPI_ACCUM_F32 = 6,  /* D[m,n] += acc                                                 fp32 */
+  FL_EPI_STORE_F32 = 7,  /* D[m,n] = acc                                                  fp32 */
   FL_EPI_COUNT
 };
 

@@ -28,7 +28,7 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;  // one 128-byte swizzle row of bf16
 constexpr int UMMA_K = 16;
-constexpr int GROUP_M = 8;
+constexpr double L2_GROUP_BUDGET = 48.0 * (1 << 20);  // bytes of operand panels kept resident per group
 constexpr int NUM_THREADS = 192;
 
 template <int BN>
@@ -148,25 +148,46 @@ FL_DEV void epilogue64(const Epi& e, int m, int n0, float* v) {
       o.x += v[4 * j]; o.y += v[4 * j + 1]; o.z += v[4 * j + 2]; o.w += v[4 * j + 3];
       d[j] = o;
     }
+  } else if (e.mode == FL_EPI_STORE_F32) {
+    float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(e.D) + (int64_t)m * e.ldd + n0);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) d[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
   } else {
     store_bf16x64(reinterpret_cast<__nv_bfloat16*>(e.D) + (int64_t)m * e.ldd + n0, v);
   }
 }
 
-FL_DEV void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
-  const int group = GROUP_M * num_n;
-  const int g = tile / group;
-  const int first_m = g * GROUP_M;
-  const int gm = min(num_m - first_m, GROUP_M);
-  const int local = tile - g * group;
-  mb = first_m + local % gm;
-  nb = local / gm;
+// Tile order.  Tiles are taken in groups of `gsz` panels of one operand: along m
+// (gsz m-blocks, m fastest) every group streams B once while its A panels stay in L2;
+// along n the roles swap.  The host picks the side and size that minimise DRAM reads.
+struct Raster {
+  int gsz;
+  int along_n;
+};
+FL_DEV void tile_coords(int tile, int num_m, int num_n, Raster r, int& mb, int& nb) {
+  if (!r.along_n) {
+    const int group = r.gsz * num_n;
+    const int g = tile / group;
+    const int first = g * r.gsz;
+    const int gm = min(num_m - first, r.gsz);
+    const int local = tile - g * group;
+    mb = first + local % gm;
+    nb = local / gm;
+  } else {
+    const int group = r.gsz * num_m;
+    const int g = tile / group;
+    const int first = g * r.gsz;
+    const int gn = min(num_n - first, r.gsz);
+    const int local = tile - g * group;
+    nb = first + local % gn;
+    mb = local / gn;
+  }
 }
 
 template <int BN, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, Epi epi,
-                   int M, int N, int K, int* status) {
+                   int M, int N, int K, Raster raster, int* status) {
   using C = Cfg<BN>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -222,7 +243,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
         int mb, nb;
-        tile_coords(tile, num_m, num_n, mb, nb);
+        tile_coords(tile, num_m, num_n, raster, mb, nb);
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1)) {
             report_status(status, FL_DEV_TIMEOUT_EMPTY);
@@ -314,7 +335,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     int local = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
       int mb, nb;
-      tile_coords(tile, num_m, num_n, mb, nb);
+      tile_coords(tile, num_m, num_n, raster, mb, nb);
       const int acc = local & 1;
       const uint32_t acc_par = (local >> 1) & 1;
       if (!mbar_wait(&acc_full[acc], acc_par)) {
@@ -421,9 +442,20 @@ int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) 
   if (!B_MN) rc = make_map(&tb, a->B, a->K, a->N, a->ldb, BN);
   else rc = make_map(&tb, a->B, a->N, a->K, a->ldb, BK);
   if (rc) return rc;
-  const int tiles = ((a->M + BM - 1) / BM) * (a->N / BN);
+  const int num_m = (a->M + BM - 1) / BM, num_n = a->N / BN;
+  const int tiles = num_m * num_n;
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<BN, A_MN, B_MN><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ta, tb, epi, a->M, a->N, a->K, status);
+  // DRAM reads of the two orders: the grouped operand once, the other once per group
+  const double pa = double(BM) * a->K * 2, pb = double(BN) * a->K * 2;
+  int gm = (int)(L2_GROUP_BUDGET / pa), gn = (int)(L2_GROUP_BUDGET / pb);
+  gm = gm < 1 ? 1 : (gm > num_m ? num_m : gm);
+  gn = gn < 1 ? 1 : (gn > num_n ? num_n : gn);
+  const double cost_m = pa * num_m + pb * num_n * ((num_m + gm - 1) / gm);
+  const double cost_n = pb * num_n + pa * num_m * ((num_n + gn - 1) / gn);
+  Raster r;
+  r.along_n = cost_n < cost_m ? 1 : 0;
+  r.gsz = r.along_n ? gn : gm;
+  gemm_tc_kernel<BN, A_MN, B_MN><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ta, tb, epi, a->M, a->N, a->K, r, status);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }

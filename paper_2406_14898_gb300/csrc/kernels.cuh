@@ -30,6 +30,8 @@ int fl_launch_gather_scatter(const CopyTable& tab, int scatter, cudaStream_t st)
 int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st);
 int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, float* out, cudaStream_t st);
 int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st);
+int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
+                    float beta2, float eps, float weight_decay, float bc1, float bc2, int zero_grad, cudaStream_t st);
 int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st);
 
 // Attention on a device tile list (built by fl_launch_meta).

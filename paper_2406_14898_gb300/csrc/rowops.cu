@@ -31,6 +31,10 @@ FL_DEV void unpack8(const uint4& w, float* f) {
   float2 a = unpack_bf16x2(w.x), b = unpack_bf16x2(w.y), c = unpack_bf16x2(w.z), d = unpack_bf16x2(w.w);
   f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y; f[4] = c.x; f[5] = c.y; f[6] = d.x; f[7] = d.y;
 }
+// Makes the compiler treat v as redefined, so that values derived from it are recomputed
+// instead of being kept live in registers across passes.
+FL_DEV void opaque(uint4& v) { asm volatile("" : "+r"(v.x), "+r"(v.y), "+r"(v.z), "+r"(v.w)); }
+
 FL_DEV uint4 pack8(const float* f) {
   uint4 w;
   w.x = pack_bf16x2(f[0], f[1]);
@@ -41,7 +45,9 @@ FL_DEV uint4 pack8(const float* f) {
 }
 
 // ------------------------------------------------------------------ LayerNorm forward
-// One warp per row; lane l owns the 8-element chunks l, l+32, l+64, ... (NV chunks).
+// One warp per row; lane l owns the 8-element chunks l, l+32, l+64, ... (NV chunks).  The
+// row stays in registers as packed bf16 (4 registers per chunk) across the mean, variance
+// and output passes, so HBM is read once and written once.
 template <int NV>
 __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bfloat16* __restrict__ x,
                                                      const float* __restrict__ gamma,
@@ -52,18 +58,29 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
   const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
-  float v[NV * 8];
+  uint4 raw[NV];
 #pragma unroll
-  for (int i = 0; i < NV; ++i) unpack8(__ldg(xr + lane + 32 * i), v + 8 * i);
+  for (int i = 0; i < NV; ++i) raw[i] = __ldg(xr + lane + 32 * i);
   float s = 0.f;
 #pragma unroll
-  for (int i = 0; i < NV * 8; ++i) s += v[i];
+  for (int i = 0; i < NV; ++i) {
+    float f[8];
+    unpack8(raw[i], f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) s += f[j];
+  }
   const float mu = warp_sum(s) / H;
   float q = 0.f;
 #pragma unroll
-  for (int i = 0; i < NV * 8; ++i) {
-    const float d = v[i] - mu;
-    q += d * d;
+  for (int i = 0; i < NV; ++i) {
+    float f[8];
+    opaque(raw[i]);
+    unpack8(raw[i], f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float d = f[j] - mu;
+      q += d * d;
+    }
   }
   const float rs = rsqrtf(warp_sum(q) / H + eps);
   uint4* yr = reinterpret_cast<uint4*>(y + (int64_t)row * H);
@@ -72,13 +89,15 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     const int c = lane + 32 * i;  // chunk index: columns [8c, 8c+8)
-    float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
-    float4 ba = __ldg(b4 + 2 * c), bb = __ldg(b4 + 2 * c + 1);
+    const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
+    const float4 ba = __ldg(b4 + 2 * c), bb = __ldg(b4 + 2 * c + 1);
     const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
     const float bt[8] = {ba.x, ba.y, ba.z, ba.w, bb.x, bb.y, bb.z, bb.w};
-    float o[8];
+    float f[8], o[8];
+    opaque(raw[i]);
+    unpack8(raw[i], f);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) o[j] = (v[8 * i + j] - mu) * rs * gg[j] + bt[j];
+    for (int j = 0; j < 8; ++j) o[j] = (f[j] - mu) * rs * gg[j] + bt[j];
     yr[c] = pack8(o);
   }
   if (lane == 0) {
@@ -88,8 +107,14 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
 }
 
 // ------------------------------------------------------------------ LayerNorm backward
-// Warp per row for dx; per-CTA column partials of dgamma/dbeta in shared memory, written
-// to workspace[blockIdx.x][2][H] and reduced by ln_bwd_reduce_kernel.
+// A CTA takes tiles of LN_R rows.  Phase 1: one warp per row computes mean(g) and
+// mean(g xhat), g = gamma dy (lane-strided 16-byte chunks).  Phase 2: thread t owns the
+// column chunks t, t+256, ... of every row of the tile; it re-reads dy and x (L2 hits),
+// writes dx and keeps its columns' dgamma/dbeta partials in registers across all the
+// CTA's tiles.  The partials go to workspace[blockIdx.x][2][H]; ln_bwd_reduce_kernel
+// adds them into dgamma/dbeta.
+constexpr int LN_R = 16;
+
 template <int NV>
 __global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bfloat16* __restrict__ dy,
                                                      const __nv_bfloat16* __restrict__ x,
@@ -98,77 +123,135 @@ __global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bf
                                                      const float* __restrict__ gamma,
                                                      const __nv_bfloat16* __restrict__ resid, float resid_alpha,
                                                      __nv_bfloat16* __restrict__ dx, float* __restrict__ ws) {
-  extern __shared__ float part[];  // [2][H]: dgamma, dbeta
-  for (int i = threadIdx.x; i < 2 * H; i += blockDim.x) part[i] = 0.f;
-  __syncthreads();
-  const int lane = threadIdx.x & 31;
-  const int wid = threadIdx.x >> 5;
+  constexpr int CPT = (NV * 32 + 255) / 256;  // column chunks per thread in phase 2
+  __shared__ float s_mg[LN_R], s_mgx[LN_R];
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const int nchunk = H / 8;
   const float4* g4 = reinterpret_cast<const float4*>(gamma);
-  for (int row = blockIdx.x * 8 + wid; row < T; row += gridDim.x * 8) {
-    const uint4* dyr = reinterpret_cast<const uint4*>(dy + (int64_t)row * H);
-    const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
-    const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
-    // pass 1: row sums of g = gamma*dy and g*xhat; column partials of dgamma, dbeta
-    float s1 = 0.f, s2 = 0.f;
-#pragma unroll 4
-    for (int i = 0; i < NV; ++i) {
-      const int c = lane + 32 * i;
-      float d[8], xv[8];
-      unpack8(__ldg(dyr + c), d);
-      unpack8(__ldg(xr + c), xv);
+  float gcol[CPT][8], accg[CPT][8], accb[CPT][8];
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) {
+    const int c = tid + 256 * j;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) accg[j][k] = accb[j][k] = gcol[j][k] = 0.f;
+    if (c < nchunk) {
       const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
-      const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const float xh = (xv[j] - mu) * rs;
-        atomicAdd(&part[8 * c + j], d[j] * xh);
-        atomicAdd(&part[H + 8 * c + j], d[j]);
-        const float g = d[j] * gg[j];
-        s1 += g;
-        s2 += g * xh;
-      }
-    }
-    const float mg = warp_sum(s1) / H;
-    const float mgx = warp_sum(s2) / H;
-    // pass 2: dx = rstd * (g - mean(g) - xhat * mean(g xhat)) (+ alpha * resid)
-    uint4* dxr = reinterpret_cast<uint4*>(dx + (int64_t)row * H);
-    const uint4* rr = resid ? reinterpret_cast<const uint4*>(resid + (int64_t)row * H) : nullptr;
-#pragma unroll 4
-    for (int i = 0; i < NV; ++i) {
-      const int c = lane + 32 * i;
-      float d[8], xv[8], o[8];
-      unpack8(__ldg(dyr + c), d);
-      unpack8(__ldg(xr + c), xv);
-      const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
-      const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
-#pragma unroll
-      for (int j = 0; j < 8; ++j) o[j] = rs * (d[j] * gg[j] - mg - (xv[j] - mu) * rs * mgx);
-      if (rr) {
-        float r[8];
-        unpack8(__ldg(rr + c), r);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = fmaf(resid_alpha, r[j], o[j]);
-      }
-      dxr[c] = pack8(o);
+      gcol[j][0] = ga.x; gcol[j][1] = ga.y; gcol[j][2] = ga.z; gcol[j][3] = ga.w;
+      gcol[j][4] = gb.x; gcol[j][5] = gb.y; gcol[j][6] = gb.z; gcol[j][7] = gb.w;
     }
   }
-  __syncthreads();
+  for (int r0 = blockIdx.x * LN_R; r0 < T; r0 += gridDim.x * LN_R) {
+    // phase 1: per-row sums
+    for (int rr = wid; rr < LN_R; rr += 8) {
+      const int row = r0 + rr;
+      float s1 = 0.f, s2 = 0.f;
+      if (row < T) {
+        const uint4* dyr = reinterpret_cast<const uint4*>(dy + (int64_t)row * H);
+        const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
+        const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
+#pragma unroll 4
+        for (int i = 0; i < NV; ++i) {
+          const int c = lane + 32 * i;
+          float d[8], xv[8];
+          unpack8(__ldg(dyr + c), d);
+          unpack8(__ldg(xr + c), xv);
+          const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
+          const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const float g = d[k] * gg[k];
+            s1 += g;
+            s2 += g * (xv[k] - mu) * rs;
+          }
+        }
+      }
+      s1 = warp_sum(s1);
+      s2 = warp_sum(s2);
+      if (lane == 0) {
+        s_mg[rr] = s1 / H;
+        s_mgx[rr] = s2 / H;
+      }
+    }
+    __syncthreads();
+    // phase 2: dx and the column partials
+    const int rows = min(LN_R, T - r0);
+    for (int rr = 0; rr < rows; ++rr) {
+      const int row = r0 + rr;
+      const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
+      const float mg = s_mg[rr], mgx = s_mgx[rr];
+      const uint4* dyr = reinterpret_cast<const uint4*>(dy + (int64_t)row * H);
+      const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
+      const uint4* rr4 = resid ? reinterpret_cast<const uint4*>(resid + (int64_t)row * H) : nullptr;
+      uint4* dxr = reinterpret_cast<uint4*>(dx + (int64_t)row * H);
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) {
+        const int c = tid + 256 * j;
+        if (c < nchunk) {
+          float d[8], xv[8], o[8];
+          unpack8(__ldg(dyr + c), d);
+          unpack8(__ldg(xr + c), xv);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const float xh = (xv[k] - mu) * rs;
+            accg[j][k] += d[k] * xh;
+            accb[j][k] += d[k];
+            o[k] = rs * (d[k] * gcol[j][k] - mg - xh * mgx);
+          }
+          if (rr4) {
+            float r[8];
+            unpack8(__ldg(rr4 + c), r);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) o[k] = fmaf(resid_alpha, r[k], o[k]);
+          }
+          dxr[c] = pack8(o);
+        }
+      }
+    }
+    __syncthreads();
+  }
   float* out = ws + (int64_t)blockIdx.x * 2 * H;
-  for (int i = threadIdx.x; i < 2 * H; i += blockDim.x) out[i] = part[i];
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) {
+    const int c = tid + 256 * j;
+    if (c < nchunk) {
+      float4* og = reinterpret_cast<float4*>(out + 8 * c);
+      float4* ob = reinterpret_cast<float4*>(out + H + 8 * c);
+      og[0] = make_float4(accg[j][0], accg[j][1], accg[j][2], accg[j][3]);
+      og[1] = make_float4(accg[j][4], accg[j][5], accg[j][6], accg[j][7]);
+      ob[0] = make_float4(accb[j][0], accb[j][1], accb[j][2], accb[j][3]);
+      ob[1] = make_float4(accb[j][4], accb[j][5], accb[j][6], accb[j][7]);
+    }
+  }
 }
 
+// dgamma/dbeta += sum over the nblk partial rows; blockIdx.y takes a slice of the rows.
 __global__ void ln_bwd_reduce_kernel(int nblk, int H, const float* __restrict__ ws, float* __restrict__ dgamma,
                                      float* __restrict__ dbeta) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= 2 * H) return;
+  const int per = (nblk + gridDim.y - 1) / gridDim.y;
+  const int b0 = blockIdx.y * per, b1 = min(nblk, b0 + per);
+  if (b0 >= b1) return;
   float s = 0.f;
-  for (int b = 0; b < nblk; ++b) s += ws[(int64_t)b * 2 * H + i];
-  if (i < H) dgamma[i] += s;
-  else dbeta[i - H] += s;
+  for (int b = b0; b < b1; ++b) s += ws[(int64_t)b * 2 * H + i];
+  atomicAdd(i < H ? dgamma + i : dbeta + (i - H), s);
+}
+
+// Launches the backward kernel and the reduction of its partials.
+template <int NV>
+int launch_ln_bwd(int nblk, int T, int H, const __nv_bfloat16* dy, const __nv_bfloat16* x, const float* mean,
+                  const float* rstd, const float* gamma, const __nv_bfloat16* resid, float alpha, __nv_bfloat16* dx,
+                  float* ws, float* dgamma, float* dbeta, cudaStream_t st) {
+  ln_bwd_kernel<NV><<<nblk, 256, 0, st>>>(T, H, dy, x, mean, rstd, gamma, resid, alpha, dx, ws);
+  FL_CUDA_TRY(cudaGetLastError());
+  const int split = nblk >= 64 ? 16 : 1;
+  ln_bwd_reduce_kernel<<<dim3((2 * H + 255) / 256, split), 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
 }
 
 int ln_bwd_blocks(int T) {
-  const int want = (T + 7) / 8;
+  const int want = (T + LN_R - 1) / LN_R;
   const int cap = 2 * sm_count();
   return want < cap ? want : cap;
 }
@@ -208,7 +291,7 @@ __global__ void __launch_bounds__(256) colsum_kernel(int T, int N, const __nv_bf
 __global__ void __launch_bounds__(256) adamw_kernel(int64_t n4, float4* __restrict__ w, float4* __restrict__ g,
                                                     float4* __restrict__ m, float4* __restrict__ v,
                                                     uint2* __restrict__ wb, float lr, float b1, float b2, float eps,
-                                                    float wd, float inv_bc1, float inv_bc2) {
+                                                    float wd, float inv_bc1, float inv_bc2, int zero_grad) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
     float4 W = w[i], G = g[i], M = m[i], V = v[i];
     float* pw = &W.x;
@@ -226,7 +309,7 @@ __global__ void __launch_bounds__(256) adamw_kernel(int64_t n4, float4* __restri
     w[i] = W;
     m[i] = M;
     v[i] = V;
-    g[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (zero_grad) g[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     if (wb) wb[i] = make_uint2(pack_bf16x2(W.x, W.y), pack_bf16x2(W.z, W.w));
   }
 }
@@ -346,31 +429,18 @@ extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const vo
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
   const int nblk = ln_bwd_blocks(T);
-  const size_t smem = 2 * (size_t)H * sizeof(float);
   float* ws = (float*)workspace;
   auto dyb = (const __nv_bfloat16*)dy;
   auto xb = (const __nv_bfloat16*)x;
   auto rb = (const __nv_bfloat16*)resid;
   auto dxb = (__nv_bfloat16*)dx;
   switch (H / 256) {
-#define FL_LNB(NV)                                                                                          \
-  case NV: {                                                                                                \
-    static bool set = false;                                                                                \
-    if (!set) {                                                                                             \
-      FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536)); \
-      set = true;                                                                                           \
-    }                                                                                                       \
-    ln_bwd_kernel<NV><<<nblk, 256, smem, st>>>(T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws); \
-    break;                                                                                                  \
-  }
+#define FL_LNB(NV) \
+  case NV: return launch_ln_bwd<NV>(nblk, T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws, dgamma, dbeta, st);
     FL_LNB(1) FL_LNB(2) FL_LNB(4) FL_LNB(8) FL_LNB(16)
 #undef FL_LNB
     default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H/256 must be a power of two");
   }
-  FL_CUDA_TRY(cudaGetLastError());
-  ln_bwd_reduce_kernel<<<(2 * H + 255) / 256, 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
-  FL_CUDA_TRY(cudaGetLastError());
-  return FL_OK;
 }
 
 extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream) {
@@ -394,7 +464,17 @@ extern "C" int fl_k_adamw(int64_t n, float* w, float* g, float* m, float* v, voi
   const int64_t n4 = n / 4;
   adamw_kernel<<<grid_for(n4), 256, 0, (cudaStream_t)stream>>>(n4, (float4*)w, (float4*)g, (float4*)m, (float4*)v,
                                                               (uint2*)w_bf16, lr, beta1, beta2, eps, weight_decay,
-                                                              1.f / bc1, 1.f / bc2);
+                                                              1.f / bc1, 1.f / bc2, 1);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
+                    float beta2, float eps, float weight_decay, float bc1, float bc2, int zero_grad, cudaStream_t st) {
+  if (n <= 0) return FL_OK;
+  const int64_t n4 = n / 4;
+  adamw_kernel<<<grid_for(n4), 256, 0, st>>>(n4, (float4*)w, (float4*)g, (float4*)m, (float4*)v, (uint2*)w_bf16, lr,
+                                             beta1, beta2, eps, weight_decay, 1.f / bc1, 1.f / bc2, zero_grad);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
@@ -530,24 +610,15 @@ extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, 
   cudaStream_t st = (cudaStream_t)stream;
   int nblk = ln_bwd_blocks(T);
   if (nblk > FL_LN_NOALLOC_MAX_BLOCKS) nblk = FL_LN_NOALLOC_MAX_BLOCKS;
-  const size_t smem = 2 * (size_t)H * sizeof(float);
   auto dyb = (const __nv_bfloat16*)dy;
   auto xb = (const __nv_bfloat16*)x;
   auto rb = (const __nv_bfloat16*)resid;
   auto dxb = (__nv_bfloat16*)dx;
   switch (H / 256) {
-#define FL_LNB_NA(NV)                                                                                          \
-  case NV: {                                                                                                   \
-    FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536));  \
-    ln_bwd_kernel<NV><<<nblk, 256, smem, st>>>(T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws);    \
-    break;                                                                                                     \
-  }
+#define FL_LNB_NA(NV) \
+  case NV: return launch_ln_bwd<NV>(nblk, T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws, dgamma, dbeta, st);
     FL_LNB_NA(1) FL_LNB_NA(2) FL_LNB_NA(4) FL_LNB_NA(8) FL_LNB_NA(16)
 #undef FL_LNB_NA
     default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd (no-alloc): H/256 must be a power of two");
   }
-  FL_CUDA_TRY(cudaGetLastError());
-  ln_bwd_reduce_kernel<<<(2 * H + 255) / 256, 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
-  FL_CUDA_TRY(cudaGetLastError());
-  return FL_OK;
 }

@@ -7,9 +7,11 @@
 //
 // Device memory (allocated once in fl_server_create, nothing allocated later):
 //   parameter arenas  fp32 master w, grad g, Adam m, v and the bf16 working copy, one flat
-//                     array each with identical offsets (tensor t of block b at
-//                     b * block_stride + tensor_off[t], every tensor 64-byte aligned), so that
-//                     one AdamW launch covers every parameter;
+//                     array each with identical offsets, so that one AdamW launch covers
+//                     every parameter: first the four weight matrices of every block
+//                     (block b at b * mat_stride), then the bias and LayerNorm vectors of
+//                     every block in one contiguous region (block b at vec_base +
+//                     b * vec_stride); every tensor 64-byte aligned;
 //   activations       per block: LN1 out A, rotated QKV, attention O, LSE, residual stream
 //                     Hres, LN2 out M, FFN pre-activation U and GeLU output G, LN statistics;
 //                     xs[0..n_blocks]: block inputs / outputs (xs[0] = packed client states);
@@ -83,13 +85,17 @@ struct fl_server {
   std::string err;
 
   // parameter arenas
-  int64_t tensor_off[FL_T_COUNT] = {};
+  int64_t tensor_off[FL_T_COUNT] = {};  // inside the block's matrix or vector slice
   int64_t tensor_n[FL_T_COUNT] = {};
-  int64_t block_stride = 0;
+  int64_t mat_stride = 0, vec_stride = 0, vec_base = 0;
   int64_t n_params = 0;  // padded total
   float *w = nullptr, *g = nullptr, *m = nullptr, *v = nullptr;
   __nv_bfloat16* wb = nullptr;
   int64_t step_t = 0;
+  // true while every gradient is zero (after create and after each step): the next
+  // backward then stores the weight gradients instead of adding to them, and AdamW
+  // does not need to clear the 4 B/parameter gradient arena
+  bool grads_zero = true;
 
   // activations
   std::vector<__nv_bfloat16*> xs;
@@ -114,9 +120,13 @@ struct fl_server {
   Prof prof;
   int64_t launches = 0;
 
-  float* wt(int b, int t) { return w + b * block_stride + tensor_off[t]; }
-  float* gt(int b, int t) { return g + b * block_stride + tensor_off[t]; }
-  __nv_bfloat16* wbt(int b, int t) { return wb + b * block_stride + tensor_off[t]; }
+  static bool is_matrix(int t) { return t == FL_T_WQKV || t == FL_T_WDENSE || t == FL_T_WUP || t == FL_T_WDOWN; }
+  int64_t off(int b, int t) const {
+    return is_matrix(t) ? b * mat_stride + tensor_off[t] : vec_base + b * vec_stride + tensor_off[t];
+  }
+  float* wt(int b, int t) { return w + off(b, t); }
+  float* gt(int b, int t) { return g + off(b, t); }
+  __nv_bfloat16* wbt(int b, int t) { return wb + off(b, t); }
 };
 
 namespace {
@@ -221,15 +231,15 @@ fl_gemm_args gemm_dgrad(int T, int Kin, int Nout, const void* dY, const void* W,
   a.epilogue = epi;
   return a;
 }
-// dW[Nout, Kin] += dY[T, Nout]^T . X[T, Kin]
-fl_gemm_args gemm_wgrad(int T, int Nout, int Kin, const void* dY, const void* X, float* dW) {
+// dW[Nout, Kin] (+)= dY[T, Nout]^T . X[T, Kin]; stores when the gradients are known zero
+fl_gemm_args gemm_wgrad(int T, int Nout, int Kin, const void* dY, const void* X, float* dW, bool store) {
   fl_gemm_args a;
   memset(&a, 0, sizeof a);
   a.M = Nout; a.N = Kin; a.K = T;
   a.A = dY; a.lda = Nout; a.a_mn_major = 1;
   a.B = X; a.ldb = Kin; a.b_mn_major = 1;
   a.D = dW; a.ldd = Kin;
-  a.epilogue = FL_EPI_ACCUM_F32;
+  a.epilogue = store ? FL_EPI_STORE_F32 : FL_EPI_ACCUM_F32;
   return a;
 }
 
@@ -302,7 +312,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* 
   d1.aux = A.u;
   d1.ld_aux = F;
   TRY(h, run_gemm(h, d1));
-  TRY(h, run_gemm(h, gemm_wgrad(T, H, F, dy, A.g, h->gt(b, FL_T_WDOWN))));
+  TRY(h, run_gemm(h, gemm_wgrad(T, H, F, dy, A.g, h->gt(b, FL_T_WDOWN), h->grads_zero)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
   prof_end(h);
@@ -314,7 +324,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* 
     d2.alpha = al;
   }
   TRY(h, run_gemm(h, d2));
-  TRY(h, run_gemm(h, gemm_wgrad(T, F, H, h->du, A.m, h->gt(b, FL_T_WUP))));
+  TRY(h, run_gemm(h, gemm_wgrad(T, F, H, h->du, A.m, h->gt(b, FL_T_WUP), h->grads_zero)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
   prof_end(h);
@@ -325,7 +335,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* 
   prof_end(h);
   // dense: do = dh Wd; dWd += dh^T o; dbd += colsum(dh)
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
-  TRY(h, run_gemm(h, gemm_wgrad(T, H, H, h->dh, A.o, h->gt(b, FL_T_WDENSE))));
+  TRY(h, run_gemm(h, gemm_wgrad(T, H, H, h->dh, A.o, h->gt(b, FL_T_WDENSE), h->grads_zero)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
   prof_end(h);
@@ -342,7 +352,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* 
     d3.alpha = al;
   }
   TRY(h, run_gemm(h, d3));
-  TRY(h, run_gemm(h, gemm_wgrad(T, 3 * H, H, h->dqkv, A.a, h->gt(b, FL_T_WQKV))));
+  TRY(h, run_gemm(h, gemm_wgrad(T, 3 * H, H, h->dqkv, A.a, h->gt(b, FL_T_WQKV), h->grads_zero)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
   prof_end(h);
@@ -433,14 +443,17 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
 
   // parameter layout
   const int64_t sizes[FL_T_COUNT] = {3 * H * H, 3 * H, H * H, H, F * H, F, H * F, H, H, H, H, H};
-  int64_t off = 0;
+  int64_t moff = 0, voff = 0;
   for (int t = 0; t < FL_T_COUNT; ++t) {
-    h->tensor_off[t] = off;
+    int64_t& o = fl_server::is_matrix(t) ? moff : voff;
+    h->tensor_off[t] = o;
     h->tensor_n[t] = sizes[t];
-    off += (sizes[t] + 15) / 16 * 16;
+    o += (sizes[t] + 15) / 16 * 16;
   }
-  h->block_stride = off;
-  h->n_params = off * c.n_blocks;
+  h->mat_stride = moff;
+  h->vec_stride = voff;
+  h->vec_base = moff * c.n_blocks;
+  h->n_params = h->vec_base + voff * c.n_blocks;
   int rc;
   if ((rc = dalloc(h, &h->w, h->n_params)) || (rc = dalloc(h, &h->g, h->n_params)) ||
       (rc = dalloc(h, &h->m, h->n_params)) || (rc = dalloc(h, &h->v, h->n_params)) ||
@@ -560,6 +573,11 @@ extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], v
   if (int rc = check_ptrs(h, grad_out, h->K, "grad_out")) return rc;
   if (int rc = check_ptrs(h, (const void* const*)grad_in, h->K, "grad_in")) return rc;
   int rc;
+  if (h->grads_zero) {
+    // bias and LayerNorm gradients accumulate (+=); one memset of their contiguous region
+    const cudaError_t e = cudaMemsetAsync(h->g + h->vec_base, 0, (h->n_params - h->vec_base) * sizeof(float), h->stream);
+    if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "cudaMemsetAsync", __FILE__, __LINE__));
+  }
   if ((rc = copy_clients(h, grad_out, h->dy, 0))) return rc;
   __nv_bfloat16* cur = h->dy;
   __nv_bfloat16* nxt = h->dx;
@@ -571,6 +589,7 @@ extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], v
   }
   if ((rc = copy_clients(h, (const void* const*)grad_in, cur, 1))) return rc;
   h->pending = false;
+  h->grads_zero = false;
   return FL_OK;
 }
 
@@ -582,9 +601,11 @@ extern "C" int fl_server_step(fl_server_t h, float lr) {
   const double bc1 = 1.0 - std::pow((double)c.adam_beta1, (double)h->step_t);
   const double bc2 = 1.0 - std::pow((double)c.adam_beta2, (double)h->step_t);
   prof_begin(h, FL_PROF_ADAMW);
-  int rc = fl_k_adamw(h->n_params, h->w, h->g, h->m, h->v, h->wb, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
-                      c.weight_decay, (float)bc1, (float)bc2, h->stream);
+  // the gradients are not cleared here: the next backward overwrites them (grads_zero)
+  int rc = fl_launch_adamw(h->n_params, h->w, h->g, h->m, h->v, h->wb, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
+                           c.weight_decay, (float)bc1, (float)bc2, 0, h->stream);
   prof_end(h);
+  if (rc == FL_OK) h->grads_zero = true;
   return fwd_err(h, rc);
 }
 
@@ -645,12 +666,16 @@ extern "C" int fl_server_get_param(fl_server_t h, int32_t b, int32_t t, float* d
 }
 extern "C" int fl_server_get_grad(fl_server_t h, int32_t b, int32_t t, float* dst, size_t n) {
   if (int rc = check_tensor(h, b, t, dst, n)) return rc;
+  if (h->grads_zero) {  // after create or a step the gradients are zero by definition
+    memset(dst, 0, n * sizeof(float));
+    return FL_OK;
+  }
   return d2h(h, dst, h->gt(b, t), n);
 }
 extern "C" int fl_server_get_adam_moments(fl_server_t h, int32_t b, int32_t t, float* hm, float* hv, size_t n) {
   if (int rc = check_tensor(h, b, t, hm, n)) return rc;
   if (!hv) return set_err(h, FL_ERR_INVALID_ARG, "null host buffer");
-  const int64_t o = b * h->block_stride + h->tensor_off[t];
+  const int64_t o = h->off(b, t);
   if (int rc = d2h(h, hm, h->m + o, n)) return rc;
   return d2h(h, hv, h->v + o, n);
 }

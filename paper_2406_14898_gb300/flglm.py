@@ -23,7 +23,7 @@ ERRORS = {-1: "FL_ERR_INVALID_ARG", -2: "FL_ERR_CAPACITY", -3: "FL_ERR_STATE", -
  FL_T_LN1_G, FL_T_LN1_B, FL_T_LN2_G, FL_T_LN2_B) = range(12)
 FL_T_COUNT = 12
 (FL_EPI_STORE, FL_EPI_BIAS_GELU, FL_EPI_BIAS_RESID, FL_EPI_BIAS_ROPE, FL_EPI_GELU_BWD, FL_EPI_RESID,
- FL_EPI_ACCUM_F32) = range(7)
+ FL_EPI_ACCUM_F32, FL_EPI_STORE_F32) = range(8)
 PROF_CLASSES = ("gemm", "attention", "layernorm", "adamw", "other")
 
 
