@@ -215,11 +215,17 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the oracle sample")
     ap.add_argument("--ref-tokens", type=int, default=256, help="tokens of the reference-arm sample")
+    ap.add_argument("--sweep", action="store_true",
+                    help="client-batching sweep: 26 blocks, 2 x 512 tokens per client, K in 1..32, "
+                         "one packed call vs K sequential single-client calls (one JSON line per K)")
     ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
     if args.impl == "reference":
         run_reference(args, cfg)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -394,6 +400,65 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def run_sweep(args):
+    """Client-batching sweep (§3.3): for each K, the K clients' step as one packed call
+    (client-batch) and as K single-client calls followed by one AdamW update (serial),
+    on one server sized for the largest K."""
+    import torch
+    from paper_2406_14898_gb300 import flglm as F
+
+    ks = syn.SWEEP_KS
+    big = syn.sweep_config(max(ks))
+    F.lib()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device=dev)
+    srv = F.Server(F.make_cfg(big, big.tokens, max(big.seq_lens)), big.seed, stream=stream)
+    sb = syn.client_states(big)
+    gb = syn.client_grads(big)
+    st = [torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev) for b in sb]
+    go = [torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev) for b in gb]
+    outs = [torch.empty_like(s) for s in st]
+    gin = [torch.empty_like(s) for s in st]
+    pk = peaks()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    for K in ks:
+        cfg = syn.sweep_config(K)
+
+        def batched():
+            srv.forward(st[:K], cfg.seq_lens, outs[:K])
+            srv.backward(go[:K], gin[:K])
+            srv.step(cfg.lr)
+
+        def sequential():
+            for k in range(K):
+                srv.forward(st[k:k + 1], cfg.seq_lens[k:k + 1], outs[k:k + 1])
+                srv.backward(go[k:k + 1], gin[k:k + 1])
+            srv.step(cfg.lr)
+
+        res = {}
+        for name, fn in (("batched", batched), ("sequential", sequential)):
+            for _ in range(args.warmup):
+                fn()
+            srv.sync()
+            e0.record(stream)
+            for _ in range(args.steps):
+                fn()
+            e1.record(stream)
+            srv.sync()
+            ms = e0.elapsed_time(e1) / args.steps
+            res[name] = {"tokens_per_s": cfg.tokens / (ms / 1e3), "ms_per_step": ms,
+                         "pct_bf16_peak": 100.0 * (gemm_flops(cfg) + attn_flops(cfg)) / (ms / 1e3)
+                         / (pk["bf16_sustained"] * 1e12)}
+        line = {"metric": METRIC, "mode": "client-batching sweep", "K": K, "value": res["batched"]["tokens_per_s"],
+                "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+                "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+                "config": {"workload": describe(cfg), "global_batch": cfg.tokens, "seq_len": 512},
+                "batched": res["batched"], "sequential": res["sequential"],
+                "batched_over_sequential": res["batched"]["tokens_per_s"] / res["sequential"]["tokens_per_s"]}
+        print(json.dumps(line), flush=True)
+    srv.close()
 
 
 def pci_bus_id(torch, dev):

@@ -22,17 +22,20 @@
 extern "C" {
 #endif
 
+/* Element types of the row kernels' and epilogues' activation operands. */
+enum { FL_DT_BF16 = 0, FL_DT_F32 = 1 };
+
 /* GEMM epilogues.  acc = sum_k A(m,k) B(n,k) in fp32 (tcgen05, TMEM accumulator). */
 enum {
   FL_EPI_STORE = 0,      /* D = acc (+ bias[n] if bias)                                   bf16 */
   FL_EPI_BIAS_GELU = 1,  /* U = acc + bias[n] -> aux_out;  D = gelu_tanh(U)               bf16 */
-  FL_EPI_BIAS_RESID = 2, /* D = acc + bias[n] + alpha * aux[m,n]                          bf16 */
+  FL_EPI_BIAS_RESID = 2, /* D = acc + bias[n] + alpha * R[m,n]                            bf16/fp32 */
   FL_EPI_BIAS_ROPE = 3,  /* D = acc + bias[n]; columns [0, 2*n_heads*head_dim) (q and k) are
                             then rotated: dims [0, rotary_dim) of each head, pairs
                             (i, i + rotary_dim/2), angle pos[m] * rope_base^(-2i/rotary_dim)
                             taken from rope_tab[pos[m]][i] = (cos, sin)                  bf16 */
   FL_EPI_GELU_BWD = 4,   /* D = acc * gelu_tanh'(aux[m,n])   (aux = pre-activation U)     bf16 */
-  FL_EPI_RESID = 5,      /* D = acc + alpha * aux[m,n]                                    bf16 */
+  FL_EPI_RESID = 5,      /* D = acc + alpha * R[m,n]                                      bf16/fp32 */
   FL_EPI_ACCUM_F32 = 6,  /* D[m,n] += acc                                                 fp32 */
   FL_EPI_STORE_F32 = 7,  /* D[m,n] = acc                                                  fp32 */
   FL_EPI_COUNT
@@ -42,6 +45,10 @@ enum {
  * A(m,k) is A[m*lda + k] when a_mn_major == 0 (row-major [M,K]) and A[k*lda + m] when
  * a_mn_major == 1 (row-major [K,M]); B(n,k) likewise with ldb / b_mn_major.
  * Forward GEMMs are (0,0), data-gradient GEMMs (0,1), weight-gradient GEMMs (1,1).
+ * Residual epilogues: R = aux (aux_dtype bf16 or fp32), or, when ln_mean != NULL, the
+ * LayerNorm of aux recomputed in fp32: R = (aux[m,n] - ln_mean[m]) ln_rstd[m] ln_gamma[n]
+ * + ln_beta[n] (this keeps the alpha-scaled residual stream of a block in fp32).
+ * d_dtype selects a bf16 or fp32 D for FL_EPI_STORE, FL_EPI_BIAS_RESID and FL_EPI_RESID.
  * Requirements: N % 128 == 0; K % 8 == 0 when a or b is K-major; lda, ldb, ldd,
  * ld_aux, ld_aux_out multiples of 8 elements; pointers 16-byte aligned.  M and K may
  * be ragged (zero-filled by the tensor-memory-accelerator loads). */
@@ -58,22 +65,30 @@ typedef struct {
   const int32_t* pos;                       /* [M] positions for BIAS_ROPE */
   const float* rope_tab;                    /* [max_pos][rotary_dim/2][2] for BIAS_ROPE */
   int32_t n_heads, head_dim, rotary_dim;
+  int32_t aux_dtype;                        /* FL_DT_BF16 or FL_DT_F32 (residual epilogues) */
+  int32_t d_dtype;                          /* FL_DT_BF16 or FL_DT_F32 (STORE / residual epilogues) */
+  const float* ln_mean;                     /* [M] or NULL: residual = LayerNorm of aux */
+  const float* ln_rstd;                     /* [M] */
+  const float* ln_gamma;                    /* [N] */
+  const float* ln_beta;                     /* [N] */
 } fl_gemm_args;
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);
 
-/* Row LayerNorm, biased variance, fp32 statistics.  x, y: bf16 [T,H]; mean, rstd: [T]. */
-int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, const float* gamma, const float* beta,
-                       float eps, void* y, float* mean, float* rstd, void* stream);
+/* Row LayerNorm, biased variance, fp32 statistics.  x: [T,H] of x_dtype (bf16 or fp32);
+ * y: bf16 [T,H]; mean, rstd: [T].  H a power of two in [256, 4096]. */
+int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x_dtype, const float* gamma,
+                       const float* beta, float eps, void* y, float* mean, float* rstd, void* stream);
 
-/* LayerNorm backward.  dy, x: bf16 [T,H]; dx = rstd (g - mean(g) - xhat mean(g xhat)),
- * g = gamma dy, plus resid_alpha * resid[t,:] when resid != NULL (bf16 [T,H]).
+/* LayerNorm backward.  dy, x and resid are [T,H] of io_dtype (bf16 or fp32);
+ * dx = rstd (g - mean(g) - xhat mean(g xhat)), g = gamma dy, plus resid_alpha * resid[t,:]
+ * when resid != NULL; written to dx_bf16 and/or dx_f32 (either may be NULL, not both).
  * dgamma[H] += sum_t dy xhat and dbeta[H] += sum_t dy (fp32, accumulated).
  * workspace: fp32 scratch of at least fl_k_layernorm_bwd_workspace(T, H) bytes. */
 size_t fl_k_layernorm_bwd_workspace(int32_t T, int32_t H);
-int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
+int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, int32_t io_dtype, const float* mean,
                        const float* rstd, const float* gamma, const void* resid, float resid_alpha,
-                       void* dx, float* dgamma, float* dbeta, void* workspace, void* stream);
+                       void* dx_bf16, float* dx_f32, float* dgamma, float* dbeta, void* workspace, void* stream);
 
 /* Allocation-free variant of fl_k_layernorm_bwd (same arguments minus the workspace,
  * same results up to the summation order of dgamma/dbeta).  The paper has no

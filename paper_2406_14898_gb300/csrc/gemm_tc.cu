@@ -55,6 +55,8 @@ struct Epi {
   const float2* rope_tab;  // [pos][rotary_dim/2]
   int rope_cols;           // 2*H: columns that hold q and k
   int head_dim, rotary_dim;
+  int aux_f32, d_f32;
+  const float *ln_mean, *ln_rstd, *ln_gamma, *ln_beta;  // residual = LayerNorm(aux) when ln_mean
 };
 
 FL_DEV void store_bf16x64(__nv_bfloat16* dst, const float* v) {
@@ -101,7 +103,29 @@ FL_DEV void epilogue64(const Epi& e, int m, int n0, float* v) {
     case FL_EPI_BIAS_RESID:
     case FL_EPI_RESID: {
       float r[64];
-      load_bf16x64(e.aux + (int64_t)m * e.ld_aux + n0, r);
+      if (e.aux_f32) {
+        const float4* a4 = reinterpret_cast<const float4*>(reinterpret_cast<const float*>(e.aux) + (int64_t)m * e.ld_aux + n0);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float4 q = __ldg(a4 + j);
+          r[4 * j] = q.x; r[4 * j + 1] = q.y; r[4 * j + 2] = q.z; r[4 * j + 3] = q.w;
+        }
+      } else {
+        load_bf16x64(e.aux + (int64_t)m * e.ld_aux + n0, r);
+      }
+      if (e.ln_mean) {  // residual = LayerNorm(aux), recomputed in fp32
+        const float mu = __ldg(e.ln_mean + m), rs = __ldg(e.ln_rstd + m);
+        const float4* g4 = reinterpret_cast<const float4*>(e.ln_gamma + n0);
+        const float4* b4 = reinterpret_cast<const float4*>(e.ln_beta + n0);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float4 g = __ldg(g4 + j), b = __ldg(b4 + j);
+          r[4 * j] = (r[4 * j] - mu) * rs * g.x + b.x;
+          r[4 * j + 1] = (r[4 * j + 1] - mu) * rs * g.y + b.y;
+          r[4 * j + 2] = (r[4 * j + 2] - mu) * rs * g.z + b.z;
+          r[4 * j + 3] = (r[4 * j + 3] - mu) * rs * g.w + b.w;
+        }
+      }
 #pragma unroll
       for (int j = 0; j < 64; ++j) v[j] = fmaf(e.alpha, r[j], v[j]);
       break;
@@ -148,7 +172,7 @@ FL_DEV void epilogue64(const Epi& e, int m, int n0, float* v) {
       o.x += v[4 * j]; o.y += v[4 * j + 1]; o.z += v[4 * j + 2]; o.w += v[4 * j + 3];
       d[j] = o;
     }
-  } else if (e.mode == FL_EPI_STORE_F32) {
+  } else if (e.mode == FL_EPI_STORE_F32 || e.d_f32) {
     float4* d = reinterpret_cast<float4*>(reinterpret_cast<float*>(e.D) + (int64_t)m * e.ldd + n0);
 #pragma unroll
     for (int j = 0; j < 16; ++j) d[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
@@ -481,6 +505,15 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   if ((mode == FL_EPI_BIAS_RESID || mode == FL_EPI_RESID || mode == FL_EPI_GELU_BWD) &&
       (!a->aux || (a->ld_aux % 8) || !aligned16(a->aux)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: epilogue needs an aligned aux tensor");
+  if ((a->aux_dtype != FL_DT_BF16 && a->aux_dtype != FL_DT_F32) || (a->d_dtype != FL_DT_BF16 && a->d_dtype != FL_DT_F32))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: aux/d dtype");
+  if (a->aux_dtype == FL_DT_F32 && !(mode == FL_EPI_BIAS_RESID || mode == FL_EPI_RESID))
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: fp32 aux only for the residual epilogues");
+  if (a->d_dtype == FL_DT_F32 && !(mode == FL_EPI_STORE || mode == FL_EPI_BIAS_RESID || mode == FL_EPI_RESID))
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: fp32 D only for STORE and the residual epilogues");
+  if (a->ln_mean && (!a->ln_rstd || !a->ln_gamma || !a->ln_beta || !aligned16(a->ln_gamma) || !aligned16(a->ln_beta) ||
+                     !(mode == FL_EPI_BIAS_RESID || mode == FL_EPI_RESID)))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: LayerNorm residual needs mean, rstd, gamma, beta");
   if (mode == FL_EPI_BIAS_GELU && (!a->aux_out || (a->ld_aux_out % 8) || !aligned16(a->aux_out)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: GeLU epilogue needs aux_out");
   if (mode == FL_EPI_BIAS_ROPE) {
@@ -505,6 +538,12 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   e.rope_cols = 2 * a->n_heads * a->head_dim;
   e.head_dim = a->head_dim > 0 ? a->head_dim : 64;
   e.rotary_dim = a->rotary_dim;
+  e.aux_f32 = a->aux_dtype == FL_DT_F32;
+  e.d_f32 = a->d_dtype == FL_DT_F32 && mode != FL_EPI_ACCUM_F32;
+  e.ln_mean = a->ln_mean;
+  e.ln_rstd = a->ln_rstd;
+  e.ln_gamma = a->ln_gamma;
+  e.ln_beta = a->ln_beta;
 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   // Tile width: 256 columns unless 128 gives clearly fewer idle SM slots in the last wave.

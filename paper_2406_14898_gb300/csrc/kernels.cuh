@@ -8,12 +8,21 @@ constexpr int FL_MAX_SEGS = 1024;     // causal segments per call
 constexpr int FL_MAX_TILES = 2048;    // 64-row attention tiles per call
 constexpr int FL_ATTN_TILE = 64;
 
+// Client <-> packed copies.  Units of 8 elements (16 bytes of bf16, 32 bytes of fp32).
+enum CopyMode {
+  COPY_GATHER_BF16 = 0,   // client bf16 -> packed bf16 (bit-exact)
+  COPY_SCATTER_BF16 = 1,  // packed bf16 -> client bf16 (bit-exact)
+  COPY_GATHER_F32 = 2,    // client bf16 -> packed fp32 (exact widening) and, if packed_bf16, a bf16 copy
+  COPY_SCATTER_F32 = 3,   // packed fp32 -> client bf16 (round to nearest even)
+};
 struct CopyTable {
   int n;
-  void* packed;
+  int mode;
+  void* packed_bf16;
+  float* packed_f32;
   void* client[FL_MAX_COPY];
-  int64_t off16[FL_MAX_COPY];  // offset into packed, 16-byte words
-  int64_t n16[FL_MAX_COPY];    // length, 16-byte words
+  int64_t off8[FL_MAX_COPY];  // offset into the packed buffer, 8-element units
+  int64_t n8[FL_MAX_COPY];    // length, 8-element units
 };
 
 // Packing metadata of one call, passed by value to the metadata kernel.
@@ -26,7 +35,7 @@ struct MetaArgs {
   uint32_t tiles[FL_MAX_TILES];
 };
 
-int fl_launch_gather_scatter(const CopyTable& tab, int scatter, cudaStream_t st);
+int fl_launch_copy_clients(const CopyTable& tab, cudaStream_t st);
 int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st);
 int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, float* out, cudaStream_t st);
 int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st);

@@ -44,12 +44,26 @@ FL_DEV uint4 pack8(const float* f) {
   return w;
 }
 
+// ------------------------------------------------------------------ typed 8-element chunks
+template <typename T>
+FL_DEV void load8(const T* base, int64_t chunk, float* f);
+template <>
+FL_DEV void load8<__nv_bfloat16>(const __nv_bfloat16* base, int64_t chunk, float* f) {
+  unpack8(__ldg(reinterpret_cast<const uint4*>(base) + chunk), f);
+}
+template <>
+FL_DEV void load8<float>(const float* base, int64_t chunk, float* f) {
+  const float4 a = __ldg(reinterpret_cast<const float4*>(base) + 2 * chunk);
+  const float4 b = __ldg(reinterpret_cast<const float4*>(base) + 2 * chunk + 1);
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+}
+
 // ------------------------------------------------------------------ LayerNorm forward
 // One warp per row; lane l owns the 8-element chunks l, l+32, l+64, ... (NV chunks).  The
-// row stays in registers as packed bf16 (4 registers per chunk) across the mean, variance
-// and output passes, so HBM is read once and written once.
-template <int NV>
-__global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bfloat16* __restrict__ x,
+// row stays in registers (packed bf16, or fp32) across the mean, variance and output
+// passes, so HBM is read once and written once.  Output y is bf16 (a GEMM operand).
+template <int NV, typename TX>
+__global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const TX* __restrict__ x,
                                                      const float* __restrict__ gamma,
                                                      const float* __restrict__ beta, float eps,
                                                      __nv_bfloat16* __restrict__ y, float* __restrict__ mean,
@@ -57,15 +71,29 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= T) return;
-  const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
-  uint4 raw[NV];
+  const TX* xr = x + (int64_t)row * H;
+  constexpr bool PACKED = sizeof(TX) == 2;
+  uint4 raw[PACKED ? NV : 1];
+  float vals[PACKED ? 1 : NV * 8];
 #pragma unroll
-  for (int i = 0; i < NV; ++i) raw[i] = __ldg(xr + lane + 32 * i);
+  for (int i = 0; i < NV; ++i) {
+    if constexpr (PACKED) raw[i] = __ldg(reinterpret_cast<const uint4*>(xr) + lane + 32 * i);
+    else load8<float>(reinterpret_cast<const float*>(xr), lane + 32 * i, vals + 8 * i);
+  }
+  auto get = [&](int i, float* f) {
+    if constexpr (PACKED) {
+      opaque(raw[i]);
+      unpack8(raw[i], f);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) f[j] = vals[8 * i + j];
+    }
+  };
   float s = 0.f;
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     float f[8];
-    unpack8(raw[i], f);
+    get(i, f);
 #pragma unroll
     for (int j = 0; j < 8; ++j) s += f[j];
   }
@@ -74,8 +102,7 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
 #pragma unroll
   for (int i = 0; i < NV; ++i) {
     float f[8];
-    opaque(raw[i]);
-    unpack8(raw[i], f);
+    get(i, f);
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const float d = f[j] - mu;
@@ -94,8 +121,7 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
     const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
     const float bt[8] = {ba.x, ba.y, ba.z, ba.w, bb.x, bb.y, bb.z, bb.w};
     float f[8], o[8];
-    opaque(raw[i]);
-    unpack8(raw[i], f);
+    get(i, f);
 #pragma unroll
     for (int j = 0; j < 8; ++j) o[j] = (f[j] - mu) * rs * gg[j] + bt[j];
     yr[c] = pack8(o);
@@ -108,21 +134,21 @@ __global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const __nv_bf
 
 // ------------------------------------------------------------------ LayerNorm backward
 // A CTA takes tiles of LN_R rows.  Phase 1: one warp per row computes mean(g) and
-// mean(g xhat), g = gamma dy (lane-strided 16-byte chunks).  Phase 2: thread t owns the
+// mean(g xhat), g = gamma dy (lane-strided 8-element chunks).  Phase 2: thread t owns the
 // column chunks t, t+256, ... of every row of the tile; it re-reads dy and x (L2 hits),
-// writes dx and keeps its columns' dgamma/dbeta partials in registers across all the
-// CTA's tiles.  The partials go to workspace[blockIdx.x][2][H]; ln_bwd_reduce_kernel
-// adds them into dgamma/dbeta.
+// writes dx (bf16 and/or fp32) and keeps its columns' dgamma/dbeta partials in registers
+// across all the CTA's tiles.  The partials go to workspace[blockIdx.x][2][H];
+// ln_bwd_reduce_kernel adds them into dgamma/dbeta.  dy, x and the optional residual
+// gradient share one element type T (bf16 or fp32).
 constexpr int LN_R = 16;
 
-template <int NV>
-__global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bfloat16* __restrict__ dy,
-                                                     const __nv_bfloat16* __restrict__ x,
+template <int NV, typename T>
+__global__ void __launch_bounds__(256) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy, const T* __restrict__ x,
                                                      const float* __restrict__ mean,
                                                      const float* __restrict__ rstd,
-                                                     const float* __restrict__ gamma,
-                                                     const __nv_bfloat16* __restrict__ resid, float resid_alpha,
-                                                     __nv_bfloat16* __restrict__ dx, float* __restrict__ ws) {
+                                                     const float* __restrict__ gamma, const T* __restrict__ resid,
+                                                     float resid_alpha, __nv_bfloat16* __restrict__ dx_bf16,
+                                                     float* __restrict__ dx_f32, float* __restrict__ ws) {
   constexpr int CPT = (NV * 32 + 255) / 256;  // column chunks per thread in phase 2
   __shared__ float s_mg[LN_R], s_mgx[LN_R];
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
@@ -140,21 +166,21 @@ __global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bf
       gcol[j][4] = gb.x; gcol[j][5] = gb.y; gcol[j][6] = gb.z; gcol[j][7] = gb.w;
     }
   }
-  for (int r0 = blockIdx.x * LN_R; r0 < T; r0 += gridDim.x * LN_R) {
+  for (int r0 = blockIdx.x * LN_R; r0 < Tn; r0 += gridDim.x * LN_R) {
     // phase 1: per-row sums
     for (int rr = wid; rr < LN_R; rr += 8) {
       const int row = r0 + rr;
       float s1 = 0.f, s2 = 0.f;
-      if (row < T) {
-        const uint4* dyr = reinterpret_cast<const uint4*>(dy + (int64_t)row * H);
-        const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
+      if (row < Tn) {
+        const T* dyr = dy + (int64_t)row * H;
+        const T* xr = x + (int64_t)row * H;
         const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
 #pragma unroll 4
         for (int i = 0; i < NV; ++i) {
           const int c = lane + 32 * i;
           float d[8], xv[8];
-          unpack8(__ldg(dyr + c), d);
-          unpack8(__ldg(xr + c), xv);
+          load8<T>(dyr, c, d);
+          load8<T>(xr, c, xv);
           const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
           const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
 #pragma unroll
@@ -174,22 +200,21 @@ __global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bf
     }
     __syncthreads();
     // phase 2: dx and the column partials
-    const int rows = min(LN_R, T - r0);
+    const int rows = min(LN_R, Tn - r0);
     for (int rr = 0; rr < rows; ++rr) {
       const int row = r0 + rr;
       const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
       const float mg = s_mg[rr], mgx = s_mgx[rr];
-      const uint4* dyr = reinterpret_cast<const uint4*>(dy + (int64_t)row * H);
-      const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)row * H);
-      const uint4* rr4 = resid ? reinterpret_cast<const uint4*>(resid + (int64_t)row * H) : nullptr;
-      uint4* dxr = reinterpret_cast<uint4*>(dx + (int64_t)row * H);
+      const T* dyr = dy + (int64_t)row * H;
+      const T* xr = x + (int64_t)row * H;
+      const T* rr4 = resid ? resid + (int64_t)row * H : nullptr;
 #pragma unroll
       for (int j = 0; j < CPT; ++j) {
         const int c = tid + 256 * j;
         if (c < nchunk) {
           float d[8], xv[8], o[8];
-          unpack8(__ldg(dyr + c), d);
-          unpack8(__ldg(xr + c), xv);
+          load8<T>(dyr, c, d);
+          load8<T>(xr, c, xv);
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const float xh = (xv[k] - mu) * rs;
@@ -199,11 +224,16 @@ __global__ void __launch_bounds__(256) ln_bwd_kernel(int T, int H, const __nv_bf
           }
           if (rr4) {
             float r[8];
-            unpack8(__ldg(rr4 + c), r);
+            load8<T>(rr4, c, r);
 #pragma unroll
             for (int k = 0; k < 8; ++k) o[k] = fmaf(resid_alpha, r[k], o[k]);
           }
-          dxr[c] = pack8(o);
+          if (dx_bf16) reinterpret_cast<uint4*>(dx_bf16 + (int64_t)row * H)[c] = pack8(o);
+          if (dx_f32) {
+            float4* df = reinterpret_cast<float4*>(dx_f32 + (int64_t)row * H) + 2 * c;
+            df[0] = make_float4(o[0], o[1], o[2], o[3]);
+            df[1] = make_float4(o[4], o[5], o[6], o[7]);
+          }
         }
       }
     }
@@ -238,14 +268,48 @@ __global__ void ln_bwd_reduce_kernel(int nblk, int H, const float* __restrict__ 
 }
 
 // Launches the backward kernel and the reduction of its partials.
-template <int NV>
-int launch_ln_bwd(int nblk, int T, int H, const __nv_bfloat16* dy, const __nv_bfloat16* x, const float* mean,
-                  const float* rstd, const float* gamma, const __nv_bfloat16* resid, float alpha, __nv_bfloat16* dx,
-                  float* ws, float* dgamma, float* dbeta, cudaStream_t st) {
-  ln_bwd_kernel<NV><<<nblk, 256, 0, st>>>(T, H, dy, x, mean, rstd, gamma, resid, alpha, dx, ws);
+template <int NV, typename T>
+int launch_ln_bwd(int nblk, int Tn, int H, const T* dy, const T* x, const float* mean, const float* rstd,
+                  const float* gamma, const T* resid, float alpha, __nv_bfloat16* dx_bf16, float* dx_f32, float* ws,
+                  float* dgamma, float* dbeta, cudaStream_t st) {
+  ln_bwd_kernel<NV, T><<<nblk, 256, 0, st>>>(Tn, H, dy, x, mean, rstd, gamma, resid, alpha, dx_bf16, dx_f32, ws);
   FL_CUDA_TRY(cudaGetLastError());
   const int split = nblk >= 64 ? 16 : 1;
   ln_bwd_reduce_kernel<<<dim3((2 * H + 255) / 256, split), 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+template <typename T>
+int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, const float* mean, const float* rstd,
+                    const float* gamma, const void* resid, float alpha, void* dx_bf16, float* dx_f32, float* ws,
+                    float* dgamma, float* dbeta, cudaStream_t st) {
+  auto dyp = (const T*)dy;
+  auto xp = (const T*)x;
+  auto rp = (const T*)resid;
+  auto dxb = (__nv_bfloat16*)dx_bf16;
+  switch (H / 256) {
+#define FL_LNB(NV) \
+  case NV: return launch_ln_bwd<NV, T>(nblk, Tn, H, dyp, xp, mean, rstd, gamma, rp, alpha, dxb, dx_f32, ws, dgamma, dbeta, st);
+    FL_LNB(1) FL_LNB(2) FL_LNB(4) FL_LNB(8) FL_LNB(16)
+#undef FL_LNB
+    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H/256 must be a power of two");
+  }
+}
+
+template <typename TX>
+int dispatch_ln_fwd(int Tn, int H, const void* x, const float* gamma, const float* beta, float eps, void* y,
+                    float* mean, float* rstd, cudaStream_t st) {
+  const dim3 grid((Tn + 7) / 8), block(256);
+  auto xp = (const TX*)x;
+  auto yb = (__nv_bfloat16*)y;
+  switch (H / 256) {
+#define FL_LNF(NV) \
+  case NV: ln_fwd_kernel<NV, TX><<<grid, block, 0, st>>>(Tn, H, xp, gamma, beta, eps, yb, mean, rstd); break;
+    FL_LNF(1) FL_LNF(2) FL_LNF(4) FL_LNF(8) FL_LNF(16)
+#undef FL_LNF
+    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H/256 must be a power of two");
+  }
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
@@ -320,17 +384,35 @@ __global__ void f32_to_bf16_kernel(int64_t n, const float* __restrict__ src, __n
 }
 
 // ------------------------------------------------------------------ pack / unpack
-__global__ void gather_scatter_kernel(CopyTable tab, int scatter) {
-  // blockIdx.y = entry; each entry copies n16 16-byte words between a client buffer and
-  // the packed buffer.
+// blockIdx.y = table entry; each entry moves n8 groups of 8 elements between a client
+// buffer (bf16) and the packed buffer (bf16 or fp32).
+__global__ void copy_clients_kernel(CopyTable tab) {
   const int e = blockIdx.y;
   if (e >= tab.n) return;
-  const int64_t n16 = tab.n16[e];
-  uint4* packed = reinterpret_cast<uint4*>(tab.packed) + tab.off16[e];
+  const int64_t n8 = tab.n8[e], off = tab.off8[e];
   uint4* client = reinterpret_cast<uint4*>(tab.client[e]);
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n16; i += (int64_t)gridDim.x * blockDim.x) {
-    if (scatter) client[i] = packed[i];
-    else packed[i] = client[i];
+  uint4* pb = tab.packed_bf16 ? reinterpret_cast<uint4*>(tab.packed_bf16) + off : nullptr;
+  float4* pf = tab.packed_f32 ? reinterpret_cast<float4*>(tab.packed_f32) + 2 * off : nullptr;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8; i += (int64_t)gridDim.x * blockDim.x) {
+    switch (tab.mode) {
+      case COPY_GATHER_BF16: pb[i] = client[i]; break;
+      case COPY_SCATTER_BF16: client[i] = pb[i]; break;
+      case COPY_GATHER_F32: {
+        const uint4 w = client[i];
+        if (pb) pb[i] = w;
+        float f[8];
+        unpack8(w, f);
+        pf[2 * i] = make_float4(f[0], f[1], f[2], f[3]);
+        pf[2 * i + 1] = make_float4(f[4], f[5], f[6], f[7]);
+        break;
+      }
+      default: {  // COPY_SCATTER_F32
+        const float4 a = pf[2 * i], b = pf[2 * i + 1];
+        const float f[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        client[i] = pack8(f);
+        break;
+      }
+    }
   }
 }
 
@@ -396,51 +478,38 @@ int grid_for(int64_t n, int per_thread_block = 256) {
 
 // ====================================================================== exported kernel API
 
-extern "C" int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, const float* gamma, const float* beta,
-                                  float eps, void* y, float* mean, float* rstd, void* stream) {
+extern "C" int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x_dtype, const float* gamma,
+                                  const float* beta, float eps, void* y, float* mean, float* rstd, void* stream) {
   if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d", H);
   if (!x || !gamma || !beta || !y || !mean || !rstd) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: null");
+  if (x_dtype != FL_DT_BF16 && x_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: dtype");
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
-  const dim3 grid((T + 7) / 8), block(256);
-  auto xb = (const __nv_bfloat16*)x;
-  auto yb = (__nv_bfloat16*)y;
-  switch (H / 256) {
-#define FL_LNF(NV) \
-  case NV: ln_fwd_kernel<NV><<<grid, block, 0, st>>>(T, H, xb, gamma, beta, eps, yb, mean, rstd); break;
-    FL_LNF(1) FL_LNF(2) FL_LNF(4) FL_LNF(8) FL_LNF(16)
-#undef FL_LNF
-    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H/256 must be a power of two");
-  }
-  FL_CUDA_TRY(cudaGetLastError());
-  return FL_OK;
+  return x_dtype == FL_DT_F32 ? dispatch_ln_fwd<float>(T, H, x, gamma, beta, eps, y, mean, rstd, st)
+                              : dispatch_ln_fwd<__nv_bfloat16>(T, H, x, gamma, beta, eps, y, mean, rstd, st);
 }
 
 extern "C" size_t fl_k_layernorm_bwd_workspace(int32_t T, int32_t H) {
   return (size_t)ln_bwd_blocks(T > 0 ? T : 1) * 2 * (size_t)H * sizeof(float);
 }
 
-extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
-                                  const float* rstd, const float* gamma, const void* resid, float resid_alpha,
-                                  void* dx, float* dgamma, float* dbeta, void* workspace, void* stream) {
+extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, int32_t io_dtype,
+                                  const float* mean, const float* rstd, const float* gamma, const void* resid,
+                                  float resid_alpha, void* dx_bf16, float* dx_f32, float* dgamma, float* dbeta,
+                                  void* workspace, void* stream) {
   if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H=%d", H);
-  if (!dy || !x || !mean || !rstd || !gamma || !dx || !dgamma || !dbeta || !workspace)
+  if (!dy || !x || !mean || !rstd || !gamma || (!dx_bf16 && !dx_f32) || !dgamma || !dbeta || !workspace)
     return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: null");
+  if (io_dtype != FL_DT_BF16 && io_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: dtype");
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
   const int nblk = ln_bwd_blocks(T);
   float* ws = (float*)workspace;
-  auto dyb = (const __nv_bfloat16*)dy;
-  auto xb = (const __nv_bfloat16*)x;
-  auto rb = (const __nv_bfloat16*)resid;
-  auto dxb = (__nv_bfloat16*)dx;
-  switch (H / 256) {
-#define FL_LNB(NV) \
-  case NV: return launch_ln_bwd<NV>(nblk, T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws, dgamma, dbeta, st);
-    FL_LNB(1) FL_LNB(2) FL_LNB(4) FL_LNB(8) FL_LNB(16)
-#undef FL_LNB
-    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H/256 must be a power of two");
-  }
+  return io_dtype == FL_DT_F32
+             ? dispatch_ln_bwd<float>(nblk, T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16, dx_f32, ws,
+                                      dgamma, dbeta, st)
+             : dispatch_ln_bwd<__nv_bfloat16>(nblk, T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16,
+                                              dx_f32, ws, dgamma, dbeta, st);
 }
 
 extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream) {
@@ -481,15 +550,15 @@ int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_b
 
 // ====================================================================== internal launchers
 
-int fl_launch_gather_scatter(const CopyTable& tab, int scatter, cudaStream_t st) {
+int fl_launch_copy_clients(const CopyTable& tab, cudaStream_t st) {
   if (tab.n <= 0) return FL_OK;
   int64_t maxn = 0;
-  for (int e = 0; e < tab.n; ++e) maxn = tab.n16[e] > maxn ? tab.n16[e] : maxn;
+  for (int e = 0; e < tab.n; ++e) maxn = tab.n8[e] > maxn ? tab.n8[e] : maxn;
   int gx = (int)((maxn + 255) / 256);
   const int cap = (2 * sm_count() + tab.n - 1) / tab.n + 1;
   if (gx > cap) gx = cap;
   if (gx < 1) gx = 1;
-  gather_scatter_kernel<<<dim3(gx, tab.n), 256, 0, st>>>(tab, scatter);
+  copy_clients_kernel<<<dim3(gx, tab.n), 256, 0, st>>>(tab);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
@@ -531,18 +600,20 @@ extern "C" int fl_k_pack_clients(int32_t K, void* const* clients_host, const int
   for (int k0 = 0; k0 < K; k0 += FL_MAX_COPY) {
     CopyTable tab;
     tab.n = (K - k0) < FL_MAX_COPY ? (K - k0) : FL_MAX_COPY;
-    tab.packed = packed;
+    tab.mode = scatter ? COPY_SCATTER_BF16 : COPY_GATHER_BF16;
+    tab.packed_bf16 = packed;
+    tab.packed_f32 = nullptr;
     for (int e = 0; e < tab.n; ++e) {
       const int k = k0 + e;
       if (!clients_host[k] || (reinterpret_cast<uintptr_t>(clients_host[k]) & 15) || bytes_host[k] < 0 ||
           (bytes_host[k] % 16))
         return fl_internal_error(FL_ERR_INVALID_ARG, "pack: client %d pointer/size", k);
       tab.client[e] = clients_host[k];
-      tab.off16[e] = off / 16;
-      tab.n16[e] = bytes_host[k] / 16;
+      tab.off8[e] = off / 16;
+      tab.n8[e] = bytes_host[k] / 16;
       off += bytes_host[k];
     }
-    if (int rc = fl_launch_gather_scatter(tab, scatter, (cudaStream_t)stream)) return rc;
+    if (int rc = fl_launch_copy_clients(tab, (cudaStream_t)stream)) return rc;
   }
   return FL_OK;
 }
@@ -610,15 +681,6 @@ extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, 
   cudaStream_t st = (cudaStream_t)stream;
   int nblk = ln_bwd_blocks(T);
   if (nblk > FL_LN_NOALLOC_MAX_BLOCKS) nblk = FL_LN_NOALLOC_MAX_BLOCKS;
-  auto dyb = (const __nv_bfloat16*)dy;
-  auto xb = (const __nv_bfloat16*)x;
-  auto rb = (const __nv_bfloat16*)resid;
-  auto dxb = (__nv_bfloat16*)dx;
-  switch (H / 256) {
-#define FL_LNB_NA(NV) \
-  case NV: return launch_ln_bwd<NV>(nblk, T, H, dyb, xb, mean, rstd, gamma, rb, resid_alpha, dxb, ws, dgamma, dbeta, st);
-    FL_LNB_NA(1) FL_LNB_NA(2) FL_LNB_NA(4) FL_LNB_NA(8) FL_LNB_NA(16)
-#undef FL_LNB_NA
-    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd (no-alloc): H/256 must be a power of two");
-  }
+  return dispatch_ln_bwd<__nv_bfloat16>(nblk, T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx, nullptr, ws,
+                                        dgamma, dbeta, st);
 }

@@ -13,9 +13,17 @@
 //                     every block in one contiguous region (block b at vec_base +
 //                     b * vec_stride); every tensor 64-byte aligned;
 //   activations       per block: LN1 out A, rotated QKV, attention O, LSE, residual stream
-//                     Hres, LN2 out M, FFN pre-activation U and GeLU output G, LN statistics;
-//                     xs[0..n_blocks]: block inputs / outputs (xs[0] = packed client states);
-//   backward scratch  one set of gradient buffers reused by every block;
+//                     Hres (fp32), LN2 out M, FFN pre-activation U and GeLU output G, LN
+//                     statistics; xs[0..n_blocks]: block inputs / outputs in fp32
+//                     (xs[0] = packed client states, widened exactly);
+//   backward scratch  one set of gradient buffers reused by every block; the gradient of
+//                     the residual stream is kept in fp32 next to the bf16 copy the GEMMs
+//                     read;
+//
+// Precision: GEMM operands are bf16 (tcgen05 kind::f16), accumulation fp32.  The
+// alpha-scaled residual path (block inputs, Hres, the alpha * LN(.) terms, and their
+// gradients) stays fp32 end to end: with alpha = sqrt(56) it carries most of each
+// block's output, and bf16 roundings on it would add up over 26 blocks.
 //   metadata          cu_seqlens, per-token positions, attention tile list, rotary table.
 #include <cuda_runtime.h>
 
@@ -24,6 +32,7 @@
 #include <cstdio>
 #include <cstring>
 #include <string>
+#include <utility>
 #include <vector>
 
 #include "../../include/flglm.h"
@@ -65,7 +74,8 @@ uint64_t stream_key(uint64_t seed, uint64_t purpose, uint64_t block, uint64_t te
 }
 
 struct BlockAct {
-  __nv_bfloat16 *a, *qkv, *o, *h, *m, *u, *g;
+  __nv_bfloat16 *a, *qkv, *o, *m, *u, *g;
+  float* h;  // residual stream after attention, fp32
   float *mean1, *rstd1, *mean2, *rstd2, *lse;
 };
 
@@ -98,11 +108,12 @@ struct fl_server {
   bool grads_zero = true;
 
   // activations
-  std::vector<__nv_bfloat16*> xs;
+  std::vector<float*> xs;  // block inputs/outputs, fp32
   std::vector<BlockAct> act;
-  // backward scratch
-  __nv_bfloat16 *dy = nullptr, *dx = nullptr, *du = nullptr, *dm = nullptr, *dh = nullptr, *d_o = nullptr,
-                *dqkv = nullptr, *da = nullptr;
+  // backward scratch: gradient of a block's output / input as bf16 (GEMM operand) and
+  // fp32 (residual chain), ping-pong
+  __nv_bfloat16 *dy = nullptr, *dx = nullptr, *du = nullptr, *dh = nullptr, *d_o = nullptr, *dqkv = nullptr;
+  float *dyf = nullptr, *dxf = nullptr, *dm = nullptr, *dhf = nullptr, *da = nullptr;
   float *delta = nullptr, *ln_ws = nullptr;
   // metadata
   int32_t *cu = nullptr, *pos = nullptr;
@@ -253,11 +264,12 @@ int block_forward(fl_server* h, int b) {
   const fl_server_cfg& c = h->cfg;
   const int T = h->T, H = c.hidden, F = c.ffn_hidden;
   BlockAct& A = h->act[b];
-  const __nv_bfloat16* x = h->xs[b];
+  const float* x = h->xs[b];
   cudaStream_t st = h->stream;
   // a = LN1(x)
   prof_begin(h, FL_PROF_LN);
-  TRY(h, fl_k_layernorm_fwd(T, H, x, h->wt(b, FL_T_LN1_G), h->wt(b, FL_T_LN1_B), c.ln_eps, A.a, A.mean1, A.rstd1, st));
+  TRY(h, fl_k_layernorm_fwd(T, H, x, FL_DT_F32, h->wt(b, FL_T_LN1_G), h->wt(b, FL_T_LN1_B), c.ln_eps, A.a, A.mean1,
+                            A.rstd1, st));
   prof_end(h);
   // qkv = a Wqkv^T + bqkv, q and k rotated
   fl_gemm_args g1 = gemm_fwd(T, 3 * H, H, A.a, h->wbt(b, FL_T_WQKV), A.qkv, FL_EPI_BIAS_ROPE);
@@ -272,16 +284,25 @@ int block_forward(fl_server* h, int b) {
   prof_begin(h, FL_PROF_ATTN);
   TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse, st));
   prof_end(h);
-  // h = alpha * (a or x) + o Wd^T + bd
+  // h = alpha * (LN1(x) or x) + o Wd^T + bd, fp32; LN1(x) recomputed in fp32 in the epilogue
   fl_gemm_args g2 = gemm_fwd(T, H, H, A.o, h->wbt(b, FL_T_WDENSE), A.h, FL_EPI_BIAS_RESID);
   g2.bias = h->wt(b, FL_T_BDENSE);
-  g2.aux = c.residual_from_ln ? (const void*)A.a : (const void*)x;
+  g2.aux = x;
+  g2.aux_dtype = FL_DT_F32;
   g2.ld_aux = H;
+  g2.d_dtype = FL_DT_F32;
   g2.alpha = c.residual_alpha;
+  if (c.residual_from_ln) {
+    g2.ln_mean = A.mean1;
+    g2.ln_rstd = A.rstd1;
+    g2.ln_gamma = h->wt(b, FL_T_LN1_G);
+    g2.ln_beta = h->wt(b, FL_T_LN1_B);
+  }
   TRY(h, run_gemm(h, g2));
   // m = LN2(h)
   prof_begin(h, FL_PROF_LN);
-  TRY(h, fl_k_layernorm_fwd(T, H, A.h, h->wt(b, FL_T_LN2_G), h->wt(b, FL_T_LN2_B), c.ln_eps, A.m, A.mean2, A.rstd2, st));
+  TRY(h, fl_k_layernorm_fwd(T, H, A.h, FL_DT_F32, h->wt(b, FL_T_LN2_G), h->wt(b, FL_T_LN2_B), c.ln_eps, A.m,
+                            A.mean2, A.rstd2, st));
   prof_end(h);
   // u = m W1^T + b1, g = gelu(u)
   fl_gemm_args g3 = gemm_fwd(T, F, H, A.m, h->wbt(b, FL_T_WUP), A.g, FL_EPI_BIAS_GELU);
@@ -289,53 +310,64 @@ int block_forward(fl_server* h, int b) {
   g3.aux_out = A.u;
   g3.ld_aux_out = F;
   TRY(h, run_gemm(h, g3));
-  // y = alpha * (m or h) + g W2^T + b2
+  // y = alpha * (LN2(h) or h) + g W2^T + b2, fp32
   fl_gemm_args g4 = gemm_fwd(T, H, F, A.g, h->wbt(b, FL_T_WDOWN), h->xs[b + 1], FL_EPI_BIAS_RESID);
   g4.bias = h->wt(b, FL_T_BDOWN);
-  g4.aux = c.residual_from_ln ? (const void*)A.m : (const void*)A.h;
+  g4.aux = A.h;
+  g4.aux_dtype = FL_DT_F32;
   g4.ld_aux = H;
+  g4.d_dtype = FL_DT_F32;
   g4.alpha = c.residual_alpha;
+  if (c.residual_from_ln) {
+    g4.ln_mean = A.mean2;
+    g4.ln_rstd = A.rstd2;
+    g4.ln_gamma = h->wt(b, FL_T_LN2_G);
+    g4.ln_beta = h->wt(b, FL_T_LN2_B);
+  }
   TRY(h, run_gemm(h, g4));
   return FL_OK;
 }
 
-// dy holds dL/dy of block b; on return dx holds dL/dx.
-int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* dx) {
+// dy / dyf hold dL/dy of block b (bf16 and fp32); on return dx / dxf hold dL/dx.
+int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dyf, __nv_bfloat16* dx, float* dxf) {
   const fl_server_cfg& c = h->cfg;
   const int T = h->T, H = c.hidden, F = c.ffn_hidden;
   const float al = c.residual_alpha;
   const bool glm = c.residual_from_ln != 0;
   BlockAct& A = h->act[b];
   cudaStream_t st = h->stream;
+  const bool store = h->grads_zero;
   // FFN down: du = (dy W2) * gelu'(u); dW2 += dy^T g; db2 += colsum(dy)
   fl_gemm_args d1 = gemm_dgrad(T, F, H, dy, h->wbt(b, FL_T_WDOWN), h->du, FL_EPI_GELU_BWD);
   d1.aux = A.u;
   d1.ld_aux = F;
   TRY(h, run_gemm(h, d1));
-  TRY(h, run_gemm(h, gemm_wgrad(T, H, F, dy, A.g, h->gt(b, FL_T_WDOWN), h->grads_zero)));
+  TRY(h, run_gemm(h, gemm_wgrad(T, H, F, dy, A.g, h->gt(b, FL_T_WDOWN), store)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
   prof_end(h);
-  // FFN up: dm = du W1 (+ alpha dy); dW1 += du^T m; db1 += colsum(du)
+  // FFN up: dm = du W1 (+ alpha dy), fp32; dW1 += du^T m; db1 += colsum(du)
   fl_gemm_args d2 = gemm_dgrad(T, H, F, h->du, h->wbt(b, FL_T_WUP), h->dm, glm ? FL_EPI_RESID : FL_EPI_STORE);
+  d2.d_dtype = FL_DT_F32;
   if (glm) {
-    d2.aux = dy;
+    d2.aux = dyf;
+    d2.aux_dtype = FL_DT_F32;
     d2.ld_aux = H;
     d2.alpha = al;
   }
   TRY(h, run_gemm(h, d2));
-  TRY(h, run_gemm(h, gemm_wgrad(T, F, H, h->du, A.m, h->gt(b, FL_T_WUP), h->grads_zero)));
+  TRY(h, run_gemm(h, gemm_wgrad(T, F, H, h->du, A.m, h->gt(b, FL_T_WUP), store)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
   prof_end(h);
-  // LN2 backward: dh = LN2'(dm) (+ alpha dy)
+  // LN2 backward: dh = LN2'(dm) (+ alpha dy), bf16 and fp32
   prof_begin(h, FL_PROF_LN, 2);
-  TRY(h, fl_k_layernorm_bwd(T, H, h->dm, A.h, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dy, al, h->dh,
-                            h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B), h->ln_ws, st));
+  TRY(h, fl_k_layernorm_bwd(T, H, h->dm, A.h, FL_DT_F32, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dyf,
+                            al, h->dh, h->dhf, h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B), h->ln_ws, st));
   prof_end(h);
   // dense: do = dh Wd; dWd += dh^T o; dbd += colsum(dh)
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
-  TRY(h, run_gemm(h, gemm_wgrad(T, H, H, h->dh, A.o, h->gt(b, FL_T_WDENSE), h->grads_zero)));
+  TRY(h, run_gemm(h, gemm_wgrad(T, H, H, h->dh, A.o, h->gt(b, FL_T_WDENSE), store)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
   prof_end(h);
@@ -344,43 +376,49 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, __nv_bfloat16* 
   TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
                             h->pos, h->rope_tab, h->rdim, h->dqkv, st));
   prof_end(h);
-  // QKV: da = dqkv Wqkv (+ alpha dh); dWqkv += dqkv^T a; dbqkv += colsum(dqkv)
+  // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a; dbqkv += colsum(dqkv)
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
+  d3.d_dtype = FL_DT_F32;
   if (glm) {
-    d3.aux = h->dh;
+    d3.aux = h->dhf;
+    d3.aux_dtype = FL_DT_F32;
     d3.ld_aux = H;
     d3.alpha = al;
   }
   TRY(h, run_gemm(h, d3));
-  TRY(h, run_gemm(h, gemm_wgrad(T, 3 * H, H, h->dqkv, A.a, h->gt(b, FL_T_WQKV), h->grads_zero)));
+  TRY(h, run_gemm(h, gemm_wgrad(T, 3 * H, H, h->dqkv, A.a, h->gt(b, FL_T_WQKV), store)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
   prof_end(h);
-  // LN1 backward: dx = LN1'(da) (+ alpha dh)
+  // LN1 backward: dx = LN1'(da) (+ alpha dh), bf16 and fp32
   prof_begin(h, FL_PROF_LN, 2);
-  TRY(h, fl_k_layernorm_bwd(T, H, h->da, h->xs[b], A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G), glm ? nullptr : h->dh, al,
-                            dx, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B), h->ln_ws, st));
+  TRY(h, fl_k_layernorm_bwd(T, H, h->da, h->xs[b], FL_DT_F32, A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G),
+                            glm ? nullptr : h->dhf, al, dx, dxf, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B), h->ln_ws,
+                            st));
   prof_end(h);
   return FL_OK;
 }
 
-int copy_clients(fl_server* h, const void* const* ptrs, __nv_bfloat16* packed, int scatter) {
-  const int64_t row16 = (int64_t)h->cfg.client_batch * h->cfg.hidden * 2 / 16;  // 16-byte words per token row group
+// Moves the K client tensors to / from the packed buffers (mode: CopyMode).
+int copy_clients(fl_server* h, const void* const* ptrs, int mode, __nv_bfloat16* packed_bf16, float* packed_f32) {
+  const int64_t row8 = (int64_t)h->cfg.client_batch * h->cfg.hidden / 8;  // 8-element groups per token
   int64_t off = 0;
   for (int k0 = 0; k0 < h->K; k0 += FL_MAX_COPY) {
     CopyTable tab;
     memset(&tab, 0, sizeof tab);
-    tab.packed = packed;
+    tab.mode = mode;
+    tab.packed_bf16 = packed_bf16;
+    tab.packed_f32 = packed_f32;
     tab.n = (h->K - k0) < FL_MAX_COPY ? (h->K - k0) : FL_MAX_COPY;
     for (int e = 0; e < tab.n; ++e) {
       const int k = k0 + e;
       tab.client[e] = const_cast<void*>(ptrs[k]);
-      tab.off16[e] = off;
-      tab.n16[e] = row16 * h->seq_lens[k];
-      off += tab.n16[e];
+      tab.off8[e] = off;
+      tab.n8[e] = row8 * h->seq_lens[k];
+      off += tab.n8[e];
     }
     prof_begin(h, FL_PROF_OTHER);
-    int rc = fl_launch_gather_scatter(tab, scatter, h->stream);
+    int rc = fl_launch_copy_clients(tab, h->stream);
     prof_end(h);
     if (rc) return fwd_err(h, rc);
   }
@@ -463,7 +501,7 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
   // activations
   h->xs.resize(c.n_blocks + 1);
   for (int b = 0; b <= c.n_blocks; ++b)
-    if ((rc = dalloc(h, &h->xs[b], Tm * H))) return fail(rc);
+    if ((rc = dalloc(h, &h->xs[b], Tm * H))) return fail(rc);  // fp32
   h->act.resize(c.n_blocks);
   for (int b = 0; b < c.n_blocks; ++b) {
     BlockAct& A = h->act[b];
@@ -475,6 +513,7 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
       return fail(rc);
   }
   if ((rc = dalloc(h, &h->dy, Tm * H)) || (rc = dalloc(h, &h->dx, Tm * H)) || (rc = dalloc(h, &h->du, Tm * F)) ||
+      (rc = dalloc(h, &h->dyf, Tm * H)) || (rc = dalloc(h, &h->dxf, Tm * H)) || (rc = dalloc(h, &h->dhf, Tm * H)) ||
       (rc = dalloc(h, &h->dm, Tm * H)) || (rc = dalloc(h, &h->dh, Tm * H)) || (rc = dalloc(h, &h->d_o, Tm * H)) ||
       (rc = dalloc(h, &h->dqkv, Tm * 3 * H)) || (rc = dalloc(h, &h->da, Tm * H)) ||
       (rc = dalloc(h, &h->delta, Tm * c.n_heads)) ||
@@ -559,10 +598,10 @@ extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[
   int rc = fl_launch_meta(meta, h->cu, h->pos, h->tiles, h->stream);
   prof_end(h);
   if (rc) return fwd_err(h, rc);
-  if ((rc = copy_clients(h, client_states, h->xs[0], 0))) return rc;
+  if ((rc = copy_clients(h, client_states, COPY_GATHER_F32, nullptr, h->xs[0]))) return rc;
   for (int blk = 0; blk < c.n_blocks; ++blk)
     if ((rc = block_forward(h, blk))) return rc;
-  if ((rc = copy_clients(h, (const void* const*)out_states, h->xs[c.n_blocks], 1))) return rc;
+  if ((rc = copy_clients(h, (const void* const*)out_states, COPY_SCATTER_F32, nullptr, h->xs[c.n_blocks]))) return rc;
   h->pending = true;
   return FL_OK;
 }
@@ -578,16 +617,17 @@ extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], v
     const cudaError_t e = cudaMemsetAsync(h->g + h->vec_base, 0, (h->n_params - h->vec_base) * sizeof(float), h->stream);
     if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "cudaMemsetAsync", __FILE__, __LINE__));
   }
-  if ((rc = copy_clients(h, grad_out, h->dy, 0))) return rc;
+  if ((rc = copy_clients(h, grad_out, COPY_GATHER_F32, h->dy, h->dyf))) return rc;
   __nv_bfloat16* cur = h->dy;
   __nv_bfloat16* nxt = h->dx;
+  float* curf = h->dyf;
+  float* nxtf = h->dxf;
   for (int blk = h->cfg.n_blocks - 1; blk >= 0; --blk) {
-    if ((rc = block_backward(h, blk, cur, nxt))) return rc;
-    __nv_bfloat16* t = cur;
-    cur = nxt;
-    nxt = t;
+    if ((rc = block_backward(h, blk, cur, curf, nxt, nxtf))) return rc;
+    std::swap(cur, nxt);
+    std::swap(curf, nxtf);
   }
-  if ((rc = copy_clients(h, (const void* const*)grad_in, cur, 1))) return rc;
+  if ((rc = copy_clients(h, (const void* const*)grad_in, COPY_SCATTER_BF16, cur, nullptr))) return rc;
   h->pending = false;
   h->grads_zero = false;
   return FL_OK;

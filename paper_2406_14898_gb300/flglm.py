@@ -25,6 +25,7 @@ FL_T_COUNT = 12
 (FL_EPI_STORE, FL_EPI_BIAS_GELU, FL_EPI_BIAS_RESID, FL_EPI_BIAS_ROPE, FL_EPI_GELU_BWD, FL_EPI_RESID,
  FL_EPI_ACCUM_F32, FL_EPI_STORE_F32) = range(8)
 PROF_CLASSES = ("gemm", "attention", "layernorm", "adamw", "other")
+FL_DT_BF16, FL_DT_F32 = 0, 1
 
 
 class FlError(RuntimeError):
@@ -50,7 +51,9 @@ class fl_gemm_args(C.Structure):
                 ("bias", C.c_void_p), ("aux", C.c_void_p), ("ld_aux", C.c_int64), ("alpha", C.c_float),
                 ("aux_out", C.c_void_p), ("ld_aux_out", C.c_int64), ("pos", C.c_void_p),
                 ("rope_tab", C.c_void_p), ("n_heads", C.c_int32), ("head_dim", C.c_int32),
-                ("rotary_dim", C.c_int32)]
+                ("rotary_dim", C.c_int32), ("aux_dtype", C.c_int32), ("d_dtype", C.c_int32),
+                ("ln_mean", C.c_void_p), ("ln_rstd", C.c_void_p), ("ln_gamma", C.c_void_p),
+                ("ln_beta", C.c_void_p)]
 
 
 _P = C.c_void_p
@@ -76,9 +79,9 @@ _SIGS = {
     "fl_server_launch_count": (_I64, [_P]),
     "fl_server_last_error": (C.c_char_p, [_P]),
     "fl_k_gemm": (C.c_int, [C.POINTER(fl_gemm_args), _P, _P]),
-    "fl_k_layernorm_fwd": (C.c_int, [_I32, _I32, _P, _P, _P, _F, _P, _P, _P, _P]),
+    "fl_k_layernorm_fwd": (C.c_int, [_I32, _I32, _P, _I32, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_layernorm_bwd_workspace": (C.c_size_t, [_I32, _I32]),
-    "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P]),
+    "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _I32, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P]),
     "fl_k_layernorm_bwd_noalloc": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_attention_tiles": (_I32, [_P, _I32]),
     "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P]),
@@ -248,14 +251,16 @@ def fl_k_gemm(args: fl_gemm_args, status=None, stream=None):
 
 def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
          alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
+         aux_dtype=FL_DT_BF16, d_dtype=FL_DT_BF16, ln_mean=None, ln_rstd=None, ln_gamma=None, ln_beta=None,
          status=None, stream=None):
     a = fl_gemm_args(M, N, K, ptr(A), lda, a_mn, ptr(B), ldb, b_mn, ptr(D), ldd, epilogue, ptr(bias), ptr(aux),
-                     ld_aux, alpha, ptr(aux_out), ld_aux_out, ptr(pos), ptr(rope_tab), n_heads, head_dim, rotary_dim)
+                     ld_aux, alpha, ptr(aux_out), ld_aux_out, ptr(pos), ptr(rope_tab), n_heads, head_dim, rotary_dim,
+                     aux_dtype, d_dtype, ptr(ln_mean), ptr(ln_rstd), ptr(ln_gamma), ptr(ln_beta))
     fl_k_gemm(a, status, stream)
 
 
-def fl_k_layernorm_fwd(T, H, x, gamma, beta, eps, y, mean, rstd, stream=None):
-    check(lib().fl_k_layernorm_fwd(T, H, ptr(x), ptr(gamma), ptr(beta), eps, ptr(y), ptr(mean), ptr(rstd),
+def fl_k_layernorm_fwd(T, H, x, gamma, beta, eps, y, mean, rstd, x_dtype=FL_DT_BF16, stream=None):
+    check(lib().fl_k_layernorm_fwd(T, H, ptr(x), x_dtype, ptr(gamma), ptr(beta), eps, ptr(y), ptr(mean), ptr(rstd),
                                    stream_ptr(stream)))
 
 
@@ -263,10 +268,10 @@ def fl_k_layernorm_bwd_workspace(T, H) -> int:
     return int(lib().fl_k_layernorm_bwd_workspace(T, H))
 
 
-def fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx, dgamma, dbeta, workspace,
-                       stream=None):
-    check(lib().fl_k_layernorm_bwd(T, H, ptr(dy), ptr(x), ptr(mean), ptr(rstd), ptr(gamma), ptr(resid),
-                                   resid_alpha, ptr(dx), ptr(dgamma), ptr(dbeta), ptr(workspace),
+def fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16, dgamma, dbeta, workspace,
+                       io_dtype=FL_DT_BF16, dx_f32=None, stream=None):
+    check(lib().fl_k_layernorm_bwd(T, H, ptr(dy), ptr(x), io_dtype, ptr(mean), ptr(rstd), ptr(gamma), ptr(resid),
+                                   resid_alpha, ptr(dx_bf16), ptr(dx_f32), ptr(dgamma), ptr(dbeta), ptr(workspace),
                                    stream_ptr(stream)))
 
 

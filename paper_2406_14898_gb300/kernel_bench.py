@@ -21,22 +21,24 @@ if ROOT not in sys.path:
 
 
 def gemm_cases(cfg):
-    """(name, M, N, K, a_mn, b_mn, epilogue) of the 12 GEMMs of one block, T tokens."""
+    """(name, M, N, K, a_mn, b_mn, epilogue, fp32 residual stream) of the 12 GEMMs of one
+    block at T tokens, with the epilogues the server uses (weight gradients as the first
+    backward after a step stores them)."""
     from paper_2406_14898_gb300 import flglm as F
     T, H, Fh = cfg.tokens, cfg.hidden, cfg.ffn_hidden
     return [
-        ("qkv_fwd", T, 3 * H, H, 0, 0, F.FL_EPI_BIAS_ROPE),
-        ("dense_fwd", T, H, H, 0, 0, F.FL_EPI_BIAS_RESID),
-        ("up_fwd", T, Fh, H, 0, 0, F.FL_EPI_BIAS_GELU),
-        ("down_fwd", T, H, Fh, 0, 0, F.FL_EPI_BIAS_RESID),
-        ("down_dgrad", T, Fh, H, 0, 1, F.FL_EPI_GELU_BWD),
-        ("down_wgrad", H, Fh, T, 1, 1, F.FL_EPI_ACCUM_F32),
-        ("up_dgrad", T, H, Fh, 0, 1, F.FL_EPI_RESID),
-        ("up_wgrad", Fh, H, T, 1, 1, F.FL_EPI_ACCUM_F32),
-        ("dense_dgrad", T, H, H, 0, 1, F.FL_EPI_STORE),
-        ("dense_wgrad", H, H, T, 1, 1, F.FL_EPI_ACCUM_F32),
-        ("qkv_dgrad", T, H, 3 * H, 0, 1, F.FL_EPI_RESID),
-        ("qkv_wgrad", 3 * H, H, T, 1, 1, F.FL_EPI_ACCUM_F32),
+        ("qkv_fwd", T, 3 * H, H, 0, 0, F.FL_EPI_BIAS_ROPE, False),
+        ("dense_fwd", T, H, H, 0, 0, F.FL_EPI_BIAS_RESID, True),
+        ("up_fwd", T, Fh, H, 0, 0, F.FL_EPI_BIAS_GELU, False),
+        ("down_fwd", T, H, Fh, 0, 0, F.FL_EPI_BIAS_RESID, True),
+        ("down_dgrad", T, Fh, H, 0, 1, F.FL_EPI_GELU_BWD, False),
+        ("down_wgrad", H, Fh, T, 1, 1, F.FL_EPI_STORE_F32, False),
+        ("up_dgrad", T, H, Fh, 0, 1, F.FL_EPI_RESID, True),
+        ("up_wgrad", Fh, H, T, 1, 1, F.FL_EPI_STORE_F32, False),
+        ("dense_dgrad", T, H, H, 0, 1, F.FL_EPI_STORE, False),
+        ("dense_wgrad", H, H, T, 1, 1, F.FL_EPI_STORE_F32, False),
+        ("qkv_dgrad", T, H, 3 * H, 0, 1, F.FL_EPI_RESID, True),
+        ("qkv_wgrad", 3 * H, H, T, 1, 1, F.FL_EPI_STORE_F32, False),
     ]
 
 
@@ -76,19 +78,25 @@ def main():
 
     T, H, Fh, nh, hd = cfg.tokens, cfg.hidden, cfg.ffn_hidden, cfg.n_heads, cfg.head_dim
     out = []
-    for (name, M, N, K, amn, bmn, epi) in gemm_cases(cfg):
+    for (name, M, N, K, amn, bmn, epi, f32res) in gemm_cases(cfg):
         if args.kernel not in ("all", "gemm", name):
             continue
         A = rnd(K, M, scale=0.1) if amn else rnd(M, K, scale=0.1)
         B = rnd(K, N, scale=0.1) if bmn else rnd(N, K, scale=0.1)
-        D = torch.zeros(M, N, device=dev, dtype=torch.float32 if epi == F.FL_EPI_ACCUM_F32 else torch.bfloat16)
+        f32_out = epi in (F.FL_EPI_ACCUM_F32, F.FL_EPI_STORE_F32) or f32res
+        D = torch.zeros(M, N, device=dev, dtype=torch.float32 if f32_out else torch.bfloat16)
         kw = {}
         if epi in (F.FL_EPI_BIAS_ROPE, F.FL_EPI_BIAS_RESID, F.FL_EPI_BIAS_GELU):
             kw["bias"] = rnd(N, dtype=torch.float32)
         if epi in (F.FL_EPI_BIAS_RESID, F.FL_EPI_RESID, F.FL_EPI_GELU_BWD):
-            kw["aux"] = rnd(M, N)
+            kw["aux"] = rnd(M, N, dtype=torch.float32 if f32res else torch.bfloat16)
             kw["ld_aux"] = N
             kw["alpha"] = 1.5
+        if f32res:
+            kw.update(aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32)
+            if epi == F.FL_EPI_BIAS_RESID:   # residual = alpha * LN(x) recomputed in the epilogue
+                kw.update(ln_mean=rnd(M, dtype=torch.float32), ln_rstd=rnd(M, dtype=torch.float32),
+                          ln_gamma=rnd(N, dtype=torch.float32), ln_beta=rnd(N, dtype=torch.float32))
         if epi == F.FL_EPI_BIAS_GELU:
             kw["aux_out"] = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
             kw["ld_aux_out"] = N
@@ -122,23 +130,27 @@ def main():
                                                 stream=st))
         out.append({"kernel": "attention_bwd", "T": T, "ms": ms, "tflops": 2.5 * fl / ms / 1e9})
     if args.kernel in ("all", "layernorm"):
-        x = rnd(T, H)
+        # as the server runs them: fp32 residual-stream input, bf16 LN output; backward with
+        # fp32 dy and x, dx written as bf16 and fp32
+        x = rnd(T, H, dtype=torch.float32)
         gm = rnd(H, dtype=torch.float32)
         bt = rnd(H, dtype=torch.float32)
-        y = torch.empty_like(x)
+        y = torch.empty(T, H, device=dev, dtype=torch.bfloat16)
         mean = torch.empty(T, device=dev, dtype=torch.float32)
         rstd = torch.empty(T, device=dev, dtype=torch.float32)
-        ms = timed(lambda: F.fl_k_layernorm_fwd(T, H, x, gm, bt, 1e-5, y, mean, rstd, stream=st))
-        nbytes = 2 * T * H * 2 + 8 * T
-        out.append({"kernel": "layernorm_fwd", "ms": ms, "gbs": nbytes / ms / 1e6})
-        dy = rnd(T, H)
-        dx = torch.empty_like(x)
+        ms = timed(lambda: F.fl_k_layernorm_fwd(T, H, x, gm, bt, 1e-5, y, mean, rstd, x_dtype=F.FL_DT_F32, stream=st))
+        nbytes = T * H * (4 + 2) + 8 * T
+        out.append({"kernel": "layernorm_fwd", "ms": ms, "gbs": nbytes / ms / 1e6, "bytes": nbytes})
+        dy = rnd(T, H, dtype=torch.float32)
+        dxb = torch.empty(T, H, device=dev, dtype=torch.bfloat16)
+        dxf = torch.empty(T, H, device=dev, dtype=torch.float32)
         ws = torch.empty(F.fl_k_layernorm_bwd_workspace(T, H) // 4 + 64, device=dev, dtype=torch.float32)
         dg = torch.zeros(H, device=dev, dtype=torch.float32)
         db = torch.zeros(H, device=dev, dtype=torch.float32)
-        ms = timed(lambda: F.fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gm, None, 0.0, dx, dg, db, ws, stream=st))
-        nbytes = 3 * T * H * 2 + 8 * T
-        out.append({"kernel": "layernorm_bwd", "ms": ms, "gbs": nbytes / ms / 1e6})
+        ms = timed(lambda: F.fl_k_layernorm_bwd(T, H, dy, x, mean, rstd, gm, None, 0.0, dxb, dg, db, ws,
+                                                io_dtype=F.FL_DT_F32, dx_f32=dxf, stream=st))
+        nbytes = T * H * (4 + 4 + 2 + 4) + 8 * T
+        out.append({"kernel": "layernorm_bwd", "ms": ms, "gbs": nbytes / ms / 1e6, "bytes": nbytes})
     if args.kernel in ("all", "adamw"):
         n = syn.params_per_block(cfg) // 4 * 4
         w = rnd(n, dtype=torch.float32)

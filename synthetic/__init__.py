@@ -114,7 +114,14 @@ def normal_f64(key: int, n: int, mean: float, std: float, start: int = 0) -> np.
 
 
 def normal_f32(key: int, n: int, mean: float, std: float, start: int = 0) -> np.ndarray:
-    return normal_f64(key, n, mean, std, start).astype(np.float32)
+    """float32(normal_f64(...)), produced in chunks so that large tensors need no
+    float64 temporaries of their full size."""
+    out = np.empty(n, np.float32)
+    chunk = 1 << 22
+    for a in range(0, n, chunk):
+        b = min(n, a + chunk)
+        out[a:b] = normal_f64(key, b - a, mean, std, start + a)
+    return out
 
 
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:

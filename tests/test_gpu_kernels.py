@@ -138,39 +138,86 @@ def test_gemm_rope_epilogue(F, hd):
 
 
 @pytest.mark.parametrize("H", [256, 4096])
-def test_layernorm_fwd_bwd(F, H):
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_layernorm_fwd_bwd(F, H, dtype):
     T = 77
-    rng = np.random.default_rng(H)
-    x = rnd_bf16_f64(rng, (T, H), 2.0) + 0.0
+    rng = np.random.default_rng(H + (dtype == "f32"))
+    if dtype == "f32":
+        x = (2.0 * rng.standard_normal((T, H))).astype(np.float32).astype(np.float64)
+        dev_io = dev_f32
+        dt = F.FL_DT_F32
+    else:
+        x = rnd_bf16_f64(rng, (T, H), 2.0)
+        dev_io = dev_bf16
+        dt = F.FL_DT_BF16
     g = (1 + 0.2 * rng.standard_normal(H)).astype(np.float32)
     be = (0.2 * rng.standard_normal(H)).astype(np.float32)
-    dx_, dg_, db_ = dev_bf16(x), dev_f32(g), dev_f32(be)
+    dx_, dg_, db_ = dev_io(x), dev_f32(g), dev_f32(be)
     y = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
     mean = torch.empty(T, dtype=torch.float32, device="cuda")
     rstd = torch.empty(T, dtype=torch.float32, device="cuda")
-    F.fl_k_layernorm_fwd(T, H, dx_, dg_, db_, 1e-5, y, mean, rstd)
+    F.fl_k_layernorm_fwd(T, H, dx_, dg_, db_, 1e-5, y, mean, rstd, x_dtype=dt)
     torch.cuda.synchronize()
     yr, mur, rsr = O.layer_norm_fwd(x, g.astype(np.float64), be.astype(np.float64), 1e-5)
     assert rel_inf(f64(y), yr) < 1e-2
     np.testing.assert_allclose(f64(mean), mur, rtol=0, atol=1e-5)
     np.testing.assert_allclose(f64(rstd), rsr, rtol=1e-4)
-    # backward, with and without the alpha-scaled residual gradient
-    dy = rnd_bf16_f64(rng, (T, H))
-    res = rnd_bf16_f64(rng, (T, H))
+    # backward, with and without the alpha-scaled residual gradient; bf16 and fp32 dx
+    if dtype == "f32":
+        dy = rng.standard_normal((T, H)).astype(np.float32).astype(np.float64)
+        res = rng.standard_normal((T, H)).astype(np.float32).astype(np.float64)
+    else:
+        dy = rnd_bf16_f64(rng, (T, H))
+        res = rnd_bf16_f64(rng, (T, H))
     ws = torch.empty(F.fl_k_layernorm_bwd_workspace(T, H) // 4 + 64, dtype=torch.float32, device="cuda")
     for use_res in (False, True):
         dxo = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+        dxf = torch.empty((T, H), dtype=torch.float32, device="cuda")
         dgam = dev_f32(np.full(H, 0.5, np.float32))
         dbet = dev_f32(np.full(H, -0.25, np.float32))
-        F.fl_k_layernorm_bwd(T, H, dev_bf16(dy), dx_, mean, rstd, dg_, dev_bf16(res) if use_res else None, 3.0,
-                             dxo, dgam, dbet, ws)
+        F.fl_k_layernorm_bwd(T, H, dev_io(dy), dx_, mean, rstd, dg_, dev_io(res) if use_res else None, 3.0,
+                             dxo, dgam, dbet, ws, io_dtype=dt, dx_f32=dxf)
         torch.cuda.synchronize()
         dxr, dgr, dbr = O.layer_norm_bwd(dy, x, mur, rsr, g.astype(np.float64))
         if use_res:
             dxr = dxr + 3.0 * res
         assert rel_inf(f64(dxo), dxr) < 1e-2
+        assert rel_inf(f64(dxf), dxr) < 1e-4
         assert rel_inf(f64(dgam) - 0.5, dgr) < 1e-4
         assert rel_inf(f64(dbet) + 0.25, dbr) < 1e-4
+
+
+def test_gemm_fp32_residual_epilogues(F):
+    """fp32 residual stream: D fp32 = acc + bias + alpha * R, with R an fp32 tensor or its
+    LayerNorm recomputed in fp32 from the row statistics."""
+    M, N, K = 200, 512, 256
+    rng = np.random.default_rng(12)
+    A = rnd_bf16_f64(rng, (M, K))
+    B = rnd_bf16_f64(rng, (N, K), 0.1)
+    bias = rng.standard_normal(N).astype(np.float32)
+    X = (3.0 * rng.standard_normal((M, N)) + 0.5).astype(np.float32)
+    g = (1 + 0.2 * rng.standard_normal(N)).astype(np.float32)
+    be = (0.2 * rng.standard_normal(N)).astype(np.float32)
+    _, mu, rs = O.layer_norm_fwd(X.astype(np.float64), g.astype(np.float64), be.astype(np.float64), 1e-5)
+    dA, lda = _store(A, False)
+    dB, ldb = _store(B, False)
+    acc = A @ B.T
+    D = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    dX = dev_f32(X)
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_RESID, bias=dev_f32(bias), aux=dX, ld_aux=N,
+           alpha=7.5, aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32)
+    torch.cuda.synchronize()
+    assert rel_inf(f64(D), acc + bias[None, :] + 7.5 * X) < 1e-5
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_RESID, bias=dev_f32(bias), aux=dX, ld_aux=N,
+           alpha=7.5, aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32, ln_mean=dev_f32(mu), ln_rstd=dev_f32(rs),
+           ln_gamma=dev_f32(g), ln_beta=dev_f32(be))
+    torch.cuda.synchronize()
+    lnx = (X - mu[:, None]) * rs[:, None] * g[None, :] + be[None, :]
+    assert rel_inf(f64(D), acc + bias[None, :] + 7.5 * lnx) < 1e-5
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_RESID, aux=dX, ld_aux=N, alpha=-2.0,
+           aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32)
+    torch.cuda.synchronize()
+    assert rel_inf(f64(D), acc - 2.0 * X) < 1e-5
 
 
 @pytest.mark.parametrize("hd", [64, 128])

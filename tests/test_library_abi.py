@@ -64,5 +64,5 @@ def test_kernel_entry_points_validate_before_launch(F):
     L = F.lib()
     a = F.fl_gemm_args()
     assert L.fl_k_gemm(ctypes.byref(a), None, None) == -1          # null operands
-    assert L.fl_k_layernorm_fwd(4, 300, None, None, None, 1e-5, None, None, None, None) == -7
+    assert L.fl_k_layernorm_fwd(4, 300, None, 0, None, None, 1e-5, None, None, None, None) == -7
     assert L.fl_k_adamw(6, None, None, None, None, None, 1e-3, .9, .999, 1e-8, 0, .1, .001, None) == -1

@@ -46,7 +46,7 @@ def test_noalloc_layernorm_bwd_matches_workspace_variant():
         dgam_ref = torch.zeros(H, dtype=torch.float32, device="cuda")
         dbet_ref = torch.zeros(H, dtype=torch.float32, device="cuda")
         F.fl_k_layernorm_bwd(T, H, ddy, dx_, mean, rstd, dg_, dres if use_res else None, 2.5, dx_ref, dgam_ref,
-                             dbet_ref, ws)
+                             dbet_ref, ws, io_dtype=F.FL_DT_BF16)
         # the allocation-free entry point, called through the C ABI
         dx_na = torch.full((T, H), float("nan"), dtype=torch.bfloat16, device="cuda")
         dgam_na = torch.zeros(H, dtype=torch.float32, device="cuda")
