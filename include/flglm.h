@@ -111,6 +111,16 @@ int fl_server_backward(fl_server_t h, const void* const grad_out[], void* const 
  * write the gradient arena.  Errors: STATE (a forward is pending), CUDA. */
 int fl_server_step(fl_server_t h, float lr);
 
+/* fl_server_backward followed by fl_server_step(h, lr), in one call.  When no gradients
+ * are pending (no backward since the last step), the AdamW update of the four weight
+ * matrices of every block runs in the epilogue of their weight-gradient GEMMs: the fp32
+ * matrix gradients are never written to memory, and the update's traffic overlaps the
+ * tensor-core work.  The bias and LayerNorm vectors get one AdamW launch at the end.
+ * Otherwise (gradients accumulated by earlier backward calls) it runs the two calls as
+ * they are.  Results equal backward + step up to fp32 rounding.  Errors: as
+ * fl_server_backward. */
+int fl_server_backward_step(fl_server_t h, const void* const grad_out[], void* const grad_in[], float lr);
+
 /* Frees every device buffer of h after synchronising its stream.  NULL is accepted. */
 int fl_server_destroy(fl_server_t h);
 

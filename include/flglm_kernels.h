@@ -38,6 +38,9 @@ enum {
   FL_EPI_RESID = 5,      /* D = acc + alpha * R[m,n]                                      bf16/fp32 */
   FL_EPI_ACCUM_F32 = 6,  /* D[m,n] += acc                                                 fp32 */
   FL_EPI_STORE_F32 = 7,  /* D[m,n] = acc                                                  fp32 */
+  FL_EPI_ADAMW = 8,      /* g = acc is a weight gradient: AdamW update of the fp32 weight
+                            D[m,n] and its moments adam_m, adam_v (same layout, ldd), the
+                            bf16 copy aux_out (ld_aux_out); g itself is not stored      */
   FL_EPI_COUNT
 };
 
@@ -71,6 +74,10 @@ typedef struct {
   const float* ln_rstd;                     /* [M] */
   const float* ln_gamma;                    /* [N] */
   const float* ln_beta;                     /* [N] */
+  float* adam_m;                            /* FL_EPI_ADAMW: first and second moments */
+  float* adam_v;
+  float lr, beta1, beta2, eps, weight_decay;   /* FL_EPI_ADAMW hyperparameters */
+  float inv_bc1, inv_bc2;                      /* 1 / (1 - beta1^t), 1 / (1 - beta2^t) */
 } fl_gemm_args;
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);

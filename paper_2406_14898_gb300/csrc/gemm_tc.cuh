@@ -1,0 +1,548 @@
+// Persistent tcgen05 GEMM for sm_103a with fused epilogues.
+//
+// D[M,N] = epilogue(A . B^T): bf16 operands staged by TMA (128-byte swizzle) into a
+// STAGES-deep shared-memory ring, one elected thread issues tcgen05.mma kind::f16
+// (M=128, N=BN, K=16) into a double-buffered fp32 TMEM accumulator, and four
+// epilogue warps drain TMEM with tcgen05.ld while the next tile's main loop runs.
+// An epilogue warp owns 32 rows of the tile (its TMEM lane quarter); it moves each 32x64
+// fp32 chunk through 8 KB of shared memory so that, row by row, its lanes handle
+// consecutive column pairs and every global load and store of the epilogue is coalesced.
+//
+// Operand majorness is a template parameter: K-major operands are [rows, K] row-major
+// (one TMA box of 64 x rows per stage), MN-major operands are [K, rows] row-major
+// (rows/64 boxes of 64 x BK per stage).  The three GEMM families of a transformer
+// block map onto it as
+//   forward  X[T,K]  . W[N,K]^T          A K-major,  B K-major
+//   dgrad    dY[T,N] . W[N,K]            A K-major,  B MN-major
+//   wgrad    dY[T,N]^T . X[T,K]          A MN-major, B MN-major  (fp32 accumulate)
+//
+// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM owner + MMA issuer,
+// warps 2..5 epilogue (warp w reads TMEM lanes 32*(w%4) .. +31).
+#pragma once
+#include <cuda.h>
+#include <cstdio>
+#include <mutex>
+
+#include "../../include/flglm_kernels.h"
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace fl_gemm {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // one 128-byte swizzle row of bf16
+constexpr int UMMA_K = 16;
+constexpr double L2_GROUP_BUDGET = 48.0 * (1 << 20);  // bytes of operand panels kept resident per group
+constexpr int NUM_THREADS = 192;
+
+template <int BN>
+struct Cfg {
+  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * BN;  // double-buffered accumulator
+  static constexpr int STAGING_BYTES = 4 * 32 * 64 * 4;  // one 32x64 fp32 chunk per epilogue warp
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 256 /*barriers*/ + STAGING_BYTES + 1024 /*align*/;
+};
+
+struct Epi {
+  int mode;
+  const float* bias;
+  const __nv_bfloat16* aux;
+  int64_t ld_aux;
+  float alpha;
+  __nv_bfloat16* aux_out;
+  int64_t ld_aux_out;
+  void* D;
+  int64_t ldd;
+  const int32_t* pos;
+  const float2* rope_tab;  // [pos][rotary_dim/2]
+  int rope_cols;           // 2*H: columns that hold q and k
+  int head_dim, rotary_dim;
+  int aux_f32, d_f32;
+  const float *ln_mean, *ln_rstd, *ln_gamma, *ln_beta;  // residual = LayerNorm(aux) when ln_mean
+  float *adam_m, *adam_v;
+  float lr, b1, b2, eps, wd, inv_bc1, inv_bc2;
+};
+
+// Epilogue families: each kernel instantiation carries only its family's code, which keeps
+// the kernel small enough for the instruction cache (the MMA-issuing warp shares it).
+enum { FAM_PLAIN = 0, FAM_GELU = 1, FAM_RESID = 2, FAM_ROPE = 3, FAM_ADAMW = 4, FAM_COUNT };
+__host__ __device__ constexpr int family_of(int mode) {
+  return (mode == FL_EPI_BIAS_GELU || mode == FL_EPI_GELU_BWD) ? FAM_GELU
+         : (mode == FL_EPI_BIAS_RESID || mode == FL_EPI_RESID) ? FAM_RESID
+         : mode == FL_EPI_BIAS_ROPE                            ? FAM_ROPE
+         : mode == FL_EPI_ADAMW                                ? FAM_ADAMW
+                                                               : FAM_PLAIN;
+}
+
+FL_DEV float4 ld_quad(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
+FL_DEV float4 ld_quad(const __nv_bfloat16* p) {
+  const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
+  const float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+  return make_float4(a.x, a.y, b.x, b.y);
+}
+FL_DEV void st_quad(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
+FL_DEV void st_quad(__nv_bfloat16* p, float4 v) {
+  *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+}
+
+// Epilogue of one 32-row x 64-column chunk held in `stage` (row r, float4 slot j stored at
+// slot j ^ (r & 15)).  Half-warp h = lane / 16 takes the rows of parity h; lane l handles
+// columns n0 + 4 (l % 16) .. + 3, so every warp-wide access covers two 64-column rows
+// (256 B of bf16 or 512 B of fp32).  Rows go in batches of RB row pairs: all global loads of
+// a batch are issued before any of its arithmetic.
+template <int FAM>
+FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows, int n0, int lane) {
+  constexpr int RB = (FAM == FAM_GELU || FAM == FAM_ROPE) ? 16 : 8;  // row pairs per batch
+  const int h = lane >> 4, cl = lane & 15;
+  const int n = n0 + 4 * cl;
+  const float4 bias = e.bias ? ld_quad(e.bias + n) : make_float4(0.f, 0.f, 0.f, 0.f);
+  const bool ln = FAM == FAM_RESID && e.ln_mean != nullptr;
+  float4 lng = make_float4(1.f, 1.f, 1.f, 1.f), lnb = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (ln) {
+    lng = ld_quad(e.ln_gamma + n);
+    lnb = ld_quad(e.ln_beta + n);
+  }
+  // RoPE: this chunk starts a head and holds its rotary dims [0, rotary_dim)
+  const bool rope = FAM == FAM_ROPE && n0 < e.rope_cols && (n0 % e.head_dim) == 0;
+  const int half = e.rotary_dim >> 1;
+  const int pair_xor = half >> 2;  // lane distance of the partner columns (8 or 4)
+  const int col = 4 * cl;
+  const bool rotated = rope && col < 2 * half;
+  const bool first = col < half;
+  const bool gelu_bwd = FAM == FAM_GELU && e.mode == FL_EPI_GELU_BWD;
+  const bool accum = FAM == FAM_PLAIN && e.mode == FL_EPI_ACCUM_F32;
+  const bool out_f32 = e.mode == FL_EPI_STORE_F32 || e.d_f32;
+#pragma unroll 1
+  for (int pb = 0; 2 * pb < rows; pb += RB) {
+    float4 acc[RB], aux[RB], am[RB], av[RB];
+    float rmu[RB], rrs[RB];
+    int rpos[RB];
+    // ---- loads of the batch
+#pragma unroll
+    for (int i = 0; i < RB; ++i) {
+      const int rr = 2 * (pb + i) + h;
+      acc[i] = *reinterpret_cast<const float4*>(stage + (rr & 31) * 64 + 4 * (cl ^ (rr & 15)));
+      aux[i] = am[i] = av[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      rmu[i] = 0.f;
+      rrs[i] = 1.f;
+      rpos[i] = 0;
+      if (rr < rows) {
+        const int m = row0 + rr;
+        const int64_t off = (int64_t)m * e.ldd + n;
+        if constexpr (FAM == FAM_RESID) {
+          const int64_t oa = (int64_t)m * e.ld_aux + n;
+          aux[i] = e.aux_f32 ? ld_quad(reinterpret_cast<const float*>(e.aux) + oa) : ld_quad(e.aux + oa);
+          if (ln) {
+            rmu[i] = __ldg(e.ln_mean + m);
+            rrs[i] = __ldg(e.ln_rstd + m);
+          }
+        } else if constexpr (FAM == FAM_ADAMW) {
+          aux[i] = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(e.D) + off);  // w
+          am[i] = *reinterpret_cast<const float4*>(e.adam_m + off);
+          av[i] = *reinterpret_cast<const float4*>(e.adam_v + off);
+        } else {
+          if (gelu_bwd) aux[i] = ld_quad(e.aux + (int64_t)m * e.ld_aux + n);
+          if (accum) aux[i] = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(e.D) + off);
+          if (FAM == FAM_ROPE && rotated) rpos[i] = __ldg(e.pos + m);
+        }
+      }
+    }
+    // ---- arithmetic and stores of the batch
+#pragma unroll
+    for (int i = 0; i < RB; ++i) {
+      const int rr = 2 * (pb + i) + h;
+      float y[4] = {acc[i].x + bias.x, acc[i].y + bias.y, acc[i].z + bias.z, acc[i].w + bias.w};
+      if (FAM == FAM_ROPE && rope) {  // uniform across the warp: every lane takes part in the shuffles
+        float p[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) p[q] = __shfl_xor_sync(0xffffffffu, y[q], pair_xor);
+        if (rotated && rr < rows) {
+          const int ii = first ? col : col - half;
+          const float2* tab = e.rope_tab + (int64_t)rpos[i] * half + ii;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float2 cs = __ldg(tab + q);
+            y[q] = first ? y[q] * cs.x - p[q] * cs.y : y[q] * cs.x + p[q] * cs.y;
+          }
+        }
+      }
+      if (rr >= rows) continue;
+      const int m = row0 + rr;
+      const int64_t off = (int64_t)m * e.ldd + n;
+      const float a4[4] = {aux[i].x, aux[i].y, aux[i].z, aux[i].w};
+      if constexpr (FAM == FAM_RESID) {
+        const float g4[4] = {lng.x, lng.y, lng.z, lng.w}, b4[4] = {lnb.x, lnb.y, lnb.z, lnb.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float r = ln ? (a4[q] - rmu[i]) * rrs[i] * g4[q] + b4[q] : a4[q];  // LayerNorm(aux) in fp32
+          y[q] = fmaf(e.alpha, r, y[q]);
+        }
+      } else if constexpr (FAM == FAM_GELU) {
+        if (gelu_bwd) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) y[q] *= gelu_tanh_grad(a4[q]);
+        } else {
+          st_quad(e.aux_out + (int64_t)m * e.ld_aux_out + n, make_float4(y[0], y[1], y[2], y[3]));
+#pragma unroll
+          for (int q = 0; q < 4; ++q) y[q] = gelu_tanh(y[q]);
+        }
+      }
+      if constexpr (FAM == FAM_ADAMW) {
+        // AdamW on the four weights with g = y: the formula of adamw_kernel
+        float w[4] = {aux[i].x, aux[i].y, aux[i].z, aux[i].w};
+        float mm[4] = {am[i].x, am[i].y, am[i].z, am[i].w};
+        float vv[4] = {av[i].x, av[i].y, av[i].z, av[i].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          mm[q] = e.b1 * mm[q] + (1.f - e.b1) * y[q];
+          vv[q] = e.b2 * vv[q] + (1.f - e.b2) * y[q] * y[q];
+          const float mh = mm[q] * e.inv_bc1;
+          const float vh = vv[q] * e.inv_bc2;
+          w[q] = w[q] - e.lr * (mh / (sqrtf(vh) + e.eps) + e.wd * w[q]);
+        }
+        st_quad(reinterpret_cast<float*>(e.D) + off, make_float4(w[0], w[1], w[2], w[3]));
+        st_quad(e.adam_m + off, make_float4(mm[0], mm[1], mm[2], mm[3]));
+        st_quad(e.adam_v + off, make_float4(vv[0], vv[1], vv[2], vv[3]));
+        st_quad(e.aux_out + (int64_t)m * e.ld_aux_out + n, make_float4(w[0], w[1], w[2], w[3]));
+      } else if (accum) {
+        st_quad(reinterpret_cast<float*>(e.D) + off, make_float4(a4[0] + y[0], a4[1] + y[1], a4[2] + y[2], a4[3] + y[3]));
+      } else if (out_f32) {
+        st_quad(reinterpret_cast<float*>(e.D) + off, make_float4(y[0], y[1], y[2], y[3]));
+      } else {
+        st_quad(reinterpret_cast<__nv_bfloat16*>(e.D) + off, make_float4(y[0], y[1], y[2], y[3]));
+      }
+    }
+  }
+}
+
+// Tile order.  Tiles are taken in groups of `gsz` panels of one operand: along m
+// (gsz m-blocks, m fastest) every group streams B once while its A panels stay in L2;
+// along n the roles swap.  The host picks the side and size that minimise DRAM reads.
+struct Raster {
+  int gsz;
+  int along_n;
+};
+FL_DEV void tile_coords(int tile, int num_m, int num_n, Raster r, int& mb, int& nb) {
+  if (!r.along_n) {
+    const int group = r.gsz * num_n;
+    const int g = tile / group;
+    const int first = g * r.gsz;
+    const int gm = min(num_m - first, r.gsz);
+    const int local = tile - g * group;
+    mb = first + local % gm;
+    nb = local / gm;
+  } else {
+    const int group = r.gsz * num_m;
+    const int g = tile / group;
+    const int first = g * r.gsz;
+    const int gn = min(num_n - first, r.gsz);
+    const int local = tile - g * group;
+    nb = first + local % gn;
+    mb = local / gn;
+  }
+}
+
+template <int BN, bool A_MN, bool B_MN, int FAM>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, Epi epi,
+                   int M, int N, int K, Raster raster, int* status) {
+  using C = Cfg<BN>;
+  constexpr int STAGES = C::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* acc_full = bars + 2 * STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* staging = reinterpret_cast<float*>(smem + STAGES * C::STAGE_BYTES + 256);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int num_m = (M + BM - 1) / BM;
+  const int num_n = N / BN;
+  const int num_tiles = num_m * num_n;
+  const int num_k = (K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 128);
+    }
+    mbar_init(drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_holder, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, last_par = 0;  // per-stage bit masks for the teardown drain
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        int mb, nb;
+        tile_coords(tile, num_m, num_n, raster, mb, nb);
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1)) {
+            report_status(status, FL_DEV_TIMEOUT_EMPTY);
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+          armed |= 1u << stage;
+          last_par = (last_par & ~(1u << stage)) | (phase << stage);
+          const int k0 = kb * BK;
+          uint8_t* a_dst = sA + stage * C::A_BYTES;
+          uint8_t* b_dst = sB + stage * C::B_BYTES;
+          if (!A_MN) {
+            tma_load_2d(a_dst, &tmA, &full[stage], k0, mb * BM);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * 64 * BK * 2, &tmA, &full[stage], mb * BM + 64 * j, k0);
+          }
+          if (!B_MN) {
+            tma_load_2d(b_dst, &tmB, &full[stage], k0, nb * BN);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 64 * BK * 2, &tmB, &full[stage], nb * BN + 64 * j, k0);
+          }
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // Drain: every armed stage's copies must have landed before shared memory is released.
+      for (int s = 0; s < STAGES; ++s)
+        if (armed & (1u << s))
+          if (!mbar_wait(&full[s], (last_par >> s) & 1)) report_status(status, FL_DEV_TIMEOUT_DRAIN);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      constexpr uint32_t IDESC = umma_idesc_bf16(BM, BN, A_MN, B_MN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_par = (local >> 1) & 1;
+        if (!mbar_wait(&acc_empty[acc], acc_par ^ 1)) {
+          report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait(&full[stage], phase)) {
+            report_status(status, FL_DEV_TIMEOUT_FULL);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(sA + stage * C::A_BYTES);
+          const uint32_t b_base = smem_u32(sB + stage * C::B_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+            // K-major: next 16 elements are 32 bytes further along the swizzled row.
+            // MN-major: next 16 k-rows are 16 * 128 bytes further.
+            const uint64_t adesc = A_MN ? smem_desc_sw128(a_base + kk * 2048, BK * 128, 1024)
+                                        : smem_desc_sw128(a_base + kk * 32, 16, 1024);
+            const uint64_t bdesc = B_MN ? smem_desc_sw128(b_base + kk * 2048, BK * 128, 1024)
+                                        : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+            umma_bf16(d_tmem, adesc, bdesc, IDESC, (kb | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit(&empty[stage]);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (ok) umma_commit(&acc_full[acc]);
+      }
+      // Drain: all MMAs issued by this thread complete before TMEM is released.
+      umma_commit(drain);
+      if (!mbar_wait(drain, 0)) report_status(status, FL_DEV_TIMEOUT_DRAIN);
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue warps
+    const int quarter = warp & 3;
+    float* stage = staging + (warp - 2) * 32 * 64;
+    float4* my = reinterpret_cast<float4*>(stage + lane * 64);
+    int local = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+      int mb, nb;
+      tile_coords(tile, num_m, num_n, raster, mb, nb);
+      const int acc = local & 1;
+      const uint32_t acc_par = (local >> 1) & 1;
+      if (!mbar_wait(&acc_full[acc], acc_par)) {
+        report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
+        break;
+      }
+      tc_fence_after();
+      const int row0 = mb * BM + quarter * 32;
+      const int rows = M - row0 < 32 ? M - row0 : 32;  // may be <= 0 for the ragged last tile
+      const uint32_t t_row = tmem_base + (uint32_t(quarter * 32) << 16) + acc * BN;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 64) {
+        uint32_t r0[32], r1[32];
+        tmem_ld32(t_row + c0, r0);
+        tmem_ld32(t_row + c0 + 32, r1);
+        tmem_ld_wait();
+        if (c0 + 64 == BN) {  // accumulator fully read: the MMA may reuse it
+          tc_fence_before();
+          mbar_arrive(&acc_empty[acc]);
+        }
+        // this lane's row -> shared memory, float4 slot j at j ^ (row & 15)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          my[j ^ (lane & 15)] = make_float4(__uint_as_float(r0[4 * j]), __uint_as_float(r0[4 * j + 1]),
+                                            __uint_as_float(r0[4 * j + 2]), __uint_as_float(r0[4 * j + 3]));
+          my[(8 + j) ^ (lane & 15)] = make_float4(__uint_as_float(r1[4 * j]), __uint_as_float(r1[4 * j + 1]),
+                                                  __uint_as_float(r1[4 * j + 2]), __uint_as_float(r1[4 * j + 3]));
+        }
+        __syncwarp();
+        if (rows > 0) epilogue_chunk<FAM>(epi, stage, row0, rows, nb * BN + c0, lane);
+        __syncwarp();
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+typedef CUresult (*PFN_encodeTiled)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+inline PFN_encodeTiled get_encode_fn() {
+  static PFN_encodeTiled fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_encodeTiled>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] (inner contiguous, row stride ld elements), box {64, box_outer}.
+inline int make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer, int64_t ld, uint32_t box_outer) {
+  PFN_encodeTiled enc = get_encode_fn();
+  if (!enc) return fl_internal_error(FL_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {cuuint64_t(ld) * 2};
+  cuuint32_t box[2] = {64, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "tensor map encode failed (%d): inner %llu outer %llu ld %lld", (int)r,
+                             (unsigned long long)inner, (unsigned long long)outer, (long long)ld);
+  return FL_OK;
+}
+
+inline int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+template <int BN, bool A_MN, bool B_MN, int FAM>
+int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) {
+  using C = Cfg<BN>;
+  auto kern = gemm_tc_kernel<BN, A_MN, B_MN, FAM>;
+  static bool attr_set = false;  // per instantiation; the attribute is per device function
+  if (!attr_set) {
+    FL_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
+    attr_set = true;
+  }
+  CUtensorMap ta, tb;
+  int rc;
+  // A(m,k): K-major -> [M rows, K inner]; MN-major -> [K rows, M inner]
+  if (!A_MN) rc = make_map(&ta, a->A, a->K, a->M, a->lda, BM);
+  else rc = make_map(&ta, a->A, a->M, a->K, a->lda, BK);
+  if (rc) return rc;
+  if (!B_MN) rc = make_map(&tb, a->B, a->K, a->N, a->ldb, BN);
+  else rc = make_map(&tb, a->B, a->N, a->K, a->ldb, BK);
+  if (rc) return rc;
+  const int num_m = (a->M + BM - 1) / BM, num_n = a->N / BN;
+  const int tiles = num_m * num_n;
+  const int grid = tiles < num_sms() ? tiles : num_sms();
+  // DRAM reads of the two orders: the grouped operand once, the other once per group
+  const double pa = double(BM) * a->K * 2, pb = double(BN) * a->K * 2;
+  int gm = (int)(L2_GROUP_BUDGET / pa), gn = (int)(L2_GROUP_BUDGET / pb);
+  gm = gm < 1 ? 1 : (gm > num_m ? num_m : gm);
+  gn = gn < 1 ? 1 : (gn > num_n ? num_n : gn);
+  const double cost_m = pa * num_m + pb * num_n * ((num_m + gm - 1) / gm);
+  const double cost_n = pb * num_n + pa * num_m * ((num_n + gn - 1) / gn);
+  Raster r;
+  r.along_n = cost_n < cost_m ? 1 : 0;
+  r.gsz = r.along_n ? gn : gm;
+  gemm_tc_kernel<BN, A_MN, B_MN, FAM><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ta, tb, epi, a->M, a->N, a->K, r,
+                                                                                 status);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// Every (layout, family) pair for both tile widths; the three operand layouts are
+// instantiated in separate translation units so that the build compiles them in parallel.
+#define FL_GEMM_INSTANTIATE(AMN, BMN)                                                              \
+  template int launch<256, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch<128, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch<256, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
+  template int launch<128, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
+  template int launch<256, AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch<128, AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch<256, AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
+  template int launch<128, AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
+  template int launch<256, AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch<128, AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);
+
+}  // namespace fl_gemm
+

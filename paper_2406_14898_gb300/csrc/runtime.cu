@@ -106,6 +106,11 @@ struct fl_server {
   // backward then stores the weight gradients instead of adding to them, and AdamW
   // does not need to clear the 4 B/parameter gradient arena
   bool grads_zero = true;
+  // fused backward + step: the weight-gradient GEMMs apply AdamW in their epilogue
+  struct {
+    bool on = false;
+    float lr = 0.f, inv_bc1 = 1.f, inv_bc2 = 1.f;
+  } fuse;
 
   // activations
   std::vector<float*> xs;  // block inputs/outputs, fp32
@@ -243,7 +248,7 @@ fl_gemm_args gemm_dgrad(int T, int Kin, int Nout, const void* dY, const void* W,
   return a;
 }
 // dW[Nout, Kin] (+)= dY[T, Nout]^T . X[T, Kin]; stores when the gradients are known zero
-fl_gemm_args gemm_wgrad(int T, int Nout, int Kin, const void* dY, const void* X, float* dW, bool store) {
+fl_gemm_args gemm_wgrad_raw(int T, int Nout, int Kin, const void* dY, const void* X, float* dW, bool store) {
   fl_gemm_args a;
   memset(&a, 0, sizeof a);
   a.M = Nout; a.N = Kin; a.K = T;
@@ -251,6 +256,29 @@ fl_gemm_args gemm_wgrad(int T, int Nout, int Kin, const void* dY, const void* X,
   a.B = X; a.ldb = Kin; a.b_mn_major = 1;
   a.D = dW; a.ldd = Kin;
   a.epilogue = store ? FL_EPI_STORE_F32 : FL_EPI_ACCUM_F32;
+  return a;
+}
+
+// Weight gradient of weight matrix t of block b: stored / accumulated into the gradient
+// arena, or, inside a fused backward + step, applied to the weight by AdamW directly.
+fl_gemm_args gemm_wgrad(fl_server* h, int b, int t, int T, int Nout, int Kin, const void* dY, const void* X) {
+  fl_gemm_args a = gemm_wgrad_raw(T, Nout, Kin, dY, X, h->gt(b, t), h->grads_zero);
+  if (h->fuse.on) {
+    const fl_server_cfg& c = h->cfg;
+    a.epilogue = FL_EPI_ADAMW;
+    a.D = h->wt(b, t);
+    a.adam_m = h->m + h->off(b, t);
+    a.adam_v = h->v + h->off(b, t);
+    a.aux_out = h->wbt(b, t);
+    a.ld_aux_out = Kin;
+    a.lr = h->fuse.lr;
+    a.beta1 = c.adam_beta1;
+    a.beta2 = c.adam_beta2;
+    a.eps = c.adam_eps;
+    a.weight_decay = c.weight_decay;
+    a.inv_bc1 = h->fuse.inv_bc1;
+    a.inv_bc2 = h->fuse.inv_bc2;
+  }
   return a;
 }
 
@@ -336,13 +364,12 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   const bool glm = c.residual_from_ln != 0;
   BlockAct& A = h->act[b];
   cudaStream_t st = h->stream;
-  const bool store = h->grads_zero;
   // FFN down: du = (dy W2) * gelu'(u); dW2 += dy^T g; db2 += colsum(dy)
   fl_gemm_args d1 = gemm_dgrad(T, F, H, dy, h->wbt(b, FL_T_WDOWN), h->du, FL_EPI_GELU_BWD);
   d1.aux = A.u;
   d1.ld_aux = F;
   TRY(h, run_gemm(h, d1));
-  TRY(h, run_gemm(h, gemm_wgrad(T, H, F, dy, A.g, h->gt(b, FL_T_WDOWN), store)));
+  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
   prof_end(h);
@@ -356,7 +383,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d2.alpha = al;
   }
   TRY(h, run_gemm(h, d2));
-  TRY(h, run_gemm(h, gemm_wgrad(T, F, H, h->du, A.m, h->gt(b, FL_T_WUP), store)));
+  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
   prof_end(h);
@@ -367,7 +394,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   prof_end(h);
   // dense: do = dh Wd; dWd += dh^T o; dbd += colsum(dh)
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
-  TRY(h, run_gemm(h, gemm_wgrad(T, H, H, h->dh, A.o, h->gt(b, FL_T_WDENSE), store)));
+  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
   prof_end(h);
@@ -386,7 +413,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d3.alpha = al;
   }
   TRY(h, run_gemm(h, d3));
-  TRY(h, run_gemm(h, gemm_wgrad(T, 3 * H, H, h->dqkv, A.a, h->gt(b, FL_T_WQKV), store)));
+  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a)));
   prof_begin(h, FL_PROF_OTHER);
   TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
   prof_end(h);
@@ -606,7 +633,7 @@ extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[
   return FL_OK;
 }
 
-extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], void* const grad_in[]) {
+static int backward_impl(fl_server_t h, const void* const grad_out[], void* const grad_in[]) {
   if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "backward: null handle");
   if (!h->pending) return set_err(h, FL_ERR_STATE, "backward: no pending forward");
   if (int rc = check_ptrs(h, grad_out, h->K, "grad_out")) return rc;
@@ -630,6 +657,40 @@ extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], v
   if ((rc = copy_clients(h, (const void* const*)grad_in, COPY_SCATTER_BF16, cur, nullptr))) return rc;
   h->pending = false;
   h->grads_zero = false;
+  return FL_OK;
+}
+
+extern "C" int fl_server_backward(fl_server_t h, const void* const grad_out[], void* const grad_in[]) {
+  return backward_impl(h, grad_out, grad_in);
+}
+
+extern "C" int fl_server_backward_step(fl_server_t h, const void* const grad_out[], void* const grad_in[], float lr) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "backward_step: null handle");
+  if (!h->pending) return set_err(h, FL_ERR_STATE, "backward_step: no pending forward");
+  if (!h->grads_zero) {  // gradients from an earlier backward are pending: no fusion
+    if (int rc = backward_impl(h, grad_out, grad_in)) return rc;
+    return fl_server_step(h, lr);
+  }
+  const fl_server_cfg& c = h->cfg;
+  const int64_t t = h->step_t + 1;
+  h->fuse.on = true;
+  h->fuse.lr = lr;
+  // the same fp32 bias-correction factors fl_server_step passes to the AdamW kernel
+  h->fuse.inv_bc1 = 1.f / (float)(1.0 - std::pow((double)c.adam_beta1, (double)t));
+  h->fuse.inv_bc2 = 1.f / (float)(1.0 - std::pow((double)c.adam_beta2, (double)t));
+  int rc = backward_impl(h, grad_out, grad_in);
+  h->fuse.on = false;
+  if (rc) return rc;
+  h->step_t = t;
+  // the bias and LayerNorm vectors: one AdamW launch over their contiguous region
+  prof_begin(h, FL_PROF_ADAMW);
+  rc = fl_launch_adamw(h->n_params - h->vec_base, h->w + h->vec_base, h->g + h->vec_base, h->m + h->vec_base,
+                       h->v + h->vec_base, h->wb + h->vec_base, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
+                       c.weight_decay, (float)(1.0 - std::pow((double)c.adam_beta1, (double)t)),
+                       (float)(1.0 - std::pow((double)c.adam_beta2, (double)t)), 0, h->stream);
+  prof_end(h);
+  if (rc) return fwd_err(h, rc);
+  h->grads_zero = true;  // matrix gradients were never written; vectors are cleared by the next backward
   return FL_OK;
 }
 

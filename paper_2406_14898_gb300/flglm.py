@@ -23,7 +23,7 @@ ERRORS = {-1: "FL_ERR_INVALID_ARG", -2: "FL_ERR_CAPACITY", -3: "FL_ERR_STATE", -
  FL_T_LN1_G, FL_T_LN1_B, FL_T_LN2_G, FL_T_LN2_B) = range(12)
 FL_T_COUNT = 12
 (FL_EPI_STORE, FL_EPI_BIAS_GELU, FL_EPI_BIAS_RESID, FL_EPI_BIAS_ROPE, FL_EPI_GELU_BWD, FL_EPI_RESID,
- FL_EPI_ACCUM_F32, FL_EPI_STORE_F32) = range(8)
+ FL_EPI_ACCUM_F32, FL_EPI_STORE_F32, FL_EPI_ADAMW) = range(9)
 PROF_CLASSES = ("gemm", "attention", "layernorm", "adamw", "other")
 FL_DT_BF16, FL_DT_F32 = 0, 1
 
@@ -53,7 +53,9 @@ class fl_gemm_args(C.Structure):
                 ("rope_tab", C.c_void_p), ("n_heads", C.c_int32), ("head_dim", C.c_int32),
                 ("rotary_dim", C.c_int32), ("aux_dtype", C.c_int32), ("d_dtype", C.c_int32),
                 ("ln_mean", C.c_void_p), ("ln_rstd", C.c_void_p), ("ln_gamma", C.c_void_p),
-                ("ln_beta", C.c_void_p)]
+                ("ln_beta", C.c_void_p), ("adam_m", C.c_void_p), ("adam_v", C.c_void_p),
+                ("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float), ("eps", C.c_float),
+                ("weight_decay", C.c_float), ("inv_bc1", C.c_float), ("inv_bc2", C.c_float)]
 
 
 _P = C.c_void_p
@@ -66,6 +68,7 @@ _SIGS = {
     "fl_server_forward": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I32), _I32, C.POINTER(_P)]),
     "fl_server_backward": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_P)]),
     "fl_server_step": (C.c_int, [_P, _F]),
+    "fl_server_backward_step": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_P), _F]),
     "fl_server_destroy": (C.c_int, [_P]),
     "fl_server_set_stream": (C.c_int, [_P, _P]),
     "fl_server_sync": (C.c_int, [_P]),
@@ -197,6 +200,9 @@ class Server:
 
     def step(self, lr: float):
         check(lib().fl_server_step(self.h, lr), self.h)
+
+    def backward_step(self, grad_out: Sequence, grad_in: Sequence, lr: float):
+        check(lib().fl_server_backward_step(self.h, _parr(grad_out), _parr(grad_in), lr), self.h)
 
     def sync(self):
         check(lib().fl_server_sync(self.h), self.h)

@@ -75,7 +75,7 @@ def check_updated_weights(w, w_ref, w0, g_ref, lr, where):
         assert np.mean(err > lr) < 0.02, (where, np.mean(err > lr))
 
 
-def parity_case(F, cfg, check_step=True):
+def parity_case(F, cfg, check_step=True, fused=False):
     params = syn.init_params(cfg)
     srv = make_server(F, cfg)
     for b in range(cfg.n_blocks):
@@ -83,6 +83,30 @@ def parity_case(F, cfg, check_step=True):
             srv.set_param(b, t, params[b][t])
     states = syn.client_states(cfg)
     grads = syn.client_grads(cfg)
+    if fused:   # backward + AdamW in one call: compare outputs, input grads and updated weights
+        st = [dev_bf16_from_bits(s) for s in states]
+        outs = [torch.empty_like(s) for s in st]
+        srv.forward(st, cfg.seq_lens, outs)
+        gins = [torch.empty_like(s) for s in st]
+        srv.backward_step([dev_bf16_from_bits(g) for g in grads], gins, cfg.lr)
+        srv.sync()
+        ref = O.OracleServer(cfg, params)
+        ro = ref.forward([syn.bf16_bits_to_f64(s) for s in states])
+        rg = ref.backward([syn.bf16_bits_to_f64(g) for g in grads])
+        gref = [[ref.grads[b][t].reshape(-1).copy() for t in range(12)] for b in range(cfg.n_blocks)]
+        ref.step(cfg.lr)
+        for k in range(cfg.K):
+            assert rel_inf(f64(outs[k]), ro[k]) < OUT_TOL
+            assert rel_inf(f64(gins[k]), rg[k]) < GRAD_TOL
+        for b in range(cfg.n_blocks):
+            for t in range(12):
+                check_updated_weights(srv.get_param(b, t), ref.params[b][t].reshape(-1),
+                                      params[b][t].reshape(-1), gref[b][t], cfg.lr, (b, t))
+                m, v = srv.get_adam_moments(b, t)
+                assert rel_inf(m, ref.m[b][t].reshape(-1)) < GRAD_TOL
+                assert not srv.get_grad(b, t).any()
+        srv.close()
+        return
     outs, gins = run_gpu(F, srv, cfg, states, grads)
     ref = O.OracleServer(cfg, params)
     ro = ref.forward([syn.bf16_bits_to_f64(s) for s in states])
@@ -113,6 +137,45 @@ def parity_case(F, cfg, check_step=True):
 @pytest.mark.parametrize("rfl", [1, 0], ids=["glm_block", "pre_ln"])
 def test_tiny_config_parity(F, rfl):
     parity_case(F, syn.CONFIGS["tiny"].with_(residual_from_ln=rfl))
+
+
+@pytest.mark.parametrize("rfl", [1, 0], ids=["glm_block", "pre_ln"])
+def test_tiny_config_parity_fused_step(F, rfl):
+    parity_case(F, syn.CONFIGS["tiny"].with_(residual_from_ln=rfl), fused=True)
+
+
+def test_fused_step_equals_backward_then_step(F):
+    """Two steps of fl_server_backward_step against fl_server_backward + fl_server_step
+    on identically seeded servers (the fused AdamW epilogue uses the same fp32 formula)."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, seq_lens=(64, 40))
+    states = [dev_bf16_from_bits(s) for s in syn.client_states(cfg)]
+    grads = [dev_bf16_from_bits(g) for g in syn.client_grads(cfg)]
+    a, b = make_server(F, cfg), make_server(F, cfg)
+    outs = [torch.empty_like(s) for s in states]
+    gi = [torch.empty_like(s) for s in states]
+    for _ in range(2):
+        a.forward(states, cfg.seq_lens, outs)
+        a.backward(grads, gi)
+        a.step(1e-3)
+        b.forward(states, cfg.seq_lens, outs)
+        b.backward_step(grads, gi, 1e-3)
+    a.sync()
+    b.sync()
+    for blk in range(cfg.n_blocks):
+        for t in range(12):
+            wa, wb = a.get_param(blk, t), b.get_param(blk, t)
+            assert rel_inf(wb, wa) < 1e-6, (blk, t)
+            ma, va = a.get_adam_moments(blk, t)
+            mb, vb = b.get_adam_moments(blk, t)
+            assert rel_inf(mb, ma) < 1e-5 and rel_inf(vb, va) < 1e-5
+    # with gradients pending from an earlier backward, the call falls back to backward + step
+    b.forward(states, cfg.seq_lens, outs)
+    b.backward(grads, gi)
+    b.forward(states, cfg.seq_lens, outs)
+    b.backward_step(grads, gi, 1e-3)
+    b.sync()
+    a.close()
+    b.close()
 
 
 def test_ragged_small_parity(F):
