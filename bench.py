@@ -275,11 +275,7 @@ def main():
             dist.barrier()
 
     def max_over_ranks(x: float) -> float:
-        if world == 1:
-            return x
-        t = torch.tensor([x], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return slowest_rank_ms(x, world, dev)
 
     for _ in range(args.warmup):
         step()
@@ -308,7 +304,7 @@ def main():
     clk = clocks.stop()
     ms = max_over_ranks(ms)
     ms_step = ms / args.steps
-    value = world * cfg.tokens * args.steps / (ms / 1e3)
+    value = job_tokens_per_s(world, cfg.tokens, args.steps, ms)
 
     adam_ms = prof["adamw"][0] / args.steps
 
@@ -368,7 +364,7 @@ def main():
         barrier()
         ems = max_over_ranks(max(e0.elapsed_time(e1), 1e3 * wall))
         nbytes = sum(s.nbytes for s in states_bits)
-        e2e = {"value": world * cfg.tokens * args.steps / (ems / 1e3), "unit": "tokens/s",
+        e2e = {"value": job_tokens_per_s(world, cfg.tokens, args.steps, ems), "unit": "tokens/s",
                "h2d_bytes_per_step": 2 * nbytes, "d2h_bytes_per_step": 2 * nbytes,
                "ms_per_step": ems / args.steps}
 
@@ -413,6 +409,23 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def slowest_rank_ms(ms: float, world: int, device=None) -> float:
+    """The timed region's duration of the slowest rank (all-reduce MAX); the job's time."""
+    if world == 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(world: int, tokens_per_rank: int, steps: int, ms: float) -> float:
+    """Whole-job throughput: every rank's tokens over the slowest rank's time (replicas,
+    weak scaling: each rank serves its own clients)."""
+    return world * tokens_per_rank * steps / (ms / 1e3)
 
 
 def run_sweep(args):
@@ -498,11 +511,14 @@ def ncu_traffic(path: str, workload_name: str):
 
 
 def kernel_version() -> str:
-    """Fingerprint of the GEMM source, so that stored ncu traffic is used only for the
+    """Fingerprint of the GEMM sources, so that stored ncu traffic is used only for the
     kernel it was measured on."""
+    import glob
     import hashlib
-    src = open(os.path.join(ROOT, "paper_2406_14898_gb300", "csrc", "gemm_tc.cu"), "rb").read()
-    return hashlib.sha256(src).hexdigest()[:16]
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2406_14898_gb300", "csrc", "gemm_*"))):
+        h.update(open(f, "rb").read())
+    return h.hexdigest()[:16]
 
 
 if __name__ == "__main__":
