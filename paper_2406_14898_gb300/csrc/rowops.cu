@@ -1,4 +1,4 @@
-// HBM-bound kernels of the server step: LayerNorm forward/backward (warp per row,
+// HBM-bound kernels of the server step: LayerNorm forward/backward (a CTA per row,
 // 128-bit loads), bias-gradient column sums, AdamW over the flat fp32 arena,
 // client pack/unpack, per-call packing metadata and the seeded parameter init.
 #include <cstdio>
@@ -58,200 +58,143 @@ FL_DEV void load8<float>(const float* base, int64_t chunk, float* f) {
   f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
 }
 
-// ------------------------------------------------------------------ LayerNorm forward
-// One warp per row; lane l owns the 8-element chunks l, l+32, l+64, ... (NV chunks).  The
-// row stays in registers (packed bf16, or fp32) across the mean, variance and output
-// passes, so HBM is read once and written once.  Output y is bf16 (a GEMM operand).
-template <int NV, typename TX>
-__global__ void __launch_bounds__(256) ln_fwd_kernel(int T, int H, const TX* __restrict__ x,
+// ------------------------------------------------------------------ LayerNorm
+// One CTA per row at a time (rows grid-strided), H/8 threads: thread c owns the 8-element
+// chunk c of every row, so a row is read from HBM exactly once and the row statistics are
+// two block reductions.  The next row of the CTA is loaded before the current row's
+// reductions to keep HBM busy across the barriers.
+
+// Sum of (a, b) over the block; `red` is a [2][32] shared buffer, `par` alternates between
+// consecutive calls so that one barrier per call suffices.
+FL_DEV float2 block_sum2(float a, float b, float2 (*red)[32], int par) {
+  a = warp_sum(a);
+  b = warp_sum(b);
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  if (lane == 0) red[par][w] = make_float2(a, b);
+  __syncthreads();
+  float2 r = make_float2(0.f, 0.f);
+  for (int i = 0; i < nw; ++i) {
+    const float2 v = red[par][i];
+    r.x += v.x;
+    r.y += v.y;
+  }
+  return r;
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(512) ln_fwd_kernel(int T, int H, const TX* __restrict__ x,
                                                      const float* __restrict__ gamma,
                                                      const float* __restrict__ beta, float eps,
                                                      __nv_bfloat16* __restrict__ y, float* __restrict__ mean,
                                                      float* __restrict__ rstd) {
-  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (row >= T) return;
-  const TX* xr = x + (int64_t)row * H;
-  constexpr bool PACKED = sizeof(TX) == 2;
-  uint4 raw[PACKED ? NV : 1];
-  float vals[PACKED ? 1 : NV * 8];
+  __shared__ float2 red[2][32];
+  const int c = threadIdx.x;
+  float gg[8], bt[8];
+  load8<float>(gamma, c, gg);
+  load8<float>(beta, c, bt);
+  int par = 0;
+  float nxt[8];
+  int row = blockIdx.x;
+  if (row < T) load8<TX>(x + (int64_t)row * H, c, nxt);
+  for (; row < T; row += gridDim.x) {
+    float v[8];
 #pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    if constexpr (PACKED) raw[i] = __ldg(reinterpret_cast<const uint4*>(xr) + lane + 32 * i);
-    else load8<float>(reinterpret_cast<const float*>(xr), lane + 32 * i, vals + 8 * i);
-  }
-  auto get = [&](int i, float* f) {
-    if constexpr (PACKED) {
-      opaque(raw[i]);
-      unpack8(raw[i], f);
-    } else {
+    for (int k = 0; k < 8; ++k) v[k] = nxt[k];
+    const int r2 = row + gridDim.x;
+    if (r2 < T) load8<TX>(x + (int64_t)r2 * H, c, nxt);
+    float s = 0.f;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) f[j] = vals[8 * i + j];
+    for (int k = 0; k < 8; ++k) s += v[k];
+    const float mu = block_sum2(s, 0.f, red, par).x / H;
+    par ^= 1;
+    float q = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) q += (v[k] - mu) * (v[k] - mu);
+    const float rs = rsqrtf(block_sum2(q, 0.f, red, par).x / H + eps);
+    par ^= 1;
+    float o[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) o[k] = (v[k] - mu) * rs * gg[k] + bt[k];
+    reinterpret_cast<uint4*>(y + (int64_t)row * H)[c] = pack8(o);
+    if (c == 0) {
+      mean[row] = mu;
+      rstd[row] = rs;
     }
-  };
-  float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    float f[8];
-    get(i, f);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) s += f[j];
-  }
-  const float mu = warp_sum(s) / H;
-  float q = 0.f;
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    float f[8];
-    get(i, f);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float d = f[j] - mu;
-      q += d * d;
-    }
-  }
-  const float rs = rsqrtf(warp_sum(q) / H + eps);
-  uint4* yr = reinterpret_cast<uint4*>(y + (int64_t)row * H);
-  const float4* g4 = reinterpret_cast<const float4*>(gamma);
-  const float4* b4 = reinterpret_cast<const float4*>(beta);
-#pragma unroll
-  for (int i = 0; i < NV; ++i) {
-    const int c = lane + 32 * i;  // chunk index: columns [8c, 8c+8)
-    const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
-    const float4 ba = __ldg(b4 + 2 * c), bb = __ldg(b4 + 2 * c + 1);
-    const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
-    const float bt[8] = {ba.x, ba.y, ba.z, ba.w, bb.x, bb.y, bb.z, bb.w};
-    float f[8], o[8];
-    get(i, f);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) o[j] = (f[j] - mu) * rs * gg[j] + bt[j];
-    yr[c] = pack8(o);
-  }
-  if (lane == 0) {
-    mean[row] = mu;
-    rstd[row] = rs;
   }
 }
 
-// ------------------------------------------------------------------ LayerNorm backward
-// A CTA takes tiles of LN_R rows.  Phase 1: one warp per row computes mean(g) and
-// mean(g xhat), g = gamma dy (lane-strided 8-element chunks).  Phase 2: thread t owns the
-// column chunks t, t+256, ... of every row of the tile; it re-reads dy and x (L2 hits),
-// writes dx (bf16 and/or fp32) and keeps its columns' dgamma/dbeta partials in registers
-// across all the CTA's tiles.  The partials go to workspace[blockIdx.x][2][H];
-// ln_bwd_reduce_kernel adds them into dgamma/dbeta.  dy, x and the optional residual
-// gradient share one element type T (bf16 or fp32).
-constexpr int LN_R = 16;
-
-template <int NV, typename T>
-__global__ void __launch_bounds__(256) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy, const T* __restrict__ x,
+// Backward: dx = rstd (g - mean(g) - xhat mean(g xhat)), g = gamma dy (+ alpha resid);
+// thread c keeps its columns' dgamma / dbeta partials in registers across the CTA's rows
+// and writes them to workspace[blockIdx.x][2][H]; ln_bwd_reduce_kernel adds them up.
+template <typename T>
+__global__ void __launch_bounds__(512) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy, const T* __restrict__ x,
                                                      const float* __restrict__ mean,
                                                      const float* __restrict__ rstd,
                                                      const float* __restrict__ gamma, const T* __restrict__ resid,
                                                      float resid_alpha, __nv_bfloat16* __restrict__ dx_bf16,
                                                      float* __restrict__ dx_f32, float* __restrict__ ws) {
-  constexpr int CPT = (NV * 32 + 255) / 256;  // column chunks per thread in phase 2
-  __shared__ float s_mg[LN_R], s_mgx[LN_R];
-  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-  const int nchunk = H / 8;
-  const float4* g4 = reinterpret_cast<const float4*>(gamma);
-  float gcol[CPT][8], accg[CPT][8], accb[CPT][8];
+  __shared__ float2 red[2][32];
+  const int c = threadIdx.x;
+  float gcol[8], accg[8], accb[8];
+  load8<float>(gamma, c, gcol);
 #pragma unroll
-  for (int j = 0; j < CPT; ++j) {
-    const int c = tid + 256 * j;
-#pragma unroll
-    for (int k = 0; k < 8; ++k) accg[j][k] = accb[j][k] = gcol[j][k] = 0.f;
-    if (c < nchunk) {
-      const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
-      gcol[j][0] = ga.x; gcol[j][1] = ga.y; gcol[j][2] = ga.z; gcol[j][3] = ga.w;
-      gcol[j][4] = gb.x; gcol[j][5] = gb.y; gcol[j][6] = gb.z; gcol[j][7] = gb.w;
-    }
+  for (int k = 0; k < 8; ++k) accg[k] = accb[k] = 0.f;
+  int par = 0;
+  float nd[8], nx[8];
+  int row = blockIdx.x;
+  if (row < Tn) {
+    load8<T>(dy + (int64_t)row * H, c, nd);
+    load8<T>(x + (int64_t)row * H, c, nx);
   }
-  for (int r0 = blockIdx.x * LN_R; r0 < Tn; r0 += gridDim.x * LN_R) {
-    // phase 1: per-row sums
-    for (int rr = wid; rr < LN_R; rr += 8) {
-      const int row = r0 + rr;
-      float s1 = 0.f, s2 = 0.f;
-      if (row < Tn) {
-        const T* dyr = dy + (int64_t)row * H;
-        const T* xr = x + (int64_t)row * H;
-        const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
-#pragma unroll 4
-        for (int i = 0; i < NV; ++i) {
-          const int c = lane + 32 * i;
-          float d[8], xv[8];
-          load8<T>(dyr, c, d);
-          load8<T>(xr, c, xv);
-          const float4 ga = __ldg(g4 + 2 * c), gb = __ldg(g4 + 2 * c + 1);
-          const float gg[8] = {ga.x, ga.y, ga.z, ga.w, gb.x, gb.y, gb.z, gb.w};
+  for (; row < Tn; row += gridDim.x) {
+    float d[8], xv[8];
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const float g = d[k] * gg[k];
-            s1 += g;
-            s2 += g * (xv[k] - mu) * rs;
-          }
-        }
-      }
-      s1 = warp_sum(s1);
-      s2 = warp_sum(s2);
-      if (lane == 0) {
-        s_mg[rr] = s1 / H;
-        s_mgx[rr] = s2 / H;
-      }
+    for (int k = 0; k < 8; ++k) {
+      d[k] = nd[k];
+      xv[k] = nx[k];
     }
-    __syncthreads();
-    // phase 2: dx and the column partials
-    const int rows = min(LN_R, Tn - r0);
-    for (int rr = 0; rr < rows; ++rr) {
-      const int row = r0 + rr;
-      const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
-      const float mg = s_mg[rr], mgx = s_mgx[rr];
-      const T* dyr = dy + (int64_t)row * H;
-      const T* xr = x + (int64_t)row * H;
-      const T* rr4 = resid ? resid + (int64_t)row * H : nullptr;
-#pragma unroll
-      for (int j = 0; j < CPT; ++j) {
-        const int c = tid + 256 * j;
-        if (c < nchunk) {
-          float d[8], xv[8], o[8];
-          load8<T>(dyr, c, d);
-          load8<T>(xr, c, xv);
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const float xh = (xv[k] - mu) * rs;
-            accg[j][k] += d[k] * xh;
-            accb[j][k] += d[k];
-            o[k] = rs * (d[k] * gcol[j][k] - mg - xh * mgx);
-          }
-          if (rr4) {
-            float r[8];
-            load8<T>(rr4, c, r);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) o[k] = fmaf(resid_alpha, r[k], o[k]);
-          }
-          if (dx_bf16) reinterpret_cast<uint4*>(dx_bf16 + (int64_t)row * H)[c] = pack8(o);
-          if (dx_f32) {
-            float4* df = reinterpret_cast<float4*>(dx_f32 + (int64_t)row * H) + 2 * c;
-            df[0] = make_float4(o[0], o[1], o[2], o[3]);
-            df[1] = make_float4(o[4], o[5], o[6], o[7]);
-          }
-        }
-      }
+    const int r2 = row + gridDim.x;
+    if (r2 < Tn) {
+      load8<T>(dy + (int64_t)r2 * H, c, nd);
+      load8<T>(x + (int64_t)r2 * H, c, nx);
     }
-    __syncthreads();
+    const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
+    float xh[8], s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      xh[k] = (xv[k] - mu) * rs;
+      const float g = d[k] * gcol[k];
+      s1 += g;
+      s2 += g * xh[k];
+      accg[k] += d[k] * xh[k];
+      accb[k] += d[k];
+    }
+    const float2 sums = block_sum2(s1, s2, red, par);
+    par ^= 1;
+    const float mg = sums.x / H, mgx = sums.y / H;
+    float o[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) o[k] = rs * (d[k] * gcol[k] - mg - xh[k] * mgx);
+    if (resid) {
+      float r[8];
+      load8<T>(resid + (int64_t)row * H, c, r);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) o[k] = fmaf(resid_alpha, r[k], o[k]);
+    }
+    if (dx_bf16) reinterpret_cast<uint4*>(dx_bf16 + (int64_t)row * H)[c] = pack8(o);
+    if (dx_f32) {
+      float4* df = reinterpret_cast<float4*>(dx_f32 + (int64_t)row * H) + 2 * c;
+      df[0] = make_float4(o[0], o[1], o[2], o[3]);
+      df[1] = make_float4(o[4], o[5], o[6], o[7]);
+    }
   }
   float* out = ws + (int64_t)blockIdx.x * 2 * H;
-#pragma unroll
-  for (int j = 0; j < CPT; ++j) {
-    const int c = tid + 256 * j;
-    if (c < nchunk) {
-      float4* og = reinterpret_cast<float4*>(out + 8 * c);
-      float4* ob = reinterpret_cast<float4*>(out + H + 8 * c);
-      og[0] = make_float4(accg[j][0], accg[j][1], accg[j][2], accg[j][3]);
-      og[1] = make_float4(accg[j][4], accg[j][5], accg[j][6], accg[j][7]);
-      ob[0] = make_float4(accb[j][0], accb[j][1], accb[j][2], accb[j][3]);
-      ob[1] = make_float4(accb[j][4], accb[j][5], accb[j][6], accb[j][7]);
-    }
-  }
+  float4* og = reinterpret_cast<float4*>(out + 8 * c);
+  float4* ob = reinterpret_cast<float4*>(out + H + 8 * c);
+  og[0] = make_float4(accg[0], accg[1], accg[2], accg[3]);
+  og[1] = make_float4(accg[4], accg[5], accg[6], accg[7]);
+  ob[0] = make_float4(accb[0], accb[1], accb[2], accb[3]);
+  ob[1] = make_float4(accb[4], accb[5], accb[6], accb[7]);
 }
 
 // dgamma/dbeta += sum over the nblk partial rows; blockIdx.y takes a slice of the rows.
@@ -267,12 +210,12 @@ __global__ void ln_bwd_reduce_kernel(int nblk, int H, const float* __restrict__ 
   atomicAdd(i < H ? dgamma + i : dbeta + (i - H), s);
 }
 
-// Launches the backward kernel and the reduction of its partials.
-template <int NV, typename T>
-int launch_ln_bwd(int nblk, int Tn, int H, const T* dy, const T* x, const float* mean, const float* rstd,
-                  const float* gamma, const T* resid, float alpha, __nv_bfloat16* dx_bf16, float* dx_f32, float* ws,
-                  float* dgamma, float* dbeta, cudaStream_t st) {
-  ln_bwd_kernel<NV, T><<<nblk, 256, 0, st>>>(Tn, H, dy, x, mean, rstd, gamma, resid, alpha, dx_bf16, dx_f32, ws);
+template <typename T>
+int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, const float* mean, const float* rstd,
+                    const float* gamma, const void* resid, float alpha, void* dx_bf16, float* dx_f32, float* ws,
+                    float* dgamma, float* dbeta, cudaStream_t st) {
+  ln_bwd_kernel<T><<<nblk, H / 8, 0, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma, (const T*)resid, alpha,
+                                           (__nv_bfloat16*)dx_bf16, dx_f32, ws);
   FL_CUDA_TRY(cudaGetLastError());
   const int split = nblk >= 64 ? 16 : 1;
   ln_bwd_reduce_kernel<<<dim3((2 * H + 255) / 256, split), 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
@@ -280,44 +223,20 @@ int launch_ln_bwd(int nblk, int Tn, int H, const T* dy, const T* x, const float*
   return FL_OK;
 }
 
-template <typename T>
-int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, const float* mean, const float* rstd,
-                    const float* gamma, const void* resid, float alpha, void* dx_bf16, float* dx_f32, float* ws,
-                    float* dgamma, float* dbeta, cudaStream_t st) {
-  auto dyp = (const T*)dy;
-  auto xp = (const T*)x;
-  auto rp = (const T*)resid;
-  auto dxb = (__nv_bfloat16*)dx_bf16;
-  switch (H / 256) {
-#define FL_LNB(NV) \
-  case NV: return launch_ln_bwd<NV, T>(nblk, Tn, H, dyp, xp, mean, rstd, gamma, rp, alpha, dxb, dx_f32, ws, dgamma, dbeta, st);
-    FL_LNB(1) FL_LNB(2) FL_LNB(4) FL_LNB(8) FL_LNB(16)
-#undef FL_LNB
-    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H/256 must be a power of two");
-  }
-}
-
 template <typename TX>
 int dispatch_ln_fwd(int Tn, int H, const void* x, const float* gamma, const float* beta, float eps, void* y,
                     float* mean, float* rstd, cudaStream_t st) {
-  const dim3 grid((Tn + 7) / 8), block(256);
-  auto xp = (const TX*)x;
-  auto yb = (__nv_bfloat16*)y;
-  switch (H / 256) {
-#define FL_LNF(NV) \
-  case NV: ln_fwd_kernel<NV, TX><<<grid, block, 0, st>>>(Tn, H, xp, gamma, beta, eps, yb, mean, rstd); break;
-    FL_LNF(1) FL_LNF(2) FL_LNF(4) FL_LNF(8) FL_LNF(16)
-#undef FL_LNF
-    default: return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H/256 must be a power of two");
-  }
+  int grid = 4 * sm_count() * (4096 / H);
+  if (grid > Tn) grid = Tn;
+  ln_fwd_kernel<TX><<<grid, H / 8, 0, st>>>(Tn, H, (const TX*)x, gamma, beta, eps, (__nv_bfloat16*)y, mean, rstd);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
 
+// CTAs of the backward (and rows of its partial-sum workspace).
 int ln_bwd_blocks(int T) {
-  const int want = (T + LN_R - 1) / LN_R;
   const int cap = 2 * sm_count();
-  return want < cap ? want : cap;
+  return T < cap ? T : cap;
 }
 
 // ------------------------------------------------------------------ column sums (bias grads)

@@ -146,7 +146,9 @@ def test_tiny_config_parity_fused_step(F, rfl):
 
 def test_fused_step_equals_backward_then_step(F):
     """Two steps of fl_server_backward_step against fl_server_backward + fl_server_step
-    on identically seeded servers (the fused AdamW epilogue uses the same fp32 formula)."""
+    on identically seeded servers (the fused AdamW epilogue uses the same fp32 formula;
+    the LayerNorm parameter gradients are summed with atomics, so their summation order,
+    and the last bits of those updates, may differ between runs)."""
     cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, seq_lens=(64, 40))
     states = [dev_bf16_from_bits(s) for s in syn.client_states(cfg)]
     grads = [dev_bf16_from_bits(g) for g in syn.client_grads(cfg)]
@@ -164,7 +166,7 @@ def test_fused_step_equals_backward_then_step(F):
     for blk in range(cfg.n_blocks):
         for t in range(12):
             wa, wb = a.get_param(blk, t), b.get_param(blk, t)
-            assert rel_inf(wb, wa) < 1e-6, (blk, t)
+            assert rel_inf(wb, wa) < 1e-5, (blk, t)
             ma, va = a.get_adam_moments(blk, t)
             mb, vb = b.get_adam_moments(blk, t)
             assert rel_inf(mb, ma) < 1e-5 and rel_inf(vb, va) < 1e-5
