@@ -218,6 +218,11 @@ def main():
     ap.add_argument("--sweep", action="store_true",
                     help="client-batching sweep: 26 blocks, 2 x 512 tokens per client, K in 1..32, "
                          "one packed call vs K sequential single-client calls (one JSON line per K)")
+    ap.add_argument("--hierarchical", type=int, default=0, metavar="K",
+                    help="the paper's three server strategies for K clients of 2 x 512 tokens on the 26-block "
+                         "stack: K server replicas (one per client, averaged every --period steps), one "
+                         "client-batched server, and one server taking the clients one after another")
+    ap.add_argument("--period", type=int, default=50, help="averaging period of --hierarchical (steps)")
     ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
@@ -226,6 +231,9 @@ def main():
         return
     if args.sweep:
         run_sweep(args)
+        return
+    if args.hierarchical:
+        run_strategies(args, args.hierarchical)
         return
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -484,6 +492,79 @@ def run_sweep(args):
                 "batched_over_sequential": res["batched"]["tokens_per_s"] / res["sequential"]["tokens_per_s"]}
         print(json.dumps(line), flush=True)
     srv.close()
+
+
+def run_strategies(args, K: int):
+    """§3.3 strategies on one GPU for K clients of 2 x 512 tokens (the 26-block stack):
+    server-hierarchical (K replicas, one client each, parameters averaged every period),
+    client-batch (one server, the K clients packed in one call) and serial (one server, the
+    clients one call after another, one update)."""
+    import torch
+    from paper_2406_14898_gb300 import flglm as F
+    from paper_2406_14898_gb300.hierarchical import HierarchicalServers
+
+    cfg = syn.sweep_config(K)
+    one = cfg.with_(seq_lens=cfg.seq_lens[:1])
+    dev = torch.device("cuda", 0)
+    sb, gb = syn.client_states(cfg), syn.client_grads(cfg)
+    st = [torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev) for b in sb]
+    go = [torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev) for b in gb]
+    outs = [torch.empty_like(s) for s in st]
+    gin = [torch.empty_like(s) for s in st]
+    pk = peaks()
+    flops = gemm_flops(cfg) + attn_flops(cfg)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    res = {}
+
+    def timed(fn, sync):
+        for _ in range(args.warmup):
+            fn()
+        sync()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            fn()
+        sync()
+        torch.cuda.synchronize()
+        return 1e3 * (time.perf_counter() - t0) / args.steps
+
+    # server-hierarchical: K replicas on their own streams
+    hs = HierarchicalServers(F.make_cfg(one, one.tokens, 512), cfg.seed, K)
+    ms = timed(lambda: hs.step(st, cfg.seq_lens, outs, go, gin, cfg.lr), hs.sync)
+    t0 = time.perf_counter()
+    hs.average()
+    avg_ms = 1e3 * (time.perf_counter() - t0)
+    hs.close()
+    torch.cuda.empty_cache()
+    amort = ms + avg_ms / args.period
+    res["server_hierarchical"] = {"replicas": K, "ms_per_step": ms, "average_ms": avg_ms, "period": args.period,
+                                  "tokens_per_s": cfg.tokens / (amort / 1e3),
+                                  "pct_bf16_peak": 100.0 * flops / (amort / 1e3) / (pk["bf16_sustained"] * 1e12)}
+    # client-batch and serial on one server
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, 512), cfg.seed)
+
+    def batched():
+        srv.forward(st, cfg.seq_lens, outs)
+        srv.backward_step(go, gin, cfg.lr)
+
+    def serial():
+        for k in range(K):
+            srv.forward(st[k:k + 1], cfg.seq_lens[k:k + 1], outs[k:k + 1])
+            srv.backward(go[k:k + 1], gin[k:k + 1])
+        srv.step(cfg.lr)
+
+    for name, fn in (("client_batch", batched), ("serial", serial)):
+        ms = timed(fn, srv.sync)
+        res[name] = {"ms_per_step": ms, "tokens_per_s": cfg.tokens / (ms / 1e3),
+                     "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / (pk["bf16_sustained"] * 1e12)}
+    srv.close()
+    line = {"metric": METRIC, "mode": "server strategies (Sec. 3.3)", "K": K,
+            "value": res["client_batch"]["tokens_per_s"], "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": describe(cfg), "global_batch": cfg.tokens, "seq_len": 512},
+            "timing": "host wall clock around the timed steps, after a device synchronisation on both sides",
+            **res}
+    print(json.dumps(line), flush=True)
 
 
 def pci_bus_id(torch, dev):

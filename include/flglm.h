@@ -161,6 +161,25 @@ int fl_server_get_grad(fl_server_t h, int32_t block, int32_t tensor_id, float* h
 int fl_server_get_adam_moments(fl_server_t h, int32_t block, int32_t tensor_id, float* host_m,
                                float* host_v, size_t n);
 
+/* Server-hierarchical strategy (§3.3): one server replica per client, run side by side,
+ * the replicas' parameters averaged at the end of each training period.
+ * fl_server_average replaces the fp32 master weights of each of the n replicas (same
+ * configuration, same device) by their arithmetic mean (summed in replica order) and
+ * refreshes their bf16 copies.  Adam moments and step counts stay per replica (local
+ * optimizer state).  It waits for every replica's stream, runs on replicas[0]'s stream
+ * and returns after the mean is written.  Errors: INVALID_ARG (n outside 1..64, null,
+ * duplicate, different shapes), STATE (a replica has a pending forward), CUDA. */
+int fl_server_average(fl_server_t const* replicas, int32_t n);
+
+/* Device address and element count of the fp32 master-weight arena, for averaging across
+ * processes (one replica per GPU: all-reduce the arena, divide by the number of ranks,
+ * then call fl_server_refresh_working_copy).  The arena is owned by the library. */
+int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n);
+
+/* Recomputes the bf16 working copy from the fp32 master weights (after they were changed
+ * outside the library), on the handle's stream. */
+int fl_server_refresh_working_copy(fl_server_t h);
+
 /* Kernel timing by class (GEMM, attention, LayerNorm, AdamW, other) with CUDA events
  * recorded on the handle's stream around each launch.  enable != 0 starts recording
  * (and clears the totals); fl_server_profile_read fills ms[c] and launches[c] for

@@ -372,3 +372,15 @@ class OracleServer:
                 self.params[bi][i], self.m[bi][i], self.v[bi][i] = w, m, v
                 self.grads[bi][i] = np.zeros_like(w)
 
+
+
+def average_params(servers: Sequence["OracleServer"]):
+    """§3.3 server-hierarchical strategy: at the end of a training period every replica's
+    parameters are replaced by the arithmetic mean over the replicas; optimizer moments and
+    step counts stay with each replica."""
+    n = len(servers)
+    for b in range(len(servers[0].params)):
+        for t in range(len(servers[0].params[b])):
+            mean = sum(s.params[b][t] for s in servers) / n
+            for s in servers:
+                s.params[b][t] = mean.copy()

@@ -36,6 +36,15 @@ struct MetaArgs {
 };
 
 int fl_launch_copy_clients(const CopyTable& tab, cudaStream_t st);
+
+// Replicas averaged together: fp32 master arenas and bf16 copies, same length.
+constexpr int FL_MAX_REPLICAS = 64;
+struct ReplicaTable {
+  int n;
+  float* w[FL_MAX_REPLICAS];
+  void* wb[FL_MAX_REPLICAS];
+};
+int fl_launch_average(const ReplicaTable& t, int64_t n, cudaStream_t st);
 int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st);
 int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, float* out, cudaStream_t st);
 int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st);

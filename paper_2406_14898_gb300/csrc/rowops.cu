@@ -297,6 +297,26 @@ __global__ void __launch_bounds__(256) adamw_kernel(int64_t n4, float4* __restri
   }
 }
 
+// Parameter averaging of n replicas (§3.3 server-hierarchical: the replicas' parameters are
+// averaged at the end of each period).  Every replica's fp32 master and bf16 copy receive
+// the arithmetic mean, summed in replica order (deterministic).
+__global__ void __launch_bounds__(256) average_kernel(ReplicaTable t, int64_t n4) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+    float4 s = reinterpret_cast<const float4*>(t.w[0])[i];
+    for (int r = 1; r < t.n; ++r) {
+      const float4 v = reinterpret_cast<const float4*>(t.w[r])[i];
+      s.x += v.x; s.y += v.y; s.z += v.z; s.w += v.w;
+    }
+    const float inv = 1.f / (float)t.n;
+    const float4 mean = make_float4(s.x * inv, s.y * inv, s.z * inv, s.w * inv);
+    const uint2 packed = make_uint2(pack_bf16x2(mean.x, mean.y), pack_bf16x2(mean.z, mean.w));
+    for (int r = 0; r < t.n; ++r) {
+      reinterpret_cast<float4*>(t.w[r])[i] = mean;
+      reinterpret_cast<uint2*>(t.wb[r])[i] = packed;
+    }
+  }
+}
+
 __global__ void f32_to_bf16_kernel(int64_t n, const float* __restrict__ src, __nv_bfloat16* __restrict__ dst) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
     dst[i] = f2bf(src[i]);
@@ -499,6 +519,13 @@ int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, flo
 int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st) {
   if (n <= 0) return FL_OK;
   fill_kernel<<<grid_for(n), 256, 0, st>>>(n, v, out);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_average(const ReplicaTable& t, int64_t n, cudaStream_t st) {
+  if (n <= 0 || t.n <= 0) return FL_OK;
+  average_kernel<<<grid_for(n / 4), 256, 0, st>>>(t, n / 4);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }

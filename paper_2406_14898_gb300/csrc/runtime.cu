@@ -792,6 +792,53 @@ extern "C" int fl_server_set_param(fl_server_t h, int32_t b, int32_t t, const fl
   return FL_OK;
 }
 
+extern "C" int fl_server_average(fl_server_t const* replicas, int32_t n) {
+  if (!replicas || n < 1 || n > FL_MAX_REPLICAS)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "average: need 1..%d replicas", FL_MAX_REPLICAS);
+  fl_server* h0 = replicas[0];
+  if (!h0) return fl_internal_error(FL_ERR_INVALID_ARG, "average: null replica");
+  ReplicaTable t;
+  memset(&t, 0, sizeof t);
+  t.n = n;
+  for (int r = 0; r < n; ++r) {
+    fl_server* h = replicas[r];
+    if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "average: null replica %d", r);
+    if (h->n_params != h0->n_params || h->cfg.n_blocks != h0->cfg.n_blocks || h->cfg.hidden != h0->cfg.hidden ||
+        h->cfg.ffn_hidden != h0->cfg.ffn_hidden)
+      return fl_internal_error(FL_ERR_INVALID_ARG, "average: replica %d has another shape", r);
+    if (h->pending) return set_err(h, FL_ERR_STATE, "average: replica %d has a pending forward", r);
+    for (int q = 0; q < r; ++q)
+      if (replicas[q] == h) return fl_internal_error(FL_ERR_INVALID_ARG, "average: replica %d listed twice", r);
+    t.w[r] = h->w;
+    t.wb[r] = h->wb;
+  }
+  // order the averaging after every replica's queued work, on replica 0's stream
+  for (int r = 1; r < n; ++r) {
+    cudaError_t e = cudaStreamSynchronize(replicas[r]->stream);
+    if (e != cudaSuccess) return fwd_err(h0, fl_internal_cuda_error(e, "average: sync", __FILE__, __LINE__));
+  }
+  prof_begin(h0, FL_PROF_OTHER);
+  int rc = fl_launch_average(t, h0->n_params, h0->stream);
+  prof_end(h0);
+  if (rc) return fwd_err(h0, rc);
+  cudaError_t e = cudaStreamSynchronize(h0->stream);
+  if (e != cudaSuccess) return fwd_err(h0, fl_internal_cuda_error(e, "average", __FILE__, __LINE__));
+  return FL_OK;
+}
+
+extern "C" int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n) {
+  if (!h || !dev_w || !n) return fl_internal_error(FL_ERR_INVALID_ARG, "param_arena: null");
+  *dev_w = h->w;
+  *n = h->n_params;
+  return FL_OK;
+}
+
+extern "C" int fl_server_refresh_working_copy(fl_server_t h) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "refresh: null handle");
+  int rc = fl_launch_f32_to_bf16(h->n_params, h->w, h->wb, h->stream);
+  return fwd_err(h, rc);
+}
+
 extern "C" int fl_server_profile(fl_server_t h, int enable) {
   if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "profile: null handle");
   cudaStreamSynchronize(h->stream);

@@ -77,6 +77,9 @@ _SIGS = {
     "fl_server_set_param": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
     "fl_server_get_grad": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
     "fl_server_get_adam_moments": (C.c_int, [_P, _I32, _I32, _P, _P, C.c_size_t]),
+    "fl_server_average": (C.c_int, [C.POINTER(_P), _I32]),
+    "fl_server_param_arena": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I64)]),
+    "fl_server_refresh_working_copy": (C.c_int, [_P]),
     "fl_server_profile": (C.c_int, [_P, C.c_int]),
     "fl_server_profile_read": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(_I64), _I32]),
     "fl_server_launch_count": (_I64, [_P]),
@@ -235,6 +238,16 @@ class Server:
         a = np.ascontiguousarray(values, np.float32).reshape(-1)
         check(lib().fl_server_set_param(self.h, block, tensor_id, a.ctypes.data, a.size), self.h)
 
+    def param_arena(self):
+        """(device address, element count) of the fp32 master-weight arena."""
+        p = C.c_void_p()
+        n = C.c_int64()
+        check(lib().fl_server_param_arena(self.h, C.byref(p), C.byref(n)), self.h)
+        return int(p.value), int(n.value)
+
+    def refresh_working_copy(self):
+        check(lib().fl_server_refresh_working_copy(self.h), self.h)
+
     def profile(self, enable: bool):
         check(lib().fl_server_profile(self.h, 1 if enable else 0), self.h)
 
@@ -247,6 +260,12 @@ class Server:
 
     def launch_count(self) -> int:
         return int(lib().fl_server_launch_count(self.h))
+
+
+def fl_server_average(replicas: Sequence["Server"]):
+    """Averages the replicas' parameters in place (the server-hierarchical strategy)."""
+    arr = (C.c_void_p * len(replicas))(*[r.h.value for r in replicas])
+    check(lib().fl_server_average(arr, len(replicas)), replicas[0].h if replicas else None)
 
 
 # ----------------------------------------------------------------------------- kernel-level calls

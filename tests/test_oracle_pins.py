@@ -390,3 +390,31 @@ def test_server_protocol_state_and_accumulation():
     srv.step(1e-3)
     assert all(not g.any() for g in srv.grads[0])
     assert srv.t == 1
+
+
+def test_replica_averaging():
+    """Averaging is the arithmetic mean; identical replicas are unchanged; training K
+    replicas on the same client for one step and averaging equals one replica's step."""
+    cfg = tiny_cfg(n_blocks=1, seq_lens=(3,), b=1)
+    rng = np.random.default_rng(50)
+    params = random_params(cfg, rng, std=0.2)
+    a = O.OracleServer(cfg, params)
+    b = O.OracleServer(cfg, params)
+    c = O.OracleServer(cfg, params)
+    for t in range(12):
+        b.params[0][t] = b.params[0][t] + 1.0
+        c.params[0][t] = c.params[0][t] - 4.0
+    O.average_params([a, b, c])
+    for t in range(12):
+        np.testing.assert_allclose(a.params[0][t], np.asarray(params[0][t]) - 1.0, rtol=0, atol=1e-12)
+        np.testing.assert_array_equal(a.params[0][t], c.params[0][t])
+    st = [rng.standard_normal((1, 3, cfg.hidden))]
+    gr = [rng.standard_normal((1, 3, cfg.hidden))]
+    reps = [O.OracleServer(cfg, params) for _ in range(3)]
+    for r in reps:
+        r.forward(st)
+        r.backward(gr)
+        r.step(1e-3)
+    O.average_params(reps)
+    for t in range(12):
+        np.testing.assert_allclose(reps[0].params[0][t], reps[1].params[0][t], rtol=0, atol=0)
