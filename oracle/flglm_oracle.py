@@ -143,8 +143,22 @@ def rope_rotate(x: np.ndarray, cos: np.ndarray, sin: np.ndarray, rotary_dim: int
 # ----------------------------------------------------------------------------- attention
 
 
-def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray):
-    """Per segment, per head: O = softmax(Q K^T / sqrt(d_h) + causal) V (App. A scale).
+def _keys_values(k, v, pk, pv, a, b, h):
+    """Keys and values one segment's queries see: the prefix (P-tuning v2, App. A:
+    K' = [prefix_key : key], V' = [prefix_value : value]) then the segment's own."""
+    if pk is None:
+        return k[a:b, h], v[a:b, h], 0
+    return np.concatenate([pk[:, h], k[a:b, h]]), np.concatenate([pv[:, h], v[a:b, h]]), pk.shape[0]
+
+
+def _mask(L: int, Lp: int):
+    """Query t sees every prefix key and the keys u <= t of its own segment."""
+    return np.concatenate([np.ones((L, Lp), bool), np.tril(np.ones((L, L), bool))], axis=1)
+
+
+def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray, pk=None, pv=None):
+    """Per segment, per head: O = softmax(Q K'^T / sqrt(d_h) + mask) V' (App. A), K' and V'
+    the optional prefix followed by the segment's causal keys.
     Returns O [T, nh, hd] and the row log-sum-exp LSE [nh, T] of the scaled scores."""
     T, nh, hd = q.shape
     scale = 1.0 / math.sqrt(hd)
@@ -155,44 +169,55 @@ def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.nd
         L = b - a
         if L == 0:
             continue
-        causal = np.tril(np.ones((L, L), bool))
         for h in range(nh):
-            S = (q[a:b, h] @ k[a:b, h].T) * scale
-            S = np.where(causal, S, -np.inf)
+            kk, vv, Lp = _keys_values(k, v, pk, pv, a, b, h)
+            S = (q[a:b, h] @ kk.T) * scale
+            S = np.where(_mask(L, Lp), S, -np.inf)
             m = S.max(axis=-1)
             P = np.exp(S - m[:, None])
             l = P.sum(axis=-1)
             P /= l[:, None]
-            o[a:b, h] = P @ v[a:b, h]
+            o[a:b, h] = P @ vv
             lse[h, a:b] = m + np.log(l)
     return o, lse
 
 
-def attention_bwd(do: np.ndarray, q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray):
-    """Chain rule of attention_fwd: dV = P^T dO, dP = dO V^T, dS = P (dP - rowsum(dP P)),
-    dQ = dS K / sqrt(d_h), dK = dS^T Q / sqrt(d_h)."""
+def attention_bwd(do: np.ndarray, q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray,
+                  pk=None, pv=None):
+    """Chain rule of attention_fwd: dV' = P^T dO, dP = dO V'^T, dS = P (dP - rowsum(dP P)),
+    dQ = dS K' / sqrt(d_h), dK' = dS^T Q / sqrt(d_h).  With a prefix, its gradients are
+    summed over every segment (the prefix is shared) and returned as dpk, dpv."""
     T, nh, hd = q.shape
     scale = 1.0 / math.sqrt(hd)
     dq = np.zeros_like(q)
     dk = np.zeros_like(k)
     dv = np.zeros_like(v)
+    dpk = None if pk is None else np.zeros_like(pk)
+    dpv = None if pv is None else np.zeros_like(pv)
     for s in range(len(cu_seqlens) - 1):
         a, b = int(cu_seqlens[s]), int(cu_seqlens[s + 1])
         L = b - a
         if L == 0:
             continue
-        causal = np.tril(np.ones((L, L), bool))
         for h in range(nh):
-            S = (q[a:b, h] @ k[a:b, h].T) * scale
-            S = np.where(causal, S, -np.inf)
+            kk, vv, Lp = _keys_values(k, v, pk, pv, a, b, h)
+            S = (q[a:b, h] @ kk.T) * scale
+            S = np.where(_mask(L, Lp), S, -np.inf)
             P = np.exp(S - S.max(axis=-1, keepdims=True))
             P /= P.sum(axis=-1, keepdims=True)
-            dP = do[a:b, h] @ v[a:b, h].T
+            dP = do[a:b, h] @ vv.T
             dS = P * (dP - (dP * P).sum(axis=-1, keepdims=True))
-            dv[a:b, h] = P.T @ do[a:b, h]
-            dq[a:b, h] = (dS @ k[a:b, h]) * scale
-            dk[a:b, h] = (dS.T @ q[a:b, h]) * scale
-    return dq, dk, dv
+            dvv = P.T @ do[a:b, h]
+            dkk = (dS.T @ q[a:b, h]) * scale
+            dq[a:b, h] = (dS @ kk) * scale
+            dv[a:b, h] = dvv[Lp:]
+            dk[a:b, h] = dkk[Lp:]
+            if Lp:
+                dpk[:, h] += dkk[:Lp]
+                dpv[:, h] += dvv[:Lp]
+    if pk is None:
+        return dq, dk, dv
+    return dq, dk, dv, dpk, dpv
 
 
 # ----------------------------------------------------------------------------- GeLU (tanh form)
@@ -231,8 +256,10 @@ class BlockShape:
                           cfg.rope_base, cfg.ln_eps, cfg.residual_alpha, cfg.residual_from_ln)
 
 
-def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShape):
-    """One server block over the packed tokens x [T, H]; returns y and the saved values."""
+def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShape, prefix=None):
+    """One server block over the packed tokens x [T, H]; returns y and the saved values.
+    prefix: optional (prefix_key, prefix_value), each [L_p, H], seen by every query (App. A);
+    the prefix keys enter the scores as they are (no rotary rotation)."""
     Wqkv, bqkv, Wd, bd, W1, b1, W2, b2, g1, be1, g2, be2 = P
     T, H = x.shape
     nh, hd = sh.n_heads, sh.head_dim
@@ -244,7 +271,11 @@ def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShap
     cos, sin = rope_cos_sin(pk.pos, sh.rotary_dim, sh.rope_base)
     qr = rope_rotate(q, cos, sin, sh.rotary_dim)
     kr = rope_rotate(k, cos, sin, sh.rotary_dim)
-    o, lse = attention_fwd(qr, kr, v, pk.cu_seqlens)
+    ppk = ppv = None
+    if prefix is not None:
+        ppk = np.asarray(prefix[0], F64).reshape(-1, nh, hd)
+        ppv = np.asarray(prefix[1], F64).reshape(-1, nh, hd)
+    o, lse = attention_fwd(qr, kr, v, pk.cu_seqlens, ppk, ppv)
     o = o.reshape(T, H)
     res1 = a if sh.residual_from_ln else x
     h = sh.alpha * res1 + (o @ Wd.T + bd[None, :])
@@ -254,12 +285,13 @@ def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShap
     res2 = m if sh.residual_from_ln else h
     y = sh.alpha * res2 + (g @ W2.T + b2[None, :])
     saved = dict(x=x, a=a, mu1=mu1, rs1=rs1, qr=qr, kr=kr, v=v, o=o, lse=lse, h=h, m=m,
-                 mu2=mu2, rs2=rs2, u=u, g=g, cos=cos, sin=sin)
+                 mu2=mu2, rs2=rs2, u=u, g=g, cos=cos, sin=sin, ppk=ppk, ppv=ppv)
     return y, saved
 
 
 def block_bwd(P: Sequence[np.ndarray], sv: dict, dy: np.ndarray, pk: Packing, sh: BlockShape):
-    """Exact chain rule of block_fwd.  Returns dx and the 12 parameter gradients (summed over T)."""
+    """Exact chain rule of block_fwd.  Returns dx and the 12 parameter gradients (summed over T),
+    followed by the prefix key and value gradients [L_p, H] when the block has a prefix."""
     Wqkv, bqkv, Wd, bd, W1, b1, W2, b2, g1, be1, g2, be2 = P
     T, H = dy.shape
     nh, hd = sh.n_heads, sh.head_dim
@@ -281,7 +313,8 @@ def block_bwd(P: Sequence[np.ndarray], sv: dict, dy: np.ndarray, pk: Packing, sh
     dWd = dh.T @ sv["o"]
     dbd = dh.sum(axis=0)
     do = (dh @ Wd).reshape(T, nh, hd)
-    dqr, dkr, dv = attention_bwd(do, sv["qr"], sv["kr"], sv["v"], pk.cu_seqlens)
+    res = attention_bwd(do, sv["qr"], sv["kr"], sv["v"], pk.cu_seqlens, sv["ppk"], sv["ppv"])
+    dqr, dkr, dv = res[:3]
     dq = rope_rotate(dqr, sv["cos"], sv["sin"], sh.rotary_dim, inverse=True)
     dk = rope_rotate(dkr, sv["cos"], sv["sin"], sh.rotary_dim, inverse=True)
     dqkv = np.concatenate([dq.reshape(T, H), dk.reshape(T, H), dv.reshape(T, H)], axis=1)
@@ -293,16 +326,19 @@ def block_bwd(P: Sequence[np.ndarray], sv: dict, dy: np.ndarray, pk: Packing, sh
     dx, dg1, dbe1 = layer_norm_bwd(da, sv["x"], sv["mu1"], sv["rs1"], g1)
     if not sh.residual_from_ln:
         dx = dx + al * dh
-    return dx, [dWqkv, dbqkv, dWd, dbd, dW1, db1, dW2, db2, dg1, dbe1, dg2, dbe2]
+    grads = [dWqkv, dbqkv, dWd, dbd, dW1, db1, dW2, db2, dg1, dbe1, dg2, dbe2]
+    if sv["ppk"] is not None:
+        grads += [res[3].reshape(-1, H), res[4].reshape(-1, H)]
+    return dx, grads
 
 
 # ----------------------------------------------------------------------------- stack + server
 
 
-def stack_fwd(params: Sequence[Sequence[np.ndarray]], x: np.ndarray, pk: Packing, sh: BlockShape):
+def stack_fwd(params: Sequence[Sequence[np.ndarray]], x: np.ndarray, pk: Packing, sh: BlockShape, prefixes=None):
     saved = []
-    for P in params:
-        x, sv = block_fwd(P, x, pk, sh)
+    for b, P in enumerate(params):
+        x, sv = block_fwd(P, x, pk, sh, None if prefixes is None else prefixes[b])
         saved.append(sv)
     return x, saved
 
@@ -327,14 +363,22 @@ def adamw_update(w, g, m, v, t: int, lr: float, beta1: float, beta2: float, eps:
 class OracleServer:
     """The server's protocol on the oracle: forward(client states) -> output states,
     backward(output-state grads) -> input-state grads (+ accumulated weight grads),
-    step(lr) -> AdamW update that clears the grads."""
+    step(lr) -> AdamW update that clears the grads.  With cfg.prefix_len > 0 every block
+    carries P-tuning v2 prefix keys and values (tensors 12 and 13 of the block); with
+    cfg.freeze_base the step updates only those (App. A: the model is frozen and only the
+    prefix is trained)."""
 
-    def __init__(self, cfg: syn.ServerConfig, params: Optional[List[List[np.ndarray]]] = None):
+    def __init__(self, cfg: syn.ServerConfig, params: Optional[List[List[np.ndarray]]] = None, prefixes=None):
         self.cfg = cfg
         self.sh = BlockShape.of(cfg)
         if params is None:
             params = syn.init_params(cfg)
+        if cfg.prefix_len and prefixes is None:
+            prefixes = [syn.init_prefix(cfg, b) for b in range(cfg.n_blocks)]
         self.params = [[np.asarray(p, F64).copy() for p in blk] for blk in params]
+        if cfg.prefix_len:
+            for blk, pre in zip(self.params, prefixes):
+                blk.extend(np.asarray(p, F64).copy() for p in pre)
         self.grads = [[np.zeros_like(p) for p in blk] for blk in self.params]
         self.m = [[np.zeros_like(p) for p in blk] for blk in self.params]
         self.v = [[np.zeros_like(p) for p in blk] for blk in self.params]
@@ -346,7 +390,9 @@ class OracleServer:
         b = client_states[0].shape[0]
         pk = make_packing(seq_lens, b)
         X = pack([np.asarray(s, F64) for s in client_states])
-        Y, saved = stack_fwd(self.params, X, pk, self.sh)
+        base = [blk[:12] for blk in self.params]
+        pre = [blk[12:14] for blk in self.params] if self.cfg.prefix_len else None
+        Y, saved = stack_fwd(base, X, pk, self.sh, pre)
         self._pending = (seq_lens, b, pk, saved)
         return unpack(Y, seq_lens, b)
 
@@ -355,9 +401,9 @@ class OracleServer:
             raise RuntimeError("backward without a pending forward")
         seq_lens, b, pk, saved = self._pending
         dY = pack([np.asarray(g, F64) for g in grad_out])
-        dX, grads = stack_bwd(self.params, saved, dY, pk, self.sh)
+        dX, grads = stack_bwd([blk[:12] for blk in self.params], saved, dY, pk, self.sh)
         for gb, acc in zip(grads, self.grads):
-            for i in range(12):
+            for i in range(len(gb)):
                 acc[i] += gb[i]
         self._pending = None
         return unpack(dX, seq_lens, b)
@@ -365,12 +411,13 @@ class OracleServer:
     def step(self, lr: float):
         c = self.cfg
         self.t += 1
+        trained = range(12, 14) if c.freeze_base else range(len(self.params[0]))
         for bi in range(len(self.params)):
-            for i in range(12):
+            for i in trained:
                 w, m, v = adamw_update(self.params[bi][i], self.grads[bi][i], self.m[bi][i], self.v[bi][i],
                                        self.t, lr, c.adam_beta1, c.adam_beta2, c.adam_eps, c.weight_decay)
                 self.params[bi][i], self.m[bi][i], self.v[bi][i] = w, m, v
-                self.grads[bi][i] = np.zeros_like(w)
+            self.grads[bi] = [np.zeros_like(g) for g in self.grads[bi]]
 
 
 

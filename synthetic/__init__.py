@@ -168,6 +168,8 @@ class ServerConfig:
     seed: int = 0
     state_std: float = 1.0
     grad_std: float = 1e-3
+    prefix_len: int = 0        # P-tuning v2 prefix keys/values per block (0: none)
+    freeze_base: int = 0       # 1: only the prefixes are trained (P-tuning v2)
 
     @property
     def K(self) -> int:
@@ -195,6 +197,25 @@ class ServerConfig:
 def param_shapes(cfg: ServerConfig) -> List[tuple]:
     H, F = cfg.hidden, cfg.ffn_hidden
     return [(3 * H, H), (3 * H,), (H, H), (H,), (F, H), (F,), (H, F), (H,), (H,), (H,), (H,), (H,)]
+
+
+# prefix tensors of a block (P-tuning v2): keys then values, [prefix_len, hidden] each,
+# head j at columns j*head_dim (ids follow the 12 block tensors)
+T_PK, T_PV = 12, 13
+
+
+def prefix_shapes(cfg: ServerConfig) -> List[tuple]:
+    return [(cfg.prefix_len, cfg.hidden), (cfg.prefix_len, cfg.hidden)]
+
+
+def init_prefix(cfg: ServerConfig, block: int, seed: Optional[int] = None) -> List[np.ndarray]:
+    """Initial fp32 prefix keys and values of a block: N(0, init_std), streams (seed, 1, block, 12|13)."""
+    seed = cfg.seed if seed is None else seed
+    out = []
+    for t, shp in zip((T_PK, T_PV), prefix_shapes(cfg)):
+        n = int(np.prod(shp))
+        out.append(normal_f32(stream_key(seed, P_WEIGHTS, block, t), n, 0.0, float(np.float32(cfg.init_std))).reshape(shp))
+    return out
 
 
 def params_per_block(cfg: ServerConfig) -> int:

@@ -418,3 +418,115 @@ def test_replica_averaging():
     O.average_params(reps)
     for t in range(12):
         np.testing.assert_allclose(reps[0].params[0][t], reps[1].params[0][t], rtol=0, atol=0)
+
+
+# ----------------------------------------------------------------------------- P-tuning v2 prefix (App. A)
+
+def test_prefix_attention_matches_torch_sdpa():
+    """Each query sees every prefix key and its own causal keys: one SDPA call per segment
+    with an explicit boolean mask over [prefix ; segment]."""
+    rng = np.random.default_rng(60)
+    seq = [5, 1, 9]
+    cu = np.cumsum([0] + seq).astype(np.int32)
+    T, nh, hd, Lp = cu[-1], 2, 8, 3
+    q, k, v = (rng.standard_normal((T, nh, hd)) for _ in range(3))
+    pk, pv = (rng.standard_normal((Lp, nh, hd)) for _ in range(2))
+    o, lse = O.attention_fwd(q, k, v, cu, pk, pv)
+    for s in range(len(seq)):
+        a, b = cu[s], cu[s + 1]
+        L = b - a
+        tq = torch.tensor(q[a:b]).transpose(0, 1)
+        tk = torch.tensor(np.concatenate([pk, k[a:b]])).transpose(0, 1)
+        tv = torch.tensor(np.concatenate([pv, v[a:b]])).transpose(0, 1)
+        mask = torch.cat([torch.ones(L, Lp, dtype=torch.bool), torch.ones(L, L, dtype=torch.bool).tril()], 1)
+        ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, attn_mask=mask).transpose(0, 1).numpy()
+        np.testing.assert_allclose(o[a:b], ref, rtol=0, atol=1e-12)
+
+
+def test_zero_value_prefix_closed_form():
+    """With zero prefix values the prefix only adds mass to the softmax denominator:
+    O' = O exp(LSE - LSE') and LSE' = log(exp(LSE) + sum_p exp(q.k_p / sqrt(d_h)))."""
+    rng = np.random.default_rng(61)
+    seq = [6, 4]
+    cu = np.cumsum([0] + seq).astype(np.int32)
+    T, nh, hd, Lp = cu[-1], 2, 8, 5
+    q, k, v = (rng.standard_normal((T, nh, hd)) for _ in range(3))
+    pk = rng.standard_normal((Lp, nh, hd))
+    o0, lse0 = O.attention_fwd(q, k, v, cu)
+    o1, lse1 = O.attention_fwd(q, k, v, cu, pk, np.zeros((Lp, nh, hd)))
+    lp = np.log(np.exp(np.einsum("thd,phd->htp", q, pk) / math.sqrt(hd)).sum(-1))
+    np.testing.assert_allclose(lse1, np.logaddexp(lse0, lp), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(o1, o0 * np.exp(lse0 - lse1).T[:, :, None], rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("rfl", [1, 0])
+def test_finite_difference_prefix_gradients(rfl):
+    cfg = tiny_cfg(residual_from_ln=rfl, n_blocks=2, seq_lens=(3, 5), b=1).with_(prefix_len=2)
+    rng = np.random.default_rng(62 + rfl)
+    params = random_params(cfg, rng)
+    prefixes = [[0.5 * rng.standard_normal((2, cfg.hidden)) for _ in range(2)] for _ in range(cfg.n_blocks)]
+    pk = O.make_packing(cfg.seq_lens, 1)
+    X = rng.standard_normal((pk.T, cfg.hidden))
+    dY = rng.standard_normal((pk.T, cfg.hidden))
+    sh = O.BlockShape.of(cfg)
+
+    def f(pre, X_):
+        Y, _ = O.stack_fwd(params, X_, pk, sh, pre)
+        return float((Y * dY).sum())
+    _, saved = O.stack_fwd(params, X, pk, sh, prefixes)
+    dX, grads = O.stack_bwd(params, saved, dY, pk, sh)
+    h = 1e-5
+    for b in range(cfg.n_blocks):
+        for j in range(2):
+            an = grads[b][12 + j].reshape(-1)
+            scale = np.abs(an).max()
+            for i in range(an.size):
+                pp = [[p.copy() for p in blk] for blk in prefixes]
+                pp[b][j].reshape(-1)[i] += h
+                fp = f(pp, X)
+                pp[b][j].reshape(-1)[i] -= 2 * h
+                fm = f(pp, X)
+                assert abs((fp - fm) / (2 * h) - an[i]) <= 1e-6 * scale, (b, j, i)
+    # the input gradient with a prefix, spot-checked
+    for i in (0, 17, 60, 127):
+        Xp = X.copy()
+        Xp.reshape(-1)[i] += h
+        fp = f(prefixes, Xp)
+        Xp.reshape(-1)[i] -= 2 * h
+        fm = f(prefixes, Xp)
+        assert abs((fp - fm) / (2 * h) - dX.reshape(-1)[i]) <= 1e-6 * np.abs(dX).max()
+
+
+def test_prefix_batching_invariant_and_frozen_step():
+    """The shared prefix keeps clients unmixed: packed results equal per-client runs and
+    prefix gradients are the sum of the per-client ones; with a frozen base only the
+    prefixes move."""
+    cfg = tiny_cfg(n_blocks=2, seq_lens=(3, 6), b=1).with_(prefix_len=3, freeze_base=1)
+    rng = np.random.default_rng(63)
+    params = random_params(cfg, rng, std=0.2)
+    prefixes = [[0.3 * rng.standard_normal((3, cfg.hidden)) for _ in range(2)] for _ in range(cfg.n_blocks)]
+    states = [rng.standard_normal((1, L, cfg.hidden)) for L in cfg.seq_lens]
+    gouts = [rng.standard_normal((1, L, cfg.hidden)) for L in cfg.seq_lens]
+    srv = O.OracleServer(cfg, params, prefixes)
+    outs = srv.forward(states)
+    gins = srv.backward(gouts)
+    gsum = [[np.zeros_like(p) for p in blk[12:]] for blk in srv.params]
+    for k in range(cfg.K):
+        s1 = O.OracleServer(cfg.with_(seq_lens=(cfg.seq_lens[k],)), params, prefixes)
+        o1 = s1.forward([states[k]])
+        g1 = s1.backward([gouts[k]])
+        np.testing.assert_allclose(o1[0], outs[k], rtol=0, atol=1e-12)
+        np.testing.assert_allclose(g1[0], gins[k], rtol=0, atol=1e-12)
+        for b in range(cfg.n_blocks):
+            for j in range(2):
+                gsum[b][j] += s1.grads[b][12 + j]
+    for b in range(cfg.n_blocks):
+        for j in range(2):
+            np.testing.assert_allclose(srv.grads[b][12 + j], gsum[b][j], rtol=1e-10, atol=1e-12)
+    w_before = [[p.copy() for p in blk] for blk in srv.params]
+    srv.step(1e-2)
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            np.testing.assert_array_equal(srv.params[b][t], w_before[b][t])
+        for t in (12, 13):
+            assert np.abs(srv.params[b][t] - w_before[b][t]).max() > 1e-3
