@@ -48,20 +48,27 @@ def workload(name: str) -> syn.ServerConfig:
 def describe(cfg: syn.ServerConfig) -> str:
     lens = sorted(set(cfg.seq_lens))
     L = f"{lens[0]}" if len(lens) == 1 else f"{min(lens)}..{max(lens)} (ragged)"
-    return (f"{cfg.name}: {cfg.n_blocks} GLM blocks, hidden {cfg.hidden}, {cfg.n_heads} heads x {cfg.head_dim}, "
-            f"FFN {cfg.ffn_hidden}, K={cfg.K} clients x {cfg.client_batch} rows x {L} tokens, T={cfg.tokens}")
+    d = (f"{cfg.name}: {cfg.n_blocks} GLM blocks, hidden {cfg.hidden}, {cfg.n_heads} heads x {cfg.head_dim}, "
+         f"FFN {cfg.ffn_hidden}, K={cfg.K} clients x {cfg.client_batch} rows x {L} tokens, T={cfg.tokens}")
+    if cfg.prefix_len:
+        d += f", P-tuning v2 prefix of {cfg.prefix_len} per block" + (", block weights frozen" if cfg.freeze_base else "")
+    return d
 
 
 def gemm_flops(cfg: syn.ServerConfig) -> float:
     """Dense contractions of one fwd+bwd: forward 2T(3H^2 + H^2 + 2HF) per block, data
-    and weight gradients the same again each."""
+    and weight gradients the same again each (no weight gradients with a frozen base)."""
     H, F, T = cfg.hidden, cfg.ffn_hidden, cfg.tokens
-    return float(cfg.n_blocks * 3 * 2 * T * (4 * H * H + 2 * H * F))
+    passes = 2 if cfg.freeze_base else 3
+    return float(cfg.n_blocks * passes * 2 * T * (4 * H * H + 2 * H * F))
 
 
 def attn_flops(cfg: syn.ServerConfig) -> float:
-    """Causal attention: 2 H L (L+1) forward and 2.5x that backward, per segment per block."""
-    return float(cfg.n_blocks * sum(7 * cfg.hidden * L * (L + 1) for L in cfg.segment_lengths))
+    """Causal attention: 2 H L (L+1) forward and 2.5x that backward, per segment per block;
+    a prefix of Lp keys adds 4 H L Lp forward (and 2.5x that backward)."""
+    Lp = cfg.prefix_len
+    return float(cfg.n_blocks * sum(3.5 * (2 * cfg.hidden * L * (L + 1) + 4 * cfg.hidden * L * Lp)
+                                    for L in cfg.segment_lengths))
 
 
 def peaks() -> dict:
@@ -223,9 +230,14 @@ def main():
                          "stack: K server replicas (one per client, averaged every --period steps), one "
                          "client-batched server, and one server taking the clients one after another")
     ap.add_argument("--period", type=int, default=50, help="averaging period of --hierarchical (steps)")
+    ap.add_argument("--ptuning", type=int, default=0, metavar="LP",
+                    help="P-tuning v2, the paper's training setting: LP prefix keys/values per block, block "
+                         "weights frozen, only the prefixes trained")
     ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
+    if args.ptuning:
+        cfg = cfg.with_(prefix_len=args.ptuning, freeze_base=1)
     if args.impl == "reference":
         run_reference(args, cfg)
         return

@@ -71,6 +71,8 @@ typedef struct {
   int32_t recompute;        /* reserved, must be 0: every activation is kept */
   float init_std;           /* N(0, init_std) for weights and biases; LN gamma = 1, beta = 0 */
   float adam_beta1, adam_beta2, adam_eps, weight_decay; /* 0.9, 0.999, 1e-8, 0 */
+  int32_t prefix_len;       /* P-tuning v2 (App. A): learnable prefix keys/values per block, 0..128 */
+  int32_t freeze_base;      /* 1: only the prefixes are trained (needs prefix_len > 0) */
 } fl_server_cfg;
 
 /* Fills *cfg with the ChatGLM-6B server defaults (26 blocks, H 4096, 32 x 128, F 16384,
@@ -80,8 +82,11 @@ void fl_server_cfg_default(fl_server_cfg* cfg);
 /* Validates cfg, allocates every device buffer (parameters, gradients, Adam moments,
  * activations for cfg->max_tokens tokens) and initialises the parameters on the
  * device from the seeded SplitMix64/Box-Muller streams: tensor t of block b uses the
- * stream keyed (seed, purpose 1, b, t); weights and biases N(0, init_std) rounded to
- * fp32, LN gamma = 1, beta = 0.  Gradients and moments start at zero, step count 0.
+ * stream keyed (seed, purpose 1, b, t); weights, biases and prefixes N(0, init_std)
+ * rounded to fp32, LN gamma = 1, beta = 0.  Gradients and moments start at zero, step 0.
+ * With prefix_len > 0 every query of block b also attends to the block's prefix keys and
+ * values (P-tuning v2, App. A); with freeze_base the backward computes no block-weight
+ * gradients and the step updates only the prefixes (the paper's training setting).
  * Errors: INVALID_ARG (null), UNSUPPORTED (shape), OOM, CUDA.  On failure *out is NULL. */
 int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_server_t* out);
 
@@ -132,7 +137,7 @@ int fl_server_set_stream(fl_server_t h, void* cuda_stream);
  * then cleared), FL_ERR_CUDA on a CUDA error, else FL_OK. */
 int fl_server_sync(fl_server_t h);
 
-/* Parameter tensor ids of a block, in arena order. */
+/* Parameter tensor ids of a block.  12 and 13 exist when cfg.prefix_len > 0. */
 enum {
   FL_T_WQKV = 0, /* [3H, H]: rows [0,H) query, [H,2H) key, [2H,3H) value; head j = rows j*hd.. */
   FL_T_BQKV,     /* [3H] */
@@ -146,6 +151,9 @@ enum {
   FL_T_LN1_B,    /* [H] */
   FL_T_LN2_G,    /* [H] */
   FL_T_LN2_B,    /* [H] */
+  FL_T_BLOCK_COUNT,              /* 12 block tensors */
+  FL_T_PREFIX_K = FL_T_BLOCK_COUNT, /* [prefix_len, H]: prefix keys (head j at column j*hd), not rotated */
+  FL_T_PREFIX_V,                 /* [prefix_len, H]: prefix values */
   FL_T_COUNT
 };
 

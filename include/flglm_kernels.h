@@ -119,20 +119,28 @@ int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, const void*
  * applied); cu_seqlens_host / cu_seqlens: host and device copies of int32 [S+1].
  * o: bf16 [T,H]; lse: fp32 [n_heads, T] (log-sum-exp of the scaled scores).
  * tile_ws: device int32 scratch of at least fl_k_attention_tiles(cu_seqlens_host, S) * 2
- * entries.  This call copies the tile list synchronously.  head_dim in {64, 128}. */
+ * entries.  This call copies the tile list synchronously.  head_dim in {64, 128}.
+ * P-tuning v2 (App. A: K' = [prefix_key : key], V' = [prefix_value : value]): with
+ * prefix_len in 1..128, prefix_k / prefix_v are bf16 [prefix_len, H] (head j at column
+ * j*head_dim), seen by every query before its causal keys; the prefix keys are not
+ * rotated.  prefix_len = 0: no prefix (the pointers are ignored). */
 int32_t fl_k_attention_tiles(const int32_t* cu_seqlens_host, int32_t S);
 int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv,
                        const int32_t* cu_seqlens_host, const int32_t* cu_seqlens, int32_t S,
-                       int32_t* tile_ws, void* o, float* lse, void* stream);
+                       int32_t* tile_ws, void* o, float* lse, const void* prefix_k, const void* prefix_v,
+                       int32_t prefix_len, void* stream);
 
 /* Attention backward: dqkv (bf16 [T, 3H]) receives dq | dk | dv.  When rope_tab != NULL
  * the inverse rotation by each token's position inside its segment is applied to dq and
  * dk (rotary_dim must be head_dim / 2), giving the gradient w.r.t. the un-rotated q, k.
+ * With a prefix, dprefix_k / dprefix_v (fp32 [prefix_len, H]) receive the ADDED gradients
+ * of the prefix summed over every segment (fp32 atomics: the summation order varies).
  * delta_ws: fp32 scratch [n_heads * T].  This call copies the tile list synchronously. */
 int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv, const void* o,
                        const float* lse, const void* dout, const int32_t* cu_seqlens_host,
                        const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,
-                       const float* rope_tab, int32_t rotary_dim, void* dqkv, void* stream);
+                       const float* rope_tab, int32_t rotary_dim, void* dqkv, const void* prefix_k,
+                       const void* prefix_v, int32_t prefix_len, float* dprefix_k, float* dprefix_v, void* stream);
 
 /* AdamW over n contiguous fp32 elements; bc1 = 1 - beta1^t, bc2 = 1 - beta2^t.
  * w_bf16 (optional) receives the rounded new weights; g is zeroed. */

@@ -91,7 +91,9 @@ template <int HD>
 __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16* __restrict__ qkv,
                                                        const int32_t* __restrict__ cu,
                                                        const uint32_t* __restrict__ tiles, bf16* __restrict__ O,
-                                                       float* __restrict__ lse, float scale_log2) {
+                                                       float* __restrict__ lse, float scale_log2,
+                                                       const bf16* __restrict__ pk, const bf16* __restrict__ pv,
+                                                       int Lp) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
   bf16* sK = sQ + AT<HD>::TILE_ELEMS;      // [2] tiles
@@ -107,9 +109,22 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
   const bf16* gK = qkv + (int64_t)seg0 * ld + H + h * HD;
   const bf16* gV = qkv + (int64_t)seg0 * ld + 2 * H + h * HD;
 
+  // key tiles: first the prefix tiles (t < npt), then the segment's causal tiles
+  const int npt = (Lp + BT - 1) / BT;
+  const int n_kv = npt + idx + 1;
+  auto load_kv = [&](int t, int buf) {
+    if (t < npt) {
+      const int k0 = t * BT;
+      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, pk + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, pv + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+    } else {
+      const int k0 = (t - npt) * BT;
+      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, gK + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, gV + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+    }
+  };
   load_tile<HD>(sQ, gQ, ld, min(BT, L - q0), tid);
-  load_tile<HD>(sK, gK, ld, min(BT, L), tid);
-  load_tile<HD>(sV, gV, ld, min(BT, L), tid);
+  load_kv(0, 0);
   cp_async_commit();
 
   float o[HD / 8][4];
@@ -117,14 +132,11 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
   for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
   uint32_t qf[HD / 16][4];
-  const int n_kv = idx + 1;
 
   for (int j = 0; j < n_kv; ++j) {
     const int buf = j & 1;
     if (j + 1 < n_kv) {
-      const int k1 = (j + 1) * BT;
-      load_tile<HD>(sK + (buf ^ 1) * AT<HD>::TILE_ELEMS, gK + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
-      load_tile<HD>(sV + (buf ^ 1) * AT<HD>::TILE_ELEMS, gV + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
+      load_kv(j + 1, buf ^ 1);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -150,18 +162,20 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
         mma_bf16_16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
       }
     }
-    const bool diag = (j == idx);
+    const bool diag = (j - npt == idx);
+    const int pvalid = j < npt ? min(BT, Lp - j * BT) : BT;  // valid prefix keys of this tile
     float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         float x = sc[nt][e] * scale_log2;
+        const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
         if (diag) {
-          const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
           const int ql = warp * 16 + (lane >> 2) + ((e >> 1) << 3);
           if (kl > ql) x = -INFINITY;
         }
+        if (kl >= pvalid) x = -INFINITY;
         sc[nt][e] = x;
         mx[e >> 1] = fmaxf(mx[e >> 1], x);
       }
@@ -272,7 +286,9 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
                                                           const int32_t* __restrict__ cu,
                                                           const uint32_t* __restrict__ tiles,
                                                           const float2* __restrict__ rope_tab, int rotary,
-                                                          float scale, bf16* __restrict__ dqkv) {
+                                                          float scale, bf16* __restrict__ dqkv,
+                                                          const bf16* __restrict__ pk, const bf16* __restrict__ pv,
+                                                          int Lp) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
   bf16* sdO = sQ + AT<HD>::TILE_ELEMS;
@@ -287,10 +303,22 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
   const int64_t ld = 3 * (int64_t)H;
   const bf16* gK = qkv + (int64_t)seg0 * ld + H + h * HD;
   const bf16* gV = qkv + (int64_t)seg0 * ld + 2 * H + h * HD;
+  const int npt = (Lp + BT - 1) / BT;
+  const int n_kv = npt + idx + 1;
+  auto load_kv = [&](int t, int buf) {
+    if (t < npt) {
+      const int k0 = t * BT;
+      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, pk + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, pv + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+    } else {
+      const int k0 = (t - npt) * BT;
+      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, gK + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, gV + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+    }
+  };
   load_tile<HD>(sQ, qkv + (int64_t)(seg0 + q0) * ld + h * HD, ld, min(BT, L - q0), tid);
   load_tile<HD>(sdO, dO + (int64_t)(seg0 + q0) * H + h * HD, H, min(BT, L - q0), tid);
-  load_tile<HD>(sK, gK, ld, min(BT, L), tid);
-  load_tile<HD>(sV, gV, ld, min(BT, L), tid);
+  load_kv(0, 0);
   cp_async_commit();
 
   const float scale_log2 = scale * LOG2E;
@@ -305,12 +333,10 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
 #pragma unroll
   for (int i = 0; i < HD / 8; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.f;
 
-  for (int j = 0; j <= idx; ++j) {
+  for (int j = 0; j < n_kv; ++j) {
     const int buf = j & 1;
-    if (j + 1 <= idx) {
-      const int k1 = (j + 1) * BT;
-      load_tile<HD>(sK + (buf ^ 1) * AT<HD>::TILE_ELEMS, gK + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
-      load_tile<HD>(sV + (buf ^ 1) * AT<HD>::TILE_ELEMS, gV + (int64_t)k1 * ld, ld, min(BT, L - k1), tid);
+    if (j + 1 < n_kv) {
+      load_kv(j + 1, buf ^ 1);
       cp_async_commit();
       cp_async_wait<1>();
     } else {
@@ -340,18 +366,20 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
         mma_bf16_16816(dp[2 * np + 1], ao, b[2], b[3]);
       }
     }
-    const bool diag = (j == idx);
+    const bool diag = (j - npt == idx);
+    const int pvalid = j < npt ? min(BT, Lp - j * BT) : BT;
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int r = e >> 1;
         float p = exp2f(sc[nt][e] * scale_log2 - lse2[r]);
+        const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
         if (diag) {
-          const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
           const int ql = warp * 16 + (lane >> 2) + (r << 3);
           if (kl > ql) p = 0.f;
         }
+        if (kl >= pvalid) p = 0.f;
         sc[nt][e] = p * (dp[nt][e] - dl[r]);  // dS
       }
     }
@@ -392,15 +420,28 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
 }
 
 // ---------------------------------------------------------------------------- dK, dV
-template <int HD>
+// One CTA per (64-key tile, head); a warp owns 16 keys.  The CTA walks the query tiles that
+// see its keys: the later tiles of its own segment (causal), or, for a prefix key tile
+// (PREFIX), a slice of every query tile of the call (the prefix is shared by all segments;
+// the slices' partial sums meet in fp32 with atomics).
+struct QTile {
+  int row0;   // global token index of the tile's first query
+  int valid;  // queries of the tile inside their segment
+  int qpos0;  // position of the first query inside its segment
+};
+
+template <int HD, bool PREFIX>
 __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const bf16* __restrict__ qkv,
                                                            const bf16* __restrict__ dO,
                                                            const float* __restrict__ lse,
                                                            const float* __restrict__ delta,
                                                            const int32_t* __restrict__ cu,
-                                                           const uint32_t* __restrict__ tiles,
+                                                           const uint32_t* __restrict__ tiles, int n_tiles,
                                                            const float2* __restrict__ rope_tab, int rotary,
-                                                           float scale, bf16* __restrict__ dqkv) {
+                                                           float scale, bf16* __restrict__ dqkv,
+                                                           const bf16* __restrict__ pk, const bf16* __restrict__ pv,
+                                                           int Lp, int nsplit, float* __restrict__ dpk,
+                                                           float* __restrict__ dpv) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sK = reinterpret_cast<bf16*>(smem);
   bf16* sV = sK + AT<HD>::TILE_ELEMS;
@@ -409,26 +450,60 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
   float* sL = reinterpret_cast<float*>(sdO + 2 * AT<HD>::TILE_ELEMS);  // [2][64] lse * log2e
   float* sD = sL + 2 * BT;                                               // [2][64] delta
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  int s, idx;
-  decode_tile(tiles[blockIdx.x], s, idx);
   const int h = blockIdx.y;
-  const int seg0 = cu[s], L = cu[s + 1] - seg0;
-  const int nq = (L + BT - 1) / BT;
-  const int kt = nq - 1 - idx;  // key tile: most work first
-  const int k0 = kt * BT;
   const int64_t ld = 3 * (int64_t)H;
-  const bf16* gQ = qkv + (int64_t)seg0 * ld + h * HD;
-  const bf16* gdO = dO + (int64_t)seg0 * H + h * HD;
-  load_tile<HD>(sK, qkv + (int64_t)(seg0 + k0) * ld + H + h * HD, ld, min(BT, L - k0), tid);
-  load_tile<HD>(sV, qkv + (int64_t)(seg0 + k0) * ld + 2 * H + h * HD, ld, min(BT, L - k0), tid);
-  load_tile<HD>(sQ, gQ + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
-  load_tile<HD>(sdO, gdO + (int64_t)k0 * H, H, min(BT, L - k0), tid);
-  cp_async_commit();
-  if (tid < BT) {
-    const int q = k0 + tid;
-    sL[tid] = q < L ? lse[(int64_t)h * T + seg0 + q] * LOG2E : 0.f;
-    sD[tid] = q < L ? delta[(int64_t)h * T + seg0 + q] : 0.f;
+  // this CTA's keys and its range of query tiles
+  int seg0 = 0, L = 0, k0, kvalid, it0, it_end;
+  if constexpr (PREFIX) {
+    const int pt = blockIdx.x / nsplit, z = blockIdx.x % nsplit;
+    k0 = pt * BT;
+    kvalid = min(BT, Lp - k0);
+    const int per = (n_tiles + nsplit - 1) / nsplit;
+    it0 = z * per;
+    it_end = min(n_tiles, it0 + per);
+    load_tile<HD>(sK, pk + (int64_t)k0 * H + h * HD, H, kvalid, tid);
+    load_tile<HD>(sV, pv + (int64_t)k0 * H + h * HD, H, kvalid, tid);
+  } else {
+    int s, idx;
+    decode_tile(tiles[blockIdx.x], s, idx);
+    seg0 = cu[s];
+    L = cu[s + 1] - seg0;
+    const int nq = (L + BT - 1) / BT;
+    const int kt = nq - 1 - idx;  // key tile: most work first
+    k0 = kt * BT;
+    kvalid = min(BT, L - k0);
+    it0 = kt;
+    it_end = nq;
+    load_tile<HD>(sK, qkv + (int64_t)(seg0 + k0) * ld + H + h * HD, ld, kvalid, tid);
+    load_tile<HD>(sV, qkv + (int64_t)(seg0 + k0) * ld + 2 * H + h * HD, ld, kvalid, tid);
   }
+  auto qtile = [&](int it) {
+    QTile q;
+    if constexpr (PREFIX) {
+      int s, idx;
+      decode_tile(tiles[it], s, idx);
+      const int sb = cu[s];
+      q.qpos0 = idx * BT;
+      q.row0 = sb + q.qpos0;
+      q.valid = min(BT, cu[s + 1] - sb - q.qpos0);
+    } else {
+      q.qpos0 = it * BT;
+      q.row0 = seg0 + q.qpos0;
+      q.valid = min(BT, L - q.qpos0);
+    }
+    return q;
+  };
+  auto load_q = [&](const QTile& q, int buf) {
+    load_tile<HD>(sQ + buf * AT<HD>::TILE_ELEMS, qkv + (int64_t)q.row0 * ld + h * HD, ld, q.valid, tid);
+    load_tile<HD>(sdO + buf * AT<HD>::TILE_ELEMS, dO + (int64_t)q.row0 * H + h * HD, H, q.valid, tid);
+    if (tid < BT) {
+      sL[buf * BT + tid] = tid < q.valid ? lse[(int64_t)h * T + q.row0 + tid] * LOG2E : 0.f;
+      sD[buf * BT + tid] = tid < q.valid ? delta[(int64_t)h * T + q.row0 + tid] : 0.f;
+    }
+  };
+  QTile cur = qtile(it0 < it_end ? it0 : 0);
+  if (it0 < it_end) load_q(cur, 0);
+  cp_async_commit();
   const float scale_log2 = scale * LOG2E;
   float dk[HD / 8][4], dv[HD / 8][4];
 #pragma unroll
@@ -436,18 +511,13 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
 #pragma unroll
     for (int e = 0; e < 4; ++e) dk[i][e] = dv[i][e] = 0.f;
 
-  for (int qt = kt; qt < nq; ++qt) {
-    const int buf = (qt - kt) & 1;
-    if (qt + 1 < nq) {
-      const int q1 = (qt + 1) * BT;
-      load_tile<HD>(sQ + (buf ^ 1) * AT<HD>::TILE_ELEMS, gQ + (int64_t)q1 * ld, ld, min(BT, L - q1), tid);
-      load_tile<HD>(sdO + (buf ^ 1) * AT<HD>::TILE_ELEMS, gdO + (int64_t)q1 * H, H, min(BT, L - q1), tid);
+  for (int it = it0; it < it_end; ++it) {
+    const int buf = (it - it0) & 1;
+    QTile nxt = cur;
+    if (it + 1 < it_end) {
+      nxt = qtile(it + 1);
+      load_q(nxt, buf ^ 1);
       cp_async_commit();
-      if (tid < BT) {
-        const int q = q1 + tid;
-        sL[(buf ^ 1) * BT + tid] = q < L ? lse[(int64_t)h * T + seg0 + q] * LOG2E : 0.f;
-        sD[(buf ^ 1) * BT + tid] = q < L ? delta[(int64_t)h * T + seg0 + q] : 0.f;
-      }
       cp_async_wait<1>();
     } else {
       cp_async_wait<0>();
@@ -486,11 +556,12 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
       for (int nt = 0; nt < 4; ++nt) {
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          const int kpos = k0 + warp * 16 + (lane >> 2) + ((e >> 1) << 3);
+          const int kl = warp * 16 + (lane >> 2) + ((e >> 1) << 3);
           const int ql = qb + nt * 8 + 2 * (lane & 3) + (e & 1);
-          const int qpos = qt * BT + ql;
+          bool ok = ql < cur.valid && kl < kvalid;
+          if constexpr (!PREFIX) ok = ok && cur.qpos0 + ql >= k0 + kl;  // causal
           float p = 0.f;
-          if (qpos >= kpos && qpos < L) p = exp2f(st[nt][e] * scale_log2 - Lq[ql]);
+          if (ok) p = exp2f(st[nt][e] * scale_log2 - Lq[ql]);
           st[nt][e] = p;
           dpt[nt][e] = p * (dpt[nt][e] - Dq[ql]);
         }
@@ -519,24 +590,38 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
       }
     }
     __syncthreads();
+    cur = nxt;
   }
 
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
-    const int kpos = k0 + warp * 16 + (lane >> 2) + 8 * r;
+    const int kl = warp * 16 + (lane >> 2) + 8 * r;
 #pragma unroll
     for (int i = 0; i < HD / 8; ++i) {
       dk[i][2 * r] *= scale;
       dk[i][2 * r + 1] *= scale;
     }
-    if (kpos < L) {
-      if (rope_tab) inverse_rope<HD>(dk, r, kpos, rope_tab, lane);
-      bf16* rk = dqkv + (int64_t)(seg0 + kpos) * ld + H + h * HD + 2 * (lane & 3);
-      bf16* rv = dqkv + (int64_t)(seg0 + kpos) * ld + 2 * H + h * HD + 2 * (lane & 3);
+    if (kl < kvalid) {
+      if constexpr (PREFIX) {  // the prefix keys enter the scores unrotated
+        float* rk = dpk + (int64_t)(k0 + kl) * H + h * HD + 2 * (lane & 3);
+        float* rv = dpv + (int64_t)(k0 + kl) * H + h * HD + 2 * (lane & 3);
 #pragma unroll
-      for (int nt = 0; nt < HD / 8; ++nt) {
-        *reinterpret_cast<uint32_t*>(rk + nt * 8) = pack_bf16x2(dk[nt][2 * r], dk[nt][2 * r + 1]);
-        *reinterpret_cast<uint32_t*>(rv + nt * 8) = pack_bf16x2(dv[nt][2 * r], dv[nt][2 * r + 1]);
+        for (int nt = 0; nt < HD / 8; ++nt) {
+          atomicAdd(rk + nt * 8, dk[nt][2 * r]);
+          atomicAdd(rk + nt * 8 + 1, dk[nt][2 * r + 1]);
+          atomicAdd(rv + nt * 8, dv[nt][2 * r]);
+          atomicAdd(rv + nt * 8 + 1, dv[nt][2 * r + 1]);
+        }
+      } else {
+        const int kpos = k0 + kl;
+        if (rope_tab) inverse_rope<HD>(dk, r, kpos, rope_tab, lane);
+        bf16* rk = dqkv + (int64_t)(seg0 + kpos) * ld + H + h * HD + 2 * (lane & 3);
+        bf16* rv = dqkv + (int64_t)(seg0 + kpos) * ld + 2 * H + h * HD + 2 * (lane & 3);
+#pragma unroll
+        for (int nt = 0; nt < HD / 8; ++nt) {
+          *reinterpret_cast<uint32_t*>(rk + nt * 8) = pack_bf16x2(dk[nt][2 * r], dk[nt][2 * r + 1]);
+          *reinterpret_cast<uint32_t*>(rv + nt * 8) = pack_bf16x2(dv[nt][2 * r], dv[nt][2 * r + 1]);
+        }
       }
     }
   }
@@ -555,8 +640,70 @@ int set_attrs() {
   if (!done) {
     FL_CUDA_TRY(cudaFuncSetAttribute(attn_fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, fwd_smem<HD>()));
     FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dq_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, dq_smem<HD>()));
-    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dkv_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, dkv_smem<HD>()));
+    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dkv_kernel<HD, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     dkv_smem<HD>()));
+    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dkv_kernel<HD, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     dkv_smem<HD>()));
     done = true;
+  }
+  return FL_OK;
+}
+
+int sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+template <int HD>
+int launch_fwd(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles, void* o,
+               float* lse, const AttnPrefix& pre, cudaStream_t st) {
+  if (int rc = set_attrs<HD>()) return rc;
+  const int H = nh * HD;
+  const float scale_log2 = (1.f / sqrtf((float)HD)) * LOG2E;
+  attn_fwd_kernel<HD><<<dim3(n_tiles, nh), 128, fwd_smem<HD>(), st>>>(
+      T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2, (const bf16*)pre.k, (const bf16*)pre.v, pre.len);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+template <int HD>
+int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, const void* dout, const int32_t* cu,
+               const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab, void* dqkv,
+               const AttnPrefix& pre, cudaStream_t st) {
+  if (int rc = set_attrs<HD>()) return rc;
+  const int H = nh * HD;
+  const float scale = 1.f / sqrtf((float)HD);
+  const int64_t pairs = (int64_t)T * nh;
+  attn_delta_kernel<<<(unsigned)((pairs * 32 + 255) / 256), 256, 0, st>>>(T, H, nh, HD, (const bf16*)o,
+                                                                          (const bf16*)dout, delta);
+  FL_CUDA_TRY(cudaGetLastError());
+  const float2* tab = reinterpret_cast<const float2*>(rope_tab);
+  const bf16* pk = (const bf16*)pre.k;
+  const bf16* pv = (const bf16*)pre.v;
+  attn_bwd_dq_kernel<HD><<<dim3(n_tiles, nh), 128, dq_smem<HD>(), st>>>(
+      T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, tab, HD / 2, scale, (bf16*)dqkv, pk, pv,
+      pre.len);
+  FL_CUDA_TRY(cudaGetLastError());
+  attn_bwd_dkv_kernel<HD, false><<<dim3(n_tiles, nh), 128, dkv_smem<HD>(), st>>>(
+      T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, (bf16*)dqkv,
+      nullptr, nullptr, 0, 1, nullptr, nullptr);
+  FL_CUDA_TRY(cudaGetLastError());
+  if (pre.len > 0) {
+    // prefix key tiles x slices of all query tiles, about two CTAs per SM in total
+    const int npt = (pre.len + BT - 1) / BT;
+    int nsplit = (2 * sms() + npt * nh - 1) / (npt * nh);
+    if (nsplit > n_tiles) nsplit = n_tiles;
+    if (nsplit < 1) nsplit = 1;
+    attn_bwd_dkv_kernel<HD, true><<<dim3(npt * nsplit, nh), 128, dkv_smem<HD>(), st>>>(
+        T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, nullptr, pk,
+        pv, pre.len, nsplit, pre.dk, pre.dv);
+    FL_CUDA_TRY(cudaGetLastError());
   }
   return FL_OK;
 }
@@ -582,55 +729,20 @@ int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles) {
 }
 
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
-                       void* o, float* lse, cudaStream_t st) {
+                       void* o, float* lse, const AttnPrefix& pre, cudaStream_t st) {
   if (n_tiles <= 0) return FL_OK;
-  const int H = nh * hd;
-  const float scale_log2 = (1.f / sqrtf((float)hd)) * LOG2E;
-  const dim3 grid(n_tiles, nh);
-  if (hd == 128) {
-    if (int rc = set_attrs<128>()) return rc;
-    attn_fwd_kernel<128><<<grid, 128, fwd_smem<128>(), st>>>(T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2);
-  } else if (hd == 64) {
-    if (int rc = set_attrs<64>()) return rc;
-    attn_fwd_kernel<64><<<grid, 128, fwd_smem<64>(), st>>>(T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2);
-  } else {
-    return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
-  }
-  FL_CUDA_TRY(cudaGetLastError());
-  return FL_OK;
+  if (hd == 128) return launch_fwd<128>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, st);
+  if (hd == 64) return launch_fwd<64>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, st);
+  return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
-                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const int32_t* /*pos*/,
-                       const float* rope_tab, int rotary, void* dqkv, cudaStream_t st) {
+                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
+                       void* dqkv, const AttnPrefix& pre, cudaStream_t st) {
   if (n_tiles <= 0) return FL_OK;
-  const int H = nh * hd;
-  const float scale = 1.f / sqrtf((float)hd);
-  const int64_t pairs = (int64_t)T * nh;
-  attn_delta_kernel<<<(unsigned)((pairs * 32 + 255) / 256), 256, 0, st>>>(T, H, nh, hd, (const bf16*)o,
-                                                                          (const bf16*)dout, delta);
-  FL_CUDA_TRY(cudaGetLastError());
-  const dim3 grid(n_tiles, nh);
-  const float2* tab = reinterpret_cast<const float2*>(rope_tab);
-  if (hd == 128) {
-    if (int rc = set_attrs<128>()) return rc;
-    attn_bwd_dq_kernel<128><<<grid, 128, dq_smem<128>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta,
-                                                              cu, tiles, tab, rotary, scale, (bf16*)dqkv);
-    FL_CUDA_TRY(cudaGetLastError());
-    attn_bwd_dkv_kernel<128><<<grid, 128, dkv_smem<128>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse,
-                                                                delta, cu, tiles, tab, rotary, scale, (bf16*)dqkv);
-  } else if (hd == 64) {
-    if (int rc = set_attrs<64>()) return rc;
-    attn_bwd_dq_kernel<64><<<grid, 128, dq_smem<64>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta,
-                                                            cu, tiles, tab, rotary, scale, (bf16*)dqkv);
-    FL_CUDA_TRY(cudaGetLastError());
-    attn_bwd_dkv_kernel<64><<<grid, 128, dkv_smem<64>(), st>>>(T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta,
-                                                              cu, tiles, tab, rotary, scale, (bf16*)dqkv);
-  } else {
-    return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
-  }
-  FL_CUDA_TRY(cudaGetLastError());
-  return FL_OK;
+  if (hd == 128) return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, st);
+  if (hd == 64) return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, st);
+  return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 
 // ====================================================================== exported kernel API
@@ -657,28 +769,46 @@ static int upload_tiles(const int32_t* cu_host, int32_t S, int32_t* tile_ws, int
 
 extern "C" int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv,
                                   const int32_t* cu_seqlens_host, const int32_t* cu_seqlens, int32_t S,
-                                  int32_t* tile_ws, void* o, float* lse, void* stream) {
+                                  int32_t* tile_ws, void* o, float* lse, const void* prefix_k, const void* prefix_v,
+                                  int32_t prefix_len, void* stream) {
   if (!qkv || !cu_seqlens_host || !cu_seqlens || !tile_ws || !o || !lse || S <= 0 || S >= 65536)
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: args");
   if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: cu_seqlens");
+  if (prefix_len < 0 || prefix_len > 128 || (prefix_len > 0 && (!prefix_k || !prefix_v)))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: prefix (length 0..128)");
   int n = 0;
   if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n)) return rc;
-  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, o, lse,
+  AttnPrefix pre;
+  pre.k = prefix_k;
+  pre.v = prefix_v;
+  pre.len = prefix_len;
+  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, o, lse, pre,
                             (cudaStream_t)stream);
 }
 
 extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv, const void* o,
                                   const float* lse, const void* dout, const int32_t* cu_seqlens_host,
                                   const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,
-                                  const float* rope_tab, int32_t rotary_dim, void* dqkv, void* stream) {
+                                  const float* rope_tab, int32_t rotary_dim, void* dqkv, const void* prefix_k,
+                                  const void* prefix_v, int32_t prefix_len, float* dprefix_k, float* dprefix_v,
+                                  void* stream) {
   if (!qkv || !o || !lse || !dout || !cu_seqlens_host || !cu_seqlens || !tile_ws || !delta_ws || !dqkv || S <= 0 ||
       S >= 65536)
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: args");
   if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: cu_seqlens");
   if (rope_tab && rotary_dim != head_dim / 2)
     return fl_internal_error(FL_ERR_UNSUPPORTED, "attention bwd: rotary_dim must be head_dim / 2");
+  if (prefix_len < 0 || prefix_len > 128 ||
+      (prefix_len > 0 && (!prefix_k || !prefix_v || !dprefix_k || !dprefix_v)))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: prefix (length 0..128, gradients required)");
   int n = 0;
   if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n)) return rc;
+  AttnPrefix pre;
+  pre.k = prefix_k;
+  pre.v = prefix_v;
+  pre.len = prefix_len;
+  pre.dk = dprefix_k;
+  pre.dv = dprefix_v;
   return fl_launch_attn_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_seqlens, (const uint32_t*)tile_ws, n, delta_ws,
-                            nullptr, rope_tab, rotary_dim, dqkv, (cudaStream_t)stream);
+                            rope_tab, dqkv, pre, (cudaStream_t)stream);
 }

@@ -52,12 +52,22 @@ int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_b
                     float beta2, float eps, float weight_decay, float bc1, float bc2, int zero_grad, cudaStream_t st);
 int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st);
 
+// P-tuning v2 prefix of one block's attention: bf16 keys/values [len, H] (head j at
+// column j*head_dim) seen by every query, and fp32 gradient accumulators (backward).
+struct AttnPrefix {
+  const void* k = nullptr;
+  const void* v = nullptr;
+  int len = 0;
+  float* dk = nullptr;
+  float* dv = nullptr;
+};
+
 // Attention on a device tile list (built by fl_launch_meta).
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
-                       int n_tiles, void* o, float* lse, cudaStream_t st);
+                       int n_tiles, void* o, float* lse, const AttnPrefix& pre, cudaStream_t st);
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
-                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const int32_t* pos,
-                       const float* rope_tab, int rotary_dim, void* dqkv, cudaStream_t st);
+                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
+                       void* dqkv, const AttnPrefix& pre, cudaStream_t st);
 
 // Host helper: builds the tile list of a packing (returns the count, -1 if over capacity).
 int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles);

@@ -97,7 +97,7 @@ struct fl_server {
   // parameter arenas
   int64_t tensor_off[FL_T_COUNT] = {};  // inside the block's matrix or vector slice
   int64_t tensor_n[FL_T_COUNT] = {};
-  int64_t mat_stride = 0, vec_stride = 0, vec_base = 0;
+  int64_t mat_stride = 0, vec_stride = 0, vec_base = 0, pre_stride = 0, pre_base = 0;
   int64_t n_params = 0;  // padded total
   float *w = nullptr, *g = nullptr, *m = nullptr, *v = nullptr;
   __nv_bfloat16* wb = nullptr;
@@ -137,8 +137,23 @@ struct fl_server {
   int64_t launches = 0;
 
   static bool is_matrix(int t) { return t == FL_T_WQKV || t == FL_T_WDENSE || t == FL_T_WUP || t == FL_T_WDOWN; }
+  static bool is_prefix(int t) { return t == FL_T_PREFIX_K || t == FL_T_PREFIX_V; }
   int64_t off(int b, int t) const {
+    if (is_prefix(t)) return pre_base + b * pre_stride + tensor_off[t];
     return is_matrix(t) ? b * mat_stride + tensor_off[t] : vec_base + b * vec_stride + tensor_off[t];
+  }
+  AttnPrefix prefix(int b, bool grads) {
+    AttnPrefix p;
+    if (cfg.prefix_len > 0) {
+      p.k = wbt(b, FL_T_PREFIX_K);
+      p.v = wbt(b, FL_T_PREFIX_V);
+      p.len = cfg.prefix_len;
+      if (grads) {
+        p.dk = gt(b, FL_T_PREFIX_K);
+        p.dv = gt(b, FL_T_PREFIX_V);
+      }
+    }
+    return p;
   }
   float* wt(int b, int t) { return w + off(b, t); }
   float* gt(int b, int t) { return g + off(b, t); }
@@ -215,6 +230,10 @@ int validate_cfg(const fl_server_cfg& c, int* rdim) {
   if (!(c.ln_eps > 0.f) || !(c.rope_base > 1.f)) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: ln_eps/rope_base");
   if (c.residual_from_ln != 0 && c.residual_from_ln != 1)
     return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: residual_from_ln must be 0 or 1");
+  if (c.prefix_len < 0 || c.prefix_len > 128) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: prefix_len in 0..128");
+  if (c.freeze_base != 0 && c.freeze_base != 1) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: freeze_base 0 or 1");
+  if (c.freeze_base && c.prefix_len == 0)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: freeze_base needs a prefix (prefix_len > 0)");
   *rdim = rd;
   return FL_OK;
 }
@@ -310,7 +329,8 @@ int block_forward(fl_server* h, int b) {
   TRY(h, run_gemm(h, g1));
   // o = causal attention within each segment
   prof_begin(h, FL_PROF_ATTN);
-  TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse, st));
+  TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse,
+                            h->prefix(b, false), st));
   prof_end(h);
   // h = alpha * (LN1(x) or x) + o Wd^T + bd, fp32; LN1(x) recomputed in fp32 in the epilogue
   fl_gemm_args g2 = gemm_fwd(T, H, H, A.o, h->wbt(b, FL_T_WDENSE), A.h, FL_EPI_BIAS_RESID);
@@ -364,15 +384,18 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   const bool glm = c.residual_from_ln != 0;
   BlockAct& A = h->act[b];
   cudaStream_t st = h->stream;
+  const bool train_base = !c.freeze_base;
   // FFN down: du = (dy W2) * gelu'(u); dW2 += dy^T g; db2 += colsum(dy)
   fl_gemm_args d1 = gemm_dgrad(T, F, H, dy, h->wbt(b, FL_T_WDOWN), h->du, FL_EPI_GELU_BWD);
   d1.aux = A.u;
   d1.ld_aux = F;
   TRY(h, run_gemm(h, d1));
-  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g)));
-  prof_begin(h, FL_PROF_OTHER);
-  TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
-  prof_end(h);
+  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g)));
+    prof_begin(h, FL_PROF_OTHER);
+    TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
+    prof_end(h);
+  }
   // FFN up: dm = du W1 (+ alpha dy), fp32; dW1 += du^T m; db1 += colsum(du)
   fl_gemm_args d2 = gemm_dgrad(T, H, F, h->du, h->wbt(b, FL_T_WUP), h->dm, glm ? FL_EPI_RESID : FL_EPI_STORE);
   d2.d_dtype = FL_DT_F32;
@@ -383,10 +406,12 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d2.alpha = al;
   }
   TRY(h, run_gemm(h, d2));
-  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m)));
-  prof_begin(h, FL_PROF_OTHER);
-  TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
-  prof_end(h);
+  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m)));
+    prof_begin(h, FL_PROF_OTHER);
+    TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
+    prof_end(h);
+  }
   // LN2 backward: dh = LN2'(dm) (+ alpha dy), bf16 and fp32
   prof_begin(h, FL_PROF_LN, 2);
   TRY(h, fl_k_layernorm_bwd(T, H, h->dm, A.h, FL_DT_F32, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dyf,
@@ -394,14 +419,16 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   prof_end(h);
   // dense: do = dh Wd; dWd += dh^T o; dbd += colsum(dh)
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
-  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)));
-  prof_begin(h, FL_PROF_OTHER);
-  TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
-  prof_end(h);
+  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)));
+    prof_begin(h, FL_PROF_OTHER);
+    TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
+    prof_end(h);
+  }
   // attention backward -> dqkv (w.r.t. the un-rotated q, k)
   prof_begin(h, FL_PROF_ATTN, 3);
   TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
-                            h->pos, h->rope_tab, h->rdim, h->dqkv, st));
+                            h->rope_tab, h->dqkv, h->prefix(b, true), st));
   prof_end(h);
   // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a; dbqkv += colsum(dqkv)
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
@@ -413,10 +440,12 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d3.alpha = al;
   }
   TRY(h, run_gemm(h, d3));
-  TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a)));
-  prof_begin(h, FL_PROF_OTHER);
-  TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
-  prof_end(h);
+  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a)));
+    prof_begin(h, FL_PROF_OTHER);
+    TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
+    prof_end(h);
+  }
   // LN1 backward: dx = LN1'(da) (+ alpha dh), bf16 and fp32
   prof_begin(h, FL_PROF_LN, 2);
   TRY(h, fl_k_layernorm_bwd(T, H, h->da, h->xs[b], FL_DT_F32, A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G),
@@ -507,18 +536,21 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
   };
 
   // parameter layout
-  const int64_t sizes[FL_T_COUNT] = {3 * H * H, 3 * H, H * H, H, F * H, F, H * F, H, H, H, H, H};
-  int64_t moff = 0, voff = 0;
+  const int64_t LpH = (int64_t)c.prefix_len * H;
+  const int64_t sizes[FL_T_COUNT] = {3 * H * H, 3 * H, H * H, H, F * H, F, H * F, H, H, H, H, H, LpH, LpH};
+  int64_t moff = 0, voff = 0, poff = 0;
   for (int t = 0; t < FL_T_COUNT; ++t) {
-    int64_t& o = fl_server::is_matrix(t) ? moff : voff;
+    int64_t& o = fl_server::is_prefix(t) ? poff : fl_server::is_matrix(t) ? moff : voff;
     h->tensor_off[t] = o;
     h->tensor_n[t] = sizes[t];
     o += (sizes[t] + 15) / 16 * 16;
   }
   h->mat_stride = moff;
   h->vec_stride = voff;
+  h->pre_stride = poff;
   h->vec_base = moff * c.n_blocks;
-  h->n_params = h->vec_base + voff * c.n_blocks;
+  h->pre_base = h->vec_base + voff * c.n_blocks;
+  h->n_params = h->pre_base + poff * c.n_blocks;
   int rc;
   if ((rc = dalloc(h, &h->w, h->n_params)) || (rc = dalloc(h, &h->g, h->n_params)) ||
       (rc = dalloc(h, &h->m, h->n_params)) || (rc = dalloc(h, &h->v, h->n_params)) ||
@@ -572,6 +604,7 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
   // seeded init: tensor t of block b from the stream (seed, purpose 1, b, t)
   for (int b = 0; b < c.n_blocks; ++b)
     for (int t = 0; t < FL_T_COUNT; ++t) {
+      if (h->tensor_n[t] == 0) continue;
       float* p = h->wt(b, t);
       if (t == FL_T_LN1_G || t == FL_T_LN2_G) rc = fl_launch_fill(h->tensor_n[t], 1.f, p, st);
       else if (t == FL_T_LN1_B || t == FL_T_LN2_B) rc = fl_launch_fill(h->tensor_n[t], 0.f, p, st);
@@ -682,10 +715,12 @@ extern "C" int fl_server_backward_step(fl_server_t h, const void* const grad_out
   h->fuse.on = false;
   if (rc) return rc;
   h->step_t = t;
-  // the bias and LayerNorm vectors: one AdamW launch over their contiguous region
+  // the bias / LayerNorm vectors and the prefixes (only the prefixes with a frozen base):
+  // one AdamW launch over their contiguous region
+  const int64_t first = c.freeze_base ? h->pre_base : h->vec_base;
   prof_begin(h, FL_PROF_ADAMW);
-  rc = fl_launch_adamw(h->n_params - h->vec_base, h->w + h->vec_base, h->g + h->vec_base, h->m + h->vec_base,
-                       h->v + h->vec_base, h->wb + h->vec_base, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
+  rc = fl_launch_adamw(h->n_params - first, h->w + first, h->g + first, h->m + first,
+                       h->v + first, h->wb + first, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
                        c.weight_decay, (float)(1.0 - std::pow((double)c.adam_beta1, (double)t)),
                        (float)(1.0 - std::pow((double)c.adam_beta2, (double)t)), 0, h->stream);
   prof_end(h);
@@ -702,9 +737,12 @@ extern "C" int fl_server_step(fl_server_t h, float lr) {
   const double bc1 = 1.0 - std::pow((double)c.adam_beta1, (double)h->step_t);
   const double bc2 = 1.0 - std::pow((double)c.adam_beta2, (double)h->step_t);
   prof_begin(h, FL_PROF_ADAMW);
-  // the gradients are not cleared here: the next backward overwrites them (grads_zero)
-  int rc = fl_launch_adamw(h->n_params, h->w, h->g, h->m, h->v, h->wb, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
-                           c.weight_decay, (float)bc1, (float)bc2, 0, h->stream);
+  // the gradients are not cleared here: the next backward overwrites them (grads_zero);
+  // with a frozen base only the prefix region is updated
+  const int64_t first = c.freeze_base ? h->pre_base : 0;
+  int rc = fl_launch_adamw(h->n_params - first, h->w + first, h->g + first, h->m + first, h->v + first, h->wb + first,
+                           lr, c.adam_beta1, c.adam_beta2, c.adam_eps, c.weight_decay, (float)bc1, (float)bc2, 0,
+                           h->stream);
   prof_end(h);
   if (rc == FL_OK) h->grads_zero = true;
   return fwd_err(h, rc);
@@ -741,12 +779,12 @@ extern "C" int fl_server_sync(fl_server_t h) {
 
 extern "C" int64_t fl_server_tensor_numel(fl_server_t h, int32_t t) {
   if (!h || t < 0 || t >= FL_T_COUNT) return -1;
-  return h->tensor_n[t];
+  return h->tensor_n[t];  // 0 for the prefix tensors when there is no prefix
 }
 
 static int check_tensor(fl_server* h, int32_t b, int32_t t, const void* p, size_t n) {
   if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "null handle");
-  if (b < 0 || b >= h->cfg.n_blocks || t < 0 || t >= FL_T_COUNT)
+  if (b < 0 || b >= h->cfg.n_blocks || t < 0 || t >= FL_T_COUNT || h->tensor_n[t] == 0)
     return set_err(h, FL_ERR_INVALID_ARG, "bad block %d / tensor %d", b, t);
   if (!p) return set_err(h, FL_ERR_INVALID_ARG, "null host buffer");
   if ((int64_t)n != h->tensor_n[t])

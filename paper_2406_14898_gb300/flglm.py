@@ -21,7 +21,9 @@ ERRORS = {-1: "FL_ERR_INVALID_ARG", -2: "FL_ERR_CAPACITY", -3: "FL_ERR_STATE", -
 
 (FL_T_WQKV, FL_T_BQKV, FL_T_WDENSE, FL_T_BDENSE, FL_T_WUP, FL_T_BUP, FL_T_WDOWN, FL_T_BDOWN,
  FL_T_LN1_G, FL_T_LN1_B, FL_T_LN2_G, FL_T_LN2_B) = range(12)
-FL_T_COUNT = 12
+FL_T_BLOCK_COUNT = 12
+FL_T_PREFIX_K, FL_T_PREFIX_V = 12, 13
+FL_T_COUNT = 14
 (FL_EPI_STORE, FL_EPI_BIAS_GELU, FL_EPI_BIAS_RESID, FL_EPI_BIAS_ROPE, FL_EPI_GELU_BWD, FL_EPI_RESID,
  FL_EPI_ACCUM_F32, FL_EPI_STORE_F32, FL_EPI_ADAMW) = range(9)
 PROF_CLASSES = ("gemm", "attention", "layernorm", "adamw", "other")
@@ -40,7 +42,8 @@ class fl_server_cfg(C.Structure):
                 ("ln_eps", C.c_float), ("residual_alpha", C.c_float), ("residual_from_ln", C.c_int32),
                 ("client_batch", C.c_int32), ("max_tokens", C.c_int32), ("max_seq_len", C.c_int32),
                 ("recompute", C.c_int32), ("init_std", C.c_float), ("adam_beta1", C.c_float),
-                ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("weight_decay", C.c_float)]
+                ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("weight_decay", C.c_float),
+                ("prefix_len", C.c_int32), ("freeze_base", C.c_int32)]
 
 
 class fl_gemm_args(C.Structure):
@@ -90,8 +93,9 @@ _SIGS = {
     "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _I32, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P]),
     "fl_k_layernorm_bwd_noalloc": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_attention_tiles": (_I32, [_P, _I32]),
-    "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P]),
-    "fl_k_attention_bwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _I32, _P, _P, _P, _I32, _P, _P]),
+    "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _I32, _P]),
+    "fl_k_attention_bwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _I32, _P, _P, _P, _I32, _P,
+                                     _P, _P, _I32, _P, _P, _P]),
     "fl_k_adamw": (C.c_int, [_I64, _P, _P, _P, _P, _P, _F, _F, _F, _F, _F, _F, _F, _P]),
     "fl_k_colsum": (C.c_int, [_I32, _I32, _P, _P, _P]),
     "fl_k_pack_clients": (C.c_int, [_I32, C.POINTER(_P), C.POINTER(_I64), _P, _I32, _P]),
@@ -165,6 +169,8 @@ def make_cfg(c, max_tokens: int, max_seq_len: int = 0) -> fl_server_cfg:
     cfg.adam_beta2 = c.adam_beta2
     cfg.adam_eps = c.adam_eps
     cfg.weight_decay = c.weight_decay
+    cfg.prefix_len = getattr(c, "prefix_len", 0)
+    cfg.freeze_base = getattr(c, "freeze_base", 0)
     return cfg
 
 
@@ -311,20 +317,24 @@ def fl_k_attention_tiles(cu_host) -> int:
     return int(lib().fl_k_attention_tiles(a.ctypes.data, a.size - 1))
 
 
-def fl_k_attention_fwd(T, n_heads, head_dim, qkv, cu_host, cu_dev, tile_ws, o, lse, stream=None):
+def fl_k_attention_fwd(T, n_heads, head_dim, qkv, cu_host, cu_dev, tile_ws, o, lse, prefix_k=None, prefix_v=None,
+                       prefix_len=0, stream=None):
     import numpy as np
     a = np.ascontiguousarray(cu_host, np.int32)
     check(lib().fl_k_attention_fwd(T, n_heads, head_dim, ptr(qkv), a.ctypes.data, ptr(cu_dev), a.size - 1,
-                                   ptr(tile_ws), ptr(o), ptr(lse), stream_ptr(stream)))
+                                   ptr(tile_ws), ptr(o), ptr(lse), ptr(prefix_k), ptr(prefix_v), prefix_len,
+                                   stream_ptr(stream)))
 
 
 def fl_k_attention_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_host, cu_dev, tile_ws, delta_ws, rope_tab,
-                       rotary_dim, dqkv, stream=None):
+                       rotary_dim, dqkv, prefix_k=None, prefix_v=None, prefix_len=0, dprefix_k=None, dprefix_v=None,
+                       stream=None):
     import numpy as np
     a = np.ascontiguousarray(cu_host, np.int32)
     check(lib().fl_k_attention_bwd(T, n_heads, head_dim, ptr(qkv), ptr(o), ptr(lse), ptr(dout), a.ctypes.data,
                                    ptr(cu_dev), a.size - 1, ptr(tile_ws), ptr(delta_ws), ptr(rope_tab), rotary_dim,
-                                   ptr(dqkv), stream_ptr(stream)))
+                                   ptr(dqkv), ptr(prefix_k), ptr(prefix_v), prefix_len, ptr(dprefix_k),
+                                   ptr(dprefix_v), stream_ptr(stream)))
 
 
 def fl_k_adamw(n, w, g, m, v, w_bf16, lr, beta1, beta2, eps, weight_decay, bc1, bc2, stream=None):

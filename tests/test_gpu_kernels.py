@@ -314,3 +314,47 @@ def test_pack_clients_bitexact(F):
     np.testing.assert_array_equal(bits(packed), want)
     for a, b in zip(back, clients):
         np.testing.assert_array_equal(bits(a), bits(b))
+
+
+@pytest.mark.parametrize("hd,Lp", [(64, 16), (128, 100)])
+def test_attention_with_prefix(F, hd, Lp):
+    """P-tuning v2 prefix (App. A): every query also sees Lp prefix keys/values (one or two
+    64-key tiles, the second partial); prefix gradients are summed over all segments."""
+    seqs = [1, 64, 100, 7, 130]
+    nh = 2
+    H = nh * hd
+    cu = np.cumsum([0] + seqs).astype(np.int32)
+    T = int(cu[-1])
+    rng = np.random.default_rng(hd + Lp)
+    qkv = rnd_bf16_f64(rng, (T, 3 * H))
+    pk = rnd_bf16_f64(rng, (Lp, H))
+    pv = rnd_bf16_f64(rng, (Lp, H))
+    do = rnd_bf16_f64(rng, (T, H))
+    dqkv_, dcu = dev_bf16(qkv), dev_i32(cu)
+    dpk_, dpv_ = dev_bf16(pk), dev_bf16(pv)
+    tiles = torch.empty(F.fl_k_attention_tiles(cu) * 2, dtype=torch.int32, device="cuda")
+    o = torch.full((T, H), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((nh, T), dtype=torch.float32, device="cuda")
+    F.fl_k_attention_fwd(T, nh, hd, dqkv_, cu, dcu, tiles, o, lse, dpk_, dpv_, Lp)
+    torch.cuda.synchronize()
+    q = qkv[:, :H].reshape(T, nh, hd)
+    k = qkv[:, H:2 * H].reshape(T, nh, hd)
+    v = qkv[:, 2 * H:].reshape(T, nh, hd)
+    ppk, ppv = pk.reshape(Lp, nh, hd), pv.reshape(Lp, nh, hd)
+    o_ref, lse_ref = O.attention_fwd(q, k, v, cu, ppk, ppv)
+    assert rel_inf(f64(o), o_ref.reshape(T, H)) < 2e-2
+    np.testing.assert_allclose(f64(lse), lse_ref, rtol=0, atol=2e-2)
+    delta = torch.empty((nh, T), dtype=torch.float32, device="cuda")
+    dq = torch.full((T, 3 * H), float("nan"), dtype=torch.bfloat16, device="cuda")
+    gpk = dev_f32(np.full((Lp, H), 0.25, np.float32))
+    gpv = torch.zeros((Lp, H), dtype=torch.float32, device="cuda")
+    F.fl_k_attention_bwd(T, nh, hd, dqkv_, o, lse, dev_bf16(do), cu, dcu, tiles, delta, None, 0, dq,
+                         dpk_, dpv_, Lp, gpk, gpv)
+    torch.cuda.synchronize()
+    dqr, dkr, dvr, dpkr, dpvr = O.attention_bwd(do.reshape(T, nh, hd), q, k, v, cu, ppk, ppv)
+    got = f64(dq)
+    assert rel_inf(got[:, :H], dqr.reshape(T, H)) < 5e-2
+    assert rel_inf(got[:, H:2 * H], dkr.reshape(T, H)) < 5e-2
+    assert rel_inf(got[:, 2 * H:], dvr.reshape(T, H)) < 5e-2
+    assert rel_inf(f64(gpk) - 0.25, dpkr.reshape(Lp, H)) < 5e-2   # accumulated onto the 0.25
+    assert rel_inf(f64(gpv), dpvr.reshape(Lp, H)) < 5e-2
