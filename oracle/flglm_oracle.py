@@ -26,6 +26,14 @@ What it computes (plain definitions, in the paper's order, float64 throughout):
   with the softmax scale 1/sqrt(d_h) of App. A (P-tuning v2 equations).
 * The optimizer of §4.1.4 (Adam, without weight decay) in the decoupled AdamW form
   with bias correction; the decay rate is a parameter that defaults to 0.
+* §4.1.1 casts every task as GLM blank infilling: a context with a mask token [M]
+  (a cloze question, or [M] appended after the text for summarisation) and an answer
+  span generated after it.  Optional per-segment GLM structure (context length c and
+  [M] position): the context attends bidirectionally within itself, the span causally
+  to the context and to its own earlier tokens; positions are two-dimensional (the
+  span takes the position of [M] and block positions 1, 2, ...), the second position
+  rotating the second half of each head.  Without it (c = 0) a segment is plainly
+  causal with positions 0..L-1.
 
 The backward is the exact chain rule of the forward, written out by hand.
 """
@@ -51,6 +59,8 @@ class Packing:
     pos: np.ndarray          # int32 [T], position of each token inside its own segment
     seg_client: np.ndarray   # int32 [S], client that owns segment s
     seg_row: np.ndarray      # int32 [S], row of that client's batch
+    ctx: Optional[np.ndarray] = None    # int32 [S], GLM context length (0: plain causal segment)
+    pos2: Optional[np.ndarray] = None   # int32 [T], GLM block position (rotates the second half)
 
     @property
     def T(self) -> int:
@@ -61,18 +71,47 @@ class Packing:
         return len(self.cu_seqlens) - 1
 
 
-def make_packing(seq_lens: Sequence[int], client_batch: int) -> Packing:
-    """Segments in client-major, then row-major order: client k row r is segment k*b + r."""
+def glm_positions(L: int, c: int, mask_pos: int):
+    """GLM's two position streams of one segment of length L with context length c and
+    the mask token at mask_pos (< c): context token t has (t, 0); span token t >= c has
+    (mask_pos, t - c + 1).  c = 0 is a plain causal segment: (t, 0)."""
+    p1 = np.arange(L, dtype=np.int32)
+    p2 = np.zeros(L, np.int32)
+    if c > 0:
+        if not 0 <= mask_pos < c <= L:
+            raise ValueError("GLM segment: need 0 <= mask_pos < context_len <= L")
+        p1[c:] = mask_pos
+        p2[c:] = np.arange(1, L - c + 1)
+    elif c < 0:
+        raise ValueError("GLM segment: negative context length")
+    return p1, p2
+
+
+def make_packing(seq_lens: Sequence[int], client_batch: int, context_lens: Optional[Sequence[int]] = None,
+                 mask_pos: Optional[Sequence[int]] = None) -> Packing:
+    """Segments in client-major, then row-major order: client k row r is segment k*b + r.
+    context_lens / mask_pos (one per segment; mask_pos defaults to the last context token,
+    the summarisation layout of §4.1.1) give every segment the GLM blank-infilling structure."""
     cu = [0]
-    pos, segc, segr = [], [], []
+    pos, pos2, segc, segr = [], [], [], []
     for k, L in enumerate(seq_lens):
         for r in range(client_batch):
+            s = len(segc)
             cu.append(cu[-1] + L)
-            pos.extend(range(L))
+            if context_lens is None:
+                pos.extend(range(L))
+            else:
+                c = int(context_lens[s])
+                mp = int(mask_pos[s]) if mask_pos is not None else c - 1
+                p1, p2 = glm_positions(L, c, mp)
+                pos.extend(p1)
+                pos2.extend(p2)
             segc.append(k)
             segr.append(r)
+    ctx = None if context_lens is None else np.array(context_lens, np.int32)
     return Packing(np.array(cu, np.int32), np.array(pos, np.int32),
-                   np.array(segc, np.int32), np.array(segr, np.int32))
+                   np.array(segc, np.int32), np.array(segr, np.int32),
+                   ctx, None if context_lens is None else np.array(pos2, np.int32))
 
 
 def pack(client_tensors: Sequence[np.ndarray]) -> np.ndarray:
@@ -140,6 +179,20 @@ def rope_rotate(x: np.ndarray, cos: np.ndarray, sin: np.ndarray, rotary_dim: int
     return out
 
 
+def rope_2d(x: np.ndarray, pk: "Packing", rotary_dim: int, base: float, inverse: bool = False):
+    """Rotary encoding of every head of x [T, nh, hd]: dims [0, rotary_dim) by the first
+    position; with GLM positions, dims [rotary_dim, 2 rotary_dim) by the block position,
+    same frequencies and pairing (ChatGLM's 2D rotary, rotary_dim = hd / 2)."""
+    cos, sin = rope_cos_sin(pk.pos, rotary_dim, base)
+    out = rope_rotate(x, cos, sin, rotary_dim, inverse)
+    if pk.pos2 is not None:
+        if 2 * rotary_dim != x.shape[-1]:
+            raise ValueError("2D rotary needs rotary_dim = head_dim / 2")
+        cos2, sin2 = rope_cos_sin(pk.pos2, rotary_dim, base)
+        out[..., rotary_dim:] = rope_rotate(out[..., rotary_dim:], cos2, sin2, rotary_dim, inverse)
+    return out
+
+
 # ----------------------------------------------------------------------------- attention
 
 
@@ -151,14 +204,24 @@ def _keys_values(k, v, pk, pv, a, b, h):
     return np.concatenate([pk[:, h], k[a:b, h]]), np.concatenate([pv[:, h], v[a:b, h]]), pk.shape[0]
 
 
-def _mask(L: int, Lp: int):
-    """Query t sees every prefix key and the keys u <= t of its own segment."""
-    return np.concatenate([np.ones((L, Lp), bool), np.tril(np.ones((L, L), bool))], axis=1)
+def _mask(L: int, Lp: int, c: int = 0):
+    """Query t sees every prefix key and the keys u of its own segment with u <= t or, in a
+    GLM segment with context length c, u < c (the context is seen by every token)."""
+    t = np.arange(L)[:, None]
+    u = np.arange(L)[None, :]
+    own = (u <= t) | (u < c)
+    return np.concatenate([np.ones((L, Lp), bool), own], axis=1)
 
 
-def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray, pk=None, pv=None):
+def _ctx(ctx, s):
+    return 0 if ctx is None else int(ctx[s])
+
+
+def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray, pk=None, pv=None,
+                  ctx=None):
     """Per segment, per head: O = softmax(Q K'^T / sqrt(d_h) + mask) V' (App. A), K' and V'
-    the optional prefix followed by the segment's causal keys.
+    the optional prefix followed by the segment's own keys (causal; with a GLM context
+    length ctx[s], the context is bidirectional).
     Returns O [T, nh, hd] and the row log-sum-exp LSE [nh, T] of the scaled scores."""
     T, nh, hd = q.shape
     scale = 1.0 / math.sqrt(hd)
@@ -172,7 +235,7 @@ def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.nd
         for h in range(nh):
             kk, vv, Lp = _keys_values(k, v, pk, pv, a, b, h)
             S = (q[a:b, h] @ kk.T) * scale
-            S = np.where(_mask(L, Lp), S, -np.inf)
+            S = np.where(_mask(L, Lp, _ctx(ctx, s)), S, -np.inf)
             m = S.max(axis=-1)
             P = np.exp(S - m[:, None])
             l = P.sum(axis=-1)
@@ -183,7 +246,7 @@ def attention_fwd(q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.nd
 
 
 def attention_bwd(do: np.ndarray, q: np.ndarray, k: np.ndarray, v: np.ndarray, cu_seqlens: np.ndarray,
-                  pk=None, pv=None):
+                  pk=None, pv=None, ctx=None):
     """Chain rule of attention_fwd: dV' = P^T dO, dP = dO V'^T, dS = P (dP - rowsum(dP P)),
     dQ = dS K' / sqrt(d_h), dK' = dS^T Q / sqrt(d_h).  With a prefix, its gradients are
     summed over every segment (the prefix is shared) and returned as dpk, dpv."""
@@ -202,7 +265,7 @@ def attention_bwd(do: np.ndarray, q: np.ndarray, k: np.ndarray, v: np.ndarray, c
         for h in range(nh):
             kk, vv, Lp = _keys_values(k, v, pk, pv, a, b, h)
             S = (q[a:b, h] @ kk.T) * scale
-            S = np.where(_mask(L, Lp), S, -np.inf)
+            S = np.where(_mask(L, Lp, _ctx(ctx, s)), S, -np.inf)
             P = np.exp(S - S.max(axis=-1, keepdims=True))
             P /= P.sum(axis=-1, keepdims=True)
             dP = do[a:b, h] @ vv.T
@@ -268,14 +331,13 @@ def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShap
     q = qkv[:, 0:H].reshape(T, nh, hd)
     k = qkv[:, H:2 * H].reshape(T, nh, hd)
     v = qkv[:, 2 * H:3 * H].reshape(T, nh, hd)
-    cos, sin = rope_cos_sin(pk.pos, sh.rotary_dim, sh.rope_base)
-    qr = rope_rotate(q, cos, sin, sh.rotary_dim)
-    kr = rope_rotate(k, cos, sin, sh.rotary_dim)
+    qr = rope_2d(q, pk, sh.rotary_dim, sh.rope_base)
+    kr = rope_2d(k, pk, sh.rotary_dim, sh.rope_base)
     ppk = ppv = None
     if prefix is not None:
         ppk = np.asarray(prefix[0], F64).reshape(-1, nh, hd)
         ppv = np.asarray(prefix[1], F64).reshape(-1, nh, hd)
-    o, lse = attention_fwd(qr, kr, v, pk.cu_seqlens, ppk, ppv)
+    o, lse = attention_fwd(qr, kr, v, pk.cu_seqlens, ppk, ppv, pk.ctx)
     o = o.reshape(T, H)
     res1 = a if sh.residual_from_ln else x
     h = sh.alpha * res1 + (o @ Wd.T + bd[None, :])
@@ -285,7 +347,7 @@ def block_fwd(P: Sequence[np.ndarray], x: np.ndarray, pk: Packing, sh: BlockShap
     res2 = m if sh.residual_from_ln else h
     y = sh.alpha * res2 + (g @ W2.T + b2[None, :])
     saved = dict(x=x, a=a, mu1=mu1, rs1=rs1, qr=qr, kr=kr, v=v, o=o, lse=lse, h=h, m=m,
-                 mu2=mu2, rs2=rs2, u=u, g=g, cos=cos, sin=sin, ppk=ppk, ppv=ppv)
+                 mu2=mu2, rs2=rs2, u=u, g=g, ppk=ppk, ppv=ppv)
     return y, saved
 
 
@@ -313,10 +375,10 @@ def block_bwd(P: Sequence[np.ndarray], sv: dict, dy: np.ndarray, pk: Packing, sh
     dWd = dh.T @ sv["o"]
     dbd = dh.sum(axis=0)
     do = (dh @ Wd).reshape(T, nh, hd)
-    res = attention_bwd(do, sv["qr"], sv["kr"], sv["v"], pk.cu_seqlens, sv["ppk"], sv["ppv"])
+    res = attention_bwd(do, sv["qr"], sv["kr"], sv["v"], pk.cu_seqlens, sv["ppk"], sv["ppv"], pk.ctx)
     dqr, dkr, dv = res[:3]
-    dq = rope_rotate(dqr, sv["cos"], sv["sin"], sh.rotary_dim, inverse=True)
-    dk = rope_rotate(dkr, sv["cos"], sv["sin"], sh.rotary_dim, inverse=True)
+    dq = rope_2d(dqr, pk, sh.rotary_dim, sh.rope_base, inverse=True)
+    dk = rope_2d(dkr, pk, sh.rotary_dim, sh.rope_base, inverse=True)
     dqkv = np.concatenate([dq.reshape(T, H), dk.reshape(T, H), dv.reshape(T, H)], axis=1)
     dWqkv = dqkv.T @ sv["a"]
     dbqkv = dqkv.sum(axis=0)
@@ -385,10 +447,12 @@ class OracleServer:
         self.t = 0
         self._pending = None
 
-    def forward(self, client_states: Sequence[np.ndarray]) -> List[np.ndarray]:
+    def forward(self, client_states: Sequence[np.ndarray], context_lens=None, mask_pos=None) -> List[np.ndarray]:
+        """context_lens / mask_pos: optional GLM structure, one entry per segment
+        (client-major, then row)."""
         seq_lens = [s.shape[1] for s in client_states]
         b = client_states[0].shape[0]
-        pk = make_packing(seq_lens, b)
+        pk = make_packing(seq_lens, b, context_lens, mask_pos)
         X = pack([np.asarray(s, F64) for s in client_states])
         base = [blk[:12] for blk in self.params]
         pre = [blk[12:14] for blk in self.params] if self.cfg.prefix_len else None

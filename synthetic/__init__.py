@@ -30,6 +30,13 @@ from this text):
     float field carries)
     ragged length k (seed 7 in the ragged workload):
         L_k = 64 + raw(key(seed, LENGTHS), k) mod 961        in [64, 1024]
+    GLM blank-infilling structure of segment s (length L >= 2; workloads with glm = 1):
+        key  = key(seed, GLM, client = s)
+        span = 1 + raw(key, 0) mod max(1, L // 4)           answer tokens, at most L/4
+        c    = L - span                                      context length
+        [M]  = c - 1 if raw(key, 1) is even (summarisation: [M] ends the context),
+               else raw(key, 1) >> 1 mod c                   (cloze: [M] inside it)
+      (L = 1: c = 1, [M] = 0)
 """
 from __future__ import annotations
 
@@ -49,6 +56,7 @@ P_WEIGHTS = 1
 P_STATES = 2
 P_GRADS = 3
 P_LENGTHS = 4
+P_GLM = 5
 
 # per-block parameter tensors, in arena order (the C library uses the same ids)
 TENSOR_NAMES = ("w_qkv", "b_qkv", "w_dense", "b_dense", "w_up", "b_up",
@@ -170,6 +178,7 @@ class ServerConfig:
     grad_std: float = 1e-3
     prefix_len: int = 0        # P-tuning v2 prefix keys/values per block (0: none)
     freeze_base: int = 0       # 1: only the prefixes are trained (P-tuning v2)
+    glm: int = 0               # 1: every segment carries a GLM blank-infilling structure
 
     @property
     def K(self) -> int:
@@ -262,6 +271,23 @@ def client_states(cfg: ServerConfig, seed: Optional[int] = None) -> List[np.ndar
 
 def client_grads(cfg: ServerConfig, seed: Optional[int] = None) -> List[np.ndarray]:
     return [client_tensor_bits(cfg, P_GRADS, k, seed) for k in range(cfg.K)]
+
+
+def glm_structure(cfg: ServerConfig, seed: Optional[int] = None):
+    """Per-segment (context length, [M] position) of a GLM workload, segments in
+    client-major then row order; see the module docstring for the recipe."""
+    seed = cfg.seed if seed is None else seed
+    ctx, mpos = [], []
+    for s, L in enumerate(cfg.segment_lengths):
+        if L < 2:
+            ctx.append(1)
+            mpos.append(0)
+            continue
+        x0, x1 = (int(v) for v in raw_u64(stream_key(seed, P_GLM, 0, 0, s), 0, 2))
+        c = L - (1 + x0 % max(1, L // 4))
+        ctx.append(c)
+        mpos.append(c - 1 if x1 % 2 == 0 else (x1 >> 1) % c)
+    return ctx, mpos
 
 
 def _glm(name, n_blocks, K, b, seq_lens, **kw) -> ServerConfig:

@@ -270,3 +270,10 @@ def test_argument_errors(F):
     assert ei.value.code == -1
     srv.sync()
     srv.close()
+
+
+@pytest.mark.parametrize("fused", [False, True], ids=["step", "backward_step"])
+def test_tiny_parity_weight_decay(F, fused):
+    """Decoupled weight decay lambda = 0.01 (the paper trains with none; the AdamW of the
+    library takes it as a parameter): the step, and the step fused into the backward."""
+    parity_case(F, syn.CONFIGS["tiny"].with_(weight_decay=0.01), fused=fused)

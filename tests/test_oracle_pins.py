@@ -530,3 +530,229 @@ def test_prefix_batching_invariant_and_frozen_step():
             np.testing.assert_array_equal(srv.params[b][t], w_before[b][t])
         for t in (12, 13):
             assert np.abs(srv.params[b][t] - w_before[b][t]).max() > 1e-3
+
+
+# ----------------------------------------------------------------------------- GLM blank infilling
+
+def glm_mask_parts(L, c):
+    """GLM's attention rule stated by parts: tokens of Part A (the context, t < c) see all
+    of Part A; tokens of Part B (the span) see Part A and the span tokens up to themselves.
+    c = 0: no Part A, the segment is plainly causal."""
+    m = np.zeros((L, L), bool)
+    for t in range(L):
+        for u in range(L):
+            if t < c:
+                m[t, u] = u < c
+            else:
+                m[t, u] = u < c or (c <= u <= t)
+    return m
+
+
+def test_glm_positions_worked_example():
+    p1, p2 = O.glm_positions(7, 4, 2)
+    assert p1.tolist() == [0, 1, 2, 3, 2, 2, 2]
+    assert p2.tolist() == [0, 0, 0, 0, 1, 2, 3]
+    p1, p2 = O.glm_positions(5, 0, 0)
+    assert p1.tolist() == [0, 1, 2, 3, 4] and p2.tolist() == [0] * 5
+    p1, p2 = O.glm_positions(3, 3, 2)      # all context: no span
+    assert p1.tolist() == [0, 1, 2] and p2.tolist() == [0, 0, 0]
+    for bad in [(4, 5, 0), (4, 2, 2), (4, -1, 0)]:
+        with pytest.raises(ValueError):
+            O.glm_positions(*bad)
+    pk = O.make_packing([4, 3], 1, context_lens=[2, 0], mask_pos=[0, 0])
+    assert pk.pos.tolist() == [0, 1, 0, 0, 0, 1, 2]
+    assert pk.pos2.tolist() == [0, 0, 1, 2, 0, 0, 0]
+    # default [M] position: the last context token (summarisation layout)
+    assert O.make_packing([4], 1, context_lens=[3]).pos.tolist() == [0, 1, 2, 2]
+
+
+@pytest.mark.parametrize("Lp", [0, 3])
+def test_glm_attention_matches_torch_sdpa(Lp):
+    """Bidirectional context + causal span, per segment, against SDPA with the mask of
+    glm_mask_parts (and every prefix key visible)."""
+    rng = np.random.default_rng(70 + Lp)
+    seq, ctx = [5, 1, 9, 6, 4], [3, 1, 0, 6, 1]
+    cu = np.cumsum([0] + seq).astype(np.int32)
+    T, nh, hd = cu[-1], 2, 8
+    q, k, v = (rng.standard_normal((T, nh, hd)) for _ in range(3))
+    pk = pv = None
+    if Lp:
+        pk, pv = (rng.standard_normal((Lp, nh, hd)) for _ in range(2))
+    o, lse = O.attention_fwd(q, k, v, cu, pk, pv, ctx=np.array(ctx))
+    for s in range(len(seq)):
+        a, b = cu[s], cu[s + 1]
+        L = b - a
+        keys = k[a:b] if not Lp else np.concatenate([pk, k[a:b]])
+        vals = v[a:b] if not Lp else np.concatenate([pv, v[a:b]])
+        tq = torch.tensor(q[a:b]).transpose(0, 1)
+        tk = torch.tensor(keys).transpose(0, 1)
+        tv = torch.tensor(vals).transpose(0, 1)
+        mask = torch.cat([torch.ones(L, Lp, dtype=torch.bool), torch.tensor(glm_mask_parts(L, ctx[s]))], 1)
+        ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv, attn_mask=mask).transpose(0, 1).numpy()
+        np.testing.assert_allclose(o[a:b], ref, rtol=0, atol=1e-12)
+        S = (torch.einsum("hid,hjd->hij", tq, tk) / math.sqrt(hd)).masked_fill(~mask, float("-inf"))
+        np.testing.assert_allclose(lse[:, a:b], torch.logsumexp(S, -1).numpy(), rtol=0, atol=1e-12)
+
+
+def test_glm_attention_special_cases():
+    """c = L is plain (non-causal) attention over the segment; c = 0 and c = 1 are the
+    causal case exactly."""
+    rng = np.random.default_rng(72)
+    seq = [7, 4]
+    cu = np.cumsum([0] + seq).astype(np.int32)
+    T, nh, hd = cu[-1], 2, 8
+    q, k, v = (rng.standard_normal((T, nh, hd)) for _ in range(3))
+    o_full, _ = O.attention_fwd(q, k, v, cu, ctx=np.array(seq))
+    for s in range(2):
+        a, b = cu[s], cu[s + 1]
+        t = [torch.tensor(z[a:b]).transpose(0, 1) for z in (q, k, v)]
+        ref = torch.nn.functional.scaled_dot_product_attention(*t, is_causal=False).transpose(0, 1).numpy()
+        np.testing.assert_allclose(o_full[a:b], ref, rtol=0, atol=1e-12)
+    o_c, l_c = O.attention_fwd(q, k, v, cu)
+    for c in (0, 1):
+        o_g, l_g = O.attention_fwd(q, k, v, cu, ctx=np.array([c, c]))
+        np.testing.assert_array_equal(o_g, o_c)
+        np.testing.assert_array_equal(l_g, l_c)
+
+
+def test_rope_2d_properties():
+    """ChatGLM's 2D rotary: the second half of each head turns by the block position with
+    the first half's frequencies; block position 0 is the identity."""
+    rng = np.random.default_rng(73)
+    hd, rd, base = 16, 8, 10000.0
+    pk = O.make_packing([9], 1, context_lens=[4], mask_pos=[1])
+    x = rng.standard_normal((9, 2, hd))
+    xr = O.rope_2d(x, pk, rd, base)
+    theta = base ** (-2.0 * np.arange(rd // 2) / rd)
+    for lo, p in ((0, pk.pos), (rd, pk.pos2)):
+        z = (x[..., lo:lo + rd // 2] + 1j * x[..., lo + rd // 2:lo + rd]) * np.exp(1j * p[:, None, None] * theta)
+        np.testing.assert_allclose(xr[..., lo:lo + rd // 2], z.real, atol=1e-13)
+        np.testing.assert_allclose(xr[..., lo + rd // 2:lo + rd], z.imag, atol=1e-13)
+    np.testing.assert_allclose(O.rope_2d(xr, pk, rd, base, inverse=True), x, atol=1e-13)
+    # no GLM structure: the 1D rotation, second half untouched
+    plain = O.make_packing([9], 1)
+    np.testing.assert_array_equal(O.rope_2d(x, plain, rd, base)[..., rd:], x[..., rd:])
+    # all block positions 0: bit-identical to the 1D rotation
+    zero2 = O.make_packing([9], 1, context_lens=[9], mask_pos=[8])
+    np.testing.assert_array_equal(O.rope_2d(x, zero2, rd, base), O.rope_2d(x, plain, rd, base))
+    # q . k depends only on the differences of both positions
+    q = rng.standard_normal((1, 1, hd))
+    kk = rng.standard_normal((1, 1, hd))
+
+    def dot(p1, p2, pp1, pp2):
+        def one(v, a, b):
+            fake = O.Packing(np.array([0, 1], np.int32), np.array([a], np.int32), np.zeros(1, np.int32),
+                             np.zeros(1, np.int32), np.array([1], np.int32), np.array([b], np.int32))
+            return O.rope_2d(v, fake, rd, base)
+        return float((one(q, p1, p2) * one(kk, pp1, pp2)).sum())
+    assert abs(dot(7, 3, 2, 1) - dot(12, 5, 7, 3)) < 1e-12
+    assert abs(dot(7, 3, 2, 1) - dot(7, 4, 2, 1)) > 1e-6   # the block position matters
+
+
+@pytest.mark.parametrize("rfl,Lp", [(1, 0), (0, 0), (1, 2)])
+def test_finite_difference_glm_gradients(rfl, Lp):
+    """Chain rule through the GLM mask and the 2D rotary (and a prefix): central
+    differences on inputs and every parameter."""
+    cfg = tiny_cfg(residual_from_ln=rfl, n_blocks=2, seq_lens=(4, 6), b=1).with_(prefix_len=Lp)
+    rng = np.random.default_rng(74 + rfl + Lp)
+    params = random_params(cfg, rng)
+    if Lp:
+        for blk in params:
+            blk.extend(0.5 * rng.standard_normal(s) for s in syn.prefix_shapes(cfg))
+    pk = O.make_packing(cfg.seq_lens, 1, context_lens=[2, 4], mask_pos=[0, 1])
+    sh = O.BlockShape.of(cfg)
+    X = rng.standard_normal((pk.T, cfg.hidden))
+    dY = rng.standard_normal((pk.T, cfg.hidden))
+    base = [blk[:12] for blk in params]
+    pre = [blk[12:] for blk in params] if Lp else None
+    Y, saved = O.stack_fwd(base, X, pk, sh, pre)
+    dX, grads = O.stack_bwd(base, saved, dY, pk, sh)
+
+    def f(pp, X_):
+        Y_, _ = O.stack_fwd([b[:12] for b in pp], X_, pk, sh, [b[12:] for b in pp] if Lp else None)
+        return float((Y_ * dY).sum())
+
+    h = 1e-5
+    irng = np.random.default_rng(98)
+
+    def check(an, perturb, n):
+        flat = an.reshape(-1)
+        scale = max(np.abs(flat).max(), 1e-8)
+        for i in irng.choice(flat.size, size=min(n, flat.size), replace=False):
+            fd = (perturb(i, +h) - perturb(i, -h)) / (2 * h)
+            assert abs(fd - flat[i]) <= 1e-6 * scale, (i, fd, flat[i], scale)
+
+    def pert_x(i, d):
+        Xp = X.copy()
+        Xp.reshape(-1)[i] += d
+        return f(params, Xp)
+    check(dX, pert_x, 60)
+    for b in range(cfg.n_blocks):
+        for t in range(len(params[b])):
+            def pert_p(i, d, b=b, t=t):
+                pp = [[p.copy() if (bb == b and tt == t) else p for tt, p in enumerate(blk)]
+                      for bb, blk in enumerate(params)]
+                pp[b][t].reshape(-1)[i] += d
+                return f(pp, X)
+            check(grads[b][t], pert_p, 20)
+
+
+def test_glm_context_is_bidirectional_and_span_causal():
+    """A later context token changes an earlier context token's output (bidirectional); a
+    span token changes neither the context nor earlier span tokens, nor another segment."""
+    cfg = tiny_cfg(n_blocks=2, seq_lens=(7, 5), b=1)
+    rng = np.random.default_rng(75)
+    params = random_params(cfg, rng)
+    pk = O.make_packing(cfg.seq_lens, 1, context_lens=[4, 2], mask_pos=[3, 0])
+    X = rng.standard_normal((pk.T, cfg.hidden))
+    Y, _ = run_stack(cfg, params, X, pk)
+    Xa = X.copy()
+    Xa[3] += 3.0 * rng.standard_normal(cfg.hidden)        # last context token of segment 0
+    Ya, _ = run_stack(cfg, params, Xa, pk)
+    assert np.abs(Ya[0] - Y[0]).max() > 1e-3
+    np.testing.assert_array_equal(Ya[7:], Y[7:])
+    Xb = X.copy()
+    Xb[5] += 3.0 * rng.standard_normal(cfg.hidden)        # second span token of segment 0
+    Yb, _ = run_stack(cfg, params, Xb, pk)
+    np.testing.assert_array_equal(Yb[:5], Y[:5])
+    assert np.abs(Yb[5:7] - Y[5:7]).max() > 1e-3
+    np.testing.assert_array_equal(Yb[7:], Y[7:])
+
+
+def test_glm_batching_invariant():
+    """§3.3 stacking with GLM segments: packed outputs and input grads equal each segment
+    alone; weight grads are the per-segment sum."""
+    cfg = tiny_cfg(n_blocks=2, seq_lens=(5, 3), b=2)
+    rng = np.random.default_rng(76)
+    params = random_params(cfg, rng, std=0.2)
+    ctx, mp = [3, 5, 1, 2], [2, 0, 0, 1]
+    states = [rng.standard_normal((2, L, cfg.hidden)) for L in cfg.seq_lens]
+    gouts = [rng.standard_normal((2, L, cfg.hidden)) for L in cfg.seq_lens]
+    srv = O.OracleServer(cfg, params)
+    outs = srv.forward(states, ctx, mp)
+    gins = srv.backward(gouts)
+    gsum = [[np.zeros_like(p) for p in blk] for blk in srv.params]
+    s = 0
+    for k in range(cfg.K):
+        for r in range(2):
+            one = O.OracleServer(cfg.with_(seq_lens=(cfg.seq_lens[k],), client_batch=1), params)
+            o1 = one.forward([states[k][r:r + 1]], [ctx[s]], [mp[s]])
+            g1 = one.backward([gouts[k][r:r + 1]])
+            np.testing.assert_array_equal(o1[0][0], outs[k][r])
+            np.testing.assert_array_equal(g1[0][0], gins[k][r])
+            for b in range(cfg.n_blocks):
+                for t in range(12):
+                    gsum[b][t] += one.grads[b][t]
+            s += 1
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            np.testing.assert_allclose(srv.grads[b][t], gsum[b][t], rtol=1e-12, atol=1e-12)
+
+
+def test_glm_structure_recipe():
+    """The synthetic GLM structure: span of 1..L/4 tokens after the context, [M] inside it."""
+    cfg = syn.CONFIGS["ragged26"]
+    ctx, mp = syn.glm_structure(cfg)
+    for L, c, m in zip(cfg.segment_lengths, ctx, mp):
+        assert 1 <= L - c <= max(1, L // 4) and 0 <= m < c
+    assert any(m == c - 1 for c, m in zip(ctx, mp)) and any(m < c - 1 for c, m in zip(ctx, mp))
