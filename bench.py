@@ -52,7 +52,18 @@ def describe(cfg: syn.ServerConfig) -> str:
          f"FFN {cfg.ffn_hidden}, K={cfg.K} clients x {cfg.client_batch} rows x {L} tokens, T={cfg.tokens}")
     if cfg.prefix_len:
         d += f", P-tuning v2 prefix of {cfg.prefix_len} per block" + (", block weights frozen" if cfg.freeze_base else "")
+    if cfg.glm:
+        d += (", GLM blank-infilling segments (bidirectional context, causal answer span of 1..L/4 tokens, "
+              "2D rotary positions)")
     return d
+
+
+def glm_args(cfg: syn.ServerConfig) -> dict:
+    """forward() keyword arguments of a workload: the GLM structure when it has one."""
+    if not cfg.glm:
+        return {}
+    ctx, mp = syn.glm_structure(cfg)
+    return {"context_lens": ctx, "mask_pos": mp}
 
 
 def gemm_flops(cfg: syn.ServerConfig) -> float:
@@ -64,11 +75,13 @@ def gemm_flops(cfg: syn.ServerConfig) -> float:
 
 
 def attn_flops(cfg: syn.ServerConfig) -> float:
-    """Causal attention: 2 H L (L+1) forward and 2.5x that backward, per segment per block;
-    a prefix of Lp keys adds 4 H L Lp forward (and 2.5x that backward)."""
+    """Attention: 4 H FLOPs per visible (query, key) pair forward and 2.5x that backward,
+    per block.  Causal: L (L+1) / 2 pairs per segment; a GLM segment with context c sees
+    c^2 + (L (L+1) - c (c+1)) / 2; a prefix of Lp keys adds L Lp."""
     Lp = cfg.prefix_len
-    return float(cfg.n_blocks * sum(3.5 * (2 * cfg.hidden * L * (L + 1) + 4 * cfg.hidden * L * Lp)
-                                    for L in cfg.segment_lengths))
+    ctx = syn.glm_structure(cfg)[0] if cfg.glm else [0] * len(cfg.segment_lengths)
+    pairs = sum(c * c + (L * (L + 1) - c * (c + 1)) / 2 + L * Lp for L, c in zip(cfg.segment_lengths, ctx))
+    return float(cfg.n_blocks * 3.5 * 4 * cfg.hidden * pairs)
 
 
 def peaks() -> dict:
@@ -155,6 +168,12 @@ class OracleSample:
         self.params = params
         self.states = [rng.standard_normal((1, L, cfg.hidden)) for _ in range(self.nseg)]
         self.grads = [1e-3 * rng.standard_normal((1, L, cfg.hidden)) for _ in range(self.nseg)]
+        # GLM workloads: the sample's segments take the GLM structure of the workload's first ones
+        self.glm = (None, None)
+        if cfg.glm:
+            ctx, mp = syn.glm_structure(cfg)
+            c = [min(x, L) for x in (ctx * self.nseg)[:self.nseg]]
+            self.glm = (c, [min(m, x - 1) if x > 0 else 0 for m, x in zip((mp * self.nseg)[:self.nseg], c)])
         n = sum(p.size for p in params[0]) // self.ADAM_FRACTION
         self.adam = [rng.standard_normal(n) * 0.02, rng.standard_normal(n) * 1e-3, np.zeros(n), np.zeros(n)]
 
@@ -162,7 +181,7 @@ class OracleSample:
         cfg, O = self.cfg, self.O
         srv = O.OracleServer(self.one, self.params)
         t0 = time.perf_counter()
-        srv.forward(self.states)
+        srv.forward(self.states, *self.glm)
         srv.backward(self.grads)
         t1 = time.perf_counter()
         w, g, m, v = self.adam
@@ -233,11 +252,16 @@ def main():
     ap.add_argument("--ptuning", type=int, default=0, metavar="LP",
                     help="P-tuning v2, the paper's training setting: LP prefix keys/values per block, block "
                          "weights frozen, only the prefixes trained")
+    ap.add_argument("--glm", action="store_true",
+                    help="GLM blank-infilling segments (the paper's task format): each segment a bidirectional "
+                         "context with a mask token and a causal answer span, GLM 2D positions")
     ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
     if args.ptuning:
         cfg = cfg.with_(prefix_len=args.ptuning, freeze_base=1)
+    if args.glm:
+        cfg = cfg.with_(glm=1)
     if args.impl == "reference":
         run_reference(args, cfg)
         return
@@ -286,8 +310,10 @@ def main():
     gins = [torch.empty_like(s) for s in states]
     torch.cuda.synchronize()
 
+    gk = glm_args(cfg)
+
     def step():
-        srv.forward(states, cfg.seq_lens, outs)
+        srv.forward(states, cfg.seq_lens, outs, **gk)
         srv.backward_step(gouts, gins, cfg.lr)
 
     def barrier():
@@ -333,7 +359,7 @@ def main():
     torch.cuda.synchronize()
     e0.record(stream)
     for _ in range(args.steps):
-        srv.forward(states, cfg.seq_lens, outs)
+        srv.forward(states, cfg.seq_lens, outs, **gk)
         srv.backward(gouts, gins)
     e1.record(stream)
     srv.sync()
@@ -359,7 +385,7 @@ def main():
             with torch.cuda.stream(stream):
                 for d, h in zip(states, h_states):
                     d.copy_(h, non_blocking=True)
-                srv.forward(states, cfg.seq_lens, outs)
+                srv.forward(states, cfg.seq_lens, outs, **gk)
                 for h, d in zip(h_outs, outs):
                     h.copy_(d, non_blocking=True)
                 for d, h in zip(gouts, h_gouts):

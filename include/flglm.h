@@ -101,6 +101,21 @@ int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_server_t* out);
 int fl_server_forward(fl_server_t h, const void* const client_states[], const int32_t seq_lens[],
                       int32_t K, void* const out_states[]);
 
+/* fl_server_forward with GLM blank-infilling segments (§4.1.1 casts every task as GLM
+ * blank infilling: a context holding a mask token [M], then the answer span).  Segment
+ * s = k * client_batch + r (client k, row r) has context_lens[s] context tokens and its
+ * [M] at mask_pos[s] (HOST int32 arrays of K * client_batch entries; mask_pos NULL = the
+ * last context token, the summarisation layout).  Context tokens attend to the whole
+ * context, span tokens to the context and causally to the span; positions are GLM's two
+ * streams: context token i has (i, 0), span token i has (mask_pos, i - c + 1); the
+ * second stream rotates dims [head_dim/2, head_dim) of q and k (needs rotary_dim =
+ * head_dim / 2).  context_lens[s] = 0 keeps segment s plainly causal.  The backward uses
+ * the same structure.  Errors: as fl_server_forward, plus INVALID_ARG when
+ * context_lens[s] > seq_len or mask_pos[s] is outside [0, context_lens[s]). */
+int fl_server_forward_glm(fl_server_t h, const void* const client_states[], const int32_t seq_lens[],
+                          int32_t K, const int32_t context_lens[], const int32_t mask_pos[],
+                          void* const out_states[]);
+
 /* Backward of the pending forward.  grad_out[k] is client k's bf16 gradient of its
  * loss w.r.t. out_states[k] (same layout); grad_in[k] receives the bf16 gradient
  * w.r.t. client_states[k].  Weight gradients are ADDED (fp32) to the gradient arena,

@@ -78,6 +78,9 @@ typedef struct {
   float* adam_v;
   float lr, beta1, beta2, eps, weight_decay;   /* FL_EPI_ADAMW hyperparameters */
   float inv_bc1, inv_bc2;                      /* 1 / (1 - beta1^t), 1 / (1 - beta2^t) */
+  const int32_t* pos2;                      /* [M] GLM block positions for BIAS_ROPE, or NULL: dims
+                                               [rotary_dim, 2*rotary_dim) of each q/k head then turn
+                                               by pos2 (2D rotary; needs rotary_dim = head_dim/2) */
 } fl_gemm_args;
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);
@@ -123,24 +126,35 @@ int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, const void*
  * P-tuning v2 (App. A: K' = [prefix_key : key], V' = [prefix_value : value]): with
  * prefix_len in 1..128, prefix_k / prefix_v are bf16 [prefix_len, H] (head j at column
  * j*head_dim), seen by every query before its causal keys; the prefix keys are not
- * rotated.  prefix_len = 0: no prefix (the pointers are ignored). */
+ * rotated.  prefix_len = 0: no prefix (the pointers are ignored).
+ * GLM blank infilling (§4.1.1: each task is a context holding a mask token followed by
+ * the generated answer span): context_lens, device int32 [S] or NULL, gives segment s a
+ * context of context_lens[s] tokens (clamped to [0, L_s]); query t then sees the keys
+ * u <= max(t, context_lens[s] - 1) of its segment (bidirectional context, causal span).
+ * NULL or 0: plainly causal. */
 int32_t fl_k_attention_tiles(const int32_t* cu_seqlens_host, int32_t S);
 int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv,
                        const int32_t* cu_seqlens_host, const int32_t* cu_seqlens, int32_t S,
                        int32_t* tile_ws, void* o, float* lse, const void* prefix_k, const void* prefix_v,
-                       int32_t prefix_len, void* stream);
+                       int32_t prefix_len, const int32_t* context_lens, void* stream);
 
 /* Attention backward: dqkv (bf16 [T, 3H]) receives dq | dk | dv.  When rope_tab != NULL
  * the inverse rotation by each token's position inside its segment is applied to dq and
  * dk (rotary_dim must be head_dim / 2), giving the gradient w.r.t. the un-rotated q, k.
  * With a prefix, dprefix_k / dprefix_v (fp32 [prefix_len, H]) receive the ADDED gradients
  * of the prefix summed over every segment (fp32 atomics: the summation order varies).
- * delta_ws: fp32 scratch [n_heads * T].  This call copies the tile list synchronously. */
+ * delta_ws: fp32 scratch [n_heads * T].  This call copies the tile list synchronously.
+ * context_lens: as in the forward.  positions / block_positions: device int32 [T] or NULL;
+ * the inverse rotation of dims [0, head_dim/2) uses positions[t] (NULL: the index inside
+ * the segment) and, when block_positions != NULL, dims [head_dim/2, head_dim) turn back by
+ * block_positions[t] (GLM 2D rotary).  Every position must be below the rows of rope_tab. */
 int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv, const void* o,
                        const float* lse, const void* dout, const int32_t* cu_seqlens_host,
                        const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,
                        const float* rope_tab, int32_t rotary_dim, void* dqkv, const void* prefix_k,
-                       const void* prefix_v, int32_t prefix_len, float* dprefix_k, float* dprefix_v, void* stream);
+                       const void* prefix_v, int32_t prefix_len, float* dprefix_k, float* dprefix_v,
+                       const int32_t* context_lens, const int32_t* positions, const int32_t* block_positions,
+                       void* stream);
 
 /* AdamW over n contiguous fp32 elements; bc1 = 1 - beta1^t, bc2 = 1 - beta2^t.
  * w_bf16 (optional) receives the rounded new weights; g is zeroed. */

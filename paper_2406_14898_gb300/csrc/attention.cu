@@ -1,6 +1,8 @@
 // Varlen causal attention over packed client segments (App. A: softmax(Q K^T / sqrt(d_h)) V),
 // each client row attending only to earlier tokens of its own segment (§3.3 stacks
-// clients; it does not mix them).
+// clients; it does not mix them).  A segment may carry a GLM blank-infilling structure
+// (§4.1.1): with context length c, query t sees the keys u <= max(t, c - 1), i.e. the
+// context is bidirectional and the answer span causal; c = 0 is the plain causal case.
 //
 // Forward: one CTA per (64-query tile, head); online softmax over 64-key tiles with
 // cp.async double buffering and bf16 mma.sync m16n8k16 (fp32 accumulate).  Saves O (bf16)
@@ -93,7 +95,7 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
                                                        const uint32_t* __restrict__ tiles, bf16* __restrict__ O,
                                                        float* __restrict__ lse, float scale_log2,
                                                        const bf16* __restrict__ pk, const bf16* __restrict__ pv,
-                                                       int Lp) {
+                                                       int Lp, const int32_t* __restrict__ ctxs) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
   bf16* sK = sQ + AT<HD>::TILE_ELEMS;      // [2] tiles
@@ -109,9 +111,12 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
   const bf16* gK = qkv + (int64_t)seg0 * ld + H + h * HD;
   const bf16* gV = qkv + (int64_t)seg0 * ld + 2 * H + h * HD;
 
-  // key tiles: first the prefix tiles (t < npt), then the segment's causal tiles
+  // key tiles: first the prefix tiles (t < npt), then the segment's tiles up to the last
+  // key any query of this tile sees (the diagonal, or the end of the GLM context)
   const int npt = (Lp + BT - 1) / BT;
-  const int n_kv = npt + idx + 1;
+  const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;  // last context key, -1 without a context
+  const int n_kv = npt + max(idx, clast >= 0 ? clast / BT : 0) + 1;
+  const int qlim0 = max(q0, clast);              // smallest key limit among the tile's queries
   auto load_kv = [&](int t, int buf) {
     if (t < npt) {
       const int k0 = t * BT;
@@ -162,7 +167,8 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
         mma_bf16_16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
       }
     }
-    const bool diag = (j - npt == idx);
+    const int kb = (j - npt) * BT;  // first key of a segment tile
+    const bool need_mask = j >= npt && kb + BT - 1 > qlim0;
     const int pvalid = j < npt ? min(BT, Lp - j * BT) : BT;  // valid prefix keys of this tile
     float mx[2] = {-INFINITY, -INFINITY};
 #pragma unroll
@@ -171,9 +177,9 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
       for (int e = 0; e < 4; ++e) {
         float x = sc[nt][e] * scale_log2;
         const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
-        if (diag) {
+        if (need_mask) {
           const int ql = warp * 16 + (lane >> 2) + ((e >> 1) << 3);
-          if (kl > ql) x = -INFINITY;
+          if (kb + kl > max(q0 + ql, clast)) x = -INFINITY;
         }
         if (kl >= pvalid) x = -INFINITY;
         sc[nt][e] = x;
@@ -256,10 +262,11 @@ __global__ void attn_delta_kernel(int T, int H, int nh, int hd, const bf16* __re
 }
 
 // Inverse rotary rotation of an accumulator fragment: the thread holds, for n-tile nt,
-// dims 8 nt + 2 (lane & 3) + {0, 1} of row r (elements 2r, 2r+1).  The rotary dims are
-// [0, HD/2) (half of each head), so the partner of dim i < HD/4 is i + HD/4, which lives
-// in n-tile nt + HD/32 of the same thread.
-template <int HD>
+// dims 8 nt + 2 (lane & 3) + {0, 1} of row r (elements 2r, 2r+1).  A rotary region is
+// half a head (HD/2 dims starting at n-tile NT0: 0 for the first position, HD/16 for the
+// GLM block position), so the partner of region dim i < HD/4 is i + HD/4, which lives in
+// n-tile nt + HD/32 of the same thread.
+template <int HD, int NT0>
 FL_DEV void inverse_rope(float (&acc)[HD / 8][4], int r, int pos, const float2* __restrict__ tab, int lane) {
   constexpr int HALF = HD / 4;
   constexpr int NTP = HALF / 8;
@@ -270,11 +277,20 @@ FL_DEV void inverse_rope(float (&acc)[HD / 8][4], int r, int pos, const float2* 
     for (int e = 0; e < 2; ++e) {
       const int i = nt * 8 + 2 * (lane & 3) + e;
       const float2 cs = __ldg(tr + i);
-      const float x1 = acc[nt][2 * r + e], x2 = acc[nt + NTP][2 * r + e];
-      acc[nt][2 * r + e] = x1 * cs.x + x2 * cs.y;
-      acc[nt + NTP][2 * r + e] = x2 * cs.x - x1 * cs.y;
+      const float x1 = acc[NT0 + nt][2 * r + e], x2 = acc[NT0 + nt + NTP][2 * r + e];
+      acc[NT0 + nt][2 * r + e] = x1 * cs.x + x2 * cs.y;
+      acc[NT0 + nt + NTP][2 * r + e] = x2 * cs.x - x1 * cs.y;
     }
   }
+}
+
+// Both rotary regions of a row at segment index i (global token index t): the first by
+// the token's position (i without GLM positions), the second by its block position.
+template <int HD>
+FL_DEV void inverse_rope_2d(float (&acc)[HD / 8][4], int r, int i, int64_t t, const float2* __restrict__ tab,
+                            const int32_t* __restrict__ gpos, const int32_t* __restrict__ gpos2, int lane) {
+  inverse_rope<HD, 0>(acc, r, gpos ? __ldg(gpos + t) : i, tab, lane);
+  if (gpos2) inverse_rope<HD, HD / 16>(acc, r, __ldg(gpos2 + t), tab, lane);
 }
 
 // ---------------------------------------------------------------------------- dQ
@@ -288,7 +304,9 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
                                                           const float2* __restrict__ rope_tab, int rotary,
                                                           float scale, bf16* __restrict__ dqkv,
                                                           const bf16* __restrict__ pk, const bf16* __restrict__ pv,
-                                                          int Lp) {
+                                                          int Lp, const int32_t* __restrict__ ctxs,
+                                                          const int32_t* __restrict__ gpos,
+                                                          const int32_t* __restrict__ gpos2) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
   bf16* sdO = sQ + AT<HD>::TILE_ELEMS;
@@ -304,7 +322,9 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
   const bf16* gK = qkv + (int64_t)seg0 * ld + H + h * HD;
   const bf16* gV = qkv + (int64_t)seg0 * ld + 2 * H + h * HD;
   const int npt = (Lp + BT - 1) / BT;
-  const int n_kv = npt + idx + 1;
+  const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
+  const int n_kv = npt + max(idx, clast >= 0 ? clast / BT : 0) + 1;
+  const int qlim0 = max(q0, clast);
   auto load_kv = [&](int t, int buf) {
     if (t < npt) {
       const int k0 = t * BT;
@@ -366,7 +386,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
         mma_bf16_16816(dp[2 * np + 1], ao, b[2], b[3]);
       }
     }
-    const bool diag = (j - npt == idx);
+    const int kb = (j - npt) * BT;
+    const bool need_mask = j >= npt && kb + BT - 1 > qlim0;
     const int pvalid = j < npt ? min(BT, Lp - j * BT) : BT;
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
@@ -375,9 +396,9 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
         const int r = e >> 1;
         float p = exp2f(sc[nt][e] * scale_log2 - lse2[r]);
         const int kl = nt * 8 + 2 * (lane & 3) + (e & 1);
-        if (diag) {
+        if (need_mask) {
           const int ql = warp * 16 + (lane >> 2) + (r << 3);
-          if (kl > ql) p = 0.f;
+          if (kb + kl > max(q0 + ql, clast)) p = 0.f;
         }
         if (kl >= pvalid) p = 0.f;
         sc[nt][e] = p * (dp[nt][e] - dl[r]);  // dS
@@ -410,7 +431,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
       dq[i][2 * r + 1] *= scale;
     }
     if (q < L) {
-      if (rope_tab) inverse_rope<HD>(dq, r, q, rope_tab, lane);
+      if (rope_tab) inverse_rope_2d<HD>(dq, r, q, seg0 + q, rope_tab, gpos, gpos2, lane);
       bf16* row = dqkv + (int64_t)(seg0 + q) * ld + h * HD + 2 * (lane & 3);
 #pragma unroll
       for (int nt = 0; nt < HD / 8; ++nt)
@@ -441,7 +462,9 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
                                                            float scale, bf16* __restrict__ dqkv,
                                                            const bf16* __restrict__ pk, const bf16* __restrict__ pv,
                                                            int Lp, int nsplit, float* __restrict__ dpk,
-                                                           float* __restrict__ dpv) {
+                                                           float* __restrict__ dpv, const int32_t* __restrict__ ctxs,
+                                                           const int32_t* __restrict__ gpos,
+                                                           const int32_t* __restrict__ gpos2) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sK = reinterpret_cast<bf16*>(smem);
   bf16* sV = sK + AT<HD>::TILE_ELEMS;
@@ -453,7 +476,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
   const int h = blockIdx.y;
   const int64_t ld = 3 * (int64_t)H;
   // this CTA's keys and its range of query tiles
-  int seg0 = 0, L = 0, k0, kvalid, it0, it_end;
+  int seg0 = 0, L = 0, k0, kvalid, it0, it_end, clast = -1;
   if constexpr (PREFIX) {
     const int pt = blockIdx.x / nsplit, z = blockIdx.x % nsplit;
     k0 = pt * BT;
@@ -472,7 +495,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
     const int kt = nq - 1 - idx;  // key tile: most work first
     k0 = kt * BT;
     kvalid = min(BT, L - k0);
-    it0 = kt;
+    clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
+    it0 = k0 <= clast ? 0 : kt;  // a tile holding context keys is seen by every query
     it_end = nq;
     load_tile<HD>(sK, qkv + (int64_t)(seg0 + k0) * ld + H + h * HD, ld, kvalid, tid);
     load_tile<HD>(sV, qkv + (int64_t)(seg0 + k0) * ld + 2 * H + h * HD, ld, kvalid, tid);
@@ -559,7 +583,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
           const int kl = warp * 16 + (lane >> 2) + ((e >> 1) << 3);
           const int ql = qb + nt * 8 + 2 * (lane & 3) + (e & 1);
           bool ok = ql < cur.valid && kl < kvalid;
-          if constexpr (!PREFIX) ok = ok && cur.qpos0 + ql >= k0 + kl;  // causal
+          if constexpr (!PREFIX) ok = ok && k0 + kl <= max(cur.qpos0 + ql, clast);  // causal / GLM context
           float p = 0.f;
           if (ok) p = exp2f(st[nt][e] * scale_log2 - Lq[ql]);
           st[nt][e] = p;
@@ -614,7 +638,7 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
         }
       } else {
         const int kpos = k0 + kl;
-        if (rope_tab) inverse_rope<HD>(dk, r, kpos, rope_tab, lane);
+        if (rope_tab) inverse_rope_2d<HD>(dk, r, kpos, seg0 + kpos, rope_tab, gpos, gpos2, lane);
         bf16* rk = dqkv + (int64_t)(seg0 + kpos) * ld + H + h * HD + 2 * (lane & 3);
         bf16* rv = dqkv + (int64_t)(seg0 + kpos) * ld + 2 * H + h * HD + 2 * (lane & 3);
 #pragma unroll
@@ -662,12 +686,13 @@ int sms() {
 
 template <int HD>
 int launch_fwd(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles, void* o,
-               float* lse, const AttnPrefix& pre, cudaStream_t st) {
+               float* lse, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
   if (int rc = set_attrs<HD>()) return rc;
   const int H = nh * HD;
   const float scale_log2 = (1.f / sqrtf((float)HD)) * LOG2E;
   attn_fwd_kernel<HD><<<dim3(n_tiles, nh), 128, fwd_smem<HD>(), st>>>(
-      T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2, (const bf16*)pre.k, (const bf16*)pre.v, pre.len);
+      T, H, (const bf16*)qkv, cu, tiles, (bf16*)o, lse, scale_log2, (const bf16*)pre.k, (const bf16*)pre.v, pre.len,
+      glm.ctx);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
@@ -675,7 +700,7 @@ int launch_fwd(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t
 template <int HD>
 int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, const void* dout, const int32_t* cu,
                const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab, void* dqkv,
-               const AttnPrefix& pre, cudaStream_t st) {
+               const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
   if (int rc = set_attrs<HD>()) return rc;
   const int H = nh * HD;
   const float scale = 1.f / sqrtf((float)HD);
@@ -688,11 +713,11 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
   const bf16* pv = (const bf16*)pre.v;
   attn_bwd_dq_kernel<HD><<<dim3(n_tiles, nh), 128, dq_smem<HD>(), st>>>(
       T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, tab, HD / 2, scale, (bf16*)dqkv, pk, pv,
-      pre.len);
+      pre.len, glm.ctx, glm.pos, glm.pos2);
   FL_CUDA_TRY(cudaGetLastError());
   attn_bwd_dkv_kernel<HD, false><<<dim3(n_tiles, nh), 128, dkv_smem<HD>(), st>>>(
       T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, (bf16*)dqkv,
-      nullptr, nullptr, 0, 1, nullptr, nullptr);
+      nullptr, nullptr, 0, 1, nullptr, nullptr, glm.ctx, glm.pos, glm.pos2);
   FL_CUDA_TRY(cudaGetLastError());
   if (pre.len > 0) {
     // prefix key tiles x slices of all query tiles, about two CTAs per SM in total
@@ -702,7 +727,7 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
     if (nsplit < 1) nsplit = 1;
     attn_bwd_dkv_kernel<HD, true><<<dim3(npt * nsplit, nh), 128, dkv_smem<HD>(), st>>>(
         T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, nullptr, pk,
-        pv, pre.len, nsplit, pre.dk, pre.dv);
+        pv, pre.len, nsplit, pre.dk, pre.dv, nullptr, nullptr, nullptr);
     FL_CUDA_TRY(cudaGetLastError());
   }
   return FL_OK;
@@ -729,19 +754,21 @@ int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles) {
 }
 
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
-                       void* o, float* lse, const AttnPrefix& pre, cudaStream_t st) {
+                       void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
   if (n_tiles <= 0) return FL_OK;
-  if (hd == 128) return launch_fwd<128>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, st);
-  if (hd == 64) return launch_fwd<64>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, st);
+  if (hd == 128) return launch_fwd<128>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, st);
+  if (hd == 64) return launch_fwd<64>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
-                       void* dqkv, const AttnPrefix& pre, cudaStream_t st) {
+                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
   if (n_tiles <= 0) return FL_OK;
-  if (hd == 128) return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, st);
-  if (hd == 64) return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, st);
+  if (hd == 128)
+    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, st);
+  if (hd == 64)
+    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 
@@ -770,7 +797,7 @@ static int upload_tiles(const int32_t* cu_host, int32_t S, int32_t* tile_ws, int
 extern "C" int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv,
                                   const int32_t* cu_seqlens_host, const int32_t* cu_seqlens, int32_t S,
                                   int32_t* tile_ws, void* o, float* lse, const void* prefix_k, const void* prefix_v,
-                                  int32_t prefix_len, void* stream) {
+                                  int32_t prefix_len, const int32_t* context_lens, void* stream) {
   if (!qkv || !cu_seqlens_host || !cu_seqlens || !tile_ws || !o || !lse || S <= 0 || S >= 65536)
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: args");
   if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: cu_seqlens");
@@ -782,7 +809,9 @@ extern "C" int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   pre.k = prefix_k;
   pre.v = prefix_v;
   pre.len = prefix_len;
-  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, o, lse, pre,
+  AttnGlm glm;
+  glm.ctx = context_lens;
+  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, o, lse, pre, glm,
                             (cudaStream_t)stream);
 }
 
@@ -791,7 +820,8 @@ extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, 
                                   const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,
                                   const float* rope_tab, int32_t rotary_dim, void* dqkv, const void* prefix_k,
                                   const void* prefix_v, int32_t prefix_len, float* dprefix_k, float* dprefix_v,
-                                  void* stream) {
+                                  const int32_t* context_lens, const int32_t* positions,
+                                  const int32_t* block_positions, void* stream) {
   if (!qkv || !o || !lse || !dout || !cu_seqlens_host || !cu_seqlens || !tile_ws || !delta_ws || !dqkv || S <= 0 ||
       S >= 65536)
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: args");
@@ -809,6 +839,10 @@ extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   pre.len = prefix_len;
   pre.dk = dprefix_k;
   pre.dv = dprefix_v;
+  AttnGlm glm;
+  glm.ctx = context_lens;
+  glm.pos = positions;
+  glm.pos2 = block_positions;
   return fl_launch_attn_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_seqlens, (const uint32_t*)tile_ws, n, delta_ws,
-                            rope_tab, dqkv, pre, (cudaStream_t)stream);
+                            rope_tab, dqkv, pre, glm, (cudaStream_t)stream);
 }

@@ -71,6 +71,10 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
     if (!a->pos || !a->rope_tab || a->head_dim <= 0 || a->head_dim % 64 ||
         !(a->rotary_dim == 32 || a->rotary_dim == 64) || a->rotary_dim > a->head_dim)
       return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: RoPE epilogue arguments");
+    if (a->pos2 && 2 * a->rotary_dim != a->head_dim)
+      return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: 2D rotary needs rotary_dim = head_dim / 2");
+  } else if (a->pos2) {
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: block positions only with the RoPE epilogue");
   }
   if (a->bias && !aligned16(a->bias)) return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: bias alignment");
 
@@ -85,6 +89,7 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   e.D = a->D;
   e.ldd = a->ldd;
   e.pos = a->pos;
+  e.pos2 = a->pos2;
   e.rope_tab = reinterpret_cast<const float2*>(a->rope_tab);
   e.rope_cols = 2 * a->n_heads * a->head_dim;
   e.head_dim = a->head_dim > 0 ? a->head_dim : 64;

@@ -57,6 +57,7 @@ struct Epi {
   void* D;
   int64_t ldd;
   const int32_t* pos;
+  const int32_t* pos2;     // GLM block positions (second rotary half) or null
   const float2* rope_tab;  // [pos][rotary_dim/2]
   int rope_cols;           // 2*H: columns that hold q and k
   int head_dim, rotary_dim;
@@ -105,13 +106,20 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
     lng = ld_quad(e.ln_gamma + n);
     lnb = ld_quad(e.ln_beta + n);
   }
-  // RoPE: this chunk starts a head and holds its rotary dims [0, rotary_dim)
-  const bool rope = FAM == FAM_ROPE && n0 < e.rope_cols && (n0 % e.head_dim) == 0;
+  // RoPE: a chunk of q/k columns that holds rotary dims.  Dims [0, rotary_dim) of a head
+  // turn by pos; with GLM block positions, dims [rotary_dim, 2 rotary_dim) turn by pos2
+  // (same frequencies and pairing).  Each rotary region is 32 or 64 columns aligned inside
+  // the 64-column chunk, so a column's partner is pair_xor lanes away.
+  const int hoff = n0 % e.head_dim;
+  const bool rope = FAM == FAM_ROPE && n0 < e.rope_cols && (hoff == 0 || e.pos2 != nullptr);
   const int half = e.rotary_dim >> 1;
   const int pair_xor = half >> 2;  // lane distance of the partner columns (8 or 4)
   const int col = 4 * cl;
-  const bool rotated = rope && col < 2 * half;
-  const bool first = col < half;
+  const int region = (hoff + col) / e.rotary_dim;  // 0: rotated by pos, 1: by pos2
+  const int rcol = hoff + col - region * e.rotary_dim;
+  const bool rotated = rope && (region == 0 || (region == 1 && e.pos2 != nullptr));
+  const int32_t* rpos_src = region == 0 ? e.pos : e.pos2;
+  const bool first = rcol < half;
   const bool gelu_bwd = FAM == FAM_GELU && e.mode == FL_EPI_GELU_BWD;
   const bool accum = FAM == FAM_PLAIN && e.mode == FL_EPI_ACCUM_F32;
   const bool out_f32 = e.mode == FL_EPI_STORE_F32 || e.d_f32;
@@ -146,7 +154,7 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
         } else {
           if (gelu_bwd) aux[i] = ld_quad(e.aux + (int64_t)m * e.ld_aux + n);
           if (accum) aux[i] = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(e.D) + off);
-          if (FAM == FAM_ROPE && rotated) rpos[i] = __ldg(e.pos + m);
+          if (FAM == FAM_ROPE && rotated) rpos[i] = __ldg(rpos_src + m);
         }
       }
     }
@@ -160,7 +168,7 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
 #pragma unroll
         for (int q = 0; q < 4; ++q) p[q] = __shfl_xor_sync(0xffffffffu, y[q], pair_xor);
         if (rotated && rr < rows) {
-          const int ii = first ? col : col - half;
+          const int ii = first ? rcol : rcol - half;
           const float2* tab = e.rope_tab + (int64_t)rpos[i] * half + ii;
 #pragma unroll
           for (int q = 0; q < 4; ++q) {

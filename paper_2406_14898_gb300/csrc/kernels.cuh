@@ -28,11 +28,16 @@ struct CopyTable {
 // Packing metadata of one call, passed by value to the metadata kernel.
 // tiles[i] = segment << 16 | tile index inside the segment, ordered by decreasing tile
 // index (the longest causal rows first).
+// With glm = 1 every segment s carries a GLM blank-infilling structure: context length
+// ctx[s] (0: plain causal segment) and mask-token position mpos[s] < ctx[s].
 struct MetaArgs {
   int S;
   int n_tiles;
+  int glm;
   int32_t cu[FL_MAX_SEGS + 1];
   uint32_t tiles[FL_MAX_TILES];
+  int32_t ctx[FL_MAX_SEGS];
+  int32_t mpos[FL_MAX_SEGS];
 };
 
 int fl_launch_copy_clients(const CopyTable& tab, cudaStream_t st);
@@ -45,7 +50,11 @@ struct ReplicaTable {
   void* wb[FL_MAX_REPLICAS];
 };
 int fl_launch_average(const ReplicaTable& t, int64_t n, cudaStream_t st);
-int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st);
+// Writes cu_seqlens, the tile list, per-token positions (and, when pos2 != NULL, the GLM
+// block positions and, when ctx != NULL, the per-segment context lengths; both zero
+// without glm).
+int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, int32_t* pos2, int32_t* ctx,
+                   cudaStream_t st);
 int fl_launch_normal_init(int64_t n, uint64_t key, double mean, double std_, float* out, cudaStream_t st);
 int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st);
 int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
@@ -62,12 +71,21 @@ struct AttnPrefix {
   float* dv = nullptr;
 };
 
+// GLM blank-infilling structure of a call (all NULL: plain causal segments, positions =
+// index inside the segment, second rotary half not rotated).
+struct AttnGlm {
+  const int32_t* ctx = nullptr;   // [S] context length per segment (key u visible to query t iff u <= max(t, ctx-1))
+  const int32_t* pos = nullptr;   // [T] first position (inverse rotary of dims [0, hd/2))
+  const int32_t* pos2 = nullptr;  // [T] block position (inverse rotary of dims [hd/2, hd))
+};
+
 // Attention on a device tile list (built by fl_launch_meta).
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
-                       int n_tiles, void* o, float* lse, const AttnPrefix& pre, cudaStream_t st);
+                       int n_tiles, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm,
+                       cudaStream_t st);
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
-                       void* dqkv, const AttnPrefix& pre, cudaStream_t st);
+                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st);
 
 // Host helper: builds the tile list of a packing (returns the count, -1 if over capacity).
 int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles);

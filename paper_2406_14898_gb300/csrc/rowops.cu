@@ -356,13 +356,17 @@ __global__ void copy_clients_kernel(CopyTable tab) {
 }
 
 // ------------------------------------------------------------------ packing metadata
+// GLM positions of token i of a segment with context length c and mask position mp:
+// (i, 0) in the context (or in a plain causal segment, c = 0), (mp, i - c + 1) in the span.
 __global__ void meta_kernel(MetaArgs a, int32_t* __restrict__ cu, int32_t* __restrict__ pos,
-                            uint32_t* __restrict__ tiles) {
+                            uint32_t* __restrict__ tiles, int32_t* __restrict__ pos2, int32_t* __restrict__ ctx) {
   const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t nth = (int64_t)gridDim.x * blockDim.x;
   const int T = a.cu[a.S];
   for (int64_t i = tid; i <= a.S; i += nth) cu[i] = a.cu[i];
   for (int64_t i = tid; i < a.n_tiles; i += nth) tiles[i] = a.tiles[i];
+  if (ctx)
+    for (int64_t i = tid; i < a.S; i += nth) ctx[i] = a.glm ? a.ctx[i] : 0;
   for (int64_t t = tid; t < T; t += nth) {
     int lo = 0, hi = a.S - 1;  // last segment with cu[s] <= t
     while (lo < hi) {
@@ -370,7 +374,14 @@ __global__ void meta_kernel(MetaArgs a, int32_t* __restrict__ cu, int32_t* __res
       if (a.cu[mid] <= t) lo = mid;
       else hi = mid - 1;
     }
-    pos[t] = int32_t(t - a.cu[lo]);
+    const int i = int(t - a.cu[lo]);
+    int p1 = i, p2 = 0;
+    if (a.glm && a.ctx[lo] > 0 && i >= a.ctx[lo]) {
+      p1 = a.mpos[lo];
+      p2 = i - a.ctx[lo] + 1;
+    }
+    pos[t] = p1;
+    if (pos2) pos2[t] = p2;
   }
 }
 
@@ -502,9 +513,10 @@ int fl_launch_copy_clients(const CopyTable& tab, cudaStream_t st) {
   return FL_OK;
 }
 
-int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, cudaStream_t st) {
+int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, int32_t* pos2, int32_t* ctx,
+                   cudaStream_t st) {
   const int T = a.cu[a.S];
-  meta_kernel<<<grid_for(T > a.n_tiles ? T : a.n_tiles), 256, 0, st>>>(a, cu, pos, tiles);
+  meta_kernel<<<grid_for(T > a.n_tiles ? T : a.n_tiles), 256, 0, st>>>(a, cu, pos, tiles, pos2, ctx);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }

@@ -121,7 +121,8 @@ struct fl_server {
   float *dyf = nullptr, *dxf = nullptr, *dm = nullptr, *dhf = nullptr, *da = nullptr;
   float *delta = nullptr, *ln_ws = nullptr;
   // metadata
-  int32_t *cu = nullptr, *pos = nullptr;
+  int32_t *cu = nullptr, *pos = nullptr, *pos2 = nullptr, *ctx = nullptr;
+  bool glm = false;  // the pending call has GLM blank-infilling segments
   uint32_t* tiles = nullptr;
   float* rope_tab = nullptr;
   int* status = nullptr;
@@ -154,6 +155,15 @@ struct fl_server {
       }
     }
     return p;
+  }
+  AttnGlm glm_args() const {
+    AttnGlm a;
+    if (glm) {
+      a.ctx = ctx;
+      a.pos = pos;
+      a.pos2 = pos2;
+    }
+    return a;
   }
   float* wt(int b, int t) { return w + off(b, t); }
   float* gt(int b, int t) { return g + off(b, t); }
@@ -322,6 +332,7 @@ int block_forward(fl_server* h, int b) {
   fl_gemm_args g1 = gemm_fwd(T, 3 * H, H, A.a, h->wbt(b, FL_T_WQKV), A.qkv, FL_EPI_BIAS_ROPE);
   g1.bias = h->wt(b, FL_T_BQKV);
   g1.pos = h->pos;
+  g1.pos2 = h->glm ? h->pos2 : nullptr;
   g1.rope_tab = h->rope_tab;
   g1.n_heads = c.n_heads;
   g1.head_dim = c.head_dim;
@@ -330,7 +341,7 @@ int block_forward(fl_server* h, int b) {
   // o = causal attention within each segment
   prof_begin(h, FL_PROF_ATTN);
   TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse,
-                            h->prefix(b, false), st));
+                            h->prefix(b, false), h->glm_args(), st));
   prof_end(h);
   // h = alpha * (LN1(x) or x) + o Wd^T + bd, fp32; LN1(x) recomputed in fp32 in the epilogue
   fl_gemm_args g2 = gemm_fwd(T, H, H, A.o, h->wbt(b, FL_T_WDENSE), A.h, FL_EPI_BIAS_RESID);
@@ -428,7 +439,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   // attention backward -> dqkv (w.r.t. the un-rotated q, k)
   prof_begin(h, FL_PROF_ATTN, 3);
   TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
-                            h->rope_tab, h->dqkv, h->prefix(b, true), st));
+                            h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st));
   prof_end(h);
   // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a; dbqkv += colsum(dqkv)
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
@@ -577,7 +588,8 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
       (rc = dalloc(h, &h->dqkv, Tm * 3 * H)) || (rc = dalloc(h, &h->da, Tm * H)) ||
       (rc = dalloc(h, &h->delta, Tm * c.n_heads)) ||
       (rc = dalloc(h, &h->ln_ws, fl_k_layernorm_bwd_workspace((int32_t)Tm, (int32_t)H) / sizeof(float))) ||
-      (rc = dalloc(h, &h->cu, FL_MAX_SEGS + 1)) || (rc = dalloc(h, &h->pos, Tm)) ||
+      (rc = dalloc(h, &h->cu, FL_MAX_SEGS + 1)) || (rc = dalloc(h, &h->pos, Tm)) || (rc = dalloc(h, &h->pos2, Tm)) ||
+      (rc = dalloc(h, &h->ctx, FL_MAX_SEGS)) ||
       (rc = dalloc(h, &h->tiles, FL_MAX_TILES)) || (rc = dalloc(h, &h->status, 1)))
     return fail(rc);
 
@@ -618,8 +630,8 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
   return FL_OK;
 }
 
-extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[], const int32_t seq_lens[], int32_t K,
-                                 void* const out_states[]) {
+static int forward_impl(fl_server_t h, const void* const client_states[], const int32_t seq_lens[], int32_t K,
+                        const int32_t* context_lens, const int32_t* mask_pos, void* const out_states[]) {
   if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "forward: null handle");
   const fl_server_cfg& c = h->cfg;
   if (h->pending) return set_err(h, FL_ERR_STATE, "forward: a forward is already pending (call backward first)");
@@ -645,6 +657,21 @@ extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[
   meta.cu[0] = 0;
   for (int k = 0, s = 0; k < K; ++k)
     for (int r = 0; r < b; ++r, ++s) meta.cu[s + 1] = meta.cu[s] + seq_lens[k];
+  meta.glm = context_lens != nullptr;
+  if (meta.glm) {
+    if (2 * h->rdim != c.head_dim)
+      return set_err(h, FL_ERR_UNSUPPORTED, "forward: GLM 2D positions need rotary_dim = head_dim / 2");
+    for (int s = 0; s < (int)S; ++s) {
+      const int L = meta.cu[s + 1] - meta.cu[s];
+      const int cl = context_lens[s];
+      const int mp = mask_pos ? mask_pos[s] : cl - 1;
+      if (cl < 0 || cl > L) return set_err(h, FL_ERR_INVALID_ARG, "forward: context_lens[%d]=%d outside [0, %d]", s, cl, L);
+      if (cl > 0 && (mp < 0 || mp >= cl))
+        return set_err(h, FL_ERR_INVALID_ARG, "forward: mask_pos[%d]=%d outside [0, %d)", s, mp, cl);
+      meta.ctx[s] = cl;
+      meta.mpos[s] = cl > 0 ? mp : 0;
+    }
+  }
   const int nt = fl_build_tiles(meta.cu, (int)S, meta.tiles, FL_MAX_TILES);
   if (nt < 0) return set_err(h, FL_ERR_CAPACITY, "forward: more than %d attention tiles", FL_MAX_TILES);
   meta.n_tiles = nt;
@@ -655,7 +682,8 @@ extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[
   h->seq_lens.assign(seq_lens, seq_lens + K);
 
   prof_begin(h, FL_PROF_OTHER);
-  int rc = fl_launch_meta(meta, h->cu, h->pos, h->tiles, h->stream);
+  h->glm = meta.glm;
+  int rc = fl_launch_meta(meta, h->cu, h->pos, h->tiles, h->pos2, h->ctx, h->stream);
   prof_end(h);
   if (rc) return fwd_err(h, rc);
   if ((rc = copy_clients(h, client_states, COPY_GATHER_F32, nullptr, h->xs[0]))) return rc;
@@ -664,6 +692,18 @@ extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[
   if ((rc = copy_clients(h, (const void* const*)out_states, COPY_SCATTER_F32, nullptr, h->xs[c.n_blocks]))) return rc;
   h->pending = true;
   return FL_OK;
+}
+
+extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[], const int32_t seq_lens[], int32_t K,
+                                 void* const out_states[]) {
+  return forward_impl(h, client_states, seq_lens, K, nullptr, nullptr, out_states);
+}
+
+extern "C" int fl_server_forward_glm(fl_server_t h, const void* const client_states[], const int32_t seq_lens[],
+                                     int32_t K, const int32_t context_lens[], const int32_t mask_pos[],
+                                     void* const out_states[]) {
+  if (h && !context_lens) return set_err(h, FL_ERR_INVALID_ARG, "forward_glm: context_lens is null");
+  return forward_impl(h, client_states, seq_lens, K, context_lens, mask_pos, out_states);
 }
 
 static int backward_impl(fl_server_t h, const void* const grad_out[], void* const grad_in[]) {

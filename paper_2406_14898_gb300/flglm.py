@@ -58,7 +58,8 @@ class fl_gemm_args(C.Structure):
                 ("ln_mean", C.c_void_p), ("ln_rstd", C.c_void_p), ("ln_gamma", C.c_void_p),
                 ("ln_beta", C.c_void_p), ("adam_m", C.c_void_p), ("adam_v", C.c_void_p),
                 ("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float), ("eps", C.c_float),
-                ("weight_decay", C.c_float), ("inv_bc1", C.c_float), ("inv_bc2", C.c_float)]
+                ("weight_decay", C.c_float), ("inv_bc1", C.c_float), ("inv_bc2", C.c_float),
+                ("pos2", C.c_void_p)]
 
 
 _P = C.c_void_p
@@ -69,6 +70,7 @@ _SIGS = {
     "fl_server_cfg_default": (None, [C.POINTER(fl_server_cfg)]),
     "fl_server_create": (C.c_int, [C.POINTER(fl_server_cfg), C.c_uint64, C.POINTER(_P)]),
     "fl_server_forward": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I32), _I32, C.POINTER(_P)]),
+    "fl_server_forward_glm": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I32), _I32, _P, _P, C.POINTER(_P)]),
     "fl_server_backward": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_P)]),
     "fl_server_step": (C.c_int, [_P, _F]),
     "fl_server_backward_step": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_P), _F]),
@@ -93,9 +95,9 @@ _SIGS = {
     "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _I32, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P]),
     "fl_k_layernorm_bwd_noalloc": (C.c_int, [_I32, _I32, _P, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_attention_tiles": (_I32, [_P, _I32]),
-    "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _I32, _P]),
+    "fl_k_attention_fwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _I32, _P, _P, _P, _P, _P, _I32, _P, _P]),
     "fl_k_attention_bwd": (C.c_int, [_I32, _I32, _I32, _P, _P, _P, _P, _P, _P, _I32, _P, _P, _P, _I32, _P,
-                                     _P, _P, _I32, _P, _P, _P]),
+                                     _P, _P, _I32, _P, _P, _P, _P, _P, _P]),
     "fl_k_adamw": (C.c_int, [_I64, _P, _P, _P, _P, _P, _F, _F, _F, _F, _F, _F, _F, _P]),
     "fl_k_colsum": (C.c_int, [_I32, _I32, _P, _P, _P]),
     "fl_k_pack_clients": (C.c_int, [_I32, C.POINTER(_P), C.POINTER(_I64), _P, _I32, _P]),
@@ -199,10 +201,19 @@ class Server:
     def set_stream(self, stream):
         check(lib().fl_server_set_stream(self.h, stream_ptr(stream)), self.h)
 
-    def forward(self, client_states: Sequence, seq_lens: Sequence[int], out_states: Sequence):
+    def forward(self, client_states: Sequence, seq_lens: Sequence[int], out_states: Sequence,
+                context_lens: Optional[Sequence[int]] = None, mask_pos: Optional[Sequence[int]] = None):
+        """context_lens / mask_pos (one per segment, client-major): GLM blank-infilling
+        segments through fl_server_forward_glm."""
         K = len(client_states)
         lens = (C.c_int32 * K)(*seq_lens)
-        check(lib().fl_server_forward(self.h, _parr(client_states), lens, K, _parr(out_states)), self.h)
+        if context_lens is None:
+            check(lib().fl_server_forward(self.h, _parr(client_states), lens, K, _parr(out_states)), self.h)
+            return
+        ctx = (C.c_int32 * len(context_lens))(*context_lens)
+        mp = None if mask_pos is None else (C.c_int32 * len(mask_pos))(*mask_pos)
+        check(lib().fl_server_forward_glm(self.h, _parr(client_states), lens, K, C.cast(ctx, _P),
+                                          None if mp is None else C.cast(mp, _P), _parr(out_states)), self.h)
 
     def backward(self, grad_out: Sequence, grad_in: Sequence):
         check(lib().fl_server_backward(self.h, _parr(grad_out), _parr(grad_in)), self.h)
@@ -283,10 +294,11 @@ def fl_k_gemm(args: fl_gemm_args, status=None, stream=None):
 def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
          alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
          aux_dtype=FL_DT_BF16, d_dtype=FL_DT_BF16, ln_mean=None, ln_rstd=None, ln_gamma=None, ln_beta=None,
-         status=None, stream=None):
+         pos2=None, status=None, stream=None):
     a = fl_gemm_args(M, N, K, ptr(A), lda, a_mn, ptr(B), ldb, b_mn, ptr(D), ldd, epilogue, ptr(bias), ptr(aux),
                      ld_aux, alpha, ptr(aux_out), ld_aux_out, ptr(pos), ptr(rope_tab), n_heads, head_dim, rotary_dim,
                      aux_dtype, d_dtype, ptr(ln_mean), ptr(ln_rstd), ptr(ln_gamma), ptr(ln_beta))
+    a.pos2 = ptr(pos2)
     fl_k_gemm(a, status, stream)
 
 
@@ -318,23 +330,24 @@ def fl_k_attention_tiles(cu_host) -> int:
 
 
 def fl_k_attention_fwd(T, n_heads, head_dim, qkv, cu_host, cu_dev, tile_ws, o, lse, prefix_k=None, prefix_v=None,
-                       prefix_len=0, stream=None):
+                       prefix_len=0, context_lens=None, stream=None):
     import numpy as np
     a = np.ascontiguousarray(cu_host, np.int32)
     check(lib().fl_k_attention_fwd(T, n_heads, head_dim, ptr(qkv), a.ctypes.data, ptr(cu_dev), a.size - 1,
                                    ptr(tile_ws), ptr(o), ptr(lse), ptr(prefix_k), ptr(prefix_v), prefix_len,
-                                   stream_ptr(stream)))
+                                   ptr(context_lens), stream_ptr(stream)))
 
 
 def fl_k_attention_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_host, cu_dev, tile_ws, delta_ws, rope_tab,
                        rotary_dim, dqkv, prefix_k=None, prefix_v=None, prefix_len=0, dprefix_k=None, dprefix_v=None,
-                       stream=None):
+                       context_lens=None, positions=None, block_positions=None, stream=None):
     import numpy as np
     a = np.ascontiguousarray(cu_host, np.int32)
     check(lib().fl_k_attention_bwd(T, n_heads, head_dim, ptr(qkv), ptr(o), ptr(lse), ptr(dout), a.ctypes.data,
                                    ptr(cu_dev), a.size - 1, ptr(tile_ws), ptr(delta_ws), ptr(rope_tab), rotary_dim,
                                    ptr(dqkv), ptr(prefix_k), ptr(prefix_v), prefix_len, ptr(dprefix_k),
-                                   ptr(dprefix_v), stream_ptr(stream)))
+                                   ptr(dprefix_v), ptr(context_lens), ptr(positions), ptr(block_positions),
+                                   stream_ptr(stream)))
 
 
 def fl_k_adamw(n, w, g, m, v, w_bf16, lr, beta1, beta2, eps, weight_decay, bc1, bc2, stream=None):
