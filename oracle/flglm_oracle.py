@@ -26,6 +26,11 @@ What it computes (plain definitions, in the paper's order, float64 throughout):
   with the softmax scale 1/sqrt(d_h) of App. A (P-tuning v2 equations).
 * The optimizer of §4.1.4 (Adam, without weight decay) in the decoupled AdamW form
   with bias correction; the decay rate is a parameter that defaults to 0.
+* §3.1 client parts: h_0 = Block_0(Embedding(x)) at the bottom; at the top
+  y' = Linear(Block_{N-1}(h_{N-2})) and the cross-entropy loss.  Reading: the
+  ChatGLM-6B top, a final LayerNorm before the bias-free LM head, the loss the mean
+  over the answer tokens that carry a target.  Clients and server parameters are
+  averaged at the end of a period (§3.3).
 * §4.1.1 casts every task as GLM blank infilling: a context with a mask token [M]
   (a cloze question, or [M] appended after the text for summarisation) and an answer
   span generated after it.  Optional per-segment GLM structure (context length c and
@@ -495,3 +500,128 @@ def average_params(servers: Sequence["OracleServer"]):
             mean = sum(s.params[b][t] for s in servers) / n
             for s in servers:
                 s.params[b][t] = mean.copy()
+
+
+# ----------------------------------------------------------------------------- client parts (§3.1)
+
+
+def embedding_fwd(E: np.ndarray, tokens: np.ndarray) -> np.ndarray:
+    """Rows of the embedding table for the token ids."""
+    return E[tokens]
+
+
+def embedding_bwd(dX: np.ndarray, tokens: np.ndarray, vocab: int) -> np.ndarray:
+    """Gradient of the table: each row receives the sum of the gradients of its occurrences."""
+    dE = np.zeros((vocab, dX.shape[1]), F64)
+    np.add.at(dE, tokens, dX)
+    return dE
+
+
+def cross_entropy(logits: np.ndarray, labels: np.ndarray):
+    """Mean over the rows with a target (label >= 0) of -log softmax(logits)[label], and its
+    gradient w.r.t. the logits (zero on rows without a target).  No target: loss 0."""
+    valid = labels >= 0
+    n = int(valid.sum())
+    m = logits.max(axis=-1, keepdims=True)
+    lse = m[:, 0] + np.log(np.exp(logits - m).sum(axis=-1))
+    d = np.exp(logits - lse[:, None])
+    rows = np.nonzero(valid)[0]
+    loss = float((lse[rows] - logits[rows, labels[rows]]).sum() / max(n, 1))
+    d[rows, labels[rows]] -= 1.0
+    d[~valid] = 0.0
+    return loss, d / max(n, 1)
+
+
+CLIENT_PARTS = ("bottom", "top", "embed", "head", "final_ln")
+
+
+class OracleClient:
+    """One client of §3.1: bottom = Embedding + Block_0, top = Block_{N-1} + final LayerNorm +
+    LM head + cross-entropy.  Protocol: bottom_forward(tokens) -> h_0 (to the server);
+    top_forward_backward(h_{N-2}, labels) -> loss and the gradient w.r.t. h_{N-2} (to the
+    server); bottom_backward(gradient w.r.t. h_0); step(lr).  Both blocks see the segment
+    structure (GLM context, positions) of the bottom call and, with prefix_len, carry their
+    own P-tuning v2 prefixes; with freeze_base only those prefixes are trained."""
+
+    def __init__(self, cfg: syn.ServerConfig, params=None):
+        self.cfg = cfg
+        self.sh = BlockShape.of(cfg)
+        p = syn.init_client(cfg) if params is None else params
+        self.params = {k: [np.asarray(x, F64).copy() for x in p[k]] for k in CLIENT_PARTS}
+        self.grads = {k: [np.zeros_like(x) for x in v] for k, v in self.params.items()}
+        self.m = {k: [np.zeros_like(x) for x in v] for k, v in self.params.items()}
+        self.v = {k: [np.zeros_like(x) for x in v] for k, v in self.params.items()}
+        self.t = 0
+        self._pk = None
+        self._bottom = None
+
+    def _block(self, name):
+        blk = self.params[name]
+        return blk[:12], (blk[12:14] if self.cfg.prefix_len else None)
+
+    def _accumulate(self, name, grads):
+        for acc, g in zip(self.grads[name], grads):
+            acc += g
+
+    def bottom_forward(self, tokens: np.ndarray, context_lens=None, mask_pos=None) -> np.ndarray:
+        b, L = tokens.shape
+        pk = make_packing([L], b, context_lens, mask_pos)
+        x = embedding_fwd(self.params["embed"][0], tokens.reshape(-1))
+        P, pre = self._block("bottom")
+        y, sv = block_fwd(P, x, pk, self.sh, pre)
+        self._pk = pk
+        self._bottom = (tokens.reshape(-1), sv)
+        return y.reshape(b, L, -1)
+
+    def top_forward_backward(self, h: np.ndarray, labels: np.ndarray):
+        b, L, H = h.shape
+        pk = self._pk
+        P, pre = self._block("top")
+        y, sv = block_fwd(P, h.reshape(-1, H), pk, self.sh, pre)
+        g, be = self.params["final_ln"]
+        z, mu, rs = layer_norm_fwd(y, g, be, self.sh.ln_eps)
+        W = self.params["head"][0]
+        logits = z @ W.T
+        loss, dlog = cross_entropy(logits, labels.reshape(-1))
+        self._accumulate("head", [dlog.T @ z])
+        dz = dlog @ W
+        dy, dg, dbe = layer_norm_bwd(dz, y, mu, rs, g)
+        self._accumulate("final_ln", [dg, dbe])
+        dx, gb = block_bwd(P, sv, dy, pk, self.sh)
+        self._accumulate("top", gb)
+        return loss, dx.reshape(b, L, H)
+
+    def bottom_backward(self, grad_h0: np.ndarray):
+        tokens, sv = self._bottom
+        P, _ = self._block("bottom")
+        H = grad_h0.shape[-1]
+        dx, gb = block_bwd(P, sv, grad_h0.reshape(-1, H), self._pk, self.sh)
+        self._accumulate("bottom", gb)
+        self._accumulate("embed", [embedding_bwd(dx, tokens, self.cfg.vocab)])
+        self._bottom = None
+
+    def trained(self):
+        """(part, tensor index) of every trained tensor."""
+        if self.cfg.freeze_base:
+            return [(k, i) for k in ("bottom", "top") for i in (12, 13)]
+        return [(k, i) for k in CLIENT_PARTS for i in range(len(self.params[k]))]
+
+    def step(self, lr: float):
+        c = self.cfg
+        self.t += 1
+        for k, i in self.trained():
+            w, m, v = adamw_update(self.params[k][i], self.grads[k][i], self.m[k][i], self.v[k][i], self.t, lr,
+                                   c.adam_beta1, c.adam_beta2, c.adam_eps, c.weight_decay)
+            self.params[k][i], self.m[k][i], self.v[k][i] = w, m, v
+        self.grads = {k: [np.zeros_like(x) for x in v] for k, v in self.params.items()}
+
+
+def average_clients(clients: Sequence[OracleClient]):
+    """§3.3: at the end of a period the client-side parameters are replaced by their mean
+    over the clients (moments and step counts stay local)."""
+    n = len(clients)
+    for k in CLIENT_PARTS:
+        for i in range(len(clients[0].params[k])):
+            mean = sum(c.params[k][i] for c in clients) / n
+            for c in clients:
+                c.params[k][i] = mean.copy()

@@ -37,6 +37,14 @@ from this text):
         [M]  = c - 1 if raw(key, 1) is even (summarisation: [M] ends the context),
                else raw(key, 1) >> 1 mod c                   (cloze: [M] inside it)
       (L = 1: c = 1, [M] = 0)
+    client parts (one client model, the same initial values for every client):
+        block 0 (bottom) tensor t: key(seed, CLIENT, block 0, t); block N-1 (top): block 1;
+        embedding [V, H]: key(seed, CLIENT, block 2, 0); LM head [V, H]: block 3;
+        final LayerNorm gamma = 1, beta = 0; N(0, init_std) like the server's weights
+    client k's token ids: raw(key(seed, TOKENS, client = k), i) mod V, i over [b, L];
+    labels (next-token targets of the answer span): label[t] = token[t + 1] when
+        t + 1 >= c (c = the segment's GLM context length, 0 without GLM) and t + 1 < L,
+        else -1 (ignored)
 """
 from __future__ import annotations
 
@@ -57,6 +65,11 @@ P_STATES = 2
 P_GRADS = 3
 P_LENGTHS = 4
 P_GLM = 5
+P_CLIENT = 6
+P_TOKENS = 7
+# client-side tensors outside the two blocks (block ids of the CLIENT streams)
+CB_BOTTOM, CB_TOP, CB_EMBED, CB_HEAD = 0, 1, 2, 3
+CHATGLM6B_VOCAB = 130528
 
 # per-block parameter tensors, in arena order (the C library uses the same ids)
 TENSOR_NAMES = ("w_qkv", "b_qkv", "w_dense", "b_dense", "w_up", "b_up",
@@ -179,6 +192,7 @@ class ServerConfig:
     prefix_len: int = 0        # P-tuning v2 prefix keys/values per block (0: none)
     freeze_base: int = 0       # 1: only the prefixes are trained (P-tuning v2)
     glm: int = 0               # 1: every segment carries a GLM blank-infilling structure
+    vocab: int = CHATGLM6B_VOCAB   # client embedding / LM head rows
 
     @property
     def K(self) -> int:
@@ -236,7 +250,8 @@ def ragged_lengths(seed: int, K: int, lo: int = 64, hi: int = 1024) -> tuple:
     return tuple(int(lo + int(v) % (hi - lo + 1)) for v in x)
 
 
-def init_tensor(cfg: ServerConfig, block: int, tensor: int, seed: Optional[int] = None) -> np.ndarray:
+def init_tensor(cfg: ServerConfig, block: int, tensor: int, seed: Optional[int] = None,
+                purpose: int = P_WEIGHTS) -> np.ndarray:
     """Initial fp32 master value of one parameter tensor: N(0, init_std) for weights and
     biases, gamma = 1, beta = 0 for the LayerNorms."""
     seed = cfg.seed if seed is None else seed
@@ -246,8 +261,47 @@ def init_tensor(cfg: ServerConfig, block: int, tensor: int, seed: Optional[int] 
         return np.ones(shape, np.float32)
     if tensor in (T_BE1, T_BE2):
         return np.zeros(shape, np.float32)
-    key = stream_key(seed, P_WEIGHTS, block, tensor)
+    key = stream_key(seed, purpose, block, tensor)
     return normal_f32(key, n, 0.0, float(np.float32(cfg.init_std))).reshape(shape)
+
+
+def init_client(cfg: ServerConfig, seed: Optional[int] = None) -> Dict[str, list]:
+    """Initial client model (see the module docstring): the two blocks (12 tensors each, plus
+    the prefix keys/values with prefix_len), embedding, final LayerNorm and LM head."""
+    seed = cfg.seed if seed is None else seed
+    std = float(np.float32(cfg.init_std))
+    out = {}
+    for name, blk in (("bottom", CB_BOTTOM), ("top", CB_TOP)):
+        ts = [init_tensor(cfg, blk, t, seed, P_CLIENT) for t in range(12)]
+        if cfg.prefix_len:
+            for t, shp in zip((T_PK, T_PV), prefix_shapes(cfg)):
+                ts.append(normal_f32(stream_key(seed, P_CLIENT, blk, t), int(np.prod(shp)), 0.0, std).reshape(shp))
+        out[name] = ts
+    V, H = cfg.vocab, cfg.hidden
+    out["embed"] = [normal_f32(stream_key(seed, P_CLIENT, CB_EMBED, 0), V * H, 0.0, std).reshape(V, H)]
+    out["head"] = [normal_f32(stream_key(seed, P_CLIENT, CB_HEAD, 0), V * H, 0.0, std).reshape(V, H)]
+    out["final_ln"] = [np.ones(H, np.float32), np.zeros(H, np.float32)]
+    return out
+
+
+def client_tokens(cfg: ServerConfig, k: int, seed: Optional[int] = None) -> np.ndarray:
+    """Client k's token ids, int32 [client_batch, L_k], uniform over the vocabulary."""
+    seed = cfg.seed if seed is None else seed
+    L = cfg.seq_lens[k]
+    x = raw_u64(stream_key(seed, P_TOKENS, 0, 0, k), 0, cfg.client_batch * L)
+    return (x % np.uint64(cfg.vocab)).astype(np.int32).reshape(cfg.client_batch, L)
+
+
+def client_labels(tokens: np.ndarray, context_lens: Optional[List[int]] = None) -> np.ndarray:
+    """Next-token targets of the answer span of each row (-1: no target)."""
+    b, L = tokens.shape
+    lab = np.full((b, L), -1, np.int32)
+    for r in range(b):
+        c = 0 if context_lens is None else int(context_lens[r])
+        for t in range(L - 1):
+            if t + 1 >= c:
+                lab[r, t] = tokens[r, t + 1]
+    return lab
 
 
 def init_params(cfg: ServerConfig, seed: Optional[int] = None) -> List[List[np.ndarray]]:

@@ -756,3 +756,163 @@ def test_glm_structure_recipe():
     for L, c, m in zip(cfg.segment_lengths, ctx, mp):
         assert 1 <= L - c <= max(1, L // 4) and 0 <= m < c
     assert any(m == c - 1 for c, m in zip(ctx, mp)) and any(m < c - 1 for c, m in zip(ctx, mp))
+
+
+# ----------------------------------------------------------------------------- client parts (§3.1)
+
+def test_cross_entropy_matches_torch():
+    rng = np.random.default_rng(80)
+    T, V = 23, 37
+    logits = 3.0 * rng.standard_normal((T, V))
+    labels = rng.integers(0, V, size=T).astype(np.int32)
+    labels[[2, 5, 11]] = -1
+    loss, d = O.cross_entropy(logits, labels)
+    tl = torch.tensor(logits, requires_grad=True)
+    ref = torch.nn.functional.cross_entropy(tl, torch.tensor(labels, dtype=torch.long), ignore_index=-1)
+    ref.backward()
+    assert abs(loss - ref.item()) < 1e-12
+    np.testing.assert_allclose(d, tl.grad.numpy(), rtol=0, atol=1e-14)
+    # no target at all: zero loss and gradient
+    l0, d0 = O.cross_entropy(logits, np.full(T, -1, np.int32))
+    assert l0 == 0.0 and not d0.any()
+
+
+def test_cross_entropy_uniform_closed_form():
+    """Equal logits: loss = log V; gradient (1/V - onehot) / n on the rows with a target."""
+    T, V = 6, 50
+    labels = np.array([3, -1, 0, 49, -1, 7], np.int32)
+    loss, d = O.cross_entropy(np.full((T, V), 0.7), labels)
+    assert abs(loss - math.log(V)) < 1e-14
+    want = np.zeros((T, V))
+    for t, y in enumerate(labels):
+        if y >= 0:
+            want[t] = 1.0 / V
+            want[t, y] -= 1.0
+    np.testing.assert_allclose(d, want / 4, rtol=0, atol=1e-15)
+
+
+def test_embedding_matches_torch():
+    rng = np.random.default_rng(81)
+    V, H = 20, 6
+    E = rng.standard_normal((V, H))
+    tokens = np.array([3, 7, 3, 19, 0, 3, 7], np.int64)
+    dX = rng.standard_normal((len(tokens), H))
+    tE = torch.tensor(E, requires_grad=True)
+    out = torch.nn.functional.embedding(torch.tensor(tokens), tE)
+    np.testing.assert_array_equal(O.embedding_fwd(E, tokens), out.detach().numpy())
+    out.backward(torch.tensor(dX))
+    np.testing.assert_allclose(O.embedding_bwd(dX, tokens, V), tE.grad.numpy(), rtol=0, atol=1e-14)
+
+
+def client_cfg(**kw):
+    return tiny_cfg(n_blocks=1, seq_lens=(5,), b=2).with_(vocab=29, **kw)
+
+
+def random_client_params(cfg, rng):
+    p = {"bottom": random_params(cfg, rng)[0], "top": random_params(cfg, rng)[0]}
+    if cfg.prefix_len:
+        for k in ("bottom", "top"):
+            p[k] += [0.5 * rng.standard_normal(s) for s in syn.prefix_shapes(cfg)]
+    p["embed"] = [rng.standard_normal((cfg.vocab, cfg.hidden))]
+    p["head"] = [0.3 * rng.standard_normal((cfg.vocab, cfg.hidden))]
+    p["final_ln"] = [1.0 + 0.3 * rng.standard_normal(cfg.hidden), 0.3 * rng.standard_normal(cfg.hidden)]
+    return p
+
+
+@pytest.mark.parametrize("Lp,glm", [(0, False), (2, True)])
+def test_client_finite_differences(Lp, glm):
+    """Loss of the client alone (bottom output handed straight to the top): central
+    differences on every client parameter, with and without GLM segments and prefixes."""
+    cfg = client_cfg(prefix_len=Lp)
+    rng = np.random.default_rng(82 + Lp)
+    params = random_client_params(cfg, rng)
+    tokens = rng.integers(0, cfg.vocab, size=(2, 5)).astype(np.int32)
+    ctx = [3, 1] if glm else None
+    labels = syn.client_labels(tokens, ctx)
+
+    def run(p, with_grads=False):
+        cl = O.OracleClient(cfg, p)
+        h0 = cl.bottom_forward(tokens, ctx)
+        loss, gh = cl.top_forward_backward(h0, labels)
+        if with_grads:
+            cl.bottom_backward(gh)
+        return loss, cl
+
+    _, cl = run(params, True)
+    h = 1e-5
+    irng = np.random.default_rng(83)
+    for part in O.CLIENT_PARTS:
+        for i, an in enumerate(cl.grads[part]):
+            flat = an.reshape(-1)
+            scale = max(np.abs(flat).max(), 1e-8)
+            if part == "embed":   # rows of tokens that occur, plus one that does not
+                rows = sorted(set(tokens.reshape(-1).tolist()))[:3] + [int(np.setdiff1d(np.arange(cfg.vocab), tokens)[0])]
+                idx = [r * cfg.hidden + c for r in rows for c in (0, 5)]
+            else:
+                idx = irng.choice(flat.size, size=min(12, flat.size), replace=False)
+            for j in idx:
+                vals = []
+                for dlt in (h, -h):
+                    pp = {k: [x.copy() for x in v] for k, v in params.items()}
+                    pp[part][i].reshape(-1)[j] += dlt
+                    vals.append(run(pp)[0])
+                fd = (vals[0] - vals[1]) / (2 * h)
+                assert abs(fd - flat[j]) <= 1e-6 * scale, (part, i, j, fd, flat[j])
+
+
+def test_split_equals_unsplit_model():
+    """§3.1 splits one model: client bottom -> server blocks -> client top gives the loss and
+    the embedding gradient of the same model run in one piece (embedding, all blocks in
+    order, final LayerNorm, head, cross-entropy)."""
+    cfg = tiny_cfg(n_blocks=2, seq_lens=(6, 4), b=1).with_(vocab=31)
+    rng = np.random.default_rng(84)
+    cp = random_client_params(cfg.with_(n_blocks=1), rng)
+    sp = random_params(cfg, rng)
+    toks = [rng.integers(0, cfg.vocab, size=(1, L)).astype(np.int32) for L in cfg.seq_lens]
+    ctx = [[4], [0]]
+    clients = [O.OracleClient(cfg, cp) for _ in toks]
+    srv = O.OracleServer(cfg, sp)
+    h0 = [c.bottom_forward(t, cx) for c, t, cx in zip(clients, toks, ctx)]
+    hs = srv.forward(h0, [cx[0] for cx in ctx])
+    out = [c.top_forward_backward(h, syn.client_labels(t, cx)) for c, h, t, cx in zip(clients, hs, toks, ctx)]
+    gi = srv.backward([g for _, g in out])
+    for c, g in zip(clients, gi):
+        c.bottom_backward(g)
+    sh = O.BlockShape.of(cfg)
+    E, W = cp["embed"][0], cp["head"][0]
+    stack = [cp["bottom"]] + sp + [cp["top"]]
+    for k, (t, cx) in enumerate(zip(toks, ctx)):
+        pk = O.make_packing([t.shape[1]], 1, cx)
+        x = E[t.reshape(-1)]
+        y, saved = O.stack_fwd(stack, x, pk, sh)
+        z, mu, rs = O.layer_norm_fwd(y, cp["final_ln"][0], cp["final_ln"][1], cfg.ln_eps)
+        loss, dlog = O.cross_entropy(z @ W.T, syn.client_labels(t, cx).reshape(-1))
+        assert abs(loss - out[k][0]) < 1e-12
+        dz = dlog @ W
+        dy, _, _ = O.layer_norm_bwd(dz, y, mu, rs, cp["final_ln"][0])
+        dx, _ = O.stack_bwd(stack, saved, dy, pk, sh)
+        np.testing.assert_allclose(clients[k].grads["embed"][0], O.embedding_bwd(dx, t.reshape(-1), cfg.vocab),
+                                   rtol=1e-10, atol=1e-12)
+
+
+def test_client_averaging_and_frozen_step():
+    cfg = client_cfg(prefix_len=2, freeze_base=1)
+    rng = np.random.default_rng(85)
+    cls = [O.OracleClient(cfg, random_client_params(cfg, rng)) for _ in range(3)]
+    want = {k: [sum(c.params[k][i] for c in cls) / 3 for i in range(len(cls[0].params[k]))] for k in O.CLIENT_PARTS}
+    O.average_clients(cls)
+    for c in cls:
+        for k in O.CLIENT_PARTS:
+            for i, w in enumerate(want[k]):
+                np.testing.assert_array_equal(c.params[k][i], w)
+    # P-tuning v2: a step moves only the client blocks' prefixes
+    c = cls[0]
+    tokens = rng.integers(0, cfg.vocab, size=(2, 5)).astype(np.int32)
+    before = {k: [x.copy() for x in v] for k, v in c.params.items()}
+    _, g = c.top_forward_backward(c.bottom_forward(tokens), syn.client_labels(tokens))
+    c.bottom_backward(g)
+    c.step(1e-2)
+    for k in O.CLIENT_PARTS:
+        for i, w in enumerate(c.params[k]):
+            moved = not np.array_equal(w, before[k][i])
+            assert moved == (k in ("bottom", "top") and i >= 12), (k, i)
