@@ -529,7 +529,9 @@ extern "C" void fl_server_cfg_default(fl_server_cfg* c) {
   c->weight_decay = 0.f;
 }
 
-extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_server_t* out) {
+// Seeded init keys: tensor t of block b from the stream (seed, purpose, block0 + b, t).
+// The server uses purpose 1 and block0 = 0; the client's blocks use their own streams.
+int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose, int block0, fl_server_t* out) {
   if (!out) return fl_internal_error(FL_ERR_INVALID_ARG, "create: out is null");
   *out = nullptr;
   if (!cfg) return fl_internal_error(FL_ERR_INVALID_ARG, "create: cfg is null");
@@ -620,7 +622,9 @@ extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_serv
       float* p = h->wt(b, t);
       if (t == FL_T_LN1_G || t == FL_T_LN2_G) rc = fl_launch_fill(h->tensor_n[t], 1.f, p, st);
       else if (t == FL_T_LN1_B || t == FL_T_LN2_B) rc = fl_launch_fill(h->tensor_n[t], 0.f, p, st);
-      else rc = fl_launch_normal_init(h->tensor_n[t], stream_key(seed, 1, b, t, 0), 0.0, (double)c.init_std, p, st);
+      else
+        rc = fl_launch_normal_init(h->tensor_n[t], stream_key(seed, (uint64_t)purpose, (uint64_t)(block0 + b), t, 0), 0.0,
+                                   (double)c.init_std, p, st);
       if (rc) return fail(rc);
     }
   if ((rc = fl_launch_f32_to_bf16(h->n_params, h->w, h->wb, st))) return fail(rc);
@@ -692,6 +696,10 @@ static int forward_impl(fl_server_t h, const void* const client_states[], const 
   if ((rc = copy_clients(h, (const void* const*)out_states, COPY_SCATTER_F32, nullptr, h->xs[c.n_blocks]))) return rc;
   h->pending = true;
   return FL_OK;
+}
+
+extern "C" int fl_server_create(const fl_server_cfg* cfg, uint64_t seed, fl_server_t* out) {
+  return fl_server_create_keyed(cfg, seed, 1, 0, out);
 }
 
 extern "C" int fl_server_forward(fl_server_t h, const void* const client_states[], const int32_t seq_lens[], int32_t K,

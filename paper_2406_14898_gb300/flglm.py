@@ -46,6 +46,13 @@ class fl_server_cfg(C.Structure):
                 ("prefix_len", C.c_int32), ("freeze_base", C.c_int32)]
 
 
+class fl_client_cfg(C.Structure):
+    _fields_ = [("block", fl_server_cfg), ("vocab", C.c_int32)]
+
+
+FL_CP_BOTTOM, FL_CP_TOP, FL_CP_EMBED, FL_CP_HEAD, FL_CP_FINAL_LN = range(5)
+
+
 class fl_gemm_args(C.Structure):
     _fields_ = [("M", C.c_int32), ("N", C.c_int32), ("K", C.c_int32),
                 ("A", C.c_void_p), ("lda", C.c_int64), ("a_mn_major", C.c_int32),
@@ -101,6 +108,22 @@ _SIGS = {
     "fl_k_adamw": (C.c_int, [_I64, _P, _P, _P, _P, _P, _F, _F, _F, _F, _F, _F, _F, _P]),
     "fl_k_colsum": (C.c_int, [_I32, _I32, _P, _P, _P]),
     "fl_k_pack_clients": (C.c_int, [_I32, C.POINTER(_P), C.POINTER(_I64), _P, _I32, _P]),
+    "fl_client_cfg_default": (None, [C.POINTER(fl_client_cfg)]),
+    "fl_client_create": (C.c_int, [C.POINTER(fl_client_cfg), C.c_uint64, C.POINTER(_P)]),
+    "fl_client_destroy": (C.c_int, [_P]),
+    "fl_client_set_stream": (C.c_int, [_P, _P]),
+    "fl_client_sync": (C.c_int, [_P]),
+    "fl_client_bottom_forward": (C.c_int, [_P, _P, _I32, _P, _P, _P]),
+    "fl_client_top_forward_backward": (C.c_int, [_P, _P, _P, _P, _P]),
+    "fl_client_bottom_backward": (C.c_int, [_P, _P]),
+    "fl_client_step": (C.c_int, [_P, _F]),
+    "fl_client_tensor_numel": (_I64, [_P, _I32, _I32]),
+    "fl_client_get_param": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
+    "fl_client_set_param": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
+    "fl_client_get_grad": (C.c_int, [_P, _I32, _I32, _P, C.c_size_t]),
+    "fl_client_average": (C.c_int, [C.POINTER(_P), _I32]),
+    "fl_client_launch_count": (_I64, [_P]),
+    "fl_client_last_error": (C.c_char_p, [_P]),
 }
 
 _lib = None
@@ -283,6 +306,97 @@ def fl_server_average(replicas: Sequence["Server"]):
     """Averages the replicas' parameters in place (the server-hierarchical strategy)."""
     arr = (C.c_void_p * len(replicas))(*[r.h.value for r in replicas])
     check(lib().fl_server_average(arr, len(replicas)), replicas[0].h if replicas else None)
+
+
+def make_client_cfg(c, max_tokens: int, max_seq_len: int = 0) -> fl_client_cfg:
+    """fl_client_cfg from a workload description (block fields as make_cfg, plus vocab)."""
+    cfg = fl_client_cfg()
+    lib().fl_client_cfg_default(C.byref(cfg))
+    cfg.block = make_cfg(c, max_tokens, max_seq_len)
+    cfg.block.n_blocks = 1
+    cfg.vocab = c.vocab
+    return cfg
+
+
+def check_client(rc: int, h):
+    if rc != FL_OK:
+        msg = lib().fl_client_last_error(h)
+        raise FlError(rc, msg.decode() if msg else "")
+
+
+class Client:
+    """Owns one fl_client handle (the client parts of §3.1).  Methods mirror fl_client_*."""
+
+    def __init__(self, cfg: fl_client_cfg, seed: int, stream=None):
+        self.h = C.c_void_p()
+        rc = lib().fl_client_create(C.byref(cfg), seed, C.byref(self.h))
+        check_client(rc, None)
+        self.cfg = cfg
+        if stream is not None:
+            self.set_stream(stream)
+
+    def close(self):
+        if self.h:
+            lib().fl_client_destroy(self.h)
+            self.h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def set_stream(self, stream):
+        check_client(lib().fl_client_set_stream(self.h, stream_ptr(stream)), self.h)
+
+    def sync(self):
+        check_client(lib().fl_client_sync(self.h), self.h)
+
+    def bottom_forward(self, tokens, seq_len: int, h0, context_lens=None, mask_pos=None):
+        ctx = None if context_lens is None else (C.c_int32 * len(context_lens))(*context_lens)
+        mp = None if mask_pos is None else (C.c_int32 * len(mask_pos))(*mask_pos)
+        check_client(lib().fl_client_bottom_forward(self.h, ptr(tokens), seq_len,
+                                                    None if ctx is None else C.cast(ctx, _P),
+                                                    None if mp is None else C.cast(mp, _P), ptr(h0)), self.h)
+
+    def top_forward_backward(self, h, labels, loss, grad_h):
+        check_client(lib().fl_client_top_forward_backward(self.h, ptr(h), ptr(labels), ptr(loss), ptr(grad_h)),
+                     self.h)
+
+    def bottom_backward(self, grad_h0):
+        check_client(lib().fl_client_bottom_backward(self.h, ptr(grad_h0)), self.h)
+
+    def step(self, lr: float):
+        check_client(lib().fl_client_step(self.h, lr), self.h)
+
+    def numel(self, part: int, tensor: int) -> int:
+        return int(lib().fl_client_tensor_numel(self.h, part, tensor))
+
+    def _get(self, fn, part, tensor):
+        import numpy as np
+        out = np.empty(self.numel(part, tensor), np.float32)
+        check_client(fn(self.h, part, tensor, out.ctypes.data, out.size), self.h)
+        return out
+
+    def get_param(self, part: int, tensor: int):
+        return self._get(lib().fl_client_get_param, part, tensor)
+
+    def get_grad(self, part: int, tensor: int):
+        return self._get(lib().fl_client_get_grad, part, tensor)
+
+    def set_param(self, part: int, tensor: int, values):
+        import numpy as np
+        a = np.ascontiguousarray(values, np.float32).reshape(-1)
+        check_client(lib().fl_client_set_param(self.h, part, tensor, a.ctypes.data, a.size), self.h)
+
+    def launch_count(self) -> int:
+        return int(lib().fl_client_launch_count(self.h))
+
+
+def fl_client_average(clients: Sequence["Client"]):
+    """Averages the clients' parameters in place (end of a training period, §3.3)."""
+    arr = (C.c_void_p * len(clients))(*[c.h.value for c in clients])
+    check_client(lib().fl_client_average(arr, len(clients)), clients[0].h if clients else None)
 
 
 # ----------------------------------------------------------------------------- kernel-level calls

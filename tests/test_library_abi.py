@@ -12,7 +12,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def declared_functions():
     names = set()
-    for h in ("flglm.h", "flglm_kernels.h"):
+    for h in ("flglm.h", "flglm_kernels.h", "flglm_client.h"):
         src = open(os.path.join(ROOT, "include", h)).read()
         src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
         for m in re.finditer(r"\b(fl_[a-z0-9_]+)\s*\(", src):
@@ -58,6 +58,15 @@ def test_cfg_default_and_validation(F):
     assert F.lib().fl_server_create(None, 0, ctypes.byref(h)) == -1
     assert F.lib().fl_server_forward(None, None, None, 1, None) == -1
     assert F.lib().fl_server_destroy(None) == 0
+    # client handles: defaults, validation before any device work
+    cc = F.fl_client_cfg()
+    F.lib().fl_client_cfg_default(ctypes.byref(cc))
+    assert cc.vocab == 130528 and cc.block.hidden == 4096
+    cc.vocab = 0
+    assert F.lib().fl_client_create(ctypes.byref(cc), 0, ctypes.byref(h)) == -1
+    assert not h.value and b"vocab" in F.lib().fl_client_last_error(None)
+    assert F.lib().fl_client_bottom_forward(None, None, 1, None, None, None) == -1
+    assert F.lib().fl_client_destroy(None) == 0
 
 
 def test_kernel_entry_points_validate_before_launch(F):
