@@ -252,6 +252,9 @@ def main():
     ap.add_argument("--ptuning", type=int, default=0, metavar="LP",
                     help="P-tuning v2, the paper's training setting: LP prefix keys/values per block, block "
                          "weights frozen, only the prefixes trained")
+    ap.add_argument("--split", action="store_true",
+                    help="the whole split-learning round: K client models (embedding + block 0, block N-1 + head "
+                         "+ cross-entropy) around the client-batched server, one GPU")
     ap.add_argument("--glm", action="store_true",
                     help="GLM blank-infilling segments (the paper's task format): each segment a bidirectional "
                          "context with a mask token and a causal answer span, GLM 2D positions")
@@ -270,6 +273,9 @@ def main():
         return
     if args.hierarchical:
         run_strategies(args, args.hierarchical)
+        return
+    if args.split:
+        run_split(args, cfg)
         return
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -603,6 +609,110 @@ def run_strategies(args, K: int):
             "timing": "host wall clock around the timed steps, after a device synchronisation on both sides",
             **res}
     print(json.dumps(line), flush=True)
+
+
+def client_flops(cfg: syn.ServerConfig) -> float:
+    """Dense work of the K clients in one round: two blocks each (the server's block FLOPs,
+    GEMM + attention, per block) and the LM head (forward and data gradient, plus the weight
+    gradient when the head is trained); the embedding is a gather."""
+    per_block = (gemm_flops(cfg) + attn_flops(cfg)) / cfg.n_blocks
+    head_passes = 2 if cfg.freeze_base else 3
+    vp = (cfg.vocab + 255) // 256 * 256
+    return 2 * per_block + head_passes * 2.0 * cfg.tokens * cfg.hidden * vp
+
+
+def run_split(args, cfg: syn.ServerConfig):
+    """The whole split-learning round of §3.1 on one GPU: K clients (each its own client
+    model: embedding + block 0, block N-1 + final LayerNorm + LM head + cross-entropy) and
+    the client-batched server, all on one stream:
+      K bottom forwards -> server forward (one packed call) -> K top forward/backward ->
+      server backward with the fused update -> K bottom backwards -> K client steps."""
+    import torch
+    from paper_2406_14898_gb300 import flglm as F
+
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.Stream(device=dev)
+    K, b = cfg.K, cfg.client_batch
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens)), cfg.seed, stream=stream)
+    ccfgs = [cfg.with_(seq_lens=(L,)) for L in cfg.seq_lens]
+    clients = [F.Client(F.make_client_cfg(c, c.tokens), cfg.seed, stream=stream) for c in ccfgs]
+    gk = glm_args(cfg)
+    ctx_all = gk.get("context_lens")
+    toks, labs = [], []
+    for k in range(K):
+        t = syn.client_tokens(cfg, k)
+        ctx = None if ctx_all is None else ctx_all[k * b:(k + 1) * b]
+        toks.append(torch.from_numpy(t).to(dev))
+        labs.append(torch.from_numpy(syn.client_labels(t, ctx)).to(dev))
+    h0 = [torch.empty((b, L, cfg.hidden), dtype=torch.bfloat16, device=dev) for L in cfg.seq_lens]
+    hs = [torch.empty_like(x) for x in h0]
+    gh = [torch.empty_like(x) for x in h0]
+    g0 = [torch.empty_like(x) for x in h0]
+    loss = torch.zeros(K, dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+
+    def round_():
+        for k in range(K):
+            ctx = None if ctx_all is None else ctx_all[k * b:(k + 1) * b]
+            mp = None if ctx_all is None else gk["mask_pos"][k * b:(k + 1) * b]
+            clients[k].bottom_forward(toks[k], cfg.seq_lens[k], h0[k], ctx, mp)
+        srv.forward(h0, cfg.seq_lens, hs, **gk)
+        for k in range(K):
+            clients[k].top_forward_backward(hs[k], labs[k], loss[k:k + 1], gh[k])
+        srv.backward_step(gh, g0, cfg.lr)
+        for k in range(K):
+            clients[k].bottom_backward(g0[k])
+            clients[k].step(cfg.lr)
+
+    for _ in range(args.warmup):
+        round_()
+    for c in clients:
+        c.sync()
+    srv.sync()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    l0 = srv.launch_count() + sum(c.launch_count() for c in clients)
+    clocks = ClockSampler(pci_bus_id(torch, dev))
+    clocks.start()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        round_()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    launches = srv.launch_count() + sum(c.launch_count() for c in clients) - l0
+    # the server's share of the round, timed alone the same way
+    srv.forward(h0, cfg.seq_lens, hs, **gk)
+    srv.backward_step(gh, g0, cfg.lr)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        srv.forward(h0, cfg.seq_lens, hs, **gk)
+        srv.backward_step(gh, g0, cfg.lr)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    srv_ms = e0.elapsed_time(e1) / args.steps
+    for c in clients:
+        c.sync()
+    pk = peaks()
+    flops = gemm_flops(cfg) + attn_flops(cfg) + client_flops(cfg)
+    line = {"metric": "split-learning round tokens/s (K clients + client-batched server, one GB300)",
+            "mode": "split round (Sec. 3.1 protocol)", "value": cfg.tokens / (ms / 1e3), "unit": "tokens/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_round": ms, "higher_is_better": True,
+            "dtype": "bf16", "data": "synthetic (seeded weights, uniform token ids, next-token labels on the answer "
+                                     "span)",
+            "config": {"workload": describe(cfg) + f"; clients: vocabulary {cfg.vocab}, embedding + block 0 and "
+                                                   "block N-1 + final LayerNorm + LM head + cross-entropy",
+                       "global_batch": cfg.tokens, "seq_len": max(cfg.seq_lens)},
+            "server_ms_per_round": srv_ms, "clients_ms_per_round": ms - srv_ms,
+            "pct_bf16_peak": 100.0 * flops / (ms / 1e3) / (pk["bf16_sustained"] * 1e12),
+            "pct_bf16_peak_basis": "algorithmic FLOPs of server and clients over the measured sustained bf16 peak",
+            "loss_mean": float(loss.mean().item()), "gpu_launches": launches, "clocks": clk}
+    print(json.dumps(line), flush=True)
+    for c in clients:
+        c.close()
+    srv.close()
 
 
 def pci_bus_id(torch, dev):
