@@ -156,6 +156,24 @@ int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void*
                        const int32_t* context_lens, const int32_t* positions, const int32_t* block_positions,
                        void* stream);
 
+/* Client parts (§3.1).  Embedding gather: out[t, :] = table[tokens[t], :] (bf16 [T, H] from
+ * a bf16 [vocab, H] table, H % 8 == 0); an id outside [0, vocab) gives a zero row and sets
+ * bit 1 of *status (device int).  Scatter-add backward: dtable[tokens[t], :] += dx[t, :]
+ * (fp32 atomics, so the order of equal tokens' additions varies; ids outside are skipped). */
+int fl_k_embedding_gather(int32_t T, int32_t H, const int32_t* tokens, const void* table, int32_t vocab,
+                          void* out, int* status, void* stream);
+int fl_k_embedding_scatter_add(int32_t T, int32_t H, const int32_t* tokens, int32_t vocab, const void* dx,
+                               float* dtable, void* stream);
+
+/* Cross-entropy of T rows of fp32 logits (row stride ld >= vocab, ld % 4 == 0, 16-byte
+ * aligned): count = #{t : 0 <= labels[t] < vocab}; row_loss[t] = logsumexp(row) -
+ * logits[t, labels[t]] (0 without a target); *loss = sum(row_loss) / max(count, 1), summed
+ * in a fixed order; dlogits (bf16, same stride) = (softmax(row) - onehot(label)) / count
+ * on rows with a target, 0 elsewhere and on the columns [vocab, ld).  A label >= vocab is
+ * ignored and sets bit 2 of *status. */
+int fl_k_cross_entropy(int32_t T, int32_t vocab, int64_t ld, const float* logits, const int32_t* labels,
+                       float* row_loss, void* dlogits, float* loss, int* count, int* status, void* stream);
+
 /* AdamW over n contiguous fp32 elements; bc1 = 1 - beta1^t, bc2 = 1 - beta2^t.
  * w_bf16 (optional) receives the rounded new weights; g is zeroed. */
 int fl_k_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,

@@ -167,6 +167,44 @@ int warps_grid(int64_t rows) { return (int)((rows * 32 + 255) / 256); }
 
 }  // namespace
 
+// ---------------------------------------------------------------------------- kernel-level API
+
+extern "C" int fl_k_embedding_gather(int32_t T, int32_t H, const int32_t* tokens, const void* table, int32_t vocab,
+                                     void* out, int* status, void* stream) {
+  if (T < 0 || H <= 0 || (H % 8) || vocab < 1 || !tokens || !table || !out || !status)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "embedding gather: args");
+  if (T == 0) return FL_OK;
+  embed_gather_kernel<<<warps_grid(T), 256, 0, (cudaStream_t)stream>>>(T, H, tokens, (const bf16*)table, vocab,
+                                                                       (bf16*)out, status);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+extern "C" int fl_k_embedding_scatter_add(int32_t T, int32_t H, const int32_t* tokens, int32_t vocab, const void* dx,
+                                          float* dtable, void* stream) {
+  if (T < 0 || H <= 0 || (H % 2) || vocab < 1 || !tokens || !dx || !dtable)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "embedding scatter: args");
+  if (T == 0) return FL_OK;
+  embed_scatter_kernel<<<warps_grid(T), 256, 0, (cudaStream_t)stream>>>(T, H, tokens, vocab, (const bf16*)dx, dtable);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+extern "C" int fl_k_cross_entropy(int32_t T, int32_t vocab, int64_t ld, const float* logits, const int32_t* labels,
+                                  float* row_loss, void* dlogits, float* loss, int* count, int* status, void* stream) {
+  if (T < 0 || vocab < 1 || ld < vocab || (ld % 4) || !logits || !labels || !row_loss || !dlogits || !loss ||
+      !count || !status)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "cross entropy: args");
+  if ((reinterpret_cast<uintptr_t>(logits) & 15) || (reinterpret_cast<uintptr_t>(dlogits) & 7))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "cross entropy: alignment");
+  cudaStream_t st = (cudaStream_t)stream;
+  count_kernel<<<1, RED_THREADS, 0, st>>>(T, labels, vocab, count, status);
+  if (T > 0) ce_kernel<<<T, CE_THREADS, 0, st>>>(vocab, ld, logits, labels, count, row_loss, (bf16*)dlogits);
+  loss_kernel<<<1, RED_THREADS, 0, st>>>(T, row_loss, count, loss);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
 // ---------------------------------------------------------------------------- client handle
 
 struct fl_client {

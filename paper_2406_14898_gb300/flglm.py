@@ -108,6 +108,9 @@ _SIGS = {
     "fl_k_adamw": (C.c_int, [_I64, _P, _P, _P, _P, _P, _F, _F, _F, _F, _F, _F, _F, _P]),
     "fl_k_colsum": (C.c_int, [_I32, _I32, _P, _P, _P]),
     "fl_k_pack_clients": (C.c_int, [_I32, C.POINTER(_P), C.POINTER(_I64), _P, _I32, _P]),
+    "fl_k_embedding_gather": (C.c_int, [_I32, _I32, _P, _P, _I32, _P, _P, _P]),
+    "fl_k_embedding_scatter_add": (C.c_int, [_I32, _I32, _P, _I32, _P, _P, _P]),
+    "fl_k_cross_entropy": (C.c_int, [_I32, _I32, _I64, _P, _P, _P, _P, _P, _P, _P, _P]),
     "fl_client_cfg_default": (None, [C.POINTER(fl_client_cfg)]),
     "fl_client_create": (C.c_int, [C.POINTER(fl_client_cfg), C.c_uint64, C.POINTER(_P)]),
     "fl_client_destroy": (C.c_int, [_P]),
@@ -462,6 +465,19 @@ def fl_k_attention_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_host, cu_dev,
                                    ptr(dqkv), ptr(prefix_k), ptr(prefix_v), prefix_len, ptr(dprefix_k),
                                    ptr(dprefix_v), ptr(context_lens), ptr(positions), ptr(block_positions),
                                    stream_ptr(stream)))
+
+
+def fl_k_embedding_gather(T, H, tokens, table, vocab, out, status, stream=None):
+    check(lib().fl_k_embedding_gather(T, H, ptr(tokens), ptr(table), vocab, ptr(out), ptr(status), stream_ptr(stream)))
+
+
+def fl_k_embedding_scatter_add(T, H, tokens, vocab, dx, dtable, stream=None):
+    check(lib().fl_k_embedding_scatter_add(T, H, ptr(tokens), vocab, ptr(dx), ptr(dtable), stream_ptr(stream)))
+
+
+def fl_k_cross_entropy(T, vocab, ld, logits, labels, row_loss, dlogits, loss, count, status, stream=None):
+    check(lib().fl_k_cross_entropy(T, vocab, ld, ptr(logits), ptr(labels), ptr(row_loss), ptr(dlogits), ptr(loss),
+                                   ptr(count), ptr(status), stream_ptr(stream)))
 
 
 def fl_k_adamw(n, w, g, m, v, w_bf16, lr, beta1, beta2, eps, weight_decay, bc1, bc2, stream=None):

@@ -2,6 +2,9 @@
 
     python -m paper_2406_14898_gb300.kernel_bench [--workload stack26] [--kernel all|<name>] [--reps 5]
 
+<name>: gemm or one GEMM case (qkv_fwd, ..., qkv_wgrad), attention, layernorm, adamw, colsum,
+client (cross-entropy over the ChatGLM-6B vocabulary and the embedding gather).
+
 Each kernel runs on random device buffers (uninitialised values are never read: every
 input is filled first) with CUDA events around `reps` launches on one stream, after one
 warm-up launch.  Prints one JSON line per kernel with its algorithmic work (FLOPs for
@@ -161,6 +164,38 @@ def main():
         ms = timed(lambda: F.fl_k_adamw(n, w, gr, m, v, wb, 1e-4, 0.9, 0.999, 1e-8, 0.0, 0.1, 0.001, stream=st))
         nbytes = n * (16 + 16 + 2)  # read w g m v, write w g m v, write bf16 copy
         out.append({"kernel": "adamw_one_block", "n": n, "ms": ms, "gbs": nbytes / ms / 1e6})
+    if args.kernel in ("all", "colsum"):
+        # bias gradient of the FFN up-projection: column sums of dU [T, F]
+        du = rnd(T, Fh)
+        db = torch.zeros(Fh, device=dev, dtype=torch.float32)
+        ms = timed(lambda: F.fl_k_colsum(T, Fh, du, db, stream=st))
+        nbytes = T * Fh * 2 + Fh * 8
+        out.append({"kernel": "colsum_dU", "ms": ms, "gbs": nbytes / ms / 1e6, "bytes": nbytes})
+        del du
+    if args.kernel in ("all", "client"):
+        # the client's cross-entropy over the ChatGLM-6B vocabulary (1024 tokens: 4 rows x 256)
+        # and the embedding gather of a full packed batch
+        V = syn.CHATGLM6B_VOCAB
+        ld = (V + 255) // 256 * 256
+        Tc = 1024
+        logits = rnd(Tc, ld, scale=2.0, dtype=torch.float32)
+        labels = torch.randint(0, V, (Tc,), device=dev, dtype=torch.int32, generator=g)
+        row = torch.empty(Tc, device=dev, dtype=torch.float32)
+        dlog = torch.empty(Tc, ld, device=dev, dtype=torch.bfloat16)
+        loss = torch.empty(1, device=dev, dtype=torch.float32)
+        cnt = torch.empty(1, device=dev, dtype=torch.int32)
+        status = torch.zeros(1, device=dev, dtype=torch.int32)
+        ms = timed(lambda: F.fl_k_cross_entropy(Tc, V, ld, logits, labels, row, dlog, loss, cnt, status, stream=st))
+        nbytes = Tc * V * 4 + Tc * ld * 2   # read the logits once, write the gradient
+        out.append({"kernel": "cross_entropy_vocab130528", "T": Tc, "ms": ms, "gbs": nbytes / ms / 1e6,
+                    "bytes": nbytes})
+        del logits, dlog
+        table = rnd(V, H)
+        toks = torch.randint(0, V, (T,), device=dev, dtype=torch.int32, generator=g)
+        emb = torch.empty(T, H, device=dev, dtype=torch.bfloat16)
+        ms = timed(lambda: F.fl_k_embedding_gather(T, H, toks, table, V, emb, status, stream=st))
+        nbytes = 2 * T * H * 2
+        out.append({"kernel": "embedding_gather", "T": T, "ms": ms, "gbs": nbytes / ms / 1e6, "bytes": nbytes})
     for r in out:
         print(json.dumps(r), flush=True)
 

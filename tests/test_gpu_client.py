@@ -260,3 +260,54 @@ def test_client_chatglm6b_shapes(F):
     params["head"] = [draw((cfg.vocab, cfg.hidden))]
     params["final_ln"] = [1.0 + draw(cfg.hidden), draw(cfg.hidden)]
     client_round(F, cfg, ctx=[70], mp=[69], check_step=False, params=params)
+
+
+@pytest.mark.parametrize("V,ld", [(1000, 1024), (130528, 130560), (5, 8)])
+def test_cross_entropy_kernel(F, V, ld):
+    """The row kernel against the oracle: loss, per-row losses and the logit gradient,
+    ragged vocabulary tails, padded columns zero, rows without a target."""
+    rng = np.random.default_rng(V)
+    T = 37
+    logits = np.zeros((T, ld), np.float32)
+    logits[:, :V] = (2.0 * rng.standard_normal((T, V))).astype(np.float32)
+    labels = rng.integers(0, V, size=T).astype(np.int32)
+    labels[[0, 9, 30]] = -1
+    dl = torch.from_numpy(logits).cuda()
+    row = torch.empty(T, dtype=torch.float32, device="cuda")
+    dlog = torch.full((T, ld), 7.0, dtype=torch.bfloat16, device="cuda")
+    loss = torch.empty(1, dtype=torch.float32, device="cuda")
+    cnt = torch.empty(1, dtype=torch.int32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    F.fl_k_cross_entropy(T, V, ld, dl, dev_i32(labels), row, dlog, loss, cnt, st)
+    torch.cuda.synchronize()
+    ref_loss, ref_d = O.cross_entropy(logits[:, :V].astype(np.float64), labels)
+    assert int(cnt.item()) == T - 3 and int(st.item()) == 0
+    assert abs(loss.item() - ref_loss) / ref_loss < 1e-5
+    got = f64(dlog)
+    assert not got[:, V:].any()
+    assert rel_inf(got[:, :V], ref_d) < 1e-2        # bf16 gradient
+    assert not got[[0, 9, 30]].any()
+
+
+def test_embedding_kernels(F):
+    rng = np.random.default_rng(5)
+    V, H, T = 300, 256, 77
+    table = rng.standard_normal((V, H)).astype(np.float32)
+    tb = syn.bf16_bits_to_f32(syn.f32_to_bf16_bits(table))
+    tokens = rng.integers(0, V, size=T).astype(np.int32)
+    tokens[[3, 4]] = tokens[2]                      # repeated ids: their gradients add up
+    tokens[10] = V                                  # out of range: zero row, flagged
+    out = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    F.fl_k_embedding_gather(T, H, dev_i32(tokens), bf16_dev(tb), V, out, st)
+    dx = rng.standard_normal((T, H))
+    dxb = syn.bf16_bits_to_f64(syn.f32_to_bf16_bits(dx.astype(np.float32)))
+    dE = torch.zeros((V, H), dtype=torch.float32, device="cuda")
+    F.fl_k_embedding_scatter_add(T, H, dev_i32(tokens), V, bf16_dev(dxb), dE)
+    torch.cuda.synchronize()
+    ok = tokens < V
+    want = np.zeros((T, H))
+    want[ok] = tb[tokens[ok]]
+    np.testing.assert_array_equal(f64(out), want)
+    assert int(st.item()) == 1
+    np.testing.assert_allclose(f64(dE), O.embedding_bwd(dxb[ok], tokens[ok], V), rtol=1e-6, atol=1e-5)
