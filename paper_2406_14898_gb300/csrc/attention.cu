@@ -242,23 +242,35 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
 }
 
 // ---------------------------------------------------------------------------- delta = rowsum(dO * O)
-__global__ void attn_delta_kernel(int T, int H, int nh, int hd, const bf16* __restrict__ O,
-                                  const bf16* __restrict__ dO, float* __restrict__ delta) {
-  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;  // (t, h) pair
-  const int lane = threadIdx.x & 31;
-  if (w >= (int64_t)T * nh) return;
-  const int t = int(w / nh), h = int(w % nh);
-  const bf16* o = O + (int64_t)t * H + h * hd;
-  const bf16* d = dO + (int64_t)t * H + h * hd;
+// G = HD/8 lanes per (token, head) pair, one 16-byte load of O and of dO each; pairs
+// ordered head-major so that a warp's pairs are consecutive tokens of one head (coalesced
+// delta stores).
+template <int HD>
+__global__ void __launch_bounds__(256) attn_delta_kernel(int T, int H, int nh, const bf16* __restrict__ O,
+                                                         const bf16* __restrict__ dO, float* __restrict__ delta) {
+  constexpr int G = HD / 8;
+  const int64_t gid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t p = gid / G;
+  const int sub = threadIdx.x % G;
+  const bool ok = p < (int64_t)T * nh;
   float s = 0.f;
-  for (int i = 2 * lane; i < hd; i += 64) {
-    const float2 a = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(o + i));
-    const float2 b = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(d + i));
-    s += a.x * b.x + a.y * b.y;
+  int h = 0, t = 0;
+  if (ok) {
+    h = int(p / T);
+    t = int(p % T);
+    const int64_t off = (int64_t)t * H + h * HD + sub * 8;
+    const uint4 a = __ldg(reinterpret_cast<const uint4*>(O + off));
+    const uint4 b = __ldg(reinterpret_cast<const uint4*>(dO + off));
+    const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 x = unpack_bf16x2(aw[e]), y = unpack_bf16x2(bw[e]);
+      s = fmaf(x.x, y.x, fmaf(x.y, y.y, s));
+    }
   }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-  if (lane == 0) delta[(int64_t)h * T + t] = s;
+  for (int off = G / 2; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  if (ok && sub == 0) delta[(int64_t)h * T + t] = s;
 }
 
 // Inverse rotary rotation of an accumulator fragment: the thread holds, for n-tile nt,
@@ -705,8 +717,8 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
   const int H = nh * HD;
   const float scale = 1.f / sqrtf((float)HD);
   const int64_t pairs = (int64_t)T * nh;
-  attn_delta_kernel<<<(unsigned)((pairs * 32 + 255) / 256), 256, 0, st>>>(T, H, nh, HD, (const bf16*)o,
-                                                                          (const bf16*)dout, delta);
+  attn_delta_kernel<HD><<<(unsigned)((pairs * (HD / 8) + 255) / 256), 256, 0, st>>>(T, H, nh, (const bf16*)o,
+                                                                                    (const bf16*)dout, delta);
   FL_CUDA_TRY(cudaGetLastError());
   const float2* tab = reinterpret_cast<const float2*>(rope_tab);
   const bf16* pk = (const bf16*)pre.k;

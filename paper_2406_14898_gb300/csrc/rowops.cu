@@ -126,43 +126,31 @@ __global__ void __launch_bounds__(512) ln_fwd_kernel(int T, int H, const TX* __r
 // Backward: dx = rstd (g - mean(g) - xhat mean(g xhat)), g = gamma dy (+ alpha resid);
 // thread c keeps its columns' dgamma / dbeta partials in registers across the CTA's rows
 // and writes them to workspace[blockIdx.x][2][H]; ln_bwd_reduce_kernel adds them up.
+// Kept at <= 64 registers (gamma re-read from L1 each row, no register prefetch of the
+// next row) so that two 512-thread CTAs share an SM and cover each other's latency.
 template <typename T>
-__global__ void __launch_bounds__(512) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy, const T* __restrict__ x,
-                                                     const float* __restrict__ mean,
-                                                     const float* __restrict__ rstd,
-                                                     const float* __restrict__ gamma, const T* __restrict__ resid,
-                                                     float resid_alpha, __nv_bfloat16* __restrict__ dx_bf16,
-                                                     float* __restrict__ dx_f32, float* __restrict__ ws) {
+__global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy,
+                                                        const T* __restrict__ x, const float* __restrict__ mean,
+                                                        const float* __restrict__ rstd,
+                                                        const float* __restrict__ gamma, const T* __restrict__ resid,
+                                                        float resid_alpha, __nv_bfloat16* __restrict__ dx_bf16,
+                                                        float* __restrict__ dx_f32, float* __restrict__ ws) {
   __shared__ float2 red[2][32];
   const int c = threadIdx.x;
-  float gcol[8], accg[8], accb[8];
-  load8<float>(gamma, c, gcol);
+  float accg[8], accb[8];
 #pragma unroll
   for (int k = 0; k < 8; ++k) accg[k] = accb[k] = 0.f;
   int par = 0;
-  float nd[8], nx[8];
-  int row = blockIdx.x;
-  if (row < Tn) {
-    load8<T>(dy + (int64_t)row * H, c, nd);
-    load8<T>(x + (int64_t)row * H, c, nx);
-  }
-  for (; row < Tn; row += gridDim.x) {
-    float d[8], xv[8];
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      d[k] = nd[k];
-      xv[k] = nx[k];
-    }
-    const int r2 = row + gridDim.x;
-    if (r2 < Tn) {
-      load8<T>(dy + (int64_t)r2 * H, c, nd);
-      load8<T>(x + (int64_t)r2 * H, c, nx);
-    }
+  for (int row = blockIdx.x; row < Tn; row += gridDim.x) {
+    float d[8], xh[8], gcol[8];
+    load8<T>(dy + (int64_t)row * H, c, d);
+    load8<T>(x + (int64_t)row * H, c, xh);
+    load8<float>(gamma, c, gcol);
     const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
-    float xh[8], s1 = 0.f, s2 = 0.f;
+    float s1 = 0.f, s2 = 0.f;
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-      xh[k] = (xv[k] - mu) * rs;
+      xh[k] = (xh[k] - mu) * rs;
       const float g = d[k] * gcol[k];
       s1 += g;
       s2 += g * xh[k];
@@ -251,6 +239,7 @@ __global__ void __launch_bounds__(256) colsum_kernel(int T, int N, const __nv_bf
   const int r1 = min(T, r0 + rows_per_block);
   float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
   if (col < N) {
+#pragma unroll 4
     for (int r = r0 + ry; r < r1; r += 8) {
       float f[8];
       unpack8(__ldg(reinterpret_cast<const uint4*>(x + (int64_t)r * N + col)), f);
@@ -466,7 +455,7 @@ extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void
   if (T < 0 || N <= 0 || (N % 8) || !x || !out) return fl_internal_error(FL_ERR_INVALID_ARG, "colsum: args");
   if (T == 0) return FL_OK;
   const int cblocks = (N + 255) / 256;
-  int rblocks = (2 * sm_count() + cblocks - 1) / cblocks;
+  int rblocks = (8 * sm_count() + cblocks - 1) / cblocks;  // ~8 CTAs (64 warps) per SM
   if (rblocks < 1) rblocks = 1;
   int rows = (T + rblocks - 1) / rblocks;
   rows = (rows + 7) / 8 * 8;
