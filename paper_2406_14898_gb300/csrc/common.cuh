@@ -47,14 +47,22 @@ FL_DEV float2 unpack_bf16x2(uint32_t u) {
 }
 
 // tanh-form GeLU and its derivative, with c = sqrt(2/pi), a = 0.044715.
+// tanh by the hardware instruction (PTX tanh.approx.f32, relative error about 2^-11): the
+// GeLU epilogues run on four warps per SM with nothing to hide an accurate tanhf's
+// instruction latency behind, and their bf16 outputs cannot resolve the difference.
+FL_DEV float tanh_hw(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 FL_DEV float gelu_tanh(float u) {
   const float c = 0.7978845608028654f, a = 0.044715f;
-  float t = tanhf(c * (u + a * u * u * u));
+  float t = tanh_hw(c * (u + a * u * u * u));
   return 0.5f * u * (1.f + t);
 }
 FL_DEV float gelu_tanh_grad(float u) {
   const float c = 0.7978845608028654f, a = 0.044715f;
-  float t = tanhf(c * (u + a * u * u * u));
+  float t = tanh_hw(c * (u + a * u * u * u));
   return 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * c * (1.f + 3.f * a * u * u);
 }
 

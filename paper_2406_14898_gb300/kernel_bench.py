@@ -56,6 +56,9 @@ def main():
     ap.add_argument("--workload", default="stack26")
     ap.add_argument("--kernel", default="all")
     ap.add_argument("--reps", type=int, default=5)
+    ap.add_argument("--wgrad-epilogue", default="store", choices=["store", "adamw"],
+                    help="epilogue of the weight-gradient GEMMs: fp32 store (the separate-step path) or the "
+                         "fused AdamW update of the backward + step call")
     args = ap.parse_args()
     cfg = syn.CONFIGS[args.workload]
     F.lib()
@@ -110,7 +113,19 @@ def main():
             kw.update(n_heads=nh, head_dim=hd, rotary_dim=hd // 2)
         lda = M if amn else K
         ldb = N if bmn else K
-        ms = timed(lambda: F.gemm(M, N, K, A, lda, amn, B, ldb, bmn, D, N, epilogue=epi, stream=st, **kw))
+        if epi == F.FL_EPI_STORE_F32 and args.wgrad_epilogue == "adamw":
+            # g = A . B^T updates fp32 weights D with their moments, writes the bf16 copy
+            mom = torch.zeros(2, M, N, device=dev, dtype=torch.float32)
+            wb16 = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
+            ga = F.fl_gemm_args(M, N, K, F.ptr(A), lda, amn, F.ptr(B), ldb, bmn, F.ptr(D), N, F.FL_EPI_ADAMW)
+            ga.aux_out, ga.ld_aux_out = F.ptr(wb16), N
+            ga.adam_m, ga.adam_v = F.ptr(mom[0]), F.ptr(mom[1])
+            ga.lr, ga.beta1, ga.beta2, ga.eps, ga.weight_decay = 1e-4, 0.9, 0.999, 1e-8, 0.0
+            ga.inv_bc1, ga.inv_bc2 = 10.0, 1000.0
+            ms = timed(lambda: F.fl_k_gemm(ga, stream=st))
+            name = name + "_adamw"
+        else:
+            ms = timed(lambda: F.gemm(M, N, K, A, lda, amn, B, ldb, bmn, D, N, epilogue=epi, stream=st, **kw))
         flops = 2.0 * M * N * K
         out.append({"kernel": f"gemm_{name}", "M": M, "N": N, "K": K, "ms": ms, "tflops": flops / ms / 1e9})
         del A, B, D, kw
