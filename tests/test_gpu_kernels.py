@@ -358,3 +358,41 @@ def test_attention_with_prefix(F, hd, Lp):
     assert rel_inf(got[:, 2 * H:], dvr.reshape(T, H)) < 5e-2
     assert rel_inf(f64(gpk) - 0.25, dpkr.reshape(Lp, H)) < 5e-2   # accumulated onto the 0.25
     assert rel_inf(f64(gpv), dpvr.reshape(Lp, H)) < 5e-2
+
+
+@pytest.mark.parametrize("M,N,K,mn", [(200, 384, 136, 1), (256, 512, 64, 1), (130, 256, 96, 0)])
+def test_gemm_adamw_epilogue(F, M, N, K, mn):
+    """The weight-gradient GEMM with the AdamW update in its epilogue equals the plain fp32
+    gradient GEMM followed by the separate AdamW kernel: weights, moments and the bf16
+    copy; ragged rows, both tile widths (N = 384 takes 128-column tiles)."""
+    rng = np.random.default_rng(M + N)
+    A = rnd_bf16_f64(rng, (M, K))
+    B = rnd_bf16_f64(rng, (N, K))
+    dA, lda = _store(A, bool(mn))
+    dB, ldb = _store(B, bool(mn))
+    w0 = (0.05 * rng.standard_normal((M, N))).astype(np.float32)
+    m0 = (0.01 * rng.standard_normal((M, N))).astype(np.float32)
+    v0 = (1e-3 * rng.random((M, N))).astype(np.float32)
+    lr, b1, b2, eps, wd, t = 1e-3, 0.9, 0.999, 1e-8, 0.01, 3
+    bc1, bc2 = 1.0 - b1 ** t, 1.0 - b2 ** t
+    # reference: g = A B^T stored in fp32, then fl_k_adamw
+    g = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    F.gemm(M, N, K, dA, lda, mn, dB, ldb, mn, g, N, epilogue=F.FL_EPI_STORE_F32)
+    wr, mr, vr = dev_f32(w0), dev_f32(m0), dev_f32(v0)
+    wbr = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    F.fl_k_adamw(M * N, wr, g, mr, vr, wbr, lr, b1, b2, eps, wd, bc1, bc2)
+    # fused
+    wf, mf, vf = dev_f32(w0), dev_f32(m0), dev_f32(v0)
+    wbf = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    ga = F.fl_gemm_args(M, N, K, F.ptr(dA), lda, mn, F.ptr(dB), ldb, mn, F.ptr(wf), N, F.FL_EPI_ADAMW)
+    ga.aux_out, ga.ld_aux_out = F.ptr(wbf), N
+    ga.adam_m, ga.adam_v = F.ptr(mf), F.ptr(vf)
+    ga.lr, ga.beta1, ga.beta2, ga.eps, ga.weight_decay = lr, b1, b2, eps, wd
+    ga.inv_bc1, ga.inv_bc2 = 1.0 / np.float32(bc1), 1.0 / np.float32(bc2)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    F.fl_k_gemm(ga, status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    for got, want in ((wf, wr), (mf, mr), (vf, vr)):
+        assert rel_inf(f64(got), f64(want)) < 1e-5
+    np.testing.assert_array_equal(bits(wbf), bits(wf.to(torch.bfloat16)))
