@@ -4,12 +4,15 @@
 // (§4.1.1): with context length c, query t sees the keys u <= max(t, c - 1), i.e. the
 // context is bidirectional and the answer span causal; c = 0 is the plain causal case.
 //
-// Forward: one CTA per (64-query tile, head); online softmax over 64-key tiles with
-// cp.async double buffering and bf16 mma.sync m16n8k16 (fp32 accumulate).  Saves O (bf16)
-// and the row log-sum-exp (fp32).
+// Forward: one CTA per (64-query tile, head); online softmax over 64-key tiles with bf16
+// mma.sync m16n8k16 (fp32 accumulate).  Saves O (bf16) and the row log-sum-exp (fp32).
+// One K/V tile buffer and Q fragments re-read from shared memory per key tile: 52 KB of
+// shared memory and 128 registers, so four CTAs share an SM and hide each other's copy
+// latency (double buffering inside the CTA would cap it at two).
 // Backward, deterministic, no atomics:
 //   delta = rowsum(dO * O);
-//   dQ  kernel: per (query tile, head), loop over key tiles: P, dP = dO V^T, dS, dQ += dS K;
+//   dQ  kernel: per (query tile, head), loop over key tiles: P, dP = dO V^T, dS, dQ += dS K
+//               (one K/V buffer, 70 KB of shared memory: three CTAs per SM);
 //   dKV kernel: per (key tile, head), loop over query tiles: dV += P^T dO, dK += dS^T Q;
 // dQ and dK leave through the inverse rotary rotation (the forward rotation is applied in
 // the QKV GEMM epilogue), so the result is the gradient w.r.t. the un-rotated q and k.
@@ -90,7 +93,7 @@ FL_DEV void decode_tile(uint32_t t, int& s, int& idx) {
 
 // ---------------------------------------------------------------------------- forward
 template <int HD>
-__global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16* __restrict__ qkv,
+__global__ void __launch_bounds__(128, 4) attn_fwd_kernel(int T, int H, const bf16* __restrict__ qkv,
                                                        const int32_t* __restrict__ cu,
                                                        const uint32_t* __restrict__ tiles, bf16* __restrict__ O,
                                                        float* __restrict__ lse, float scale_log2,
@@ -98,8 +101,8 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
                                                        int Lp, const int32_t* __restrict__ ctxs) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
-  bf16* sK = sQ + AT<HD>::TILE_ELEMS;      // [2] tiles
-  bf16* sV = sK + 2 * AT<HD>::TILE_ELEMS;  // [2] tiles
+  bf16* sK = sQ + AT<HD>::TILE_ELEMS;      // one tile
+  bf16* sV = sK + AT<HD>::TILE_ELEMS;      // one tile
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   int s, idx;
   decode_tile(tiles[blockIdx.x], s, idx);
@@ -117,54 +120,44 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
   const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;  // last context key, -1 without a context
   const int n_kv = npt + max(idx, clast >= 0 ? clast / BT : 0) + 1;
   const int qlim0 = max(q0, clast);              // smallest key limit among the tile's queries
-  auto load_kv = [&](int t, int buf) {
+  auto load_kv = [&](int t) {
     if (t < npt) {
       const int k0 = t * BT;
-      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, pk + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
-      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, pv + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+      load_tile<HD>(sK, pk + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+      load_tile<HD>(sV, pv + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
     } else {
       const int k0 = (t - npt) * BT;
-      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, gK + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
-      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, gV + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+      load_tile<HD>(sK, gK + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+      load_tile<HD>(sV, gV + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
     }
   };
   load_tile<HD>(sQ, gQ, ld, min(BT, L - q0), tid);
-  load_kv(0, 0);
+  load_kv(0);
   cp_async_commit();
 
   float o[HD / 8][4];
 #pragma unroll
   for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
-  uint32_t qf[HD / 16][4];
 
   for (int j = 0; j < n_kv; ++j) {
-    const int buf = j & 1;
-    if (j + 1 < n_kv) {
-      load_kv(j + 1, buf ^ 1);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
+    cp_async_wait<0>();
     __syncthreads();
-    if (j == 0) {
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) ld_a<HD>(sQ, warp * 16, kk * 16, lane, qf[kk]);
-    }
-    const bf16* K = sK + buf * AT<HD>::TILE_ELEMS;
-    const bf16* V = sV + buf * AT<HD>::TILE_ELEMS;
+    const bf16* K = sK;
+    const bf16* V = sV;
     float sc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < HD / 16; ++kk) {
+      uint32_t qa[4];
+      ld_a<HD>(sQ, warp * 16, kk * 16, lane, qa);
 #pragma unroll
       for (int np = 0; np < 4; ++np) {
         uint32_t b[4];
         ld_b_rows<HD>(K, np * 16, kk * 16, lane, b);
-        mma_bf16_16816(sc[2 * np], qf[kk], b[0], b[1]);
-        mma_bf16_16816(sc[2 * np + 1], qf[kk], b[2], b[3]);
+        mma_bf16_16816(sc[2 * np], qa, b[0], b[1]);
+        mma_bf16_16816(sc[2 * np + 1], qa, b[2], b[3]);
       }
     }
     const int kb = (j - npt) * BT;  // first key of a segment tile
@@ -224,6 +217,10 @@ __global__ void __launch_bounds__(128) attn_fwd_kernel(int T, int H, const bf16*
       }
     }
     __syncthreads();
+    if (j + 1 < n_kv) {  // every warp is done with the tile: load the next one into it
+      load_kv(j + 1);
+      cp_async_commit();
+    }
   }
 
 #pragma unroll
@@ -322,8 +319,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
   bf16* sdO = sQ + AT<HD>::TILE_ELEMS;
-  bf16* sK = sdO + AT<HD>::TILE_ELEMS;     // [2]
-  bf16* sV = sK + 2 * AT<HD>::TILE_ELEMS;  // [2]
+  bf16* sK = sdO + AT<HD>::TILE_ELEMS;  // one tile
+  bf16* sV = sK + AT<HD>::TILE_ELEMS;   // one tile
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   int s, idx;
   decode_tile(tiles[blockIdx.x], s, idx);
@@ -337,20 +334,20 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
   const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
   const int n_kv = npt + max(idx, clast >= 0 ? clast / BT : 0) + 1;
   const int qlim0 = max(q0, clast);
-  auto load_kv = [&](int t, int buf) {
+  auto load_kv = [&](int t) {
     if (t < npt) {
       const int k0 = t * BT;
-      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, pk + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
-      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, pv + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+      load_tile<HD>(sK, pk + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
+      load_tile<HD>(sV, pv + (int64_t)k0 * H + h * HD, H, min(BT, Lp - k0), tid);
     } else {
       const int k0 = (t - npt) * BT;
-      load_tile<HD>(sK + buf * AT<HD>::TILE_ELEMS, gK + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
-      load_tile<HD>(sV + buf * AT<HD>::TILE_ELEMS, gV + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+      load_tile<HD>(sK, gK + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
+      load_tile<HD>(sV, gV + (int64_t)k0 * ld, ld, min(BT, L - k0), tid);
     }
   };
   load_tile<HD>(sQ, qkv + (int64_t)(seg0 + q0) * ld + h * HD, ld, min(BT, L - q0), tid);
   load_tile<HD>(sdO, dO + (int64_t)(seg0 + q0) * H + h * HD, H, min(BT, L - q0), tid);
-  load_kv(0, 0);
+  load_kv(0);
   cp_async_commit();
 
   const float scale_log2 = scale * LOG2E;
@@ -366,17 +363,10 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
   for (int i = 0; i < HD / 8; ++i) dq[i][0] = dq[i][1] = dq[i][2] = dq[i][3] = 0.f;
 
   for (int j = 0; j < n_kv; ++j) {
-    const int buf = j & 1;
-    if (j + 1 < n_kv) {
-      load_kv(j + 1, buf ^ 1);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
+    cp_async_wait<0>();
     __syncthreads();
-    const bf16* K = sK + buf * AT<HD>::TILE_ELEMS;
-    const bf16* V = sV + buf * AT<HD>::TILE_ELEMS;
+    const bf16* K = sK;
+    const bf16* V = sV;
     float sc[8][4], dp[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
@@ -432,6 +422,10 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
       }
     }
     __syncthreads();
+    if (j + 1 < n_kv) {  // every warp is done with the tile: load the next one into it
+      load_kv(j + 1);
+      cp_async_commit();
+    }
   }
 
 #pragma unroll
@@ -664,9 +658,9 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
 }
 
 template <int HD>
-constexpr int fwd_smem() { return 5 * AT<HD>::TILE_BYTES; }
+constexpr int fwd_smem() { return 3 * AT<HD>::TILE_BYTES; }
 template <int HD>
-constexpr int dq_smem() { return 6 * AT<HD>::TILE_BYTES; }
+constexpr int dq_smem() { return 4 * AT<HD>::TILE_BYTES; }
 template <int HD>
 constexpr int dkv_smem() { return 6 * AT<HD>::TILE_BYTES + 4 * BT * 4; }
 
