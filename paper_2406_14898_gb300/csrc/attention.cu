@@ -760,9 +760,9 @@ int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles) {
 }
 
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
-                       void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
+                       void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st, int* status) {
   if (n_tiles <= 0) return FL_OK;
-  if (hd == 128) return launch_fwd<128>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, st);
+  if (hd == 128) return fl_launch_attn_fwd_tc(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, status, st);
   if (hd == 64) return launch_fwd<64>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }

@@ -80,9 +80,14 @@ struct AttnGlm {
 };
 
 // Attention on a device tile list (built by fl_launch_meta).
+// head_dim 128 runs on tcgen05 (attention_tc.cu), head_dim 64 on mma.sync; `status`
+// (device int or null) receives a code if a bounded wait inside the kernel gave up.
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
                        int n_tiles, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm,
-                       cudaStream_t st);
+                       cudaStream_t st, int* status = nullptr);
+int fl_launch_attn_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
+                          void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
+                          cudaStream_t st);
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
                        void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st);

@@ -341,7 +341,7 @@ int block_forward(fl_server* h, int b) {
   // o = causal attention within each segment
   prof_begin(h, FL_PROF_ATTN);
   TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse,
-                            h->prefix(b, false), h->glm_args(), st));
+                            h->prefix(b, false), h->glm_args(), st, h->status));
   prof_end(h);
   // h = alpha * (LN1(x) or x) + o Wd^T + bd, fp32; LN1(x) recomputed in fp32 in the epilogue
   fl_gemm_args g2 = gemm_fwd(T, H, H, A.o, h->wbt(b, FL_T_WDENSE), A.h, FL_EPI_BIAS_RESID);
