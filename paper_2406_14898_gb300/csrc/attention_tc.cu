@@ -139,47 +139,44 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
       break;
     }
     tc_fence_after();
-    // ---- masked row max (pass 1)
+    // ---- the thread's S row, read once (4 x 32 columns, one wait)
     const bool prefix = j < npt;
     const int kb = prefix ? 0 : (j - npt) * TBK;  // first key of the tile inside its sequence
     const int klim = prefix ? Lp - 1 : min(L - 1, max(q, clast));  // last visible key
+    const bool full = kb + TBK - 1 <= klim;      // every key of the tile visible to this row
+    uint32_t r[TBK];
+    tmem_ld32(t_s, *reinterpret_cast<uint32_t(*)[32]>(r));
+    tmem_ld32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
+    tmem_ld32(t_s + 64, *reinterpret_cast<uint32_t(*)[32]>(r + 64));
+    tmem_ld32(t_s + 96, *reinterpret_cast<uint32_t(*)[32]>(r + 96));
+    tmem_ld_wait();
+    // masked row max; invisible keys become -inf
     float mt = -INFINITY;
-#pragma unroll 1
-    for (int c = 0; c < TBK; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(t_s + c, r);
-      tmem_ld_wait();
 #pragma unroll
-      for (int e = 0; e < 32; ++e)
-        if (kb + c + e <= klim) mt = fmaxf(mt, __uint_as_float(r[e]) * scale_log2);
+    for (int e = 0; e < TBK; ++e) {
+      float x = __uint_as_float(r[e]) * scale_log2;
+      if (!full && kb + e > klim) x = -INFINITY;
+      r[e] = __float_as_uint(x);
+      mt = fmaxf(mt, x);
     }
     const float m_new = fmaxf(m_run, mt);
     const float mref = m_new == -INFINITY ? 0.f : m_new;
     const float corr = exp2f(m_run - mref);  // 0 on the first tile (m_run = -inf)
-    // ---- P = exp2(S - m) (pass 2) into the K buffer: row `tid`, 16-byte chunk c of the
-    // 64-key box b at position c ^ (row & 7), the layout of a 128-byte-swizzled TMA box
+    // ---- P = exp2(S - m) into the K buffer: row `tid`, 16-byte chunk c of the 64-key box b
+    // at position c ^ (row & 7), the layout of a 128-byte-swizzled TMA box
     float lt = 0.f;
-#pragma unroll 1
-    for (int c = 0; c < TBK; c += 32) {
-      uint32_t r[32];
-      tmem_ld32(t_s + c, r);
-      tmem_ld_wait();
-      uint32_t pk2[16];
 #pragma unroll
-      for (int e = 0; e < 32; e += 2) {
-        float p0 = 0.f, p1 = 0.f;
-        if (kb + c + e <= klim) p0 = exp2f(__uint_as_float(r[e]) * scale_log2 - mref);
-        if (kb + c + e + 1 <= klim) p1 = exp2f(__uint_as_float(r[e + 1]) * scale_log2 - mref);
-        lt += p0 + p1;
-        pk2[e >> 1] = pack_bf16x2(p0, p1);
-      }
-      uint8_t* row = sK + (c >> 6) * BOX + tid * 128;
+    for (int c = 0; c < TBK; c += 8) {
+      float p[8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int chunk = ((c & 63) >> 3) + u;  // 16-byte chunk inside the 128-byte row
-        *reinterpret_cast<uint4*>(row + ((chunk ^ (tid & 7)) << 4)) =
-            make_uint4(pk2[4 * u], pk2[4 * u + 1], pk2[4 * u + 2], pk2[4 * u + 3]);
+      for (int e = 0; e < 8; ++e) {
+        p[e] = exp2f(__uint_as_float(r[c + e]) - mref);
+        lt += p[e];
       }
+      const int chunk = (c & 63) >> 3;
+      *reinterpret_cast<uint4*>(sK + (c >> 6) * BOX + tid * 128 + ((chunk ^ (tid & 7)) << 4)) =
+          make_uint4(pack_bf16x2(p[0], p[1]), pack_bf16x2(p[2], p[3]), pack_bf16x2(p[4], p[5]),
+                     pack_bf16x2(p[6], p[7]));
     }
     l_run = l_run * corr + lt;
     m_run = m_new;
