@@ -740,12 +740,16 @@ def ncu_traffic(path: str, workload_name: str):
 
 
 def kernel_version() -> str:
-    """Fingerprint of the GEMM sources, so that stored ncu traffic is used only for the
-    kernel it was measured on."""
+    """Fingerprint of the GEMM sources (the kernel, its instantiations and the device
+    helpers its epilogues call), so that stored ncu traffic is used only for the kernel it
+    was measured on."""
     import glob
     import hashlib
     h = hashlib.sha256()
-    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2406_14898_gb300", "csrc", "gemm_*"))):
+    csrc = os.path.join(ROOT, "paper_2406_14898_gb300", "csrc")
+    files = sorted(glob.glob(os.path.join(csrc, "gemm_*"))) + [os.path.join(csrc, "common.cuh"),
+                                                                 os.path.join(csrc, "ptx.cuh")]
+    for f in files:
         h.update(open(f, "rb").read())
     return h.hexdigest()[:16]
 
