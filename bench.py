@@ -74,6 +74,13 @@ def gemm_flops(cfg: syn.ServerConfig) -> float:
     return float(cfg.n_blocks * passes * 2 * T * (4 * H * H + 2 * H * F))
 
 
+def recompute_flops(cfg: syn.ServerConfig) -> float:
+    """GEMM work the backward repeats with activation recompute: the QKV, dense and FFN-up
+    forward contractions of every block, 2T(3H^2 + H^2 + HF) each (not algorithmic work)."""
+    H, F, T = cfg.hidden, cfg.ffn_hidden, cfg.tokens
+    return float(cfg.n_blocks * 2 * T * (4 * H * H + H * F))
+
+
 def attn_flops(cfg: syn.ServerConfig) -> float:
     """Attention: 4 H FLOPs per visible (query, key) pair forward and 2.5x that backward,
     per block.  Causal: L (L+1) / 2 pairs per segment; a GLM segment with context c sees
@@ -258,6 +265,9 @@ def main():
     ap.add_argument("--glm", action="store_true",
                     help="GLM blank-infilling segments (the paper's task format): each segment a bidirectional "
                          "context with a mask token and a causal answer span, GLM 2D positions")
+    ap.add_argument("--recompute", action="store_true",
+                    help="keep only the block inputs and recompute each block's activations in the backward "
+                         "(for workloads whose activations do not fit, e.g. --workload sweep26_K64)")
     ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
@@ -302,7 +312,8 @@ def main():
     dev = torch.device("cuda", local_rank)
     F.lib()
     stream = torch.cuda.Stream(device=dev)
-    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens)), cfg.seed, stream=stream)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens), recompute=int(args.recompute)), cfg.seed,
+                   stream=stream)
 
     states_bits = syn.client_states(cfg)
     grads_bits = syn.client_grads(cfg)
@@ -315,6 +326,7 @@ def main():
     outs = [torch.empty_like(s) for s in states]
     gins = [torch.empty_like(s) for s in states]
     torch.cuda.synchronize()
+    free_b, total_b = torch.cuda.mem_get_info(dev)
 
     gk = glm_args(cfg)
 
@@ -375,7 +387,9 @@ def main():
     pk = peaks()
     flops = gemm_flops(cfg) + attn_flops(cfg)
     gemm_ms, gemm_n = prof["gemm"]
-    gemm_per_launch_flops = gemm_flops(cfg) * args.steps / max(gemm_n, 1)
+    # executed contractions per GEMM launch: the recomputed forward GEMMs are work the kernel does
+    gemm_exec = gemm_flops(cfg) + (recompute_flops(cfg) if args.recompute else 0.0)
+    gemm_per_launch_flops = gemm_exec * args.steps / max(gemm_n, 1)
     achieved = gemm_per_launch_flops / (gemm_ms / max(gemm_n, 1) / 1e3) / 1e12
     traffic = ncu_traffic(args.ncu_traffic, cfg.name)
 
@@ -433,7 +447,11 @@ def main():
                              "than L2; no flush needed",
                        "step": "pack + forward + unpack + backward with the AdamW update of every parameter "
                                "(fl_server_forward + fl_server_backward_step: the weight-matrix update runs in "
-                               "the weight-gradient GEMM epilogues)"},
+                               "the weight-gradient GEMM epilogues)",
+                       "recompute": (f"on: each block's activations recomputed in the backward "
+                                     f"({recompute_flops(cfg) / 1e12:.1f} TFLOP per step beyond the algorithmic "
+                                     f"FLOPs; counted in roofline.achieved, not in pct_bf16_peak)")
+                       if args.recompute else "off: every activation kept"},
             "pct_bf16_peak": 100.0 * flops / (ms_step / 1e3) / (pk["bf16_sustained"] * 1e12),
             "pct_bf16_peak_basis": f"algorithmic FLOPs (GEMM + causal attention) of the whole step over the "
                                    f"{pk['source']} sustained bf16 peak {pk['bf16_sustained']} TFLOP/s",
@@ -452,6 +470,7 @@ def main():
                          "share_of_step": gemm_ms / ms},
             "gpu_launches": launches,
             "clocks": clk,
+            "hbm_used_gb": (total_b - free_b) / 1e9,
         }
         if cpu is not None:
             line["cpu_baseline"] = {"value": cpu["tokens_per_s"], "unit": "tokens/s", "cores": cpu_cores(),

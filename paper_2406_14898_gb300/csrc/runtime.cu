@@ -15,7 +15,9 @@
 //   activations       per block: LN1 out A, rotated QKV, attention O, LSE, residual stream
 //                     Hres (fp32), LN2 out M, FFN pre-activation U and GeLU output G, LN
 //                     statistics; xs[0..n_blocks]: block inputs / outputs in fp32
-//                     (xs[0] = packed client states, widened exactly);
+//                     (xs[0] = packed client states, widened exactly); with cfg.recompute
+//                     only one block's set, refilled before each block's backward by
+//                     running that block's forward again from its kept input xs[b];
 //   backward scratch  one set of gradient buffers reused by every block; the gradient of
 //                     the residual stream is kept in fp32 next to the bf16 copy the GEMMs
 //                     read;
@@ -114,7 +116,8 @@ struct fl_server {
 
   // activations
   std::vector<float*> xs;  // block inputs/outputs, fp32
-  std::vector<BlockAct> act;
+  std::vector<BlockAct> act;  // one per block, or a single shared set with recompute
+  BlockAct& act_of(int b) { return act[cfg.recompute ? 0 : b]; }
   // backward scratch: gradient of a block's output / input as bf16 (GEMM operand) and
   // fp32 (residual chain), ping-pong
   __nv_bfloat16 *dy = nullptr, *dx = nullptr, *du = nullptr, *dh = nullptr, *d_o = nullptr, *dqkv = nullptr;
@@ -236,7 +239,7 @@ int validate_cfg(const fl_server_cfg& c, int* rdim) {
   if (rd != c.head_dim / 2) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: rotary_dim must be head_dim/2");
   if (c.max_tokens < 1) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: max_tokens < 1");
   if (c.client_batch < 1) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: client_batch < 1");
-  if (c.recompute != 0) return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: recompute is not built");
+  if (c.recompute != 0 && c.recompute != 1) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: recompute must be 0 or 1");
   if (!(c.ln_eps > 0.f) || !(c.rope_base > 1.f)) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: ln_eps/rope_base");
   if (c.residual_from_ln != 0 && c.residual_from_ln != 1)
     return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: residual_from_ln must be 0 or 1");
@@ -317,10 +320,13 @@ fl_gemm_args gemm_wgrad(fl_server* h, int b, int t, int T, int Nout, int Kin, co
     if (_rc != FL_OK) return fwd_err(h, _rc); \
   } while (0)
 
-int block_forward(fl_server* h, int b) {
+// Forward of block b from xs[b] into its activations and xs[b + 1].  Without `output`
+// (recomputing the activations for the backward) the FFN down-projection, whose result
+// xs[b + 1] is already kept and which the backward does not read, is skipped.
+int block_forward(fl_server* h, int b, bool output = true) {
   const fl_server_cfg& c = h->cfg;
   const int T = h->T, H = c.hidden, F = c.ffn_hidden;
-  BlockAct& A = h->act[b];
+  BlockAct& A = h->act_of(b);
   const float* x = h->xs[b];
   cudaStream_t st = h->stream;
   // a = LN1(x)
@@ -369,6 +375,7 @@ int block_forward(fl_server* h, int b) {
   g3.aux_out = A.u;
   g3.ld_aux_out = F;
   TRY(h, run_gemm(h, g3));
+  if (!output) return FL_OK;
   // y = alpha * (LN2(h) or h) + g W2^T + b2, fp32
   fl_gemm_args g4 = gemm_fwd(T, H, F, A.g, h->wbt(b, FL_T_WDOWN), h->xs[b + 1], FL_EPI_BIAS_RESID);
   g4.bias = h->wt(b, FL_T_BDOWN);
@@ -393,7 +400,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   const int T = h->T, H = c.hidden, F = c.ffn_hidden;
   const float al = c.residual_alpha;
   const bool glm = c.residual_from_ln != 0;
-  BlockAct& A = h->act[b];
+  BlockAct& A = h->act_of(b);
   cudaStream_t st = h->stream;
   const bool train_base = !c.freeze_base;
   // FFN down: du = (dy W2) * gelu'(u); dW2 += dy^T g; db2 += colsum(dy)
@@ -574,8 +581,8 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
   h->xs.resize(c.n_blocks + 1);
   for (int b = 0; b <= c.n_blocks; ++b)
     if ((rc = dalloc(h, &h->xs[b], Tm * H))) return fail(rc);  // fp32
-  h->act.resize(c.n_blocks);
-  for (int b = 0; b < c.n_blocks; ++b) {
+  h->act.resize(c.recompute ? 1 : c.n_blocks);
+  for (size_t b = 0; b < h->act.size(); ++b) {
     BlockAct& A = h->act[b];
     if ((rc = dalloc(h, &A.a, Tm * H)) || (rc = dalloc(h, &A.qkv, Tm * 3 * H)) || (rc = dalloc(h, &A.o, Tm * H)) ||
         (rc = dalloc(h, &A.h, Tm * H)) || (rc = dalloc(h, &A.m, Tm * H)) || (rc = dalloc(h, &A.u, Tm * F)) ||
@@ -731,6 +738,10 @@ static int backward_impl(fl_server_t h, const void* const grad_out[], void* cons
   float* curf = h->dyf;
   float* nxtf = h->dxf;
   for (int blk = h->cfg.n_blocks - 1; blk >= 0; --blk) {
+    // with recompute the shared activations hold another block's (or stale) values:
+    // refill them from the kept block input; every kernel is deterministic, so they are
+    // the same bits the forward computed
+    if (h->cfg.recompute && (rc = block_forward(h, blk, false))) return rc;
     if ((rc = block_backward(h, blk, cur, curf, nxt, nxtf))) return rc;
     std::swap(cur, nxt);
     std::swap(curf, nxtf);

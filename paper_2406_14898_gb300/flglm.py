@@ -173,9 +173,10 @@ def _parr(xs) -> "C.Array":
     return (C.c_void_p * len(xs))(*[ptr(x) for x in xs])
 
 
-def make_cfg(c, max_tokens: int, max_seq_len: int = 0) -> fl_server_cfg:
+def make_cfg(c, max_tokens: int, max_seq_len: int = 0, recompute: int = 0) -> fl_server_cfg:
     """fl_server_cfg from a workload description with the attributes of
-    ``synthetic.ServerConfig`` (n_blocks, hidden, ... , weight_decay)."""
+    ``synthetic.ServerConfig`` (n_blocks, hidden, ... , weight_decay); ``recompute``
+    keeps one block's activations and recomputes the rest in the backward."""
     cfg = fl_server_cfg()
     lib().fl_server_cfg_default(C.byref(cfg))
     cfg.n_blocks = c.n_blocks
@@ -191,7 +192,7 @@ def make_cfg(c, max_tokens: int, max_seq_len: int = 0) -> fl_server_cfg:
     cfg.client_batch = c.client_batch
     cfg.max_tokens = max_tokens
     cfg.max_seq_len = max_seq_len
-    cfg.recompute = 0
+    cfg.recompute = recompute
     cfg.init_std = c.init_std
     cfg.adam_beta1 = c.adam_beta1
     cfg.adam_beta2 = c.adam_beta2
