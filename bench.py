@@ -460,7 +460,7 @@ def main():
             "fwd_bwd_basis": "separate timed loop of fl_server_forward + fl_server_backward, no optimizer step",
             "vector_adamw_ms": adam_ms,
             "kernel_ms_per_step": {k: v[0] / args.steps for k, v in prof.items()},
-            "roofline": {"kernel": "gemm_tc_kernel (tcgen05)", "bound": "tensor", "achieved": achieved,
+            "roofline": {"kernel": "gemm_pair_kernel (tcgen05.mma.cta_group::2, 256 x 256 tiles on SM pairs)", "bound": "tensor", "achieved": achieved,
                          "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
                          "peak_basis": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
                          "traffic": traffic["bytes_per_launch"] if traffic else None,

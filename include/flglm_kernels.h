@@ -44,6 +44,13 @@ enum {
   FL_EPI_COUNT
 };
 
+/* Tile shapes of fl_gemm_args.tile. */
+#define FL_TILE_AUTO 0
+#define FL_TILE_128x128 1      /* one SM per 128 x 128 tile */
+#define FL_TILE_128x256 2      /* one SM per 128 x 256 tile (N % 256 == 0) */
+#define FL_TILE_256x256_PAIR 3 /* a cluster of two SMs per 256 x 256 tile, tcgen05.mma.cta_group::2
+                                  (N % 256 == 0) */
+
 /* D[M,N] = epilogue(A . B^T) with bf16 operands.
  * A(m,k) is A[m*lda + k] when a_mn_major == 0 (row-major [M,K]) and A[k*lda + m] when
  * a_mn_major == 1 (row-major [K,M]); B(n,k) likewise with ldb / b_mn_major.
@@ -81,6 +88,9 @@ typedef struct {
   const int32_t* pos2;                      /* [M] GLM block positions for BIAS_ROPE, or NULL: dims
                                                [rotary_dim, 2*rotary_dim) of each q/k head then turn
                                                by pos2 (2D rotary; needs rotary_dim = head_dim/2) */
+  int32_t tile;                             /* FL_TILE_*: tile shape, FL_TILE_AUTO (0) lets the library
+                                               pick (256-column tiles on CTA pairs unless smaller tiles
+                                               leave clearly fewer SMs idle in the last wave) */
 } fl_gemm_args;
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);

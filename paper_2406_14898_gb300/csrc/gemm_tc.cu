@@ -5,6 +5,8 @@
 
 namespace fl_gemm {
 #define FL_GEMM_EXTERN(AMN, BMN, FAM)                                                                   \
+  extern template int pair_slots<AMN, BMN, FAM>();                                                      \
+  extern template int launch_pair<AMN, BMN, FAM>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
   extern template int launch<256, AMN, BMN, FAM>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
   extern template int launch<128, AMN, BMN, FAM>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);
 #define FL_GEMM_EXTERN_ALL(AMN, BMN)                                                                   \
@@ -14,8 +16,19 @@ FL_GEMM_EXTERN_ALL(false, false)
 FL_GEMM_EXTERN_ALL(false, true)
 FL_GEMM_EXTERN_ALL(true, true)
 
+// Tile shape: 0 = 128 x 128 on one SM, 1 = 128 x 256 on one SM, 2 = 256 x 256 on a CTA pair.
 template <bool AMN, bool BMN>
-int dispatch_layout(int fam, bool wide, const fl_gemm_args* a, const Epi& e, int* status, cudaStream_t st) {
+int dispatch_layout(int fam, int shape, const fl_gemm_args* a, const Epi& e, int* status, cudaStream_t st) {
+  if (shape == 2) {
+    switch (fam) {
+      case FAM_GELU: return launch_pair<AMN, BMN, FAM_GELU>(a, e, status, st);
+      case FAM_RESID: return launch_pair<AMN, BMN, FAM_RESID>(a, e, status, st);
+      case FAM_ROPE: return launch_pair<AMN, BMN, FAM_ROPE>(a, e, status, st);
+      case FAM_ADAMW: return launch_pair<AMN, BMN, FAM_ADAMW>(a, e, status, st);
+      default: return launch_pair<AMN, BMN, FAM_PLAIN>(a, e, status, st);
+    }
+  }
+  const bool wide = shape == 1;
   switch (fam) {
     case FAM_GELU: return wide ? launch<256, AMN, BMN, FAM_GELU>(a, e, status, st) : launch<128, AMN, BMN, FAM_GELU>(a, e, status, st);
     case FAM_RESID: return wide ? launch<256, AMN, BMN, FAM_RESID>(a, e, status, st) : launch<128, AMN, BMN, FAM_RESID>(a, e, status, st);
@@ -25,11 +38,26 @@ int dispatch_layout(int fam, bool wide, const fl_gemm_args* a, const Epi& e, int
   }
 }
 
-int dispatch_fam(int fam, bool wide, bool amn, bool bmn, const fl_gemm_args* a, const Epi& e, int* status,
+int dispatch_fam(int fam, int shape, bool amn, bool bmn, const fl_gemm_args* a, const Epi& e, int* status,
                  cudaStream_t st) {
-  if (!amn && !bmn) return dispatch_layout<false, false>(fam, wide, a, e, status, st);
-  if (!amn && bmn) return dispatch_layout<false, true>(fam, wide, a, e, status, st);
-  return dispatch_layout<true, true>(fam, wide, a, e, status, st);
+  if (!amn && !bmn) return dispatch_layout<false, false>(fam, shape, a, e, status, st);
+  if (!amn && bmn) return dispatch_layout<false, true>(fam, shape, a, e, status, st);
+  return dispatch_layout<true, true>(fam, shape, a, e, status, st);
+}
+
+int pair_slots_for(int fam, bool amn, bool bmn) {
+#define FL_SLOTS(AMN, BMN)                                          \
+  switch (fam) {                                                    \
+    case FAM_GELU: return pair_slots<AMN, BMN, FAM_GELU>();         \
+    case FAM_RESID: return pair_slots<AMN, BMN, FAM_RESID>();       \
+    case FAM_ROPE: return pair_slots<AMN, BMN, FAM_ROPE>();         \
+    case FAM_ADAMW: return pair_slots<AMN, BMN, FAM_ADAMW>();       \
+    default: return pair_slots<AMN, BMN, FAM_PLAIN>();              \
+  }
+  if (!amn && !bmn) { FL_SLOTS(false, false) }
+  if (!amn && bmn) { FL_SLOTS(false, true) }
+  FL_SLOTS(true, true)
+#undef FL_SLOTS
 }
 }  // namespace fl_gemm
 
@@ -111,17 +139,35 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   e.inv_bc2 = a->inv_bc2;
 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  // Tile width: 256 columns unless 128 gives clearly fewer idle SM slots in the last wave.
-  bool wide = (a->N % 256) == 0;
-  if (wide) {
-    const int sms = num_sms();
-    const long t256 = (long)((a->M + BM - 1) / BM) * (a->N / 256);
-    const long t128 = 2 * t256;
-    const double eff256 = double(t256) / double(((t256 + sms - 1) / sms) * sms);
-    const double eff128 = double(t128) / double(((t128 + sms - 1) / sms) * sms);
-    if (eff128 > eff256 * 1.15) wide = false;
-  }
   const bool amn = a->a_mn_major != 0, bmn = a->b_mn_major != 0;
   if (amn && !bmn) return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: MN-major A with K-major B is not built");
-  return dispatch_fam(family_of(mode), wide, amn, bmn, a, e, status, st);
+  const int fam = family_of(mode);
+  if (a->tile < FL_TILE_AUTO || a->tile > FL_TILE_256x256_PAIR)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: tile %d", a->tile);
+  if (a->tile >= FL_TILE_128x256 && (a->N % 256))
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: 256-column tiles need N %% 256 == 0 (N=%d)", a->N);
+  if (a->tile == FL_TILE_256x256_PAIR && pair_slots_for(fam, amn, bmn) <= 0)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: this device cannot hold the CTA-pair kernel");
+  if (a->tile != FL_TILE_AUTO) return dispatch_fam(fam, a->tile - 1, amn, bmn, a, e, status, st);
+  // Tile shape: 256 columns (on a CTA pair where the device can hold pairs) unless
+  // 128 x 128 tiles give clearly fewer idle SM slots in the last wave.
+  int shape = 0;
+  if ((a->N % 256) == 0) {
+    const int sms = num_sms();
+    const int pairs = pair_slots_for(fam, amn, bmn);
+    const long t128 = (long)((a->M + BM - 1) / BM) * (a->N / 128);
+    const double eff128 = double(t128) / double(((t128 + sms - 1) / sms) * sms);
+    double eff_wide;
+    if (pairs > 0) {
+      const long tp = (long)((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
+      eff_wide = double(tp) / double(((tp + pairs - 1) / pairs) * pairs);
+      shape = 2;
+    } else {
+      const long t256 = (long)((a->M + BM - 1) / BM) * (a->N / 256);
+      eff_wide = double(t256) / double(((t256 + sms - 1) / sms) * sms);
+      shape = 1;
+    }
+    if (eff128 > eff_wide * 1.15) shape = 0;
+  }
+  return dispatch_fam(fam, shape, amn, bmn, a, e, status, st);
 }

@@ -451,6 +451,232 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+// ------------------------------------------------------------------ CTA-pair kernel
+// A cluster of two CTAs on two SMs computes one 256 x 256 tile with tcgen05.mma
+// .cta_group::2.  Each CTA stages its own 128 rows of A and 128 columns of B (32 KB per
+// k-block, against 48 KB for a 128 x 256 tile on one SM, which leaves room for a 6-deep
+// ring); the even CTA issues 256 x 256 x 16 MMAs that read both CTAs' stages and write
+// accumulator rows 0..127 into its own TMEM and rows 128..255 into the odd CTA's; each
+// CTA's four epilogue warps drain their own half exactly as in gemm_tc_kernel.
+// Barriers: both producers' loads complete on the even CTA's full[s]; the MMA commits
+// arrive on empty[s] and acc_full[a] of both CTAs; every epilogue warp of the pair
+// arrives once on the even CTA's acc_empty[a].
+constexpr int PAIR_BM = 256, PAIR_BN = 256;
+struct CfgPair {
+  static constexpr int STAGES = 6;
+  static constexpr int A_BYTES = 128 * BK * 2;  // this CTA's 128 rows of A
+  static constexpr int B_BYTES = 128 * BK * 2;  // this CTA's 128 columns of B
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int TMEM_COLS = 2 * PAIR_BN;  // double-buffered 256-column accumulator
+  static constexpr int STAGING_BYTES = 4 * 32 * 64 * 4;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 256 /*barriers*/ + STAGING_BYTES + 1024 /*align*/;
+};
+
+template <bool A_MN, bool B_MN, int FAM>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, Epi epi,
+                     int M, int N, int K, Raster raster, int* status) {
+  using C = CfgPair;
+  constexpr int STAGES = C::STAGES;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* acc_full = bars + 2 * STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* staging = reinterpret_cast<float*>(smem + STAGES * C::STAGE_BYTES + 256);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  const int num_m = (M + PAIR_BM - 1) / PAIR_BM;
+  const int num_n = N / PAIR_BN;
+  const int num_tiles = num_m * num_n;
+  const int num_k = (K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);   // the even CTA's producer (expect_tx of both CTAs' bytes)
+      mbar_init(&empty[s], 1);  // one MMA commit
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 8);  // four epilogue warps in each CTA
+    }
+    mbar_init(drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_holder, C::TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();  // both CTAs' barriers initialised and TMEM allocated
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer (both CTAs)
+      const uint32_t full0 = mapa_shared(smem_u32(full), 0);  // the even CTA's full[0]
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t armed = 0, last_par = 0;  // per-stage bit masks for the teardown drain
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += n_pairs) {
+        int mb, nb;
+        tile_coords(tile, num_m, num_n, raster, mb, nb);
+        const int m0 = mb * PAIR_BM + int(rank) * 128, n0 = nb * PAIR_BN + int(rank) * 128;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1)) {
+            report_status(status, FL_DEV_TIMEOUT_EMPTY);
+            ok = false;
+            break;
+          }
+          if (leader) mbar_arrive_expect_tx(&full[stage], 2 * C::STAGE_BYTES);
+          armed |= 1u << stage;
+          last_par = (last_par & ~(1u << stage)) | (phase << stage);
+          const uint32_t fb = full0 + 8u * stage;
+          const int k0 = kb * BK;
+          uint8_t* a_dst = sA + stage * C::A_BYTES;
+          uint8_t* b_dst = sB + stage * C::B_BYTES;
+          if (!A_MN) {
+            tma_load_2d_pair(a_dst, &tmA, fb, k0, m0);
+          } else {
+            tma_load_2d_pair(a_dst, &tmA, fb, m0, k0);
+            tma_load_2d_pair(a_dst + 64 * BK * 2, &tmA, fb, m0 + 64, k0);
+          }
+          if (!B_MN) {
+            tma_load_2d_pair(b_dst, &tmB, fb, k0, n0);
+          } else {
+            tma_load_2d_pair(b_dst, &tmB, fb, n0, k0);
+            tma_load_2d_pair(b_dst + 64 * BK * 2, &tmB, fb, n0 + 64, k0);
+          }
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // Drain: a stage loaded in phase p is released (empty phase p completes) only after
+      // the MMAs that read it, and so after its copies landed.
+      for (int s = 0; s < STAGES; ++s)
+        if (armed & (1u << s))
+          if (!mbar_wait(&empty[s], (last_par >> s) & 1)) report_status(status, FL_DEV_TIMEOUT_DRAIN);
+    }
+  } else if (warp == 1) {
+    if (leader && lane == 0) {
+      // ------------------------------------------------------------ MMA issuer (even CTA)
+      constexpr uint32_t IDESC = umma_idesc_bf16(PAIR_BM, PAIR_BN, A_MN, B_MN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += n_pairs, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_par = (local >> 1) & 1;
+        if (!mbar_wait(&acc_empty[acc], acc_par ^ 1)) {
+          report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * PAIR_BN;
+        for (int kb = 0; kb < num_k; ++kb) {
+          if (!mbar_wait(&full[stage], phase)) {
+            report_status(status, FL_DEV_TIMEOUT_FULL);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(sA + stage * C::A_BYTES);
+          const uint32_t b_base = smem_u32(sB + stage * C::B_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < BK / UMMA_K; ++kk) {
+            const uint64_t adesc = A_MN ? smem_desc_sw128(a_base + kk * 2048, BK * 128, 1024)
+                                        : smem_desc_sw128(a_base + kk * 32, 16, 1024);
+            const uint64_t bdesc = B_MN ? smem_desc_sw128(b_base + kk * 2048, BK * 128, 1024)
+                                        : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+            umma_bf16_pair(d_tmem, adesc, bdesc, IDESC, (kb | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit_pair(&empty[stage], 3);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (ok) umma_commit_pair(&acc_full[acc], 3);
+      }
+      // Drain: all MMAs issued by this thread (and their arrivals) complete before the pair
+      // releases TMEM and shared memory.
+      umma_commit_pair(drain, 1);
+      if (!mbar_wait(drain, 0)) report_status(status, FL_DEV_TIMEOUT_DRAIN);
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue warps (both CTAs)
+    const int quarter = warp & 3;
+    float* stage = staging + (warp - 2) * 32 * 64;
+    float4* my = reinterpret_cast<float4*>(stage + lane * 64);
+    const uint32_t acc_empty0 = mapa_shared(smem_u32(acc_empty), 0);
+    int local = 0;
+    for (int tile = pair; tile < num_tiles; tile += n_pairs, ++local) {
+      int mb, nb;
+      tile_coords(tile, num_m, num_n, raster, mb, nb);
+      const int acc = local & 1;
+      const uint32_t acc_par = (local >> 1) & 1;
+      if (!mbar_wait(&acc_full[acc], acc_par)) {
+        report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
+        break;
+      }
+      tc_fence_after();
+      const int row0 = mb * PAIR_BM + int(rank) * 128 + quarter * 32;
+      const int rows = M - row0 < 32 ? M - row0 : 32;  // may be <= 0 for the ragged last tile
+      const uint32_t t_row = tmem_base + (uint32_t(quarter * 32) << 16) + acc * PAIR_BN;
+#pragma unroll 1
+      for (int c0 = 0; c0 < PAIR_BN; c0 += 64) {
+        uint32_t r0[32], r1[32];
+        tmem_ld32(t_row + c0, r0);
+        tmem_ld32(t_row + c0 + 32, r1);
+        tmem_ld_wait();
+        if (c0 + 64 == PAIR_BN) {  // accumulator fully read: the MMA may reuse it
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(acc_empty0 + 8u * acc);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          my[j ^ (lane & 15)] = make_float4(__uint_as_float(r0[4 * j]), __uint_as_float(r0[4 * j + 1]),
+                                            __uint_as_float(r0[4 * j + 2]), __uint_as_float(r0[4 * j + 3]));
+          my[(8 + j) ^ (lane & 15)] = make_float4(__uint_as_float(r1[4 * j]), __uint_as_float(r1[4 * j + 1]),
+                                                  __uint_as_float(r1[4 * j + 2]), __uint_as_float(r1[4 * j + 3]));
+        }
+        __syncwarp();
+        if (rows > 0) epilogue_chunk<FAM>(epi, stage, row0, rows, nb * PAIR_BN + c0, lane);
+        __syncwarp();
+      }
+    }
+  }
+
+  tc_fence_before();
+  cluster_sync();  // neither CTA leaves while the pair's MMAs or arrivals may still touch it
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
+  }
+}
+
 // ------------------------------------------------------------------ host side
 
 typedef CUresult (*PFN_encodeTiled)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -499,6 +725,21 @@ inline int num_sms() {
   return n;
 }
 
+// Row-group raster that minimises DRAM reads for tiles of bm x bn (see Raster).
+inline Raster pick_raster(int M, int N, int K, int bm, int bn) {
+  const int num_m = (M + bm - 1) / bm, num_n = N / bn;
+  const double pa = double(bm) * K * 2, pb = double(bn) * K * 2;
+  int gm = (int)(L2_GROUP_BUDGET / pa), gn = (int)(L2_GROUP_BUDGET / pb);
+  gm = gm < 1 ? 1 : (gm > num_m ? num_m : gm);
+  gn = gn < 1 ? 1 : (gn > num_n ? num_n : gn);
+  const double cost_m = pa * num_m + pb * num_n * ((num_m + gm - 1) / gm);
+  const double cost_n = pb * num_n + pa * num_m * ((num_n + gn - 1) / gn);
+  Raster r;
+  r.along_n = cost_n < cost_m ? 1 : 0;
+  r.gsz = r.along_n ? gn : gm;
+  return r;
+}
+
 template <int BN, bool A_MN, bool B_MN, int FAM>
 int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) {
   using C = Cfg<BN>;
@@ -520,27 +761,88 @@ int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) 
   const int num_m = (a->M + BM - 1) / BM, num_n = a->N / BN;
   const int tiles = num_m * num_n;
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  // DRAM reads of the two orders: the grouped operand once, the other once per group
-  const double pa = double(BM) * a->K * 2, pb = double(BN) * a->K * 2;
-  int gm = (int)(L2_GROUP_BUDGET / pa), gn = (int)(L2_GROUP_BUDGET / pb);
-  gm = gm < 1 ? 1 : (gm > num_m ? num_m : gm);
-  gn = gn < 1 ? 1 : (gn > num_n ? num_n : gn);
-  const double cost_m = pa * num_m + pb * num_n * ((num_m + gm - 1) / gm);
-  const double cost_n = pb * num_n + pa * num_m * ((num_n + gn - 1) / gn);
-  Raster r;
-  r.along_n = cost_n < cost_m ? 1 : 0;
-  r.gsz = r.along_n ? gn : gm;
+  const Raster r = pick_raster(a->M, a->N, a->K, BM, BN);
   gemm_tc_kernel<BN, A_MN, B_MN, FAM><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ta, tb, epi, a->M, a->N, a->K, r,
                                                                                  status);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
 
+// CTA pairs the device keeps resident at once for the pair kernel (0 if it cannot run).
+template <bool A_MN, bool B_MN, int FAM>
+int pair_slots() {
+  static int slots = -1;
+  if (slots < 0) {
+    auto kern = gemm_pair_kernel<A_MN, B_MN, FAM>;
+    slots = 0;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, CfgPair::SMEM_BYTES) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 2;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.gridDim = dim3(2 * num_sms());
+      cfg.blockDim = dim3(NUM_THREADS);
+      cfg.dynamicSmemBytes = CfgPair::SMEM_BYTES;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0) slots = n;
+    }
+    cudaGetLastError();  // a refused query leaves the single-SM kernel in use
+  }
+  return slots;
+}
+
+template <bool A_MN, bool B_MN, int FAM>
+int launch_pair(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) {
+  auto kern = gemm_pair_kernel<A_MN, B_MN, FAM>;
+  const int slots = pair_slots<A_MN, B_MN, FAM>();
+  if (slots <= 0) return fl_internal_error(FL_ERR_CUDA, "gemm: the CTA-pair kernel cannot be resident");
+  CUtensorMap ta, tb;
+  int rc;
+  // each CTA loads 128 rows of A and 128 columns of B per k-block
+  if (!A_MN) rc = make_map(&ta, a->A, a->K, a->M, a->lda, 128);
+  else rc = make_map(&ta, a->A, a->M, a->K, a->lda, BK);
+  if (rc) return rc;
+  if (!B_MN) rc = make_map(&tb, a->B, a->K, a->N, a->ldb, 128);
+  else rc = make_map(&tb, a->B, a->N, a->K, a->ldb, BK);
+  if (rc) return rc;
+  const int tiles = ((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
+  const int pairs = tiles < slots ? tiles : slots;
+  const Raster r = pick_raster(a->M, a->N, a->K, PAIR_BM, PAIR_BN);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(2 * pairs);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = CfgPair::SMEM_BYTES;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  FL_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, ta, tb, epi, a->M, a->N, a->K, r, status));
+  return FL_OK;
+}
+
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
-// Every (layout, family) pair for both tile widths; the three operand layouts are
+// Every (layout, family) pair for the CTA-pair kernel and both single-SM tile widths; the three operand layouts are
 // instantiated in separate translation units so that the build compiles them in parallel.
 #define FL_GEMM_INSTANTIATE(AMN, BMN)                                                              \
+  template int pair_slots<AMN, BMN, FAM_PLAIN>();                                                      \
+  template int pair_slots<AMN, BMN, FAM_GELU>();                                                       \
+  template int pair_slots<AMN, BMN, FAM_RESID>();                                                      \
+  template int pair_slots<AMN, BMN, FAM_ROPE>();                                                       \
+  template int pair_slots<AMN, BMN, FAM_ADAMW>();                                                      \
+  template int launch_pair<AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch_pair<AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
+  template int launch_pair<AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
+  template int launch_pair<AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
+  template int launch_pair<AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
   template int launch<256, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
   template int launch<128, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
   template int launch<256, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \

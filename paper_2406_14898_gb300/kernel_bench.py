@@ -59,7 +59,13 @@ def main():
     ap.add_argument("--wgrad-epilogue", default="store", choices=["store", "adamw"],
                     help="epilogue of the weight-gradient GEMMs: fp32 store (the separate-step path) or the "
                          "fused AdamW update of the backward + step call")
+    ap.add_argument("--tiles", default="auto",
+                    help="comma-separated GEMM tile shapes to time: auto, 128x128, 128x256, pair (256 x 256 on a "
+                         "CTA pair)")
     args = ap.parse_args()
+    tile_ids = {"auto": F.FL_TILE_AUTO, "128x128": F.FL_TILE_128x128, "128x256": F.FL_TILE_128x256,
+                "pair": F.FL_TILE_256x256_PAIR}
+    tiles_wanted = [t.strip() for t in args.tiles.split(",") if t.strip()]
     cfg = syn.CONFIGS[args.workload]
     F.lib()
     dev = torch.device("cuda", 0)
@@ -113,7 +119,8 @@ def main():
             kw.update(n_heads=nh, head_dim=hd, rotary_dim=hd // 2)
         lda = M if amn else K
         ldb = N if bmn else K
-        if epi == F.FL_EPI_STORE_F32 and args.wgrad_epilogue == "adamw":
+        adamw = epi == F.FL_EPI_STORE_F32 and args.wgrad_epilogue == "adamw"
+        if adamw:
             # g = A . B^T updates fp32 weights D with their moments, writes the bf16 copy
             mom = torch.zeros(2, M, N, device=dev, dtype=torch.float32)
             wb16 = torch.empty(M, N, device=dev, dtype=torch.bfloat16)
@@ -122,12 +129,22 @@ def main():
             ga.adam_m, ga.adam_v = F.ptr(mom[0]), F.ptr(mom[1])
             ga.lr, ga.beta1, ga.beta2, ga.eps, ga.weight_decay = 1e-4, 0.9, 0.999, 1e-8, 0.0
             ga.inv_bc1, ga.inv_bc2 = 10.0, 1000.0
-            ms = timed(lambda: F.fl_k_gemm(ga, stream=st))
-            name = name + "_adamw"
-        else:
-            ms = timed(lambda: F.gemm(M, N, K, A, lda, amn, B, ldb, bmn, D, N, epilogue=epi, stream=st, **kw))
-        flops = 2.0 * M * N * K
-        out.append({"kernel": f"gemm_{name}", "M": M, "N": N, "K": K, "ms": ms, "tflops": flops / ms / 1e9})
+        for tname in tiles_wanted:
+            tile = tile_ids[tname]
+            if tile >= F.FL_TILE_128x256 and N % 256:
+                continue
+            if adamw:
+                ga.tile = tile
+                ms = timed(lambda: F.fl_k_gemm(ga, stream=st))
+            else:
+                ms = timed(lambda: F.gemm(M, N, K, A, lda, amn, B, ldb, bmn, D, N, epilogue=epi, tile=tile, stream=st,
+                                          **kw))
+            flops = 2.0 * M * N * K
+            rec = {"kernel": f"gemm_{name}" + ("_adamw" if adamw else ""), "M": M, "N": N, "K": K, "ms": ms,
+                   "tflops": flops / ms / 1e9}
+            if tname != "auto":
+                rec["tile"] = tname
+            out.append(rec)
         del A, B, D, kw
     if args.kernel in ("all", "attention"):
         seqs = cfg.segment_lengths

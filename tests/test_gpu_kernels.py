@@ -36,19 +36,33 @@ def _store(mat: np.ndarray, mn_major: bool):
     return dev_bf16(mat), mat.shape[1]
 
 
+TILES = ["auto", "128x128", "128x256", "pair"]
+
+
+def tile_id(F, name):
+    return {"auto": F.FL_TILE_AUTO, "128x128": F.FL_TILE_128x128, "128x256": F.FL_TILE_128x256,
+            "pair": F.FL_TILE_256x256_PAIR}[name]
+
+
+@pytest.mark.parametrize("tile", TILES)
 @pytest.mark.parametrize("layout", [(0, 0), (0, 1), (1, 1)], ids=["fwd", "dgrad", "wgrad"])
 @pytest.mark.parametrize("shape", [(200, 256, 320), (136, 384, 200), (1000, 1024, 512), (64, 128, 64),
-                                   (8, 256, 4096), (520, 768, 72)])
-def test_gemm_layouts(F, layout, shape):
+                                   (8, 256, 4096), (520, 768, 72), (104, 512, 256), (4000, 4096, 520)])
+def test_gemm_layouts(F, layout, shape, tile):
+    """Every operand layout and tile shape.  (104, 512, 256): the odd CTA of a pair loads
+    rows wholly past M; (4000, 4096, 520): several 256 x 256 tiles per CTA pair, so both
+    accumulator buffers and the 6-stage ring wrap, with a ragged last k-block."""
     M, N, K = shape
     a_mn, b_mn = layout
+    if tile in ("128x256", "pair") and N % 256:
+        pytest.skip("256-column tiles need N % 256 == 0")
     rng = np.random.default_rng(M * 7 + N + K + 31 * a_mn + 17 * b_mn)
     A = rnd_bf16_f64(rng, (M, K))
     B = rnd_bf16_f64(rng, (N, K))
     dA, lda = _store(A, bool(a_mn))
     dB, ldb = _store(B, bool(b_mn))
     D = torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda")
-    F.gemm(M, N, K, dA, lda, a_mn, dB, ldb, b_mn, D, N)
+    F.gemm(M, N, K, dA, lda, a_mn, dB, ldb, b_mn, D, N, tile=tile_id(F, tile))
     torch.cuda.synchronize()
     ref = A @ B.T
     assert rel_inf(f64(D), ref) < GEMM_TOL
@@ -71,8 +85,10 @@ def test_gemm_accumulate_f32_repeated(F):
     assert rel_inf(f64(D), ref) < 1e-5
 
 
-def test_gemm_epilogues(F):
+@pytest.mark.parametrize("tile", ["auto", "pair"])
+def test_gemm_epilogues(F, tile):
     M, N, K = 192, 512, 256
+    t = tile_id(F, tile)
     rng = np.random.default_rng(11)
     A = rnd_bf16_f64(rng, (M, K))
     B = rnd_bf16_f64(rng, (N, K), 0.1)
@@ -87,35 +103,38 @@ def test_gemm_epilogues(F):
     # bias + gelu, pre-activation kept
     D = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
     U = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_GELU, bias=db, aux_out=U, ld_aux_out=N)
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_BIAS_GELU, bias=db, aux_out=U, ld_aux_out=N)
     torch.cuda.synchronize()
     u = acc + bias[None, :]
     assert rel_inf(f64(U), u) < GEMM_TOL
     assert rel_inf(f64(D), O.gelu(u)) < GEMM_TOL
     # bias + alpha * residual
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_RESID, bias=db, aux=dR, ld_aux=N,
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_BIAS_RESID, bias=db, aux=dR, ld_aux=N,
            alpha=alpha)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), u + alpha * R) < GEMM_TOL
     # alpha * residual, no bias
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_RESID, aux=dR, ld_aux=N, alpha=alpha)
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_RESID, aux=dR, ld_aux=N, alpha=alpha)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), acc + alpha * R) < GEMM_TOL
     # gelu' of a stored pre-activation
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_GELU_BWD, aux=dR, ld_aux=N)
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_GELU_BWD, aux=dR, ld_aux=N)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), acc * O.gelu_grad(R)) < GEMM_TOL
     # plain store with bias
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_STORE, bias=db)
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_STORE, bias=db)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), u) < GEMM_TOL
 
 
+@pytest.mark.parametrize("tile", ["auto", "pair"])
 @pytest.mark.parametrize("hd", [64, 128])
-def test_gemm_rope_epilogue(F, hd):
+def test_gemm_rope_epilogue(F, hd, tile):
     nh = 2
     H = nh * hd
     M, N, K = 130, 3 * H, 256
+    if tile == "pair" and N % 256:
+        pytest.skip("256-column tiles need N % 256 == 0")
     rng = np.random.default_rng(hd)
     A = rnd_bf16_f64(rng, (M, K))
     B = rnd_bf16_f64(rng, (N, K), 0.1)
@@ -127,7 +146,7 @@ def test_gemm_rope_epilogue(F, hd):
     dB, ldb = _store(B, False)
     D = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
     F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_ROPE, bias=dev_f32(bias),
-           pos=dev_i32(pos), rope_tab=dev_f32(tab), n_heads=nh, head_dim=hd, rotary_dim=rd)
+           pos=dev_i32(pos), rope_tab=dev_f32(tab), n_heads=nh, head_dim=hd, rotary_dim=rd, tile=tile_id(F, tile))
     torch.cuda.synchronize()
     qkv = A @ B.T + bias[None, :]
     cos, sin = O.rope_cos_sin(pos, rd, 10000.0)
@@ -187,10 +206,12 @@ def test_layernorm_fwd_bwd(F, H, dtype):
         assert rel_inf(f64(dbet) + 0.25, dbr) < 1e-4
 
 
-def test_gemm_fp32_residual_epilogues(F):
+@pytest.mark.parametrize("tile", ["auto", "pair"])
+def test_gemm_fp32_residual_epilogues(F, tile):
     """fp32 residual stream: D fp32 = acc + bias + alpha * R, with R an fp32 tensor or its
     LayerNorm recomputed in fp32 from the row statistics."""
     M, N, K = 200, 512, 256
+    t = tile_id(F, tile)
     rng = np.random.default_rng(12)
     A = rnd_bf16_f64(rng, (M, K))
     B = rnd_bf16_f64(rng, (N, K), 0.1)
@@ -204,17 +225,17 @@ def test_gemm_fp32_residual_epilogues(F):
     acc = A @ B.T
     D = torch.empty((M, N), dtype=torch.float32, device="cuda")
     dX = dev_f32(X)
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_RESID, bias=dev_f32(bias), aux=dX, ld_aux=N,
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_BIAS_RESID, bias=dev_f32(bias), aux=dX, ld_aux=N,
            alpha=7.5, aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), acc + bias[None, :] + 7.5 * X) < 1e-5
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_BIAS_RESID, bias=dev_f32(bias), aux=dX, ld_aux=N,
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_BIAS_RESID, bias=dev_f32(bias), aux=dX, ld_aux=N,
            alpha=7.5, aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32, ln_mean=dev_f32(mu), ln_rstd=dev_f32(rs),
            ln_gamma=dev_f32(g), ln_beta=dev_f32(be))
     torch.cuda.synchronize()
     lnx = (X - mu[:, None]) * rs[:, None] * g[None, :] + be[None, :]
     assert rel_inf(f64(D), acc + bias[None, :] + 7.5 * lnx) < 1e-5
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, epilogue=F.FL_EPI_RESID, aux=dX, ld_aux=N, alpha=-2.0,
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_RESID, aux=dX, ld_aux=N, alpha=-2.0,
            aux_dtype=F.FL_DT_F32, d_dtype=F.FL_DT_F32)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), acc - 2.0 * X) < 1e-5
@@ -360,11 +381,14 @@ def test_attention_with_prefix(F, hd, Lp):
     assert rel_inf(f64(gpv), dpvr.reshape(Lp, H)) < 5e-2
 
 
-@pytest.mark.parametrize("M,N,K,mn", [(200, 384, 136, 1), (256, 512, 64, 1), (130, 256, 96, 0)])
-def test_gemm_adamw_epilogue(F, M, N, K, mn):
+@pytest.mark.parametrize("tile", ["auto", "pair"])
+@pytest.mark.parametrize("M,N,K,mn", [(200, 384, 136, 1), (256, 512, 64, 1), (130, 256, 96, 0), (600, 1024, 520, 1)])
+def test_gemm_adamw_epilogue(F, M, N, K, mn, tile):
     """The weight-gradient GEMM with the AdamW update in its epilogue equals the plain fp32
     gradient GEMM followed by the separate AdamW kernel: weights, moments and the bf16
-    copy; ragged rows, both tile widths (N = 384 takes 128-column tiles)."""
+    copy; ragged rows, every tile shape (N = 384 takes 128-column tiles)."""
+    if tile == "pair" and N % 256:
+        pytest.skip("256-column tiles need N % 256 == 0")
     rng = np.random.default_rng(M + N)
     A = rnd_bf16_f64(rng, (M, K))
     B = rnd_bf16_f64(rng, (N, K))
@@ -389,6 +413,7 @@ def test_gemm_adamw_epilogue(F, M, N, K, mn):
     ga.adam_m, ga.adam_v = F.ptr(mf), F.ptr(vf)
     ga.lr, ga.beta1, ga.beta2, ga.eps, ga.weight_decay = lr, b1, b2, eps, wd
     ga.inv_bc1, ga.inv_bc2 = 1.0 / np.float32(bc1), 1.0 / np.float32(bc2)
+    ga.tile = tile_id(F, tile)
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
     F.fl_k_gemm(ga, status=status)
     torch.cuda.synchronize()

@@ -73,5 +73,13 @@ def test_kernel_entry_points_validate_before_launch(F):
     L = F.lib()
     a = F.fl_gemm_args()
     assert L.fl_k_gemm(ctypes.byref(a), None, None) == -1          # null operands
+    # tile shape checks come before any device call (addresses are never dereferenced)
+    a = F.fl_gemm_args(8, 384, 64, 0x10000, 64, 0, 0x20000, 64, 0, 0x30000, 384, F.FL_EPI_STORE)
+    a.tile = 7
+    assert L.fl_k_gemm(ctypes.byref(a), None, None) == -1
+    a.tile = F.FL_TILE_128x256                                      # N % 256 != 0
+    assert L.fl_k_gemm(ctypes.byref(a), None, None) == -7
+    a.tile = F.FL_TILE_256x256_PAIR
+    assert L.fl_k_gemm(ctypes.byref(a), None, None) == -7
     assert L.fl_k_layernorm_fwd(4, 300, None, 0, None, None, 1e-5, None, None, None, None) == -7
     assert L.fl_k_adamw(6, None, None, None, None, None, 1e-3, .9, .999, 1e-8, 0, .1, .001, None) == -1
