@@ -268,7 +268,7 @@ def main():
     ap.add_argument("--recompute", action="store_true",
                     help="keep only the block inputs and recompute each block's activations in the backward "
                          "(for workloads whose activations do not fit, e.g. --workload sweep26_K64)")
-    ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_tc_up_fwd_stack26.md"))
+    ap.add_argument("--ncu-traffic", default=os.path.join(ROOT, "profiles", "gemm_pair_up_fwd_stack26.md"))
     args = ap.parse_args()
     cfg = workload(args.workload)
     if args.ptuning:
