@@ -78,6 +78,12 @@ typedef struct {
   float adam_beta1, adam_beta2, adam_eps, weight_decay; /* 0.9, 0.999, 1e-8, 0 */
   int32_t prefix_len;       /* P-tuning v2 (App. A): learnable prefix keys/values per block, 0..128 */
   int32_t freeze_base;      /* 1: only the prefixes are trained (needs prefix_len > 0) */
+  int32_t fused_step_min_tokens; /* fl_server_backward_step applies AdamW inside the weight-
+                             * gradient GEMMs when the pending call has at least this many
+                             * tokens, else it runs the backward and then fl_server_step;
+                             * 0 -> 4608 (the crossover measured on GB300: with fewer tokens
+                             * the weight-gradient main loop is too short to hide the 26 B per
+                             * parameter of the fused update); 1 -> always fused */
 } fl_server_cfg;
 
 /* Fills *cfg with the ChatGLM-6B server defaults (26 blocks, H 4096, 32 x 128, F 16384,
@@ -141,9 +147,9 @@ int fl_server_step(fl_server_t h, float lr);
  * matrices of every block runs in the epilogue of their weight-gradient GEMMs: the fp32
  * matrix gradients are never written to memory, and the update's traffic overlaps the
  * tensor-core work.  The bias and LayerNorm vectors get one AdamW launch at the end.
- * Otherwise (gradients accumulated by earlier backward calls) it runs the two calls as
- * they are.  Results equal backward + step up to fp32 rounding.  Errors: as
- * fl_server_backward. */
+ * Otherwise (gradients accumulated by earlier backward calls, or fewer tokens in the
+ * pending call than cfg.fused_step_min_tokens) it runs the two calls as they are.
+ * Results equal backward + step up to fp32 rounding.  Errors: as fl_server_backward. */
 int fl_server_backward_step(fl_server_t h, const void* const grad_out[], void* const grad_in[], float lr);
 
 /* Frees every device buffer of h after synchronising its stream.  NULL is accepted. */

@@ -44,7 +44,7 @@ class fl_server_cfg(C.Structure):
                 ("client_batch", C.c_int32), ("max_tokens", C.c_int32), ("max_seq_len", C.c_int32),
                 ("recompute", C.c_int32), ("init_std", C.c_float), ("adam_beta1", C.c_float),
                 ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("weight_decay", C.c_float),
-                ("prefix_len", C.c_int32), ("freeze_base", C.c_int32)]
+                ("prefix_len", C.c_int32), ("freeze_base", C.c_int32), ("fused_step_min_tokens", C.c_int32)]
 
 
 class fl_client_cfg(C.Structure):
@@ -174,10 +174,12 @@ def _parr(xs) -> "C.Array":
     return (C.c_void_p * len(xs))(*[ptr(x) for x in xs])
 
 
-def make_cfg(c, max_tokens: int, max_seq_len: int = 0, recompute: int = 0) -> fl_server_cfg:
+def make_cfg(c, max_tokens: int, max_seq_len: int = 0, recompute: int = 0,
+             fused_step_min_tokens: int = 0) -> fl_server_cfg:
     """fl_server_cfg from a workload description with the attributes of
     ``synthetic.ServerConfig`` (n_blocks, hidden, ... , weight_decay); ``recompute``
-    keeps one block's activations and recomputes the rest in the backward."""
+    keeps one block's activations and recomputes the rest in the backward;
+    ``fused_step_min_tokens`` as in fl_server_cfg (0: the library's crossover)."""
     cfg = fl_server_cfg()
     lib().fl_server_cfg_default(C.byref(cfg))
     cfg.n_blocks = c.n_blocks
@@ -201,6 +203,7 @@ def make_cfg(c, max_tokens: int, max_seq_len: int = 0, recompute: int = 0) -> fl
     cfg.weight_decay = c.weight_decay
     cfg.prefix_len = getattr(c, "prefix_len", 0)
     cfg.freeze_base = getattr(c, "freeze_base", 0)
+    cfg.fused_step_min_tokens = fused_step_min_tokens
     return cfg
 
 

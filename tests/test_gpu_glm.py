@@ -128,7 +128,7 @@ def glm_case(F, cfg, ctx, mp, fused=False, check_grads=True):
     """Server forward/backward(/step) with GLM segments against the oracle server."""
     params = syn.init_params(cfg)
     prefixes = [syn.init_prefix(cfg, b) for b in range(cfg.n_blocks)] if cfg.prefix_len else None
-    srv = F.Server(F.make_cfg(cfg, cfg.tokens), cfg.seed)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, fused_step_min_tokens=1), cfg.seed)
     for b in range(cfg.n_blocks):
         for t in range(12):
             srv.set_param(b, t, params[b][t])
@@ -214,7 +214,7 @@ def test_glm_batching_invariant_bitexact(F):
     states, grads = syn.client_states(cfg), syn.client_grads(cfg)
 
     def run(c, st_bits, g_bits, cl, mpl, max_tokens):
-        srv = F.Server(F.make_cfg(c, max_tokens), cfg.seed)
+        srv = F.Server(F.make_cfg(c, max_tokens, fused_step_min_tokens=1), cfg.seed)
         st = [dev_bf16_from_bits(s) for s in st_bits]
         outs = [torch.empty_like(s) for s in st]
         srv.forward(st, c.seq_lens, outs, context_lens=cl, mask_pos=mpl)
@@ -235,7 +235,7 @@ def test_glm_batching_invariant_bitexact(F):
 
 def test_glm_argument_errors(F):
     cfg = syn.CONFIGS["tiny"]
-    srv = F.Server(F.make_cfg(cfg, cfg.tokens), cfg.seed)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, fused_step_min_tokens=1), cfg.seed)
     st = [torch.zeros((2, 64, 256), dtype=torch.bfloat16, device="cuda")]
     for ctx, mp in [([65, 1], None), ([-1, 1], None), ([10, 4], [10, 0]), ([10, 4], [-1, 0])]:
         with pytest.raises(F.FlError) as ei:

@@ -20,7 +20,7 @@ def F():
 
 def test_prefix_init_matches_generator(F):
     cfg = syn.CONFIGS["tiny"].with_(prefix_len=16)
-    srv = F.Server(F.make_cfg(cfg, cfg.tokens), cfg.seed)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, fused_step_min_tokens=1), cfg.seed)
     want = syn.init_prefix(cfg, 0)
     for j, t in enumerate((F.FL_T_PREFIX_K, F.FL_T_PREFIX_V)):
         got = srv.get_param(0, t)
@@ -36,7 +36,7 @@ def test_ptuning_parity(F, freeze, fused):
                                     freeze_base=freeze, lr=1e-3)
     params = syn.init_params(cfg)
     prefixes = [syn.init_prefix(cfg, b) for b in range(cfg.n_blocks)]
-    srv = F.Server(F.make_cfg(cfg, cfg.tokens), cfg.seed)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, fused_step_min_tokens=1), cfg.seed)
     for b in range(cfg.n_blocks):
         for t in range(12):
             srv.set_param(b, t, params[b][t])

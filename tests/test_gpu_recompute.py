@@ -34,7 +34,8 @@ def glm_kwargs(cfg):
 
 def run(F, cfg, recompute, fused):
     """One forward and one backward (fused: backward + AdamW step) from the seeded state."""
-    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens), recompute=recompute), cfg.seed)
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens), recompute=recompute, fused_step_min_tokens=1),
+                   cfg.seed)
     states = [dev_bf16_from_bits(s) for s in syn.client_states(cfg)]
     grads = [dev_bf16_from_bits(g) for g in syn.client_grads(cfg)]
     outs = [torch.empty_like(s) for s in states]

@@ -24,9 +24,12 @@ def F():
     return flglm()
 
 
-def make_server(F, cfg, max_tokens=None, seed=None):
+def make_server(F, cfg, max_tokens=None, seed=None, fused_step_min_tokens=1):
+    """fused_step_min_tokens=1: fl_server_backward_step always takes the fused path (the
+    test shapes are far below the library's crossover)."""
     mt = max_tokens or cfg.tokens
-    return F.Server(F.make_cfg(cfg, mt), cfg.seed if seed is None else seed)
+    return F.Server(F.make_cfg(cfg, mt, fused_step_min_tokens=fused_step_min_tokens),
+                    cfg.seed if seed is None else seed)
 
 
 def run_gpu(F, srv, cfg, states_bits, grads_bits):
@@ -176,6 +179,29 @@ def test_fused_step_equals_backward_then_step(F):
     b.forward(states, cfg.seq_lens, outs)
     b.backward_step(grads, gi, 1e-3)
     b.sync()
+    a.close()
+    b.close()
+
+
+def test_backward_step_below_the_fusion_crossover(F):
+    """With the library's default crossover a small call takes backward + step inside
+    fl_server_backward_step; two steps of it give the weights of the forced fused path
+    (up to the rounding of the atomic bias sums)."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, seq_lens=(64, 40))
+    states = [dev_bf16_from_bits(s) for s in syn.client_states(cfg)]
+    grads = [dev_bf16_from_bits(g) for g in syn.client_grads(cfg)]
+    a, b = make_server(F, cfg, fused_step_min_tokens=0), make_server(F, cfg)
+    outs = [torch.empty_like(s) for s in states]
+    gi = [torch.empty_like(s) for s in states]
+    for _ in range(2):
+        for srv in (a, b):
+            srv.forward(states, cfg.seq_lens, outs)
+            srv.backward_step(grads, gi, 1e-3)
+    a.sync()
+    b.sync()
+    for blk in range(cfg.n_blocks):
+        for t in range(12):
+            assert rel_inf(a.get_param(blk, t), b.get_param(blk, t)) < 1e-5, (blk, t)
     a.close()
     b.close()
 

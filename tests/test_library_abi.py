@@ -58,6 +58,12 @@ def test_cfg_default_and_validation(F):
     assert F.lib().fl_server_create(None, 0, ctypes.byref(h)) == -1
     assert F.lib().fl_server_forward(None, None, None, 1, None) == -1
     assert F.lib().fl_server_destroy(None) == 0
+    cfg = F.fl_server_cfg()
+    F.lib().fl_server_cfg_default(ctypes.byref(cfg))
+    assert cfg.fused_step_min_tokens == 0
+    cfg.fused_step_min_tokens = -1
+    assert F.lib().fl_server_create(ctypes.byref(cfg), 0, ctypes.byref(h)) == -1
+    assert not h.value and b"fused_step_min_tokens" in F.lib().fl_server_last_error(None)
     # client handles: defaults, validation before any device work
     cc = F.fl_client_cfg()
     F.lib().fl_client_cfg_default(ctypes.byref(cc))
