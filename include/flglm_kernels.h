@@ -91,6 +91,9 @@ typedef struct {
   int32_t tile;                             /* FL_TILE_*: tile shape, FL_TILE_AUTO (0) lets the library
                                                pick (256-column tiles on CTA pairs unless smaller tiles
                                                leave clearly fewer SMs idle in the last wave) */
+  float* colsum;                            /* FL_EPI_GELU_BWD only, or NULL: colsum[n] += sum over m of
+                                               D[m,n] (fp32, before rounding; fp32 atomics, so the
+                                               order of the additions is not fixed) */
 } fl_gemm_args;
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);

@@ -302,6 +302,28 @@ FL_DEV void inverse_rope_2d(float (&acc)[HD / 8][4], int r, int i, int64_t t, co
   if (gpos2) inverse_rope<HD, HD / 16>(acc, r, __ldg(gpos2 + t), tab, lane);
 }
 
+// Adds the column sums of a warp's 16 x HD fragment rows (dq-style accumulator layout:
+// thread holds rows lane/4 and lane/4 + 8, columns nt*8 + 2*(lane%4) + {0,1}) of all four
+// warps of the CTA to out[0..HD): rows already summed into acc[nt][0..1] by the caller,
+// reduced over the warp's 8 row groups with shuffles and over the warps through `red`
+// (4 * HD floats of shared memory no thread still reads); one atomic per column.
+template <int HD>
+FL_DEV void cta_colsum_add(float (&acc)[HD / 8][4], float* red, float* out, int warp, int lane, int tid) {
+#pragma unroll
+  for (int nt = 0; nt < HD / 8; ++nt)
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      float v = acc[nt][c];
+      v += __shfl_xor_sync(0xffffffffu, v, 4);
+      v += __shfl_xor_sync(0xffffffffu, v, 8);
+      v += __shfl_xor_sync(0xffffffffu, v, 16);
+      if (lane < 4) red[warp * HD + nt * 8 + 2 * lane + c] = v;
+    }
+  __syncthreads();
+  if (tid < HD) atomicAdd(out + tid, red[tid] + red[HD + tid] + red[2 * HD + tid] + red[3 * HD + tid]);
+  __syncthreads();
+}
+
 // ---------------------------------------------------------------------------- dQ
 template <int HD>
 __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf16* __restrict__ qkv,
@@ -315,7 +337,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
                                                           const bf16* __restrict__ pk, const bf16* __restrict__ pv,
                                                           int Lp, const int32_t* __restrict__ ctxs,
                                                           const int32_t* __restrict__ gpos,
-                                                          const int32_t* __restrict__ gpos2) {
+                                                          const int32_t* __restrict__ gpos2,
+                                                          float* __restrict__ dbias) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sQ = reinterpret_cast<bf16*>(smem);
   bf16* sdO = sQ + AT<HD>::TILE_ELEMS;
@@ -444,6 +467,16 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(int T, int H, const bf
         *reinterpret_cast<uint32_t*>(row + nt * 8) = pack_bf16x2(dq[nt][2 * r], dq[nt][2 * r + 1]);
     }
   }
+  if (dbias) {  // bias gradient of the q columns: sum of the valid rows' (unrotated) dq
+    const int qa = q0 + warp * 16 + (lane >> 2);
+    const bool va = qa < L, vb = qa + 8 < L;
+#pragma unroll
+    for (int nt = 0; nt < HD / 8; ++nt) {
+      dq[nt][0] = (va ? dq[nt][0] : 0.f) + (vb ? dq[nt][2] : 0.f);
+      dq[nt][1] = (va ? dq[nt][1] : 0.f) + (vb ? dq[nt][3] : 0.f);
+    }
+    cta_colsum_add<HD>(dq, reinterpret_cast<float*>(smem), dbias + h * HD, warp, lane, tid);
+  }
 }
 
 // ---------------------------------------------------------------------------- dK, dV
@@ -470,7 +503,8 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
                                                            int Lp, int nsplit, float* __restrict__ dpk,
                                                            float* __restrict__ dpv, const int32_t* __restrict__ ctxs,
                                                            const int32_t* __restrict__ gpos,
-                                                           const int32_t* __restrict__ gpos2) {
+                                                           const int32_t* __restrict__ gpos2,
+                                                           float* __restrict__ dbias) {
   extern __shared__ __align__(128) uint8_t smem[];
   bf16* sK = reinterpret_cast<bf16*>(smem);
   bf16* sV = sK + AT<HD>::TILE_ELEMS;
@@ -655,6 +689,21 @@ __global__ void __launch_bounds__(128) attn_bwd_dkv_kernel(int T, int H, const b
       }
     }
   }
+  if constexpr (!PREFIX) {
+    if (dbias) {  // bias gradients of the k and v columns: sums of the valid keys' dk, dv
+      const int ka = warp * 16 + (lane >> 2);
+      const bool va = ka < kvalid, vb = ka + 8 < kvalid;
+#pragma unroll
+      for (int nt = 0; nt < HD / 8; ++nt) {
+        dk[nt][0] = (va ? dk[nt][0] : 0.f) + (vb ? dk[nt][2] : 0.f);
+        dk[nt][1] = (va ? dk[nt][1] : 0.f) + (vb ? dk[nt][3] : 0.f);
+        dv[nt][0] = (va ? dv[nt][0] : 0.f) + (vb ? dv[nt][2] : 0.f);
+        dv[nt][1] = (va ? dv[nt][1] : 0.f) + (vb ? dv[nt][3] : 0.f);
+      }
+      cta_colsum_add<HD>(dk, reinterpret_cast<float*>(smem), dbias + H + h * HD, warp, lane, tid);
+      cta_colsum_add<HD>(dv, reinterpret_cast<float*>(smem), dbias + 2 * H + h * HD, warp, lane, tid);
+    }
+  }
 }
 
 template <int HD>
@@ -706,7 +755,7 @@ int launch_fwd(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t
 template <int HD>
 int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, const void* dout, const int32_t* cu,
                const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab, void* dqkv,
-               const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
+               const AttnPrefix& pre, const AttnGlm& glm, float* dbias, cudaStream_t st) {
   if (int rc = set_attrs<HD>()) return rc;
   const int H = nh * HD;
   const float scale = 1.f / sqrtf((float)HD);
@@ -719,11 +768,11 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
   const bf16* pv = (const bf16*)pre.v;
   attn_bwd_dq_kernel<HD><<<dim3(n_tiles, nh), 128, dq_smem<HD>(), st>>>(
       T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, tab, HD / 2, scale, (bf16*)dqkv, pk, pv,
-      pre.len, glm.ctx, glm.pos, glm.pos2);
+      pre.len, glm.ctx, glm.pos, glm.pos2, dbias);
   FL_CUDA_TRY(cudaGetLastError());
   attn_bwd_dkv_kernel<HD, false><<<dim3(n_tiles, nh), 128, dkv_smem<HD>(), st>>>(
       T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, (bf16*)dqkv,
-      nullptr, nullptr, 0, 1, nullptr, nullptr, glm.ctx, glm.pos, glm.pos2);
+      nullptr, nullptr, 0, 1, nullptr, nullptr, glm.ctx, glm.pos, glm.pos2, dbias);
   FL_CUDA_TRY(cudaGetLastError());
   if (pre.len > 0) {
     // prefix key tiles x slices of all query tiles, about two CTAs per SM in total
@@ -733,7 +782,7 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
     if (nsplit < 1) nsplit = 1;
     attn_bwd_dkv_kernel<HD, true><<<dim3(npt * nsplit, nh), 128, dkv_smem<HD>(), st>>>(
         T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, nullptr, pk,
-        pv, pre.len, nsplit, pre.dk, pre.dv, nullptr, nullptr, nullptr);
+        pv, pre.len, nsplit, pre.dk, pre.dv, nullptr, nullptr, nullptr, nullptr);
     FL_CUDA_TRY(cudaGetLastError());
   }
   return FL_OK;
@@ -769,12 +818,12 @@ int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu
 
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
-                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st) {
+                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st, float* dbias) {
   if (n_tiles <= 0) return FL_OK;
   if (hd == 128)
-    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, st);
+    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias, st);
   if (hd == 64)
-    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, st);
+    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 

@@ -105,6 +105,8 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
     return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: block positions only with the RoPE epilogue");
   }
   if (a->bias && !aligned16(a->bias)) return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: bias alignment");
+  if (a->colsum && mode != FL_EPI_GELU_BWD)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: column sums only with the GeLU-backward epilogue");
 
   Epi e;
   e.mode = mode;
@@ -137,6 +139,7 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   e.wd = a->weight_decay;
   e.inv_bc1 = a->inv_bc1;
   e.inv_bc2 = a->inv_bc2;
+  e.colsum = a->colsum;
 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const bool amn = a->a_mn_major != 0, bmn = a->b_mn_major != 0;

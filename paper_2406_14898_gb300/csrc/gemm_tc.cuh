@@ -65,6 +65,7 @@ struct Epi {
   const float *ln_mean, *ln_rstd, *ln_gamma, *ln_beta;  // residual = LayerNorm(aux) when ln_mean
   float *adam_m, *adam_v;
   float lr, b1, b2, eps, wd, inv_bc1, inv_bc2;
+  float* colsum;  // GELU_BWD: column sums of D added here (bias gradient of the up-projection)
 };
 
 // Epilogue families: each kernel instantiation carries only its family's code, which keeps
@@ -121,6 +122,8 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
   const int32_t* rpos_src = region == 0 ? e.pos : e.pos2;
   const bool first = rcol < half;
   const bool gelu_bwd = FAM == FAM_GELU && e.mode == FL_EPI_GELU_BWD;
+  const bool colsum = FAM == FAM_GELU && gelu_bwd && e.colsum != nullptr;
+  float cs[4] = {0.f, 0.f, 0.f, 0.f};  // this lane's column sums over its rows of the chunk
   const bool accum = FAM == FAM_PLAIN && e.mode == FL_EPI_ACCUM_F32;
   const bool out_f32 = e.mode == FL_EPI_STORE_F32 || e.d_f32;
 #pragma unroll 1
@@ -192,6 +195,10 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
         if (gelu_bwd) {
 #pragma unroll
           for (int q = 0; q < 4; ++q) y[q] *= gelu_tanh_grad(a4[q]);
+          if (colsum) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) cs[q] += y[q];
+          }
         } else {
           st_quad(e.aux_out + (int64_t)m * e.ld_aux_out + n, make_float4(y[0], y[1], y[2], y[3]));
 #pragma unroll
@@ -222,6 +229,14 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
       } else {
         st_quad(reinterpret_cast<__nv_bfloat16*>(e.D) + off, make_float4(y[0], y[1], y[2], y[3]));
       }
+    }
+  }
+  if (colsum) {  // the two half-warps hold the same columns for rows of either parity
+#pragma unroll
+    for (int q = 0; q < 4; ++q) cs[q] += __shfl_xor_sync(0xffffffffu, cs[q], 16);
+    if (h == 0 && rows > 0) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) atomicAdd(e.colsum + n + q, cs[q]);
     }
   }
 }

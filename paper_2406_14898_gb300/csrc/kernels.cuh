@@ -1,5 +1,6 @@
 // Internal launch interfaces shared by the kernels and the server runtime.
 #pragma once
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -88,9 +89,19 @@ int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu
 int fl_launch_attn_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
                           void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
                           cudaStream_t st);
+// dbias (or null): += the column sums of dqkv [3H] (the QKV bias gradient), per CTA.
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
-                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st);
+                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
+                       float* dbias = nullptr);
+
+// LayerNorm backward on fp32 dy / x (rowops.cu): fl_k_layernorm_bwd, and, when dcol is not
+// null, dcol += the column sums of dx.  workspace: fl_launch_layernorm_bwd_workspace bytes.
+size_t fl_launch_layernorm_bwd_workspace(int T, int H);
+int fl_launch_layernorm_bwd_f32(int T, int H, const float* dy, const float* x, const float* mean, const float* rstd,
+                                const float* gamma, const float* resid, float resid_alpha, __nv_bfloat16* dx_bf16,
+                                float* dx_f32, float* dgamma, float* dbeta, float* dcol, float* workspace,
+                                cudaStream_t st);
 
 // Host helper: builds the tile list of a packing (returns the count, -1 if over capacity).
 int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles);

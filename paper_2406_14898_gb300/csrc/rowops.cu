@@ -134,11 +134,13 @@ __global__ void __launch_bounds__(128) ln_fwd_row_kernel(int H, const TX* __rest
 }
 
 // Backward: dx = rstd (g - mean(g) - xhat mean(g xhat)), g = gamma dy (+ alpha resid);
-// thread c keeps its columns' dgamma / dbeta partials in registers across the CTA's rows
-// and writes them to workspace[blockIdx.x][2][H]; ln_bwd_reduce_kernel adds them up.
-// Kept at <= 64 registers (gamma re-read from L1 each row, no register prefetch of the
-// next row) so that two 512-thread CTAs share an SM and cover each other's latency.
-template <typename T>
+// thread c keeps its columns' dgamma / dbeta partials (and with CS the column sums of dx,
+// the bias gradient of the GEMM whose output gradient dx is) in registers across the
+// CTA's rows and writes them to workspace[blockIdx.x][2 + CS][H]; ln_bwd_reduce_kernel
+// adds them up.  Kept at <= 64 registers (gamma re-read from L1 each row, no register
+// prefetch of the next row) so that two 512-thread CTAs share an SM and cover each
+// other's latency.
+template <typename T, bool CS>
 __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy,
                                                         const T* __restrict__ x, const float* __restrict__ mean,
                                                         const float* __restrict__ rstd,
@@ -147,9 +149,11 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
                                                         float* __restrict__ dx_f32, float* __restrict__ ws) {
   __shared__ float2 red[2][32];
   const int c = threadIdx.x;
-  float accg[8], accb[8];
+  float accg[8], accb[8], accd[CS ? 8 : 1];
 #pragma unroll
   for (int k = 0; k < 8; ++k) accg[k] = accb[k] = 0.f;
+#pragma unroll
+  for (int k = 0; k < (CS ? 8 : 1); ++k) accd[k] = 0.f;
   int par = 0;
   for (int row = blockIdx.x; row < Tn; row += gridDim.x) {
     float d[8], xh[8], gcol[8];
@@ -179,6 +183,10 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
 #pragma unroll
       for (int k = 0; k < 8; ++k) o[k] = fmaf(resid_alpha, r[k], o[k]);
     }
+    if constexpr (CS) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) accd[k] += o[k];
+    }
     if (dx_bf16) reinterpret_cast<uint4*>(dx_bf16 + (int64_t)row * H)[c] = pack8(o);
     if (dx_f32) {
       float4* df = reinterpret_cast<float4*>(dx_f32 + (int64_t)row * H) + 2 * c;
@@ -186,37 +194,48 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
       df[1] = make_float4(o[4], o[5], o[6], o[7]);
     }
   }
-  float* out = ws + (int64_t)blockIdx.x * 2 * H;
+  float* out = ws + (int64_t)blockIdx.x * (CS ? 3 : 2) * H;
   float4* og = reinterpret_cast<float4*>(out + 8 * c);
   float4* ob = reinterpret_cast<float4*>(out + H + 8 * c);
   og[0] = make_float4(accg[0], accg[1], accg[2], accg[3]);
   og[1] = make_float4(accg[4], accg[5], accg[6], accg[7]);
   ob[0] = make_float4(accb[0], accb[1], accb[2], accb[3]);
   ob[1] = make_float4(accb[4], accb[5], accb[6], accb[7]);
+  if constexpr (CS) {
+    float4* od = reinterpret_cast<float4*>(out + 2 * H + 8 * c);
+    od[0] = make_float4(accd[0], accd[1], accd[2], accd[3]);
+    od[1] = make_float4(accd[4], accd[5], accd[6], accd[7]);
+  }
 }
 
-// dgamma/dbeta += sum over the nblk partial rows; blockIdx.y takes a slice of the rows.
-__global__ void ln_bwd_reduce_kernel(int nblk, int H, const float* __restrict__ ws, float* __restrict__ dgamma,
-                                     float* __restrict__ dbeta) {
+// dgamma, dbeta (and dcol) += sum over the nblk partial rows of the nv = 2 (3) vectors;
+// blockIdx.y takes a slice of the rows.
+__global__ void ln_bwd_reduce_kernel(int nblk, int H, int nv, const float* __restrict__ ws, float* __restrict__ dgamma,
+                                     float* __restrict__ dbeta, float* __restrict__ dcol) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= 2 * H) return;
+  if (i >= nv * H) return;
   const int per = (nblk + gridDim.y - 1) / gridDim.y;
   const int b0 = blockIdx.y * per, b1 = min(nblk, b0 + per);
   if (b0 >= b1) return;
   float s = 0.f;
-  for (int b = b0; b < b1; ++b) s += ws[(int64_t)b * 2 * H + i];
-  atomicAdd(i < H ? dgamma + i : dbeta + (i - H), s);
+  for (int b = b0; b < b1; ++b) s += ws[(int64_t)b * nv * H + i];
+  atomicAdd(i < H ? dgamma + i : i < 2 * H ? dbeta + (i - H) : dcol + (i - 2 * H), s);
 }
 
 template <typename T>
 int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, const float* mean, const float* rstd,
                     const float* gamma, const void* resid, float alpha, void* dx_bf16, float* dx_f32, float* ws,
-                    float* dgamma, float* dbeta, cudaStream_t st) {
-  ln_bwd_kernel<T><<<nblk, H / 8, 0, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma, (const T*)resid, alpha,
-                                           (__nv_bfloat16*)dx_bf16, dx_f32, ws);
+                    float* dgamma, float* dbeta, float* dcol, cudaStream_t st) {
+  if (dcol)
+    ln_bwd_kernel<T, true><<<nblk, H / 8, 0, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
+                                                   (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws);
+  else
+    ln_bwd_kernel<T, false><<<nblk, H / 8, 0, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
+                                                    (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws);
   FL_CUDA_TRY(cudaGetLastError());
   const int split = nblk >= 64 ? 16 : 1;
-  ln_bwd_reduce_kernel<<<dim3((2 * H + 255) / 256, split), 256, 0, st>>>(nblk, H, ws, dgamma, dbeta);
+  const int nv = dcol ? 3 : 2;
+  ln_bwd_reduce_kernel<<<dim3((nv * H + 255) / 256, split), 256, 0, st>>>(nblk, H, nv, ws, dgamma, dbeta, dcol);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
@@ -462,9 +481,24 @@ extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const vo
   float* ws = (float*)workspace;
   return io_dtype == FL_DT_F32
              ? dispatch_ln_bwd<float>(nblk, T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16, dx_f32, ws,
-                                      dgamma, dbeta, st)
+                                      dgamma, dbeta, nullptr, st)
              : dispatch_ln_bwd<__nv_bfloat16>(nblk, T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16,
-                                              dx_f32, ws, dgamma, dbeta, st);
+                                              dx_f32, ws, dgamma, dbeta, nullptr, st);
+}
+
+// The runtime's LayerNorm backward on the fp32 residual stream: fl_k_layernorm_bwd plus
+// dcol += column sums of dx (the bias gradient of the GEMM whose output gradient dx is).
+// The workspace holds fl_launch_layernorm_bwd_workspace(T, H) bytes.
+size_t fl_launch_layernorm_bwd_workspace(int T, int H) {
+  return (size_t)ln_bwd_blocks(T > 0 ? T : 1) * 3 * (size_t)H * sizeof(float);
+}
+int fl_launch_layernorm_bwd_f32(int T, int H, const float* dy, const float* x, const float* mean, const float* rstd,
+                                const float* gamma, const float* resid, float resid_alpha, __nv_bfloat16* dx_bf16,
+                                float* dx_f32, float* dgamma, float* dbeta, float* dcol, float* workspace,
+                                cudaStream_t st) {
+  if (T == 0) return FL_OK;
+  return dispatch_ln_bwd<float>(ln_bwd_blocks(T), T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16, dx_f32,
+                                workspace, dgamma, dbeta, dcol, st);
 }
 
 extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream) {
@@ -645,5 +679,5 @@ extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, 
   int nblk = ln_bwd_blocks(T);
   if (nblk > FL_LN_NOALLOC_MAX_BLOCKS) nblk = FL_LN_NOALLOC_MAX_BLOCKS;
   return dispatch_ln_bwd<__nv_bfloat16>(nblk, T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx, nullptr, ws,
-                                        dgamma, dbeta, st);
+                                        dgamma, dbeta, nullptr, st);
 }

@@ -410,18 +410,25 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   BlockAct& A = h->act_of(b);
   cudaStream_t st = h->stream;
   const bool train_base = !c.freeze_base;
-  // FFN down: du = (dy W2) * gelu'(u); dW2 += dy^T g; db2 += colsum(dy)
+  // Bias gradients are column sums of the output gradients, added by the kernels that
+  // produce those: db2 (dy) by the LayerNorm-1 backward of block b + 1 (here by a column-sum
+  // kernel for the top block, whose dy comes from the clients), db1 (du) by the GeLU'
+  // epilogue, dbd (dh) by the LayerNorm-2 backward, dbqkv (dqkv) by the attention backward.
+  // FFN down: du = (dy W2) * gelu'(u), db1 += colsum(du); dW2 += dy^T g
   fl_gemm_args d1 = gemm_dgrad(T, F, H, dy, h->wbt(b, FL_T_WDOWN), h->du, FL_EPI_GELU_BWD);
   d1.aux = A.u;
   d1.ld_aux = F;
+  d1.colsum = train_base ? h->gt(b, FL_T_BUP) : nullptr;
   TRY(h, run_gemm(h, d1));
   if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
     TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g)));
-    prof_begin(h, FL_PROF_OTHER);
-    TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
-    prof_end(h);
+    if (b == c.n_blocks - 1) {
+      prof_begin(h, FL_PROF_OTHER);
+      TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
+      prof_end(h);
+    }
   }
-  // FFN up: dm = du W1 (+ alpha dy), fp32; dW1 += du^T m; db1 += colsum(du)
+  // FFN up: dm = du W1 (+ alpha dy), fp32; dW1 += du^T m
   fl_gemm_args d2 = gemm_dgrad(T, H, F, h->du, h->wbt(b, FL_T_WUP), h->dm, glm ? FL_EPI_RESID : FL_EPI_STORE);
   d2.d_dtype = FL_DT_F32;
   if (glm) {
@@ -431,31 +438,25 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d2.alpha = al;
   }
   TRY(h, run_gemm(h, d2));
-  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+  if (train_base)  // weight gradient (skipped when only the prefixes train)
     TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m)));
-    prof_begin(h, FL_PROF_OTHER);
-    TRY(h, fl_k_colsum(T, F, h->du, h->gt(b, FL_T_BUP), st));
-    prof_end(h);
-  }
-  // LN2 backward: dh = LN2'(dm) (+ alpha dy), bf16 and fp32
+  // LN2 backward: dh = LN2'(dm) (+ alpha dy), bf16 and fp32; dbd += colsum(dh)
   prof_begin(h, FL_PROF_LN, 2);
-  TRY(h, fl_k_layernorm_bwd(T, H, h->dm, A.h, FL_DT_F32, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dyf,
-                            al, h->dh, h->dhf, h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B), h->ln_ws, st));
+  TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->dm, A.h, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dyf, al,
+                                     h->dh, h->dhf, h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B),
+                                     train_base ? h->gt(b, FL_T_BDENSE) : nullptr, h->ln_ws, st));
   prof_end(h);
-  // dense: do = dh Wd; dWd += dh^T o; dbd += colsum(dh)
+  // dense: do = dh Wd; dWd += dh^T o
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
-  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+  if (train_base)  // weight gradient (skipped when only the prefixes train)
     TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)));
-    prof_begin(h, FL_PROF_OTHER);
-    TRY(h, fl_k_colsum(T, H, h->dh, h->gt(b, FL_T_BDENSE), st));
-    prof_end(h);
-  }
-  // attention backward -> dqkv (w.r.t. the un-rotated q, k)
+  // attention backward -> dqkv (w.r.t. the un-rotated q, k); dbqkv += colsum(dqkv)
   prof_begin(h, FL_PROF_ATTN, 3);
   TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
-                            h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st));
+                            h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st,
+                            train_base ? h->gt(b, FL_T_BQKV) : nullptr));
   prof_end(h);
-  // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a; dbqkv += colsum(dqkv)
+  // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
   d3.d_dtype = FL_DT_F32;
   if (glm) {
@@ -465,17 +466,14 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d3.alpha = al;
   }
   TRY(h, run_gemm(h, d3));
-  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+  if (train_base)  // weight gradient (skipped when only the prefixes train)
     TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a)));
-    prof_begin(h, FL_PROF_OTHER);
-    TRY(h, fl_k_colsum(T, 3 * H, h->dqkv, h->gt(b, FL_T_BQKV), st));
-    prof_end(h);
-  }
-  // LN1 backward: dx = LN1'(da) (+ alpha dh), bf16 and fp32
+  // LN1 backward: dx = LN1'(da) (+ alpha dh), bf16 and fp32; dx is dy of block b - 1, whose
+  // down-projection bias gradient is its column sum
   prof_begin(h, FL_PROF_LN, 2);
-  TRY(h, fl_k_layernorm_bwd(T, H, h->da, h->xs[b], FL_DT_F32, A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G),
-                            glm ? nullptr : h->dhf, al, dx, dxf, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B), h->ln_ws,
-                            st));
+  TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->da, h->xs[b], A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G),
+                                     glm ? nullptr : h->dhf, al, dx, dxf, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B),
+                                     train_base && b > 0 ? h->gt(b - 1, FL_T_BDOWN) : nullptr, h->ln_ws, st));
   prof_end(h);
   return FL_OK;
 }
@@ -603,7 +601,7 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
       (rc = dalloc(h, &h->dm, Tm * H)) || (rc = dalloc(h, &h->dh, Tm * H)) || (rc = dalloc(h, &h->d_o, Tm * H)) ||
       (rc = dalloc(h, &h->dqkv, Tm * 3 * H)) || (rc = dalloc(h, &h->da, Tm * H)) ||
       (rc = dalloc(h, &h->delta, Tm * c.n_heads)) ||
-      (rc = dalloc(h, &h->ln_ws, fl_k_layernorm_bwd_workspace((int32_t)Tm, (int32_t)H) / sizeof(float))) ||
+      (rc = dalloc(h, &h->ln_ws, fl_launch_layernorm_bwd_workspace((int)Tm, (int)H) / sizeof(float))) ||
       (rc = dalloc(h, &h->cu, FL_MAX_SEGS + 1)) || (rc = dalloc(h, &h->pos, Tm)) || (rc = dalloc(h, &h->pos2, Tm)) ||
       (rc = dalloc(h, &h->ctx, FL_MAX_SEGS)) ||
       (rc = dalloc(h, &h->tiles, FL_MAX_TILES)) || (rc = dalloc(h, &h->status, 1)))

@@ -67,7 +67,7 @@ class fl_gemm_args(C.Structure):
                 ("ln_beta", C.c_void_p), ("adam_m", C.c_void_p), ("adam_v", C.c_void_p),
                 ("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float), ("eps", C.c_float),
                 ("weight_decay", C.c_float), ("inv_bc1", C.c_float), ("inv_bc2", C.c_float),
-                ("pos2", C.c_void_p), ("tile", C.c_int32)]
+                ("pos2", C.c_void_p), ("tile", C.c_int32), ("colsum", C.c_void_p)]
 
 
 _P = C.c_void_p
@@ -416,12 +416,13 @@ def fl_k_gemm(args: fl_gemm_args, status=None, stream=None):
 def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
          alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
          aux_dtype=FL_DT_BF16, d_dtype=FL_DT_BF16, ln_mean=None, ln_rstd=None, ln_gamma=None, ln_beta=None,
-         pos2=None, tile=0, status=None, stream=None):
+         pos2=None, tile=0, colsum=None, status=None, stream=None):
     a = fl_gemm_args(M, N, K, ptr(A), lda, a_mn, ptr(B), ldb, b_mn, ptr(D), ldd, epilogue, ptr(bias), ptr(aux),
                      ld_aux, alpha, ptr(aux_out), ld_aux_out, ptr(pos), ptr(rope_tab), n_heads, head_dim, rotary_dim,
                      aux_dtype, d_dtype, ptr(ln_mean), ptr(ln_rstd), ptr(ln_gamma), ptr(ln_beta))
     a.pos2 = ptr(pos2)
     a.tile = tile
+    a.colsum = ptr(colsum)
     fl_k_gemm(a, status, stream)
 
 

@@ -117,10 +117,15 @@ def test_gemm_epilogues(F, tile):
     F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_RESID, aux=dR, ld_aux=N, alpha=alpha)
     torch.cuda.synchronize()
     assert rel_inf(f64(D), acc + alpha * R) < GEMM_TOL
-    # gelu' of a stored pre-activation
-    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_GELU_BWD, aux=dR, ld_aux=N)
+    # gelu' of a stored pre-activation; its column sums added to a vector (the up-projection
+    # bias gradient of the backward)
+    c0 = rng.standard_normal(N).astype(np.float32)
+    cs = dev_f32(c0)
+    F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_GELU_BWD, aux=dR, ld_aux=N, colsum=cs)
     torch.cuda.synchronize()
-    assert rel_inf(f64(D), acc * O.gelu_grad(R)) < GEMM_TOL
+    du = acc * O.gelu_grad(R)
+    assert rel_inf(f64(D), du) < GEMM_TOL
+    assert rel_inf(f64(cs) - c0, du.sum(axis=0)) < 1e-4
     # plain store with bias
     F.gemm(M, N, K, dA, lda, 0, dB, ldb, 0, D, N, tile=t, epilogue=F.FL_EPI_STORE, bias=db)
     torch.cuda.synchronize()

@@ -87,5 +87,8 @@ def test_kernel_entry_points_validate_before_launch(F):
     assert L.fl_k_gemm(ctypes.byref(a), None, None) == -7
     a.tile = F.FL_TILE_256x256_PAIR
     assert L.fl_k_gemm(ctypes.byref(a), None, None) == -7
+    a.tile = F.FL_TILE_AUTO
+    a.colsum = 0x40000                                              # only with FL_EPI_GELU_BWD
+    assert L.fl_k_gemm(ctypes.byref(a), None, None) == -7
     assert L.fl_k_layernorm_fwd(4, 300, None, 0, None, None, 1e-5, None, None, None, None) == -7
     assert L.fl_k_adamw(6, None, None, None, None, None, 1e-3, .9, .999, 1e-8, 0, .1, .001, None) == -1
