@@ -755,7 +755,7 @@ int launch_fwd(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t
 template <int HD>
 int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, const void* dout, const int32_t* cu,
                const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab, void* dqkv,
-               const AttnPrefix& pre, const AttnGlm& glm, float* dbias, cudaStream_t st) {
+               const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st) {
   if (int rc = set_attrs<HD>()) return rc;
   const int H = nh * HD;
   const float scale = 1.f / sqrtf((float)HD);
@@ -770,10 +770,16 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
       T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, tab, HD / 2, scale, (bf16*)dqkv, pk, pv,
       pre.len, glm.ctx, glm.pos, glm.pos2, dbias);
   FL_CUDA_TRY(cudaGetLastError());
-  attn_bwd_dkv_kernel<HD, false><<<dim3(n_tiles, nh), 128, dkv_smem<HD>(), st>>>(
-      T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, (bf16*)dqkv,
-      nullptr, nullptr, 0, 1, nullptr, nullptr, glm.ctx, glm.pos, glm.pos2, dbias);
-  FL_CUDA_TRY(cudaGetLastError());
+  if (HD == 128) {  // the segment's own keys on tcgen05 (attention_bwd_tc.cu)
+    if (int rc = fl_launch_attn_bwd_dkv_tc(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, glm, dbias,
+                                           status, st))
+      return rc;
+  } else {
+    attn_bwd_dkv_kernel<HD, false><<<dim3(n_tiles, nh), 128, dkv_smem<HD>(), st>>>(
+        T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, n_tiles, tab, HD / 2, scale, (bf16*)dqkv,
+        nullptr, nullptr, 0, 1, nullptr, nullptr, glm.ctx, glm.pos, glm.pos2, dbias);
+    FL_CUDA_TRY(cudaGetLastError());
+  }
   if (pre.len > 0) {
     // prefix key tiles x slices of all query tiles, about two CTAs per SM in total
     const int npt = (pre.len + BT - 1) / BT;
@@ -818,12 +824,15 @@ int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu
 
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
-                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st, float* dbias) {
+                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st, float* dbias,
+                       int* status) {
   if (n_tiles <= 0) return FL_OK;
   if (hd == 128)
-    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias, st);
+    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias,
+                           status, st);
   if (hd == 64)
-    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias, st);
+    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias,
+                          status, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 

@@ -454,7 +454,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   prof_begin(h, FL_PROF_ATTN, 3);
   TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
                             h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st,
-                            train_base ? h->gt(b, FL_T_BQKV) : nullptr));
+                            train_base ? h->gt(b, FL_T_BQKV) : nullptr, h->status));
   prof_end(h);
   // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);

@@ -248,7 +248,7 @@ def test_gemm_fp32_residual_epilogues(F, tile):
 
 @pytest.mark.parametrize("hd", [64, 128])
 def test_attention_fwd_bwd(F, hd):
-    seqs = [1, 64, 100, 130, 7, 64, 200]
+    seqs = [1, 64, 100, 130, 7, 64, 200] + ([520, 1030] if hd == 128 else [])
     nh = 2
     H = nh * hd
     cu = np.cumsum([0] + seqs).astype(np.int32)
@@ -274,7 +274,7 @@ def test_attention_fwd_bwd(F, hd):
     # backward (inverse rotary rotation folded in, as the server uses it)
     rd = hd // 2
     pos = np.concatenate([np.arange(L) for L in seqs]).astype(np.int32)
-    tab = rope_table(256, rd, 10000.0)
+    tab = rope_table(max(seqs), rd, 10000.0)
     delta = torch.empty((nh, T), dtype=torch.float32, device="cuda")
     dq = torch.full((T, 3 * H), float("nan"), dtype=torch.bfloat16, device="cuda")
     # the kernel differentiates through its own saved O (bf16), as the server does
