@@ -766,10 +766,16 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
   const float2* tab = reinterpret_cast<const float2*>(rope_tab);
   const bf16* pk = (const bf16*)pre.k;
   const bf16* pv = (const bf16*)pre.v;
-  attn_bwd_dq_kernel<HD><<<dim3(n_tiles, nh), 128, dq_smem<HD>(), st>>>(
-      T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, tab, HD / 2, scale, (bf16*)dqkv, pk, pv,
-      pre.len, glm.ctx, glm.pos, glm.pos2, dbias);
-  FL_CUDA_TRY(cudaGetLastError());
+  if (HD == 128) {  // tcgen05 (attention_bwd_tc.cu)
+    if (int rc = fl_launch_attn_bwd_dq_tc(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, pre, glm,
+                                          dbias, status, st))
+      return rc;
+  } else {
+    attn_bwd_dq_kernel<HD><<<dim3(n_tiles, nh), 128, dq_smem<HD>(), st>>>(
+        T, H, (const bf16*)qkv, (const bf16*)dout, lse, delta, cu, tiles, tab, HD / 2, scale, (bf16*)dqkv, pk, pv,
+        pre.len, glm.ctx, glm.pos, glm.pos2, dbias);
+    FL_CUDA_TRY(cudaGetLastError());
+  }
   if (HD == 128) {  // the segment's own keys on tcgen05 (attention_bwd_tc.cu)
     if (int rc = fl_launch_attn_bwd_dkv_tc(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, glm, dbias,
                                            status, st))

@@ -1,7 +1,8 @@
-// Attention backward, dK and dV, on the 5th-generation tensor cores (head_dim 128): the
-// same computation as attn_bwd_dkv_kernel<128, false> in attention.cu (the gradient of
-// App. A's softmax(Q K^T / sqrt(d_h)) V for the segment's own keys, causal or with a
-// bidirectional GLM context; the shared P-tuning prefix keys stay on the mma.sync kernel).
+// Attention backward on the 5th-generation tensor cores (head_dim 128): dQ, and dK / dV of
+// the segment's own keys, the same computations as attn_bwd_dq_kernel<128> and
+// attn_bwd_dkv_kernel<128, false> in attention.cu (the gradient of App. A's
+// softmax(Q K^T / sqrt(d_h)) V, causal or with a bidirectional GLM context, with the
+// P-tuning prefix keys in dQ; the prefix keys' own gradients stay on the mma.sync kernel).
 //
 // One CTA (8 warps) per (128-key tile, head).  Warp w reads TMEM lanes 32 (w % 4) .. + 31,
 // so thread (w, lane) owns key row r = 32 (w % 4) + lane, and takes query half w / 4 of
@@ -322,6 +323,243 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   }
 }
 
+// dQ: one CTA (8 warps) per (128-query tile, head); thread (w, lane) owns query row
+// r = 32 (w % 4) + lane and takes key half w / 4 of every key tile.  Per 128-key tile j
+// the queries see (the prefix tile first, then the segment's own keys):
+//   TMA: K_j and V_j (Q and dO once);  S = Q K_j^T -> TMEM [0, 128), dP = dO V_j^T ->
+//   TMEM [128, 256);  threads: dS = P (dP - delta_q), P = exp2(S scale log2e - lse_q
+//   log2e) on the visible keys, bf16 into shared memory as a K-major operand (rows =
+//   queries, K = keys);  dQ += dS K_j -> TMEM [256, 384) (K_j as an MN-major operand).
+// Epilogue as in the dK / dV kernel: dQ * scale, inverse rotary rotation(s), coalesced bf16
+// rows, q column sums for the bias gradient.
+__global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
+    const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do,
+    const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int T, int H,
+    const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, const float* __restrict__ lse,
+    const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale, float scale_log2, int Lp,
+    bf16* __restrict__ dqkv, const int32_t* __restrict__ ctxs, const int32_t* __restrict__ gpos,
+    const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int* status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sdO = smem + TILE;
+  uint8_t* sK = smem + 2 * TILE;
+  uint8_t* sV = smem + 3 * TILE;
+  uint8_t* sdS = smem + 4 * TILE;  // then, with the spare tile after it, the epilogue's scratch
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 6 * TILE + 2 * TB * 4);
+  uint64_t* bar_load = bars;
+  uint64_t* bar_mma1 = bars + 1;
+  uint64_t* bar_mma2 = bars + 2;
+  uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 4);
+
+  const int s = int(tiles[blockIdx.x] >> 16), idx64 = int(tiles[blockIdx.x] & 0xFFFFu);
+  if (idx64 & 1) return;
+  const int idx = idx64 >> 1;
+  const int h = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int quarter = warp & 3, kh = warp >> 2;
+  const int r = quarter * 32 + lane;  // this thread's query row (TMEM lane)
+  const int seg0 = cu[s], L = cu[s + 1] - seg0;
+  const int q0 = idx * TB;
+  const int q = q0 + r;
+  const bool q_ok = q < L;
+  const int npt = Lp > 0 ? 1 : 0;  // at most one prefix tile (Lp <= 128)
+  const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
+  const int n_kv = npt + max(idx, clast >= 0 ? clast / TB : 0) + 1;
+  const float lse2 = q_ok ? __ldg(lse + (int64_t)h * T + seg0 + q) * LOG2E_B : 0.f;
+  const float dl = q_ok ? __ldg(delta + (int64_t)h * T + seg0 + q) : 0.f;
+  const int ulim = q_ok ? max(q, clast) : -1;  // last own key visible to the row
+
+  if (tid == 0) {
+    mbar_init(bar_load, 1);
+    mbar_init(bar_mma1, 1);
+    mbar_init(bar_mma2, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_qkv);
+    tma_prefetch_desc(&tm_do);
+  }
+  if (warp == 0) {
+    tmem_alloc(holder, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *holder;
+  const uint32_t t_lane = tmem + (uint32_t(quarter * 32) << 16);
+
+  auto issue_kv = [&](int j) {  // one elected thread
+    if (j < npt) {
+      tma_load_2d(sK, &tm_pk, bar_load, h * HDT, 0);
+      tma_load_2d(sK + BOX, &tm_pk, bar_load, h * HDT + 64, 0);
+      tma_load_2d(sV, &tm_pv, bar_load, h * HDT, 0);
+      tma_load_2d(sV + BOX, &tm_pv, bar_load, h * HDT + 64, 0);
+    } else {
+      const int row = seg0 + (j - npt) * TB;
+      tma_load_2d(sK, &tm_qkv, bar_load, H + h * HDT, row);
+      tma_load_2d(sK + BOX, &tm_qkv, bar_load, H + h * HDT + 64, row);
+      tma_load_2d(sV, &tm_qkv, bar_load, 2 * H + h * HDT, row);
+      tma_load_2d(sV + BOX, &tm_qkv, bar_load, 2 * H + h * HDT + 64, row);
+    }
+  };
+  if (tid == 0) {
+    mbar_arrive_expect_tx(bar_load, 4 * TILE);
+    tma_load_2d(sQ, &tm_qkv, bar_load, h * HDT, seg0 + q0);
+    tma_load_2d(sQ + BOX, &tm_qkv, bar_load, h * HDT + 64, seg0 + q0);
+    tma_load_2d(sdO, &tm_do, bar_load, h * HDT, seg0 + q0);
+    tma_load_2d(sdO + BOX, &tm_do, bar_load, h * HDT + 64, seg0 + q0);
+    issue_kv(0);
+  }
+
+  constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
+  constexpr uint32_t IDESC_G = umma_idesc_bf16(TB, HDT, false, true);
+  bool ok = true;
+  uint32_t ph = 0;
+  for (int j = 0; j < n_kv && ok; ++j, ph ^= 1) {
+    if (!__syncthreads_and(mbar_wait(bar_load, ph))) {
+      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+      ok = false;
+      break;
+    }
+    // ---- S = Q K_j^T, dP = dO V_j^T
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t aq = smem_u32(sQ), ao = smem_u32(sdO), bk = smem_u32(sK), bv = smem_u32(sV);
+#pragma unroll
+      for (int kk = 0; kk < HDT / 16; ++kk) umma_bf16(tmem, desc_k(aq, kk), desc_k(bk, kk), IDESC_S, kk > 0);
+#pragma unroll
+      for (int kk = 0; kk < HDT / 16; ++kk) umma_bf16(tmem + 128, desc_k(ao, kk), desc_k(bv, kk), IDESC_S, kk > 0);
+      umma_commit(bar_mma1);
+    }
+    if (!__syncthreads_and(mbar_wait(bar_mma1, ph))) {
+      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
+      ok = false;
+      break;
+    }
+    tc_fence_after();
+    // ---- dS of query row r for keys kh * 64 .. + 63 of the tile, in two halves of 32
+    {
+      const bool prefix = j < npt;
+      const int u0 = (prefix ? 0 : (j - npt) * TB) + kh * 64;  // first key of the half
+      const int uend = prefix ? (q_ok ? Lp : 0) : ulim + 1;    // keys [u0, uend) are visible
+#pragma unroll 1
+      for (int hf = 0; hf < 2; ++hf) {
+        uint32_t sr[32], dr[32];
+        tmem_ld32(t_lane + kh * 64 + 32 * hf, sr);
+        tmem_ld32(t_lane + 128 + kh * 64 + 32 * hf, dr);
+        tmem_ld_wait();
+#pragma unroll
+        for (int c8 = 0; c8 < 4; ++c8) {
+          float ds[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int c = 8 * c8 + e;
+            const bool vis = u0 + 32 * hf + c < uend;
+            const float pv = vis ? exp2_hw(fmaf(__uint_as_float(sr[c]), scale_log2, -lse2)) : 0.f;
+            ds[e] = pv * (__uint_as_float(dr[c]) - dl);
+          }
+          put_chunk8(sdS, kh, r, 4 * hf + c8, ds);
+        }
+      }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    // ---- dQ += dS K_j
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t as = smem_u32(sdS), bk = smem_u32(sK);
+#pragma unroll
+      for (int kk = 0; kk < TB / 16; ++kk)
+        umma_bf16(tmem + 256, desc_k(as, kk), desc_mn(bk, kk), IDESC_G, (j > 0 || kk > 0) ? 1u : 0u);
+      umma_commit(bar_mma2);
+    }
+    if (!__syncthreads_and(mbar_wait(bar_mma2, ph))) {
+      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
+      ok = false;
+      break;
+    }
+    tc_fence_after();
+    if (tid == 0 && j + 1 < n_kv) {
+      mbar_arrive_expect_tx(bar_load, 2 * TILE);
+      issue_kv(j + 1);
+    }
+  }
+
+  // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * 64 .. + 63 of query row r,
+  // staged in the freed K buffer and written as whole coalesced rows; the rotary rows of
+  // the tile's queries in the freed V buffer (32 KB: one region) or, with GLM block
+  // positions, V and dO (64 KB); the bias scratch in dS + the spare buffer (64 KB).
+  if (ok) {
+    float* scratch = reinterpret_cast<float*>(sdS) + warp * 32 * 64;
+    const int nreg = rope_tab ? (gpos2 ? 2 : 1) : 0;
+    for (int reg = 0; reg < nreg; ++reg) {  // warp w loads rows w, w + 8, ...: 16 in flight
+      float2* rtr = reg == 0 ? reinterpret_cast<float2*>(sV) : reinterpret_cast<float2*>(sdO);
+      const int32_t* gp = reg == 0 ? gpos : gpos2;
+      int pos[TB / 8];
+#pragma unroll
+      for (int jj = 0; jj < TB / 8; ++jj) {
+        const int qq = min(q0 + warp + 8 * jj, L - 1);
+        pos[jj] = gp ? __ldg(gp + seg0 + qq) : qq;
+      }
+      float2 cs[TB / 8];
+#pragma unroll
+      for (int jj = 0; jj < TB / 8; ++jj) cs[jj] = __ldg(rope_tab + (int64_t)pos[jj] * 32 + lane);
+#pragma unroll
+      for (int jj = 0; jj < TB / 8; ++jj) {
+        const int rr = warp + 8 * jj;
+        rtr[rr * 32 + (lane ^ (rr & 31))] = cs[jj];
+      }
+    }
+    __syncthreads();
+    uint32_t vr[64];
+    tmem_ld32(t_lane + 256 + kh * 64, *reinterpret_cast<uint32_t(*)[32]>(vr));
+    tmem_ld32(t_lane + 256 + kh * 64 + 32, *reinterpret_cast<uint32_t(*)[32]>(vr + 32));
+    tmem_ld_wait();
+    float* v = reinterpret_cast<float*>(vr);
+#pragma unroll
+    for (int c = 0; c < 64; ++c) v[c] = __uint_as_float(vr[c]) * scale;
+    if (kh < nreg && q_ok)
+      inverse_rope_row(v, reinterpret_cast<float2*>(kh == 0 ? sV : sdO) + r * 32, r & 31);
+#pragma unroll
+    for (int c8 = 0; c8 < 8; ++c8) {
+      const int jc = kh * 8 + c8;
+      *reinterpret_cast<uint4*>(sK + r * 256 + ((jc ^ (r & 15)) << 4)) =
+          make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
+                     pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
+    }
+    const int col = blockIdx.y * HDT;
+    if (dbias) {
+#pragma unroll
+      for (int c = 0; c < 64; ++c) scratch[lane * 64 + (c ^ lane)] = q_ok ? v[c] : 0.f;
+      __syncwarp();
+      float s0 = 0.f, s1 = 0.f;
+#pragma unroll 8
+      for (int rr = 0; rr < 32; ++rr) {
+        s0 += scratch[rr * 64 + (lane ^ rr)];
+        s1 += scratch[rr * 64 + ((lane + 32) ^ rr)];
+      }
+      atomicAdd(dbias + col + kh * 64 + lane, s0);
+      atomicAdd(dbias + col + kh * 64 + lane + 32, s1);
+    }
+    __syncthreads();  // the tile is staged
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int id = tid + 256 * i, row = id >> 4, jc = id & 15;
+      if (q0 + row < L) {
+        const uint4 w = *reinterpret_cast<const uint4*>(sK + row * 256 + ((jc ^ (row & 15)) << 4));
+        *reinterpret_cast<uint4*>(dqkv + ((int64_t)seg0 + q0 + row) * 3 * H + col + jc * 8) = w;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
 }  // namespace
 
 int fl_launch_attn_bwd_dkv_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
@@ -340,6 +578,33 @@ int fl_launch_attn_bwd_dkv_tc(int T, int nh, const void* qkv, const void* dout, 
   attn_bwd_dkv_tc_kernel<<<dim3(n_tiles, nh), 256, SMEM, st>>>(
       tq, tdo, T, H, cu, tiles, lse, delta, reinterpret_cast<const float2*>(rope_tab), scale, scale * LOG2E_B,
       (bf16*)dqkv, glm.ctx, glm.pos, glm.pos2, dbias, status);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
+int fl_launch_attn_bwd_dq_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
+                             const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab, void* dqkv,
+                             const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st) {
+  static bool attr = false;
+  if (!attr) {
+    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dq_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM));
+    attr = true;
+  }
+  const int H = nh * HDT;
+  CUtensorMap tq, tdo, tpk, tpv;
+  if (int rc = fl_gemm::make_map(&tq, qkv, (uint64_t)3 * H, (uint64_t)T, 3 * (int64_t)H, 128)) return rc;
+  if (int rc = fl_gemm::make_map(&tdo, dout, (uint64_t)H, (uint64_t)T, H, 128)) return rc;
+  if (pre.len > 0) {
+    if (int rc = fl_gemm::make_map(&tpk, pre.k, (uint64_t)H, (uint64_t)pre.len, H, 128)) return rc;
+    if (int rc = fl_gemm::make_map(&tpv, pre.v, (uint64_t)H, (uint64_t)pre.len, H, 128)) return rc;
+  } else {
+    tpk = tq;
+    tpv = tq;
+  }
+  const float scale = 1.f / sqrtf((float)HDT);
+  attn_bwd_dq_tc_kernel<<<dim3(n_tiles, nh), 256, SMEM, st>>>(
+      tq, tdo, tpk, tpv, T, H, cu, tiles, lse, delta, reinterpret_cast<const float2*>(rope_tab), scale,
+      scale * LOG2E_B, pre.len, (bf16*)dqkv, glm.ctx, glm.pos, glm.pos2, dbias, status);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }

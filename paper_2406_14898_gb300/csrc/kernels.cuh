@@ -90,12 +90,15 @@ int fl_launch_attn_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, con
                           void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
                           cudaStream_t st);
 // dbias (or null): += the column sums of dqkv [3H] (the QKV bias gradient), per CTA.
-// head_dim 128 computes dK / dV of the segments' own keys on tcgen05 (attention_bwd_tc.cu),
-// whose bounded waits report into `status` (device int or null).
+// head_dim 128 computes dQ and dK / dV of the segments' own keys on tcgen05
+// (attention_bwd_tc.cu), whose bounded waits report into `status` (device int or null).
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
                        void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
                        float* dbias = nullptr, int* status = nullptr);
+int fl_launch_attn_bwd_dq_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
+                             const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab, void* dqkv,
+                             const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st);
 int fl_launch_attn_bwd_dkv_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
                               const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab,
                               void* dqkv, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st);
