@@ -15,7 +15,7 @@
 //   dV += P^T dO_i  -> TMEM [256, 384)   dK += dS^T Q_i -> TMEM [384, 512)
 //            (dO_i and Q_i as MN-major operands).
 // Epilogue: dK * scale, the inverse rotary rotation(s), bf16 rows of dqkv, and the k / v
-// column sums for the QKV bias gradient.  Shared memory 197 KB and 512 TMEM columns: one
+// column sums for the QKV bias gradient.  Shared memory 195 KB and 512 TMEM columns: one
 // CTA per SM.  Every mbarrier wait is bounded (2 s): on expiry the CTA records a status
 // code and leaves its remaining work undone.
 #include <cuda.h>
