@@ -71,6 +71,19 @@ FL_DEV float exp2_hw(float x) {
   return y;
 }
 
+// Adds the column sums of a staged 128 x 128 bf16 tile (rows of 256 bytes, 16-byte chunk j
+// of row r at j ^ (r & 15)) over its first `rows` rows to out[0..128): thread c < 128 sums
+// column c in row order, one atomic per column.
+FL_DEV void staged_colsum(const uint8_t* stage, int rows, float* out, int tid) {
+  if (tid >= TB) return;
+  const int jc = tid >> 3, e = tid & 7;
+  float acc = 0.f;
+#pragma unroll 8
+  for (int row = 0; row < rows; ++row)
+    acc += __bfloat162float(*reinterpret_cast<const bf16*>(stage + row * 256 + ((jc ^ (row & 15)) << 4) + 2 * e));
+  atomicAdd(out + tid, acc);
+}
+
 __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do, int T, int H,
     const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, const float* __restrict__ lse,
@@ -243,11 +256,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   // ---- dK (scaled, rotated back) and dV: thread (r, qh) takes dims qh * 64 .. + 63 of key
   // row r from TMEM, stages the bf16 rows in the freed K (dK) and V (dV) buffers (16-byte
   // chunk j of row r at position j ^ (r & 15)), then the CTA writes whole rows with
-  // coalesced 16-byte stores.  The freed Q / dO buffers (64 KB) hold a per-warp 32 x 64
-  // fp32 scratch for the bias column sums (entry c of row l at c ^ l), the freed P / dS
-  // buffers (64 KB) the rotary table rows of the tile's keys.
+  // coalesced 16-byte stores; the bias column sums are taken from the staged rows (the
+  // values stored).  The freed P / dS buffers (64 KB) hold the rotary table rows of the
+  // tile's keys.
   if (ok && it0 < nq) {
-    float* scratch = reinterpret_cast<float*>(sQ) + warp * 32 * 64;
     // rotary rows: region 0 (position) and, with GLM block positions, region 1; entry e of
     // row rr at e ^ (rr & 31), loaded with coalesced reads
     float2* rt = reinterpret_cast<float2*>(sP);
@@ -289,21 +301,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
                        pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
       }
       const int col = (part ? 2 * H : H) + blockIdx.y * HDT;
-      if (dbias) {  // column sums over the warp's valid rows, then one atomic per column
-#pragma unroll
-        for (int c = 0; c < 64; ++c) scratch[lane * 64 + (c ^ lane)] = key_ok ? v[c] : 0.f;
-        __syncwarp();
-        float s0 = 0.f, s1 = 0.f;
-#pragma unroll 8
-        for (int rr = 0; rr < 32; ++rr) {
-          s0 += scratch[rr * 64 + (lane ^ rr)];
-          s1 += scratch[rr * 64 + ((lane + 32) ^ rr)];
-        }
-        atomicAdd(dbias + col + qh * 64 + lane, s0);
-        atomicAdd(dbias + col + qh * 64 + lane + 32, s1);
-        __syncwarp();
-      }
       __syncthreads();  // the tile is staged
+      if (dbias) staged_colsum(stage, min(TB, L - kb), dbias + col, tid);
       // 128 rows x 16 chunks: consecutive threads write consecutive chunks of a row
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
@@ -331,7 +330,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
 //   log2e) on the visible keys, bf16 into shared memory as a K-major operand (rows =
 //   queries, K = keys);  dQ += dS K_j -> TMEM [256, 384) (K_j as an MN-major operand).
 // Epilogue as in the dK / dV kernel: dQ * scale, inverse rotary rotation(s), coalesced bf16
-// rows, q column sums for the bias gradient.
+// rows, q column sums for the bias gradient.  Shared memory: five tiles used of the
+// kernels' common allocation.
 __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do,
     const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int T, int H,
@@ -345,7 +345,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   uint8_t* sdO = smem + TILE;
   uint8_t* sK = smem + 2 * TILE;
   uint8_t* sV = smem + 3 * TILE;
-  uint8_t* sdS = smem + 4 * TILE;  // then, with the spare tile after it, the epilogue's scratch
+  uint8_t* sdS = smem + 4 * TILE;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 6 * TILE + 2 * TB * 4);
   uint64_t* bar_load = bars;
   uint64_t* bar_mma1 = bars + 1;
@@ -487,11 +487,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   }
 
   // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * 64 .. + 63 of query row r,
-  // staged in the freed K buffer and written as whole coalesced rows; the rotary rows of
-  // the tile's queries in the freed V buffer (32 KB: one region) or, with GLM block
-  // positions, V and dO (64 KB); the bias scratch in dS + the spare buffer (64 KB).
+  // staged in the freed K buffer and written as whole coalesced rows, the bias column sums
+  // taken from the staged rows; the rotary rows of the tile's queries in the freed V buffer
+  // (32 KB: one region) or, with GLM block positions, V and dO (64 KB).
   if (ok) {
-    float* scratch = reinterpret_cast<float*>(sdS) + warp * 32 * 64;
     const int nreg = rope_tab ? (gpos2 ? 2 : 1) : 0;
     for (int reg = 0; reg < nreg; ++reg) {  // warp w loads rows w, w + 8, ...: 16 in flight
       float2* rtr = reg == 0 ? reinterpret_cast<float2*>(sV) : reinterpret_cast<float2*>(sdO);
@@ -529,20 +528,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
                      pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
     }
     const int col = blockIdx.y * HDT;
-    if (dbias) {
-#pragma unroll
-      for (int c = 0; c < 64; ++c) scratch[lane * 64 + (c ^ lane)] = q_ok ? v[c] : 0.f;
-      __syncwarp();
-      float s0 = 0.f, s1 = 0.f;
-#pragma unroll 8
-      for (int rr = 0; rr < 32; ++rr) {
-        s0 += scratch[rr * 64 + (lane ^ rr)];
-        s1 += scratch[rr * 64 + ((lane + 32) ^ rr)];
-      }
-      atomicAdd(dbias + col + kh * 64 + lane, s0);
-      atomicAdd(dbias + col + kh * 64 + lane + 32, s1);
-    }
     __syncthreads();  // the tile is staged
+    if (dbias) staged_colsum(sK, min(TB, L - q0), dbias + col, tid);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int id = tid + 256 * i, row = id >> 4, jc = id & 15;
