@@ -93,7 +93,7 @@ typedef struct {
                                                leave clearly fewer SMs idle in the last wave) */
   float* colsum;                            /* FL_EPI_GELU_BWD only, or NULL: colsum[n] += sum over m of
                                                D[m,n] (fp32, before rounding; fp32 atomics, so the
-                                               order of the additions is not fixed) */
+                                               order of the additions is not fixed); 16-byte aligned */
 } fl_gemm_args;
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);

@@ -107,6 +107,8 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   if (a->bias && !aligned16(a->bias)) return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: bias alignment");
   if (a->colsum && mode != FL_EPI_GELU_BWD)
     return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: column sums only with the GeLU-backward epilogue");
+  if (a->colsum && !aligned16(a->colsum))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: colsum must be 16-byte aligned");
 
   Epi e;
   e.mode = mode;

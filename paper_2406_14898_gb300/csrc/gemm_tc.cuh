@@ -234,10 +234,7 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
   if (colsum) {  // the two half-warps hold the same columns for rows of either parity
 #pragma unroll
     for (int q = 0; q < 4; ++q) cs[q] += __shfl_xor_sync(0xffffffffu, cs[q], 16);
-    if (h == 0 && rows > 0) {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) atomicAdd(e.colsum + n + q, cs[q]);
-    }
+    if (h == 0 && rows > 0) red_add_v4(e.colsum + n, cs[0], cs[1], cs[2], cs[3]);
   }
 }
 

@@ -202,6 +202,12 @@ FL_DEV void umma_commit_pair(uint64_t* bar, uint16_t cta_mask) {
       : "memory");
 }
 
+// out[0..4) += v, one vector reduction in the memory system (16-byte aligned address).
+FL_DEV void red_add_v4(float* out, float a, float b, float c, float d) {
+  asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(out), "f"(a), "f"(b), "f"(c), "f"(d)
+               : "memory");
+}
+
 // ------------------------------------------------------------------ warp-level MMA (attention)
 FL_DEV void ldmatrix_x4(uint32_t saddr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
