@@ -44,3 +44,19 @@ def test_single_rank_is_identity():
     import bench
     assert bench.slowest_rank_ms(12.5, 1) == 12.5
     assert bench.job_tokens_per_s(1, 1000, 2, 500.0) == pytest.approx(4000.0)
+
+
+def test_stored_traffic_used_only_for_the_current_gemm_sources(tmp_path):
+    """The roofline's DRAM traffic comes from a committed ncu summary only while the GEMM
+    sources it was measured on are unchanged (their fingerprint is in the summary) and
+    only for the workload it names."""
+    import bench
+    fp = bench.kernel_version()
+    good = tmp_path / "gemm_x_stack26.md"
+    good.write_text(f"fingerprint: {fp}\ntraffic_bytes_per_launch: 123456\n")
+    assert bench.ncu_traffic(str(good), "stack26")["bytes_per_launch"] == 123456
+    assert bench.ncu_traffic(str(good), "block6b") is None            # another workload
+    stale = tmp_path / "gemm_y_stack26.md"
+    stale.write_text("fingerprint: 0000000000000000\ntraffic_bytes_per_launch: 123456\n")
+    assert bench.ncu_traffic(str(stale), "stack26") is None            # other GEMM sources
+    assert bench.ncu_traffic(str(tmp_path / "missing_stack26.md"), "stack26") is None
