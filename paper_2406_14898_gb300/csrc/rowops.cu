@@ -31,9 +31,6 @@ FL_DEV void unpack8(const uint4& w, float* f) {
   float2 a = unpack_bf16x2(w.x), b = unpack_bf16x2(w.y), c = unpack_bf16x2(w.z), d = unpack_bf16x2(w.w);
   f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y; f[4] = c.x; f[5] = c.y; f[6] = d.x; f[7] = d.y;
 }
-// Makes the compiler treat v as redefined, so that values derived from it are recomputed
-// instead of being kept live in registers across passes.
-FL_DEV void opaque(uint4& v) { asm volatile("" : "+r"(v.x), "+r"(v.y), "+r"(v.z), "+r"(v.w)); }
 
 FL_DEV uint4 pack8(const float* f) {
   uint4 w;
