@@ -754,7 +754,7 @@ int launch_fwd(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t
 
 template <int HD>
 int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, const void* dout, const int32_t* cu,
-               const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab, void* dqkv,
+               const uint32_t* tiles, int n_tiles, int n_tiles128, float* delta, const float* rope_tab, void* dqkv,
                const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st) {
   if (int rc = set_attrs<HD>()) return rc;
   const int H = nh * HD;
@@ -767,8 +767,8 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
   const bf16* pk = (const bf16*)pre.k;
   const bf16* pv = (const bf16*)pre.v;
   if (HD == 128) {  // tcgen05 (attention_bwd_tc.cu)
-    if (int rc = fl_launch_attn_bwd_dq_tc(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, pre, glm,
-                                          dbias, status, st))
+    if (int rc = fl_launch_attn_bwd_dq_tc(T, nh, qkv, dout, lse, delta, cu, tiles + n_tiles, n_tiles128, rope_tab,
+                                          dqkv, pre, glm, dbias, status, st))
       return rc;
   } else {
     attn_bwd_dq_kernel<HD><<<dim3(n_tiles, nh), 128, dq_smem<HD>(), st>>>(
@@ -777,8 +777,8 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
     FL_CUDA_TRY(cudaGetLastError());
   }
   if (HD == 128) {  // the segment's own keys on tcgen05 (attention_bwd_tc.cu)
-    if (int rc = fl_launch_attn_bwd_dkv_tc(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, glm, dbias,
-                                           status, st))
+    if (int rc = fl_launch_attn_bwd_dkv_tc(T, nh, qkv, dout, lse, delta, cu, tiles + n_tiles, n_tiles128, rope_tab,
+                                           dqkv, glm, dbias, status, st))
       return rc;
   } else {
     attn_bwd_dkv_kernel<HD, false><<<dim3(n_tiles, nh), 128, dkv_smem<HD>(), st>>>(
@@ -802,16 +802,16 @@ int launch_bwd(int T, int nh, const void* qkv, const void* o, const float* lse, 
 
 }  // namespace
 
-int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles) {
+int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles, int rows) {
   int maxq = 0;
   for (int s = 0; s < S; ++s) {
-    const int nq = (cu[s + 1] - cu[s] + BT - 1) / BT;
+    const int nq = (cu[s + 1] - cu[s] + rows - 1) / rows;
     maxq = nq > maxq ? nq : maxq;
   }
   int n = 0;
   for (int i = maxq - 1; i >= 0; --i)
     for (int s = 0; s < S; ++s) {
-      const int nq = (cu[s + 1] - cu[s] + BT - 1) / BT;
+      const int nq = (cu[s + 1] - cu[s] + rows - 1) / rows;
       if (i < nq) {
         if (n >= max_tiles) return -1;
         tiles[n++] = (uint32_t(s) << 16) | uint32_t(i);
@@ -821,24 +821,25 @@ int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles) {
 }
 
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
+                       int n_tiles128,
                        void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st, int* status) {
   if (n_tiles <= 0) return FL_OK;
-  if (hd == 128) return fl_launch_attn_fwd_tc(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, status, st);
+  if (hd == 128) return fl_launch_attn_fwd_tc(T, nh, qkv, cu, tiles + n_tiles, n_tiles128, o, lse, pre, glm, status, st);
   if (hd == 64) return launch_fwd<64>(T, nh, qkv, cu, tiles, n_tiles, o, lse, pre, glm, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
-                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
-                       void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st, float* dbias,
-                       int* status) {
+                       const int32_t* cu, const uint32_t* tiles, int n_tiles, int n_tiles128, float* delta,
+                       const float* rope_tab, void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
+                       float* dbias, int* status) {
   if (n_tiles <= 0) return FL_OK;
   if (hd == 128)
-    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias,
-                           status, st);
+    return launch_bwd<128>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, n_tiles128, delta, rope_tab, dqkv, pre, glm,
+                           dbias, status, st);
   if (hd == 64)
-    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, delta, rope_tab, dqkv, pre, glm, dbias,
-                          status, st);
+    return launch_bwd<64>(T, nh, qkv, o, lse, dout, cu, tiles, n_tiles, n_tiles128, delta, rope_tab, dqkv, pre, glm,
+                          dbias, status, st);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }
 
@@ -851,16 +852,20 @@ extern "C" int32_t fl_k_attention_tiles(const int32_t* cu_host, int32_t S) {
   return n;
 }
 
-static int upload_tiles(const int32_t* cu_host, int32_t S, int32_t* tile_ws, int* n_out) {
+// The 64-row tile list followed by the 128-row one (at most as long) in tile_ws.
+static int upload_tiles(const int32_t* cu_host, int32_t S, int32_t* tile_ws, int* n_out, int* n128_out) {
   const int n = fl_k_attention_tiles(cu_host, S);
-  std::vector<uint32_t> t(n > 0 ? n : 1);
-  const int got = fl_build_tiles(cu_host, S, t.data(), n);
-  if (got != n) return fl_internal_error(FL_ERR_INVALID_ARG, "attention: bad cu_seqlens");
   for (int s = 0; s < S; ++s)
     if (cu_host[s + 1] < cu_host[s] || cu_host[s + 1] - cu_host[s] > 65535 * BT)
       return fl_internal_error(FL_ERR_INVALID_ARG, "attention: bad cu_seqlens");
-  if (n > 0) FL_CUDA_TRY(cudaMemcpy(tile_ws, t.data(), n * sizeof(uint32_t), cudaMemcpyHostToDevice));
+  std::vector<uint32_t> t(2 * (n > 0 ? n : 1));
+  const int got = fl_build_tiles(cu_host, S, t.data(), n);
+  if (got != n) return fl_internal_error(FL_ERR_INVALID_ARG, "attention: bad cu_seqlens");
+  const int n128 = n > 0 ? fl_build_tiles(cu_host, S, t.data() + n, n, 2 * BT) : 0;
+  if (n128 < 0) return fl_internal_error(FL_ERR_INVALID_ARG, "attention: bad cu_seqlens");
+  if (n > 0) FL_CUDA_TRY(cudaMemcpy(tile_ws, t.data(), (n + n128) * sizeof(uint32_t), cudaMemcpyHostToDevice));
   *n_out = n;
+  *n128_out = n128;
   return FL_OK;
 }
 
@@ -873,15 +878,15 @@ extern "C" int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: cu_seqlens");
   if (prefix_len < 0 || prefix_len > 128 || (prefix_len > 0 && (!prefix_k || !prefix_v)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: prefix (length 0..128)");
-  int n = 0;
-  if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n)) return rc;
+  int n = 0, n128 = 0;
+  if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n, &n128)) return rc;
   AttnPrefix pre;
   pre.k = prefix_k;
   pre.v = prefix_v;
   pre.len = prefix_len;
   AttnGlm glm;
   glm.ctx = context_lens;
-  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, o, lse, pre, glm,
+  return fl_launch_attn_fwd(T, n_heads, head_dim, qkv, cu_seqlens, (const uint32_t*)tile_ws, n, n128, o, lse, pre, glm,
                             (cudaStream_t)stream);
 }
 
@@ -901,8 +906,8 @@ extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   if (prefix_len < 0 || prefix_len > 128 ||
       (prefix_len > 0 && (!prefix_k || !prefix_v || !dprefix_k || !dprefix_v)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: prefix (length 0..128, gradients required)");
-  int n = 0;
-  if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n)) return rc;
+  int n = 0, n128 = 0;
+  if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n, &n128)) return rc;
   AttnPrefix pre;
   pre.k = prefix_k;
   pre.v = prefix_v;
@@ -913,6 +918,6 @@ extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   glm.ctx = context_lens;
   glm.pos = positions;
   glm.pos2 = block_positions;
-  return fl_launch_attn_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_seqlens, (const uint32_t*)tile_ws, n, delta_ws,
-                            rope_tab, dqkv, pre, glm, (cudaStream_t)stream);
+  return fl_launch_attn_bwd(T, n_heads, head_dim, qkv, o, lse, dout, cu_seqlens, (const uint32_t*)tile_ws, n, n128,
+                            delta_ws, rope_tab, dqkv, pre, glm, (cudaStream_t)stream);
 }

@@ -106,16 +106,15 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   uint64_t* bar_mma2 = bars + 2;
   uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 4);
 
-  // the 64-row tile list of the other kernels: even entries are this kernel's 128-row tiles
-  const int s = int(tiles[blockIdx.x] >> 16), idx64 = int(tiles[blockIdx.x] & 0xFFFFu);
-  if (idx64 & 1) return;
+  // the 128-row tile list: (segment, tile), tile i standing for key tile nq - 1 - i
+  const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
   const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, qh = warp >> 2;
   const int r = quarter * 32 + lane;  // this thread's key row (TMEM lane)
   const int seg0 = cu[s], L = cu[s + 1] - seg0;
   const int nq = (L + TB - 1) / TB;
-  const int kt = nq - 1 - (idx64 >> 1);  // key tile: most work first
+  const int kt = nq - 1 - idx;  // key tile: most work first
   const int kb = kt * TB;
   const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
   const int it0 = kb <= clast ? 0 : kt;  // a tile holding context keys is seen by every query
@@ -352,9 +351,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   uint64_t* bar_mma2 = bars + 2;
   uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 4);
 
-  const int s = int(tiles[blockIdx.x] >> 16), idx64 = int(tiles[blockIdx.x] & 0xFFFFu);
-  if (idx64 & 1) return;
-  const int idx = idx64 >> 1;
+  // the 128-row tile list: (segment, query tile)
+  const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
   const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, kh = warp >> 2;

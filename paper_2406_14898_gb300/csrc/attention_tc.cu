@@ -61,10 +61,8 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   uint64_t* bar_pv = bars + 2;
   uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 4);
 
-  // the 64-row tile list of the other kernels: even entries are this kernel's 128-row tiles
-  const int s = int(tiles[blockIdx.x] >> 16), idx64 = int(tiles[blockIdx.x] & 0xFFFFu);
-  if (idx64 & 1) return;
-  const int idx = idx64 >> 1;
+  // the 128-row tile list: (segment, query tile)
+  const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
   const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5;
   const int seg0 = cu[s], L = cu[s + 1] - seg0;

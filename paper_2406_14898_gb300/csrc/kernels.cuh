@@ -33,10 +33,11 @@ struct CopyTable {
 // ctx[s] (0: plain causal segment) and mask-token position mpos[s] < ctx[s].
 struct MetaArgs {
   int S;
-  int n_tiles;
+  int n_tiles;    // 64-row tiles, then n_tiles128 128-row tiles (the tcgen05 attention kernels)
+  int n_tiles128;
   int glm;
   int32_t cu[FL_MAX_SEGS + 1];
-  uint32_t tiles[FL_MAX_TILES];
+  uint32_t tiles[2 * FL_MAX_TILES];
   int32_t ctx[FL_MAX_SEGS];
   int32_t mpos[FL_MAX_SEGS];
 };
@@ -84,7 +85,7 @@ struct AttnGlm {
 // head_dim 128 runs on tcgen05 (attention_tc.cu), head_dim 64 on mma.sync; `status`
 // (device int or null) receives a code if a bounded wait inside the kernel gave up.
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
-                       int n_tiles, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm,
+                       int n_tiles, int n_tiles128, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm,
                        cudaStream_t st, int* status = nullptr);
 int fl_launch_attn_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
                           void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
@@ -93,7 +94,8 @@ int fl_launch_attn_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, con
 // head_dim 128 computes dQ and dK / dV of the segments' own keys on tcgen05
 // (attention_bwd_tc.cu), whose bounded waits report into `status` (device int or null).
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
-                       const int32_t* cu, const uint32_t* tiles, int n_tiles, float* delta, const float* rope_tab,
+                       const int32_t* cu, const uint32_t* tiles, int n_tiles, int n_tiles128, float* delta,
+                       const float* rope_tab,
                        void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
                        float* dbias = nullptr, int* status = nullptr);
 int fl_launch_attn_bwd_dq_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
@@ -111,5 +113,8 @@ int fl_launch_layernorm_bwd_f32(int T, int H, const float* dy, const float* x, c
                                 float* dx_f32, float* dgamma, float* dbeta, float* dcol, float* workspace,
                                 cudaStream_t st);
 
-// Host helper: builds the tile list of a packing (returns the count, -1 if over capacity).
-int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles);
+// Host helper: builds the tile list of a packing, tiles of `rows` query rows (64 for the
+// mma.sync kernels, 128 for the tcgen05 ones), segments' last tiles first (returns the
+// count, -1 if over capacity).  A device tile list holds the 64-row list followed by the
+// 128-row one.
+int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles, int rows = 64);

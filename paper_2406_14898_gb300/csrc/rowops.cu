@@ -385,7 +385,7 @@ __global__ void meta_kernel(MetaArgs a, int32_t* __restrict__ cu, int32_t* __res
   const int64_t nth = (int64_t)gridDim.x * blockDim.x;
   const int T = a.cu[a.S];
   for (int64_t i = tid; i <= a.S; i += nth) cu[i] = a.cu[i];
-  for (int64_t i = tid; i < a.n_tiles; i += nth) tiles[i] = a.tiles[i];
+  for (int64_t i = tid; i < a.n_tiles + a.n_tiles128; i += nth) tiles[i] = a.tiles[i];
   if (ctx)
     for (int64_t i = tid; i < a.S; i += nth) ctx[i] = a.glm ? a.ctx[i] : 0;
   for (int64_t t = tid; t < T; t += nth) {

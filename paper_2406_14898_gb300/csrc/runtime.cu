@@ -140,7 +140,7 @@ struct fl_server {
 
   // pending step
   bool pending = false;
-  int T = 0, S = 0, K = 0, n_tiles = 0;
+  int T = 0, S = 0, K = 0, n_tiles = 0, n_tiles128 = 0;
   std::vector<int32_t> seq_lens;
 
   Prof prof;
@@ -353,7 +353,7 @@ int block_forward(fl_server* h, int b, bool output = true) {
   TRY(h, run_gemm(h, g1));
   // o = causal attention within each segment
   prof_begin(h, FL_PROF_ATTN);
-  TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, A.o, A.lse,
+  TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, h->n_tiles128, A.o, A.lse,
                             h->prefix(b, false), h->glm_args(), st, h->status));
   prof_end(h);
   // h = alpha * (LN1(x) or x) + o Wd^T + bd, fp32; LN1(x) recomputed in fp32 in the epilogue
@@ -452,7 +452,8 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)));
   // attention backward -> dqkv (w.r.t. the un-rotated q, k); dbqkv += colsum(dqkv)
   prof_begin(h, FL_PROF_ATTN, 3);
-  TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles, h->delta,
+  TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles,
+                            h->n_tiles128, h->delta,
                             h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st,
                             train_base ? h->gt(b, FL_T_BQKV) : nullptr, h->status));
   prof_end(h);
@@ -604,7 +605,7 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
       (rc = dalloc(h, &h->ln_ws, fl_launch_layernorm_bwd_workspace((int)Tm, (int)H) / sizeof(float))) ||
       (rc = dalloc(h, &h->cu, FL_MAX_SEGS + 1)) || (rc = dalloc(h, &h->pos, Tm)) || (rc = dalloc(h, &h->pos2, Tm)) ||
       (rc = dalloc(h, &h->ctx, FL_MAX_SEGS)) ||
-      (rc = dalloc(h, &h->tiles, FL_MAX_TILES)) || (rc = dalloc(h, &h->status, 1)))
+      (rc = dalloc(h, &h->tiles, 2 * FL_MAX_TILES)) || (rc = dalloc(h, &h->status, 1)))
     return fail(rc);
 
   // rotary table: [position][pair i] = (cos, sin) of p * base^(-2i/rdim), in double
@@ -690,11 +691,14 @@ static int forward_impl(fl_server_t h, const void* const client_states[], const 
   }
   const int nt = fl_build_tiles(meta.cu, (int)S, meta.tiles, FL_MAX_TILES);
   if (nt < 0) return set_err(h, FL_ERR_CAPACITY, "forward: more than %d attention tiles", FL_MAX_TILES);
+  const int nt128 = fl_build_tiles(meta.cu, (int)S, meta.tiles + nt, FL_MAX_TILES, 128);  // never more than nt
   meta.n_tiles = nt;
+  meta.n_tiles128 = nt128;
   h->T = (int)T;
   h->S = (int)S;
   h->K = K;
   h->n_tiles = nt;
+  h->n_tiles128 = nt128;
   h->seq_lens.assign(seq_lens, seq_lens + K);
 
   prof_begin(h, FL_PROF_OTHER);
