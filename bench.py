@@ -58,6 +58,21 @@ def describe(cfg: syn.ServerConfig) -> str:
     return d
 
 
+def config_dict(cfg: syn.ServerConfig, world: int = 1, recompute: bool = False) -> dict:
+    """The `config` object of the JSON line; the GPU arm and the reference arm print the same one."""
+    return {"workload": describe(cfg), "global_batch": world * cfg.tokens, "seq_len": max(cfg.seq_lens),
+            "parallelism": "replicas" if world > 1 else "single GPU",
+            "l2": "working set (~125 GB of weights, optimizer state and activations) is far larger "
+                  "than L2; no flush needed",
+            "step": "pack + forward + unpack + backward with the AdamW update of every parameter "
+                    "(fl_server_forward + fl_server_backward_step: the weight-matrix update runs in "
+                    "the weight-gradient GEMM epilogues)",
+            "recompute": (f"on: each block's activations recomputed in the backward "
+                          f"({recompute_flops(cfg) / 1e12:.1f} TFLOP per step beyond the algorithmic "
+                          f"FLOPs; counted in roofline.achieved, not in pct_bf16_peak)")
+            if recompute else "off: every activation kept"}
+
+
 def glm_args(cfg: syn.ServerConfig) -> dict:
     """forward() keyword arguments of a workload: the GLM structure when it has one."""
     if not cfg.glm:
@@ -197,7 +212,10 @@ class OracleSample:
         sample_tokens = self.nseg * self.L
         t_step = cfg.n_blocks * ((t1 - t0) * cfg.tokens / sample_tokens + (t2 - t1) * self.ADAM_FRACTION)
         return {"t_fwd_bwd_s": t1 - t0, "t_adamw_s": t2 - t1, "sample_tokens": sample_tokens,
-                "t_step_s": t_step, "tokens_per_s": cfg.tokens / t_step,
+                "t_sample_s": t2 - t0, "t_step_s": t_step, "tokens_per_s": cfg.tokens / t_step,
+                "dtype": "f64", "cores": cpu_cores(),
+                "rule": (f"full step = n_blocks x (t_fwd_bwd x {cfg.tokens}/{sample_tokens} + t_adamw x "
+                         f"{self.ADAM_FRACTION})"),
                 "sample": (f"1 of {cfg.n_blocks} blocks at the workload's shapes, {self.nseg} segment(s) x {self.L} "
                            f"tokens fwd+bwd, plus AdamW over 1/{self.ADAM_FRACTION} of that block's parameters; "
                            f"fp64 numpy; full step estimated as n_blocks x (t_fwd_bwd x {cfg.tokens}/"
@@ -212,24 +230,35 @@ def cpu_cores() -> int:
 
 
 def run_reference(args, cfg: syn.ServerConfig):
+    """The reference arm: the oracle as it stands, on the host cores.  Each of the K timed
+    steps is one bounded sample of the workload (see OracleSample); `ms_per_step` is the
+    sample's own measured time, and `value` the workload's tokens/s extrapolated from it
+    (flagged, with the factor)."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     sample = OracleSample(cfg, min(cfg.tokens, args.ref_tokens))
     for _ in range(args.warmup):
         sample.run()
-    ts, last = [], None
+    runs = []
+    t0 = time.perf_counter()
     for _ in range(args.steps):
-        last = sample.run()
-        ts.append(last["t_step_s"])
-    t = statistics.mean(ts)
-    value = cfg.tokens / t
+        runs.append(sample.run())
+    wall = time.perf_counter() - t0
+    t_sample = statistics.mean(r["t_sample_s"] for r in runs)
+    t_step = statistics.mean(r["t_step_s"] for r in runs)
+    value = cfg.tokens / t_step
+    last = runs[-1]
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": describe(cfg), "global_batch": cfg.tokens,
-                       "seq_len": max(cfg.seq_lens), "parallelism": "cpu"},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_sample,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": last["dtype"],
+            "data": "synthetic", "config": config_dict(cfg, int(os.environ.get("WORLD_SIZE", "1"))),
+            "extrapolated": True,
+            "extrapolation": {"factor": t_step / t_sample,
+                              "basis": "each timed step is one sample (ms_per_step is its measured time); value = "
+                                       "the workload's tokens / (sample time x factor), " + last["rule"],
+                              "sample_tokens": last["sample_tokens"], "timed_wall_s": wall},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": last["cores"], "kind": "oracle",
                              "sample": last["sample"]},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -246,6 +275,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-other-configs", action="store_true",
+                    help="skip the ragged workload and the packed-vs-sequential points after the main line")
     ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the oracle sample")
     ap.add_argument("--ref-tokens", type=int, default=256, help="tokens of the reference-arm sample")
     ap.add_argument("--sweep", action="store_true",
@@ -435,23 +466,19 @@ def main():
                "ms_per_step": ems / args.steps}
 
     srv.close()
+    del states, gouts, outs, gins
+    torch.cuda.empty_cache()
+    others = None
+    if world == 1 and args.workload == "stack26" and not (args.ptuning or args.glm or args.recompute) \
+            and not args.no_other_configs:
+        others = run_other_configs(max(3, min(args.steps, 5)), 3, dev, stream)
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded N(0,0.02) weights, N(0,1) states, "
                                                        "N(0,1e-3) output-state grads)",
-            "config": {"workload": describe(cfg), "global_batch": world * cfg.tokens, "seq_len": max(cfg.seq_lens),
-                       "parallelism": "replicas" if world > 1 else "single GPU",
-                       "l2": "working set (~125 GB of weights, optimizer state and activations) is far larger "
-                             "than L2; no flush needed",
-                       "step": "pack + forward + unpack + backward with the AdamW update of every parameter "
-                               "(fl_server_forward + fl_server_backward_step: the weight-matrix update runs in "
-                               "the weight-gradient GEMM epilogues)",
-                       "recompute": (f"on: each block's activations recomputed in the backward "
-                                     f"({recompute_flops(cfg) / 1e12:.1f} TFLOP per step beyond the algorithmic "
-                                     f"FLOPs; counted in roofline.achieved, not in pct_bf16_peak)")
-                       if args.recompute else "off: every activation kept"},
+            "config": config_dict(cfg, world, args.recompute),
             "pct_bf16_peak": 100.0 * flops / (ms_step / 1e3) / (pk["bf16_sustained"] * 1e12),
             "pct_bf16_peak_basis": f"algorithmic FLOPs (GEMM + causal attention) of the whole step over the "
                                    f"{pk['source']} sustained bf16 peak {pk['bf16_sustained']} TFLOP/s",
@@ -477,6 +504,8 @@ def main():
                                     "kind": "oracle", "sample": cpu["sample"]}
         if e2e is not None:
             line["e2e"] = e2e
+        if others is not None:
+            line["other_configs"] = others
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -518,35 +547,9 @@ def run_sweep(args):
     go = [torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev) for b in gb]
     outs = [torch.empty_like(s) for s in st]
     gin = [torch.empty_like(s) for s in st]
-    pk = peaks()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     for K in ks:
         cfg = syn.sweep_config(K)
-
-        def batched():
-            srv.forward(st[:K], cfg.seq_lens, outs[:K])
-            srv.backward_step(go[:K], gin[:K], cfg.lr)
-
-        def sequential():
-            for k in range(K):
-                srv.forward(st[k:k + 1], cfg.seq_lens[k:k + 1], outs[k:k + 1])
-                srv.backward(go[k:k + 1], gin[k:k + 1])
-            srv.step(cfg.lr)
-
-        res = {}
-        for name, fn in (("batched", batched), ("sequential", sequential)):
-            for _ in range(args.warmup):
-                fn()
-            srv.sync()
-            e0.record(stream)
-            for _ in range(args.steps):
-                fn()
-            e1.record(stream)
-            srv.sync()
-            ms = e0.elapsed_time(e1) / args.steps
-            res[name] = {"tokens_per_s": cfg.tokens / (ms / 1e3), "ms_per_step": ms,
-                         "pct_bf16_peak": 100.0 * (gemm_flops(cfg) + attn_flops(cfg)) / (ms / 1e3)
-                         / (pk["bf16_sustained"] * 1e12)}
+        res = sweep_point(srv, K, st, go, outs, gin, args.steps, args.warmup, stream)
         line = {"metric": METRIC, "mode": "client-batching sweep", "K": K, "value": res["batched"]["tokens_per_s"],
                 "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
                 "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
@@ -555,6 +558,96 @@ def run_sweep(args):
                 "batched_over_sequential": res["batched"]["tokens_per_s"] / res["sequential"]["tokens_per_s"]}
         print(json.dumps(line), flush=True)
     srv.close()
+
+
+def sweep_point(srv, K: int, st, go, outs, gin, steps: int, warmup: int, stream) -> dict:
+    """One client-batching point (§3.3) on a server sized for at least K clients of the
+    sweep workload: the K clients' step as one packed call (client-batch) and as K
+    single-client calls followed by one AdamW update (serial), CUDA events on `stream`."""
+    import torch
+    cfg = syn.sweep_config(K)
+    pk = peaks()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def batched():
+        srv.forward(st[:K], cfg.seq_lens, outs[:K])
+        srv.backward_step(go[:K], gin[:K], cfg.lr)
+
+    def sequential():
+        for k in range(K):
+            srv.forward(st[k:k + 1], cfg.seq_lens[k:k + 1], outs[k:k + 1])
+            srv.backward(go[k:k + 1], gin[k:k + 1])
+        srv.step(cfg.lr)
+
+    res = {}
+    for name, fn in (("batched", batched), ("sequential", sequential)):
+        for _ in range(warmup):
+            fn()
+        srv.sync()
+        e0.record(stream)
+        for _ in range(steps):
+            fn()
+        e1.record(stream)
+        srv.sync()
+        ms = e0.elapsed_time(e1) / steps
+        res[name] = {"tokens_per_s": cfg.tokens / (ms / 1e3), "ms_per_step": ms, "steps": steps, "warmup": warmup,
+                     "pct_bf16_peak": 100.0 * (gemm_flops(cfg) + attn_flops(cfg)) / (ms / 1e3)
+                     / (pk["bf16_sustained"] * 1e12)}
+    return res
+
+
+def dev_bf16(torch, bits_list, dev):
+    return [torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).to(dev) for b in bits_list]
+
+
+def run_other_configs(steps: int, warmup: int, dev, stream) -> dict:
+    """The workload's sibling configurations, a few steps each, on fresh servers after the
+    main measurement: the ragged client-batching workload (26 blocks, K=16 clients x 1 row,
+    lengths U[64,1024] drawn with seed 7) and client-batching points of the sweep (26
+    blocks, K clients x 2 x 512 tokens): one packed call against K single-client calls."""
+    import torch
+    from paper_2406_14898_gb300 import flglm as F
+    pk = peaks()
+    out = {}
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    cfg = syn.CONFIGS["ragged26"]
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens, max(cfg.seq_lens)), cfg.seed, stream=stream)
+    st, go = dev_bf16(torch, syn.client_states(cfg), dev), dev_bf16(torch, syn.client_grads(cfg), dev)
+    outs, gin = [torch.empty_like(x) for x in st], [torch.empty_like(x) for x in st]
+    for _ in range(warmup):
+        srv.forward(st, cfg.seq_lens, outs)
+        srv.backward_step(go, gin, cfg.lr)
+    srv.sync()
+    e0.record(stream)
+    for _ in range(steps):
+        srv.forward(st, cfg.seq_lens, outs)
+        srv.backward_step(go, gin, cfg.lr)
+    e1.record(stream)
+    srv.sync()
+    ms = e0.elapsed_time(e1) / steps
+    out[cfg.name] = {"workload": describe(cfg), "tokens": cfg.tokens, "steps": steps, "warmup": warmup,
+                     "ms_per_step": ms, "tokens_per_s": cfg.tokens / (ms / 1e3),
+                     "pct_bf16_peak": 100.0 * (gemm_flops(cfg) + attn_flops(cfg)) / (ms / 1e3)
+                     / (pk["bf16_sustained"] * 1e12)}
+    srv.close()
+    del st, go, outs, gin
+    torch.cuda.empty_cache()
+    big = syn.sweep_config(max(OTHER_SWEEP_KS))
+    srv = F.Server(F.make_cfg(big, big.tokens, max(big.seq_lens)), big.seed, stream=stream)
+    st, go = dev_bf16(torch, syn.client_states(big), dev), dev_bf16(torch, syn.client_grads(big), dev)
+    outs, gin = [torch.empty_like(x) for x in st], [torch.empty_like(x) for x in st]
+    for K in OTHER_SWEEP_KS:
+        cfg = syn.sweep_config(K)
+        r = sweep_point(srv, K, st, go, outs, gin, steps, warmup, stream)
+        out[cfg.name] = {"workload": describe(cfg), "tokens": cfg.tokens, **r,
+                         "batched_over_sequential": r["batched"]["tokens_per_s"] / r["sequential"]["tokens_per_s"]}
+    srv.close()
+    del st, go, outs, gin
+    torch.cuda.empty_cache()
+    return out
+
+
+OTHER_SWEEP_KS = (2, 8)
 
 
 def run_strategies(args, K: int):

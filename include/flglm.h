@@ -42,7 +42,8 @@ extern "C" {
 
 #define FL_OK 0
 #define FL_ERR_INVALID_ARG (-1)  /* null pointer, bad size, misaligned buffer, bad id */
-#define FL_ERR_CAPACITY (-2)     /* total tokens of a call exceed cfg.max_tokens */
+#define FL_ERR_CAPACITY (-2)     /* a size exceeds a fixed capacity: total tokens of a call over
+                                  * cfg.max_tokens, or a fixed scratch array's limit */
 #define FL_ERR_STATE (-3)        /* protocol order violated (e.g. backward without forward) */
 #define FL_ERR_OOM (-4)          /* device allocation failed in fl_server_create */
 #define FL_ERR_CUDA (-5)         /* a CUDA runtime/driver call failed */
@@ -206,9 +207,16 @@ int fl_server_get_adam_moments(fl_server_t h, int32_t block, int32_t tensor_id, 
 int fl_server_average(fl_server_t const* replicas, int32_t n);
 
 /* Device address and element count of the fp32 master-weight arena, for averaging across
- * processes (one replica per GPU: all-reduce the arena, divide by the number of ranks,
- * then call fl_server_refresh_working_copy).  The arena is owned by the library. */
+ * processes (one replica per GPU: all-reduce (sum) the arena, then call
+ * fl_server_average_finish).  The arena is owned by the library. */
 int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n);
+
+/* Completes the §3.3 period-end average across processes: the caller has replaced this
+ * replica's master arena by the sum over n_replicas replicas (an all-reduce); this call
+ * scales it by 1/n_replicas in fp32, as fl_server_average does (so two replicas give the
+ * same bits either way), and refreshes the bf16 working copy, on the handle's stream.
+ * Errors: INVALID_ARG (null, n_replicas < 1), STATE (a forward is pending), CUDA. */
+int fl_server_average_finish(fl_server_t h, int32_t n_replicas);
 
 /* Recomputes the bf16 working copy from the fp32 master weights (after they were changed
  * outside the library), on the handle's stream. */

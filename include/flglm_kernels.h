@@ -113,17 +113,20 @@ int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const void* x, int3
                        const float* rstd, const float* gamma, const void* resid, float resid_alpha,
                        void* dx_bf16, float* dx_f32, float* dgamma, float* dbeta, void* workspace, void* stream);
 
-/* Allocation-free variant of fl_k_layernorm_bwd (same arguments minus the workspace,
- * same results up to the summation order of dgamma/dbeta).  The paper has no
+/* Allocation-free variant of fl_k_layernorm_bwd for bf16 tensors only: dy, x, resid and
+ * the single dx output are bf16 [T,H] (no io_dtype, no fp32 dx, no workspace); results
+ * equal fl_k_layernorm_bwd's bf16 dx up to the summation order of dgamma/dbeta.  The paper has no
  * counterpart: this exists for callers that cannot call cudaMalloc, such as a plug-in
  * inside a host framework that owns all device memory through its own pool, a serving
  * loop that must not pay cudaMalloc's implicit device synchronisation, or a process whose
  * device-memory budget is fully reserved.  Its per-CTA partial sums live in a fixed
  * 8 MiB array inside the library image (held by every GPU that loads the library until
  * the process exits); the call allocates nothing.  Limits: H <= 4096 (larger H returns
- * FL_ERR_CAPACITY), at most 256 CTAs.  The first call on each device looks up the
- * array's device address (cudaGetSymbolAddress) with that device current; make that
- * first call before any stream capture.  All calls share the array: calls that overlap
+ * FL_ERR_CAPACITY), at most 256 CTAs; T < 0 returns FL_ERR_INVALID_ARG.  The first call on
+ * each device looks up the array's device address (cudaGetSymbolAddress) with that device
+ * current and keeps it for the life of the process; make that first call before any stream
+ * capture, and do not call this function after cudaDeviceReset in the same process (the
+ * kept address would be stale).  All calls share the array: calls that overlap
  * on the GPU race, so serialise them (one stream, or events).  Nothing in the array
  * needs to start at zero: every CTA overwrites its slice before it is read. */
 int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,

@@ -52,6 +52,8 @@ struct ReplicaTable {
   void* wb[FL_MAX_REPLICAS];
 };
 int fl_launch_average(const ReplicaTable& t, int64_t n, cudaStream_t st);
+// w[i] *= 1/n_replicas (the factor fl_launch_average applies) and wb[i] = bf16(w[i]).
+int fl_launch_mean_finish(int64_t n, int n_replicas, float* w, void* wb, cudaStream_t st);
 // Writes cu_seqlens, the tile list, per-token positions (and, when pos2 != NULL, the GLM
 // block positions and, when ctx != NULL, the per-segment context lengths; both zero
 // without glm).

@@ -338,6 +338,18 @@ __global__ void __launch_bounds__(256) average_kernel(ReplicaTable t, int64_t n4
   }
 }
 
+// The last step of a mean taken across processes: the arena holds the sum of n replicas'
+// weights (an all-reduce), scaled here by 1/n as average_kernel does, bf16 copy refreshed.
+__global__ void __launch_bounds__(256) mean_finish_kernel(int64_t n4, float inv, float* __restrict__ w,
+                                                          __nv_bfloat16* __restrict__ wb) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+    const float4 s = reinterpret_cast<const float4*>(w)[i];
+    const float4 mean = make_float4(s.x * inv, s.y * inv, s.z * inv, s.w * inv);
+    reinterpret_cast<float4*>(w)[i] = mean;
+    reinterpret_cast<uint2*>(wb)[i] = make_uint2(pack_bf16x2(mean.x, mean.y), pack_bf16x2(mean.z, mean.w));
+  }
+}
+
 __global__ void f32_to_bf16_kernel(int64_t n, const float* __restrict__ src, __nv_bfloat16* __restrict__ dst) {
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
     dst[i] = f2bf(src[i]);
@@ -578,6 +590,14 @@ int fl_launch_average(const ReplicaTable& t, int64_t n, cudaStream_t st) {
   return FL_OK;
 }
 
+int fl_launch_mean_finish(int64_t n, int n_replicas, float* w, void* wb, cudaStream_t st) {
+  if (n % 4) return fl_internal_error(FL_ERR_INVALID_ARG, "mean finish: length %lld not a multiple of 4", (long long)n);
+  if (n <= 0) return FL_OK;
+  mean_finish_kernel<<<grid_for(n / 4), 256, 0, st>>>(n / 4, 1.f / (float)n_replicas, w, (__nv_bfloat16*)wb);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
 int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st) {
   if (n <= 0) return FL_OK;
   f32_to_bf16_kernel<<<grid_for(n), 256, 0, st>>>(n, src, (__nv_bfloat16*)dst);
@@ -641,7 +661,9 @@ std::mutex g_ln_scratch_mu;
 
 // Device address of the scratch array on the current device.  The host-side name of a
 // __device__ array is only a stand-in, so the address is looked up once per device with
-// that device current (the first call on each device does this).
+// that device current (the first call on each device does this) and kept for the life of
+// the process: after a cudaDeviceReset the cached address is stale, so the entry point
+// must not be called again in a process that has reset the device.
 int ln_scratch_address(float** out) {
   int dev = 0;
   FL_CUDA_TRY(cudaGetDevice(&dev));
@@ -661,7 +683,8 @@ int ln_scratch_address(float** out) {
 extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, const void* x, const float* mean,
                                           const float* rstd, const float* gamma, const void* resid,
                                           float resid_alpha, void* dx, float* dgamma, float* dbeta, void* stream) {
-  if (T < 0 || H <= 0 || (H % 256))
+  if (T < 0) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): T=%d is negative", T);
+  if (H <= 0 || (H % 256))
     return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd (no-alloc): H=%d must be a positive multiple of 256", H);
   if (H > FL_LN_NOALLOC_MAX_H)
     return fl_internal_error(FL_ERR_CAPACITY,

@@ -942,6 +942,16 @@ extern "C" int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n) {
   return FL_OK;
 }
 
+extern "C" int fl_server_average_finish(fl_server_t h, int32_t n_replicas) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "average finish: null handle");
+  if (n_replicas < 1) return set_err(h, FL_ERR_INVALID_ARG, "average finish: n_replicas=%d < 1", n_replicas);
+  if (h->pending) return set_err(h, FL_ERR_STATE, "average finish: a forward is pending");
+  prof_begin(h, FL_PROF_OTHER);
+  int rc = fl_launch_mean_finish(h->n_params, n_replicas, h->w, h->wb, h->stream);
+  prof_end(h);
+  return fwd_err(h, rc);
+}
+
 extern "C" int fl_server_refresh_working_copy(fl_server_t h) {
   if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "refresh: null handle");
   int rc = fl_launch_f32_to_bf16(h->n_params, h->w, h->wb, h->stream);

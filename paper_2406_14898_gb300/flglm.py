@@ -93,6 +93,7 @@ _SIGS = {
     "fl_server_average": (C.c_int, [C.POINTER(_P), _I32]),
     "fl_server_param_arena": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I64)]),
     "fl_server_refresh_working_copy": (C.c_int, [_P]),
+    "fl_server_average_finish": (C.c_int, [_P, _I32]),
     "fl_server_profile": (C.c_int, [_P, C.c_int]),
     "fl_server_profile_read": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(_I64), _I32]),
     "fl_server_launch_count": (_I64, [_P]),
@@ -295,6 +296,9 @@ class Server:
 
     def refresh_working_copy(self):
         check(lib().fl_server_refresh_working_copy(self.h), self.h)
+
+    def average_finish(self, n_replicas: int):
+        check(lib().fl_server_average_finish(self.h, n_replicas), self.h)
 
     def profile(self, enable: bool):
         check(lib().fl_server_profile(self.h, 1 if enable else 0), self.h)

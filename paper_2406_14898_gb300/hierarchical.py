@@ -3,10 +3,10 @@ replicas trained side by side and their parameters averaged at the end of every 
 
 On one GPU the replicas are independent fl_server handles, each on its own CUDA stream, so
 their kernels can overlap; fl_server_average forms the mean on the device.  Across GPUs
-(one replica per rank) the mean is an all-reduce of each replica's fp32 master-weight
-arena divided by the number of ranks, followed by a refresh of the bf16 working copy.
-All arithmetic runs in the CUDA library or in the collective; this module only orders
-the calls.
+(one replica per rank) the mean is an all-reduce (sum) of each replica's fp32 master-weight
+arena, then fl_server_average_finish scales it by 1/ranks and refreshes the bf16 working
+copy.  All arithmetic runs in the CUDA library or in the collective; this module only
+orders the calls.
 """
 from __future__ import annotations
 
@@ -30,24 +30,26 @@ def arena_tensor(server: F.Server):
     return torch.as_tensor(_ArenaView(ptr, n), device="cuda")
 
 
-def allreduce_mean_(tensor, group=None):
-    """In-place mean of `tensor` over the ranks of `group` (sum all-reduce, then divide)."""
+def allreduce_sum_(tensor, group=None):
+    """In-place sum of `tensor` over the ranks of `group` (the collective alone)."""
     import torch.distributed as dist
-    world = dist.get_world_size(group)
     dist.all_reduce(tensor, op=dist.ReduceOp.SUM, group=group)
-    tensor.div_(world)
     return tensor
 
 
-def average_across_ranks(server: F.Server, group=None):
-    """Period-end averaging with one replica per rank: all-reduce-mean of the master weights,
-    then the bf16 working copy is recomputed from them."""
+def average_across_ranks(server, group=None, arena=None):
+    """Period-end averaging with one replica per rank: all-reduce (sum) of the master
+    weights, then the library scales the sum by 1/ranks and refreshes the bf16 working copy.
+    `arena` (default: the server's master arena as a CUDA tensor) is the buffer the
+    collective sums."""
     import torch
+    import torch.distributed as dist
     server.sync()
-    w = arena_tensor(server)
-    allreduce_mean_(w, group)
-    torch.cuda.synchronize()
-    server.refresh_working_copy()
+    w = arena_tensor(server) if arena is None else arena
+    allreduce_sum_(w, group)
+    if w.is_cuda:
+        torch.cuda.synchronize()
+    server.average_finish(dist.get_world_size(group))
     server.sync()
 
 

@@ -10,7 +10,11 @@ At these sizes the oracle cannot run the whole packed batch, so the checks use w
 * the same segment run alone on the GPU gives weight gradients (first and last block,
   all 12 tensors) that must match the oracle's single-segment gradients (5e-2);
 * the packed call's weight gradients equal the serial strategy's (one client per call,
-  accumulated), and each client's outputs are bit-identical in both.
+  accumulated), and each client's outputs are bit-identical in both;
+* on the bench workload, one segment through fl_server_backward_step with the AdamW update
+  fused into the weight-gradient GEMM epilogues (the path bench.py times): the updated
+  weights and first Adam moments of the first and last block against the oracle's AdamW
+  step from its own gradients.
 
 The oracle uses the seeded weights of the synthetic generator; the library draws the
 same streams on the device (equal to within one fp32 ulp, tested elsewhere).
@@ -24,6 +28,7 @@ import torch
 import synthetic as syn
 from oracle import flglm_oracle as O
 from tests._gpu import bits, dev_bf16_from_bits, f64, flglm, need_gpu, rel_inf
+from tests.test_gpu_server import check_updated_weights
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
@@ -120,6 +125,39 @@ def serial_calls(F, cfg, states, grads, keep_clients):
     return res, wg
 
 
+def gpu_step_call(F, cfg, x_bits, g_bits):
+    """One segment alone through forward + fl_server_backward_step with the update fused into
+    the weight-gradient GEMMs (fused_step_min_tokens = 1: fused whatever the call's size).
+    Returns the updated fp32 weights and Adam moments (m) of CHECK_BLOCKS."""
+    L = x_bits.shape[0]
+    srv = F.Server(F.make_cfg(cfg, L, L, fused_step_min_tokens=1), cfg.seed)
+    st = [dev_bf16_from_bits(x_bits[None])]
+    outs = [torch.empty_like(st[0])]
+    srv.forward(st, [L], outs)
+    gi = [torch.empty_like(st[0])]
+    srv.backward_step([dev_bf16_from_bits(g_bits[None])], gi, cfg.lr)
+    srv.sync()
+    res = {b: [(srv.get_param(b, t), srv.get_adam_moments(b, t)[0]) for t in range(12)] for b in CHECK_BLOCKS}
+    assert not any(srv.get_grad(b, t).any() for b in CHECK_BLOCKS for t in range(12))
+    srv.close()
+    torch.cuda.empty_cache()
+    return res
+
+
+def check_fused_step(cfg, weights, stepped, wg_ref):
+    """Updated weights and m of CHECK_BLOCKS against the oracle's first AdamW step (t = 1,
+    zero moments) taken from the oracle's gradients of the same segment."""
+    for b in CHECK_BLOCKS:
+        for t in range(12):
+            w0 = weights[b][t].reshape(-1)
+            g = wg_ref[b][t].reshape(-1)
+            w_ref, m_ref, _ = O.adamw_update(w0.astype(np.float64), g, np.zeros_like(g), np.zeros_like(g), 1,
+                                             cfg.lr, cfg.adam_beta1, cfg.adam_beta2, cfg.adam_eps, cfg.weight_decay)
+            w, m = stepped[b][t]
+            check_updated_weights(w, w_ref, w0, g, cfg.lr, (cfg.name, "step", b, syn.TENSOR_NAMES[t]))
+            assert rel_inf(m, m_ref) < GRAD_TOL, (cfg.name, "adam m", b, syn.TENSOR_NAMES[t], rel_inf(m, m_ref))
+
+
 def sampled_segments(cfg):
     """(client, row) pairs to check: first and last; shortest and longest if ragged."""
     picks = {(0, 0), (cfg.K - 1, cfg.client_batch - 1)}
@@ -129,7 +167,7 @@ def sampled_segments(cfg):
     return sorted(picks)
 
 
-def run_workload(F, weights, cfg, n_oracle_segments=None, serial=True):
+def run_workload(F, weights, cfg, n_oracle_segments=None, serial=True, step=False):
     states = syn.client_states(cfg)
     grads = syn.client_grads(cfg)
     picks = sampled_segments(cfg)[:n_oracle_segments]
@@ -161,16 +199,28 @@ def run_workload(F, weights, cfg, n_oracle_segments=None, serial=True):
             for t in range(12):
                 e = rel_inf(wg1[b][t], wg_ref[b][t].reshape(-1))
                 assert e < GRAD_TOL, (cfg.name, k, r, "wgrad", b, syn.TENSOR_NAMES[t], e)
+        if step:
+            check_fused_step(cfg, weights, gpu_step_call(F, one, x, g), wg_ref)
+            step = False   # one segment is enough: the update is per element
 
 
 def test_stack26_fullsize(F, weights):
-    """26 blocks, K=8 clients x 4 rows x 256 tokens (T=8192), the bench workload."""
-    run_workload(F, weights, syn.CONFIGS["stack26"])
+    """26 blocks, K=8 clients x 4 rows x 256 tokens (T=8192), the bench workload, with the
+    fused backward + AdamW step of one segment."""
+    run_workload(F, weights, syn.CONFIGS["stack26"], step=True)
 
 
 def test_ragged26_fullsize(F, weights):
     """26 blocks, K=16 clients x 1 row, lengths U[64,1024] (seed 7), no padding."""
     run_workload(F, weights, syn.CONFIGS["ragged26"])
+
+
+@pytest.mark.parametrize("K", [1, 8])
+def test_sweep26_fullsize_vs_serial(F, weights, K):
+    """Sweep points K=1 and K=8 (2 rows x 512 tokens per client): the packed call against
+    the serial strategy (bit-identical per client, equal weight gradients) and one segment
+    against the oracle."""
+    run_workload(F, weights, syn.sweep_config(K), n_oracle_segments=1, serial=True)
 
 
 def test_sweep26_K32_fullsize(F, weights):

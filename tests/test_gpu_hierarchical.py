@@ -35,6 +35,37 @@ def test_average_is_the_mean(F):
         r.close()
 
 
+def test_average_finish_matches_average(F):
+    """The cross-process form: a replica whose arena holds the sum of two replicas' weights
+    (what an all-reduce leaves), finished by fl_server_average_finish(2), has the bits
+    fl_server_average gives, fp32 master and bf16 working copy (checked through a forward)."""
+    from paper_2406_14898_gb300.hierarchical import arena_tensor
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2)
+    a, b, c = (F.Server(F.make_cfg(cfg, cfg.tokens), seed) for seed in (4, 5, 6))
+    wa, wb, wc = arena_tensor(a), arena_tensor(b), arena_tensor(c)
+    torch.cuda.synchronize()
+    wc.copy_(wa + wb)
+    torch.cuda.synchronize()
+    c.average_finish(2)
+    F.fl_server_average([a, b])
+    c.sync()
+    torch.testing.assert_close(wc, wa, rtol=0, atol=0)
+    st = [dev_bf16_from_bits(s) for s in syn.client_states(cfg)]
+    outs = {}
+    for name, srv in (("a", a), ("c", c)):
+        o = [torch.empty_like(x) for x in st]
+        srv.forward(st, cfg.seq_lens, o)
+        srv.backward([torch.zeros_like(x) for x in st], [torch.empty_like(x) for x in st])
+        srv.sync()
+        outs[name] = o
+    for x, y in zip(outs["a"], outs["c"]):
+        assert torch.equal(x.view(torch.int16), y.view(torch.int16))
+    with pytest.raises(F.FlError):
+        c.average_finish(0)
+    for s_ in (a, b, c):
+        s_.close()
+
+
 def test_hierarchical_period_matches_oracle(F):
     """Two replicas, each trained two steps on its own client, then averaged; the averaged
     server's outputs for both clients match the oracle run of the same schedule."""

@@ -62,9 +62,28 @@ def test_noalloc_layernorm_bwd_matches_workspace_variant():
 
 
 def test_noalloc_layernorm_bwd_rejects_oversized_hidden():
+    """H above the fixed array's 4096 columns is refused before any launch.  The buffers
+    are real and sized for H = 8192, so that even a launch that slipped past the check
+    would stay inside memory the test owns."""
     need_gpu()
     F = flglm()
     L = F.lib()
-    rc = L.fl_k_layernorm_bwd_noalloc(4, 8192, 16, 16, 16, 16, 16, None, ctypes.c_float(0.0), 16, 16, 16, None)
+    T, H = 4, 8192
+    bf = [torch.zeros((T, H), dtype=torch.bfloat16, device="cuda") for _ in range(4)]  # dy, x, resid, dx
+    rows = [torch.ones(T, dtype=torch.float32, device="cuda") for _ in range(2)]         # mean, rstd
+    cols = [torch.zeros(H, dtype=torch.float32, device="cuda") for _ in range(3)]        # gamma, dgamma, dbeta
+    dy, x, res, dx = bf
+    mean, rstd = rows
+    gamma, dgam, dbet = cols
+    rc = L.fl_k_layernorm_bwd_noalloc(T, H, dy.data_ptr(), x.data_ptr(), mean.data_ptr(), rstd.data_ptr(),
+                                      gamma.data_ptr(), res.data_ptr(), ctypes.c_float(0.0), dx.data_ptr(),
+                                      dgam.data_ptr(), dbet.data_ptr(), None)
     assert rc == -2
     assert b"4096" in L.fl_server_last_error(None)
+    rc = L.fl_k_layernorm_bwd_noalloc(-1, 256, dy.data_ptr(), x.data_ptr(), mean.data_ptr(), rstd.data_ptr(),
+                                      gamma.data_ptr(), res.data_ptr(), ctypes.c_float(0.0), dx.data_ptr(),
+                                      dgam.data_ptr(), dbet.data_ptr(), None)
+    assert rc == -1
+    assert b"negative" in L.fl_server_last_error(None)
+    torch.cuda.synchronize()
+    assert not dgam.any() and not dbet.any() and not dx.view(torch.int16).any()
