@@ -14,7 +14,7 @@ Under torchrun (N > 1) each rank runs an independent replica of the server (the 
 is one GPU; there is no collective on the data path) and `value` counts every rank's
 tokens over the slowest rank's time.
 
---impl reference times the fp64 CPU oracle on a bounded sample of the same workload
+--impl reference times the fp32 C++ CPU oracle on a bounded sample of the same workload
 (the repository's reference arm; rank 0 only).
 """
 from __future__ import annotations
@@ -169,57 +169,58 @@ class ClockSampler:
 # ----------------------------------------------------------------------------- oracle CPU sample
 
 class OracleSample:
-    """Times the fp64 oracle on a bounded sample of `cfg`'s step: forward + backward of one
-    block at the workload's shapes over `tokens` tokens (segments of the workload's first
-    length), and one AdamW update over 1/ADAM_FRACTION of that block's parameters.  The
-    full step is estimated as n_blocks x (t_fwd_bwd x T / tokens + t_adamw x ADAM_FRACTION)."""
+    """Times the fp32 C++ oracle (oracle/flglm_oracle32.cpp, OpenMP over the host cores) on a
+    bounded sample of `cfg`'s step: forward + backward of one block at the workload's shapes
+    over `tokens` tokens (segments of the workload's first length), and one AdamW update over
+    1/ADAM_FRACTION of that block's parameters.  The full step is estimated as
+    n_blocks x (t_fwd_bwd x T / tokens + t_adamw x ADAM_FRACTION).  GLM and prefix workloads
+    are timed on their plain-causal block (the fp32 oracle covers the base path)."""
     ADAM_FRACTION = 16
 
     def __init__(self, cfg: syn.ServerConfig, tokens: int, seed: int = 0):
-        from oracle import flglm_oracle as O
-        self.O = O
+        from oracle import oracle32 as O32
+        self.O32 = O32
         self.cfg = cfg
         rng = np.random.default_rng(seed)
-        L = cfg.segment_lengths[0]
+        L = min(cfg.segment_lengths[0], tokens)
         self.nseg = max(1, tokens // L)
         self.L = L
-        self.one = cfg.with_(n_blocks=1, client_batch=1, seq_lens=(L,) * self.nseg)
-        params = [[cfg.init_std * rng.standard_normal(s) for s in syn.param_shapes(self.one)]]
+        self.one = cfg.with_(n_blocks=1, client_batch=1, seq_lens=(L,) * self.nseg, prefix_len=0, glm=0)
+        shapes = syn.param_shapes(self.one)
+        params = [[(cfg.init_std * rng.standard_normal(s)).astype(np.float32) for s in shapes]]
         for t, v in ((syn.T_G1, 1.0), (syn.T_G2, 1.0), (syn.T_BE1, 0.0), (syn.T_BE2, 0.0)):
             params[0][t][:] = v
         self.params = params
-        self.states = [rng.standard_normal((1, L, cfg.hidden)) for _ in range(self.nseg)]
-        self.grads = [1e-3 * rng.standard_normal((1, L, cfg.hidden)) for _ in range(self.nseg)]
-        # GLM workloads: the sample's segments take the GLM structure of the workload's first ones
-        self.glm = (None, None)
-        if cfg.glm:
-            ctx, mp = syn.glm_structure(cfg)
-            c = [min(x, L) for x in (ctx * self.nseg)[:self.nseg]]
-            self.glm = (c, [min(m, x - 1) if x > 0 else 0 for m, x in zip((mp * self.nseg)[:self.nseg], c)])
+        self.grads = [[np.zeros(s, np.float32) for s in shapes]]
+        T = self.nseg * L
+        self.cu = np.arange(self.nseg + 1, dtype=np.int32) * L
+        self.x = rng.standard_normal((T, cfg.hidden)).astype(np.float32)
+        self.dy = (1e-3 * rng.standard_normal((T, cfg.hidden))).astype(np.float32)
         n = sum(p.size for p in params[0]) // self.ADAM_FRACTION
-        self.adam = [rng.standard_normal(n) * 0.02, rng.standard_normal(n) * 1e-3, np.zeros(n), np.zeros(n)]
+        self.adam = [(rng.standard_normal(n) * 0.02).astype(np.float32),
+                     (rng.standard_normal(n) * 1e-3).astype(np.float32), np.zeros(n, np.float32),
+                     np.zeros(n, np.float32)]
 
     def run(self) -> dict:
-        cfg, O = self.cfg, self.O
-        srv = O.OracleServer(self.one, self.params)
+        cfg, O32 = self.cfg, self.O32
         t0 = time.perf_counter()
-        srv.forward(self.states, *self.glm)
-        srv.backward(self.grads)
+        O32.server_fwd_bwd(self.one, self.params, self.grads, self.cu, self.x, self.dy)
         t1 = time.perf_counter()
         w, g, m, v = self.adam
-        O.adamw_update(w, g, m, v, 1, cfg.lr, cfg.adam_beta1, cfg.adam_beta2, cfg.adam_eps, cfg.weight_decay)
+        O32.adamw(w, g, m, v, 1, cfg.lr, cfg.adam_beta1, cfg.adam_beta2, cfg.adam_eps, cfg.weight_decay)
         t2 = time.perf_counter()
         sample_tokens = self.nseg * self.L
         t_step = cfg.n_blocks * ((t1 - t0) * cfg.tokens / sample_tokens + (t2 - t1) * self.ADAM_FRACTION)
         return {"t_fwd_bwd_s": t1 - t0, "t_adamw_s": t2 - t1, "sample_tokens": sample_tokens,
                 "t_sample_s": t2 - t0, "t_step_s": t_step, "tokens_per_s": cfg.tokens / t_step,
-                "dtype": "f64", "cores": cpu_cores(),
+                "dtype": "f32", "cores": O32.threads(),
                 "rule": (f"full step = n_blocks x (t_fwd_bwd x {cfg.tokens}/{sample_tokens} + t_adamw x "
                          f"{self.ADAM_FRACTION})"),
                 "sample": (f"1 of {cfg.n_blocks} blocks at the workload's shapes, {self.nseg} segment(s) x {self.L} "
                            f"tokens fwd+bwd, plus AdamW over 1/{self.ADAM_FRACTION} of that block's parameters; "
-                           f"fp64 numpy; full step estimated as n_blocks x (t_fwd_bwd x {cfg.tokens}/"
-                           f"{sample_tokens} + t_adamw x {self.ADAM_FRACTION})")}
+                           f"fp32 C++ oracle (plain loops, OpenMP on {O32.threads()} threads, no BLAS); full step "
+                           f"estimated as n_blocks x (t_fwd_bwd x {cfg.tokens}/{sample_tokens} + t_adamw x "
+                           f"{self.ADAM_FRACTION})")}
 
 
 def cpu_cores() -> int:
@@ -278,7 +279,7 @@ def main():
     ap.add_argument("--no-other-configs", action="store_true",
                     help="skip the ragged workload and the packed-vs-sequential points after the main line")
     ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the oracle sample")
-    ap.add_argument("--ref-tokens", type=int, default=256, help="tokens of the reference-arm sample")
+    ap.add_argument("--ref-tokens", type=int, default=128, help="tokens of the reference-arm sample")
     ap.add_argument("--sweep", action="store_true",
                     help="client-batching sweep: 26 blocks, 2 x 512 tokens per client, K in 1..32, "
                          "one packed call vs K sequential single-client calls (one JSON line per K)")
@@ -329,7 +330,6 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         sample = OracleSample(cfg, min(cfg.tokens, args.cpu_tokens))
-        sample.run()
         cpu = sample.run()
         del sample
 

@@ -303,3 +303,43 @@ def test_tiny_parity_weight_decay(F, fused):
     """Decoupled weight decay lambda = 0.01 (the paper trains with none; the AdamW of the
     library takes it as a parameter): the step, and the step fused into the backward."""
     parity_case(F, syn.CONFIGS["tiny"].with_(weight_decay=0.01), fused=fused)
+
+
+def fp32_oracle_case(F, cfg):
+    """GPU forward + backward against the fp32 C++ oracle (single precision throughout, the
+    precision the tolerances were written for), the same seeded weights and inputs."""
+    from oracle import oracle32 as O32
+    params = syn.init_params(cfg)
+    srv = make_server(F, cfg)
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            srv.set_param(b, t, params[b][t])
+    states = syn.client_states(cfg)
+    grads = syn.client_grads(cfg)
+    outs, gins = run_gpu(F, srv, cfg, states, grads)
+    H = cfg.hidden
+    x = np.concatenate([syn.bf16_bits_to_f64(s).reshape(-1, H) for s in states])
+    dy = np.concatenate([syn.bf16_bits_to_f64(g).reshape(-1, H) for g in grads])
+    cu = np.concatenate([[0], np.cumsum([L for L in cfg.seq_lens for _ in range(cfg.client_batch)])])
+    g32 = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+    y, dx = O32.server_fwd_bwd(cfg, params, g32, cu, x, dy)
+    y_gpu = np.concatenate([f64(o).reshape(-1, H) for o in outs])
+    dx_gpu = np.concatenate([f64(g).reshape(-1, H) for g in gins])
+    assert rel_inf(y_gpu, y) < OUT_TOL, rel_inf(y_gpu, y)
+    assert rel_inf(dx_gpu, dx) < GRAD_TOL, rel_inf(dx_gpu, dx)
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            e = rel_inf(srv.get_grad(b, t), g32[b][t].reshape(-1))
+            assert e < GRAD_TOL, ("wgrad", b, syn.TENSOR_NAMES[t], e)
+    srv.close()
+
+
+def test_tiny_parity_vs_fp32_oracle(F):
+    """The one-block H=256 workload (K=2 x 2 rows x 64 tokens) against the fp32 oracle."""
+    fp32_oracle_case(F, syn.CONFIGS["tiny"])
+
+
+def test_block6b_segment_parity_vs_fp32_oracle(F):
+    """One ChatGLM-6B-shaped block (H=4096, 32 x 128, F=16384) on one 512-token client of
+    the one-block workload, against the fp32 oracle."""
+    fp32_oracle_case(F, syn.CONFIGS["block6b"].with_(seq_lens=(512,)))

@@ -1,0 +1,141 @@
+"""The fp32 C++ oracle (oracle/flglm_oracle32.cpp) against what fixes it independently of
+itself: the pinned fp64 oracle (an independent implementation of the same definitions),
+the zero-weight closed form, the batching invariant of §3.3, causality and segment
+isolation, and the first-step closed form of AdamW (CPU only)."""
+import numpy as np
+import pytest
+
+import synthetic as syn
+from oracle import flglm_oracle as O
+from oracle import oracle32 as O32
+
+
+def _rel(a, b):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.abs(a - b).max() / max(np.abs(b).max(), 1e-30))
+
+
+def _inputs(cfg):
+    states = syn.client_states(cfg)
+    grads = syn.client_grads(cfg)
+    x = np.concatenate([syn.bf16_bits_to_f64(s).reshape(-1, cfg.hidden) for s in states])
+    dy = np.concatenate([syn.bf16_bits_to_f64(g).reshape(-1, cfg.hidden) for g in grads])
+    cu = np.concatenate([[0], np.cumsum([L for L in cfg.seq_lens for _ in range(cfg.client_batch)])])
+    return states, grads, x, dy, cu
+
+
+def _run32(cfg, params, cu, x, dy):
+    g = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+    y, dx = O32.server_fwd_bwd(cfg, params, g, cu, x, dy)
+    return y, dx, g
+
+
+@pytest.mark.parametrize("rfl", [1, 0], ids=["glm_block", "pre_ln"])
+def test_matches_fp64_oracle(rfl):
+    """Two blocks over ragged segments (64, 37 and a 1-token one), both residual readings:
+    outputs, input gradients and every weight gradient within fp32 rounding of the fp64
+    oracle."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, client_batch=1, seq_lens=(64, 37, 1), residual_from_ln=rfl,
+                                    residual_alpha=2.0 if rfl else 1.0)
+    params = syn.init_params(cfg)
+    states, grads, x, dy, cu = _inputs(cfg)
+    ref = O.OracleServer(cfg, params)
+    ro = np.concatenate([r.reshape(-1, cfg.hidden) for r in ref.forward([syn.bf16_bits_to_f64(s) for s in states])])
+    rg = np.concatenate([r.reshape(-1, cfg.hidden) for r in ref.backward([syn.bf16_bits_to_f64(g) for g in grads])])
+    y, dx, g = _run32(cfg, params, cu, x, dy)
+    assert _rel(y, ro) < 1e-5
+    assert _rel(dx, rg) < 1e-5
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            assert _rel(g[b][t], ref.grads[b][t]) < 1e-5, (b, syn.TENSOR_NAMES[t])
+
+
+def test_matches_fp64_oracle_head_dim_128():
+    """One block with 128-dim heads (the ChatGLM-6B head size) at a small hidden size."""
+    cfg = syn.CONFIGS["tiny"].with_(hidden=256, n_heads=2, head_dim=128, ffn_hidden=1024, client_batch=2,
+                                    seq_lens=(40, 17))
+    params = syn.init_params(cfg)
+    states, grads, x, dy, cu = _inputs(cfg)
+    ref = O.OracleServer(cfg, params)
+    ro = np.concatenate([r.reshape(-1, cfg.hidden) for r in ref.forward([syn.bf16_bits_to_f64(s) for s in states])])
+    rg = np.concatenate([r.reshape(-1, cfg.hidden) for r in ref.backward([syn.bf16_bits_to_f64(g) for g in grads])])
+    y, dx, g = _run32(cfg, params, cu, x, dy)
+    assert _rel(y, ro) < 1e-5 and _rel(dx, rg) < 1e-5
+    assert max(_rel(g[0][t], ref.grads[0][t]) for t in range(12)) < 1e-5
+
+
+def test_zero_weights_closed_form():
+    """Wd = W1 = W2 = 0 and zero biases, gamma = 1, beta = 0: y = alpha LN(alpha LN(x))."""
+    cfg = syn.CONFIGS["tiny"].with_(client_batch=1, seq_lens=(9, 4))
+    params = syn.init_params(cfg)
+    for t in (syn.T_WD, syn.T_BD, syn.T_W1, syn.T_B1, syn.T_W2, syn.T_B2):
+        params[0][t][:] = 0
+    _, _, x, dy, cu = _inputs(cfg)
+    y, _, _ = _run32(cfg, params, cu, x, dy)
+
+    def ln(v):
+        v = v - v.mean(axis=1, keepdims=True)
+        return v / np.sqrt((v * v).mean(axis=1, keepdims=True) + cfg.ln_eps)
+    a = cfg.residual_alpha
+    assert _rel(y, a * ln(a * ln(x))) < 1e-5
+
+
+def test_batching_invariant_and_isolation():
+    """Packed segments equal each segment run alone bit for bit (row-independent loops,
+    sums in a fixed order); weight gradients equal the sum of the per-segment runs within
+    fp32 rounding; changing a later token or another segment leaves an output bit-identical."""
+    cfg = syn.CONFIGS["tiny"].with_(client_batch=1, seq_lens=(20, 11, 5))
+    params = syn.init_params(cfg)
+    _, _, x, dy, cu = _inputs(cfg)
+    y, dx, g = _run32(cfg, params, cu, x, dy)
+    gsum = [np.zeros(p.shape, np.float64) for p in params[0]]
+    for s in range(3):
+        a, b = cu[s], cu[s + 1]
+        ys, dxs, gs = _run32(cfg, params, [0, b - a], x[a:b], dy[a:b])
+        np.testing.assert_array_equal(ys, y[a:b])
+        np.testing.assert_array_equal(dxs, dx[a:b])
+        for t in range(12):
+            gsum[t] += gs[0][t]
+    for t in range(12):
+        assert _rel(g[0][t], gsum[t]) < 1e-5
+    x2 = x.copy()
+    rng = np.random.default_rng(5)   # not a constant shift, which LayerNorm removes exactly
+    x2[cu[1] - 1] += rng.standard_normal(cfg.hidden)          # last token of segment 0
+    x2[cu[2]:cu[3]] += rng.standard_normal((cu[3] - cu[2], cfg.hidden))  # all of segment 2
+    y2, _, _ = _run32(cfg, params, cu, x2, dy)
+    np.testing.assert_array_equal(y2[:cu[1] - 1], y[:cu[1] - 1])
+    np.testing.assert_array_equal(y2[cu[1]:cu[2]], y[cu[1]:cu[2]])
+    assert not np.array_equal(y2[cu[1] - 1], y[cu[1] - 1])
+
+
+def test_adamw_first_step_and_fp64():
+    """First step (zero moments, no decay): w1 = w0 - lr g / (|g| + eps) within fp32
+    rounding; five steps against the fp64 AdamW."""
+    rng = np.random.default_rng(3)
+    n = 1000
+    w0 = rng.standard_normal(n).astype(np.float32)
+    g = (1e-3 * rng.standard_normal(n)).astype(np.float32)
+    w, m, v = w0.copy(), np.zeros(n, np.float32), np.zeros(n, np.float32)
+    O32.adamw(w, g, m, v, 1, 1e-2, 0.9, 0.999, 1e-8, 0.0)
+    want = w0.astype(np.float64) - 1e-2 * g / (np.abs(g.astype(np.float64)) + 1e-8)
+    assert np.abs(w - want).max() < 1e-6
+    w64, m64, v64 = w0.astype(np.float64), np.zeros(n), np.zeros(n)
+    w, m, v = w0.copy(), np.zeros(n, np.float32), np.zeros(n, np.float32)
+    for t in range(1, 6):
+        gt = (1e-3 * rng.standard_normal(n)).astype(np.float32)
+        O32.adamw(w, gt, m, v, t, 1e-3, 0.9, 0.999, 1e-8, 0.01)
+        w64, m64, v64 = O.adamw_update(w64, gt.astype(np.float64), m64, v64, t, 1e-3, 0.9, 0.999, 1e-8, 0.01)
+    assert np.abs(w - w64).max() < 1e-6
+    assert _rel(m, m64) < 1e-5
+
+
+def test_bad_arguments():
+    cfg = syn.CONFIGS["tiny"].with_(client_batch=1, seq_lens=(4,))
+    params = syn.init_params(cfg)
+    x = np.zeros((4, cfg.hidden), np.float32)
+    with pytest.raises(ValueError):
+        _run32(cfg, params, [0, 3, 2, 4], x, x)
+    with pytest.raises(ValueError):
+        O32.adamw(np.zeros(2, np.float32), np.zeros(2, np.float32), np.zeros(2, np.float32),
+                  np.zeros(2, np.float32), 0, 1e-3, 0.9, 0.999, 1e-8, 0.0)
