@@ -83,29 +83,30 @@ struct AttnGlm {
   const int32_t* pos2 = nullptr;  // [T] block position (inverse rotary of dims [hd/2, hd))
 };
 
-// Attention on a device tile list (built by fl_launch_meta).
-// head_dim 128 runs on tcgen05 (attention_tc.cu), head_dim 64 on mma.sync; `status`
-// (device int or null) receives a code if a bounded wait inside the kernel gave up.
+// Attention on a device tile list (built by fl_launch_meta): the 64-row list (n_tiles
+// entries) followed by the 128-row one (n_tiles128) that the tcgen05 kernels walk.
+// head_dim 64 or 128; `status` (device int or null) receives a code if a bounded wait
+// inside a kernel gave up.
 int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
                        int n_tiles, int n_tiles128, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm,
                        cudaStream_t st, int* status = nullptr);
-int fl_launch_attn_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles,
-                          void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
+// tiles: the 128-row list alone (attention_tc.cu).
+int fl_launch_attn_fwd_tc(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
+                          int n_tiles, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
                           cudaStream_t st);
 // dbias (or null): += the column sums of dqkv [3H] (the QKV bias gradient), per CTA.
-// head_dim 128 computes dQ and dK / dV of the segments' own keys on tcgen05
-// (attention_bwd_tc.cu), whose bounded waits report into `status` (device int or null).
+// delta: fp32 [nh, T] scratch (rowsum(dO * O), written here).
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, int n_tiles128, float* delta,
                        const float* rope_tab,
                        void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
                        float* dbias = nullptr, int* status = nullptr);
-int fl_launch_attn_bwd_dq_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
-                             const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab, void* dqkv,
-                             const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st);
-int fl_launch_attn_bwd_dkv_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
-                              const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab,
-                              void* dqkv, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st);
+// dQ, dK / dV and, with a prefix, the prefix keys' gradients (attention_bwd_tc.cu); tiles:
+// the 128-row list alone; delta already computed.
+int fl_launch_attn_bwd_tc(int T, int nh, int hd, const void* qkv, const void* dout, const float* lse,
+                          const float* delta, const int32_t* cu, const uint32_t* tiles, int n_tiles,
+                          const float* rope_tab, void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, float* dbias,
+                          int* status, cudaStream_t st);
 
 // LayerNorm backward on fp32 dy / x (rowops.cu): fl_k_layernorm_bwd, and, when dcol is not
 // null, dcol += the column sums of dx.  workspace: fl_launch_layernorm_bwd_workspace bytes.
