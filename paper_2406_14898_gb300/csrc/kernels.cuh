@@ -114,7 +114,11 @@ size_t fl_launch_layernorm_bwd_workspace(int T, int H);
 int fl_launch_layernorm_bwd_f32(int T, int H, const float* dy, const float* x, const float* mean, const float* rstd,
                                 const float* gamma, const float* resid, float resid_alpha, __nv_bfloat16* dx_bf16,
                                 float* dx_f32, float* dgamma, float* dbeta, float* dcol, float* workspace,
-                                cudaStream_t st);
+                                cudaStream_t st, int* status = nullptr);
+// LayerNorm forward of fp32 rows (fl_k_layernorm_fwd); x 16-byte aligned; `status` (device int
+// or null) receives a code if a bounded wait gave up.
+int fl_launch_layernorm_fwd_f32(int T, int H, const float* x, const float* gamma, const float* beta, float eps,
+                                __nv_bfloat16* y, float* mean, float* rstd, cudaStream_t st, int* status = nullptr);
 
 // Host helper: builds the tile list of a packing, tiles of `rows` query rows (64 for the
 // mma.sync kernels, 128 for the tcgen05 ones), segments' last tiles first (returns the

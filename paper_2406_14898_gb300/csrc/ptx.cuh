@@ -57,6 +57,15 @@ FL_DEV void tma_load_2d(void* dst, const CUtensorMap* m, uint64_t* bar, int x, i
       : "memory");
 }
 
+// Untiled bulk copy of `bytes` from global to this CTA's shared memory; completes tx bytes
+// on `bar`.  Both addresses 16-byte aligned, bytes a multiple of 16.
+FL_DEV void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
 // ------------------------------------------------------------------ tcgen05
 FL_DEV void tmem_alloc(uint32_t* dst, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)),

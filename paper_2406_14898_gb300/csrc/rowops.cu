@@ -7,6 +7,7 @@
 #include "../../include/flglm_kernels.h"
 #include "common.cuh"
 #include "kernels.cuh"
+#include "ptx.cuh"
 
 namespace {
 
@@ -75,87 +76,172 @@ FL_DEV float2 block_sum2(float a, float b, float2 (*red)[32], int par) {
   return r;
 }
 
-// Forward: a CTA of max(32, H/32) threads takes one row, each thread CH chunks of 8
-// elements (chunk c + k * blockDim.x) held in registers; with small CTAs an SM keeps 7
-// rows (for H = 4096, 112 KB of fp32 loads) in flight.  (One 512-thread CTA per row with
-// the next row prefetched kept only one row per CTA in flight: 4.0 against 5.2 TB/s.)
+// Forward: persistent CTAs of max(32, H/16) threads, each thread CH chunks of 8 elements
+// (chunk c + k * blockDim.x) of every row.  The CTA walks rows blockIdx.x, + gridDim.x, ...
+// and keeps the next LN_STAGES of them in flight: one elected thread copies each whole row
+// into a shared-memory stage with one bulk copy (cp.async.bulk, completion on the stage's
+// mbarrier) and refills the stage as soon as every thread has read it.  Three CTAs per SM
+// at H = 4096 (fp32 rows: 4 x 16 KB of stages each) keep 12 rows in flight per SM.  The
+// statistics are two block reductions (mean, then the centred variance).  Every wait is
+// bounded: on expiry the CTA records a status code and stops.
+constexpr int LN_STAGES = 4;
+
 template <typename TX, int CH>
-__global__ void __launch_bounds__(128) ln_fwd_row_kernel(int H, const TX* __restrict__ x,
-                                                         const float* __restrict__ gamma,
-                                                         const float* __restrict__ beta, float eps,
-                                                         __nv_bfloat16* __restrict__ y, float* __restrict__ mean,
-                                                         float* __restrict__ rstd) {
-  __shared__ float red[2][4];
-  const int row = blockIdx.x, c = threadIdx.x, nt = blockDim.x;
+__global__ void __launch_bounds__(256) ln_fwd_bulk_kernel(int T, int H, const TX* __restrict__ x,
+                                                          const float* __restrict__ gamma,
+                                                          const float* __restrict__ beta, float eps,
+                                                          __nv_bfloat16* __restrict__ y, float* __restrict__ mean,
+                                                          float* __restrict__ rstd, int* status) {
+  extern __shared__ __align__(128) uint8_t ln_smem[];
+  const uint32_t row_bytes = (uint32_t)H * sizeof(TX);
+  uint64_t* full = reinterpret_cast<uint64_t*>(ln_smem + LN_STAGES * row_bytes);
+  __shared__ float red[2][8];
+  const int c = threadIdx.x, nt = blockDim.x;
   const int lane = c & 31, w = c >> 5, nw = nt >> 5;
-  const TX* xr = x + (int64_t)row * H;
-  float v[CH][8];
-#pragma unroll
-  for (int k = 0; k < CH; ++k) load8<TX>(xr, c + k * nt, v[k]);
-  float s = 0.f;
-#pragma unroll
-  for (int k = 0; k < CH; ++k)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) s += v[k][j];
-  s = warp_sum(s);
-  if (lane == 0) red[0][w] = s;
-  __syncthreads();
-  float tot = 0.f;
-  for (int i = 0; i < nw; ++i) tot += red[0][i];
-  const float mu = tot / H;
-  float q = 0.f;
-#pragma unroll
-  for (int k = 0; k < CH; ++k)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) q += (v[k][j] - mu) * (v[k][j] - mu);
-  q = warp_sum(q);
-  if (lane == 0) red[1][w] = q;
-  __syncthreads();
-  tot = 0.f;
-  for (int i = 0; i < nw; ++i) tot += red[1][i];
-  const float rs = rsqrtf(tot / H + eps);
-  __nv_bfloat16* yr = y + (int64_t)row * H;
+  if (c == 0) {
+    for (int i = 0; i < LN_STAGES; ++i) mbar_init(full + i, 1);
+    fence_mbar_init();
+    for (int i = 0; i < LN_STAGES; ++i) {
+      const int row = blockIdx.x + i * gridDim.x;
+      if (row < T) {
+        mbar_arrive_expect_tx(full + i, row_bytes);
+        bulk_load(ln_smem + i * row_bytes, x + (int64_t)row * H, row_bytes, full + i);
+      }
+    }
+  }
+  float gg[CH][8], bt[CH][8];
 #pragma unroll
   for (int k = 0; k < CH; ++k) {
-    float gg[8], bt[8], o[8];
-    load8<float>(gamma, c + k * nt, gg);
-    load8<float>(beta, c + k * nt, bt);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) o[j] = (v[k][j] - mu) * rs * gg[j] + bt[j];
-    reinterpret_cast<uint4*>(yr)[c + k * nt] = pack8(o);
+    load8<float>(gamma, c + k * nt, gg[k]);
+    load8<float>(beta, c + k * nt, bt[k]);
   }
-  if (c == 0) {
-    mean[row] = mu;
-    rstd[row] = rs;
+  __syncthreads();
+  for (int it = 0;; ++it) {
+    const int row = blockIdx.x + it * gridDim.x;
+    if (row >= T) break;
+    const int st = it % LN_STAGES;
+    if (!__syncthreads_and(mbar_wait(full + st, (it / LN_STAGES) & 1))) {
+      if (c == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+      break;
+    }
+    const TX* xr = reinterpret_cast<const TX*>(ln_smem + st * row_bytes);
+    float v[CH][8];
+#pragma unroll
+    for (int k = 0; k < CH; ++k) {
+      if constexpr (sizeof(TX) == 4) {
+        const float4 a = reinterpret_cast<const float4*>(xr)[2 * (c + k * nt)];
+        const float4 b = reinterpret_cast<const float4*>(xr)[2 * (c + k * nt) + 1];
+        v[k][0] = a.x; v[k][1] = a.y; v[k][2] = a.z; v[k][3] = a.w;
+        v[k][4] = b.x; v[k][5] = b.y; v[k][6] = b.z; v[k][7] = b.w;
+      } else {
+        unpack8(reinterpret_cast<const uint4*>(xr)[c + k * nt], v[k]);
+      }
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < CH; ++k)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) s += v[k][j];
+    s = warp_sum(s);
+    if (lane == 0) red[0][w] = s;
+    __syncthreads();  // also: every thread has read the stage
+    if (c == 0) {
+      const int nxt = row + LN_STAGES * gridDim.x;
+      if (nxt < T) {
+        fence_proxy_async_smem();
+        mbar_arrive_expect_tx(full + st, row_bytes);
+        bulk_load(ln_smem + st * row_bytes, x + (int64_t)nxt * H, row_bytes, full + st);
+      }
+    }
+    float tot = 0.f;
+    for (int i = 0; i < nw; ++i) tot += red[0][i];
+    const float mu = tot / H;
+    float q = 0.f;
+#pragma unroll
+    for (int k = 0; k < CH; ++k)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) q += (v[k][j] - mu) * (v[k][j] - mu);
+    q = warp_sum(q);
+    if (lane == 0) red[1][w] = q;
+    __syncthreads();
+    tot = 0.f;
+    for (int i = 0; i < nw; ++i) tot += red[1][i];
+    const float rs = rsqrtf(tot / H + eps);
+    __nv_bfloat16* yr = y + (int64_t)row * H;
+#pragma unroll
+    for (int k = 0; k < CH; ++k) {
+      float o[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) o[j] = (v[k][j] - mu) * rs * gg[k][j] + bt[k][j];
+      reinterpret_cast<uint4*>(yr)[c + k * nt] = pack8(o);
+    }
+    if (c == 0) {
+      mean[row] = mu;
+      rstd[row] = rs;
+    }
   }
 }
 
 // Backward: dx = rstd (g - mean(g) - xhat mean(g xhat)), g = gamma dy (+ alpha resid);
-// thread c keeps its columns' dgamma / dbeta partials (and with CS the column sums of dx,
-// the bias gradient of the GEMM whose output gradient dx is) in registers across the
-// CTA's rows and writes them to workspace[blockIdx.x][2 + CS][H]; ln_bwd_reduce_kernel
-// adds them up.  Kept at <= 64 registers (gamma re-read from L1 each row, no register
-// prefetch of the next row) so that two 512-thread CTAs share an SM and cover each
-// other's latency.
+// persistent CTAs of H/8 threads walk rows blockIdx.x, + gridDim.x, ...; one elected thread
+// bulk-copies each row's dy and x into a shared-memory stage (LNB_STAGES in flight, refilled
+// once every thread has read it).  Thread c keeps its 8 columns' dgamma / dbeta partials (and
+// with CS the column sums of dx, the bias gradient of the GEMM whose output gradient dx is)
+// in registers across the CTA's rows and writes them to workspace[blockIdx.x][2 + CS][H];
+// ln_bwd_reduce_kernel adds them up.  At <= 64 registers two 512-thread CTAs (3 x 32 KB of
+// stages each at H = 4096, fp32) share an SM: six rows in flight.  Every wait is bounded.
+constexpr int LNB_STAGES = 3;
+
 template <typename T, bool CS>
 __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* __restrict__ dy,
                                                         const T* __restrict__ x, const float* __restrict__ mean,
                                                         const float* __restrict__ rstd,
                                                         const float* __restrict__ gamma, const T* __restrict__ resid,
                                                         float resid_alpha, __nv_bfloat16* __restrict__ dx_bf16,
-                                                        float* __restrict__ dx_f32, float* __restrict__ ws) {
+                                                        float* __restrict__ dx_f32, float* __restrict__ ws,
+                                                        int* status) {
+  extern __shared__ __align__(128) uint8_t lnb_smem[];
+  const uint32_t row_bytes = (uint32_t)H * sizeof(T);
+  uint64_t* full = reinterpret_cast<uint64_t*>(lnb_smem + 2 * LNB_STAGES * row_bytes);
   __shared__ float2 red[2][32];
   const int c = threadIdx.x;
+  auto issue = [&](int st, int row) {  // one elected thread: dy and x of `row` into stage st
+    mbar_arrive_expect_tx(full + st, 2 * row_bytes);
+    bulk_load(lnb_smem + (2 * st) * row_bytes, dy + (int64_t)row * H, row_bytes, full + st);
+    bulk_load(lnb_smem + (2 * st + 1) * row_bytes, x + (int64_t)row * H, row_bytes, full + st);
+  };
+  if (c == 0) {
+    for (int i = 0; i < LNB_STAGES; ++i) mbar_init(full + i, 1);
+    fence_mbar_init();
+    for (int i = 0; i < LNB_STAGES; ++i)
+      if (blockIdx.x + i * gridDim.x < Tn) issue(i, blockIdx.x + i * gridDim.x);
+  }
   float accg[8], accb[8], accd[CS ? 8 : 1];
 #pragma unroll
   for (int k = 0; k < 8; ++k) accg[k] = accb[k] = 0.f;
 #pragma unroll
   for (int k = 0; k < (CS ? 8 : 1); ++k) accd[k] = 0.f;
+  __syncthreads();
   int par = 0;
-  for (int row = blockIdx.x; row < Tn; row += gridDim.x) {
+  for (int it = 0;; ++it) {
+    const int row = blockIdx.x + it * gridDim.x;
+    if (row >= Tn) break;
+    const int st = it % LNB_STAGES;
+    if (!__syncthreads_and(mbar_wait(full + st, (it / LNB_STAGES) & 1))) {
+      if (c == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+      break;
+    }
     float d[8], xh[8], gcol[8];
-    load8<T>(dy + (int64_t)row * H, c, d);
-    load8<T>(x + (int64_t)row * H, c, xh);
+    if constexpr (sizeof(T) == 4) {
+      const float4* sd = reinterpret_cast<const float4*>(lnb_smem + (2 * st) * row_bytes) + 2 * c;
+      const float4* sx = reinterpret_cast<const float4*>(lnb_smem + (2 * st + 1) * row_bytes) + 2 * c;
+      const float4 d0 = sd[0], d1 = sd[1], x0 = sx[0], x1 = sx[1];
+      d[0] = d0.x; d[1] = d0.y; d[2] = d0.z; d[3] = d0.w; d[4] = d1.x; d[5] = d1.y; d[6] = d1.z; d[7] = d1.w;
+      xh[0] = x0.x; xh[1] = x0.y; xh[2] = x0.z; xh[3] = x0.w; xh[4] = x1.x; xh[5] = x1.y; xh[6] = x1.z; xh[7] = x1.w;
+    } else {
+      unpack8(reinterpret_cast<const uint4*>(lnb_smem + (2 * st) * row_bytes)[c], d);
+      unpack8(reinterpret_cast<const uint4*>(lnb_smem + (2 * st + 1) * row_bytes)[c], xh);
+    }
     load8<float>(gamma, c, gcol);
     const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
     float s1 = 0.f, s2 = 0.f;
@@ -168,8 +254,15 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
       accg[k] += d[k] * xh[k];
       accb[k] += d[k];
     }
-    const float2 sums = block_sum2(s1, s2, red, par);
+    const float2 sums = block_sum2(s1, s2, red, par);  // its barrier: every thread has read the stage
     par ^= 1;
+    if (c == 0) {
+      const int nxt = row + LNB_STAGES * gridDim.x;
+      if (nxt < Tn) {
+        fence_proxy_async_smem();
+        issue(st, nxt);
+      }
+    }
     const float mg = sums.x / H, mgx = sums.y / H;
     float o[8];
 #pragma unroll
@@ -222,13 +315,23 @@ __global__ void ln_bwd_reduce_kernel(int nblk, int H, int nv, const float* __res
 template <typename T>
 int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, const float* mean, const float* rstd,
                     const float* gamma, const void* resid, float alpha, void* dx_bf16, float* dx_f32, float* ws,
-                    float* dgamma, float* dbeta, float* dcol, cudaStream_t st) {
+                    float* dgamma, float* dbeta, float* dcol, cudaStream_t st, int* status = nullptr) {
+  const int smem = 2 * LNB_STAGES * H * (int)sizeof(T) + LNB_STAGES * 8;
+  static bool attr = false;
+  if (!attr) {
+    const int mx = 2 * LNB_STAGES * 4096 * (int)sizeof(T) + LNB_STAGES * 8;
+    FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx));
+    FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx));
+    attr = true;
+  }
   if (dcol)
-    ln_bwd_kernel<T, true><<<nblk, H / 8, 0, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
-                                                   (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws);
+    ln_bwd_kernel<T, true><<<nblk, H / 8, smem, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
+                                                      (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws,
+                                                      status);
   else
-    ln_bwd_kernel<T, false><<<nblk, H / 8, 0, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
-                                                    (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws);
+    ln_bwd_kernel<T, false><<<nblk, H / 8, smem, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
+                                                       (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws,
+                                                       status);
   FL_CUDA_TRY(cudaGetLastError());
   const int split = nblk >= 64 ? 16 : 1;
   const int nv = dcol ? 3 : 2;
@@ -239,16 +342,27 @@ int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, cons
 
 template <typename TX>
 int dispatch_ln_fwd(int Tn, int H, const void* x, const float* gamma, const float* beta, float eps, void* y,
-                    float* mean, float* rstd, cudaStream_t st) {
-  // one CTA per row: max(32, H/32) threads of CH = H / (8 * threads) chunks (H a power of
-  // two in [256, 4096]: 32 x 1, 32 x 2, then H/32 x 4)
-  const int threads = H / 32 > 32 ? H / 32 : 32;
+                    float* mean, float* rstd, cudaStream_t st, int* status = nullptr) {
+  // max(32, H/16) threads of CH = H / (8 * threads) chunks (H a multiple of 256 up to 4096)
+  const int threads = H / 16 > 32 ? H / 16 : 32;
   const int ch = H / (8 * threads);
+  const int smem = LN_STAGES * H * (int)sizeof(TX) + LN_STAGES * 8;
+  static bool attr = false;
+  if (!attr) {
+    FL_CUDA_TRY(cudaFuncSetAttribute(ln_fwd_bulk_kernel<TX, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
+    FL_CUDA_TRY(cudaFuncSetAttribute(ln_fwd_bulk_kernel<TX, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
+    attr = true;
+  }
+  int grid = 3 * sm_count();
+  if (grid > Tn) grid = Tn;
   const TX* xx = (const TX*)x;
   __nv_bfloat16* yy = (__nv_bfloat16*)y;
-  if (ch == 4) ln_fwd_row_kernel<TX, 4><<<Tn, threads, 0, st>>>(H, xx, gamma, beta, eps, yy, mean, rstd);
-  else if (ch == 2) ln_fwd_row_kernel<TX, 2><<<Tn, threads, 0, st>>>(H, xx, gamma, beta, eps, yy, mean, rstd);
-  else ln_fwd_row_kernel<TX, 1><<<Tn, threads, 0, st>>>(H, xx, gamma, beta, eps, yy, mean, rstd);
+  if (ch == 2)
+    ln_fwd_bulk_kernel<TX, 2><<<grid, threads, smem, st>>>(Tn, H, xx, gamma, beta, eps, yy, mean, rstd, status);
+  else
+    ln_fwd_bulk_kernel<TX, 1><<<grid, threads, smem, st>>>(Tn, H, xx, gamma, beta, eps, yy, mean, rstd, status);
   FL_CUDA_TRY(cudaGetLastError());
   return FL_OK;
 }
@@ -466,6 +580,7 @@ extern "C" int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x
   if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d", H);
   if (!x || !gamma || !beta || !y || !mean || !rstd) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: null");
   if (x_dtype != FL_DT_BF16 && x_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: dtype");
+  if (reinterpret_cast<uintptr_t>(x) & 15) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: x not 16-byte aligned");
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
   return x_dtype == FL_DT_F32 ? dispatch_ln_fwd<float>(T, H, x, gamma, beta, eps, y, mean, rstd, st)
@@ -484,6 +599,8 @@ extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const vo
   if (!dy || !x || !mean || !rstd || !gamma || (!dx_bf16 && !dx_f32) || !dgamma || !dbeta || !workspace)
     return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: null");
   if (io_dtype != FL_DT_BF16 && io_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: dtype");
+  if ((reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(x)) & 15)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: dy / x not 16-byte aligned");
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
   const int nblk = ln_bwd_blocks(T);
@@ -504,10 +621,16 @@ size_t fl_launch_layernorm_bwd_workspace(int T, int H) {
 int fl_launch_layernorm_bwd_f32(int T, int H, const float* dy, const float* x, const float* mean, const float* rstd,
                                 const float* gamma, const float* resid, float resid_alpha, __nv_bfloat16* dx_bf16,
                                 float* dx_f32, float* dgamma, float* dbeta, float* dcol, float* workspace,
-                                cudaStream_t st) {
+                                cudaStream_t st, int* status) {
   if (T == 0) return FL_OK;
   return dispatch_ln_bwd<float>(ln_bwd_blocks(T), T, H, dy, x, mean, rstd, gamma, resid, resid_alpha, dx_bf16, dx_f32,
-                                workspace, dgamma, dbeta, dcol, st);
+                                workspace, dgamma, dbeta, dcol, st, status);
+}
+
+int fl_launch_layernorm_fwd_f32(int T, int H, const float* x, const float* gamma, const float* beta, float eps,
+                                __nv_bfloat16* y, float* mean, float* rstd, cudaStream_t st, int* status) {
+  if (T == 0) return FL_OK;
+  return dispatch_ln_fwd<float>(T, H, x, gamma, beta, eps, y, mean, rstd, st, status);
 }
 
 extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream) {
@@ -692,6 +815,8 @@ extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, 
                              FL_LN_NOALLOC_MAX_H);
   if (!dy || !x || !mean || !rstd || !gamma || !dx || !dgamma || !dbeta)
     return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): null pointer");
+  if ((reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(x)) & 15)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): dy / x not 16-byte aligned");
   float* ws = nullptr;
   if (int rc = ln_scratch_address(&ws)) return rc;
   if (T == 0) return FL_OK;

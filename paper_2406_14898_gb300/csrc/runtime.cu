@@ -338,8 +338,8 @@ int block_forward(fl_server* h, int b, bool output = true) {
   cudaStream_t st = h->stream;
   // a = LN1(x)
   prof_begin(h, FL_PROF_LN);
-  TRY(h, fl_k_layernorm_fwd(T, H, x, FL_DT_F32, h->wt(b, FL_T_LN1_G), h->wt(b, FL_T_LN1_B), c.ln_eps, A.a, A.mean1,
-                            A.rstd1, st));
+  TRY(h, fl_launch_layernorm_fwd_f32(T, H, x, h->wt(b, FL_T_LN1_G), h->wt(b, FL_T_LN1_B), c.ln_eps,
+                                     (__nv_bfloat16*)A.a, A.mean1, A.rstd1, st, h->status));
   prof_end(h);
   // qkv = a Wqkv^T + bqkv, q and k rotated
   fl_gemm_args g1 = gemm_fwd(T, 3 * H, H, A.a, h->wbt(b, FL_T_WQKV), A.qkv, FL_EPI_BIAS_ROPE);
@@ -373,8 +373,8 @@ int block_forward(fl_server* h, int b, bool output = true) {
   TRY(h, run_gemm(h, g2));
   // m = LN2(h)
   prof_begin(h, FL_PROF_LN);
-  TRY(h, fl_k_layernorm_fwd(T, H, A.h, FL_DT_F32, h->wt(b, FL_T_LN2_G), h->wt(b, FL_T_LN2_B), c.ln_eps, A.m,
-                            A.mean2, A.rstd2, st));
+  TRY(h, fl_launch_layernorm_fwd_f32(T, H, A.h, h->wt(b, FL_T_LN2_G), h->wt(b, FL_T_LN2_B), c.ln_eps,
+                                     (__nv_bfloat16*)A.m, A.mean2, A.rstd2, st, h->status));
   prof_end(h);
   // u = m W1^T + b1, g = gelu(u)
   fl_gemm_args g3 = gemm_fwd(T, F, H, A.m, h->wbt(b, FL_T_WUP), A.g, FL_EPI_BIAS_GELU);
@@ -444,7 +444,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   prof_begin(h, FL_PROF_LN, 2);
   TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->dm, A.h, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dyf, al,
                                      h->dh, h->dhf, h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B),
-                                     train_base ? h->gt(b, FL_T_BDENSE) : nullptr, h->ln_ws, st));
+                                     train_base ? h->gt(b, FL_T_BDENSE) : nullptr, h->ln_ws, st, h->status));
   prof_end(h);
   // dense: do = dh Wd; dWd += dh^T o
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
@@ -474,7 +474,8 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   prof_begin(h, FL_PROF_LN, 2);
   TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->da, h->xs[b], A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G),
                                      glm ? nullptr : h->dhf, al, dx, dxf, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B),
-                                     train_base && b > 0 ? h->gt(b - 1, FL_T_BDOWN) : nullptr, h->ln_ws, st));
+                                     train_base && b > 0 ? h->gt(b - 1, FL_T_BDOWN) : nullptr, h->ln_ws, st,
+                                     h->status));
   prof_end(h);
   return FL_OK;
 }
