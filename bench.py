@@ -376,10 +376,10 @@ def main():
         step()
     srv.sync()
 
-    # ---- device-resident timed region
+    # ---- device-resident timed region (no per-launch events: consecutive kernels overlap
+    # their launch with the previous kernel's tail)
     clocks = ClockSampler(pci_bus_id(torch, dev))
     clocks.start()
-    srv.profile(True)
     l0 = srv.launch_count()
     barrier()
     torch.cuda.synchronize()
@@ -394,13 +394,24 @@ def main():
     barrier()
     ms = e0.elapsed_time(e1)
     launches = srv.launch_count() - l0
-    prof = srv.profile_read()
-    srv.profile(False)
     clk = clocks.stop()
     ms = max_over_ranks(ms)
     ms_step = ms / args.steps
     value = job_tokens_per_s(world, cfg.tokens, args.steps, ms)
 
+    # ---- the same steps again with CUDA events around every launch on the library's
+    # stream: per-class kernel time and the GEMM's live throughput (the roofline line)
+    srv.profile(True)
+    barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    srv.sync()
+    prof_ms_step = max_over_ranks(e0.elapsed_time(e1)) / args.steps
+    prof = srv.profile_read()
+    srv.profile(False)
     adam_ms = prof["adamw"][0] / args.steps
 
     # forward + backward alone (no optimizer), the metric's "fwd+bwd" in the narrow sense
@@ -487,6 +498,8 @@ def main():
             "fwd_bwd_basis": "separate timed loop of fl_server_forward + fl_server_backward, no optimizer step",
             "vector_adamw_ms": adam_ms,
             "kernel_ms_per_step": {k: v[0] / args.steps for k, v in prof.items()},
+            "kernel_ms_basis": (f"a second timed region of the same {args.steps} steps with CUDA events around every "
+                                f"launch ({prof_ms_step:.2f} ms per step there)"),
             "roofline": {"kernel": "gemm_pair_kernel (tcgen05.mma.cta_group::2, 256 x 256 tiles on SM pairs)", "bound": "tensor", "achieved": achieved,
                          "peak": pk["bf16_sustained"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_sustained"],
                          "peak_basis": f"{pk['source']} sustained bf16 (kernel timed inside a long step)",
@@ -494,7 +507,8 @@ def main():
                          "traffic_basis": (f"{traffic['launch']}, one ncu capture ({traffic['source']}); achieved is "
                                            f"the mean over all GEMM launches of the step") if traffic else None,
                          "launches_per_step": gemm_n / args.steps,
-                         "share_of_step": gemm_ms / ms},
+                         "share_of_step": gemm_ms / (prof_ms_step * args.steps),
+                         "timed_region": "the profiled repeat of the timed steps (kernel_ms_basis)"},
             "gpu_launches": launches,
             "clocks": clk,
             "hbm_used_gb": (total_b - free_b) / 1e9,
@@ -603,8 +617,9 @@ def dev_bf16(torch, bits_list, dev):
 def run_other_configs(steps: int, warmup: int, dev, stream) -> dict:
     """The workload's sibling configurations, a few steps each, on fresh servers after the
     main measurement: the ragged client-batching workload (26 blocks, K=16 clients x 1 row,
-    lengths U[64,1024] drawn with seed 7) and client-batching points of the sweep (26
-    blocks, K clients x 2 x 512 tokens): one packed call against K single-client calls."""
+    lengths U[64,1024] drawn with seed 7) and the client-batching sweep (26 blocks, K in
+    1..32 clients x 2 x 512 tokens, one server sized for K=32): one packed call against K
+    single-client calls."""
     import torch
     from paper_2406_14898_gb300 import flglm as F
     pk = peaks()
@@ -647,7 +662,7 @@ def run_other_configs(steps: int, warmup: int, dev, stream) -> dict:
     return out
 
 
-OTHER_SWEEP_KS = (2, 8)
+OTHER_SWEEP_KS = syn.SWEEP_KS
 
 
 def run_strategies(args, K: int):

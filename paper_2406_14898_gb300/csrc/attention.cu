@@ -30,6 +30,8 @@ constexpr int BT = 64;  // rows of the 64-row tile list (the first part of a til
 template <int HD>
 __global__ void __launch_bounds__(256) attn_delta_kernel(int T, int H, int nh, const bf16* __restrict__ O,
                                                          const bf16* __restrict__ dO, float* __restrict__ delta) {
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   constexpr int G = HD / 8;
   const int64_t gid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t p = gid / G;
@@ -92,12 +94,11 @@ int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, co
   const int64_t pairs = (int64_t)T * nh;
   const int H = nh * hd;
   if (hd == 128)
-    attn_delta_kernel<128><<<(unsigned)((pairs * 16 + 255) / 256), 256, 0, st>>>(T, H, nh, (const bf16*)o,
-                                                                                (const bf16*)dout, delta);
+    FL_CUDA_TRY(fl_launch(attn_delta_kernel<128>, dim3((unsigned)((pairs * 16 + 255) / 256)), dim3(256), 0, st, T, H,
+                          nh, (const bf16*)o, (const bf16*)dout, delta));
   else
-    attn_delta_kernel<64><<<(unsigned)((pairs * 8 + 255) / 256), 256, 0, st>>>(T, H, nh, (const bf16*)o,
-                                                                              (const bf16*)dout, delta);
-  FL_CUDA_TRY(cudaGetLastError());
+    FL_CUDA_TRY(fl_launch(attn_delta_kernel<64>, dim3((unsigned)((pairs * 8 + 255) / 256)), dim3(256), 0, st, T, H,
+                          nh, (const bf16*)o, (const bf16*)dout, delta));
   return fl_launch_attn_bwd_tc(T, nh, hd, qkv, dout, lse, delta, cu, tiles + n_tiles, n_tiles128, rope_tab, dqkv, pre,
                                glm, dbias, status, st);
 }

@@ -149,6 +149,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     bf16* __restrict__ dqkv, float* __restrict__ dpk, float* __restrict__ dpv, const int32_t* __restrict__ ctxs,
     const int32_t* __restrict__ gpos, const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int* status) {
   constexpr int NB = BwdCfg<HD>::NB, TILE = BwdCfg<HD>::TILE, CH = BwdCfg<HD>::CH, E = BwdCfg<HD>::E;
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sK = smem;
@@ -437,6 +439,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     bf16* __restrict__ dqkv, const int32_t* __restrict__ ctxs, const int32_t* __restrict__ gpos,
     const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int* status) {
   constexpr int NB = BwdCfg<HD>::NB, TILE = BwdCfg<HD>::TILE, CH = BwdCfg<HD>::CH, E = BwdCfg<HD>::E;
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
@@ -668,23 +672,20 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
   }
   const float scale = 1.f / sqrtf((float)HD);
   const float2* tab = reinterpret_cast<const float2*>(rope_tab);
-  attn_bwd_dq_tc_kernel<HD><<<dim3(n_tiles, nh), 256, BwdCfg<HD>::SMEM, st>>>(
-      tq, tdo, tpk, tpv, T, H, cu, tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv, glm.ctx,
-      glm.pos, glm.pos2, dbias, status);
-  FL_CUDA_TRY(cudaGetLastError());
-  attn_bwd_dkv_tc_kernel<HD, false><<<dim3(n_tiles, nh), 256, BwdCfg<HD>::SMEM, st>>>(
-      tq, tdo, tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, 0, (bf16*)dqkv, nullptr,
-      nullptr, glm.ctx, glm.pos, glm.pos2, dbias, status);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(attn_bwd_dq_tc_kernel<HD>, dim3(n_tiles, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo, tpk,
+                        tpv, T, H, cu, tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv, glm.ctx,
+                        glm.pos, glm.pos2, dbias, status));
+  FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, false>, dim3(n_tiles, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo,
+                        tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, 0, (bf16*)dqkv,
+                        (float*)nullptr, (float*)nullptr, glm.ctx, glm.pos, glm.pos2, dbias, status));
   if (pre.len > 0) {
     // the prefix keys of each head against slices of the query tiles, about one CTA per SM
     int nsplit = (sm_count_bwd() + nh - 1) / nh;
     if (nsplit > n_tiles) nsplit = n_tiles;
     if (nsplit < 1) nsplit = 1;
-    attn_bwd_dkv_tc_kernel<HD, true><<<dim3(nsplit, nh), 256, BwdCfg<HD>::SMEM, st>>>(
-        tq, tdo, tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv,
-        pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2, nullptr, status);
-    FL_CUDA_TRY(cudaGetLastError());
+    FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, true>, dim3(nsplit, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq,
+                          tdo, tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len,
+                          (bf16*)dqkv, pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2, (float*)nullptr, status));
   }
   return FL_OK;
 }

@@ -60,6 +60,8 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     const uint32_t* __restrict__ tiles, bf16* __restrict__ O, float* __restrict__ lse, float scale_log2, int Lp,
     const int32_t* __restrict__ ctxs, int* status) {
   constexpr int NB = FwdCfg<HD>::NB, TILE = FwdCfg<HD>::TILE;
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
@@ -275,9 +277,8 @@ int launch_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint3
     tpv = tq;
   }
   const float scale_log2 = (1.f / sqrtf((float)HD)) * LOG2E_T;
-  attn_fwd_tc_kernel<HD><<<dim3(n_tiles, nh), 128, FwdCfg<HD>::SMEM, st>>>(
-      tq, tpk, tpv, T, H, cu, tiles, (bf16*)o, lse, scale_log2, pre.len, glm.ctx, status);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(attn_fwd_tc_kernel<HD>, dim3(n_tiles, nh), dim3(128), FwdCfg<HD>::SMEM, st, tq, tpk, tpv, T, H,
+                        cu, tiles, (bf16*)o, lse, scale_log2, pre.len, glm.ctx, status));
   return FL_OK;
 }
 

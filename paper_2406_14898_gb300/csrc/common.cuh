@@ -30,6 +30,14 @@ FL_DEV uint64_t globaltimer_ns() {
   return t;
 }
 
+// Programmatic dependent launch.  A kernel launched with fl_launch (programmatic stream
+// serialization) may start while the previous kernel on the stream is still running; it
+// calls pdl_wait() before its first access to global memory (which returns once that
+// kernel has completed and its writes are visible) and then pdl_trigger(), which lets the
+// next kernel's CTAs be scheduled as SMs free up.  Without the attribute both are no-ops.
+FL_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+FL_DEV void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 FL_DEV void report_status(int* status, int code) {
   if (status) atomicCAS(status, 0, code);
 }
@@ -64,6 +72,23 @@ FL_DEV float gelu_tanh_grad(float u) {
   const float c = 0.7978845608028654f, a = 0.044715f;
   float t = tanh_hw(c * (u + a * u * u * u));
   return 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * c * (1.f + 3.f * a * u * u);
+}
+
+// Launches `kern` on `st` with programmatic stream serialization (see pdl_wait): the
+// kernel must call pdl_wait() before touching global memory.
+template <typename... KArgs, typename... Args>
+cudaError_t fl_launch(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
 #define FL_CUDA_TRY(expr)                                  \

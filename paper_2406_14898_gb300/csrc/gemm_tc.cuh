@@ -315,6 +315,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  pdl_wait();  // the previous kernel's outputs (operands, epilogue inputs) are complete
+  pdl_trigger();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -537,6 +539,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   cluster_sync();  // both CTAs' barriers initialised and TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  pdl_wait();  // the previous kernel's outputs (operands, epilogue inputs) are complete
+  pdl_trigger();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -774,9 +778,8 @@ int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) 
   const int tiles = num_m * num_n;
   const int grid = tiles < num_sms() ? tiles : num_sms();
   const Raster r = pick_raster(a->M, a->N, a->K, BM, BN);
-  gemm_tc_kernel<BN, A_MN, B_MN, FAM><<<grid, NUM_THREADS, C::SMEM_BYTES, st>>>(ta, tb, epi, a->M, a->N, a->K, r,
-                                                                                 status);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(gemm_tc_kernel<BN, A_MN, B_MN, FAM>, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, st, ta, tb,
+                        epi, a->M, a->N, a->K, r, status));
   return FL_OK;
 }
 
@@ -825,17 +828,19 @@ int launch_pair(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t
   const int pairs = tiles < slots ? tiles : slots;
   const Raster r = pick_raster(a->M, a->N, a->K, PAIR_BM, PAIR_BN);
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see pdl_wait
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(2 * pairs);
   cfg.blockDim = dim3(NUM_THREADS);
   cfg.dynamicSmemBytes = CfgPair::SMEM_BYTES;
   cfg.stream = st;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   FL_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, ta, tb, epi, a->M, a->N, a->K, r, status));
   return FL_OK;
 }

@@ -93,6 +93,8 @@ __global__ void __launch_bounds__(256) ln_fwd_bulk_kernel(int T, int H, const TX
                                                           __nv_bfloat16* __restrict__ y, float* __restrict__ mean,
                                                           float* __restrict__ rstd, int* status) {
   extern __shared__ __align__(128) uint8_t ln_smem[];
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   const uint32_t row_bytes = (uint32_t)H * sizeof(TX);
   uint64_t* full = reinterpret_cast<uint64_t*>(ln_smem + LN_STAGES * row_bytes);
   __shared__ float red[2][8];
@@ -201,6 +203,8 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
                                                         float* __restrict__ dx_f32, float* __restrict__ ws,
                                                         int* status) {
   extern __shared__ __align__(128) uint8_t lnb_smem[];
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   const uint32_t row_bytes = (uint32_t)H * sizeof(T);
   uint64_t* full = reinterpret_cast<uint64_t*>(lnb_smem + 2 * LNB_STAGES * row_bytes);
   __shared__ float2 red[2][32];
@@ -302,6 +306,8 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
 // blockIdx.y takes a slice of the rows.
 __global__ void ln_bwd_reduce_kernel(int nblk, int H, int nv, const float* __restrict__ ws, float* __restrict__ dgamma,
                                      float* __restrict__ dbeta, float* __restrict__ dcol) {
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= nv * H) return;
   const int per = (nblk + gridDim.y - 1) / gridDim.y;
@@ -325,18 +331,16 @@ int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, cons
     attr = true;
   }
   if (dcol)
-    ln_bwd_kernel<T, true><<<nblk, H / 8, smem, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
-                                                      (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws,
-                                                      status);
+    FL_CUDA_TRY(fl_launch(ln_bwd_kernel<T, true>, dim3(nblk), dim3(H / 8), smem, st, Tn, H, (const T*)dy, (const T*)x,
+                          mean, rstd, gamma, (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws, status));
   else
-    ln_bwd_kernel<T, false><<<nblk, H / 8, smem, st>>>(Tn, H, (const T*)dy, (const T*)x, mean, rstd, gamma,
-                                                       (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws,
-                                                       status);
-  FL_CUDA_TRY(cudaGetLastError());
+    FL_CUDA_TRY(fl_launch(ln_bwd_kernel<T, false>, dim3(nblk), dim3(H / 8), smem, st, Tn, H, (const T*)dy,
+                          (const T*)x, mean, rstd, gamma, (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws,
+                          status));
   const int split = nblk >= 64 ? 16 : 1;
   const int nv = dcol ? 3 : 2;
-  ln_bwd_reduce_kernel<<<dim3((nv * H + 255) / 256, split), 256, 0, st>>>(nblk, H, nv, ws, dgamma, dbeta, dcol);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(ln_bwd_reduce_kernel, dim3((nv * H + 255) / 256, split), dim3(256), 0, st, nblk, H, nv,
+                        (const float*)ws, dgamma, dbeta, dcol));
   return FL_OK;
 }
 
@@ -360,10 +364,11 @@ int dispatch_ln_fwd(int Tn, int H, const void* x, const float* gamma, const floa
   const TX* xx = (const TX*)x;
   __nv_bfloat16* yy = (__nv_bfloat16*)y;
   if (ch == 2)
-    ln_fwd_bulk_kernel<TX, 2><<<grid, threads, smem, st>>>(Tn, H, xx, gamma, beta, eps, yy, mean, rstd, status);
+    FL_CUDA_TRY(fl_launch(ln_fwd_bulk_kernel<TX, 2>, dim3(grid), dim3(threads), smem, st, Tn, H, xx, gamma, beta, eps,
+                          yy, mean, rstd, status));
   else
-    ln_fwd_bulk_kernel<TX, 1><<<grid, threads, smem, st>>>(Tn, H, xx, gamma, beta, eps, yy, mean, rstd, status);
-  FL_CUDA_TRY(cudaGetLastError());
+    FL_CUDA_TRY(fl_launch(ln_fwd_bulk_kernel<TX, 1>, dim3(grid), dim3(threads), smem, st, Tn, H, xx, gamma, beta, eps,
+                          yy, mean, rstd, status));
   return FL_OK;
 }
 
@@ -377,6 +382,8 @@ int ln_bwd_blocks(int T) {
 // Block: 32 column-threads (8 columns each = 256 columns) x 8 row groups.
 __global__ void __launch_bounds__(256) colsum_kernel(int T, int N, const __nv_bfloat16* __restrict__ x,
                                                      float* __restrict__ out, int rows_per_block) {
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   __shared__ float red[8][256];
   const int cx = threadIdx.x & 31;
   const int ry = threadIdx.x >> 5;
@@ -410,6 +417,8 @@ __global__ void __launch_bounds__(256) adamw_kernel(int64_t n4, float4* __restri
                                                     float4* __restrict__ m, float4* __restrict__ v,
                                                     uint2* __restrict__ wb, float lr, float b1, float b2, float eps,
                                                     float wd, float inv_bc1, float inv_bc2, int zero_grad) {
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
     float4 W = w[i], G = g[i], M = m[i], V = v[i];
     float* pw = &W.x;
@@ -473,6 +482,8 @@ __global__ void f32_to_bf16_kernel(int64_t n, const float* __restrict__ src, __n
 // blockIdx.y = table entry; each entry moves n8 groups of 8 elements between a client
 // buffer (bf16) and the packed buffer (bf16 or fp32).
 __global__ void copy_clients_kernel(CopyTable tab) {
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   const int e = blockIdx.y;
   if (e >= tab.n) return;
   const int64_t n8 = tab.n8[e], off = tab.off8[e];
@@ -507,6 +518,8 @@ __global__ void copy_clients_kernel(CopyTable tab) {
 // (i, 0) in the context (or in a plain causal segment, c = 0), (mp, i - c + 1) in the span.
 __global__ void meta_kernel(MetaArgs a, int32_t* __restrict__ cu, int32_t* __restrict__ pos,
                             uint32_t* __restrict__ tiles, int32_t* __restrict__ pos2, int32_t* __restrict__ ctx) {
+  pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
+  pdl_trigger();
   const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t nth = (int64_t)gridDim.x * blockDim.x;
   const int T = a.cu[a.S];
@@ -642,8 +655,8 @@ extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void
   int rows = (T + rblocks - 1) / rblocks;
   rows = (rows + 7) / 8 * 8;
   rblocks = (T + rows - 1) / rows;
-  colsum_kernel<<<dim3(cblocks, rblocks), 256, 0, (cudaStream_t)stream>>>(T, N, (const __nv_bfloat16*)x, out, rows);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(colsum_kernel, dim3(cblocks, rblocks), dim3(256), 0, (cudaStream_t)stream, T, N,
+                        (const __nv_bfloat16*)x, out, rows));
   return FL_OK;
 }
 
@@ -663,9 +676,9 @@ int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_b
                     float beta2, float eps, float weight_decay, float bc1, float bc2, int zero_grad, cudaStream_t st) {
   if (n <= 0) return FL_OK;
   const int64_t n4 = n / 4;
-  adamw_kernel<<<grid_for(n4), 256, 0, st>>>(n4, (float4*)w, (float4*)g, (float4*)m, (float4*)v, (uint2*)w_bf16, lr,
-                                             beta1, beta2, eps, weight_decay, 1.f / bc1, 1.f / bc2, zero_grad);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(adamw_kernel, dim3(grid_for(n4)), dim3(256), 0, st, n4, (float4*)w, (float4*)g, (float4*)m,
+                        (float4*)v, (uint2*)w_bf16, lr, beta1, beta2, eps, weight_decay, 1.f / bc1, 1.f / bc2,
+                        zero_grad));
   return FL_OK;
 }
 
@@ -679,16 +692,15 @@ int fl_launch_copy_clients(const CopyTable& tab, cudaStream_t st) {
   const int cap = (2 * sm_count() + tab.n - 1) / tab.n + 1;
   if (gx > cap) gx = cap;
   if (gx < 1) gx = 1;
-  copy_clients_kernel<<<dim3(gx, tab.n), 256, 0, st>>>(tab);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(copy_clients_kernel, dim3(gx, tab.n), dim3(256), 0, st, tab));
   return FL_OK;
 }
 
 int fl_launch_meta(const MetaArgs& a, int32_t* cu, int32_t* pos, uint32_t* tiles, int32_t* pos2, int32_t* ctx,
                    cudaStream_t st) {
   const int T = a.cu[a.S];
-  meta_kernel<<<grid_for(T > a.n_tiles ? T : a.n_tiles), 256, 0, st>>>(a, cu, pos, tiles, pos2, ctx);
-  FL_CUDA_TRY(cudaGetLastError());
+  FL_CUDA_TRY(fl_launch(meta_kernel, dim3(grid_for(T > a.n_tiles ? T : a.n_tiles)), dim3(256), 0, st, a, cu, pos,
+                        tiles, pos2, ctx));
   return FL_OK;
 }
 
