@@ -279,7 +279,7 @@ def main():
     ap.add_argument("--no-other-configs", action="store_true",
                     help="skip the ragged workload and the packed-vs-sequential points after the main line")
     ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the oracle sample")
-    ap.add_argument("--ref-tokens", type=int, default=128, help="tokens of the reference-arm sample")
+    ap.add_argument("--ref-tokens", type=int, default=256, help="tokens of the reference-arm sample")
     ap.add_argument("--sweep", action="store_true",
                     help="client-batching sweep: 26 blocks, 2 x 512 tokens per client, K in 1..32, "
                          "one packed call vs K sequential single-client calls (one JSON line per K)")

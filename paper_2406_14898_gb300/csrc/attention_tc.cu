@@ -3,8 +3,9 @@
 // keys, causal within the segment or with a bidirectional GLM context; §3.3 segments are
 // never mixed), with both tile contractions on tcgen05 and their accumulators in TMEM.
 //
-// One CTA (4 warps) per (128-query tile, head).  Thread i owns query row i, which is TMEM
-// lane i.  Per 128-key tile j:
+// Persistent CTAs (4 warps, two per SM) walk the (128-query tile, head) units; the next
+// unit's Q and first K / V tiles load while a unit's output is written.  Thread i owns
+// query row i, which is TMEM lane i.  Per 128-key tile j:
 //   TMA: K_j and V_j (128 rows x head_dim, 64-column 128-byte-swizzled boxes; Q once),
 //        each on its own barrier;
 //   S = Q K_j^T     -> TMEM columns [0, 128)   (tcgen05.mma, both operands in shared memory);
@@ -56,9 +57,9 @@ FL_DEV uint64_t desc_mnmajor(uint32_t base, int kk) { return smem_desc_sw128(bas
 template <int HD>
 __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_pk,
-    const __grid_constant__ CUtensorMap tm_pv, int T, int H, const int32_t* __restrict__ cu,
-    const uint32_t* __restrict__ tiles, bf16* __restrict__ O, float* __restrict__ lse, float scale_log2, int Lp,
-    const int32_t* __restrict__ ctxs, int* status) {
+    const __grid_constant__ CUtensorMap tm_pv, int T, int H, int n_heads, const int32_t* __restrict__ cu,
+    const uint32_t* __restrict__ tiles, int n_units, bf16* __restrict__ O, float* __restrict__ lse,
+    float scale_log2, int Lp, const int32_t* __restrict__ ctxs, int* status) {
   constexpr int NB = FwdCfg<HD>::NB, TILE = FwdCfg<HD>::TILE;
   pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
   pdl_trigger();
@@ -74,16 +75,26 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   uint64_t* bar_s = bars + 3;
   uint64_t* bar_pv = bars + 4;
   uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 6);
-
-  // the 128-row tile list: (segment, query tile)
-  const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
-  const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5;
-  const int seg0 = cu[s], L = cu[s + 1] - seg0;
-  const int q0 = idx * TB;
   const int npt = Lp > 0 ? 1 : 0;  // at most one prefix tile (Lp <= 128)
-  const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
-  const int n_kv = npt + max(idx, clast >= 0 ? clast / TB : 0) + 1;
+
+  // A work unit u is (entry u / n_heads of the 128-row tile list, head u % n_heads): the
+  // list's longest causal rows first.
+  struct Unit {
+    int h, seg0, L, q0, clast, n_kv;
+  };
+  auto unit = [&](int u) {
+    Unit w;
+    const uint32_t t = tiles[u / n_heads];
+    const int s = int(t >> 16), idx = int(t & 0xFFFFu);
+    w.h = u % n_heads;
+    w.seg0 = cu[s];
+    w.L = cu[s + 1] - w.seg0;
+    w.q0 = idx * TB;
+    w.clast = (ctxs ? min(max(ctxs[s], 0), w.L) : 0) - 1;
+    w.n_kv = npt + max(idx, w.clast >= 0 ? w.clast / TB : 0) + 1;
+    return w;
+  };
 
   if (tid == 0) {
     for (int i = 0; i < 5; ++i) mbar_init(bars + i, 1);
@@ -101,137 +112,153 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   const uint32_t t_lane = tmem + (uint32_t(warp * 32) << 16);  // this warp's TMEM lanes
   const uint32_t t_s = t_lane, t_o = t_lane + 128;
 
-  // one elected thread: the key (part 0) or value (part 1) tile j into its buffer
-  auto issue = [&](int j, int part) {
+  // one elected thread: the key (part 0) or value (part 1) tile j of unit w into its buffer
+  auto issue = [&](const Unit& w, int j, int part) {
     uint8_t* dst = part ? sV : sK;
     uint64_t* bar = part ? bar_v : bar_k;
     mbar_arrive_expect_tx(bar, TILE);
     if (j < npt) {
       const CUtensorMap* m = part ? &tm_pv : &tm_pk;
 #pragma unroll
-      for (int b = 0; b < NB; ++b) tma_load_2d(dst + b * BOX, m, bar, h * HD + 64 * b, 0);
+      for (int b = 0; b < NB; ++b) tma_load_2d(dst + b * BOX, m, bar, w.h * HD + 64 * b, 0);
     } else {
-      const int row = seg0 + (j - npt) * TB;
+      const int row = w.seg0 + (j - npt) * TB;
 #pragma unroll
-      for (int b = 0; b < NB; ++b) tma_load_2d(dst + b * BOX, &tm_qkv, bar, (1 + part) * H + h * HD + 64 * b, row);
+      for (int b = 0; b < NB; ++b)
+        tma_load_2d(dst + b * BOX, &tm_qkv, bar, (1 + part) * H + w.h * HD + 64 * b, row);
     }
   };
-  if (tid == 0) {
+  auto issue_unit = [&](const Unit& w) {  // Q and the first key / value tiles of a unit
     mbar_arrive_expect_tx(bar_q, TILE);
 #pragma unroll
-    for (int b = 0; b < NB; ++b) tma_load_2d(sQ + b * BOX, &tm_qkv, bar_q, h * HD + 64 * b, seg0 + q0);
-    issue(0, 0);
-    issue(0, 1);
-  }
+    for (int b = 0; b < NB; ++b) tma_load_2d(sQ + b * BOX, &tm_qkv, bar_q, w.h * HD + 64 * b, w.seg0 + w.q0);
+    issue(w, 0, 0);
+    issue(w, 0, 1);
+  };
 
   constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
   constexpr uint32_t IDESC_PV = umma_idesc_bf16(TB, HD, false, true);
-  const int q = q0 + tid;  // this thread's query row (inside the segment)
-  float m_run = -INFINITY, l_run = 0.f;
-  bool ok = __syncthreads_and(mbar_wait(bar_q, 0));
-  if (!ok && tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
-  uint32_t ph = 0;
-  for (int j = 0; j < n_kv && ok; ++j, ph ^= 1) {
+  // completed phases of each barrier so far (a wait takes the parity of its count)
+  uint32_t nq = 0, nk = 0, nv = 0, ns = 0, npv = 0;
+  bool ok = true;
+  int u = blockIdx.x;
+  Unit w = u < n_units ? unit(u) : Unit{};
+  if (tid == 0 && u < n_units) issue_unit(w);
+  while (u < n_units && ok) {
+    const int q = w.q0 + tid;  // this thread's query row (inside the segment)
+    float m_run = -INFINITY, l_run = 0.f;
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
-    if (!__syncthreads_and(mbar_wait(bar_k, ph))) {
+    if (!__syncthreads_and(mbar_wait(bar_q, (nq++) & 1))) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
       ok = false;
       break;
     }
-    // ---- S = Q K_j^T (the previous P V, which read the S columns, has completed)
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t aq = smem_u32(sQ), bk = smem_u32(sK);
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_kmajor(aq, kk), desc_kmajor(bk, kk), IDESC_S, kk > 0);
-      umma_commit(bar_s);
-    }
-    if (!__syncthreads_and(mbar_wait(bar_s, ph))) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
-      ok = false;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && j + 1 < n_kv) issue(j + 1, 0);  // K_j has been read
-    // ---- the thread's S row, read once (4 x 32 columns, one wait)
-    const bool prefix = j < npt;
-    const int kb = prefix ? 0 : (j - npt) * TB;  // first key of the tile inside its sequence
-    const int klim = prefix ? Lp - 1 : min(L - 1, max(q, clast));  // last visible key
-    const bool full = kb + TB - 1 <= klim;       // every key of the tile visible to this row
-    uint32_t r[TB];
-    tmem_ld32(t_s, *reinterpret_cast<uint32_t(*)[32]>(r));
-    tmem_ld32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
-    tmem_ld32(t_s + 64, *reinterpret_cast<uint32_t(*)[32]>(r + 64));
-    tmem_ld32(t_s + 96, *reinterpret_cast<uint32_t(*)[32]>(r + 96));
-    tmem_ld_wait();
-    // masked row max; invisible keys become -inf
-    float mt = -INFINITY;
-#pragma unroll
-    for (int e = 0; e < TB; ++e) {
-      float x = __uint_as_float(r[e]) * scale_log2;
-      if (!full && kb + e > klim) x = -INFINITY;
-      r[e] = __float_as_uint(x);
-      mt = fmaxf(mt, x);
-    }
-    const float m_new = fmaxf(m_run, mt);
-    const float mref = m_new == -INFINITY ? 0.f : m_new;
-    const float corr = exp2f(m_run - mref);  // 0 on the first tile (m_run = -inf)
-    // ---- P = exp2(S - m), bf16 pairs (keys 2c, 2c + 1 in column c) into S's columns [0, 64)
-    float lt = 0.f;
-#pragma unroll
-    for (int c = 0; c < TB / 2; ++c) {
-      const float p0 = exp2f(__uint_as_float(r[2 * c]) - mref);
-      const float p1 = exp2f(__uint_as_float(r[2 * c + 1]) - mref);
-      lt += p0 + p1;
-      r[c] = pack_bf16x2(p0, p1);
-    }
-    tmem_st32(t_s, *reinterpret_cast<uint32_t(*)[32]>(r));
-    tmem_st32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
-    l_run = l_run * corr + lt;
-    m_run = m_new;
-    // ---- rescale the O rows when a row max moved (not before the first P V); TMEM
-    // loads and stores are warp-wide, so the whole warp takes part (factor 1 elsewhere)
-    if (j > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
-#pragma unroll 1
-      for (int c = 0; c < HD; c += 32) {
-        uint32_t o[32];
-        tmem_ld32(t_o + c, o);
-        tmem_ld_wait();
-#pragma unroll
-        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * corr);
-        tmem_st32(t_o + c, o);
+    for (int j = 0; j < w.n_kv && ok; ++j) {
+      if (!__syncthreads_and(mbar_wait(bar_k, (nk++) & 1))) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+        ok = false;
+        break;
       }
-    }
-    tmem_st_wait();
-    tc_fence_before();
-    if (!__syncthreads_and(mbar_wait(bar_v, ph))) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
-      ok = false;
-      break;
-    }
-    // ---- O += P V_j
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t bv = smem_u32(sV);
+      // ---- S = Q K_j^T (the previous P V, which read the S columns, has completed)
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t aq = smem_u32(sQ), bk = smem_u32(sK);
 #pragma unroll
-      for (int kk = 0; kk < TB / 16; ++kk)
-        umma_bf16_ts(tmem + 128, tmem + kk * 8, desc_mnmajor(bv, kk), IDESC_PV, (j > 0 || kk > 0) ? 1u : 0u);
-      umma_commit(bar_pv);
+        for (int kk = 0; kk < HD / 16; ++kk)
+          umma_bf16(tmem, desc_kmajor(aq, kk), desc_kmajor(bk, kk), IDESC_S, kk > 0);
+        umma_commit(bar_s);
+      }
+      if (!__syncthreads_and(mbar_wait(bar_s, (ns++) & 1))) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (tid == 0 && j + 1 < w.n_kv) issue(w, j + 1, 0);  // K_j has been read
+      // ---- the thread's S row, read once (4 x 32 columns, one wait)
+      const bool prefix = j < npt;
+      const int kb = prefix ? 0 : (j - npt) * TB;  // first key of the tile inside its sequence
+      const int klim = prefix ? Lp - 1 : min(w.L - 1, max(q, w.clast));  // last visible key
+      const bool full = kb + TB - 1 <= klim;       // every key of the tile visible to this row
+      uint32_t r[TB];
+      tmem_ld32(t_s, *reinterpret_cast<uint32_t(*)[32]>(r));
+      tmem_ld32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
+      tmem_ld32(t_s + 64, *reinterpret_cast<uint32_t(*)[32]>(r + 64));
+      tmem_ld32(t_s + 96, *reinterpret_cast<uint32_t(*)[32]>(r + 96));
+      tmem_ld_wait();
+      // masked row max; invisible keys become -inf
+      float mt = -INFINITY;
+#pragma unroll
+      for (int e = 0; e < TB; ++e) {
+        float x = __uint_as_float(r[e]) * scale_log2;
+        if (!full && kb + e > klim) x = -INFINITY;
+        r[e] = __float_as_uint(x);
+        mt = fmaxf(mt, x);
+      }
+      const float m_new = fmaxf(m_run, mt);
+      const float mref = m_new == -INFINITY ? 0.f : m_new;
+      const float corr = exp2f(m_run - mref);  // 0 on the first tile (m_run = -inf)
+      // ---- P = exp2(S - m), bf16 pairs (keys 2c, 2c + 1 in column c) into S's columns [0, 64)
+      float lt = 0.f;
+#pragma unroll
+      for (int c = 0; c < TB / 2; ++c) {
+        const float p0 = exp2f(__uint_as_float(r[2 * c]) - mref);
+        const float p1 = exp2f(__uint_as_float(r[2 * c + 1]) - mref);
+        lt += p0 + p1;
+        r[c] = pack_bf16x2(p0, p1);
+      }
+      tmem_st32(t_s, *reinterpret_cast<uint32_t(*)[32]>(r));
+      tmem_st32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(r + 32));
+      l_run = l_run * corr + lt;
+      m_run = m_new;
+      // ---- rescale the O rows when a row max moved (not before the first P V); TMEM
+      // loads and stores are warp-wide, so the whole warp takes part (factor 1 elsewhere)
+      if (j > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
+#pragma unroll 1
+        for (int c = 0; c < HD; c += 32) {
+          uint32_t o[32];
+          tmem_ld32(t_o + c, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * corr);
+          tmem_st32(t_o + c, o);
+        }
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      if (!__syncthreads_and(mbar_wait(bar_v, (nv++) & 1))) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+        ok = false;
+        break;
+      }
+      // ---- O += P V_j
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t bv = smem_u32(sV);
+#pragma unroll
+        for (int kk = 0; kk < TB / 16; ++kk)
+          umma_bf16_ts(tmem + 128, tmem + kk * 8, desc_mnmajor(bv, kk), IDESC_PV, (j > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(bar_pv);
+      }
+      if (!__syncthreads_and(mbar_wait(bar_pv, (npv++) & 1))) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (tid == 0 && j + 1 < w.n_kv) issue(w, j + 1, 1);  // V_j has been read
     }
-    if (!__syncthreads_and(mbar_wait(bar_pv, ph))) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
-      ok = false;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && j + 1 < n_kv) issue(j + 1, 1);  // V_j has been read
-  }
-  // ---- O / l and the log-sum-exp (every lane reads TMEM; rows past the segment end
-  // store nothing)
-  if (ok) {
-    const bool valid = q < L;
+    if (!ok) break;
+    // ---- every product of the unit is complete and Q / K / V are free: the next unit's
+    // first tiles load while this one's O leaves
+    const int un = u + gridDim.x;
+    const Unit wn = un < n_units ? unit(un) : Unit{};
+    if (tid == 0 && un < n_units) issue_unit(wn);
+    // ---- O / l and the log-sum-exp (every lane reads TMEM; rows past the segment end
+    // store nothing)
+    const bool valid = q < w.L;
     const float inv = valid ? 1.f / l_run : 0.f;
-    bf16* orow = O + (int64_t)(seg0 + (valid ? q : 0)) * H + h * HD;
+    bf16* orow = O + (int64_t)(w.seg0 + (valid ? q : 0)) * H + w.h * HD;
 #pragma unroll 1
     for (int c = 0; c < HD; c += 32) {
       uint32_t o[32];
@@ -239,15 +266,19 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
       tmem_ld_wait();
       if (valid) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-          *reinterpret_cast<uint4*>(orow + c + 8 * u) = make_uint4(
-              pack_bf16x2(__uint_as_float(o[8 * u]) * inv, __uint_as_float(o[8 * u + 1]) * inv),
-              pack_bf16x2(__uint_as_float(o[8 * u + 2]) * inv, __uint_as_float(o[8 * u + 3]) * inv),
-              pack_bf16x2(__uint_as_float(o[8 * u + 4]) * inv, __uint_as_float(o[8 * u + 5]) * inv),
-              pack_bf16x2(__uint_as_float(o[8 * u + 6]) * inv, __uint_as_float(o[8 * u + 7]) * inv));
+        for (int v = 0; v < 4; ++v)
+          *reinterpret_cast<uint4*>(orow + c + 8 * v) = make_uint4(
+              pack_bf16x2(__uint_as_float(o[8 * v]) * inv, __uint_as_float(o[8 * v + 1]) * inv),
+              pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv),
+              pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv),
+              pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv));
       }
     }
-    if (valid) lse[(int64_t)h * T + seg0 + q] = (m_run + log2f(l_run)) * LN2_T;
+    if (valid) lse[(int64_t)w.h * T + w.seg0 + q] = (m_run + log2f(l_run)) * LN2_T;
+    // the O columns are read before the next unit's first P V overwrites them
+    tc_fence_before();
+    u = un;
+    w = wn;
   }
   tc_fence_before();
   __syncthreads();
@@ -277,8 +308,11 @@ int launch_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint3
     tpv = tq;
   }
   const float scale_log2 = (1.f / sqrtf((float)HD)) * LOG2E_T;
-  FL_CUDA_TRY(fl_launch(attn_fwd_tc_kernel<HD>, dim3(n_tiles, nh), dim3(128), FwdCfg<HD>::SMEM, st, tq, tpk, tpv, T, H,
-                        cu, tiles, (bf16*)o, lse, scale_log2, pre.len, glm.ctx, status));
+  // persistent: two CTAs per SM walk the (tile, head) units
+  const int n_units = n_tiles * nh;
+  const int grid = n_units < 2 * fl_gemm::num_sms() ? n_units : 2 * fl_gemm::num_sms();
+  FL_CUDA_TRY(fl_launch(attn_fwd_tc_kernel<HD>, dim3(grid), dim3(128), FwdCfg<HD>::SMEM, st, tq, tpk, tpv, T, H, nh,
+                        cu, tiles, n_units, (bf16*)o, lse, scale_log2, pre.len, glm.ctx, status));
   return FL_OK;
 }
 
