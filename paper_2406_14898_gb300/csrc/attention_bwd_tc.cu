@@ -47,6 +47,7 @@
 #include "gemm_tc.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
+#include "waits.cuh"
 
 namespace {
 
@@ -221,9 +222,11 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   const uint32_t tmem = *holder;
   const uint32_t t_lane = tmem + (uint32_t(quarter * 32) << 16);
 
+  BarTrack tkv, tq0, tq1, tm1, tm2;
   auto issue_q = [&](int it, int b) {  // one elected thread: Q_it, dO_it into buffer pair b
     int row0, qpos0, valid;
     qtile(it, row0, qpos0, valid);
+    (b ? tq1 : tq0).pend = true;
     mbar_arrive_expect_tx(bar_q + b, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
@@ -232,6 +235,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     }
   };
   if (tid == 0 && it0 < it_end) {
+    tkv.pend = true;
     mbar_arrive_expect_tx(bar_kv, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
@@ -249,11 +253,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
 
   constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
   constexpr uint32_t IDESC_G = umma_idesc_bf16(TB, HD, false, true);
-  bool ok = it0 >= it_end || __syncthreads_and(mbar_wait(bar_kv, 0));
+  bool ok = it0 >= it_end || track_wait_all(bar_kv, tkv);
   if (!ok && tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
   for (int it = it0; it < it_end && ok; ++it) {
     const int n = it - it0, b = n & 1;
-    const uint32_t ph = n & 1, phq = (n >> 1) & 1;
     int row0, qpos0, valid;
     qtile(it, row0, qpos0, valid);
     {  // lse and delta of the query tile (rows past its segment are never visible)
@@ -264,7 +267,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       else sD[b * TB + c] = v;
     }
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
-    if (!__syncthreads_and(mbar_wait(bar_q + b, phq))) {
+    if (!track_wait_all(bar_q + b, b ? tq1 : tq0)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
       ok = false;
       break;
@@ -279,9 +282,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_k(ak, kk), desc_k(bq, kk), IDESC_S, kk > 0);
 #pragma unroll
       for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem + 128, desc_k(av, kk), desc_k(bo, kk), IDESC_S, kk > 0);
+      tm1.pend = true;
       umma_commit(bar_mma1);
     }
-    if (!__syncthreads_and(mbar_wait(bar_mma1, ph))) {
+    if (!track_wait_all(bar_mma1, tm1)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
       ok = false;
       break;
@@ -350,9 +354,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
 #pragma unroll
       for (int kk = 0; kk < TB / 16; ++kk)
         umma_bf16_ts(tmem + 256 + HD, tmem + 128 + a_col(kk), desc_mn(bq, kk), IDESC_G, (acc || kk > 0) ? 1u : 0u);
+      tm2.pend = true;
       umma_commit(bar_mma2);
     }
-    if (!__syncthreads_and(mbar_wait(bar_mma2, ph))) {
+    if (!track_wait_all(bar_mma2, tm2)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
       ok = false;
       break;
@@ -422,6 +427,13 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       }
     }
   }
+  if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
+    track_drain(bar_kv, tkv);
+    track_drain(bar_q, tq0);
+    track_drain(bar_q + 1, tq1);
+    track_drain(bar_mma1, tm1);
+    track_drain(bar_mma2, tm2);
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
@@ -487,7 +499,9 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   const uint32_t tmem = *holder;
   const uint32_t t_lane = tmem + (uint32_t(quarter * 32) << 16);
 
+  BarTrack tqdo, tkv0, tkv1, tm1, tm2;
   auto issue_kv = [&](int j, int b) {  // one elected thread: K_j, V_j into buffer pair b
+    (b ? tkv1 : tkv0).pend = true;
     mbar_arrive_expect_tx(bar_kv + b, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
@@ -502,6 +516,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     }
   };
   if (tid == 0) {
+    tqdo.pend = true;
     mbar_arrive_expect_tx(bar_qdo, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
@@ -514,12 +529,11 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
 
   constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
   constexpr uint32_t IDESC_G = umma_idesc_bf16(TB, HD, false, true);
-  bool ok = __syncthreads_and(mbar_wait(bar_qdo, 0));
+  bool ok = track_wait_all(bar_qdo, tqdo);
   if (!ok && tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
   for (int j = 0; j < n_kv && ok; ++j) {
     const int b = j & 1;
-    const uint32_t ph = j & 1, phk = (j >> 1) & 1;
-    if (!__syncthreads_and(mbar_wait(bar_kv + b, phk))) {
+    if (!track_wait_all(bar_kv + b, b ? tkv1 : tkv0)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
       ok = false;
       break;
@@ -534,9 +548,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
       for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_k(aq, kk), desc_k(bk, kk), IDESC_S, kk > 0);
 #pragma unroll
       for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem + 128, desc_k(ao, kk), desc_k(bv, kk), IDESC_S, kk > 0);
+      tm1.pend = true;
       umma_commit(bar_mma1);
     }
-    if (!__syncthreads_and(mbar_wait(bar_mma1, ph))) {
+    if (!track_wait_all(bar_mma1, tm1)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
       ok = false;
       break;
@@ -581,9 +596,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
 #pragma unroll
       for (int kk = 0; kk < TB / 16; ++kk)
         umma_bf16_ts(tmem + 256, tmem + a_col(kk), desc_mn(bk, kk), IDESC_G, (j > 0 || kk > 0) ? 1u : 0u);
+      tm2.pend = true;
       umma_commit(bar_mma2);
     }
-    if (!__syncthreads_and(mbar_wait(bar_mma2, ph))) {
+    if (!track_wait_all(bar_mma2, tm2)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
       ok = false;
       break;
@@ -625,6 +641,13 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
         *reinterpret_cast<uint4*>(dqkv + ((int64_t)seg0 + q0 + row) * 3 * H + col + jc * 8) =
             *reinterpret_cast<const uint4*>(stage_chunk<HD>(sK, row, jc));
     }
+  }
+  if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
+    track_drain(bar_qdo, tqdo);
+    track_drain(bar_kv, tkv0);
+    track_drain(bar_kv + 1, tkv1);
+    track_drain(bar_mma1, tm1);
+    track_drain(bar_mma2, tm2);
   }
   tc_fence_before();
   __syncthreads();

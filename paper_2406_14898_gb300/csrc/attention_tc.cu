@@ -28,6 +28,7 @@
 #include "gemm_tc.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
+#include "waits.cuh"
 
 namespace {
 
@@ -112,10 +113,12 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   const uint32_t t_lane = tmem + (uint32_t(warp * 32) << 16);  // this warp's TMEM lanes
   const uint32_t t_s = t_lane, t_o = t_lane + 128;
 
+  BarTrack tq, tk, tv, ts, tpv;
   // one elected thread: the key (part 0) or value (part 1) tile j of unit w into its buffer
   auto issue = [&](const Unit& w, int j, int part) {
     uint8_t* dst = part ? sV : sK;
     uint64_t* bar = part ? bar_v : bar_k;
+    (part ? tv : tk).pend = true;
     mbar_arrive_expect_tx(bar, TILE);
     if (j < npt) {
       const CUtensorMap* m = part ? &tm_pv : &tm_pk;
@@ -129,6 +132,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     }
   };
   auto issue_unit = [&](const Unit& w) {  // Q and the first key / value tiles of a unit
+    tq.pend = true;
     mbar_arrive_expect_tx(bar_q, TILE);
 #pragma unroll
     for (int b = 0; b < NB; ++b) tma_load_2d(sQ + b * BOX, &tm_qkv, bar_q, w.h * HD + 64 * b, w.seg0 + w.q0);
@@ -138,8 +142,6 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
 
   constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
   constexpr uint32_t IDESC_PV = umma_idesc_bf16(TB, HD, false, true);
-  // completed phases of each barrier so far (a wait takes the parity of its count)
-  uint32_t nq = 0, nk = 0, nv = 0, ns = 0, npv = 0;
   bool ok = true;
   int u = blockIdx.x;
   Unit w = u < n_units ? unit(u) : Unit{};
@@ -148,13 +150,13 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     const int q = w.q0 + tid;  // this thread's query row (inside the segment)
     float m_run = -INFINITY, l_run = 0.f;
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
-    if (!__syncthreads_and(mbar_wait(bar_q, (nq++) & 1))) {
+    if (!track_wait_all(bar_q, tq)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
       ok = false;
       break;
     }
     for (int j = 0; j < w.n_kv && ok; ++j) {
-      if (!__syncthreads_and(mbar_wait(bar_k, (nk++) & 1))) {
+      if (!track_wait_all(bar_k, tk)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
         ok = false;
         break;
@@ -166,9 +168,10 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
           umma_bf16(tmem, desc_kmajor(aq, kk), desc_kmajor(bk, kk), IDESC_S, kk > 0);
+        ts.pend = true;
         umma_commit(bar_s);
       }
-      if (!__syncthreads_and(mbar_wait(bar_s, (ns++) & 1))) {
+      if (!track_wait_all(bar_s, ts)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
         ok = false;
         break;
@@ -226,7 +229,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
       }
       tmem_st_wait();
       tc_fence_before();
-      if (!__syncthreads_and(mbar_wait(bar_v, (nv++) & 1))) {
+      if (!track_wait_all(bar_v, tv)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
         ok = false;
         break;
@@ -238,9 +241,10 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
 #pragma unroll
         for (int kk = 0; kk < TB / 16; ++kk)
           umma_bf16_ts(tmem + 128, tmem + kk * 8, desc_mnmajor(bv, kk), IDESC_PV, (j > 0 || kk > 0) ? 1u : 0u);
+        tpv.pend = true;
         umma_commit(bar_pv);
       }
-      if (!__syncthreads_and(mbar_wait(bar_pv, (npv++) & 1))) {
+      if (!track_wait_all(bar_pv, tpv)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
         ok = false;
         break;
@@ -279,6 +283,13 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     tc_fence_before();
     u = un;
     w = wn;
+  }
+  if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
+    track_drain(bar_q, tq);
+    track_drain(bar_k, tk);
+    track_drain(bar_v, tv);
+    track_drain(bar_s, ts);
+    track_drain(bar_pv, tpv);
   }
   tc_fence_before();
   __syncthreads();

@@ -86,6 +86,16 @@ FL_DEV float2 block_sum2(float a, float b, float2 (*red)[32], int par) {
 // bounded: on expiry the CTA records a status code and stops.
 constexpr int LN_STAGES = 4;
 
+// After a stage wait gave up at iteration `it`: the elected thread waits (bounded) for every
+// row copy still in flight into the CTA's NS stages (the next row of each stage, if the
+// schedule issued it), so that none lands after the CTA has left.
+FL_DEV void ln_drain(uint64_t* full, int NS, int it, int T) {
+  for (int s = 0; s < NS; ++s) {
+    const int it2 = ((it - s + NS - 1) / NS) * NS + s;  // next iteration that uses stage s
+    if (blockIdx.x + (int64_t)it2 * gridDim.x < T) mbar_wait(full + s, (it2 / NS) & 1);
+  }
+}
+
 template <typename TX, int CH>
 __global__ void __launch_bounds__(256) ln_fwd_bulk_kernel(int T, int H, const TX* __restrict__ x,
                                                           const float* __restrict__ gamma,
@@ -123,7 +133,10 @@ __global__ void __launch_bounds__(256) ln_fwd_bulk_kernel(int T, int H, const TX
     if (row >= T) break;
     const int st = it % LN_STAGES;
     if (!__syncthreads_and(mbar_wait(full + st, (it / LN_STAGES) & 1))) {
-      if (c == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+      if (c == 0) {
+        report_status(status, FL_DEV_TIMEOUT_FULL);
+        ln_drain(full, LN_STAGES, it, T);
+      }
       break;
     }
     const TX* xr = reinterpret_cast<const TX*>(ln_smem + st * row_bytes);
@@ -232,7 +245,10 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
     if (row >= Tn) break;
     const int st = it % LNB_STAGES;
     if (!__syncthreads_and(mbar_wait(full + st, (it / LNB_STAGES) & 1))) {
-      if (c == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+      if (c == 0) {
+        report_status(status, FL_DEV_TIMEOUT_FULL);
+        ln_drain(full, LNB_STAGES, it, Tn);
+      }
       break;
     }
     float d[8], xh[8], gcol[8];
