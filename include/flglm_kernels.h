@@ -94,7 +94,21 @@ typedef struct {
   float* colsum;                            /* FL_EPI_GELU_BWD only, or NULL: colsum[n] += sum over m of
                                                D[m,n] (fp32, before rounding; fp32 atomics, so the
                                                order of the additions is not fixed); 16-byte aligned */
+  /* Batched launch (the replicas of the server-hierarchical strategy, §3.3): `batch`
+   * independent problems of the same shape and epilogue in one launch (0 or 1: one problem;
+   * at most FL_GEMM_MAX_BATCH).  Problem r reads A + r*a_bstride and B + r*b_bstride and its
+   * epilogue uses every pointer above offset by r times its stride, in elements of the
+   * pointer's own type: D by d_bstride, aux by aux_bstride, aux_out by aux_out_bstride,
+   * bias and colsum by bias_bstride, pos, pos2, ln_mean and ln_rstd by row_bstride,
+   * ln_gamma and ln_beta by lnp_bstride, adam_m and adam_v by adam_bstride.  Strides keep
+   * every problem's pointers 16-byte aligned.  Each problem's result is bit-identical to
+   * its own unbatched launch. */
+  int32_t batch;
+  int64_t a_bstride, b_bstride, d_bstride, aux_bstride, aux_out_bstride;
+  int64_t bias_bstride, row_bstride, lnp_bstride, adam_bstride;
 } fl_gemm_args;
+
+#define FL_GEMM_MAX_BATCH 4
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);
 

@@ -109,6 +109,21 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
     return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: column sums only with the GeLU-backward epilogue");
   if (a->colsum && !aligned16(a->colsum))
     return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: colsum must be 16-byte aligned");
+  if (a->batch < 0 || a->batch > FL_GEMM_MAX_BATCH)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: batch %d outside 0..%d", a->batch, FL_GEMM_MAX_BATCH);
+  const int batch = a->batch > 1 ? a->batch : 1;
+  if (batch > 1) {
+    // every problem's pointers keep the 16-byte alignment of the first problem's: strides in
+    // bf16 elements multiples of 8, in fp32 elements multiples of 4 (and of 4 for the
+    // per-row int32 / fp32 arrays read one element at a time)
+    const bool d32 = a->d_dtype == FL_DT_F32 || mode == FL_EPI_STORE_F32 || mode == FL_EPI_ACCUM_F32 ||
+                     mode == FL_EPI_ADAMW;
+    if ((a->a_bstride % 8) || (a->b_bstride % 8) || (a->d_bstride % (d32 ? 4 : 8)) ||
+        (a->aux && (a->aux_bstride % (a->aux_dtype == FL_DT_F32 ? 4 : 8))) || (a->aux_out && (a->aux_out_bstride % 8)) ||
+        ((a->bias || a->colsum) && (a->bias_bstride % 4)) || (a->ln_mean && (a->lnp_bstride % 4)) ||
+        (a->adam_m && (a->adam_bstride % 4)))
+      return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: batch strides break the 16-byte alignment");
+  }
 
   Epi e;
   e.mode = mode;
@@ -142,6 +157,13 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   e.inv_bc1 = a->inv_bc1;
   e.inv_bc2 = a->inv_bc2;
   e.colsum = a->colsum;
+  e.bs_d = a->d_bstride;
+  e.bs_aux = a->aux_bstride;
+  e.bs_aux_out = a->aux_out_bstride;
+  e.bs_bias = a->bias_bstride;
+  e.bs_row = a->row_bstride;
+  e.bs_lnp = a->lnp_bstride;
+  e.bs_adam = a->adam_bstride;
 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const bool amn = a->a_mn_major != 0, bmn = a->b_mn_major != 0;
@@ -160,15 +182,15 @@ extern "C" int fl_k_gemm(const fl_gemm_args* a, int* status, void* stream) {
   if ((a->N % 256) == 0) {
     const int sms = num_sms();
     const int pairs = pair_slots_for(fam, amn, bmn);
-    const long t128 = (long)((a->M + BM - 1) / BM) * (a->N / 128);
+    const long t128 = (long)batch * ((a->M + BM - 1) / BM) * (a->N / 128);
     const double eff128 = double(t128) / double(((t128 + sms - 1) / sms) * sms);
     double eff_wide;
     if (pairs > 0) {
-      const long tp = (long)((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
+      const long tp = (long)batch * ((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
       eff_wide = double(tp) / double(((tp + pairs - 1) / pairs) * pairs);
       shape = 2;
     } else {
-      const long t256 = (long)((a->M + BM - 1) / BM) * (a->N / 256);
+      const long t256 = (long)batch * ((a->M + BM - 1) / BM) * (a->N / 256);
       eff_wide = double(t256) / double(((t256 + sms - 1) / sms) * sms);
       shape = 1;
     }

@@ -66,6 +66,15 @@ struct Epi {
   float *adam_m, *adam_v;
   float lr, b1, b2, eps, wd, inv_bc1, inv_bc2;
   float* colsum;  // GELU_BWD: column sums of D added here (bias gradient of the up-projection)
+  // batched launch: element strides between the problems' pointers (fl_gemm_args)
+  int64_t bs_d, bs_aux, bs_aux_out, bs_bias, bs_row, bs_lnp, bs_adam;
+};
+
+// Tensor maps of the A and B operands of up to FL_GEMM_MAX_BATCH problems (a kernel
+// parameter: TMA reads each map from parameter space).
+struct GemmMaps {
+  CUtensorMap a[FL_GEMM_MAX_BATCH];
+  CUtensorMap b[FL_GEMM_MAX_BATCH];
 };
 
 // Epilogue families: each kernel instantiation carries only its family's code, which keeps
@@ -96,16 +105,19 @@ FL_DEV void st_quad(__nv_bfloat16* p, float4 v) {
 // (256 B of bf16 or 512 B of fp32).  Rows go in batches of RB row pairs: all global loads of
 // a batch are issued before any of its arithmetic.
 template <int FAM>
-FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows, int n0, int lane) {
+FL_DEV void epilogue_chunk(const Epi& e, int r, const float* stage, int row0, int rows, int n0, int lane) {
+  // problem r of a batched launch: element offsets of its pointers (0 for r = 0)
+  const int64_t od = r * e.bs_d, oaux = r * e.bs_aux, oauxo = r * e.bs_aux_out, ob = r * e.bs_bias,
+                orow = r * e.bs_row, olnp = r * e.bs_lnp, oad = r * e.bs_adam;
   constexpr int RB = (FAM == FAM_GELU || FAM == FAM_ROPE) ? 16 : 8;  // row pairs per batch
   const int h = lane >> 4, cl = lane & 15;
   const int n = n0 + 4 * cl;
-  const float4 bias = e.bias ? ld_quad(e.bias + n) : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4 bias = e.bias ? ld_quad(e.bias + ob + n) : make_float4(0.f, 0.f, 0.f, 0.f);
   const bool ln = FAM == FAM_RESID && e.ln_mean != nullptr;
   float4 lng = make_float4(1.f, 1.f, 1.f, 1.f), lnb = make_float4(0.f, 0.f, 0.f, 0.f);
   if (ln) {
-    lng = ld_quad(e.ln_gamma + n);
-    lnb = ld_quad(e.ln_beta + n);
+    lng = ld_quad(e.ln_gamma + olnp + n);
+    lnb = ld_quad(e.ln_beta + olnp + n);
   }
   // RoPE: a chunk of q/k columns that holds rotary dims.  Dims [0, rotary_dim) of a head
   // turn by pos; with GLM block positions, dims [rotary_dim, 2 rotary_dim) turn by pos2
@@ -142,22 +154,22 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
       rpos[i] = 0;
       if (rr < rows) {
         const int m = row0 + rr;
-        const int64_t off = (int64_t)m * e.ldd + n;
+        const int64_t off = (int64_t)m * e.ldd + n + od;
         if constexpr (FAM == FAM_RESID) {
           const int64_t oa = (int64_t)m * e.ld_aux + n;
-          aux[i] = e.aux_f32 ? ld_quad(reinterpret_cast<const float*>(e.aux) + oa) : ld_quad(e.aux + oa);
+          aux[i] = e.aux_f32 ? ld_quad(reinterpret_cast<const float*>(e.aux) + oaux + oa) : ld_quad(e.aux + oaux + oa);
           if (ln) {
-            rmu[i] = __ldg(e.ln_mean + m);
-            rrs[i] = __ldg(e.ln_rstd + m);
+            rmu[i] = __ldg(e.ln_mean + orow + m);
+            rrs[i] = __ldg(e.ln_rstd + orow + m);
           }
         } else if constexpr (FAM == FAM_ADAMW) {
           aux[i] = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(e.D) + off);  // w
-          am[i] = *reinterpret_cast<const float4*>(e.adam_m + off);
-          av[i] = *reinterpret_cast<const float4*>(e.adam_v + off);
+          am[i] = *reinterpret_cast<const float4*>(e.adam_m + (off - od + oad));
+          av[i] = *reinterpret_cast<const float4*>(e.adam_v + (off - od + oad));
         } else {
-          if (gelu_bwd) aux[i] = ld_quad(e.aux + (int64_t)m * e.ld_aux + n);
+          if (gelu_bwd) aux[i] = ld_quad(e.aux + oaux + (int64_t)m * e.ld_aux + n);
           if (accum) aux[i] = *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(e.D) + off);
-          if (FAM == FAM_ROPE && rotated) rpos[i] = __ldg(rpos_src + m);
+          if (FAM == FAM_ROPE && rotated) rpos[i] = __ldg(rpos_src + orow + m);
         }
       }
     }
@@ -182,7 +194,7 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
       }
       if (rr >= rows) continue;
       const int m = row0 + rr;
-      const int64_t off = (int64_t)m * e.ldd + n;
+      const int64_t off = (int64_t)m * e.ldd + n + od;
       const float a4[4] = {aux[i].x, aux[i].y, aux[i].z, aux[i].w};
       if constexpr (FAM == FAM_RESID) {
         const float g4[4] = {lng.x, lng.y, lng.z, lng.w}, b4[4] = {lnb.x, lnb.y, lnb.z, lnb.w};
@@ -200,7 +212,7 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
             for (int q = 0; q < 4; ++q) cs[q] += y[q];
           }
         } else {
-          st_quad(e.aux_out + (int64_t)m * e.ld_aux_out + n, make_float4(y[0], y[1], y[2], y[3]));
+          st_quad(e.aux_out + oauxo + (int64_t)m * e.ld_aux_out + n, make_float4(y[0], y[1], y[2], y[3]));
 #pragma unroll
           for (int q = 0; q < 4; ++q) y[q] = gelu_tanh(y[q]);
         }
@@ -219,9 +231,9 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
           w[q] = w[q] - e.lr * (mh / (sqrtf(vh) + e.eps) + e.wd * w[q]);
         }
         st_quad(reinterpret_cast<float*>(e.D) + off, make_float4(w[0], w[1], w[2], w[3]));
-        st_quad(e.adam_m + off, make_float4(mm[0], mm[1], mm[2], mm[3]));
-        st_quad(e.adam_v + off, make_float4(vv[0], vv[1], vv[2], vv[3]));
-        st_quad(e.aux_out + (int64_t)m * e.ld_aux_out + n, make_float4(w[0], w[1], w[2], w[3]));
+        st_quad(e.adam_m + (off - od + oad), make_float4(mm[0], mm[1], mm[2], mm[3]));
+        st_quad(e.adam_v + (off - od + oad), make_float4(vv[0], vv[1], vv[2], vv[3]));
+        st_quad(e.aux_out + oauxo + (int64_t)m * e.ld_aux_out + n, make_float4(w[0], w[1], w[2], w[3]));
       } else if (accum) {
         st_quad(reinterpret_cast<float*>(e.D) + off, make_float4(a4[0] + y[0], a4[1] + y[1], a4[2] + y[2], a4[3] + y[3]));
       } else if (out_f32) {
@@ -234,7 +246,7 @@ FL_DEV void epilogue_chunk(const Epi& e, const float* stage, int row0, int rows,
   if (colsum) {  // the two half-warps hold the same columns for rows of either parity
 #pragma unroll
     for (int q = 0; q < 4; ++q) cs[q] += __shfl_xor_sync(0xffffffffu, cs[q], 16);
-    if (h == 0 && rows > 0) red_add_v4(e.colsum + n, cs[0], cs[1], cs[2], cs[3]);
+    if (h == 0 && rows > 0) red_add_v4(e.colsum + ob + n, cs[0], cs[1], cs[2], cs[3]);
   }
 }
 
@@ -245,6 +257,10 @@ struct Raster {
   int gsz;
   int along_n;
 };
+// Problem r of a batched launch and the tile's coordinates inside it: the problems' tile
+// ranges follow each other, each in its own raster order.
+FL_DEV void batch_tile(int tile, int num_m, int num_n, Raster rs, int& r, int& mb, int& nb);
+
 FL_DEV void tile_coords(int tile, int num_m, int num_n, Raster r, int& mb, int& nb) {
   if (!r.along_n) {
     const int group = r.gsz * num_n;
@@ -265,10 +281,16 @@ FL_DEV void tile_coords(int tile, int num_m, int num_n, Raster r, int& mb, int& 
   }
 }
 
+FL_DEV void batch_tile(int tile, int num_m, int num_n, Raster rs, int& r, int& mb, int& nb) {
+  const int per = num_m * num_n;
+  r = tile / per;
+  tile_coords(tile - r * per, num_m, num_n, rs, mb, nb);
+}
+
 template <int BN, bool A_MN, bool B_MN, int FAM>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, Epi epi,
-                   int M, int N, int K, Raster raster, int* status) {
+    gemm_tc_kernel(const __grid_constant__ GemmMaps maps, Epi epi, int M, int N, int K, int batch, Raster raster,
+                   int* status) {
   using C = Cfg<BN>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -288,7 +310,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int lane = threadIdx.x & 31;
   const int num_m = (M + BM - 1) / BM;
   const int num_n = N / BN;
-  const int num_tiles = num_m * num_n;
+  const int num_tiles = batch * num_m * num_n;
   const int num_k = (K + BK - 1) / BK;
 
   if (threadIdx.x == 0) {
@@ -304,8 +326,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
+    for (int r = 0; r < batch; ++r) {
+      tma_prefetch_desc(&maps.a[r]);
+      tma_prefetch_desc(&maps.b[r]);
+    }
   }
   if (warp == 1) {
     tmem_alloc(tmem_holder, C::TMEM_COLS);
@@ -326,8 +350,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t armed = 0, last_par = 0;  // per-stage bit masks for the teardown drain
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        int mb, nb;
-        tile_coords(tile, num_m, num_n, raster, mb, nb);
+        int r, mb, nb;
+        batch_tile(tile, num_m, num_n, raster, r, mb, nb);
+        const CUtensorMap* tmA = &maps.a[r];
+        const CUtensorMap* tmB = &maps.b[r];
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1)) {
             report_status(status, FL_DEV_TIMEOUT_EMPTY);
@@ -341,16 +367,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           uint8_t* a_dst = sA + stage * C::A_BYTES;
           uint8_t* b_dst = sB + stage * C::B_BYTES;
           if (!A_MN) {
-            tma_load_2d(a_dst, &tmA, &full[stage], k0, mb * BM);
+            tma_load_2d(a_dst, tmA, &full[stage], k0, mb * BM);
           } else {
 #pragma unroll
-            for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * 64 * BK * 2, &tmA, &full[stage], mb * BM + 64 * j, k0);
+            for (int j = 0; j < BM / 64; ++j) tma_load_2d(a_dst + j * 64 * BK * 2, tmA, &full[stage], mb * BM + 64 * j, k0);
           }
           if (!B_MN) {
-            tma_load_2d(b_dst, &tmB, &full[stage], k0, nb * BN);
+            tma_load_2d(b_dst, tmB, &full[stage], k0, nb * BN);
           } else {
 #pragma unroll
-            for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 64 * BK * 2, &tmB, &full[stage], nb * BN + 64 * j, k0);
+            for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 64 * BK * 2, tmB, &full[stage], nb * BN + 64 * j, k0);
           }
           if (++stage == STAGES) {
             stage = 0;
@@ -419,8 +445,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     float4* my = reinterpret_cast<float4*>(stage + lane * 64);
     int local = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
-      int mb, nb;
-      tile_coords(tile, num_m, num_n, raster, mb, nb);
+      int r, mb, nb;
+      batch_tile(tile, num_m, num_n, raster, r, mb, nb);
       const int acc = local & 1;
       const uint32_t acc_par = (local >> 1) & 1;
       if (!mbar_wait(&acc_full[acc], acc_par)) {
@@ -450,7 +476,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                                   __uint_as_float(r1[4 * j + 2]), __uint_as_float(r1[4 * j + 3]));
         }
         __syncwarp();
-        if (rows > 0) epilogue_chunk<FAM>(epi, stage, row0, rows, nb * BN + c0, lane);
+        if (rows > 0) epilogue_chunk<FAM>(epi, r, stage, row0, rows, nb * BN + c0, lane);
         __syncwarp();
       }
     }
@@ -488,8 +514,8 @@ struct CfgPair {
 
 template <bool A_MN, bool B_MN, int FAM>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, Epi epi,
-                     int M, int N, int K, Raster raster, int* status) {
+    gemm_pair_kernel(const __grid_constant__ GemmMaps maps, Epi epi, int M, int N, int K, int batch, Raster raster,
+                     int* status) {
   using C = CfgPair;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -512,7 +538,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
   const int num_m = (M + PAIR_BM - 1) / PAIR_BM;
   const int num_n = N / PAIR_BN;
-  const int num_tiles = num_m * num_n;
+  const int num_tiles = batch * num_m * num_n;
   const int num_k = (K + BK - 1) / BK;
 
   if (threadIdx.x == 0) {
@@ -528,8 +554,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
+    for (int r = 0; r < batch; ++r) {
+      tma_prefetch_desc(&maps.a[r]);
+      tma_prefetch_desc(&maps.b[r]);
+    }
   }
   if (warp == 1) {
     tmem_alloc_pair(tmem_holder, C::TMEM_COLS);
@@ -551,8 +579,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t armed = 0, last_par = 0;  // per-stage bit masks for the teardown drain
       bool ok = true;
       for (int tile = pair; tile < num_tiles && ok; tile += n_pairs) {
-        int mb, nb;
-        tile_coords(tile, num_m, num_n, raster, mb, nb);
+        int r, mb, nb;
+        batch_tile(tile, num_m, num_n, raster, r, mb, nb);
+        const CUtensorMap* tmA = &maps.a[r];
+        const CUtensorMap* tmB = &maps.b[r];
         const int m0 = mb * PAIR_BM + int(rank) * 128, n0 = nb * PAIR_BN + int(rank) * 128;
         for (int kb = 0; kb < num_k; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1)) {
@@ -568,16 +598,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           uint8_t* a_dst = sA + stage * C::A_BYTES;
           uint8_t* b_dst = sB + stage * C::B_BYTES;
           if (!A_MN) {
-            tma_load_2d_pair(a_dst, &tmA, fb, k0, m0);
+            tma_load_2d_pair(a_dst, tmA, fb, k0, m0);
           } else {
-            tma_load_2d_pair(a_dst, &tmA, fb, m0, k0);
-            tma_load_2d_pair(a_dst + 64 * BK * 2, &tmA, fb, m0 + 64, k0);
+            tma_load_2d_pair(a_dst, tmA, fb, m0, k0);
+            tma_load_2d_pair(a_dst + 64 * BK * 2, tmA, fb, m0 + 64, k0);
           }
           if (!B_MN) {
-            tma_load_2d_pair(b_dst, &tmB, fb, k0, n0);
+            tma_load_2d_pair(b_dst, tmB, fb, k0, n0);
           } else {
-            tma_load_2d_pair(b_dst, &tmB, fb, n0, k0);
-            tma_load_2d_pair(b_dst + 64 * BK * 2, &tmB, fb, n0 + 64, k0);
+            tma_load_2d_pair(b_dst, tmB, fb, n0, k0);
+            tma_load_2d_pair(b_dst + 64 * BK * 2, tmB, fb, n0 + 64, k0);
           }
           if (++stage == STAGES) {
             stage = 0;
@@ -647,8 +677,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const uint32_t acc_empty0 = mapa_shared(smem_u32(acc_empty), 0);
     int local = 0;
     for (int tile = pair; tile < num_tiles; tile += n_pairs, ++local) {
-      int mb, nb;
-      tile_coords(tile, num_m, num_n, raster, mb, nb);
+      int r, mb, nb;
+      batch_tile(tile, num_m, num_n, raster, r, mb, nb);
       const int acc = local & 1;
       const uint32_t acc_par = (local >> 1) & 1;
       if (!mbar_wait(&acc_full[acc], acc_par)) {
@@ -678,7 +708,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                                   __uint_as_float(r1[4 * j + 2]), __uint_as_float(r1[4 * j + 3]));
         }
         __syncwarp();
-        if (rows > 0) epilogue_chunk<FAM>(epi, stage, row0, rows, nb * PAIR_BN + c0, lane);
+        if (rows > 0) epilogue_chunk<FAM>(epi, r, stage, row0, rows, nb * PAIR_BN + c0, lane);
         __syncwarp();
       }
     }
@@ -765,21 +795,26 @@ int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) 
     FL_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
     attr_set = true;
   }
-  CUtensorMap ta, tb;
-  int rc;
-  // A(m,k): K-major -> [M rows, K inner]; MN-major -> [K rows, M inner]
-  if (!A_MN) rc = make_map(&ta, a->A, a->K, a->M, a->lda, BM);
-  else rc = make_map(&ta, a->A, a->M, a->K, a->lda, BK);
-  if (rc) return rc;
-  if (!B_MN) rc = make_map(&tb, a->B, a->K, a->N, a->ldb, BN);
-  else rc = make_map(&tb, a->B, a->N, a->K, a->ldb, BK);
-  if (rc) return rc;
+  GemmMaps maps;
+  const int batch = a->batch > 1 ? a->batch : 1;
+  for (int r = 0; r < batch; ++r) {
+    const void* A = static_cast<const __nv_bfloat16*>(a->A) + r * a->a_bstride;
+    const void* B = static_cast<const __nv_bfloat16*>(a->B) + r * a->b_bstride;
+    int rc;
+    // A(m,k): K-major -> [M rows, K inner]; MN-major -> [K rows, M inner]
+    if (!A_MN) rc = make_map(&maps.a[r], A, a->K, a->M, a->lda, BM);
+    else rc = make_map(&maps.a[r], A, a->M, a->K, a->lda, BK);
+    if (rc) return rc;
+    if (!B_MN) rc = make_map(&maps.b[r], B, a->K, a->N, a->ldb, BN);
+    else rc = make_map(&maps.b[r], B, a->N, a->K, a->ldb, BK);
+    if (rc) return rc;
+  }
   const int num_m = (a->M + BM - 1) / BM, num_n = a->N / BN;
-  const int tiles = num_m * num_n;
+  const int tiles = batch * num_m * num_n;
   const int grid = tiles < num_sms() ? tiles : num_sms();
   const Raster r = pick_raster(a->M, a->N, a->K, BM, BN);
-  FL_CUDA_TRY(fl_launch(gemm_tc_kernel<BN, A_MN, B_MN, FAM>, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, st, ta, tb,
-                        epi, a->M, a->N, a->K, r, status));
+  FL_CUDA_TRY(fl_launch(gemm_tc_kernel<BN, A_MN, B_MN, FAM>, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, st, maps,
+                        epi, a->M, a->N, a->K, batch, r, status));
   return FL_OK;
 }
 
@@ -815,16 +850,21 @@ int launch_pair(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t
   auto kern = gemm_pair_kernel<A_MN, B_MN, FAM>;
   const int slots = pair_slots<A_MN, B_MN, FAM>();
   if (slots <= 0) return fl_internal_error(FL_ERR_CUDA, "gemm: the CTA-pair kernel cannot be resident");
-  CUtensorMap ta, tb;
-  int rc;
-  // each CTA loads 128 rows of A and 128 columns of B per k-block
-  if (!A_MN) rc = make_map(&ta, a->A, a->K, a->M, a->lda, 128);
-  else rc = make_map(&ta, a->A, a->M, a->K, a->lda, BK);
-  if (rc) return rc;
-  if (!B_MN) rc = make_map(&tb, a->B, a->K, a->N, a->ldb, 128);
-  else rc = make_map(&tb, a->B, a->N, a->K, a->ldb, BK);
-  if (rc) return rc;
-  const int tiles = ((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
+  GemmMaps maps;
+  const int batch = a->batch > 1 ? a->batch : 1;
+  for (int r = 0; r < batch; ++r) {
+    const void* A = static_cast<const __nv_bfloat16*>(a->A) + r * a->a_bstride;
+    const void* B = static_cast<const __nv_bfloat16*>(a->B) + r * a->b_bstride;
+    int rc;
+    // each CTA loads 128 rows of A and 128 columns of B per k-block
+    if (!A_MN) rc = make_map(&maps.a[r], A, a->K, a->M, a->lda, 128);
+    else rc = make_map(&maps.a[r], A, a->M, a->K, a->lda, BK);
+    if (rc) return rc;
+    if (!B_MN) rc = make_map(&maps.b[r], B, a->K, a->N, a->ldb, 128);
+    else rc = make_map(&maps.b[r], B, a->N, a->K, a->ldb, BK);
+    if (rc) return rc;
+  }
+  const int tiles = batch * ((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
   const int pairs = tiles < slots ? tiles : slots;
   const Raster r = pick_raster(a->M, a->N, a->K, PAIR_BM, PAIR_BN);
   cudaLaunchConfig_t cfg = {};
@@ -841,7 +881,7 @@ int launch_pair(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t
   cfg.stream = st;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  FL_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, ta, tb, epi, a->M, a->N, a->K, r, status));
+  FL_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, maps, epi, a->M, a->N, a->K, batch, r, status));
   return FL_OK;
 }
 

@@ -27,6 +27,7 @@ FL_T_COUNT = 14
 (FL_EPI_STORE, FL_EPI_BIAS_GELU, FL_EPI_BIAS_RESID, FL_EPI_BIAS_ROPE, FL_EPI_GELU_BWD, FL_EPI_RESID,
  FL_EPI_ACCUM_F32, FL_EPI_STORE_F32, FL_EPI_ADAMW) = range(9)
 FL_TILE_AUTO, FL_TILE_128x128, FL_TILE_128x256, FL_TILE_256x256_PAIR = range(4)
+FL_GEMM_MAX_BATCH = 4
 PROF_CLASSES = ("gemm", "attention", "layernorm", "adamw", "other")
 FL_DT_BF16, FL_DT_F32 = 0, 1
 
@@ -67,7 +68,11 @@ class fl_gemm_args(C.Structure):
                 ("ln_beta", C.c_void_p), ("adam_m", C.c_void_p), ("adam_v", C.c_void_p),
                 ("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float), ("eps", C.c_float),
                 ("weight_decay", C.c_float), ("inv_bc1", C.c_float), ("inv_bc2", C.c_float),
-                ("pos2", C.c_void_p), ("tile", C.c_int32), ("colsum", C.c_void_p)]
+                ("pos2", C.c_void_p), ("tile", C.c_int32), ("colsum", C.c_void_p),
+                ("batch", C.c_int32), ("a_bstride", C.c_int64), ("b_bstride", C.c_int64),
+                ("d_bstride", C.c_int64), ("aux_bstride", C.c_int64), ("aux_out_bstride", C.c_int64),
+                ("bias_bstride", C.c_int64), ("row_bstride", C.c_int64), ("lnp_bstride", C.c_int64),
+                ("adam_bstride", C.c_int64)]
 
 
 _P = C.c_void_p
@@ -420,13 +425,21 @@ def fl_k_gemm(args: fl_gemm_args, status=None, stream=None):
 def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
          alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
          aux_dtype=FL_DT_BF16, d_dtype=FL_DT_BF16, ln_mean=None, ln_rstd=None, ln_gamma=None, ln_beta=None,
-         pos2=None, tile=0, colsum=None, status=None, stream=None):
+         pos2=None, tile=0, colsum=None, status=None, stream=None, batch=1, bstrides=None, **fields):
+    """bstrides: {"a": .., "b": .., "d": .., "aux": .., "aux_out": .., "bias": .., "row": .., "lnp": ..,
+    "adam": ..} element strides between the problems of a batched launch; `fields` sets any
+    other fl_gemm_args field by name (tensors as device pointers)."""
     a = fl_gemm_args(M, N, K, ptr(A), lda, a_mn, ptr(B), ldb, b_mn, ptr(D), ldd, epilogue, ptr(bias), ptr(aux),
                      ld_aux, alpha, ptr(aux_out), ld_aux_out, ptr(pos), ptr(rope_tab), n_heads, head_dim, rotary_dim,
                      aux_dtype, d_dtype, ptr(ln_mean), ptr(ln_rstd), ptr(ln_gamma), ptr(ln_beta))
     a.pos2 = ptr(pos2)
     a.tile = tile
     a.colsum = ptr(colsum)
+    a.batch = batch
+    for k, v in (bstrides or {}).items():
+        setattr(a, f"{k}_bstride", int(v))
+    for k, v in fields.items():
+        setattr(a, k, v if isinstance(v, (int, float)) else ptr(v))
     fl_k_gemm(a, status, stream)
 
 
