@@ -85,6 +85,13 @@ typedef struct {
                              * 0 -> 4608 (the crossover measured on GB300: with fewer tokens
                              * the weight-gradient main loop is too short to hide the 26 B per
                              * parameter of the fused update); 1 -> always fused */
+  int32_t n_replicas;       /* server-hierarchical strategy (§3.3) on one GPU: 0 or 1 = one
+                             * server; 2..4 = that many replicas in one handle, each with its
+                             * own parameters, gradients and Adam state (arena of replica r at
+                             * r * the per-replica size), started from the same seeded values.
+                             * A call's K clients are split in order into n_replicas equal groups
+                             * of equal token counts, group r trained by replica r: the block GEMMs
+                             * of all replicas run as one batched launch each.  No prefix. */
 } fl_server_cfg;
 
 /* Fills *cfg with the ChatGLM-6B server defaults (26 blocks, H 4096, 32 x 128, F 16384,
@@ -189,7 +196,8 @@ int64_t fl_server_tensor_numel(fl_server_t h, int32_t tensor_id);
 
 /* Synchronous copies between a host fp32 buffer of exactly n elements and the fp32
  * master weights / accumulated gradients / Adam moments of (block, tensor_id).
- * set_param also refreshes the bf16 working copy.  Errors: INVALID_ARG (ids, n, null). */
+ * set_param also refreshes the bf16 working copy.  With cfg.n_replicas > 1 the getters read
+ * replica 0 and set_param writes every replica.  Errors: INVALID_ARG (ids, n, null). */
 int fl_server_get_param(fl_server_t h, int32_t block, int32_t tensor_id, float* host_dst, size_t n);
 int fl_server_set_param(fl_server_t h, int32_t block, int32_t tensor_id, const float* host_src, size_t n);
 int fl_server_get_grad(fl_server_t h, int32_t block, int32_t tensor_id, float* host_dst, size_t n);
@@ -208,7 +216,8 @@ int fl_server_average(fl_server_t const* replicas, int32_t n);
 
 /* Device address and element count of the fp32 master-weight arena, for averaging across
  * processes (one replica per GPU: all-reduce (sum) the arena, then call
- * fl_server_average_finish).  The arena is owned by the library. */
+ * fl_server_average_finish).  With cfg.n_replicas > 1 it spans every replica's arena.
+ * The arena is owned by the library. */
 int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n);
 
 /* Completes the §3.3 period-end average across processes: the caller has replaced this
@@ -217,6 +226,19 @@ int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n);
  * same bits either way), and refreshes the bf16 working copy, on the handle's stream.
  * Errors: INVALID_ARG (null, n_replicas < 1), STATE (a forward is pending), CUDA. */
 int fl_server_average_finish(fl_server_t h, int32_t n_replicas);
+
+/* The period-end average of the replicas of one handle (cfg.n_replicas > 1): every
+ * replica's fp32 master weights are replaced by their mean over the replicas (summed in
+ * replica order, scaled by 1/n as fl_server_average does) and the bf16 copies refreshed;
+ * Adam moments and the step count stay per replica.  Errors: INVALID_ARG (null handle),
+ * STATE (a forward is pending), CUDA. */
+int fl_server_average_replicas(fl_server_t h);
+
+/* fp32 master values of tensor_id of block `block` of replica `replica` (0 <=
+ * replica < cfg.n_replicas, or 0 with one replica) into host_dst[n] (n = the tensor's
+ * element count); fl_server_get_param reads replica 0. */
+int fl_server_get_replica_param(fl_server_t h, int32_t replica, int32_t block, int32_t tensor_id, float* host_dst,
+                                size_t n);
 
 /* Recomputes the bf16 working copy from the fp32 master weights (after they were changed
  * outside the library), on the handle's stream. */

@@ -37,7 +37,8 @@ typedef struct fl_client* fl_client_t;
 
 typedef struct {
   fl_server_cfg block; /* block shape, optimizer, prefix_len, freeze_base, client_batch (rows b per
-                          call), max_tokens (capacity b * L), max_seq_len; n_blocks is ignored */
+                          call), max_tokens (capacity b * L), max_seq_len; n_blocks is ignored;
+                          n_replicas must be 0 or 1 */
   int32_t vocab;       /* embedding and LM head rows (ChatGLM-6B: 130528) */
 } fl_client_cfg;
 

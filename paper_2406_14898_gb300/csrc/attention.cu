@@ -88,7 +88,7 @@ int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, int n_tiles128, float* delta,
                        const float* rope_tab, void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
-                       float* dbias, int* status) {
+                       float* dbias, int* status, int dbias_segs, int64_t dbias_rstride) {
   if (n_tiles <= 0) return FL_OK;
   if (hd != 64 && hd != 128) return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
   const int64_t pairs = (int64_t)T * nh;
@@ -100,7 +100,7 @@ int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, co
     FL_CUDA_TRY(fl_launch(attn_delta_kernel<64>, dim3((unsigned)((pairs * 8 + 255) / 256)), dim3(256), 0, st, T, H,
                           nh, (const bf16*)o, (const bf16*)dout, delta));
   return fl_launch_attn_bwd_tc(T, nh, hd, qkv, dout, lse, delta, cu, tiles + n_tiles, n_tiles128, rope_tab, dqkv, pre,
-                               glm, dbias, status, st);
+                               glm, dbias, status, st, dbias_segs, dbias_rstride);
 }
 
 // ====================================================================== exported kernel API

@@ -148,7 +148,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, int n_tiles, const float* __restrict__ lse,
     const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale, float scale_log2, int Lp,
     bf16* __restrict__ dqkv, float* __restrict__ dpk, float* __restrict__ dpv, const int32_t* __restrict__ ctxs,
-    const int32_t* __restrict__ gpos, const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int* status) {
+    const int32_t* __restrict__ gpos, const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int dbias_segs,
+    int64_t dbias_rstride, int* status) {
   constexpr int NB = BwdCfg<HD>::NB, TILE = BwdCfg<HD>::TILE, CH = BwdCfg<HD>::CH, E = BwdCfg<HD>::E;
   pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
   pdl_trigger();
@@ -180,6 +181,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   } else {
     // the 128-row tile list: (segment, tile), tile i standing for key tile nq - 1 - i
     const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
+    if (dbias && dbias_segs > 0) dbias += (int64_t)(s / dbias_segs) * dbias_rstride;  // the segment's replica
     seg0 = cu[s];
     L = cu[s + 1] - seg0;
     const int nq = (L + TB - 1) / TB;
@@ -449,7 +451,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, const float* __restrict__ lse,
     const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale, float scale_log2, int Lp,
     bf16* __restrict__ dqkv, const int32_t* __restrict__ ctxs, const int32_t* __restrict__ gpos,
-    const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int* status) {
+    const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int dbias_segs, int64_t dbias_rstride, int* status) {
   constexpr int NB = BwdCfg<HD>::NB, TILE = BwdCfg<HD>::TILE, CH = BwdCfg<HD>::CH, E = BwdCfg<HD>::E;
   pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
   pdl_trigger();
@@ -468,6 +470,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
 
   // the 128-row tile list: (segment, query tile)
   const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
+  if (dbias && dbias_segs > 0) dbias += (int64_t)(s / dbias_segs) * dbias_rstride;  // the segment's replica
   const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5;
   const int quarter = warp & 3, kh = warp >> 2;
@@ -671,7 +674,8 @@ int sm_count_bwd() {
 template <int HD>
 int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
                   const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab, void* dqkv,
-                  const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st) {
+                  const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st,
+                  int dbias_segs, int64_t dbias_rstride) {
   static bool attr = false;
   if (!attr) {
     FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dq_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -697,10 +701,11 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
   const float2* tab = reinterpret_cast<const float2*>(rope_tab);
   FL_CUDA_TRY(fl_launch(attn_bwd_dq_tc_kernel<HD>, dim3(n_tiles, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo, tpk,
                         tpv, T, H, cu, tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv, glm.ctx,
-                        glm.pos, glm.pos2, dbias, status));
+                        glm.pos, glm.pos2, dbias, dbias_segs, dbias_rstride, status));
   FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, false>, dim3(n_tiles, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo,
                         tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, 0, (bf16*)dqkv,
-                        (float*)nullptr, (float*)nullptr, glm.ctx, glm.pos, glm.pos2, dbias, status));
+                        (float*)nullptr, (float*)nullptr, glm.ctx, glm.pos, glm.pos2, dbias, dbias_segs, dbias_rstride,
+                        status));
   if (pre.len > 0) {
     // the prefix keys of each head against slices of the query tiles, about one CTA per SM
     int nsplit = (sm_count_bwd() + nh - 1) / nh;
@@ -708,7 +713,8 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
     if (nsplit < 1) nsplit = 1;
     FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, true>, dim3(nsplit, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq,
                           tdo, tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len,
-                          (bf16*)dqkv, pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2, (float*)nullptr, status));
+                          (bf16*)dqkv, pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2, (float*)nullptr, 0, (int64_t)0,
+                          status));
   }
   return FL_OK;
 }
@@ -718,12 +724,12 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
 int fl_launch_attn_bwd_tc(int T, int nh, int hd, const void* qkv, const void* dout, const float* lse,
                           const float* delta, const int32_t* cu, const uint32_t* tiles, int n_tiles,
                           const float* rope_tab, void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, float* dbias,
-                          int* status, cudaStream_t st) {
+                          int* status, cudaStream_t st, int dbias_segs, int64_t dbias_rstride) {
   if (hd == 128)
     return launch_bwd_tc<128>(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, pre, glm, dbias,
-                              status, st);
+                              status, st, dbias_segs, dbias_rstride);
   if (hd == 64)
     return launch_bwd_tc<64>(T, nh, qkv, dout, lse, delta, cu, tiles, n_tiles, rope_tab, dqkv, pre, glm, dbias,
-                             status, st);
+                             status, st, dbias_segs, dbias_rstride);
   return fl_internal_error(FL_ERR_UNSUPPORTED, "attention: head_dim %d", hd);
 }

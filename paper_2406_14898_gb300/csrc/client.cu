@@ -342,6 +342,9 @@ extern "C" int fl_client_create(const fl_client_cfg* cfg, uint64_t seed, fl_clie
   if (!cfg) return fl_internal_error(FL_ERR_INVALID_ARG, "client create: cfg is null");
   if (cfg->vocab < 1 || cfg->vocab >= (1 << 24))
     return fl_internal_error(FL_ERR_INVALID_ARG, "client create: vocab %d outside [1, 2^24)", cfg->vocab);
+  if (cfg->block.n_replicas > 1)
+    return fl_internal_error(FL_ERR_INVALID_ARG, "client create: block.n_replicas %d (a client has one replica)",
+                             cfg->block.n_replicas);
   fl_client* c = new fl_client();
   c->cfg = *cfg;
   c->cfg.block.n_blocks = 1;

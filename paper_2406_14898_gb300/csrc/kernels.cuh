@@ -94,19 +94,21 @@ int fl_launch_attn_fwd(int T, int nh, int hd, const void* qkv, const int32_t* cu
 int fl_launch_attn_fwd_tc(int T, int nh, int hd, const void* qkv, const int32_t* cu, const uint32_t* tiles,
                           int n_tiles, void* o, float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status,
                           cudaStream_t st);
-// dbias (or null): += the column sums of dqkv [3H] (the QKV bias gradient), per CTA.
+// dbias (or null): += the column sums of dqkv [3H] (the QKV bias gradient), per CTA; with
+// dbias_segs > 0 the sums of segment s go to dbias + (s / dbias_segs) * dbias_rstride (the
+// replicas of one handle, dbias_segs segments each).
 // delta: fp32 [nh, T] scratch (rowsum(dO * O), written here).
 int fl_launch_attn_bwd(int T, int nh, int hd, const void* qkv, const void* o, const float* lse, const void* dout,
                        const int32_t* cu, const uint32_t* tiles, int n_tiles, int n_tiles128, float* delta,
                        const float* rope_tab,
                        void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, cudaStream_t st,
-                       float* dbias = nullptr, int* status = nullptr);
+                       float* dbias = nullptr, int* status = nullptr, int dbias_segs = 0, int64_t dbias_rstride = 0);
 // dQ, dK / dV and, with a prefix, the prefix keys' gradients (attention_bwd_tc.cu); tiles:
 // the 128-row list alone; delta already computed.
 int fl_launch_attn_bwd_tc(int T, int nh, int hd, const void* qkv, const void* dout, const float* lse,
                           const float* delta, const int32_t* cu, const uint32_t* tiles, int n_tiles,
                           const float* rope_tab, void* dqkv, const AttnPrefix& pre, const AttnGlm& glm, float* dbias,
-                          int* status, cudaStream_t st);
+                          int* status, cudaStream_t st, int dbias_segs = 0, int64_t dbias_rstride = 0);
 
 // LayerNorm backward on fp32 dy / x (rowops.cu): fl_k_layernorm_bwd, and, when dcol is not
 // null, dcol += the column sums of dx.  workspace: fl_launch_layernorm_bwd_workspace bytes.

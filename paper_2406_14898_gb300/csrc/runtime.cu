@@ -11,7 +11,13 @@
 //                     every parameter: first the four weight matrices of every block
 //                     (block b at b * mat_stride), then the bias and LayerNorm vectors of
 //                     every block in one contiguous region (block b at vec_base +
-//                     b * vec_stride); every tensor 64-byte aligned;
+//                     b * vec_stride); every tensor 64-byte aligned; with cfg.n_replicas
+//                     = R > 1 each arena holds R such layouts back to back (replica r at
+//                     r * n_params), and replica r trains on the r-th of R equal, contiguous
+//                     token groups of each call (§3.3 server-hierarchical on one GPU): the
+//                     GEMMs of all replicas run as one batched launch, attention over
+//                     the whole packed batch (segments are independent), the LayerNorm
+//                     and vector kernels once per replica;
 //   activations       per block: LN1 out A, rotated QKV, attention O, LSE, residual stream
 //                     Hres (fp32), LN2 out M, FFN pre-activation U and GeLU output G, LN
 //                     statistics; xs[0..n_blocks]: block inputs / outputs in fp32
@@ -106,7 +112,9 @@ struct fl_server {
   int64_t tensor_off[FL_T_COUNT] = {};  // inside the block's matrix or vector slice
   int64_t tensor_n[FL_T_COUNT] = {};
   int64_t mat_stride = 0, vec_stride = 0, vec_base = 0, pre_stride = 0, pre_base = 0;
-  int64_t n_params = 0;  // padded total
+  int64_t n_params = 0;  // padded total of one replica
+  int R = 1;             // replicas in the handle (cfg.n_replicas, at least 1)
+  int64_t n_all() const { return R * n_params; }  // every replica's arena
   float *w = nullptr, *g = nullptr, *m = nullptr, *v = nullptr;
   __nv_bfloat16* wb = nullptr;
   int64_t step_t = 0;
@@ -141,6 +149,7 @@ struct fl_server {
   // pending step
   bool pending = false;
   int T = 0, S = 0, K = 0, n_tiles = 0, n_tiles128 = 0;
+  int Tr = 0, Sr = 0;  // tokens and segments of one replica's group (T and S with one replica)
   std::vector<int32_t> seq_lens;
 
   Prof prof;
@@ -174,9 +183,9 @@ struct fl_server {
     }
     return a;
   }
-  float* wt(int b, int t) { return w + off(b, t); }
-  float* gt(int b, int t) { return g + off(b, t); }
-  __nv_bfloat16* wbt(int b, int t) { return wb + off(b, t); }
+  float* wt(int b, int t, int r = 0) { return w + r * n_params + off(b, t); }
+  float* gt(int b, int t, int r = 0) { return g + r * n_params + off(b, t); }
+  __nv_bfloat16* wbt(int b, int t, int r = 0) { return wb + r * n_params + off(b, t); }
 };
 
 namespace {
@@ -254,11 +263,38 @@ int validate_cfg(const fl_server_cfg& c, int* rdim) {
   if (c.freeze_base && c.prefix_len == 0)
     return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: freeze_base needs a prefix (prefix_len > 0)");
   if (c.fused_step_min_tokens < 0) return fl_internal_error(FL_ERR_INVALID_ARG, "cfg: fused_step_min_tokens < 0");
+  if (c.n_replicas < 0 || c.n_replicas > FL_GEMM_MAX_BATCH)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: n_replicas in 0..%d", FL_GEMM_MAX_BATCH);
+  if (c.n_replicas > 1 && c.prefix_len > 0)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "cfg: n_replicas > 1 with a prefix");
   *rdim = rd;
   return FL_OK;
 }
 
-int run_gemm(fl_server* h, const fl_gemm_args& a) {
+// Launches one block GEMM; with R > 1 replicas one batched launch runs it for every replica:
+// problem r reads and writes replica r's Tr token rows and replica r's parameter arena.
+// A weight gradient (wgrad) contracts over the tokens: its A and B are token-major, its
+// output (gradient, or weight + Adam state + bf16 copy when fused) is a parameter.
+int run_gemm(fl_server* h, fl_gemm_args a, bool wgrad = false) {
+  if (h->R > 1) {
+    const int64_t P = h->n_params, Tr = h->Tr;
+    a.batch = h->R;
+    a.a_bstride = Tr * a.lda;
+    if (wgrad) {
+      a.b_bstride = Tr * a.ldb;
+      a.d_bstride = P;
+      a.adam_bstride = P;
+      a.aux_out_bstride = P;
+    } else {
+      a.b_bstride = P;
+      a.d_bstride = Tr * a.ldd;
+      a.aux_bstride = Tr * a.ld_aux;
+      a.aux_out_bstride = Tr * a.ld_aux_out;
+      a.bias_bstride = P;  // the bias, or the column sums of a bias gradient
+      a.row_bstride = Tr;  // positions, LayerNorm statistics
+      a.lnp_bstride = P;   // LayerNorm gain and shift
+    }
+  }
   prof_begin(h, FL_PROF_GEMM);
   int rc = fl_k_gemm(&a, h->status, h->stream);
   prof_end(h);
@@ -332,14 +368,17 @@ fl_gemm_args gemm_wgrad(fl_server* h, int b, int t, int T, int Nout, int Kin, co
 // xs[b + 1] is already kept and which the backward does not read, is skipped.
 int block_forward(fl_server* h, int b, bool output = true) {
   const fl_server_cfg& c = h->cfg;
-  const int T = h->T, H = c.hidden, F = c.ffn_hidden;
+  const int T = h->Tr, H = c.hidden, F = c.ffn_hidden;  // T: the token rows of one replica's GEMM
   BlockAct& A = h->act_of(b);
   const float* x = h->xs[b];
   cudaStream_t st = h->stream;
   // a = LN1(x)
-  prof_begin(h, FL_PROF_LN);
-  TRY(h, fl_launch_layernorm_fwd_f32(T, H, x, h->wt(b, FL_T_LN1_G), h->wt(b, FL_T_LN1_B), c.ln_eps,
-                                     (__nv_bfloat16*)A.a, A.mean1, A.rstd1, st, h->status));
+  prof_begin(h, FL_PROF_LN, h->R);
+  for (int r = 0; r < h->R; ++r) {
+    const int64_t r0 = (int64_t)r * T;
+    TRY(h, fl_launch_layernorm_fwd_f32(T, H, x + r0 * H, h->wt(b, FL_T_LN1_G, r), h->wt(b, FL_T_LN1_B, r), c.ln_eps,
+                                       (__nv_bfloat16*)A.a + r0 * H, A.mean1 + r0, A.rstd1 + r0, st, h->status));
+  }
   prof_end(h);
   // qkv = a Wqkv^T + bqkv, q and k rotated
   fl_gemm_args g1 = gemm_fwd(T, 3 * H, H, A.a, h->wbt(b, FL_T_WQKV), A.qkv, FL_EPI_BIAS_ROPE);
@@ -353,8 +392,8 @@ int block_forward(fl_server* h, int b, bool output = true) {
   TRY(h, run_gemm(h, g1));
   // o = causal attention within each segment
   prof_begin(h, FL_PROF_ATTN);
-  TRY(h, fl_launch_attn_fwd(T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, h->n_tiles128, A.o, A.lse,
-                            h->prefix(b, false), h->glm_args(), st, h->status));
+  TRY(h, fl_launch_attn_fwd(h->T, c.n_heads, c.head_dim, A.qkv, h->cu, h->tiles, h->n_tiles, h->n_tiles128, A.o,
+                            A.lse, h->prefix(b, false), h->glm_args(), st, h->status));
   prof_end(h);
   // h = alpha * (LN1(x) or x) + o Wd^T + bd, fp32; LN1(x) recomputed in fp32 in the epilogue
   fl_gemm_args g2 = gemm_fwd(T, H, H, A.o, h->wbt(b, FL_T_WDENSE), A.h, FL_EPI_BIAS_RESID);
@@ -372,9 +411,12 @@ int block_forward(fl_server* h, int b, bool output = true) {
   }
   TRY(h, run_gemm(h, g2));
   // m = LN2(h)
-  prof_begin(h, FL_PROF_LN);
-  TRY(h, fl_launch_layernorm_fwd_f32(T, H, A.h, h->wt(b, FL_T_LN2_G), h->wt(b, FL_T_LN2_B), c.ln_eps,
-                                     (__nv_bfloat16*)A.m, A.mean2, A.rstd2, st, h->status));
+  prof_begin(h, FL_PROF_LN, h->R);
+  for (int r = 0; r < h->R; ++r) {
+    const int64_t r0 = (int64_t)r * T;
+    TRY(h, fl_launch_layernorm_fwd_f32(T, H, A.h + r0 * H, h->wt(b, FL_T_LN2_G, r), h->wt(b, FL_T_LN2_B, r), c.ln_eps,
+                                       (__nv_bfloat16*)A.m + r0 * H, A.mean2 + r0, A.rstd2 + r0, st, h->status));
+  }
   prof_end(h);
   // u = m W1^T + b1, g = gelu(u)
   fl_gemm_args g3 = gemm_fwd(T, F, H, A.m, h->wbt(b, FL_T_WUP), A.g, FL_EPI_BIAS_GELU);
@@ -404,7 +446,7 @@ int block_forward(fl_server* h, int b, bool output = true) {
 // dy / dyf hold dL/dy of block b (bf16 and fp32); on return dx / dxf hold dL/dx.
 int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dyf, __nv_bfloat16* dx, float* dxf) {
   const fl_server_cfg& c = h->cfg;
-  const int T = h->T, H = c.hidden, F = c.ffn_hidden;
+  const int T = h->Tr, H = c.hidden, F = c.ffn_hidden;  // T: the token rows of one replica's GEMM
   const float al = c.residual_alpha;
   const bool glm = c.residual_from_ln != 0;
   BlockAct& A = h->act_of(b);
@@ -421,10 +463,10 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   d1.colsum = train_base ? h->gt(b, FL_T_BUP) : nullptr;
   TRY(h, run_gemm(h, d1));
   if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g)));
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g), true));
     if (b == c.n_blocks - 1) {
-      prof_begin(h, FL_PROF_OTHER);
-      TRY(h, fl_k_colsum(T, H, dy, h->gt(b, FL_T_BDOWN), st));
+      prof_begin(h, FL_PROF_OTHER, h->R);
+      for (int r = 0; r < h->R; ++r) TRY(h, fl_k_colsum(T, H, dy + (int64_t)r * T * H, h->gt(b, FL_T_BDOWN, r), st));
       prof_end(h);
     }
   }
@@ -439,23 +481,27 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   }
   TRY(h, run_gemm(h, d2));
   if (train_base)  // weight gradient (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m)));
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m), true));
   // LN2 backward: dh = LN2'(dm) (+ alpha dy), bf16 and fp32; dbd += colsum(dh)
-  prof_begin(h, FL_PROF_LN, 2);
-  TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->dm, A.h, A.mean2, A.rstd2, h->wt(b, FL_T_LN2_G), glm ? nullptr : dyf, al,
-                                     h->dh, h->dhf, h->gt(b, FL_T_LN2_G), h->gt(b, FL_T_LN2_B),
-                                     train_base ? h->gt(b, FL_T_BDENSE) : nullptr, h->ln_ws, st, h->status));
+  prof_begin(h, FL_PROF_LN, 2 * h->R);
+  for (int r = 0; r < h->R; ++r) {
+    const int64_t r0 = (int64_t)r * T, e0 = r0 * H;
+    TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->dm + e0, A.h + e0, A.mean2 + r0, A.rstd2 + r0,
+                                       h->wt(b, FL_T_LN2_G, r), glm ? nullptr : dyf + e0, al, h->dh + e0, h->dhf + e0,
+                                       h->gt(b, FL_T_LN2_G, r), h->gt(b, FL_T_LN2_B, r),
+                                       train_base ? h->gt(b, FL_T_BDENSE, r) : nullptr, h->ln_ws, st, h->status));
+  }
   prof_end(h);
   // dense: do = dh Wd; dWd += dh^T o
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
   if (train_base)  // weight gradient (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)));
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o), true));
   // attention backward -> dqkv (w.r.t. the un-rotated q, k); dbqkv += colsum(dqkv)
   prof_begin(h, FL_PROF_ATTN, 3);
-  TRY(h, fl_launch_attn_bwd(T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles,
-                            h->n_tiles128, h->delta,
-                            h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st,
-                            train_base ? h->gt(b, FL_T_BQKV) : nullptr, h->status));
+  TRY(h, fl_launch_attn_bwd(h->T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles,
+                            h->n_tiles128, h->delta, h->rope_tab, h->dqkv, h->prefix(b, true), h->glm_args(), st,
+                            train_base ? h->gt(b, FL_T_BQKV) : nullptr, h->status, h->R > 1 ? h->Sr : 0,
+                            h->n_params));
   prof_end(h);
   // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
@@ -468,14 +514,18 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   }
   TRY(h, run_gemm(h, d3));
   if (train_base)  // weight gradient (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a)));
+    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a), true));
   // LN1 backward: dx = LN1'(da) (+ alpha dh), bf16 and fp32; dx is dy of block b - 1, whose
   // down-projection bias gradient is its column sum
-  prof_begin(h, FL_PROF_LN, 2);
-  TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->da, h->xs[b], A.mean1, A.rstd1, h->wt(b, FL_T_LN1_G),
-                                     glm ? nullptr : h->dhf, al, dx, dxf, h->gt(b, FL_T_LN1_G), h->gt(b, FL_T_LN1_B),
-                                     train_base && b > 0 ? h->gt(b - 1, FL_T_BDOWN) : nullptr, h->ln_ws, st,
-                                     h->status));
+  prof_begin(h, FL_PROF_LN, 2 * h->R);
+  for (int r = 0; r < h->R; ++r) {
+    const int64_t r0 = (int64_t)r * T, e0 = r0 * H;
+    TRY(h, fl_launch_layernorm_bwd_f32(T, H, h->da + e0, h->xs[b] + e0, A.mean1 + r0, A.rstd1 + r0,
+                                       h->wt(b, FL_T_LN1_G, r), glm ? nullptr : h->dhf + e0, al, dx + e0, dxf + e0,
+                                       h->gt(b, FL_T_LN1_G, r), h->gt(b, FL_T_LN1_B, r),
+                                       train_base && b > 0 ? h->gt(b - 1, FL_T_BDOWN, r) : nullptr, h->ln_ws, st,
+                                       h->status));
+  }
   prof_end(h);
   return FL_OK;
 }
@@ -578,10 +628,11 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
   h->vec_base = moff * c.n_blocks;
   h->pre_base = h->vec_base + voff * c.n_blocks;
   h->n_params = h->pre_base + poff * c.n_blocks;
+  h->R = c.n_replicas > 1 ? c.n_replicas : 1;
+  const int64_t n_all = h->n_all();
   int rc;
-  if ((rc = dalloc(h, &h->w, h->n_params)) || (rc = dalloc(h, &h->g, h->n_params)) ||
-      (rc = dalloc(h, &h->m, h->n_params)) || (rc = dalloc(h, &h->v, h->n_params)) ||
-      (rc = dalloc(h, &h->wb, h->n_params)))
+  if ((rc = dalloc(h, &h->w, n_all)) || (rc = dalloc(h, &h->g, n_all)) || (rc = dalloc(h, &h->m, n_all)) ||
+      (rc = dalloc(h, &h->v, n_all)) || (rc = dalloc(h, &h->wb, n_all)))
     return fail(rc);
 
   // activations
@@ -622,10 +673,10 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
   if ((rc = dalloc(h, &h->rope_tab, tab.size()))) return fail(rc);
   cudaStream_t st = nullptr;
   if (cudaMemcpy(h->rope_tab, tab.data(), tab.size() * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess ||
-      cudaMemset(h->g, 0, h->n_params * sizeof(float)) != cudaSuccess ||
-      cudaMemset(h->m, 0, h->n_params * sizeof(float)) != cudaSuccess ||
-      cudaMemset(h->v, 0, h->n_params * sizeof(float)) != cudaSuccess ||
-      cudaMemset(h->w, 0, h->n_params * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->g, 0, n_all * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->m, 0, n_all * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->v, 0, n_all * sizeof(float)) != cudaSuccess ||
+      cudaMemset(h->w, 0, n_all * sizeof(float)) != cudaSuccess ||
       cudaMemset(h->status, 0, sizeof(int)) != cudaSuccess)
     return fail(fl_internal_cuda_error(cudaGetLastError(), "create: memset/copy", __FILE__, __LINE__));
 
@@ -641,7 +692,12 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
                                    (double)c.init_std, p, st);
       if (rc) return fail(rc);
     }
-  if ((rc = fl_launch_f32_to_bf16(h->n_params, h->w, h->wb, st))) return fail(rc);
+  // every replica starts from replica 0's values
+  for (int r = 1; r < h->R; ++r)
+    if (cudaMemcpyAsync(h->w + r * h->n_params, h->w, h->n_params * sizeof(float), cudaMemcpyDeviceToDevice, st) !=
+        cudaSuccess)
+      return fail(fl_internal_cuda_error(cudaGetLastError(), "create: replica copy", __FILE__, __LINE__));
+  if ((rc = fl_launch_f32_to_bf16(n_all, h->w, h->wb, st))) return fail(rc);
   if (cudaDeviceSynchronize() != cudaSuccess)
     return fail(fl_internal_cuda_error(cudaGetLastError(), "create: init", __FILE__, __LINE__));
   *out = h;
@@ -668,6 +724,19 @@ static int forward_impl(fl_server_t h, const void* const client_states[], const 
   if (T > c.max_tokens) return set_err(h, FL_ERR_CAPACITY, "forward: %lld tokens > max_tokens %d", (long long)T, c.max_tokens);
   const int64_t S = (int64_t)K * b;
   if (S > FL_MAX_SEGS) return set_err(h, FL_ERR_CAPACITY, "forward: %lld segments > %d", (long long)S, FL_MAX_SEGS);
+  // replicas: clients [r K/R, (r+1) K/R) are replica r's group; every group the same tokens
+  const int R = h->R;
+  if (K % R) return set_err(h, FL_ERR_INVALID_ARG, "forward: K=%d is not a multiple of n_replicas %d", K, R);
+  int64_t Tr = T;
+  if (R > 1) {
+    std::vector<int64_t> group(R, 0);
+    for (int k = 0; k < K; ++k) group[k / (K / R)] += (int64_t)b * seq_lens[k];
+    for (int r = 1; r < R; ++r)
+      if (group[r] != group[0])
+        return set_err(h, FL_ERR_INVALID_ARG, "forward: replica %d's clients hold %lld tokens, replica 0's %lld", r,
+                       (long long)group[r], (long long)group[0]);
+    Tr = group[0];
+  }
 
   // packing metadata: client k row r is segment k*b + r
   static thread_local MetaArgs meta;
@@ -697,6 +766,8 @@ static int forward_impl(fl_server_t h, const void* const client_states[], const 
   meta.n_tiles128 = nt128;
   h->T = (int)T;
   h->S = (int)S;
+  h->Tr = (int)Tr;
+  h->Sr = (int)(S / R);
   h->K = K;
   h->n_tiles = nt;
   h->n_tiles128 = nt128;
@@ -739,8 +810,12 @@ static int backward_impl(fl_server_t h, const void* const grad_out[], void* cons
   int rc;
   if (h->grads_zero) {
     // bias and LayerNorm gradients accumulate (+=); one memset of their contiguous region
-    const cudaError_t e = cudaMemsetAsync(h->g + h->vec_base, 0, (h->n_params - h->vec_base) * sizeof(float), h->stream);
-    if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "cudaMemsetAsync", __FILE__, __LINE__));
+    // (per replica)
+    for (int r = 0; r < h->R; ++r) {
+      const cudaError_t e = cudaMemsetAsync(h->g + r * h->n_params + h->vec_base, 0,
+                                            (h->n_params - h->vec_base) * sizeof(float), h->stream);
+      if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "cudaMemsetAsync", __FILE__, __LINE__));
+    }
   }
   if ((rc = copy_clients(h, grad_out, COPY_GATHER_F32, h->dy, h->dyf))) return rc;
   __nv_bfloat16* cur = h->dy;
@@ -772,7 +847,7 @@ extern "C" int fl_server_backward_step(fl_server_t h, const void* const grad_out
   // no fusion while gradients from an earlier backward are pending, nor for calls too
   // short for the weight-gradient main loop to hide the update
   const int min_tokens = h->cfg.fused_step_min_tokens > 0 ? h->cfg.fused_step_min_tokens : FL_FUSED_STEP_MIN_TOKENS;
-  if (!h->grads_zero || h->T < min_tokens) {
+  if (!h->grads_zero || h->Tr < min_tokens) {
     if (int rc = backward_impl(h, grad_out, grad_in)) return rc;
     return fl_server_step(h, lr);
   }
@@ -789,12 +864,16 @@ extern "C" int fl_server_backward_step(fl_server_t h, const void* const grad_out
   h->step_t = t;
   // the bias / LayerNorm vectors and the prefixes (only the prefixes with a frozen base):
   // one AdamW launch over their contiguous region
+  // (per replica)
   const int64_t first = c.freeze_base ? h->pre_base : h->vec_base;
-  prof_begin(h, FL_PROF_ADAMW);
-  rc = fl_launch_adamw(h->n_params - first, h->w + first, h->g + first, h->m + first,
-                       h->v + first, h->wb + first, lr, c.adam_beta1, c.adam_beta2, c.adam_eps,
-                       c.weight_decay, (float)(1.0 - std::pow((double)c.adam_beta1, (double)t)),
-                       (float)(1.0 - std::pow((double)c.adam_beta2, (double)t)), 0, h->stream);
+  prof_begin(h, FL_PROF_ADAMW, h->R);
+  for (int r = 0; r < h->R && rc == FL_OK; ++r) {
+    const int64_t o = r * h->n_params + first;
+    rc = fl_launch_adamw(h->n_params - first, h->w + o, h->g + o, h->m + o, h->v + o, h->wb + o, lr, c.adam_beta1,
+                         c.adam_beta2, c.adam_eps, c.weight_decay,
+                         (float)(1.0 - std::pow((double)c.adam_beta1, (double)t)),
+                         (float)(1.0 - std::pow((double)c.adam_beta2, (double)t)), 0, h->stream);
+  }
   prof_end(h);
   if (rc) return fwd_err(h, rc);
   h->grads_zero = true;  // matrix gradients were never written; vectors are cleared by the next backward
@@ -810,9 +889,10 @@ extern "C" int fl_server_step(fl_server_t h, float lr) {
   const double bc2 = 1.0 - std::pow((double)c.adam_beta2, (double)h->step_t);
   prof_begin(h, FL_PROF_ADAMW);
   // the gradients are not cleared here: the next backward overwrites them (grads_zero);
-  // with a frozen base only the prefix region is updated
+  // with a frozen base only the prefix region is updated (there is one replica then); with
+  // replicas one launch covers every replica's arena
   const int64_t first = c.freeze_base ? h->pre_base : 0;
-  int rc = fl_launch_adamw(h->n_params - first, h->w + first, h->g + first, h->m + first, h->v + first, h->wb + first,
+  int rc = fl_launch_adamw(h->n_all() - first, h->w + first, h->g + first, h->m + first, h->v + first, h->wb + first,
                            lr, c.adam_beta1, c.adam_beta2, c.adam_eps, c.weight_decay, (float)bc1, (float)bc2, 0,
                            h->stream);
   prof_end(h);
@@ -890,12 +970,20 @@ extern "C" int fl_server_get_adam_moments(fl_server_t h, int32_t b, int32_t t, f
   if (int rc = d2h(h, hm, h->m + o, n)) return rc;
   return d2h(h, hv, h->v + o, n);
 }
+extern "C" int fl_server_get_replica_param(fl_server_t h, int32_t r, int32_t b, int32_t t, float* dst, size_t n) {
+  if (int rc = check_tensor(h, b, t, dst, n)) return rc;
+  if (r < 0 || r >= h->R) return set_err(h, FL_ERR_INVALID_ARG, "replica %d outside [0, %d)", r, h->R);
+  return d2h(h, dst, h->wt(b, t, r), n);
+}
 extern "C" int fl_server_set_param(fl_server_t h, int32_t b, int32_t t, const float* src, size_t n) {
   if (int rc = check_tensor(h, b, t, src, n)) return rc;
   cudaError_t e = cudaStreamSynchronize(h->stream);
-  if (e == cudaSuccess) e = cudaMemcpy(h->wt(b, t), src, n * sizeof(float), cudaMemcpyHostToDevice);
+  for (int r = 0; r < h->R && e == cudaSuccess; ++r)  // every replica
+    e = cudaMemcpy(h->wt(b, t, r), src, n * sizeof(float), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "host to device copy", __FILE__, __LINE__));
-  int rc = fl_launch_f32_to_bf16((int64_t)n, h->wt(b, t), h->wbt(b, t), h->stream);
+  int rc = FL_OK;
+  for (int r = 0; r < h->R && rc == FL_OK; ++r)
+    rc = fl_launch_f32_to_bf16((int64_t)n, h->wt(b, t, r), h->wbt(b, t, r), h->stream);
   if (rc) return fwd_err(h, rc);
   e = cudaStreamSynchronize(h->stream);
   if (e != cudaSuccess) return fwd_err(h, fl_internal_cuda_error(e, "set_param", __FILE__, __LINE__));
@@ -913,8 +1001,8 @@ extern "C" int fl_server_average(fl_server_t const* replicas, int32_t n) {
   for (int r = 0; r < n; ++r) {
     fl_server* h = replicas[r];
     if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "average: null replica %d", r);
-    if (h->n_params != h0->n_params || h->cfg.n_blocks != h0->cfg.n_blocks || h->cfg.hidden != h0->cfg.hidden ||
-        h->cfg.ffn_hidden != h0->cfg.ffn_hidden)
+    if (h->n_params != h0->n_params || h->R != h0->R || h->cfg.n_blocks != h0->cfg.n_blocks ||
+        h->cfg.hidden != h0->cfg.hidden || h->cfg.ffn_hidden != h0->cfg.ffn_hidden)
       return fl_internal_error(FL_ERR_INVALID_ARG, "average: replica %d has another shape", r);
     if (h->pending) return set_err(h, FL_ERR_STATE, "average: replica %d has a pending forward", r);
     for (int q = 0; q < r; ++q)
@@ -928,7 +1016,7 @@ extern "C" int fl_server_average(fl_server_t const* replicas, int32_t n) {
     if (e != cudaSuccess) return fwd_err(h0, fl_internal_cuda_error(e, "average: sync", __FILE__, __LINE__));
   }
   prof_begin(h0, FL_PROF_OTHER);
-  int rc = fl_launch_average(t, h0->n_params, h0->stream);
+  int rc = fl_launch_average(t, h0->n_all(), h0->stream);
   prof_end(h0);
   if (rc) return fwd_err(h0, rc);
   cudaError_t e = cudaStreamSynchronize(h0->stream);
@@ -939,7 +1027,7 @@ extern "C" int fl_server_average(fl_server_t const* replicas, int32_t n) {
 extern "C" int fl_server_param_arena(fl_server_t h, float** dev_w, int64_t* n) {
   if (!h || !dev_w || !n) return fl_internal_error(FL_ERR_INVALID_ARG, "param_arena: null");
   *dev_w = h->w;
-  *n = h->n_params;
+  *n = h->n_all();
   return FL_OK;
 }
 
@@ -948,14 +1036,31 @@ extern "C" int fl_server_average_finish(fl_server_t h, int32_t n_replicas) {
   if (n_replicas < 1) return set_err(h, FL_ERR_INVALID_ARG, "average finish: n_replicas=%d < 1", n_replicas);
   if (h->pending) return set_err(h, FL_ERR_STATE, "average finish: a forward is pending");
   prof_begin(h, FL_PROF_OTHER);
-  int rc = fl_launch_mean_finish(h->n_params, n_replicas, h->w, h->wb, h->stream);
+  int rc = fl_launch_mean_finish(h->n_all(), n_replicas, h->w, h->wb, h->stream);
+  prof_end(h);
+  return fwd_err(h, rc);
+}
+
+extern "C" int fl_server_average_replicas(fl_server_t h) {
+  if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "average replicas: null handle");
+  if (h->pending) return set_err(h, FL_ERR_STATE, "average replicas: a forward is pending");
+  if (h->R < 2) return FL_OK;
+  ReplicaTable t;
+  memset(&t, 0, sizeof t);
+  t.n = h->R;
+  for (int r = 0; r < h->R; ++r) {
+    t.w[r] = h->w + r * h->n_params;
+    t.wb[r] = h->wb + r * h->n_params;
+  }
+  prof_begin(h, FL_PROF_OTHER);
+  int rc = fl_launch_average(t, h->n_params, h->stream);
   prof_end(h);
   return fwd_err(h, rc);
 }
 
 extern "C" int fl_server_refresh_working_copy(fl_server_t h) {
   if (!h) return fl_internal_error(FL_ERR_INVALID_ARG, "refresh: null handle");
-  int rc = fl_launch_f32_to_bf16(h->n_params, h->w, h->wb, h->stream);
+  int rc = fl_launch_f32_to_bf16(h->n_all(), h->w, h->wb, h->stream);
   return fwd_err(h, rc);
 }
 

@@ -45,7 +45,8 @@ class fl_server_cfg(C.Structure):
                 ("client_batch", C.c_int32), ("max_tokens", C.c_int32), ("max_seq_len", C.c_int32),
                 ("recompute", C.c_int32), ("init_std", C.c_float), ("adam_beta1", C.c_float),
                 ("adam_beta2", C.c_float), ("adam_eps", C.c_float), ("weight_decay", C.c_float),
-                ("prefix_len", C.c_int32), ("freeze_base", C.c_int32), ("fused_step_min_tokens", C.c_int32)]
+                ("prefix_len", C.c_int32), ("freeze_base", C.c_int32), ("fused_step_min_tokens", C.c_int32),
+                ("n_replicas", C.c_int32)]
 
 
 class fl_client_cfg(C.Structure):
@@ -99,6 +100,8 @@ _SIGS = {
     "fl_server_param_arena": (C.c_int, [_P, C.POINTER(_P), C.POINTER(_I64)]),
     "fl_server_refresh_working_copy": (C.c_int, [_P]),
     "fl_server_average_finish": (C.c_int, [_P, _I32]),
+    "fl_server_average_replicas": (C.c_int, [_P]),
+    "fl_server_get_replica_param": (C.c_int, [_P, _I32, _I32, _I32, _P, C.c_size_t]),
     "fl_server_profile": (C.c_int, [_P, C.c_int]),
     "fl_server_profile_read": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(_I64), _I32]),
     "fl_server_launch_count": (_I64, [_P]),
@@ -181,11 +184,12 @@ def _parr(xs) -> "C.Array":
 
 
 def make_cfg(c, max_tokens: int, max_seq_len: int = 0, recompute: int = 0,
-             fused_step_min_tokens: int = 0) -> fl_server_cfg:
+             fused_step_min_tokens: int = 0, n_replicas: int = 0) -> fl_server_cfg:
     """fl_server_cfg from a workload description with the attributes of
     ``synthetic.ServerConfig`` (n_blocks, hidden, ... , weight_decay); ``recompute``
     keeps one block's activations and recomputes the rest in the backward;
-    ``fused_step_min_tokens`` as in fl_server_cfg (0: the library's crossover)."""
+    ``fused_step_min_tokens`` as in fl_server_cfg (0: the library's crossover);
+    ``n_replicas`` > 1 holds that many server replicas in the handle (§3.3)."""
     cfg = fl_server_cfg()
     lib().fl_server_cfg_default(C.byref(cfg))
     cfg.n_blocks = c.n_blocks
@@ -210,6 +214,7 @@ def make_cfg(c, max_tokens: int, max_seq_len: int = 0, recompute: int = 0,
     cfg.prefix_len = getattr(c, "prefix_len", 0)
     cfg.freeze_base = getattr(c, "freeze_base", 0)
     cfg.fused_step_min_tokens = fused_step_min_tokens
+    cfg.n_replicas = n_replicas
     return cfg
 
 
@@ -276,6 +281,12 @@ class Server:
     def get_param(self, block: int, tensor_id: int):
         return self._get(lib().fl_server_get_param, block, tensor_id)
 
+    def get_replica_param(self, replica: int, block: int, tensor_id: int):
+        import numpy as np
+        out = np.empty(self.numel(tensor_id), np.float32)
+        check(lib().fl_server_get_replica_param(self.h, replica, block, tensor_id, out.ctypes.data, out.size), self.h)
+        return out
+
     def get_grad(self, block: int, tensor_id: int):
         return self._get(lib().fl_server_get_grad, block, tensor_id)
 
@@ -304,6 +315,10 @@ class Server:
 
     def average_finish(self, n_replicas: int):
         check(lib().fl_server_average_finish(self.h, n_replicas), self.h)
+
+    def average_replicas(self):
+        """The §3.3 period-end average of the replicas held in this handle."""
+        check(lib().fl_server_average_replicas(self.h), self.h)
 
     def profile(self, enable: bool):
         check(lib().fl_server_profile(self.h, 1 if enable else 0), self.h)

@@ -1,11 +1,15 @@
 """Server-hierarchical training (§3.3 of the paper): one server replica per client, the
 replicas trained side by side and their parameters averaged at the end of every period.
 
-On one GPU the replicas are independent fl_server handles, each on its own CUDA stream, so
-their kernels can overlap; fl_server_average forms the mean on the device.  Across GPUs
-(one replica per rank) the mean is an all-reduce (sum) of each replica's fp32 master-weight
-arena, then fl_server_average_finish scales it by 1/ranks and refreshes the bf16 working
-copy.  All arithmetic runs in the CUDA library or in the collective; this module only
+On one GPU the replicas are either independent fl_server handles, each on its own CUDA
+stream, averaged by fl_server_average (HierarchicalServers), or up to four replicas held in
+one handle (cfg.n_replicas), whose block GEMMs run as one batched launch per GEMM and which
+fl_server_average_replicas averages (BatchedReplicas; every replica's clients must hold the
+same number of tokens).  Across GPUs (replicas on every rank) the mean is the in-handle
+mean, then an all-reduce (sum) of each rank's fp32 master-weight arena, then
+fl_server_average_finish scales it by 1/ranks and refreshes the bf16 working copy (with an
+equal number of replicas on every rank, the mean of the ranks' means is the mean over all
+replicas).  All arithmetic runs in the CUDA library or in the collective; this module only
 orders the calls.
 """
 from __future__ import annotations
@@ -38,12 +42,14 @@ def allreduce_sum_(tensor, group=None):
 
 
 def average_across_ranks(server, group=None, arena=None):
-    """Period-end averaging with one replica per rank: all-reduce (sum) of the master
-    weights, then the library scales the sum by 1/ranks and refreshes the bf16 working copy.
-    `arena` (default: the server's master arena as a CUDA tensor) is the buffer the
-    collective sums."""
+    """Period-end averaging with the replicas of `server` on every rank: the replicas held in
+    the handle are averaged first (nothing to do with one), then the master weights are
+    all-reduced (sum) and the library scales the sum by 1/ranks and refreshes the bf16
+    working copy.  `arena` (default: the server's master arena as a CUDA tensor) is the
+    buffer the collective sums."""
     import torch
     import torch.distributed as dist
+    server.average_replicas()
     server.sync()
     w = arena_tensor(server) if arena is None else arena
     allreduce_sum_(w, group)
@@ -82,3 +88,34 @@ class HierarchicalServers:
         for srv in self.replicas:
             srv.close()
         self.replicas = []
+
+
+class BatchedReplicas:
+    """n_replicas (2..4) server replicas in one handle: a call's K clients are split in
+    order into n_replicas groups holding the same number of tokens, group r trained by
+    replica r; every block GEMM of all replicas is one batched launch."""
+
+    def __init__(self, cfg: F.fl_server_cfg, seed: int, n_replicas: int, stream=None):
+        c = F.fl_server_cfg.from_buffer_copy(cfg)
+        c.n_replicas = n_replicas
+        self.n_replicas = n_replicas
+        # every replica starts from the same parameters, as after an averaging
+        self.server = F.Server(c, seed, stream=stream)
+
+    def step(self, client_states: Sequence, seq_lens: Sequence[int], out_states: Sequence, grad_out: Sequence,
+             grad_in: Sequence, lr: float):
+        """One training step of every replica on its group of clients."""
+        self.server.forward(client_states, seq_lens, out_states)
+        self.server.backward_step(grad_out, grad_in, lr)
+
+    def average(self):
+        self.server.average_replicas()
+
+    def get_param(self, replica: int, block: int, tensor_id: int):
+        return self.server.get_replica_param(replica, block, tensor_id)
+
+    def sync(self):
+        self.server.sync()
+
+    def close(self):
+        self.server.close()
