@@ -672,7 +672,7 @@ def run_strategies(args, K: int):
     clients one call after another, one update)."""
     import torch
     from paper_2406_14898_gb300 import flglm as F
-    from paper_2406_14898_gb300.hierarchical import HierarchicalServers
+    from paper_2406_14898_gb300.hierarchical import BatchedReplicas, HierarchicalServers
 
     cfg = syn.sweep_config(K)
     one = cfg.with_(seq_lens=cfg.seq_lens[:1])
@@ -711,6 +711,21 @@ def run_strategies(args, K: int):
     res["server_hierarchical"] = {"replicas": K, "ms_per_step": ms, "average_ms": avg_ms, "period": args.period,
                                   "tokens_per_s": cfg.tokens / (amort / 1e3),
                                   "pct_bf16_peak": 100.0 * flops / (amort / 1e3) / (pk["bf16_sustained"] * 1e12)}
+    # the same K replicas held in one handle, every block GEMM one batched launch
+    if 2 <= K <= F.FL_GEMM_MAX_BATCH:
+        br = BatchedReplicas(F.make_cfg(cfg, cfg.tokens, 512), cfg.seed, K)
+        ms = timed(lambda: br.step(st, cfg.seq_lens, outs, go, gin, cfg.lr), br.sync)
+        t0 = time.perf_counter()
+        br.average()
+        br.sync()
+        avg_ms = 1e3 * (time.perf_counter() - t0)
+        br.close()
+        torch.cuda.empty_cache()
+        amort = ms + avg_ms / args.period
+        res["server_hierarchical_batched"] = {
+            "replicas": K, "ms_per_step": ms, "average_ms": avg_ms, "period": args.period,
+            "tokens_per_s": cfg.tokens / (amort / 1e3),
+            "pct_bf16_peak": 100.0 * flops / (amort / 1e3) / (pk["bf16_sustained"] * 1e12)}
     # client-batch and serial on one server
     srv = F.Server(F.make_cfg(cfg, cfg.tokens, 512), cfg.seed)
 
