@@ -177,7 +177,8 @@ int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, const void*
  * context_lens: as in the forward.  positions / block_positions: device int32 [T] or NULL;
  * the inverse rotation of dims [0, head_dim/2) uses positions[t] (NULL: the index inside
  * the segment) and, when block_positions != NULL, dims [head_dim/2, head_dim) turn back by
- * block_positions[t] (GLM 2D rotary).  Every position must be below the rows of rope_tab. */
+ * block_positions[t] (GLM 2D rotary).  Every position must be below the rows of rope_tab,
+ * and rope_tab 16-byte aligned (INVALID_ARG otherwise). */
 int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, const void* qkv, const void* o,
                        const float* lse, const void* dout, const int32_t* cu_seqlens_host,
                        const int32_t* cu_seqlens, int32_t S, int32_t* tile_ws, float* delta_ws,

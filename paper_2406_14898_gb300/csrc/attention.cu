@@ -163,6 +163,8 @@ extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: cu_seqlens");
   if (rope_tab && rotary_dim != head_dim / 2)
     return fl_internal_error(FL_ERR_UNSUPPORTED, "attention bwd: rotary_dim must be head_dim / 2");
+  if (rope_tab && (reinterpret_cast<uintptr_t>(rope_tab) & 15))  // rows are read as 16-byte vectors
+    return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: rope_tab is not 16-byte aligned");
   if (prefix_len < 0 || prefix_len > 128 ||
       (prefix_len > 0 && (!prefix_k || !prefix_v || !dprefix_k || !dprefix_v)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: prefix (length 0..128, gradients required)");

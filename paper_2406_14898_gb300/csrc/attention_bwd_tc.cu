@@ -10,9 +10,15 @@
 // double-buffer the tiles the CTA walks through, so their loads overlap the work on the
 // previous tile.
 //
-// dK / dV: one CTA (8 warps) per (128-key tile, head).  Warp w reads TMEM lanes
-// 32 (w % 4) .. + 31, so thread (w, lane) owns key row r = 32 (w % 4) + lane, and takes
-// query half w / 4 of every query tile.  Per 128-query tile i that sees the key tile:
+// Both kernels are persistent: one CTA per SM (192 KB of shared memory at head_dim 128,
+// 512 TMEM columns) walks work units u = blockIdx.x, + gridDim.x, ...  Once a unit's last
+// product has completed, the next unit's first tiles are loaded into buffer pair 0 while
+// the unit's output is staged in buffer pair 1 and written; the next unit's pair-1 tiles
+// follow once the staged rows have been read.
+//
+// dK / dV: unit = (128-key tile, head).  Warp w reads TMEM lanes 32 (w % 4) .. + 31, so
+// thread (w, lane) owns key row r = 32 (w % 4) + lane, and takes query half w / 4 of every
+// query tile.  Per 128-query tile i that sees the key tile:
 //   TMA: Q_i and dO_i into the buffer pair (i % 2), the next tile's while this one works;
 //   S^T = K Q_i^T -> TMEM [0, 128)      dP^T = V dO_i^T -> TMEM [128, 256);
 //   threads: P^T = exp2(S^T scale log2e - lse_q log2e) where key r is visible to query q,
@@ -20,13 +26,13 @@
 //   dV += P^T dO_i -> TMEM [256, 256 + hd)   dK += dS^T Q_i -> TMEM [256 + hd, 256 + 2 hd)
 //            (A from TMEM, dO_i and Q_i as MN-major operands).
 // Epilogue: dK * scale, the inverse rotary rotation(s), bf16 rows of dqkv and the k / v
-// column sums for the QKV bias gradient; the prefix variant (PREFIX: the CTA's keys are
-// the prefix, its query tiles a slice of the call's tile list) adds dK * scale and dV into
-// the fp32 prefix gradients instead.
+// column sums for the QKV bias gradient; the prefix variant (PREFIX: the unit's keys are
+// the prefix of its head, its query tiles a slice of the call's tile list) adds dK * scale
+// and dV into the fp32 prefix gradients instead.
 //
-// dQ: one CTA (8 warps) per (128-query tile, head); thread (w, lane) owns query row
-// r = 32 (w % 4) + lane and key half w / 4 of every key tile.  Per key tile j (the prefix
-// tile first, then the segment's own keys), K_j / V_j double-buffered:
+// dQ: unit = (128-query tile, head); thread (w, lane) owns query row r = 32 (w % 4) + lane
+// and key half w / 4 of every key tile.  Per key tile j (the prefix tile first, then the
+// segment's own keys), K_j / V_j double-buffered:
 //   S = Q K_j^T -> TMEM [0, 128), dP = dO V_j^T -> TMEM [128, 256);
 //   threads: dS = P (dP - delta_q), P = exp2(S scale log2e - lse_q log2e) on the visible
 //            keys, bf16 over the S values just read;
@@ -34,9 +40,8 @@
 // Epilogue as in dK / dV: dQ * scale, inverse rotary rotation(s), coalesced bf16 rows, q
 // column sums.
 //
-// Both kernels take 192 KB of shared memory (head_dim 128) and 512 TMEM columns: one CTA
-// per SM.  Every mbarrier wait is bounded (2 s): on expiry the CTA records a status code
-// and leaves its remaining work undone.
+// Every mbarrier wait is bounded (2 s): on expiry the CTA records a status code, lets what
+// it armed land and leaves its remaining work undone.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -77,17 +82,22 @@ FL_DEV uint64_t desc_mn(uint32_t base, int kk) { return smem_desc_sw128(base + k
 FL_DEV uint32_t a_col(int kk) { return (kk >> 2) * 64 + ((kk >> 1) & 1) * 16 + (kk & 1) * 8; }
 
 // Inverse rotary rotation of one rotary region held by a thread: HD/2 consecutive dims,
-// pairs (i, i + HD/4), angle (cos, sin) of pair i at tr[i ^ sw] (a row of the rotary table
-// staged in shared memory, entries XOR-swizzled by the row).
+// pairs (i, i + HD/4), angle (cos, sin) of pair i at row[i] (the row of the rotary table
+// for the token's position, read from global memory: the table is small and L2-resident).
 template <int HD>
-FL_DEV void inverse_rope_row(float* v, const float2* tr, int sw) {
+FL_DEV void inverse_rope_row(float* v, const float2* __restrict__ row) {
   constexpr int Q = HD / 4;
+  const float4* r4 = reinterpret_cast<const float4*>(row);
 #pragma unroll
-  for (int i = 0; i < Q; ++i) {
-    const float2 cs = tr[i ^ sw];
-    const float x1 = v[i], x2 = v[i + Q];
+  for (int i = 0; i < Q; i += 2) {
+    const float4 cs = __ldg(r4 + i / 2);  // pairs i and i + 1
+    float x1 = v[i], x2 = v[i + Q];
     v[i] = x1 * cs.x + x2 * cs.y;
     v[i + Q] = x2 * cs.x - x1 * cs.y;
+    x1 = v[i + 1];
+    x2 = v[i + 1 + Q];
+    v[i + 1] = x1 * cs.z + x2 * cs.w;
+    v[i + 1 + Q] = x2 * cs.z - x1 * cs.w;
   }
 }
 
@@ -120,36 +130,19 @@ FL_DEV void staged_colsum(uint8_t* stage, int rows, float* out, int tid) {
   atomicAdd(out + tid, acc);
 }
 
-// The rotary table rows of a tile's 128 tokens, staged for inverse_rope_row: region `reg`
-// (0: first position, 1: GLM block position) at rt + reg * 128 * E, entry e of row rr at
-// e ^ (rr & (E - 1)).  pos(rr) = gp[tok0 + rr] (or rr + pos0 without a position stream),
-// rows past the segment clamped to its last token.
-template <int HD>
-FL_DEV void stage_rope(float2* rt, int nreg, const float2* __restrict__ tab, const int32_t* gpos,
-                       const int32_t* gpos2, int tok0, int pos0, int rows_valid, int tid) {
-  constexpr int E = BwdCfg<HD>::E;
-  for (int reg = 0; reg < nreg; ++reg) {
-    const int32_t* gp = reg == 0 ? gpos : gpos2;
-    for (int i = tid; i < TB * E; i += 256) {
-      const int rr = i / E, e = i % E;
-      const int t = min(rr, rows_valid - 1);
-      const int pos = gp ? __ldg(gp + tok0 + t) : pos0 + t;
-      rt[(reg * TB + rr) * E + (e ^ (rr & (E - 1)))] = __ldg(tab + (int64_t)pos * E + e);
-    }
-  }
-}
-
-// dK / dV.  PREFIX: the CTA's keys are the Lp prefix keys of its head and its query tiles
-// the slice blockIdx.x of the 128-row tile list (n_tiles entries cut into gridDim.x slices).
+// dK / dV.  Non-prefix: unit u = (entry u / nh of the 128-row tile list, head u % nh), the
+// entry's tile index i standing for key tile nq - 1 - i (the list's most work first).
+// PREFIX: unit u = (slice u / nh of the tile list cut into n_split slices, head u % nh),
+// the unit's keys the Lp prefix keys of its head.
 template <int HD, bool PREFIX>
 __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do,
     const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int T, int H,
-    const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, int n_tiles, const float* __restrict__ lse,
-    const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale, float scale_log2, int Lp,
-    bf16* __restrict__ dqkv, float* __restrict__ dpk, float* __restrict__ dpv, const int32_t* __restrict__ ctxs,
-    const int32_t* __restrict__ gpos, const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int dbias_segs,
-    int64_t dbias_rstride, int* status) {
+    const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, int n_tiles, int n_units, int n_split,
+    const float* __restrict__ lse, const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale,
+    float scale_log2, int Lp, bf16* __restrict__ dqkv, float* __restrict__ dpk, float* __restrict__ dpv,
+    const int32_t* __restrict__ ctxs, const int32_t* __restrict__ gpos, const int32_t* __restrict__ gpos2,
+    float* __restrict__ dbias, int dbias_segs, int64_t dbias_rstride, int* status) {
   constexpr int NB = BwdCfg<HD>::NB, TILE = BwdCfg<HD>::TILE, CH = BwdCfg<HD>::CH, E = BwdCfg<HD>::E;
   pdl_wait();  // the previous kernel on the stream has completed (see fl_launch)
   pdl_trigger();
@@ -168,33 +161,47 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   uint64_t* bar_mma2 = bars + 4;
   uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 6);
 
-  const int h = blockIdx.y;
+  const int nh = H / HD;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, qh = warp >> 2;
   const int r = quarter * 32 + lane;  // this thread's key row (TMEM lane)
-  // this CTA's keys and its query tiles [it0, it_end)
-  int seg0 = 0, L = 0, kb = 0, clast = -1, it0, it_end;
-  if constexpr (PREFIX) {
-    const int per = (n_tiles + gridDim.x - 1) / gridDim.x;
-    it0 = blockIdx.x * per;
-    it_end = min(n_tiles, it0 + per);
-  } else {
-    // the 128-row tile list: (segment, tile), tile i standing for key tile nq - 1 - i
-    const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
-    if (dbias && dbias_segs > 0) dbias += (int64_t)(s / dbias_segs) * dbias_rstride;  // the segment's replica
-    seg0 = cu[s];
-    L = cu[s + 1] - seg0;
-    const int nq = (L + TB - 1) / TB;
-    const int kt = nq - 1 - idx;  // key tile: most work first
-    kb = kt * TB;
-    clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
-    it0 = kb <= clast ? 0 : kt;  // a tile holding context keys is seen by every query
-    it_end = nq;
-  }
-  const int k = kb + r;  // the key inside its segment (or the prefix)
-  const bool key_ok = PREFIX ? r < Lp : k < L;
-  // a query tile: its first token, the position of that token in its segment, valid rows
-  auto qtile = [&](int it, int& row0, int& qpos0, int& valid) {
+  const int nreg = rope_tab ? (gpos2 ? 2 : 1) : 0;  // rotary regions of a head
+
+  // a unit: its head, keys (segment start and length, first key kb), the last context key
+  // of the segment (GLM; -1 when causal), its query tiles [it0, it_end), and the QKV bias
+  // gradient of the segment's replica
+  struct Unit {
+    int h, seg0, L, kb, clast, it0, it_end;
+    float* db;
+  };
+  auto unit = [&](int u) {
+    Unit w;
+    w.h = u % nh;
+    if constexpr (PREFIX) {
+      const int per = (n_tiles + n_split - 1) / n_split;
+      w.it0 = (u / nh) * per;
+      w.it_end = min(n_tiles, w.it0 + per);
+      w.seg0 = w.L = w.kb = 0;
+      w.clast = -1;
+      w.db = nullptr;
+    } else {
+      const uint32_t t = tiles[u / nh];
+      const int s = int(t >> 16), idx = int(t & 0xFFFFu);
+      w.seg0 = cu[s];
+      w.L = cu[s + 1] - w.seg0;
+      const int nq = (w.L + TB - 1) / TB;
+      const int kt = nq - 1 - idx;
+      w.kb = kt * TB;
+      w.clast = (ctxs ? min(max(ctxs[s], 0), w.L) : 0) - 1;
+      w.it0 = w.kb <= w.clast ? 0 : kt;  // a tile holding context keys is seen by every query
+      w.it_end = nq;
+      w.db = dbias ? dbias + (dbias_segs > 0 ? (int64_t)(s / dbias_segs) * dbias_rstride : 0) : nullptr;
+    }
+    return w;
+  };
+  // a query tile of unit w: its first token, the position of that token in its segment,
+  // valid rows
+  auto qtile = [&](const Unit& w, int it, int& row0, int& qpos0, int& valid) {
     if constexpr (PREFIX) {
       const int s = int(tiles[it] >> 16), idx = int(tiles[it] & 0xFFFFu);
       const int sb = cu[s];
@@ -203,8 +210,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       valid = min(TB, cu[s + 1] - sb - qpos0);
     } else {
       qpos0 = it * TB;
-      row0 = seg0 + qpos0;
-      valid = min(TB, L - qpos0);
+      row0 = w.seg0 + qpos0;
+      valid = min(TB, w.L - qpos0);
     }
   };
 
@@ -225,209 +232,242 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   const uint32_t t_lane = tmem + (uint32_t(quarter * 32) << 16);
 
   BarTrack tkv, tq0, tq1, tm1, tm2;
-  auto issue_q = [&](int it, int b) {  // one elected thread: Q_it, dO_it into buffer pair b
+  auto issue_q = [&](const Unit& w, int it, int b) {  // one elected thread: Q_it, dO_it into pair b
     int row0, qpos0, valid;
-    qtile(it, row0, qpos0, valid);
+    qtile(w, it, row0, qpos0, valid);
     (b ? tq1 : tq0).pend = true;
     mbar_arrive_expect_tx(bar_q + b, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
-      tma_load_2d(sQ + b * TILE + x * BOX, &tm_qkv, bar_q + b, h * HD + 64 * x, row0);
-      tma_load_2d(sdO + b * TILE + x * BOX, &tm_do, bar_q + b, h * HD + 64 * x, row0);
+      tma_load_2d(sQ + b * TILE + x * BOX, &tm_qkv, bar_q + b, w.h * HD + 64 * x, row0);
+      tma_load_2d(sdO + b * TILE + x * BOX, &tm_do, bar_q + b, w.h * HD + 64 * x, row0);
     }
   };
-  if (tid == 0 && it0 < it_end) {
+  auto issue_kv = [&](const Unit& w) {  // one elected thread: the unit's K and V
     tkv.pend = true;
     mbar_arrive_expect_tx(bar_kv, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
       if constexpr (PREFIX) {
-        tma_load_2d(sK + x * BOX, &tm_pk, bar_kv, h * HD + 64 * x, 0);
-        tma_load_2d(sV + x * BOX, &tm_pv, bar_kv, h * HD + 64 * x, 0);
+        tma_load_2d(sK + x * BOX, &tm_pk, bar_kv, w.h * HD + 64 * x, 0);
+        tma_load_2d(sV + x * BOX, &tm_pv, bar_kv, w.h * HD + 64 * x, 0);
       } else {
-        tma_load_2d(sK + x * BOX, &tm_qkv, bar_kv, H + h * HD + 64 * x, seg0 + kb);
-        tma_load_2d(sV + x * BOX, &tm_qkv, bar_kv, 2 * H + h * HD + 64 * x, seg0 + kb);
+        tma_load_2d(sK + x * BOX, &tm_qkv, bar_kv, H + w.h * HD + 64 * x, w.seg0 + w.kb);
+        tma_load_2d(sV + x * BOX, &tm_qkv, bar_kv, 2 * H + w.h * HD + 64 * x, w.seg0 + w.kb);
       }
     }
-    issue_q(it0, 0);
-    if (it0 + 1 < it_end) issue_q(it0 + 1, 1);
-  }
+  };
 
   constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
   constexpr uint32_t IDESC_G = umma_idesc_bf16(TB, HD, false, true);
-  bool ok = it0 >= it_end || track_wait_all(bar_kv, tkv);
-  if (!ok && tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
-  for (int it = it0; it < it_end && ok; ++it) {
-    const int n = it - it0, b = n & 1;
-    int row0, qpos0, valid;
-    qtile(it, row0, qpos0, valid);
-    {  // lse and delta of the query tile (rows past its segment are never visible)
-      const int c = tid & (TB - 1);
-      const float* src = tid < TB ? lse : delta;
-      const float v = c < valid ? __ldg(src + (int64_t)h * T + row0 + c) : 0.f;
-      if (tid < TB) sL[b * TB + c] = v * LOG2E_B;
-      else sD[b * TB + c] = v;
-    }
+  bool ok = true;
+  int u = blockIdx.x;
+  Unit w = u < n_units ? unit(u) : Unit{};
+  if (tid == 0 && u < n_units && w.it0 < w.it_end) {
+    issue_kv(w);
+    issue_q(w, w.it0, 0);
+    if (w.it0 + 1 < w.it_end) issue_q(w, w.it0 + 1, 1);
+  }
+  while (u < n_units && ok) {
+    const int k = w.kb + r;  // the key inside its segment (or the prefix)
+    const bool key_ok = PREFIX ? r < Lp : k < w.L;
+    const bool work = w.it0 < w.it_end;
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
-    if (!track_wait_all(bar_q + b, b ? tq1 : tq0)) {
+    if (work && !track_wait_all(bar_kv, tkv)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
       ok = false;
       break;
     }
-    // ---- S^T = K Q^T, dP^T = V dO^T (the previous dV / dK products, which read these
-    // columns, have completed)
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t ak = smem_u32(sK), av = smem_u32(sV), bq = smem_u32(sQ + b * TILE),
-                     bo = smem_u32(sdO + b * TILE);
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_k(ak, kk), desc_k(bq, kk), IDESC_S, kk > 0);
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem + 128, desc_k(av, kk), desc_k(bo, kk), IDESC_S, kk > 0);
-      tm1.pend = true;
-      umma_commit(bar_mma1);
-    }
-    if (!track_wait_all(bar_mma1, tm1)) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
-      ok = false;
-      break;
-    }
-    tc_fence_after();
-    // ---- P^T and dS^T of key row r for queries qh * 64 .. + 63, in two groups of 32,
-    // each written (bf16 pairs) into the 16 columns at 64 qh + 16 hf it has just read
-    {
-      const int q0 = qpos0 + qh * 64;
-      // key k is visible to queries [qfirst, qlim) of the tile's segment
-      int qlim, qfirst;
-      if constexpr (PREFIX) {
-        qlim = key_ok ? qpos0 + valid : q0;
-        qfirst = q0;
-      } else {
-        qlim = key_ok ? min(L, q0 + 64) : q0;
-        qfirst = k <= clast ? q0 : max(q0, k);
+    for (int it = w.it0; it < w.it_end && ok; ++it) {
+      const int b = (it - w.it0) & 1;
+      int row0, qpos0, valid;
+      qtile(w, it, row0, qpos0, valid);
+      {  // lse and delta of the query tile (rows past its segment are never visible)
+        const int c = tid & (TB - 1);
+        const float* src = tid < TB ? lse : delta;
+        const float v = c < valid ? __ldg(src + (int64_t)w.h * T + row0 + c) : 0.f;
+        if (tid < TB) sL[b * TB + c] = v * LOG2E_B;
+        else sD[b * TB + c] = v;
       }
-      const float* Lb = sL + b * TB;
-      const float* Db = sD + b * TB;
+      if (!track_wait_all(bar_q + b, b ? tq1 : tq0)) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+        ok = false;
+        break;
+      }
+      // ---- S^T = K Q^T, dP^T = V dO^T (the previous dV / dK products, which read these
+      // columns, have completed)
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t ak = smem_u32(sK), av = smem_u32(sV), bq = smem_u32(sQ + b * TILE),
+                       bo = smem_u32(sdO + b * TILE);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_k(ak, kk), desc_k(bq, kk), IDESC_S, kk > 0);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem + 128, desc_k(av, kk), desc_k(bo, kk), IDESC_S, kk > 0);
+        tm1.pend = true;
+        umma_commit(bar_mma1);
+      }
+      if (!track_wait_all(bar_mma1, tm1)) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      // ---- P^T and dS^T of key row r for queries qh * 64 .. + 63, in two groups of 32,
+      // each written (bf16 pairs) into the 16 columns at 64 qh + 16 hf it has just read
+      {
+        const int q0 = qpos0 + qh * 64;
+        // key k is visible to queries [qfirst, qlim) of the tile's segment
+        int qlim, qfirst;
+        if constexpr (PREFIX) {
+          qlim = key_ok ? qpos0 + valid : q0;
+          qfirst = q0;
+        } else {
+          qlim = key_ok ? min(w.L, q0 + 64) : q0;
+          qfirst = k <= w.clast ? q0 : max(q0, k);
+        }
+        const float* Lb = sL + b * TB;
+        const float* Db = sD + b * TB;
 #pragma unroll 1
-      for (int hf = 0; hf < 2; ++hf) {
-        uint32_t sr[32], dr[32];
-        tmem_ld32(t_lane + qh * 64 + 32 * hf, sr);
-        tmem_ld32(t_lane + 128 + qh * 64 + 32 * hf, dr);
-        tmem_ld_wait();
-        const float4* L4 = reinterpret_cast<const float4*>(Lb + qh * 64 + 32 * hf);
-        const float4* D4 = reinterpret_cast<const float4*>(Db + qh * 64 + 32 * hf);
-        uint32_t pp[16], dd[16];
+        for (int hf = 0; hf < 2; ++hf) {
+          uint32_t sr[32], dr[32];
+          tmem_ld32(t_lane + qh * 64 + 32 * hf, sr);
+          tmem_ld32(t_lane + 128 + qh * 64 + 32 * hf, dr);
+          tmem_ld_wait();
+          const float4* L4 = reinterpret_cast<const float4*>(Lb + qh * 64 + 32 * hf);
+          const float4* D4 = reinterpret_cast<const float4*>(Db + qh * 64 + 32 * hf);
+          uint32_t pp[16], dd[16];
 #pragma unroll
-        for (int c8 = 0; c8 < 4; ++c8) {
-          const float4 la = L4[2 * c8], lb = L4[2 * c8 + 1], da = D4[2 * c8], db = D4[2 * c8 + 1];
-          const float lq[8] = {la.x, la.y, la.z, la.w, lb.x, lb.y, lb.z, lb.w};
-          const float dq[8] = {da.x, da.y, da.z, da.w, db.x, db.y, db.z, db.w};
-          float p[8], ds[8];
+          for (int c8 = 0; c8 < 4; ++c8) {
+            const float4 la = L4[2 * c8], lb = L4[2 * c8 + 1], da = D4[2 * c8], db = D4[2 * c8 + 1];
+            const float lq[8] = {la.x, la.y, la.z, la.w, lb.x, lb.y, lb.z, lb.w};
+            const float dq[8] = {da.x, da.y, da.z, da.w, db.x, db.y, db.z, db.w};
+            float p[8], ds[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int c = 8 * c8 + e, q = q0 + 32 * hf + c;
-            const bool vis = q >= qfirst && q < qlim;
-            const float pv = vis ? exp2_hw(fmaf(__uint_as_float(sr[c]), scale_log2, -lq[e])) : 0.f;
-            p[e] = pv;
-            ds[e] = pv * (__uint_as_float(dr[c]) - dq[e]);
+            for (int e = 0; e < 8; ++e) {
+              const int c = 8 * c8 + e, q = q0 + 32 * hf + c;
+              const bool vis = q >= qfirst && q < qlim;
+              const float pv = vis ? exp2_hw(fmaf(__uint_as_float(sr[c]), scale_log2, -lq[e])) : 0.f;
+              p[e] = pv;
+              ds[e] = pv * (__uint_as_float(dr[c]) - dq[e]);
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              pp[4 * c8 + e] = pack_bf16x2(p[2 * e], p[2 * e + 1]);
+              dd[4 * c8 + e] = pack_bf16x2(ds[2 * e], ds[2 * e + 1]);
+            }
           }
+          tmem_st16(t_lane + qh * 64 + 16 * hf, pp);
+          tmem_st16(t_lane + 128 + qh * 64 + 16 * hf, dd);
+        }
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      __syncthreads();
+      // ---- dV += P^T dO, dK += dS^T Q (A from TMEM); then the tile after next into this
+      // buffer pair once both products have read it
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t bq = smem_u32(sQ + b * TILE), bo = smem_u32(sdO + b * TILE);
+        const bool acc = it > w.it0;
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            pp[4 * c8 + e] = pack_bf16x2(p[2 * e], p[2 * e + 1]);
-            dd[4 * c8 + e] = pack_bf16x2(ds[2 * e], ds[2 * e + 1]);
+        for (int kk = 0; kk < TB / 16; ++kk)
+          umma_bf16_ts(tmem + 256, tmem + a_col(kk), desc_mn(bo, kk), IDESC_G, (acc || kk > 0) ? 1u : 0u);
+#pragma unroll
+        for (int kk = 0; kk < TB / 16; ++kk)
+          umma_bf16_ts(tmem + 256 + HD, tmem + 128 + a_col(kk), desc_mn(bq, kk), IDESC_G, (acc || kk > 0) ? 1u : 0u);
+        tm2.pend = true;
+        umma_commit(bar_mma2);
+      }
+      if (!track_wait_all(bar_mma2, tm2)) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (tid == 0 && it + 2 < w.it_end) issue_q(w, it + 2, b);
+    }
+    if (!ok) break;
+
+    // ---- every product of the unit is complete: the next unit's K / V and first query
+    // tile load into their buffers (pair 0) while this unit's dK / dV leave through pair 1
+    const int un = u + gridDim.x;
+    const Unit wn = un < n_units ? unit(un) : Unit{};
+    const bool next = un < n_units && wn.it0 < wn.it_end;
+    if (tid == 0 && next) {
+      issue_kv(wn);
+      issue_q(wn, wn.it0, 0);
+    }
+    if (work) {
+      if constexpr (PREFIX) {
+        // ---- dK * scale and dV added into the fp32 prefix gradients: thread (r, qh) adds
+        // dims qh * HD/2 .. + HD/2 - 1 of prefix key r
+#pragma unroll 1
+        for (int part = 0; part < 2; ++part) {  // 0: dK, 1: dV
+          uint32_t vr[HD / 2];
+#pragma unroll
+          for (int c = 0; c < HD / 2; c += 32)
+            tmem_ld32(t_lane + (part ? 256 : 256 + HD) + qh * (HD / 2) + c,
+                      *reinterpret_cast<uint32_t(*)[32]>(vr + c));
+          tmem_ld_wait();
+          if (key_ok) {
+            const float f = part ? 1.f : scale;
+            float* dst = (part ? dpv : dpk) + (int64_t)r * H + w.h * HD + qh * (HD / 2);
+#pragma unroll
+            for (int c = 0; c < HD / 2; c += 4)
+              red_add_v4(dst + c, __uint_as_float(vr[c]) * f, __uint_as_float(vr[c + 1]) * f,
+                         __uint_as_float(vr[c + 2]) * f, __uint_as_float(vr[c + 3]) * f);
           }
         }
-        tmem_st16(t_lane + qh * 64 + 16 * hf, pp);
-        tmem_st16(t_lane + 128 + qh * 64 + 16 * hf, dd);
+      } else {
+        // ---- dK (scaled, rotated back) and dV: thread (r, qh) takes dims qh * HD/2 .. +
+        // HD/2 - 1 of key row r from TMEM and stages the bf16 rows in the pair-1 Q (dK) and
+        // dO (dV) buffers, then the CTA writes whole rows with coalesced 16-byte stores; the
+        // bias column sums are taken from the staged rows (the values stored)
+#pragma unroll 1
+        for (int part = 0; part < 2; ++part) {  // 0: dK, 1: dV
+          uint8_t* stage = part ? sdO + TILE : sQ + TILE;
+          uint32_t vr[HD / 2];
+#pragma unroll
+          for (int c = 0; c < HD / 2; c += 32)
+            tmem_ld32(t_lane + (part ? 256 : 256 + HD) + qh * (HD / 2) + c,
+                      *reinterpret_cast<uint32_t(*)[32]>(vr + c));
+          tmem_ld_wait();
+          float* v = reinterpret_cast<float*>(vr);
+#pragma unroll
+          for (int c = 0; c < HD / 2; ++c) v[c] = __uint_as_float(vr[c]) * (part ? 1.f : scale);
+          if (part == 0 && qh < nreg && key_ok) {  // rotary region qh: by pos, or by the GLM block position
+            const int32_t* gp = qh == 0 ? gpos : gpos2;
+            const int pos = gp ? __ldg(gp + w.seg0 + k) : k;
+            inverse_rope_row<HD>(v, rope_tab + (int64_t)pos * E);
+          }
+#pragma unroll
+          for (int c8 = 0; c8 < HD / 16; ++c8)
+            *reinterpret_cast<uint4*>(stage_chunk<HD>(stage, r, qh * (HD / 16) + c8)) =
+                make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
+                           pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
+          const int col = (part ? 2 * H : H) + w.h * HD;
+          __syncthreads();  // the tile is staged
+          if (w.db) staged_colsum<HD>(stage, min(TB, w.L - w.kb), w.db + col, tid);
+          // 128 rows x CH chunks: consecutive threads write consecutive chunks of a row
+#pragma unroll
+          for (int i = 0; i < TB * CH / 256; ++i) {
+            const int id = tid + 256 * i, row = id / CH, jc = id % CH;
+            if (w.kb + row < w.L)
+              *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.kb + row) * 3 * H + col + jc * 8) =
+                  *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
+          }
+        }
       }
     }
-    tmem_st_wait();
+    // the staged rows have been read and the dK / dV columns loaded before the pair-1
+    // buffers are loaded again and the next unit's products overwrite the accumulators
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
-    // ---- dV += P^T dO, dK += dS^T Q (A from TMEM); then the tile after next into this
-    // buffer pair once both products have read it
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t bq = smem_u32(sQ + b * TILE), bo = smem_u32(sdO + b * TILE);
-      const bool acc = it > it0;
-#pragma unroll
-      for (int kk = 0; kk < TB / 16; ++kk)
-        umma_bf16_ts(tmem + 256, tmem + a_col(kk), desc_mn(bo, kk), IDESC_G, (acc || kk > 0) ? 1u : 0u);
-#pragma unroll
-      for (int kk = 0; kk < TB / 16; ++kk)
-        umma_bf16_ts(tmem + 256 + HD, tmem + 128 + a_col(kk), desc_mn(bq, kk), IDESC_G, (acc || kk > 0) ? 1u : 0u);
-      tm2.pend = true;
-      umma_commit(bar_mma2);
-    }
-    if (!track_wait_all(bar_mma2, tm2)) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
-      ok = false;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && it + 2 < it_end) issue_q(it + 2, b);
-  }
-
-  if (ok && it0 < it_end) {
-    if constexpr (PREFIX) {
-      // ---- dK * scale and dV added into the fp32 prefix gradients: thread (r, qh) adds
-      // dims qh * HD/2 .. + HD/2 - 1 of prefix key r
-#pragma unroll 1
-      for (int part = 0; part < 2; ++part) {  // 0: dK, 1: dV
-        uint32_t vr[HD / 2];
-#pragma unroll
-        for (int c = 0; c < HD / 2; c += 32)
-          tmem_ld32(t_lane + (part ? 256 : 256 + HD) + qh * (HD / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(vr + c));
-        tmem_ld_wait();
-        if (key_ok) {
-          const float f = part ? 1.f : scale;
-          float* dst = (part ? dpv : dpk) + (int64_t)r * H + h * HD + qh * (HD / 2);
-#pragma unroll
-          for (int c = 0; c < HD / 2; c += 4)
-            red_add_v4(dst + c, __uint_as_float(vr[c]) * f, __uint_as_float(vr[c + 1]) * f,
-                       __uint_as_float(vr[c + 2]) * f, __uint_as_float(vr[c + 3]) * f);
-        }
-      }
-    } else {
-      // ---- dK (scaled, rotated back) and dV: thread (r, qh) takes dims qh * HD/2 .. + HD/2
-      // - 1 of key row r from TMEM, stages the bf16 rows in the freed K (dK) and V (dV)
-      // buffers, then the CTA writes whole rows with coalesced 16-byte stores; the bias
-      // column sums are taken from the staged rows (the values stored).  The freed Q / dO
-      // buffers hold the rotary table rows of the tile's keys.
-      float2* rt = reinterpret_cast<float2*>(sQ);
-      const int nreg = rope_tab ? (gpos2 ? 2 : 1) : 0;
-      stage_rope<HD>(rt, nreg, rope_tab, gpos, gpos2, seg0 + kb, kb, L - kb, tid);
-      __syncthreads();
-#pragma unroll 1
-      for (int part = 0; part < 2; ++part) {  // 0: dK, 1: dV
-        uint8_t* stage = part ? sV : sK;
-        uint32_t vr[HD / 2];
-#pragma unroll
-        for (int c = 0; c < HD / 2; c += 32)
-          tmem_ld32(t_lane + (part ? 256 : 256 + HD) + qh * (HD / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(vr + c));
-        tmem_ld_wait();
-        float* v = reinterpret_cast<float*>(vr);
-#pragma unroll
-        for (int c = 0; c < HD / 2; ++c) v[c] = __uint_as_float(vr[c]) * (part ? 1.f : scale);
-        if (part == 0 && qh < nreg && key_ok) inverse_rope_row<HD>(v, rt + (qh * TB + r) * E, r & (E - 1));
-#pragma unroll
-        for (int c8 = 0; c8 < HD / 16; ++c8)
-          *reinterpret_cast<uint4*>(stage_chunk<HD>(stage, r, qh * (HD / 16) + c8)) =
-              make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
-                         pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
-        const int col = (part ? 2 * H : H) + h * HD;
-        __syncthreads();  // the tile is staged
-        if (dbias) staged_colsum<HD>(stage, min(TB, L - kb), dbias + col, tid);
-        // 128 rows x CH chunks: consecutive threads write consecutive chunks of a row
-#pragma unroll
-        for (int i = 0; i < TB * CH / 256; ++i) {
-          const int id = tid + 256 * i, row = id / CH, jc = id % CH;
-          if (kb + row < L)
-            *reinterpret_cast<uint4*>(dqkv + ((int64_t)seg0 + kb + row) * 3 * H + col + jc * 8) =
-                *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
-        }
-      }
-    }
+    if (tid == 0 && next && wn.it0 + 1 < wn.it_end) issue_q(wn, wn.it0 + 1, 1);
+    u = un;
+    w = wn;
   }
   if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
     track_drain(bar_kv, tkv);
@@ -444,11 +484,12 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   }
 }
 
+// dQ.  Unit u = (entry u / nh of the 128-row tile list, head u % nh).
 template <int HD>
 __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do,
     const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int T, int H,
-    const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, const float* __restrict__ lse,
+    const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, int n_units, const float* __restrict__ lse,
     const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale, float scale_log2, int Lp,
     bf16* __restrict__ dqkv, const int32_t* __restrict__ ctxs, const int32_t* __restrict__ gpos,
     const int32_t* __restrict__ gpos2, float* __restrict__ dbias, int dbias_segs, int64_t dbias_rstride, int* status) {
@@ -468,23 +509,38 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   uint64_t* bar_mma2 = bars + 4;
   uint32_t* holder = reinterpret_cast<uint32_t*>(bars + 6);
 
-  // the 128-row tile list: (segment, query tile)
-  const int s = int(tiles[blockIdx.x] >> 16), idx = int(tiles[blockIdx.x] & 0xFFFFu);
-  if (dbias && dbias_segs > 0) dbias += (int64_t)(s / dbias_segs) * dbias_rstride;  // the segment's replica
-  const int h = blockIdx.y;
+  const int nh = H / HD;
   const int tid = threadIdx.x, warp = tid >> 5;
   const int quarter = warp & 3, kh = warp >> 2;
   const int r = quarter * 32 + (tid & 31);  // this thread's query row (TMEM lane)
-  const int seg0 = cu[s], L = cu[s + 1] - seg0;
-  const int q0 = idx * TB;
-  const int q = q0 + r;
-  const bool q_ok = q < L;
-  const int npt = Lp > 0 ? 1 : 0;  // at most one prefix tile (Lp <= 128)
-  const int clast = (ctxs ? min(max(ctxs[s], 0), L) : 0) - 1;
-  const int n_kv = npt + max(idx, clast >= 0 ? clast / TB : 0) + 1;
-  const float lse2 = q_ok ? __ldg(lse + (int64_t)h * T + seg0 + q) * LOG2E_B : 0.f;
-  const float dl = q_ok ? __ldg(delta + (int64_t)h * T + seg0 + q) : 0.f;
-  const int ulim = q_ok ? max(q, clast) : -1;  // last own key visible to the row
+  const int npt = Lp > 0 ? 1 : 0;           // at most one prefix tile (Lp <= 128)
+  const int nreg = rope_tab ? (gpos2 ? 2 : 1) : 0;
+
+  // a unit: its head, segment, first query q0, last context key (-1 when causal), key
+  // tiles (the prefix tile first), and the QKV bias gradient of the segment's replica
+  struct Unit {
+    int h, seg0, L, q0, clast, n_kv;
+    float* db;
+  };
+  auto unit = [&](int u) {
+    Unit w;
+    const uint32_t t = tiles[u / nh];
+    const int s = int(t >> 16), idx = int(t & 0xFFFFu);
+    w.h = u % nh;
+    w.seg0 = cu[s];
+    w.L = cu[s + 1] - w.seg0;
+    w.q0 = idx * TB;
+    w.clast = (ctxs ? min(max(ctxs[s], 0), w.L) : 0) - 1;
+    w.n_kv = npt + max(idx, w.clast >= 0 ? w.clast / TB : 0) + 1;
+    w.db = dbias ? dbias + (dbias_segs > 0 ? (int64_t)(s / dbias_segs) * dbias_rstride : 0) : nullptr;
+    return w;
+  };
+  // the thread's row statistics in unit w: lse * log2e and delta
+  auto row_stats = [&](const Unit& w, float& lse2, float& dl) {
+    const bool q_ok = w.q0 + r < w.L;
+    lse2 = q_ok ? __ldg(lse + (int64_t)w.h * T + w.seg0 + w.q0 + r) * LOG2E_B : 0.f;
+    dl = q_ok ? __ldg(delta + (int64_t)w.h * T + w.seg0 + w.q0 + r) : 0.f;
+  };
 
   if (tid == 0) {
     for (int i = 0; i < 5; ++i) mbar_init(bars + i, 1);
@@ -503,147 +559,185 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   const uint32_t t_lane = tmem + (uint32_t(quarter * 32) << 16);
 
   BarTrack tqdo, tkv0, tkv1, tm1, tm2;
-  auto issue_kv = [&](int j, int b) {  // one elected thread: K_j, V_j into buffer pair b
+  auto issue_kv = [&](const Unit& w, int j, int b) {  // one elected thread: K_j, V_j into pair b
     (b ? tkv1 : tkv0).pend = true;
     mbar_arrive_expect_tx(bar_kv + b, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
       if (j < npt) {
-        tma_load_2d(sK + b * TILE + x * BOX, &tm_pk, bar_kv + b, h * HD + 64 * x, 0);
-        tma_load_2d(sV + b * TILE + x * BOX, &tm_pv, bar_kv + b, h * HD + 64 * x, 0);
+        tma_load_2d(sK + b * TILE + x * BOX, &tm_pk, bar_kv + b, w.h * HD + 64 * x, 0);
+        tma_load_2d(sV + b * TILE + x * BOX, &tm_pv, bar_kv + b, w.h * HD + 64 * x, 0);
       } else {
-        const int row = seg0 + (j - npt) * TB;
-        tma_load_2d(sK + b * TILE + x * BOX, &tm_qkv, bar_kv + b, H + h * HD + 64 * x, row);
-        tma_load_2d(sV + b * TILE + x * BOX, &tm_qkv, bar_kv + b, 2 * H + h * HD + 64 * x, row);
+        const int row = w.seg0 + (j - npt) * TB;
+        tma_load_2d(sK + b * TILE + x * BOX, &tm_qkv, bar_kv + b, H + w.h * HD + 64 * x, row);
+        tma_load_2d(sV + b * TILE + x * BOX, &tm_qkv, bar_kv + b, 2 * H + w.h * HD + 64 * x, row);
       }
     }
   };
-  if (tid == 0) {
+  auto issue_qdo = [&](const Unit& w) {  // one elected thread: the unit's Q and dO
     tqdo.pend = true;
     mbar_arrive_expect_tx(bar_qdo, 2 * TILE);
 #pragma unroll
     for (int x = 0; x < NB; ++x) {
-      tma_load_2d(sQ + x * BOX, &tm_qkv, bar_qdo, h * HD + 64 * x, seg0 + q0);
-      tma_load_2d(sdO + x * BOX, &tm_do, bar_qdo, h * HD + 64 * x, seg0 + q0);
+      tma_load_2d(sQ + x * BOX, &tm_qkv, bar_qdo, w.h * HD + 64 * x, w.seg0 + w.q0);
+      tma_load_2d(sdO + x * BOX, &tm_do, bar_qdo, w.h * HD + 64 * x, w.seg0 + w.q0);
     }
-    issue_kv(0, 0);
-    if (n_kv > 1) issue_kv(1, 1);
-  }
+  };
 
   constexpr uint32_t IDESC_S = umma_idesc_bf16(TB, TB, false, false);
   constexpr uint32_t IDESC_G = umma_idesc_bf16(TB, HD, false, true);
-  bool ok = track_wait_all(bar_qdo, tqdo);
-  if (!ok && tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
-  for (int j = 0; j < n_kv && ok; ++j) {
-    const int b = j & 1;
-    if (!track_wait_all(bar_kv + b, b ? tkv1 : tkv0)) {
+  bool ok = true;
+  int u = blockIdx.x;
+  Unit w = u < n_units ? unit(u) : Unit{};
+  float lse2 = 0.f, dl = 0.f;
+  if (u < n_units) row_stats(w, lse2, dl);
+  if (tid == 0 && u < n_units) {
+    issue_qdo(w);
+    issue_kv(w, 0, 0);
+    if (w.n_kv > 1) issue_kv(w, 1, 1);
+  }
+  while (u < n_units && ok) {
+    const int q = w.q0 + r;
+    const bool q_ok = q < w.L;
+    const int ulim = q_ok ? max(q, w.clast) : -1;  // last own key visible to the row
+    // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
+    if (!track_wait_all(bar_qdo, tqdo)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
       ok = false;
       break;
     }
-    // ---- S = Q K_j^T, dP = dO V_j^T (the previous dQ product, which read these columns,
-    // has completed)
-    if (tid == 0) {
+    for (int j = 0; j < w.n_kv && ok; ++j) {
+      const int b = j & 1;
+      if (!track_wait_all(bar_kv + b, b ? tkv1 : tkv0)) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
+        ok = false;
+        break;
+      }
+      // ---- S = Q K_j^T, dP = dO V_j^T (the previous dQ product, which read these
+      // columns, has completed)
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t aq = smem_u32(sQ), ao = smem_u32(sdO), bk = smem_u32(sK + b * TILE),
+                       bv = smem_u32(sV + b * TILE);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_k(aq, kk), desc_k(bk, kk), IDESC_S, kk > 0);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem + 128, desc_k(ao, kk), desc_k(bv, kk), IDESC_S, kk > 0);
+        tm1.pend = true;
+        umma_commit(bar_mma1);
+      }
+      if (!track_wait_all(bar_mma1, tm1)) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
+        ok = false;
+        break;
+      }
       tc_fence_after();
-      const uint32_t aq = smem_u32(sQ), ao = smem_u32(sdO), bk = smem_u32(sK + b * TILE),
-                     bv = smem_u32(sV + b * TILE);
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem, desc_k(aq, kk), desc_k(bk, kk), IDESC_S, kk > 0);
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) umma_bf16(tmem + 128, desc_k(ao, kk), desc_k(bv, kk), IDESC_S, kk > 0);
-      tm1.pend = true;
-      umma_commit(bar_mma1);
-    }
-    if (!track_wait_all(bar_mma1, tm1)) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
-      ok = false;
-      break;
-    }
-    tc_fence_after();
-    // ---- dS of query row r for keys kh * 64 .. + 63 of the tile, in two groups of 32,
-    // each written (bf16 pairs) into the 16 S columns at 64 kh + 16 hf it has just read
-    {
-      const bool prefix = j < npt;
-      const int u0 = (prefix ? 0 : (j - npt) * TB) + kh * 64;  // first key of the half
-      const int uend = prefix ? (q_ok ? Lp : 0) : ulim + 1;    // keys [u0, uend) are visible
+      // ---- dS of query row r for keys kh * 64 .. + 63 of the tile, in two groups of 32,
+      // each written (bf16 pairs) into the 16 S columns at 64 kh + 16 hf it has just read
+      {
+        const bool prefix = j < npt;
+        const int u0 = (prefix ? 0 : (j - npt) * TB) + kh * 64;  // first key of the half
+        const int uend = prefix ? (q_ok ? Lp : 0) : ulim + 1;    // keys [u0, uend) are visible
 #pragma unroll 1
-      for (int hf = 0; hf < 2; ++hf) {
-        uint32_t sr[32], dr[32];
-        tmem_ld32(t_lane + kh * 64 + 32 * hf, sr);
-        tmem_ld32(t_lane + 128 + kh * 64 + 32 * hf, dr);
-        tmem_ld_wait();
-        uint32_t dd[16];
+        for (int hf = 0; hf < 2; ++hf) {
+          uint32_t sr[32], dr[32];
+          tmem_ld32(t_lane + kh * 64 + 32 * hf, sr);
+          tmem_ld32(t_lane + 128 + kh * 64 + 32 * hf, dr);
+          tmem_ld_wait();
+          uint32_t dd[16];
 #pragma unroll
-        for (int c2 = 0; c2 < 16; ++c2) {
-          float ds[2];
+          for (int c2 = 0; c2 < 16; ++c2) {
+            float ds[2];
 #pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int c = 2 * c2 + e;
-            const bool vis = u0 + 32 * hf + c < uend;
-            const float pv = vis ? exp2_hw(fmaf(__uint_as_float(sr[c]), scale_log2, -lse2)) : 0.f;
-            ds[e] = pv * (__uint_as_float(dr[c]) - dl);
+            for (int e = 0; e < 2; ++e) {
+              const int c = 2 * c2 + e;
+              const bool vis = u0 + 32 * hf + c < uend;
+              const float pv = vis ? exp2_hw(fmaf(__uint_as_float(sr[c]), scale_log2, -lse2)) : 0.f;
+              ds[e] = pv * (__uint_as_float(dr[c]) - dl);
+            }
+            dd[c2] = pack_bf16x2(ds[0], ds[1]);
           }
-          dd[c2] = pack_bf16x2(ds[0], ds[1]);
+          tmem_st16(t_lane + kh * 64 + 16 * hf, dd);
         }
-        tmem_st16(t_lane + kh * 64 + 16 * hf, dd);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      __syncthreads();
+      // ---- dQ += dS K_j (A from TMEM); then the tile after next into this buffer pair
+      // once both products have read it
+      if (tid == 0) {
+        tc_fence_after();
+        const uint32_t bk = smem_u32(sK + b * TILE);
+#pragma unroll
+        for (int kk = 0; kk < TB / 16; ++kk)
+          umma_bf16_ts(tmem + 256, tmem + a_col(kk), desc_mn(bk, kk), IDESC_G, (j > 0 || kk > 0) ? 1u : 0u);
+        tm2.pend = true;
+        umma_commit(bar_mma2);
+      }
+      if (!track_wait_all(bar_mma2, tm2)) {
+        if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (tid == 0 && j + 2 < w.n_kv) issue_kv(w, j + 2, b);
+    }
+    if (!ok) break;
+
+    // ---- every product of the unit is complete: the next unit's Q, dO and first key /
+    // value tiles load (pair 0) while this unit's dQ leaves through the pair-1 K buffer
+    const int un = u + gridDim.x;
+    const Unit wn = un < n_units ? unit(un) : Unit{};
+    if (tid == 0 && un < n_units) {
+      issue_qdo(wn);
+      issue_kv(wn, 0, 0);
+    }
+    float lse2n = 0.f, dln = 0.f;
+    if (un < n_units) row_stats(wn, lse2n, dln);
+    // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * HD/2 .. + HD/2 - 1 of
+    // query row r, staged and written as whole coalesced rows, the bias column sums taken
+    // from the staged rows
+    {
+      uint8_t* stage = sK + TILE;
+      uint32_t vr[HD / 2];
+#pragma unroll
+      for (int c = 0; c < HD / 2; c += 32)
+        tmem_ld32(t_lane + 256 + kh * (HD / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(vr + c));
+      tmem_ld_wait();
+      float* v = reinterpret_cast<float*>(vr);
+#pragma unroll
+      for (int c = 0; c < HD / 2; ++c) v[c] = __uint_as_float(vr[c]) * scale;
+      if (kh < nreg && q_ok) {  // rotary region kh: by pos, or by the GLM block position
+        const int32_t* gp = kh == 0 ? gpos : gpos2;
+        const int pos = gp ? __ldg(gp + w.seg0 + q) : q;
+        inverse_rope_row<HD>(v, rope_tab + (int64_t)pos * E);
+      }
+#pragma unroll
+      for (int c8 = 0; c8 < HD / 16; ++c8)
+        *reinterpret_cast<uint4*>(stage_chunk<HD>(stage, r, kh * (HD / 16) + c8)) =
+            make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
+                       pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
+      const int col = w.h * HD;
+      __syncthreads();  // the tile is staged
+      if (w.db) staged_colsum<HD>(stage, min(TB, w.L - w.q0), w.db + col, tid);
+#pragma unroll
+      for (int i = 0; i < TB * CH / 256; ++i) {
+        const int id = tid + 256 * i, row = id / CH, jc = id % CH;
+        if (w.q0 + row < w.L)
+          *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.q0 + row) * 3 * H + col + jc * 8) =
+              *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
       }
     }
-    tmem_st_wait();
+    // the staged rows have been read and the dQ columns loaded before the pair-1 buffers
+    // are loaded again and the next unit's products overwrite the accumulator
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
-    // ---- dQ += dS K_j (A from TMEM); then the tile after next into this buffer pair once
-    // both products have read it
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t bk = smem_u32(sK + b * TILE);
-#pragma unroll
-      for (int kk = 0; kk < TB / 16; ++kk)
-        umma_bf16_ts(tmem + 256, tmem + a_col(kk), desc_mn(bk, kk), IDESC_G, (j > 0 || kk > 0) ? 1u : 0u);
-      tm2.pend = true;
-      umma_commit(bar_mma2);
-    }
-    if (!track_wait_all(bar_mma2, tm2)) {
-      if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
-      ok = false;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && j + 2 < n_kv) issue_kv(j + 2, b);
-  }
-
-  // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * HD/2 .. + HD/2 - 1 of
-  // query row r, staged in the freed K buffers and written as whole coalesced rows, the bias
-  // column sums taken from the staged rows; the rotary rows of the tile's queries in the
-  // freed V buffers.
-  if (ok) {
-    float2* rt = reinterpret_cast<float2*>(sV);
-    const int nreg = rope_tab ? (gpos2 ? 2 : 1) : 0;
-    stage_rope<HD>(rt, nreg, rope_tab, gpos, gpos2, seg0 + q0, q0, L - q0, tid);
-    __syncthreads();
-    uint32_t vr[HD / 2];
-#pragma unroll
-    for (int c = 0; c < HD / 2; c += 32)
-      tmem_ld32(t_lane + 256 + kh * (HD / 2) + c, *reinterpret_cast<uint32_t(*)[32]>(vr + c));
-    tmem_ld_wait();
-    float* v = reinterpret_cast<float*>(vr);
-#pragma unroll
-    for (int c = 0; c < HD / 2; ++c) v[c] = __uint_as_float(vr[c]) * scale;
-    if (kh < nreg && q_ok) inverse_rope_row<HD>(v, rt + (kh * TB + r) * E, r & (E - 1));
-#pragma unroll
-    for (int c8 = 0; c8 < HD / 16; ++c8)
-      *reinterpret_cast<uint4*>(stage_chunk<HD>(sK, r, kh * (HD / 16) + c8)) =
-          make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
-                     pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
-    const int col = h * HD;
-    __syncthreads();  // the tile is staged
-    if (dbias) staged_colsum<HD>(sK, min(TB, L - q0), dbias + col, tid);
-#pragma unroll
-    for (int i = 0; i < TB * CH / 256; ++i) {
-      const int id = tid + 256 * i, row = id / CH, jc = id % CH;
-      if (q0 + row < L)
-        *reinterpret_cast<uint4*>(dqkv + ((int64_t)seg0 + q0 + row) * 3 * H + col + jc * 8) =
-            *reinterpret_cast<const uint4*>(stage_chunk<HD>(sK, row, jc));
-    }
+    if (tid == 0 && un < n_units && wn.n_kv > 1) issue_kv(wn, 1, 1);
+    u = un;
+    w = wn;
+    lse2 = lse2n;
+    dl = dln;
   }
   if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
     track_drain(bar_qdo, tqdo);
@@ -699,22 +793,27 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
   }
   const float scale = 1.f / sqrtf((float)HD);
   const float2* tab = reinterpret_cast<const float2*>(rope_tab);
-  FL_CUDA_TRY(fl_launch(attn_bwd_dq_tc_kernel<HD>, dim3(n_tiles, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo, tpk,
-                        tpv, T, H, cu, tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv, glm.ctx,
-                        glm.pos, glm.pos2, dbias, dbias_segs, dbias_rstride, status));
-  FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, false>, dim3(n_tiles, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo,
-                        tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, 0, (bf16*)dqkv,
-                        (float*)nullptr, (float*)nullptr, glm.ctx, glm.pos, glm.pos2, dbias, dbias_segs, dbias_rstride,
-                        status));
-  if (pre.len > 0) {
+  // persistent: one CTA per SM (512 TMEM columns each) walks the (tile, head) units
+  const int n_units = n_tiles * nh;
+  const int grid = n_units < sm_count_bwd() ? n_units : sm_count_bwd();
+  if (n_units > 0) {
+    FL_CUDA_TRY(fl_launch(attn_bwd_dq_tc_kernel<HD>, dim3(grid), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo, tpk, tpv,
+                          T, H, cu, tiles, n_units, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv,
+                          glm.ctx, glm.pos, glm.pos2, dbias, dbias_segs, dbias_rstride, status));
+    FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, false>, dim3(grid), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo,
+                          tpk, tpv, T, H, cu, tiles, n_tiles, n_units, 0, lse, delta, tab, scale, scale * LOG2E_B, 0,
+                          (bf16*)dqkv, (float*)nullptr, (float*)nullptr, glm.ctx, glm.pos, glm.pos2, dbias,
+                          dbias_segs, dbias_rstride, status));
+  }
+  if (pre.len > 0 && n_tiles > 0) {
     // the prefix keys of each head against slices of the query tiles, about one CTA per SM
     int nsplit = (sm_count_bwd() + nh - 1) / nh;
     if (nsplit > n_tiles) nsplit = n_tiles;
     if (nsplit < 1) nsplit = 1;
-    FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, true>, dim3(nsplit, nh), dim3(256), BwdCfg<HD>::SMEM, st, tq,
-                          tdo, tpk, tpv, T, H, cu, tiles, n_tiles, lse, delta, tab, scale, scale * LOG2E_B, pre.len,
-                          (bf16*)dqkv, pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2, (float*)nullptr, 0, (int64_t)0,
-                          status));
+    FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, true>, dim3(nsplit * nh), dim3(256), BwdCfg<HD>::SMEM, st, tq,
+                          tdo, tpk, tpv, T, H, cu, tiles, n_tiles, nsplit * nh, nsplit, lse, delta, tab, scale,
+                          scale * LOG2E_B, pre.len, (bf16*)dqkv, pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2,
+                          (float*)nullptr, 0, (int64_t)0, status));
   }
   return FL_OK;
 }

@@ -342,6 +342,50 @@ def test_pack_clients_bitexact(F):
         np.testing.assert_array_equal(bits(a), bits(b))
 
 
+@pytest.mark.parametrize("hd", [64, 128])
+def test_attention_bwd_many_units(F, hd):
+    """Many more (tile, head) units than SMs, so that every persistent backward CTA walks
+    several units (the next unit's tiles loading while a unit's output leaves): every
+    element of dqkv written (NaN-filled before), sampled heads against the oracle, and the
+    rope table's alignment checked before any launch."""
+    nh = 32 if hd == 128 else 40
+    H = nh * hd
+    seqs = [256] * 24 + [1, 130, 300, 77, 512, 64]
+    cu = np.cumsum([0] + seqs).astype(np.int32)
+    T = int(cu[-1])
+    rng = np.random.default_rng(hd + 11)
+    qkv = rnd_bf16_f64(rng, (T, 3 * H))
+    do = rnd_bf16_f64(rng, (T, H))
+    dqkv_, dcu = dev_bf16(qkv), dev_i32(cu)
+    tiles = torch.empty(F.fl_k_attention_tiles(cu) * 2, dtype=torch.int32, device="cuda")
+    o = torch.empty((T, H), dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty((nh, T), dtype=torch.float32, device="cuda")
+    F.fl_k_attention_fwd(T, nh, hd, dqkv_, cu, dcu, tiles, o, lse)
+    rd = hd // 2
+    pos = np.concatenate([np.arange(L) for L in seqs]).astype(np.int32)
+    tab = dev_f32(rope_table(max(seqs), rd, 10000.0))
+    delta = torch.empty((nh, T), dtype=torch.float32, device="cuda")
+    dq = torch.full((T, 3 * H), float("nan"), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(F.FlError, match="aligned"):
+        F.fl_k_attention_bwd(T, nh, hd, dqkv_, o, lse, dev_bf16(do), cu, dcu, tiles, delta, tab.view(-1)[2:], rd, dq)
+    F.fl_k_attention_bwd(T, nh, hd, dqkv_, o, lse, dev_bf16(do), cu, dcu, tiles, delta, tab, rd, dq)
+    torch.cuda.synchronize()
+    got = f64(dq)
+    assert np.isfinite(got).all()
+    cos, sin = O.rope_cos_sin(pos, rd, 10000.0)
+    heads = [0, nh // 2 + 1, nh - 1]
+    sel = lambda base: np.concatenate([np.arange(base + h * hd, base + (h + 1) * hd) for h in heads])
+    q = qkv[:, sel(0)].reshape(T, len(heads), hd)
+    k = qkv[:, sel(H)].reshape(T, len(heads), hd)
+    v = qkv[:, sel(2 * H)].reshape(T, len(heads), hd)
+    dos = do[:, sel(0)].reshape(T, len(heads), hd)
+    dqr, dkr, dvr = O.attention_bwd(dos, q, k, v, cu)
+    n = len(heads) * hd
+    assert rel_inf(got[:, sel(0)], O.rope_rotate(dqr, cos, sin, rd, inverse=True).reshape(T, n)) < 5e-2
+    assert rel_inf(got[:, sel(H)], O.rope_rotate(dkr, cos, sin, rd, inverse=True).reshape(T, n)) < 5e-2
+    assert rel_inf(got[:, sel(2 * H)], dvr.reshape(T, n)) < 5e-2
+
+
 @pytest.mark.parametrize("hd,Lp", [(64, 16), (128, 100)])
 def test_attention_with_prefix(F, hd, Lp):
     """P-tuning v2 prefix (App. A): every query also sees Lp prefix keys/values (one or two
