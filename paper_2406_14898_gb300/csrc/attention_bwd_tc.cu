@@ -272,6 +272,11 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     const int k = w.kb + r;  // the key inside its segment (or the prefix)
     const bool key_ok = PREFIX ? r < Lp : k < w.L;
     const bool work = w.it0 < w.it_end;
+    // the next unit: its K / V load once this unit's last S^T / dP^T products have read K
+    // and V, its first query tile once buffer pair 0 has had its last use here
+    const int un = u + gridDim.x;
+    const Unit wn = un < n_units ? unit(un) : Unit{};
+    const bool next = un < n_units && wn.it0 < wn.it_end;
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
     if (work && !track_wait_all(bar_kv, tkv)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
@@ -313,6 +318,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
         break;
       }
       tc_fence_after();
+      if (tid == 0 && next && it + 1 == w.it_end) issue_kv(wn);
       // ---- P^T and dS^T of key row r for queries qh * 64 .. + 63, in two groups of 32,
       // each written (bf16 pairs) into the 16 columns at 64 qh + 16 hf it has just read
       {
@@ -385,16 +391,16 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
         break;
       }
       tc_fence_after();
-      if (tid == 0 && it + 2 < w.it_end) issue_q(w, it + 2, b);
+      if (tid == 0) {
+        if (it + 2 < w.it_end) issue_q(w, it + 2, b);
+        else if (b == 0 && next) issue_q(wn, wn.it0, 0);  // pair 0's last use in this unit
+      }
     }
     if (!ok) break;
 
-    // ---- every product of the unit is complete: the next unit's K / V and first query
-    // tile load into their buffers (pair 0) while this unit's dK / dV leave through pair 1
-    const int un = u + gridDim.x;
-    const Unit wn = un < n_units ? unit(un) : Unit{};
-    const bool next = un < n_units && wn.it0 < wn.it_end;
-    if (tid == 0 && next) {
+    // ---- every product of the unit is complete: this unit's dK / dV leave through pair 1
+    // while the next unit's K / V and first query tile load
+    if (tid == 0 && next && !work) {
       issue_kv(wn);
       issue_q(wn, wn.it0, 0);
     }
@@ -600,6 +606,11 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     const int q = w.q0 + r;
     const bool q_ok = q < w.L;
     const int ulim = q_ok ? max(q, w.clast) : -1;  // last own key visible to the row
+    // the next unit: its Q / dO load once this unit's last S / dP products have read them,
+    // its first key / value tile once buffer pair 0 has had its last use here
+    const int un = u + gridDim.x;
+    const Unit wn = un < n_units ? unit(un) : Unit{};
+    const bool next = un < n_units;
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
     if (!track_wait_all(bar_qdo, tqdo)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
@@ -632,6 +643,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
         break;
       }
       tc_fence_after();
+      if (tid == 0 && next && j + 1 == w.n_kv) issue_qdo(wn);
       // ---- dS of query row r for keys kh * 64 .. + 63 of the tile, in two groups of 32,
       // each written (bf16 pairs) into the 16 S columns at 64 kh + 16 hf it has just read
       {
@@ -680,20 +692,17 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
         break;
       }
       tc_fence_after();
-      if (tid == 0 && j + 2 < w.n_kv) issue_kv(w, j + 2, b);
+      if (tid == 0) {
+        if (j + 2 < w.n_kv) issue_kv(w, j + 2, b);
+        else if (b == 0 && next) issue_kv(wn, 0, 0);  // pair 0's last use in this unit
+      }
     }
     if (!ok) break;
 
-    // ---- every product of the unit is complete: the next unit's Q, dO and first key /
-    // value tiles load (pair 0) while this unit's dQ leaves through the pair-1 K buffer
-    const int un = u + gridDim.x;
-    const Unit wn = un < n_units ? unit(un) : Unit{};
-    if (tid == 0 && un < n_units) {
-      issue_qdo(wn);
-      issue_kv(wn, 0, 0);
-    }
+    // ---- every product of the unit is complete: this unit's dQ leaves through the pair-1
+    // K buffer while the next unit's Q, dO and first key / value tiles load
     float lse2n = 0.f, dln = 0.f;
-    if (un < n_units) row_stats(wn, lse2n, dln);
+    if (next) row_stats(wn, lse2n, dln);
     // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * HD/2 .. + HD/2 - 1 of
     // query row r, staged and written as whole coalesced rows, the bias column sums taken
     // from the staged rows
@@ -733,7 +742,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && un < n_units && wn.n_kv > 1) issue_kv(wn, 1, 1);
+    if (tid == 0 && next && wn.n_kv > 1) issue_kv(wn, 1, 1);
     u = un;
     w = wn;
     lse2 = lse2n;
