@@ -10,11 +10,11 @@
 // double-buffer the tiles the CTA walks through, so their loads overlap the work on the
 // previous tile.
 //
-// Both kernels are persistent: one CTA per SM (192 KB of shared memory at head_dim 128,
-// 512 TMEM columns) walks work units u = blockIdx.x, + gridDim.x, ...  Once a unit's last
-// product has completed, the next unit's first tiles are loaded into buffer pair 0 while
-// the unit's output is staged in buffer pair 1 and written; the next unit's pair-1 tiles
-// follow once the staged rows have been read.
+// Both kernels are persistent: one CTA per SM (226 KB of shared memory at head_dim 128,
+// 512 TMEM columns) walks work units u = blockIdx.x, + gridDim.x, ...  Each of the next
+// unit's tiles is loaded as soon as its buffer has had its last use in the current unit,
+// so they arrive while the unit's last products run and its output is staged (in a tile
+// of its own) and written.
 //
 // dK / dV: unit = (128-key tile, head).  Warp w reads TMEM lanes 32 (w % 4) .. + 31, so
 // thread (w, lane) owns key row r = 32 (w % 4) + lane, and takes query half w / 4 of every
@@ -67,9 +67,9 @@ struct BwdCfg {
   static constexpr int TILE = NB * BOX;  // one 128 x HD bf16 tile
   static constexpr int CH = HD / 8;      // 16-byte chunks per staged bf16 row
   static constexpr int E = HD / 4;       // rotary (cos, sin) entries per position
-  // six tiles + lse / delta of two query tiles; padded at head_dim 64 so that one CTA
-  // (512 TMEM columns) has an SM to itself
-  static constexpr int USED = 6 * TILE + 4 * TB * 4 + 1024 /*barriers, holder*/ + 1024 /*alignment*/;
+  // six operand tiles, a staging tile for the output rows, lse / delta of one query tile;
+  // padded at head_dim 64 so that one CTA (512 TMEM columns) has an SM to itself
+  static constexpr int USED = 7 * TILE + 2 * TB * 4 + 128 /*barriers, holder*/ + 1024 /*alignment*/;
   static constexpr int SMEM = USED > 120 * 1024 ? USED : 120 * 1024;
 };
 
@@ -152,9 +152,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   uint8_t* sV = smem + TILE;
   uint8_t* sQ = smem + 2 * TILE;   // [2]
   uint8_t* sdO = smem + 4 * TILE;  // [2]
-  float* sL = reinterpret_cast<float*>(smem + 6 * TILE);  // [2][128] lse * log2e of the query tile
-  float* sD = sL + 2 * TB;                                // [2][128] delta of the query tile
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sD + 2 * TB);
+  uint8_t* sST = smem + 6 * TILE;  // staging of the bf16 output rows
+  float* sL = reinterpret_cast<float*>(smem + 7 * TILE);  // [128] lse * log2e of the query tile
+  float* sD = sL + TB;                                    // [128] delta of the query tile
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sD + TB);
   uint64_t* bar_kv = bars;
   uint64_t* bar_q = bars + 1;  // [2]
   uint64_t* bar_mma1 = bars + 3;
@@ -291,8 +292,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
         const int c = tid & (TB - 1);
         const float* src = tid < TB ? lse : delta;
         const float v = c < valid ? __ldg(src + (int64_t)w.h * T + row0 + c) : 0.f;
-        if (tid < TB) sL[b * TB + c] = v * LOG2E_B;
-        else sD[b * TB + c] = v;
+        if (tid < TB) sL[c] = v * LOG2E_B;  // the previous tile's readers passed a barrier since
+        else sD[c] = v;
       }
       if (!track_wait_all(bar_q + b, b ? tq1 : tq0)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
@@ -332,8 +333,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
           qlim = key_ok ? min(w.L, q0 + 64) : q0;
           qfirst = k <= w.clast ? q0 : max(q0, k);
         }
-        const float* Lb = sL + b * TB;
-        const float* Db = sD + b * TB;
+        const float* Lb = sL;
+        const float* Db = sD;
 #pragma unroll 1
         for (int hf = 0; hf < 2; ++hf) {
           uint32_t sr[32], dr[32];
@@ -392,17 +393,22 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       }
       tc_fence_after();
       if (tid == 0) {
-        if (it + 2 < w.it_end) issue_q(w, it + 2, b);
-        else if (b == 0 && next) issue_q(wn, wn.it0, 0);  // pair 0's last use in this unit
+        if (it + 2 < w.it_end) {
+          issue_q(w, it + 2, b);
+        } else if (next) {  // pair b's last use in this unit: the next unit's tile of pair b
+          if (wn.it0 + b < wn.it_end) issue_q(wn, wn.it0 + b, b);
+          if (w.it0 + 1 == w.it_end && wn.it0 + 1 < wn.it_end) issue_q(wn, wn.it0 + 1, 1);  // pair 1 unused here
+        }
       }
     }
     if (!ok) break;
 
-    // ---- every product of the unit is complete: this unit's dK / dV leave through pair 1
-    // while the next unit's K / V and first query tile load
+    // ---- every product of the unit is complete: its dK / dV leave while the next unit's
+    // tiles load
     if (tid == 0 && next && !work) {
       issue_kv(wn);
       issue_q(wn, wn.it0, 0);
+      if (wn.it0 + 1 < wn.it_end) issue_q(wn, wn.it0 + 1, 1);
     }
     if (work) {
       if constexpr (PREFIX) {
@@ -426,13 +432,13 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
           }
         }
       } else {
-        // ---- dK (scaled, rotated back) and dV: thread (r, qh) takes dims qh * HD/2 .. +
-        // HD/2 - 1 of key row r from TMEM and stages the bf16 rows in the pair-1 Q (dK) and
-        // dO (dV) buffers, then the CTA writes whole rows with coalesced 16-byte stores; the
-        // bias column sums are taken from the staged rows (the values stored)
+        // ---- dK (scaled, rotated back), then dV: thread (r, qh) takes dims qh * HD/2 .. +
+        // HD/2 - 1 of key row r from TMEM and stages the bf16 rows, then the CTA writes whole
+        // rows with coalesced 16-byte stores; the bias column sums are taken from the staged
+        // rows (the values stored)
 #pragma unroll 1
         for (int part = 0; part < 2; ++part) {  // 0: dK, 1: dV
-          uint8_t* stage = part ? sdO + TILE : sQ + TILE;
+          uint8_t* stage = sST;
           uint32_t vr[HD / 2];
 #pragma unroll
           for (int c = 0; c < HD / 2; c += 32)
@@ -463,15 +469,13 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
               *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.kb + row) * 3 * H + col + jc * 8) =
                   *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
           }
+          __syncthreads();  // the staged rows have been read
         }
       }
     }
-    // the staged rows have been read and the dK / dV columns loaded before the pair-1
-    // buffers are loaded again and the next unit's products overwrite the accumulators
-    fence_proxy_async_smem();
+    // the dK / dV columns are loaded before the next unit's products overwrite them
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && next && wn.it0 + 1 < wn.it_end) issue_q(wn, wn.it0 + 1, 1);
     u = un;
     w = wn;
   }
@@ -508,7 +512,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   uint8_t* sdO = smem + TILE;
   uint8_t* sK = smem + 2 * TILE;  // [2]
   uint8_t* sV = smem + 4 * TILE;  // [2]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 6 * TILE + 4 * TB * 4);
+  uint8_t* sST = smem + 6 * TILE;  // staging of the bf16 output rows
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * TILE + 2 * TB * 4);
   uint64_t* bar_qdo = bars;
   uint64_t* bar_kv = bars + 1;  // [2]
   uint64_t* bar_mma1 = bars + 3;
@@ -693,21 +698,25 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
       }
       tc_fence_after();
       if (tid == 0) {
-        if (j + 2 < w.n_kv) issue_kv(w, j + 2, b);
-        else if (b == 0 && next) issue_kv(wn, 0, 0);  // pair 0's last use in this unit
+        if (j + 2 < w.n_kv) {
+          issue_kv(w, j + 2, b);
+        } else if (next) {  // pair b's last use in this unit: the next unit's tile of pair b
+          if (b < wn.n_kv) issue_kv(wn, b, b);
+          if (w.n_kv == 1 && wn.n_kv > 1) issue_kv(wn, 1, 1);  // pair 1 unused here
+        }
       }
     }
     if (!ok) break;
 
-    // ---- every product of the unit is complete: this unit's dQ leaves through the pair-1
-    // K buffer while the next unit's Q, dO and first key / value tiles load
+    // ---- every product of the unit is complete: its dQ leaves while the next unit's tiles
+    // load
     float lse2n = 0.f, dln = 0.f;
     if (next) row_stats(wn, lse2n, dln);
     // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * HD/2 .. + HD/2 - 1 of
     // query row r, staged and written as whole coalesced rows, the bias column sums taken
     // from the staged rows
     {
-      uint8_t* stage = sK + TILE;
+      uint8_t* stage = sST;
       uint32_t vr[HD / 2];
 #pragma unroll
       for (int c = 0; c < HD / 2; c += 32)
@@ -737,12 +746,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
               *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
       }
     }
-    // the staged rows have been read and the dQ columns loaded before the pair-1 buffers
-    // are loaded again and the next unit's products overwrite the accumulator
-    fence_proxy_async_smem();
+    // the staged rows have been read and the dQ columns loaded before the next unit's
+    // epilogue and products reuse them
     tc_fence_before();
     __syncthreads();
-    if (tid == 0 && next && wn.n_kv > 1) issue_kv(wn, 1, 1);
     u = un;
     w = wn;
     lse2 = lse2n;
