@@ -112,6 +112,21 @@ typedef struct {
 
 int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);
 
+/* n (1..FL_GEMM_MAX_BATCH) problems of one shape run as one launch, each with its own
+ * pointers: problem r's tiles follow problem r-1's in one persistent grid, so the last wave
+ * of one problem is filled by the next (e.g. the weight gradients of several matrices of
+ * one block, which the backward of §3.1 produces side by side).  Every problem is checked
+ * as by fl_k_gemm and must share M, N, K, the operand layouts, the epilogue and its
+ * scalars (alpha, AdamW hyper-parameters, RoPE arguments and table), tile, and the output
+ * leading dimensions ldd, ld_aux, ld_aux_out; A, B, lda and ldb are free per problem.  An
+ * optional operand (aux, aux_out, bias, colsum, pos, pos2, LayerNorm, Adam moments) is
+ * given for every problem or for none; pos / pos2 / ln_mean / ln_rstd of one problem lie
+ * at one offset from problem 0's, as do ln_gamma / ln_beta, bias / colsum, adam_m /
+ * adam_v.  batch must be 0 or 1 in every entry.  Results are bit-identical to launching
+ * the problems one by one.  Errors: INVALID_ARG (as fl_k_gemm, or the problems differ),
+ * UNSUPPORTED, CUDA. */
+int fl_k_gemm_multi(const fl_gemm_args* probs, int32_t n, int* status, void* stream);
+
 /* Row LayerNorm, biased variance, fp32 statistics.  x: [T,H] of x_dtype (bf16 or fp32);
  * y: bf16 [T,H]; mean, rstd: [T].  H a power of two in [256, 4096]. */
 int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x_dtype, const float* gamma,

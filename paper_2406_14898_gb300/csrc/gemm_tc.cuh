@@ -66,8 +66,20 @@ struct Epi {
   float *adam_m, *adam_v;
   float lr, b1, b2, eps, wd, inv_bc1, inv_bc2;
   float* colsum;  // GELU_BWD: column sums of D added here (bias gradient of the up-projection)
-  // batched launch: element strides between the problems' pointers (fl_gemm_args)
-  int64_t bs_d, bs_aux, bs_aux_out, bs_bias, bs_row, bs_lnp, bs_adam;
+  // launch of several problems: element offsets of problem r's pointers from problem 0's
+  // (entry 0 unused, always 0): D, aux, aux_out, bias / colsum, the per-row arrays (pos,
+  // pos2, LayerNorm statistics), LayerNorm gain / shift, Adam moments
+  int64_t o_d[FL_GEMM_MAX_BATCH], o_aux[FL_GEMM_MAX_BATCH], o_aux_out[FL_GEMM_MAX_BATCH],
+      o_bias[FL_GEMM_MAX_BATCH], o_row[FL_GEMM_MAX_BATCH], o_lnp[FL_GEMM_MAX_BATCH], o_adam[FL_GEMM_MAX_BATCH];
+};
+
+// The operands of the problems of one launch: A and B of problem r with their leading
+// dimensions (tensor maps are built from these on the host).
+struct Problems {
+  int n;
+  const void* A[FL_GEMM_MAX_BATCH];
+  const void* B[FL_GEMM_MAX_BATCH];
+  int64_t lda[FL_GEMM_MAX_BATCH], ldb[FL_GEMM_MAX_BATCH];
 };
 
 // Tensor maps of the A and B operands of up to FL_GEMM_MAX_BATCH problems (a kernel
@@ -104,11 +116,19 @@ FL_DEV void st_quad(__nv_bfloat16* p, float4 v) {
 // columns n0 + 4 (l % 16) .. + 3, so every warp-wide access covers two 64-column rows
 // (256 B of bf16 or 512 B of fp32).  Rows go in batches of RB row pairs: all global loads of
 // a batch are issued before any of its arithmetic.
+// Entry r of a per-problem offset array (constant indices only: no local copy of the
+// parameter struct).
+FL_DEV int64_t prob_off(const int64_t (&o)[FL_GEMM_MAX_BATCH], int r) {
+  static_assert(FL_GEMM_MAX_BATCH == 4, "prob_off selects among four problems");
+  return r == 0 ? 0 : r == 1 ? o[1] : r == 2 ? o[2] : o[3];
+}
+
 template <int FAM>
 FL_DEV void epilogue_chunk(const Epi& e, int r, const float* stage, int row0, int rows, int n0, int lane) {
-  // problem r of a batched launch: element offsets of its pointers (0 for r = 0)
-  const int64_t od = r * e.bs_d, oaux = r * e.bs_aux, oauxo = r * e.bs_aux_out, ob = r * e.bs_bias,
-                orow = r * e.bs_row, olnp = r * e.bs_lnp, oad = r * e.bs_adam;
+  // problem r of a multi-problem launch: element offsets of its pointers (0 for r = 0)
+  const int64_t od = prob_off(e.o_d, r), oaux = prob_off(e.o_aux, r), oauxo = prob_off(e.o_aux_out, r),
+                ob = prob_off(e.o_bias, r), orow = prob_off(e.o_row, r), olnp = prob_off(e.o_lnp, r),
+                oad = prob_off(e.o_adam, r);
   constexpr int RB = (FAM == FAM_GELU || FAM == FAM_ROPE) ? 16 : 8;  // row pairs per batch
   const int h = lane >> 4, cl = lane & 15;
   const int n = n0 + 4 * cl;
@@ -787,7 +807,7 @@ inline Raster pick_raster(int M, int N, int K, int bm, int bn) {
 }
 
 template <int BN, bool A_MN, bool B_MN, int FAM>
-int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) {
+int launch(const fl_gemm_args* a, const Problems& pr, const Epi& epi, int* status, cudaStream_t st) {
   using C = Cfg<BN>;
   auto kern = gemm_tc_kernel<BN, A_MN, B_MN, FAM>;
   static bool attr_set = false;  // per instantiation; the attribute is per device function
@@ -796,17 +816,15 @@ int launch(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) 
     attr_set = true;
   }
   GemmMaps maps;
-  const int batch = a->batch > 1 ? a->batch : 1;
+  const int batch = pr.n;
   for (int r = 0; r < batch; ++r) {
-    const void* A = static_cast<const __nv_bfloat16*>(a->A) + r * a->a_bstride;
-    const void* B = static_cast<const __nv_bfloat16*>(a->B) + r * a->b_bstride;
     int rc;
     // A(m,k): K-major -> [M rows, K inner]; MN-major -> [K rows, M inner]
-    if (!A_MN) rc = make_map(&maps.a[r], A, a->K, a->M, a->lda, BM);
-    else rc = make_map(&maps.a[r], A, a->M, a->K, a->lda, BK);
+    if (!A_MN) rc = make_map(&maps.a[r], pr.A[r], a->K, a->M, pr.lda[r], BM);
+    else rc = make_map(&maps.a[r], pr.A[r], a->M, a->K, pr.lda[r], BK);
     if (rc) return rc;
-    if (!B_MN) rc = make_map(&maps.b[r], B, a->K, a->N, a->ldb, BN);
-    else rc = make_map(&maps.b[r], B, a->N, a->K, a->ldb, BK);
+    if (!B_MN) rc = make_map(&maps.b[r], pr.B[r], a->K, a->N, pr.ldb[r], BN);
+    else rc = make_map(&maps.b[r], pr.B[r], a->N, a->K, pr.ldb[r], BK);
     if (rc) return rc;
   }
   const int num_m = (a->M + BM - 1) / BM, num_n = a->N / BN;
@@ -846,22 +864,20 @@ int pair_slots() {
 }
 
 template <bool A_MN, bool B_MN, int FAM>
-int launch_pair(const fl_gemm_args* a, const Epi& epi, int* status, cudaStream_t st) {
+int launch_pair(const fl_gemm_args* a, const Problems& pr, const Epi& epi, int* status, cudaStream_t st) {
   auto kern = gemm_pair_kernel<A_MN, B_MN, FAM>;
   const int slots = pair_slots<A_MN, B_MN, FAM>();
   if (slots <= 0) return fl_internal_error(FL_ERR_CUDA, "gemm: the CTA-pair kernel cannot be resident");
   GemmMaps maps;
-  const int batch = a->batch > 1 ? a->batch : 1;
+  const int batch = pr.n;
   for (int r = 0; r < batch; ++r) {
-    const void* A = static_cast<const __nv_bfloat16*>(a->A) + r * a->a_bstride;
-    const void* B = static_cast<const __nv_bfloat16*>(a->B) + r * a->b_bstride;
     int rc;
     // each CTA loads 128 rows of A and 128 columns of B per k-block
-    if (!A_MN) rc = make_map(&maps.a[r], A, a->K, a->M, a->lda, 128);
-    else rc = make_map(&maps.a[r], A, a->M, a->K, a->lda, BK);
+    if (!A_MN) rc = make_map(&maps.a[r], pr.A[r], a->K, a->M, pr.lda[r], 128);
+    else rc = make_map(&maps.a[r], pr.A[r], a->M, a->K, pr.lda[r], BK);
     if (rc) return rc;
-    if (!B_MN) rc = make_map(&maps.b[r], B, a->K, a->N, a->ldb, 128);
-    else rc = make_map(&maps.b[r], B, a->N, a->K, a->ldb, BK);
+    if (!B_MN) rc = make_map(&maps.b[r], pr.B[r], a->K, a->N, pr.ldb[r], 128);
+    else rc = make_map(&maps.b[r], pr.B[r], a->N, a->K, pr.ldb[r], BK);
     if (rc) return rc;
   }
   const int tiles = batch * ((a->M + PAIR_BM - 1) / PAIR_BM) * (a->N / PAIR_BN);
@@ -895,21 +911,21 @@ inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
   template int pair_slots<AMN, BMN, FAM_RESID>();                                                      \
   template int pair_slots<AMN, BMN, FAM_ROPE>();                                                       \
   template int pair_slots<AMN, BMN, FAM_ADAMW>();                                                      \
-  template int launch_pair<AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch_pair<AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
-  template int launch_pair<AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch_pair<AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
-  template int launch_pair<AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch<256, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch<128, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch<256, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
-  template int launch<128, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
-  template int launch<256, AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch<128, AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch<256, AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
-  template int launch<128, AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);  \
-  template int launch<256, AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Epi&, int*, cudaStream_t); \
-  template int launch<128, AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Epi&, int*, cudaStream_t);
+  template int launch_pair<AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch_pair<AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);  \
+  template int launch_pair<AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch_pair<AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);  \
+  template int launch_pair<AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch<256, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch<128, AMN, BMN, FAM_PLAIN>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch<256, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);  \
+  template int launch<128, AMN, BMN, FAM_GELU>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);  \
+  template int launch<256, AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch<128, AMN, BMN, FAM_RESID>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch<256, AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);  \
+  template int launch<128, AMN, BMN, FAM_ROPE>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);  \
+  template int launch<256, AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t); \
+  template int launch<128, AMN, BMN, FAM_ADAMW>(const fl_gemm_args*, const Problems&, const Epi&, int*, cudaStream_t);
 
 }  // namespace fl_gemm
 

@@ -64,6 +64,8 @@ int fl_launch_fill(int64_t n, float v, float* out, cudaStream_t st);
 int fl_launch_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
                     float beta2, float eps, float weight_decay, float bc1, float bc2, int zero_grad, cudaStream_t st);
 int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st);
+// dst [cols, rows] = the transpose of src [rows, cols] (fp32; src and dst do not overlap).
+int fl_launch_transpose_f32(int64_t rows, int64_t cols, const float* src, float* dst, cudaStream_t st);
 
 // P-tuning v2 prefix of one block's attention: bf16 keys/values [len, H] (head j at
 // column j*head_dim) seen by every query, and fp32 gradient accumulators (backward).

@@ -749,6 +749,32 @@ int fl_launch_mean_finish(int64_t n, int n_replicas, float* w, void* wb, cudaStr
   return FL_OK;
 }
 
+// dst[c][r] = src[r][c] for src [rows, cols] (fp32), through 32 x 32 shared-memory tiles so
+// that both the reads and the writes are coalesced; blockDim (32, 8).
+__global__ void transpose_f32_kernel(int64_t rows, int64_t cols, const float* __restrict__ src,
+                                     float* __restrict__ dst) {
+  __shared__ float tile[32][33];
+  const int64_t r0 = (int64_t)blockIdx.y * 32, c0 = (int64_t)blockIdx.x * 32;
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int64_t r = r0 + i, c = c0 + threadIdx.x;
+    if (r < rows && c < cols) tile[i][threadIdx.x] = src[r * cols + c];
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += 8) {
+    const int64_t c = c0 + i, r = r0 + threadIdx.x;
+    if (r < rows && c < cols) dst[c * rows + r] = tile[threadIdx.x][i];
+  }
+}
+
+int fl_launch_transpose_f32(int64_t rows, int64_t cols, const float* src, float* dst, cudaStream_t st) {
+  if (rows <= 0 || cols <= 0) return FL_OK;
+  const int64_t gx = (cols + 31) / 32, gy = (rows + 31) / 32;
+  if (gy > 65535) return fl_internal_error(FL_ERR_UNSUPPORTED, "transpose: %lld rows", (long long)rows);
+  transpose_f32_kernel<<<dim3((unsigned)gx, (unsigned)gy), dim3(32, 8), 0, st>>>(rows, cols, src, dst);
+  FL_CUDA_TRY(cudaGetLastError());
+  return FL_OK;
+}
+
 int fl_launch_f32_to_bf16(int64_t n, const float* src, void* dst, cudaStream_t st) {
   if (n <= 0) return FL_OK;
   f32_to_bf16_kernel<<<grid_for(n), 256, 0, st>>>(n, src, (__nv_bfloat16*)dst);

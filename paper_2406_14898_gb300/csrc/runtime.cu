@@ -11,7 +11,10 @@
 //                     every parameter: first the four weight matrices of every block
 //                     (block b at b * mat_stride), then the bias and LayerNorm vectors of
 //                     every block in one contiguous region (block b at vec_base +
-//                     b * vec_stride); every tensor 64-byte aligned; with cfg.n_replicas
+//                     b * vec_stride); every tensor 64-byte aligned; the FFN up-projection
+//                     weight is stored transposed ([H, F]: its weight gradient then has the
+//                     down-projection's shape and the two run as one launch; the parameter
+//                     access functions transpose on the host); with cfg.n_replicas
 //                     = R > 1 each arena holds R such layouts back to back (replica r at
 //                     r * n_params), and replica r trains on the r-th of R equal, contiguous
 //                     token groups of each call (§3.3 server-hierarchical on one GPU): the
@@ -301,6 +304,14 @@ int run_gemm(fl_server* h, fl_gemm_args a, bool wgrad = false) {
   return rc;
 }
 
+// Several problems of one shape as one launch (fl_k_gemm_multi; one replica).
+int run_gemm_multi(fl_server* h, const fl_gemm_args* probs, int n) {
+  prof_begin(h, FL_PROF_GEMM);
+  int rc = fl_k_gemm_multi(probs, n, h->status, h->stream);
+  prof_end(h);
+  return rc;
+}
+
 fl_gemm_args gemm_fwd(int M, int N, int K, const void* A, const void* W, void* D, int epi) {
   fl_gemm_args a;
   memset(&a, 0, sizeof a);
@@ -334,17 +345,20 @@ fl_gemm_args gemm_wgrad_raw(int T, int Nout, int Kin, const void* dY, const void
   return a;
 }
 
-// Weight gradient of weight matrix t of block b: stored / accumulated into the gradient
-// arena, or, inside a fused backward + step, applied to the weight by AdamW directly.
-fl_gemm_args gemm_wgrad(fl_server* h, int b, int t, int T, int Nout, int Kin, const void* dY, const void* X) {
-  fl_gemm_args a = gemm_wgrad_raw(T, Nout, Kin, dY, X, h->gt(b, t), h->grads_zero);
+// Weight gradient of weight matrix t of block b (from element e0 of it on: a block of rows,
+// whose gradient dY has row stride ldy): stored / accumulated into the gradient arena, or,
+// inside a fused backward + step, applied to the weight by AdamW directly.
+fl_gemm_args gemm_wgrad(fl_server* h, int b, int t, int T, int Nout, int Kin, const void* dY, const void* X,
+                        int64_t e0 = 0, int64_t ldy = 0) {
+  fl_gemm_args a = gemm_wgrad_raw(T, Nout, Kin, dY, X, h->gt(b, t) + e0, h->grads_zero);
+  if (ldy) a.lda = ldy;
   if (h->fuse.on) {
     const fl_server_cfg& c = h->cfg;
     a.epilogue = FL_EPI_ADAMW;
-    a.D = h->wt(b, t);
-    a.adam_m = h->m + h->off(b, t);
-    a.adam_v = h->v + h->off(b, t);
-    a.aux_out = h->wbt(b, t);
+    a.D = h->wt(b, t) + e0;
+    a.adam_m = h->m + h->off(b, t) + e0;
+    a.adam_v = h->v + h->off(b, t) + e0;
+    a.aux_out = h->wbt(b, t) + e0;
     a.ld_aux_out = Kin;
     a.lr = h->fuse.lr;
     a.beta1 = c.adam_beta1;
@@ -420,6 +434,8 @@ int block_forward(fl_server* h, int b, bool output = true) {
   prof_end(h);
   // u = m W1^T + b1, g = gelu(u)
   fl_gemm_args g3 = gemm_fwd(T, F, H, A.m, h->wbt(b, FL_T_WUP), A.g, FL_EPI_BIAS_GELU);
+  g3.b_mn_major = 1;  // W1 stored transposed, [H, F]
+  g3.ldb = F;
   g3.bias = h->wt(b, FL_T_BUP);
   g3.aux_out = A.u;
   g3.ld_aux_out = F;
@@ -456,22 +472,20 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
   // produce those: db2 (dy) by the LayerNorm-1 backward of block b + 1 (here by a column-sum
   // kernel for the top block, whose dy comes from the clients), db1 (du) by the GeLU'
   // epilogue, dbd (dh) by the LayerNorm-2 backward, dbqkv (dqkv) by the attention backward.
-  // FFN down: du = (dy W2) * gelu'(u), db1 += colsum(du); dW2 += dy^T g
+  // Weight gradients run after the data gradients that read the same weights (a fused
+  // step updates the weight in the gradient's epilogue), two or four matrices per launch
+  // with one replica: [dW2, dW1^T] (both [H, F]) and [dWd, dWq, dWk, dWv] (all [H, H]), so
+  // that one matrix's last wave is filled by the next.
+  // FFN down: du = (dy W2) * gelu'(u), db1 += colsum(du)
   fl_gemm_args d1 = gemm_dgrad(T, F, H, dy, h->wbt(b, FL_T_WDOWN), h->du, FL_EPI_GELU_BWD);
   d1.aux = A.u;
   d1.ld_aux = F;
   d1.colsum = train_base ? h->gt(b, FL_T_BUP) : nullptr;
   TRY(h, run_gemm(h, d1));
-  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g), true));
-    if (b == c.n_blocks - 1) {
-      prof_begin(h, FL_PROF_OTHER, h->R);
-      for (int r = 0; r < h->R; ++r) TRY(h, fl_k_colsum(T, H, dy + (int64_t)r * T * H, h->gt(b, FL_T_BDOWN, r), st));
-      prof_end(h);
-    }
-  }
-  // FFN up: dm = du W1 (+ alpha dy), fp32; dW1 += du^T m
+  // FFN up: dm = du W1 (+ alpha dy), fp32 (W1 stored transposed: a K-major operand)
   fl_gemm_args d2 = gemm_dgrad(T, H, F, h->du, h->wbt(b, FL_T_WUP), h->dm, glm ? FL_EPI_RESID : FL_EPI_STORE);
+  d2.b_mn_major = 0;
+  d2.ldb = F;
   d2.d_dtype = FL_DT_F32;
   if (glm) {
     d2.aux = dyf;
@@ -480,8 +494,22 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d2.alpha = al;
   }
   TRY(h, run_gemm(h, d2));
-  if (train_base)  // weight gradient (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WUP, T, F, H, h->du, A.m), true));
+  if (train_base) {  // weight and bias gradients (skipped when only the prefixes train)
+    // dW2 (+)= dy^T g, dW1^T (+)= m^T du
+    const fl_gemm_args ffn[2] = {gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g),
+                                 gemm_wgrad(h, b, FL_T_WUP, T, H, F, A.m, h->du)};
+    if (h->R == 1) {
+      TRY(h, run_gemm_multi(h, ffn, 2));
+    } else {
+      TRY(h, run_gemm(h, ffn[0], true));
+      TRY(h, run_gemm(h, ffn[1], true));
+    }
+    if (b == c.n_blocks - 1) {
+      prof_begin(h, FL_PROF_OTHER, h->R);
+      for (int r = 0; r < h->R; ++r) TRY(h, fl_k_colsum(T, H, dy + (int64_t)r * T * H, h->gt(b, FL_T_BDOWN, r), st));
+      prof_end(h);
+    }
+  }
   // LN2 backward: dh = LN2'(dm) (+ alpha dy), bf16 and fp32; dbd += colsum(dh)
   prof_begin(h, FL_PROF_LN, 2 * h->R);
   for (int r = 0; r < h->R; ++r) {
@@ -492,10 +520,8 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
                                        train_base ? h->gt(b, FL_T_BDENSE, r) : nullptr, h->ln_ws, st, h->status));
   }
   prof_end(h);
-  // dense: do = dh Wd; dWd += dh^T o
+  // dense: do = dh Wd
   TRY(h, run_gemm(h, gemm_dgrad(T, H, H, h->dh, h->wbt(b, FL_T_WDENSE), h->d_o, FL_EPI_STORE)));
-  if (train_base)  // weight gradient (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o), true));
   // attention backward -> dqkv (w.r.t. the un-rotated q, k); dbqkv += colsum(dqkv)
   prof_begin(h, FL_PROF_ATTN, 3);
   TRY(h, fl_launch_attn_bwd(h->T, c.n_heads, c.head_dim, A.qkv, A.o, A.lse, h->d_o, h->cu, h->tiles, h->n_tiles,
@@ -503,7 +529,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
                             train_base ? h->gt(b, FL_T_BQKV) : nullptr, h->status, h->R > 1 ? h->Sr : 0,
                             h->n_params));
   prof_end(h);
-  // QKV: da = dqkv Wqkv (+ alpha dh), fp32; dWqkv += dqkv^T a
+  // QKV: da = dqkv Wqkv (+ alpha dh), fp32
   fl_gemm_args d3 = gemm_dgrad(T, H, 3 * H, h->dqkv, h->wbt(b, FL_T_WQKV), h->da, glm ? FL_EPI_RESID : FL_EPI_STORE);
   d3.d_dtype = FL_DT_F32;
   if (glm) {
@@ -513,8 +539,18 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     d3.alpha = al;
   }
   TRY(h, run_gemm(h, d3));
-  if (train_base)  // weight gradient (skipped when only the prefixes train)
-    TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a), true));
+  if (train_base) {  // weight gradients (skipped when only the prefixes train)
+    if (h->R == 1) {
+      // dWd (+)= dh^T o; rows r H .. of dWqkv (+)= dqkv[:, r H ..]^T a, r = 0, 1, 2
+      fl_gemm_args att[4] = {gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)};
+      for (int r = 0; r < 3; ++r)
+        att[1 + r] = gemm_wgrad(h, b, FL_T_WQKV, T, H, H, h->dqkv + (int64_t)r * H, A.a, (int64_t)r * H * H, 3 * H);
+      TRY(h, run_gemm_multi(h, att, 4));
+    } else {
+      TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o), true));
+      TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a), true));
+    }
+  }
   // LN1 backward: dx = LN1'(da) (+ alpha dh), bf16 and fp32; dx is dy of block b - 1, whose
   // down-projection bias gradient is its column sum
   prof_begin(h, FL_PROF_LN, 2 * h->R);
@@ -687,7 +723,16 @@ int fl_server_create_keyed(const fl_server_cfg* cfg, uint64_t seed, int purpose,
       float* p = h->wt(b, t);
       if (t == FL_T_LN1_G || t == FL_T_LN2_G) rc = fl_launch_fill(h->tensor_n[t], 1.f, p, st);
       else if (t == FL_T_LN1_B || t == FL_T_LN2_B) rc = fl_launch_fill(h->tensor_n[t], 0.f, p, st);
-      else
+      else if (t == FL_T_WUP) {
+        // drawn in the [F, H] order of its stream into the (zero) gradient arena, then
+        // transposed into place and the scratch cleared
+        float* tmp = h->gt(b, t);
+        rc = fl_launch_normal_init(h->tensor_n[t], stream_key(seed, (uint64_t)purpose, (uint64_t)(block0 + b), t, 0),
+                                   0.0, (double)c.init_std, tmp, st);
+        if (!rc) rc = fl_launch_transpose_f32(F, H, tmp, p, st);
+        if (!rc && cudaMemsetAsync(tmp, 0, h->tensor_n[t] * sizeof(float), st) != cudaSuccess)
+          rc = fl_internal_cuda_error(cudaGetLastError(), "create: clear", __FILE__, __LINE__);
+      } else
         rc = fl_launch_normal_init(h->tensor_n[t], stream_key(seed, (uint64_t)purpose, (uint64_t)(block0 + b), t, 0), 0.0,
                                    (double)c.init_std, p, st);
       if (rc) return fail(rc);
@@ -944,6 +989,12 @@ static int check_tensor(fl_server* h, int32_t b, int32_t t, const void* p, size_
   return FL_OK;
 }
 
+// dst[c * rows + r] = src[r * cols + c]
+static void transpose_host(const float* src, float* dst, int64_t rows, int64_t cols) {
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t c = 0; c < cols; ++c) dst[c * rows + r] = src[r * cols + c];
+}
+
 static int d2h(fl_server* h, float* dst, const float* src, size_t n) {
   cudaError_t e = cudaStreamSynchronize(h->stream);
   if (e == cudaSuccess) e = cudaMemcpy(dst, src, n * sizeof(float), cudaMemcpyDeviceToHost);
@@ -951,9 +1002,19 @@ static int d2h(fl_server* h, float* dst, const float* src, size_t n) {
   return FL_OK;
 }
 
+// Copies tensor t's arena values (at src) to dst in the tensor's own [rows, cols] order:
+// the FFN up-projection weight, stored [H, F], is transposed back to [F, H].
+static int d2h_tensor(fl_server* h, int t, float* dst, const float* src, size_t n) {
+  if (t != FL_T_WUP) return d2h(h, dst, src, n);
+  std::vector<float> tmp(n);
+  if (int rc = d2h(h, tmp.data(), src, n)) return rc;
+  transpose_host(tmp.data(), dst, h->cfg.hidden, h->cfg.ffn_hidden);
+  return FL_OK;
+}
+
 extern "C" int fl_server_get_param(fl_server_t h, int32_t b, int32_t t, float* dst, size_t n) {
   if (int rc = check_tensor(h, b, t, dst, n)) return rc;
-  return d2h(h, dst, h->wt(b, t), n);
+  return d2h_tensor(h, t, dst, h->wt(b, t), n);
 }
 extern "C" int fl_server_get_grad(fl_server_t h, int32_t b, int32_t t, float* dst, size_t n) {
   if (int rc = check_tensor(h, b, t, dst, n)) return rc;
@@ -961,22 +1022,28 @@ extern "C" int fl_server_get_grad(fl_server_t h, int32_t b, int32_t t, float* ds
     memset(dst, 0, n * sizeof(float));
     return FL_OK;
   }
-  return d2h(h, dst, h->gt(b, t), n);
+  return d2h_tensor(h, t, dst, h->gt(b, t), n);
 }
 extern "C" int fl_server_get_adam_moments(fl_server_t h, int32_t b, int32_t t, float* hm, float* hv, size_t n) {
   if (int rc = check_tensor(h, b, t, hm, n)) return rc;
   if (!hv) return set_err(h, FL_ERR_INVALID_ARG, "null host buffer");
   const int64_t o = h->off(b, t);
-  if (int rc = d2h(h, hm, h->m + o, n)) return rc;
-  return d2h(h, hv, h->v + o, n);
+  if (int rc = d2h_tensor(h, t, hm, h->m + o, n)) return rc;
+  return d2h_tensor(h, t, hv, h->v + o, n);
 }
 extern "C" int fl_server_get_replica_param(fl_server_t h, int32_t r, int32_t b, int32_t t, float* dst, size_t n) {
   if (int rc = check_tensor(h, b, t, dst, n)) return rc;
   if (r < 0 || r >= h->R) return set_err(h, FL_ERR_INVALID_ARG, "replica %d outside [0, %d)", r, h->R);
-  return d2h(h, dst, h->wt(b, t, r), n);
+  return d2h_tensor(h, t, dst, h->wt(b, t, r), n);
 }
 extern "C" int fl_server_set_param(fl_server_t h, int32_t b, int32_t t, const float* src, size_t n) {
   if (int rc = check_tensor(h, b, t, src, n)) return rc;
+  std::vector<float> tmp;
+  if (t == FL_T_WUP) {  // stored transposed, [H, F]
+    tmp.resize(n);
+    transpose_host(src, tmp.data(), h->cfg.ffn_hidden, h->cfg.hidden);
+    src = tmp.data();
+  }
   cudaError_t e = cudaStreamSynchronize(h->stream);
   for (int r = 0; r < h->R && e == cudaSuccess; ++r)  // every replica
     e = cudaMemcpy(h->wt(b, t, r), src, n * sizeof(float), cudaMemcpyHostToDevice);

@@ -107,6 +107,7 @@ _SIGS = {
     "fl_server_launch_count": (_I64, [_P]),
     "fl_server_last_error": (C.c_char_p, [_P]),
     "fl_k_gemm": (C.c_int, [C.POINTER(fl_gemm_args), _P, _P]),
+    "fl_k_gemm_multi": (C.c_int, [C.POINTER(fl_gemm_args), _I32, _P, _P]),
     "fl_k_layernorm_fwd": (C.c_int, [_I32, _I32, _P, _I32, _P, _P, _F, _P, _P, _P, _P]),
     "fl_k_layernorm_bwd_workspace": (C.c_size_t, [_I32, _I32]),
     "fl_k_layernorm_bwd": (C.c_int, [_I32, _I32, _P, _P, _I32, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P, _P]),
@@ -437,10 +438,20 @@ def fl_k_gemm(args: fl_gemm_args, status=None, stream=None):
     check(lib().fl_k_gemm(C.byref(args), ptr(status), stream_ptr(stream)))
 
 
-def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
-         alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
-         aux_dtype=FL_DT_BF16, d_dtype=FL_DT_BF16, ln_mean=None, ln_rstd=None, ln_gamma=None, ln_beta=None,
-         pos2=None, tile=0, colsum=None, status=None, stream=None, batch=1, bstrides=None, **fields):
+def fl_k_gemm_multi(args: Sequence[fl_gemm_args], status=None, stream=None):
+    arr = (fl_gemm_args * len(args))(*args)
+    check(lib().fl_k_gemm_multi(arr, len(args), ptr(status), stream_ptr(stream)))
+
+
+def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, status=None, stream=None, **kw):
+    """One fl_k_gemm call; arguments as gemm_args."""
+    fl_k_gemm(gemm_args(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, **kw), status, stream)
+
+
+def gemm_args(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bias=None, aux=None, ld_aux=0,
+              alpha=0.0, aux_out=None, ld_aux_out=0, pos=None, rope_tab=None, n_heads=0, head_dim=0, rotary_dim=0,
+              aux_dtype=FL_DT_BF16, d_dtype=FL_DT_BF16, ln_mean=None, ln_rstd=None, ln_gamma=None, ln_beta=None,
+              pos2=None, tile=0, colsum=None, batch=1, bstrides=None, **fields) -> fl_gemm_args:
     """bstrides: {"a": .., "b": .., "d": .., "aux": .., "aux_out": .., "bias": .., "row": .., "lnp": ..,
     "adam": ..} element strides between the problems of a batched launch; `fields` sets any
     other fl_gemm_args field by name (tensors as device pointers)."""
@@ -455,7 +466,7 @@ def gemm(M, N, K, A, lda, a_mn, B, ldb, b_mn, D, ldd, epilogue=FL_EPI_STORE, bia
         setattr(a, f"{k}_bstride", int(v))
     for k, v in fields.items():
         setattr(a, k, v if isinstance(v, (int, float)) else ptr(v))
-    fl_k_gemm(a, status, stream)
+    return a
 
 
 def fl_k_layernorm_fwd(T, H, x, gamma, beta, eps, y, mean, rstd, x_dtype=FL_DT_BF16, stream=None):

@@ -200,3 +200,98 @@ def test_batched_adamw(F, tile):
                                     inv_bc2=1 / 0.002997)
     for k in ("D", "adam_m", "adam_v", "aux_out"):
         _cmp(bat[k], sep[k])
+
+
+# ---------------------------------------------------------------- fl_k_gemm_multi
+def test_multi_argument_errors(F):
+    A = torch.zeros((128, 64), dtype=torch.bfloat16, device="cuda")
+    D = torch.zeros((128, 128), dtype=torch.bfloat16, device="cuda")
+    a0 = F.gemm_args(128, 128, 64, A, 64, 0, A, 64, 0, D, 128)
+    with pytest.raises(F.FlError):
+        F.fl_k_gemm_multi([a0] * (F.FL_GEMM_MAX_BATCH + 1))
+    with pytest.raises(F.FlError, match="differs"):  # another M
+        F.fl_k_gemm_multi([a0, F.gemm_args(64, 128, 64, A, 64, 0, A, 64, 0, D, 128)])
+    with pytest.raises(F.FlError, match="differs"):  # another epilogue
+        F.fl_k_gemm_multi([a0, F.gemm_args(128, 128, 64, A, 64, 0, A, 64, 0, D, 128, epilogue=F.FL_EPI_STORE_F32)])
+    bias = torch.zeros(128, dtype=torch.float32, device="cuda")
+    with pytest.raises(F.FlError, match="lacks"):  # a bias in one problem only
+        F.fl_k_gemm_multi([a0, F.gemm_args(128, 128, 64, A, 64, 0, A, 64, 0, D, 128, bias=bias)])
+    with pytest.raises(F.FlError):  # a batched entry
+        F.fl_k_gemm_multi([a0, F.gemm_args(128, 128, 64, A, 64, 0, A, 64, 0, D, 128, batch=2)])
+
+
+@pytest.mark.parametrize("tile", TILES)
+def test_multi_weight_gradients_adamw(F, tile):
+    """The backward's grouped weight gradients: problems 0-2 read column slices of one
+    [K, 3M] gradient (lda = 3M, as the q, k, v rows of a QKV weight), problem 3 its own
+    [K, M] tensor; the four updated weights, moments and bf16 copies sit at irregular
+    offsets of shared arenas.  Bit-identical to four separate launches."""
+    M, N, K = 256, 512, 200
+    n = 4
+    rng = np.random.default_rng(7)
+    dqkv = dev_bf16(rnd_bf16_f64(rng, (K, 3 * M)))
+    dh = dev_bf16(rnd_bf16_f64(rng, (K, M)))
+    X = [dev_bf16(rnd_bf16_f64(rng, (K, N), 0.1)) for _ in range(2)]
+    offs = [0, M * N + 64, 2 * M * N + 128, 3 * M * N + 1024]  # element offsets in the arenas
+    size = offs[-1] + M * N
+    w0 = (0.02 * rng.standard_normal(size)).astype(np.float32)
+    m0 = (1e-3 * rng.standard_normal(size)).astype(np.float32)
+    v0 = (1e-6 * rng.random(size)).astype(np.float32)
+    hyper = dict(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.01, inv_bc1=1 / 0.19, inv_bc2=1 / 0.002997)
+
+    def run(multi):
+        w, m, v = dev_f32(w0), dev_f32(m0), dev_f32(v0)
+        wb = torch.full((size,), float("nan"), dtype=torch.bfloat16, device="cuda")
+        args = []
+        for r in range(n):
+            A, lda = (dqkv[:, r * M:], 3 * M) if r < 3 else (dh, M)
+            o = offs[r]
+            args.append(F.gemm_args(M, N, K, A, lda, 1, X[r % 2], N, 1, w[o:], N, epilogue=F.FL_EPI_ADAMW,
+                                    aux_out=wb[o:], ld_aux_out=N, adam_m=m[o:], adam_v=v[o:], tile=tile_id(F, tile),
+                                    **hyper))
+        if multi:
+            F.fl_k_gemm_multi(args)
+        else:
+            for a in args:
+                F.fl_k_gemm(a)
+        torch.cuda.synchronize()
+        return w, m, v, wb
+
+    got, want = run(True), run(False)
+    for g, x in zip(got, want):
+        _cmp(g, x)
+
+
+@pytest.mark.parametrize("tile", TILES)
+def test_multi_forward_bias_residual_layernorm(F, tile):
+    """Three forward problems in separate buffers (K-major A with different row strides),
+    bias + fp32 residual with the LayerNorm recomputed, each problem's per-row statistics
+    and gain / shift at their own offsets; bit-identical to separate launches."""
+    M, N, K = 130, 256, 192
+    rng = np.random.default_rng(8)
+    n = 3
+    As = [dev_bf16(rnd_bf16_f64(rng, (M, K + 64 * r))) for r in range(n)]
+    Bs = [dev_bf16(rnd_bf16_f64(rng, (N, K), 0.1)) for _ in range(n)]
+    X = dev_f32(rng.standard_normal((n, M, N)).astype(np.float32))
+    stats = dev_f32(rng.standard_normal((2, n * M + 32)).astype(np.float32))
+    lnp = dev_f32(rng.standard_normal((2, n * N + 64)).astype(np.float32))
+    bias = dev_f32(rng.standard_normal(n * N + 16).astype(np.float32))
+
+    def run(multi):
+        D = torch.full((n, M, N), float("nan"), dtype=torch.float32, device="cuda")
+        args = []
+        for r in range(n):
+            ro, co = r * M + 8 * r, r * N + 16 * r
+            args.append(F.gemm_args(M, N, K, As[r], K + 64 * r, 0, Bs[r], K, 0, D[r], N, epilogue=F.FL_EPI_BIAS_RESID,
+                                    bias=bias[r * N + 4 * r:], aux=X[r], ld_aux=N, alpha=1.5, aux_dtype=F.FL_DT_F32,
+                                    d_dtype=F.FL_DT_F32, ln_mean=stats[0, ro:], ln_rstd=stats[1, ro:],
+                                    ln_gamma=lnp[0, co:], ln_beta=lnp[1, co:], tile=tile_id(F, tile)))
+        if multi:
+            F.fl_k_gemm_multi(args)
+        else:
+            for a in args:
+                F.fl_k_gemm(a)
+        torch.cuda.synchronize()
+        return D
+
+    _cmp(run(True), run(False))
