@@ -25,19 +25,20 @@ if ROOT not in sys.path:
 
 def gemm_cases(cfg):
     """(name, M, N, K, a_mn, b_mn, epilogue, fp32 residual stream) of the 12 GEMMs of one
-    block at T tokens, with the epilogues the server uses (weight gradients as the first
-    backward after a step stores them)."""
+    block at T tokens, with the operand layouts and epilogues the server uses (the FFN
+    up-projection weight stored transposed, [H, F]; weight gradients as the first backward
+    after a step stores them)."""
     from paper_2406_14898_gb300 import flglm as F
     T, H, Fh = cfg.tokens, cfg.hidden, cfg.ffn_hidden
     return [
         ("qkv_fwd", T, 3 * H, H, 0, 0, F.FL_EPI_BIAS_ROPE, False),
         ("dense_fwd", T, H, H, 0, 0, F.FL_EPI_BIAS_RESID, True),
-        ("up_fwd", T, Fh, H, 0, 0, F.FL_EPI_BIAS_GELU, False),
+        ("up_fwd", T, Fh, H, 0, 1, F.FL_EPI_BIAS_GELU, False),
         ("down_fwd", T, H, Fh, 0, 0, F.FL_EPI_BIAS_RESID, True),
         ("down_dgrad", T, Fh, H, 0, 1, F.FL_EPI_GELU_BWD, False),
         ("down_wgrad", H, Fh, T, 1, 1, F.FL_EPI_STORE_F32, False),
-        ("up_dgrad", T, H, Fh, 0, 1, F.FL_EPI_RESID, True),
-        ("up_wgrad", Fh, H, T, 1, 1, F.FL_EPI_STORE_F32, False),
+        ("up_dgrad", T, H, Fh, 0, 0, F.FL_EPI_RESID, True),
+        ("up_wgrad", H, Fh, T, 1, 1, F.FL_EPI_STORE_F32, False),
         ("dense_dgrad", T, H, H, 0, 1, F.FL_EPI_STORE, False),
         ("dense_wgrad", H, H, T, 1, 1, F.FL_EPI_STORE_F32, False),
         ("qkv_dgrad", T, H, 3 * H, 0, 1, F.FL_EPI_RESID, True),
