@@ -10,6 +10,7 @@
 // exported kernel entry points.  dQ and dK leave the backward through the inverse rotary
 // rotation (the forward rotation is applied in the QKV GEMM epilogue), so the result is
 // the gradient w.r.t. the un-rotated q and k.
+#include <algorithm>
 #include <cmath>
 #include <vector>
 
@@ -60,19 +61,17 @@ __global__ void __launch_bounds__(256) attn_delta_kernel(int T, int H, int nh, c
 }  // namespace
 
 int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles, int rows) {
-  int maxq = 0;
-  for (int s = 0; s < S; ++s) {
-    const int nq = (cu[s + 1] - cu[s] + rows - 1) / rows;
-    maxq = nq > maxq ? nq : maxq;
-  }
+  // segments by decreasing tile count (stable), each segment's tiles next to each other,
+  // its last (longest causal) tile first
+  std::vector<int> order(S > 0 ? S : 0);
+  for (int s = 0; s < S; ++s) order[s] = s;
+  auto ntiles = [&](int s) { return (cu[s + 1] - cu[s] + rows - 1) / rows; };
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return ntiles(a) > ntiles(b); });
   int n = 0;
-  for (int i = maxq - 1; i >= 0; --i)
-    for (int s = 0; s < S; ++s) {
-      const int nq = (cu[s + 1] - cu[s] + rows - 1) / rows;
-      if (i < nq) {
-        if (n >= max_tiles) return -1;
-        tiles[n++] = (uint32_t(s) << 16) | uint32_t(i);
-      }
+  for (int s : order)
+    for (int i = ntiles(s) - 1; i >= 0; --i) {
+      if (n >= max_tiles) return -1;
+      tiles[n++] = (uint32_t(s) << 16) | uint32_t(i);
     }
   return n;
 }

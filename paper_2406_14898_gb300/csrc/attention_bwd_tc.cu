@@ -131,7 +131,8 @@ FL_DEV void staged_colsum(uint8_t* stage, int rows, float* out, int tid) {
 }
 
 // dK / dV.  Non-prefix: unit u = (entry u / nh of the 128-row tile list, head u % nh), the
-// entry's tile index i standing for key tile nq - 1 - i (the list's most work first).
+// entry's tile index i standing for key tile nq - 1 - i (a segment's key tile 0, seen by
+// every query tile, first).
 // PREFIX: unit u = (slice u / nh of the tile list cut into n_split slices, head u % nh),
 // the unit's keys the Lp prefix keys of its head.
 template <int HD, bool PREFIX>

@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   const int npt = Lp > 0 ? 1 : 0;  // at most one prefix tile (Lp <= 128)
 
   // A work unit u is (entry u / n_heads of the 128-row tile list, head u % n_heads): the
-  // list's longest causal rows first.
+  // list's longest segments first, each segment's tiles together (last tile first).
   struct Unit {
     int h, seg0, L, q0, clast, n_kv;
   };

@@ -124,8 +124,11 @@ int fl_launch_layernorm_bwd_f32(int T, int H, const float* dy, const float* x, c
 int fl_launch_layernorm_fwd_f32(int T, int H, const float* x, const float* gamma, const float* beta, float eps,
                                 __nv_bfloat16* y, float* mean, float* rstd, cudaStream_t st, int* status = nullptr);
 
-// Host helper: builds the tile list of a packing, tiles of `rows` query rows (64 for the
-// mma.sync kernels, 128 for the tcgen05 ones), segments' last tiles first (returns the
-// count, -1 if over capacity).  A device tile list holds the 64-row list followed by the
+// Host helper: builds the tile list of a packing, tiles of `rows` query rows (128 for the
+// tcgen05 kernels): segments by decreasing length, each segment's tiles consecutive, its
+// last tile first (returns the count, -1 if over capacity).  The units of the persistent
+// attention kernels are (list entry, head), so the tiles of one segment and head, which
+// read the same key / value (or query / output-gradient) tiles, run at about the same
+// time and share them in L2.  A device tile list holds the 64-row list followed by the
 // 128-row one.
 int fl_build_tiles(const int32_t* cu, int S, uint32_t* tiles, int max_tiles, int rows = 64);
