@@ -304,10 +304,33 @@ int run_gemm(fl_server* h, fl_gemm_args a, bool wgrad = false) {
   return rc;
 }
 
-// Several problems of one shape as one launch (fl_k_gemm_multi; one replica).
-int run_gemm_multi(fl_server* h, const fl_gemm_args* probs, int n) {
+// Several weight-gradient problems of one shape (ms[0..n), for replica 0) as one launch
+// for every replica (fl_k_gemm_multi) when n x R problems fit one launch, else one
+// launch per problem batched over the replicas.  Problem m of replica r reads replica r's
+// Tr token rows and updates replica r's arena.
+int run_wgrad_group(fl_server* h, const fl_gemm_args* ms, int n) {
+  if (n * h->R > FL_GEMM_MAX_BATCH) {
+    for (int i = 0; i < n; ++i)
+      if (int rc = run_gemm(h, ms[i], true)) return rc;
+    return FL_OK;
+  }
+  fl_gemm_args probs[FL_GEMM_MAX_BATCH];
+  const int64_t P = h->n_params, Tr = h->Tr;
+  for (int r = 0; r < h->R; ++r)
+    for (int i = 0; i < n; ++i) {
+      fl_gemm_args a = ms[i];
+      a.A = static_cast<const __nv_bfloat16*>(a.A) + r * Tr * a.lda;
+      a.B = static_cast<const __nv_bfloat16*>(a.B) + r * Tr * a.ldb;
+      a.D = static_cast<float*>(a.D) + r * P;
+      if (a.adam_m) {
+        a.adam_m += r * P;
+        a.adam_v += r * P;
+        a.aux_out = static_cast<__nv_bfloat16*>(a.aux_out) + r * P;
+      }
+      probs[r * n + i] = a;
+    }
   prof_begin(h, FL_PROF_GEMM);
-  int rc = fl_k_gemm_multi(probs, n, h->status, h->stream);
+  int rc = fl_k_gemm_multi(probs, n * h->R, h->status, h->stream);
   prof_end(h);
   return rc;
 }
@@ -498,12 +521,7 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
     // dW2 (+)= dy^T g, dW1^T (+)= m^T du
     const fl_gemm_args ffn[2] = {gemm_wgrad(h, b, FL_T_WDOWN, T, H, F, dy, A.g),
                                  gemm_wgrad(h, b, FL_T_WUP, T, H, F, A.m, h->du)};
-    if (h->R == 1) {
-      TRY(h, run_gemm_multi(h, ffn, 2));
-    } else {
-      TRY(h, run_gemm(h, ffn[0], true));
-      TRY(h, run_gemm(h, ffn[1], true));
-    }
+    TRY(h, run_wgrad_group(h, ffn, 2));
     if (b == c.n_blocks - 1) {
       prof_begin(h, FL_PROF_OTHER, h->R);
       for (int r = 0; r < h->R; ++r) TRY(h, fl_k_colsum(T, H, dy + (int64_t)r * T * H, h->gt(b, FL_T_BDOWN, r), st));
@@ -545,8 +563,8 @@ int block_backward(fl_server* h, int b, const __nv_bfloat16* dy, const float* dy
       fl_gemm_args att[4] = {gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o)};
       for (int r = 0; r < 3; ++r)
         att[1 + r] = gemm_wgrad(h, b, FL_T_WQKV, T, H, H, h->dqkv + (int64_t)r * H, A.a, (int64_t)r * H * H, 3 * H);
-      TRY(h, run_gemm_multi(h, att, 4));
-    } else {
+      TRY(h, run_wgrad_group(h, att, 4));
+    } else {  // [dWd, dWqkv] batched over the replicas
       TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WDENSE, T, H, H, h->dh, A.o), true));
       TRY(h, run_gemm(h, gemm_wgrad(h, b, FL_T_WQKV, T, 3 * H, H, h->dqkv, A.a), true));
     }
