@@ -14,7 +14,10 @@
 // 512 TMEM columns) walks work units u = blockIdx.x, + gridDim.x, ...  Each of the next
 // unit's tiles is loaded as soon as its buffer has had its last use in the current unit,
 // so they arrive while the unit's last products run and its output is staged (in a tile
-// of its own) and written.
+// of its own) and written; a whole tile of output rows leaves by bulk tensor stores
+// (TMA), which the next unit's epilogue waits for only before it stages again.  Per-row
+// values that a unit needs later (the next tile's lse / delta, the rotary rows of the
+// epilogue, the descriptor of the unit after next) are read while products run.
 //
 // dK / dV: unit = (128-key tile, head).  Warp w reads TMEM lanes 32 (w % 4) .. + 31, so
 // thread (w, lane) owns key row r = 32 (w % 4) + lane, and takes query half w / 4 of every
@@ -81,23 +84,34 @@ FL_DEV uint64_t desc_mn(uint32_t base, int kk) { return smem_desc_sw128(base + k
 // as two groups of 32 values at 64 g + 16 hf (hf = (kk / 2) % 2), 8 columns per k-step.
 FL_DEV uint32_t a_col(int kk) { return (kk >> 2) * 64 + ((kk >> 1) & 1) * 16 + (kk & 1) * 8; }
 
-// Inverse rotary rotation of one rotary region held by a thread: HD/2 consecutive dims,
-// pairs (i, i + HD/4), angle (cos, sin) of pair i at row[i] (the row of the rotary table
-// for the token's position, read from global memory: the table is small and L2-resident).
+// The rotary table row of one token's position, (cos, sin) of pairs 2j, 2j + 1 in cs[j]:
+// read from global memory (the table is small and L2-resident) while the unit's last
+// products run, applied in the epilogue.
 template <int HD>
-FL_DEV void inverse_rope_row(float* v, const float2* __restrict__ row) {
-  constexpr int Q = HD / 4;
+struct RopeRow {
+  float4 cs[HD / 8];
+};
+template <int HD>
+FL_DEV void rope_load(RopeRow<HD>& rr, const float2* __restrict__ row) {
   const float4* r4 = reinterpret_cast<const float4*>(row);
 #pragma unroll
-  for (int i = 0; i < Q; i += 2) {
-    const float4 cs = __ldg(r4 + i / 2);  // pairs i and i + 1
+  for (int j = 0; j < HD / 8; ++j) rr.cs[j] = __ldg(r4 + j);
+}
+// Inverse rotary rotation of one rotary region held by a thread: HD/2 consecutive dims,
+// pairs (i, i + HD/4), angle (cos, sin) of pair i from the token's table row.
+template <int HD>
+FL_DEV void inverse_rope_row(float* v, const RopeRow<HD>& rr) {
+  constexpr int Q = HD / 4;
+#pragma unroll
+  for (int j = 0; j < Q / 2; ++j) {
+    const int i = 2 * j;  // pairs i and i + 1
     float x1 = v[i], x2 = v[i + Q];
-    v[i] = x1 * cs.x + x2 * cs.y;
-    v[i + Q] = x2 * cs.x - x1 * cs.y;
+    v[i] = x1 * rr.cs[j].x + x2 * rr.cs[j].y;
+    v[i + Q] = x2 * rr.cs[j].x - x1 * rr.cs[j].y;
     x1 = v[i + 1];
     x2 = v[i + 1 + Q];
-    v[i + 1] = x1 * cs.z + x2 * cs.w;
-    v[i + 1 + Q] = x2 * cs.z - x1 * cs.w;
+    v[i + 1] = x1 * rr.cs[j].z + x2 * rr.cs[j].w;
+    v[i + 1 + Q] = x2 * rr.cs[j].z - x1 * rr.cs[j].w;
   }
 }
 
@@ -109,13 +123,25 @@ FL_DEV float exp2_hw(float x) {
   return y;
 }
 
-// Staged bf16 tile: rows of HD values (CH chunks of 16 bytes), chunk j of row r at
-// position j ^ (r & (CH - 1)).
+// Staged bf16 tile in the layout of 128-byte-swizzled TMA boxes of 64 columns x 128 rows:
+// 16-byte chunk j of row r in box j / 8, at chunk (j % 8) ^ (r % 8) of the box's row r.
 template <int HD>
 FL_DEV uint8_t* stage_chunk(uint8_t* stage, int r, int j) {
-  constexpr int CH = BwdCfg<HD>::CH;
-  return stage + r * (HD * 2) + ((j ^ (r & (CH - 1))) << 4);
+  return stage + (j >> 3) * (TB * 128) + r * 128 + (((j & 7) ^ (r & 7)) << 4);
 }
+
+// 2-D tiled store of one box from shared memory to global memory (bulk-group completion).
+FL_DEV void tma_store_2d(const CUtensorMap* m, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(m)),
+               "r"(smem_u32(src)), "r"(x), "r"(y)
+               : "memory");
+}
+FL_DEV void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// The committed bulk stores have read their shared memory (it may be written again).
+FL_DEV void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// The committed bulk stores are complete.
+FL_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // Adds the column sums of a staged tile over its first `rows` rows to out[0..HD): thread
 // c < HD sums column c in row order, one atomic per column.
@@ -138,7 +164,8 @@ FL_DEV void staged_colsum(uint8_t* stage, int rows, float* out, int tid) {
 template <int HD, bool PREFIX>
 __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do,
-    const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int T, int H,
+    const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv,
+    const __grid_constant__ CUtensorMap tm_dqkv, int T, int H,
     const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, int n_tiles, int n_units, int n_split,
     const float* __restrict__ lse, const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale,
     float scale_log2, int Lp, bf16* __restrict__ dqkv, float* __restrict__ dpk, float* __restrict__ dpv,
@@ -176,7 +203,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     int h, seg0, L, kb, clast, it0, it_end;
     float* db;
   };
-  auto unit = [&](int u) {
+  auto unit_t = [&](int u, uint32_t t) {
     Unit w;
     w.h = u % nh;
     if constexpr (PREFIX) {
@@ -187,7 +214,6 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       w.clast = -1;
       w.db = nullptr;
     } else {
-      const uint32_t t = tiles[u / nh];
       const int s = int(t >> 16), idx = int(t & 0xFFFFu);
       w.seg0 = cu[s];
       w.L = cu[s + 1] - w.seg0;
@@ -201,6 +227,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     }
     return w;
   };
+  auto tile_word = [&](int u) { return PREFIX ? 0u : tiles[u / nh]; };
+  auto unit = [&](int u) { return unit_t(u, tile_word(u)); };
   // a query tile of unit w: its first token, the position of that token in its segment,
   // valid rows
   auto qtile = [&](const Unit& w, int it, int& row0, int& qpos0, int& valid) {
@@ -265,6 +293,17 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
   bool ok = true;
   int u = blockIdx.x;
   Unit w = u < n_units ? unit(u) : Unit{};
+  Unit wn = u + (int)gridDim.x < n_units ? unit(u + gridDim.x) : Unit{};
+  // the thread's lse (tid < 128) or delta value of the next query tile, loaded a tile early
+  auto stat_of = [&](const Unit& x, int it) {
+    int row0, qpos0, valid;
+    qtile(x, it, row0, qpos0, valid);
+    const int c = tid & (TB - 1);
+    const float* src = tid < TB ? lse : delta;
+    return c < valid ? __ldg(src + (int64_t)x.h * T + row0 + c) : 0.f;
+  };
+  float pf = (u < n_units && w.it0 < w.it_end) ? stat_of(w, w.it0) : 0.f;
+  RopeRow<HD> rrow;
   if (tid == 0 && u < n_units && w.it0 < w.it_end) {
     issue_kv(w);
     issue_q(w, w.it0, 0);
@@ -277,8 +316,9 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     // the next unit: its K / V load once this unit's last S^T / dP^T products have read K
     // and V, its first query tile once buffer pair 0 has had its last use here
     const int un = u + gridDim.x;
-    const Unit wn = un < n_units ? unit(un) : Unit{};
     const bool next = un < n_units && wn.it0 < wn.it_end;
+    Unit wnn = Unit{};  // the unit after next: its tile word read while the first score
+    uint32_t tnn = 0;   // products run, the rest while the first gradient products run
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
     if (work && !track_wait_all(bar_kv, tkv)) {
       if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
@@ -291,10 +331,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
       qtile(w, it, row0, qpos0, valid);
       {  // lse and delta of the query tile (rows past its segment are never visible)
         const int c = tid & (TB - 1);
-        const float* src = tid < TB ? lse : delta;
-        const float v = c < valid ? __ldg(src + (int64_t)w.h * T + row0 + c) : 0.f;
-        if (tid < TB) sL[c] = v * LOG2E_B;  // the previous tile's readers passed a barrier since
-        else sD[c] = v;
+        if (tid < TB) sL[c] = pf * LOG2E_B;  // the previous tile's readers passed a barrier since
+        else sD[c] = pf;
       }
       if (!track_wait_all(bar_q + b, b ? tq1 : tq0)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_FULL);
@@ -314,6 +352,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
         tm1.pend = true;
         umma_commit(bar_mma1);
       }
+      // while the products run: the next tile's statistics, the unit after next
+      if (it + 1 < w.it_end) pf = stat_of(w, it + 1);
+      else if (next) pf = stat_of(wn, wn.it0);
+      if (it == w.it0 && un + (int)gridDim.x < n_units) tnn = tile_word(un + gridDim.x);
       if (!track_wait_all(bar_mma1, tm1)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
         ok = false;
@@ -387,6 +429,11 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
         tm2.pend = true;
         umma_commit(bar_mma2);
       }
+      if (it == w.it0 && un + (int)gridDim.x < n_units) wnn = unit_t(un + gridDim.x, tnn);
+      if (!PREFIX && it + 1 == w.it_end && qh < nreg && key_ok) {  // the key's rotary row, for the epilogue
+        const int32_t* gp = qh == 0 ? gpos : gpos2;
+        rope_load<HD>(rrow, rope_tab + (int64_t)(gp ? __ldg(gp + w.seg0 + k) : k) * E);
+      }
       if (!track_wait_all(bar_mma2, tm2)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
         ok = false;
@@ -433,12 +480,14 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
           }
         }
       } else {
-        // ---- dK (scaled, rotated back), then dV: thread (r, qh) takes dims qh * HD/2 .. +
-        // HD/2 - 1 of key row r from TMEM and stages the bf16 rows, then the CTA writes whole
-        // rows with coalesced 16-byte stores; the bias column sums are taken from the staged
-        // rows (the values stored)
+        // ---- dV, then dK (scaled, rotated back): thread (r, qh) takes dims qh * HD/2 .. +
+        // HD/2 - 1 of key row r from TMEM and stages the bf16 rows; a tile inside the
+        // segment leaves by bulk tensor stores, a ragged last tile by coalesced 16-byte
+        // stores of its valid rows; the bias column sums are taken from the staged rows
+        // (the values stored)
 #pragma unroll 1
-        for (int part = 0; part < 2; ++part) {  // 0: dK, 1: dV
+        for (int pi = 0; pi < 2; ++pi) {
+          const int part = 1 - pi;  // dV, then dK
           uint8_t* stage = sST;
           uint32_t vr[HD / 2];
 #pragma unroll
@@ -449,28 +498,36 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
           float* v = reinterpret_cast<float*>(vr);
 #pragma unroll
           for (int c = 0; c < HD / 2; ++c) v[c] = __uint_as_float(vr[c]) * (part ? 1.f : scale);
-          if (part == 0 && qh < nreg && key_ok) {  // rotary region qh: by pos, or by the GLM block position
-            const int32_t* gp = qh == 0 ? gpos : gpos2;
-            const int pos = gp ? __ldg(gp + w.seg0 + k) : k;
-            inverse_rope_row<HD>(v, rope_tab + (int64_t)pos * E);
-          }
+          if (part == 0 && qh < nreg && key_ok) inverse_rope_row<HD>(v, rrow);  // rotary region qh
+          // the staging tile is free once the previous bulk store has read it
+          if (tid == 0) bulk_wait_read();
+          __syncthreads();
 #pragma unroll
           for (int c8 = 0; c8 < HD / 16; ++c8)
             *reinterpret_cast<uint4*>(stage_chunk<HD>(stage, r, qh * (HD / 16) + c8)) =
                 make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
                            pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
           const int col = (part ? 2 * H : H) + w.h * HD;
+          const bool full = w.kb + TB <= w.L;  // a whole tile of the segment: TMA stores
+          if (full) fence_proxy_async_smem();  // the staged rows, visible to the bulk copies
           __syncthreads();  // the tile is staged
-          if (w.db) staged_colsum<HD>(stage, min(TB, w.L - w.kb), w.db + col, tid);
-          // 128 rows x CH chunks: consecutive threads write consecutive chunks of a row
+          if (full && tid == 0) {
 #pragma unroll
-          for (int i = 0; i < TB * CH / 256; ++i) {
-            const int id = tid + 256 * i, row = id / CH, jc = id % CH;
-            if (w.kb + row < w.L)
-              *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.kb + row) * 3 * H + col + jc * 8) =
-                  *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
+            for (int x = 0; x < NB; ++x) tma_store_2d(&tm_dqkv, stage + x * (TB * 128), col + 64 * x, w.seg0 + w.kb);
+            bulk_commit();
           }
-          __syncthreads();  // the staged rows have been read
+          if (w.db) staged_colsum<HD>(stage, min(TB, w.L - w.kb), w.db + col, tid);
+          if (!full) {
+            // 128 rows x CH chunks: consecutive threads write consecutive chunks of a row
+#pragma unroll
+            for (int i = 0; i < TB * CH / 256; ++i) {
+              const int id = tid + 256 * i, row = id / CH, jc = id % CH;
+              if (w.kb + row < w.L)
+                *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.kb + row) * 3 * H + col + jc * 8) =
+                    *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
+            }
+          }
+          __syncthreads();  // the staged rows have been read (the bulk store reads them on)
         }
       }
     }
@@ -479,7 +536,9 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
     __syncthreads();
     u = un;
     w = wn;
+    wn = wnn;
   }
+  if (tid == 0) bulk_wait_all();  // this CTA's bulk stores are complete before it leaves
   if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
     track_drain(bar_kv, tkv);
     track_drain(bar_q, tq0);
@@ -499,7 +558,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dkv_tc_kernel(
 template <int HD>
 __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     const __grid_constant__ CUtensorMap tm_qkv, const __grid_constant__ CUtensorMap tm_do,
-    const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv, int T, int H,
+    const __grid_constant__ CUtensorMap tm_pk, const __grid_constant__ CUtensorMap tm_pv,
+    const __grid_constant__ CUtensorMap tm_dqkv, int T, int H,
     const int32_t* __restrict__ cu, const uint32_t* __restrict__ tiles, int n_units, const float* __restrict__ lse,
     const float* __restrict__ delta, const float2* __restrict__ rope_tab, float scale, float scale_log2, int Lp,
     bf16* __restrict__ dqkv, const int32_t* __restrict__ ctxs, const int32_t* __restrict__ gpos,
@@ -603,6 +663,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   Unit w = u < n_units ? unit(u) : Unit{};
   float lse2 = 0.f, dl = 0.f;
   if (u < n_units) row_stats(w, lse2, dl);
+  RopeRow<HD> rrow;
   if (tid == 0 && u < n_units) {
     issue_qdo(w);
     issue_kv(w, 0, 0);
@@ -692,6 +753,10 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
         tm2.pend = true;
         umma_commit(bar_mma2);
       }
+      if (j + 1 == w.n_kv && kh < nreg && q_ok) {  // the query's rotary row, for the epilogue
+        const int32_t* gp = kh == 0 ? gpos : gpos2;
+        rope_load<HD>(rrow, rope_tab + (int64_t)(gp ? __ldg(gp + w.seg0 + q) : q) * E);
+      }
       if (!track_wait_all(bar_mma2, tm2)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
         ok = false;
@@ -714,8 +779,8 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     float lse2n = 0.f, dln = 0.f;
     if (next) row_stats(wn, lse2n, dln);
     // ---- dQ (scaled, rotated back): thread (r, kh) takes dims kh * HD/2 .. + HD/2 - 1 of
-    // query row r, staged and written as whole coalesced rows, the bias column sums taken
-    // from the staged rows
+    // query row r, staged and written by bulk tensor stores (coalesced row stores for a
+    // ragged last tile), the bias column sums taken from the staged rows
     {
       uint8_t* stage = sST;
       uint32_t vr[HD / 2];
@@ -726,25 +791,33 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
       float* v = reinterpret_cast<float*>(vr);
 #pragma unroll
       for (int c = 0; c < HD / 2; ++c) v[c] = __uint_as_float(vr[c]) * scale;
-      if (kh < nreg && q_ok) {  // rotary region kh: by pos, or by the GLM block position
-        const int32_t* gp = kh == 0 ? gpos : gpos2;
-        const int pos = gp ? __ldg(gp + w.seg0 + q) : q;
-        inverse_rope_row<HD>(v, rope_tab + (int64_t)pos * E);
-      }
+      if (kh < nreg && q_ok) inverse_rope_row<HD>(v, rrow);  // rotary region kh
+      // the staging tile is free once the previous bulk store has read it
+      if (tid == 0) bulk_wait_read();
+      __syncthreads();
 #pragma unroll
       for (int c8 = 0; c8 < HD / 16; ++c8)
         *reinterpret_cast<uint4*>(stage_chunk<HD>(stage, r, kh * (HD / 16) + c8)) =
             make_uint4(pack_bf16x2(v[8 * c8], v[8 * c8 + 1]), pack_bf16x2(v[8 * c8 + 2], v[8 * c8 + 3]),
                        pack_bf16x2(v[8 * c8 + 4], v[8 * c8 + 5]), pack_bf16x2(v[8 * c8 + 6], v[8 * c8 + 7]));
       const int col = w.h * HD;
+      const bool full = w.q0 + TB <= w.L;  // a whole tile of the segment: TMA stores
+      if (full) fence_proxy_async_smem();
       __syncthreads();  // the tile is staged
-      if (w.db) staged_colsum<HD>(stage, min(TB, w.L - w.q0), w.db + col, tid);
+      if (full && tid == 0) {
 #pragma unroll
-      for (int i = 0; i < TB * CH / 256; ++i) {
-        const int id = tid + 256 * i, row = id / CH, jc = id % CH;
-        if (w.q0 + row < w.L)
-          *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.q0 + row) * 3 * H + col + jc * 8) =
-              *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
+        for (int x = 0; x < NB; ++x) tma_store_2d(&tm_dqkv, stage + x * (TB * 128), col + 64 * x, w.seg0 + w.q0);
+        bulk_commit();
+      }
+      if (w.db) staged_colsum<HD>(stage, min(TB, w.L - w.q0), w.db + col, tid);
+      if (!full) {
+#pragma unroll
+        for (int i = 0; i < TB * CH / 256; ++i) {
+          const int id = tid + 256 * i, row = id / CH, jc = id % CH;
+          if (w.q0 + row < w.L)
+            *reinterpret_cast<uint4*>(dqkv + ((int64_t)w.seg0 + w.q0 + row) * 3 * H + col + jc * 8) =
+                *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
+        }
       }
     }
     // the staged rows have been read and the dQ columns loaded before the next unit's
@@ -756,6 +829,7 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
     lse2 = lse2n;
     dl = dln;
   }
+  if (tid == 0) bulk_wait_all();  // this CTA's bulk stores are complete before it leaves
   if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
     track_drain(bar_qdo, tqdo);
     track_drain(bar_kv, tkv0);
@@ -798,8 +872,9 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
     attr = true;
   }
   const int H = nh * HD;
-  CUtensorMap tq, tdo, tpk, tpv;
+  CUtensorMap tq, tdo, tpk, tpv, tdq;
   if (int rc = fl_gemm::make_map(&tq, qkv, (uint64_t)3 * H, (uint64_t)T, 3 * (int64_t)H, 128)) return rc;
+  if (int rc = fl_gemm::make_map(&tdq, dqkv, (uint64_t)3 * H, (uint64_t)T, 3 * (int64_t)H, 128)) return rc;
   if (int rc = fl_gemm::make_map(&tdo, dout, (uint64_t)H, (uint64_t)T, H, 128)) return rc;
   if (pre.len > 0) {
     if (int rc = fl_gemm::make_map(&tpk, pre.k, (uint64_t)H, (uint64_t)pre.len, H, 128)) return rc;
@@ -815,10 +890,10 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
   const int grid = n_units < sm_count_bwd() ? n_units : sm_count_bwd();
   if (n_units > 0) {
     FL_CUDA_TRY(fl_launch(attn_bwd_dq_tc_kernel<HD>, dim3(grid), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo, tpk, tpv,
-                          T, H, cu, tiles, n_units, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv,
+                          tdq, T, H, cu, tiles, n_units, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv,
                           glm.ctx, glm.pos, glm.pos2, dbias, dbias_segs, dbias_rstride, status));
     FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, false>, dim3(grid), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo,
-                          tpk, tpv, T, H, cu, tiles, n_tiles, n_units, 0, lse, delta, tab, scale, scale * LOG2E_B, 0,
+                          tpk, tpv, tdq, T, H, cu, tiles, n_tiles, n_units, 0, lse, delta, tab, scale, scale * LOG2E_B, 0,
                           (bf16*)dqkv, (float*)nullptr, (float*)nullptr, glm.ctx, glm.pos, glm.pos2, dbias,
                           dbias_segs, dbias_rstride, status));
   }
@@ -828,7 +903,7 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
     if (nsplit > n_tiles) nsplit = n_tiles;
     if (nsplit < 1) nsplit = 1;
     FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, true>, dim3(nsplit * nh), dim3(256), BwdCfg<HD>::SMEM, st, tq,
-                          tdo, tpk, tpv, T, H, cu, tiles, n_tiles, nsplit * nh, nsplit, lse, delta, tab, scale,
+                          tdo, tpk, tpv, tdq, T, H, cu, tiles, n_tiles, nsplit * nh, nsplit, lse, delta, tab, scale,
                           scale * LOG2E_B, pre.len, (bf16*)dqkv, pre.dk, pre.dv, glm.ctx, glm.pos, glm.pos2,
                           (float*)nullptr, 0, (int64_t)0, status));
   }
