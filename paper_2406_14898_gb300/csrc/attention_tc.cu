@@ -84,9 +84,8 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   struct Unit {
     int h, seg0, L, q0, clast, n_kv;
   };
-  auto unit = [&](int u) {
+  auto unit_t = [&](int u, uint32_t t) {
     Unit w;
-    const uint32_t t = tiles[u / n_heads];
     const int s = int(t >> 16), idx = int(t & 0xFFFFu);
     w.h = u % n_heads;
     w.seg0 = cu[s];
@@ -96,6 +95,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     w.n_kv = npt + max(idx, w.clast >= 0 ? w.clast / TB : 0) + 1;
     return w;
   };
+  auto unit = [&](int u) { return unit_t(u, tiles[u / n_heads]); };
 
   if (tid == 0) {
     for (int i = 0; i < 5; ++i) mbar_init(bars + i, 1);
@@ -145,9 +145,14 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
   bool ok = true;
   int u = blockIdx.x;
   Unit w = u < n_units ? unit(u) : Unit{};
+  Unit wn = u + (int)gridDim.x < n_units ? unit(u + gridDim.x) : Unit{};
   if (tid == 0 && u < n_units) issue_unit(w);
   while (u < n_units && ok) {
     const int q = w.q0 + tid;  // this thread's query row (inside the segment)
+    const int un = u + gridDim.x, unn = un + gridDim.x;
+    // the descriptor of the unit after next, read in two steps while products run
+    Unit wnn = Unit{};
+    uint32_t tnn = 0;
     float m_run = -INFINITY, l_run = 0.f;
     // every wait's outcome is agreed on by the whole CTA, so that all threads leave together
     if (!track_wait_all(bar_q, tq)) {
@@ -171,6 +176,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
         ts.pend = true;
         umma_commit(bar_s);
       }
+      if (j == 0 && unn < n_units) tnn = tiles[unn / n_heads];
       if (!track_wait_all(bar_s, ts)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_FULL);
         ok = false;
@@ -244,6 +250,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
         tpv.pend = true;
         umma_commit(bar_pv);
       }
+      if (j == 0 && unn < n_units) wnn = unit_t(unn, tnn);
       if (!track_wait_all(bar_pv, tpv)) {
         if (tid == 0) report_status(status, FL_DEV_TIMEOUT_ACC_EMPTY);
         ok = false;
@@ -255,23 +262,21 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     if (!ok) break;
     // ---- every product of the unit is complete and Q / K / V are free: the next unit's
     // first tiles load while this one's O leaves
-    const int un = u + gridDim.x;
-    const Unit wn = un < n_units ? unit(un) : Unit{};
     if (tid == 0 && un < n_units) issue_unit(wn);
-    // ---- O / l and the log-sum-exp (every lane reads TMEM; rows past the segment end
-    // store nothing)
+    // ---- O / l and the log-sum-exp (every lane reads TMEM, all of the row at once; rows
+    // past the segment end store nothing)
     const bool valid = q < w.L;
     const float inv = valid ? 1.f / l_run : 0.f;
     bf16* orow = O + (int64_t)(w.seg0 + (valid ? q : 0)) * H + w.h * HD;
-#pragma unroll 1
-    for (int c = 0; c < HD; c += 32) {
-      uint32_t o[32];
-      tmem_ld32(t_o + c, o);
+    {
+      uint32_t o[HD];
+#pragma unroll
+      for (int c = 0; c < HD; c += 32) tmem_ld32(t_o + c, *reinterpret_cast<uint32_t(*)[32]>(o + c));
       tmem_ld_wait();
       if (valid) {
 #pragma unroll
-        for (int v = 0; v < 4; ++v)
-          *reinterpret_cast<uint4*>(orow + c + 8 * v) = make_uint4(
+        for (int v = 0; v < HD / 8; ++v)
+          *reinterpret_cast<uint4*>(orow + 8 * v) = make_uint4(
               pack_bf16x2(__uint_as_float(o[8 * v]) * inv, __uint_as_float(o[8 * v + 1]) * inv),
               pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv),
               pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv),
@@ -283,6 +288,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
     tc_fence_before();
     u = un;
     w = wn;
+    wn = wnn;
   }
   if (!ok && tid == 0) {  // a wait gave up: let what this CTA armed land before leaving
     track_drain(bar_q, tq);
