@@ -159,12 +159,11 @@ def check_fused_step(cfg, weights, stepped, wg_ref):
 
 
 def sampled_segments(cfg):
-    """(client, row) pairs to check: first and last; shortest and longest if ragged."""
-    picks = {(0, 0), (cfg.K - 1, cfg.client_batch - 1)}
+    """(client, row) pairs to check: the shortest and the longest segment when the lengths
+    are ragged (one and eight query tiles at ragged26), else the first and the last."""
     if len(set(cfg.seq_lens)) > 1:
-        picks.add((int(np.argmin(cfg.seq_lens)), 0))
-        picks.add((int(np.argmax(cfg.seq_lens)), 0))
-    return sorted(picks)
+        return sorted({(int(np.argmin(cfg.seq_lens)), 0), (int(np.argmax(cfg.seq_lens)), 0)})
+    return sorted({(0, 0), (cfg.K - 1, cfg.client_batch - 1)})
 
 
 def run_workload(F, weights, cfg, n_oracle_segments=None, serial=True, step=False):
