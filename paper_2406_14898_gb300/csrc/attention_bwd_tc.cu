@@ -143,17 +143,41 @@ FL_DEV void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" :
 // The committed bulk stores are complete.
 FL_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-// Adds the column sums of a staged tile over its first `rows` rows to out[0..HD): thread
-// c < HD sums column c in row order, one atomic per column.
+// Adds the column sums of a staged tile over its first `rows` rows to out[0..HD); called by
+// all 256 threads.  Warp wp takes the HD/64 16-byte chunks wp*HD/64 ..: LPC = 32*64/HD
+// lanes per chunk, lane l reading rows l % LPC, + LPC, ... (8 consecutive lanes read 8
+// consecutive rows of one chunk: distinct swizzled 16-byte slots, no bank conflict), then
+// a butterfly over the chunk's lanes and one atomic per column.
 template <int HD>
 FL_DEV void staged_colsum(uint8_t* stage, int rows, float* out, int tid) {
-  if (tid >= HD) return;
-  const int jc = tid >> 3, e = tid & 7;
-  float acc = 0.f;
-#pragma unroll 8
-  for (int row = 0; row < rows; ++row)
-    acc += __bfloat162float(*reinterpret_cast<const bf16*>(stage_chunk<HD>(stage, row, jc) + 2 * e));
-  atomicAdd(out + tid, acc);
+  constexpr int CPW = HD / 64, LPC = 32 / CPW;
+  const int lane = tid & 31, jc = (tid >> 5) * CPW + lane / LPC, r0 = lane % LPC;
+  float acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+#pragma unroll
+  for (int i = 0; i < TB / LPC; ++i) {
+    const int row = r0 + LPC * i;
+    if (row < rows) {
+      const uint4 q = *reinterpret_cast<const uint4*>(stage_chunk<HD>(stage, row, jc));
+      const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 f = unpack_bf16x2(qw[e]);
+        acc[2 * e] += f.x;
+        acc[2 * e + 1] += f.y;
+      }
+    }
+  }
+#pragma unroll
+  for (int off = LPC / 2; off > 0; off >>= 1)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], off);
+  float mine = acc[0];
+#pragma unroll
+  for (int e = 1; e < 8; ++e)
+    if (r0 == e) mine = acc[e];
+  if (r0 < 8) atomicAdd(out + jc * 8 + r0, mine);
 }
 
 // dK / dV.  Non-prefix: unit u = (entry u / nh of the 128-row tile list, head u % nh), the
