@@ -869,32 +869,14 @@ __global__ void __launch_bounds__(256, 1) attn_bwd_dq_tc_kernel(
   }
 }
 
-int sm_count_bwd() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 148;
-  }
-  return n;
-}
-
 template <int HD>
 int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float* lse, const float* delta,
                   const int32_t* cu, const uint32_t* tiles, int n_tiles, const float* rope_tab, void* dqkv,
                   const AttnPrefix& pre, const AttnGlm& glm, float* dbias, int* status, cudaStream_t st,
                   int dbias_segs, int64_t dbias_rstride) {
-  static bool attr = false;
-  if (!attr) {
-    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dq_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BwdCfg<HD>::SMEM));
-    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dkv_tc_kernel<HD, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BwdCfg<HD>::SMEM));
-    FL_CUDA_TRY(cudaFuncSetAttribute(attn_bwd_dkv_tc_kernel<HD, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     BwdCfg<HD>::SMEM));
-    attr = true;
-  }
+  FL_CUDA_TRY(fl_func_smem((const void*)attn_bwd_dq_tc_kernel<HD>, BwdCfg<HD>::SMEM));
+  FL_CUDA_TRY(fl_func_smem((const void*)attn_bwd_dkv_tc_kernel<HD, false>, BwdCfg<HD>::SMEM));
+  FL_CUDA_TRY(fl_func_smem((const void*)attn_bwd_dkv_tc_kernel<HD, true>, BwdCfg<HD>::SMEM));
   const int H = nh * HD;
   CUtensorMap tq, tdo, tpk, tpv, tdq;
   if (int rc = fl_gemm::make_map(&tq, qkv, (uint64_t)3 * H, (uint64_t)T, 3 * (int64_t)H, 128)) return rc;
@@ -911,7 +893,7 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
   const float2* tab = reinterpret_cast<const float2*>(rope_tab);
   // persistent: one CTA per SM (512 TMEM columns each) walks the (tile, head) units
   const int n_units = n_tiles * nh;
-  const int grid = n_units < sm_count_bwd() ? n_units : sm_count_bwd();
+  const int grid = n_units < fl_sm_count() ? n_units : fl_sm_count();
   if (n_units > 0) {
     FL_CUDA_TRY(fl_launch(attn_bwd_dq_tc_kernel<HD>, dim3(grid), dim3(256), BwdCfg<HD>::SMEM, st, tq, tdo, tpk, tpv,
                           tdq, T, H, cu, tiles, n_units, lse, delta, tab, scale, scale * LOG2E_B, pre.len, (bf16*)dqkv,
@@ -923,7 +905,7 @@ int launch_bwd_tc(int T, int nh, const void* qkv, const void* dout, const float*
   }
   if (pre.len > 0 && n_tiles > 0) {
     // the prefix keys of each head against slices of the query tiles, about one CTA per SM
-    int nsplit = (sm_count_bwd() + nh - 1) / nh;
+    int nsplit = (fl_sm_count() + nh - 1) / nh;
     if (nsplit > n_tiles) nsplit = n_tiles;
     if (nsplit < 1) nsplit = 1;
     FL_CUDA_TRY(fl_launch(attn_bwd_dkv_tc_kernel<HD, true>, dim3(nsplit * nh), dim3(256), BwdCfg<HD>::SMEM, st, tq,

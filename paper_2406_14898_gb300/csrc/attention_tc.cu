@@ -308,12 +308,7 @@ __global__ void __launch_bounds__(128) attn_fwd_tc_kernel(
 template <int HD>
 int launch_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint32_t* tiles, int n_tiles, void* o,
                   float* lse, const AttnPrefix& pre, const AttnGlm& glm, int* status, cudaStream_t st) {
-  static bool attr = false;
-  if (!attr) {
-    FL_CUDA_TRY(cudaFuncSetAttribute(attn_fwd_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     FwdCfg<HD>::SMEM));
-    attr = true;
-  }
+  FL_CUDA_TRY(fl_func_smem((const void*)attn_fwd_tc_kernel<HD>, FwdCfg<HD>::SMEM));
   const int H = nh * HD;
   CUtensorMap tq, tpk, tpv;
   if (int rc = fl_gemm::make_map(&tq, qkv, (uint64_t)3 * H, (uint64_t)T, 3 * (int64_t)H, 128)) return rc;
@@ -327,7 +322,7 @@ int launch_fwd_tc(int T, int nh, const void* qkv, const int32_t* cu, const uint3
   const float scale_log2 = (1.f / sqrtf((float)HD)) * LOG2E_T;
   // persistent: two CTAs per SM walk the (tile, head) units
   const int n_units = n_tiles * nh;
-  const int grid = n_units < 2 * fl_gemm::num_sms() ? n_units : 2 * fl_gemm::num_sms();
+  const int grid = n_units < 2 * fl_sm_count() ? n_units : 2 * fl_sm_count();
   FL_CUDA_TRY(fl_launch(attn_fwd_tc_kernel<HD>, dim3(grid), dim3(128), FwdCfg<HD>::SMEM, st, tq, tpk, tpv, T, H, nh,
                         cu, tiles, n_units, (bf16*)o, lse, scale_log2, pre.len, glm.ctx, status));
   return FL_OK;

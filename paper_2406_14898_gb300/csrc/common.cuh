@@ -100,3 +100,11 @@ cudaError_t fl_launch(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem
 // Records a CUDA error in the thread-local error string and returns FL_ERR_CUDA.
 int fl_internal_cuda_error(cudaError_t e, const char* what, const char* file, int line);
 int fl_internal_error(int code, const char* fmt, ...);
+
+// Launch set-up shared by every launcher, kept per device and safe to call from several
+// host threads (runtime.cu).  fl_sm_count: the current device's multiprocessor count.
+// fl_func_smem: raises kernel `func`'s dynamic shared-memory limit to `bytes` on the
+// current device (an attribute the driver keeps per device), once per (kernel, device,
+// bytes); later calls return at once.
+int fl_sm_count();
+cudaError_t fl_func_smem(const void* func, int bytes);

@@ -20,6 +20,7 @@
 // warps 2..5 epilogue (warp w reads TMEM lanes 32*(w%4) .. +31).
 #pragma once
 #include <cuda.h>
+#include <atomic>
 #include <cstdio>
 #include <mutex>
 
@@ -785,16 +786,7 @@ inline int make_map(CUtensorMap* map, const void* base, uint64_t inner, uint64_t
   return FL_OK;
 }
 
-inline int num_sms() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 148;
-  }
-  return n;
-}
+inline int num_sms() { return fl_sm_count(); }
 
 // Row-group raster that minimises DRAM reads for tiles of bm x bn (see Raster).
 inline Raster pick_raster(int M, int N, int K, int bm, int bn) {
@@ -816,11 +808,7 @@ template <int BN, bool A_MN, bool B_MN, int FAM>
 int launch(const fl_gemm_args* a, const Problems& pr, const Epi& epi, int* status, cudaStream_t st) {
   using C = Cfg<BN>;
   auto kern = gemm_tc_kernel<BN, A_MN, B_MN, FAM>;
-  static bool attr_set = false;  // per instantiation; the attribute is per device function
-  if (!attr_set) {
-    FL_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES));
-    attr_set = true;
-  }
+  FL_CUDA_TRY(fl_func_smem((const void*)kern, C::SMEM_BYTES));
   GemmMaps maps;
   const int batch = pr.n;
   for (int r = 0; r < batch; ++r) {
@@ -842,30 +830,41 @@ int launch(const fl_gemm_args* a, const Problems& pr, const Epi& epi, int* statu
   return FL_OK;
 }
 
-// CTA pairs the device keeps resident at once for the pair kernel (0 if it cannot run).
+// CTA pairs the current device keeps resident at once for the pair kernel (0 if it cannot
+// run there); queried once per device (each of the first 64 devices caches its answer).
 template <bool A_MN, bool B_MN, int FAM>
 int pair_slots() {
-  static int slots = -1;
-  if (slots < 0) {
-    auto kern = gemm_pair_kernel<A_MN, B_MN, FAM>;
-    slots = 0;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, CfgPair::SMEM_BYTES) == cudaSuccess) {
-      cudaLaunchConfig_t cfg = {};
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = 2;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.gridDim = dim3(2 * num_sms());
-      cfg.blockDim = dim3(NUM_THREADS);
-      cfg.dynamicSmemBytes = CfgPair::SMEM_BYTES;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0) slots = n;
-    }
-    cudaGetLastError();  // a refused query leaves the single-SM kernel in use
+  constexpr int MAX_DEV = 64;
+  static std::atomic<int> cache[MAX_DEV];  // slots + 1; 0: not queried yet
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
   }
+  const bool cached = dev >= 0 && dev < MAX_DEV;
+  if (cached) {
+    const int c = cache[dev].load(std::memory_order_relaxed);
+    if (c > 0) return c - 1;
+  }
+  auto kern = gemm_pair_kernel<A_MN, B_MN, FAM>;
+  int slots = 0;
+  if (fl_func_smem((const void*)kern, CfgPair::SMEM_BYTES) == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(2 * num_sms());
+    cfg.blockDim = dim3(NUM_THREADS);
+    cfg.dynamicSmemBytes = CfgPair::SMEM_BYTES;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0) slots = n;
+  }
+  cudaGetLastError();  // a refused query leaves the single-SM kernel in use
+  if (cached) cache[dev].store(slots + 1, std::memory_order_relaxed);
   return slots;
 }
 

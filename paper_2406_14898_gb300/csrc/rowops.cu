@@ -12,14 +12,7 @@
 namespace {
 
 int sm_count() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 148;
-  }
-  return n;
+  return fl_sm_count();
 }
 
 FL_DEV float warp_sum(float v) {
@@ -330,7 +323,8 @@ __global__ void ln_bwd_reduce_kernel(int nblk, int H, int nv, const float* __res
   const int b0 = blockIdx.y * per, b1 = min(nblk, b0 + per);
   if (b0 >= b1) return;
   float s = 0.f;
-  for (int b = b0; b < b1; ++b) s += ws[(int64_t)b * nv * H + i];
+#pragma unroll 8
+  for (int b = b0; b < b1; ++b) s += ws[(int64_t)b * nv * H + i];  // independent loads: eight in flight
   atomicAdd(i < H ? dgamma + i : i < 2 * H ? dbeta + (i - H) : dcol + (i - 2 * H), s);
 }
 
@@ -339,13 +333,9 @@ int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, cons
                     const float* gamma, const void* resid, float alpha, void* dx_bf16, float* dx_f32, float* ws,
                     float* dgamma, float* dbeta, float* dcol, cudaStream_t st, int* status = nullptr) {
   const int smem = 2 * LNB_STAGES * H * (int)sizeof(T) + LNB_STAGES * 8;
-  static bool attr = false;
-  if (!attr) {
-    const int mx = 2 * LNB_STAGES * 4096 * (int)sizeof(T) + LNB_STAGES * 8;
-    FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<T, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx));
-    FL_CUDA_TRY(cudaFuncSetAttribute(ln_bwd_kernel<T, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx));
-    attr = true;
-  }
+  const int mx = 2 * LNB_STAGES * 4096 * (int)sizeof(T) + LNB_STAGES * 8;
+  FL_CUDA_TRY(fl_func_smem((const void*)ln_bwd_kernel<T, true>, mx));
+  FL_CUDA_TRY(fl_func_smem((const void*)ln_bwd_kernel<T, false>, mx));
   if (dcol)
     FL_CUDA_TRY(fl_launch(ln_bwd_kernel<T, true>, dim3(nblk), dim3(H / 8), smem, st, Tn, H, (const T*)dy, (const T*)x,
                           mean, rstd, gamma, (const T*)resid, alpha, (__nv_bfloat16*)dx_bf16, dx_f32, ws, status));
@@ -367,14 +357,8 @@ int dispatch_ln_fwd(int Tn, int H, const void* x, const float* gamma, const floa
   const int threads = H / 16 > 32 ? H / 16 : 32;
   const int ch = H / (8 * threads);
   const int smem = LN_STAGES * H * (int)sizeof(TX) + LN_STAGES * 8;
-  static bool attr = false;
-  if (!attr) {
-    FL_CUDA_TRY(cudaFuncSetAttribute(ln_fwd_bulk_kernel<TX, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
-    FL_CUDA_TRY(cudaFuncSetAttribute(ln_fwd_bulk_kernel<TX, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
-    attr = true;
-  }
+  FL_CUDA_TRY(fl_func_smem((const void*)ln_fwd_bulk_kernel<TX, 1>, LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
+  FL_CUDA_TRY(fl_func_smem((const void*)ln_fwd_bulk_kernel<TX, 2>, LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
   int grid = 3 * sm_count();
   if (grid > Tn) grid = Tn;
   const TX* xx = (const TX*)x;
