@@ -5,7 +5,6 @@ inputs that are exactly representable in bf16, and compares with the oracle's
 function of the same step (or, for the plain contractions, with the fp64 product
 that defines them).  Shapes span several tiles and a ragged tail.
 """
-import math
 
 import numpy as np
 import pytest
