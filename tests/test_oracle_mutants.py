@@ -154,6 +154,34 @@ def _alpha_ignored(orig):
     return f
 
 
+def _embedding_bwd_overwrites(orig):
+    def f(dX, tokens, vocab):
+        dE = np.zeros((vocab, dX.shape[1]))
+        dE[tokens] = dX  # a repeated token keeps one occurrence's gradient, not the sum
+        return dE
+    return f
+
+
+def _ce_mean_over_all_rows(orig):
+    def f(logits, labels):
+        loss, d = orig(logits, labels)
+        n, T = int((labels >= 0).sum()), labels.shape[0]
+        return (loss * n / T, d * n / T) if n else (loss, d)
+    return f
+
+
+def _ce_ignored_rows_keep_gradient(orig):
+    def f(logits, labels):
+        loss, d = orig(logits, labels)
+        d = d.copy()
+        ign = labels < 0
+        if ign.any() and (~ign).any():
+            sm = np.exp(logits[ign] - logits[ign].max(-1, keepdims=True))
+            d[ign] = sm / sm.sum(-1, keepdims=True) / int((~ign).sum())
+        return loss, d
+    return f
+
+
 FD = lambda: P.test_finite_difference_gradients(1)  # noqa: E731
 
 # (mistake, oracle attribute, mutant factory, pins that should catch it)
@@ -188,6 +216,12 @@ CASES = [
      [P.test_adamw_first_step_closed_form, P.test_adamw_matches_torch_over_steps]),
     ("AdamW with coupled (L2) decay", "adamw_update", _adamw_coupled_decay,
      [P.test_adamw_first_step_closed_form, P.test_adamw_matches_torch_over_steps]),
+    ("embedding gradient overwrites repeated tokens", "embedding_bwd", _embedding_bwd_overwrites,
+     [P.test_embedding_matches_torch]),
+    ("cross-entropy averaged over rows without a target", "cross_entropy", _ce_mean_over_all_rows,
+     [P.test_cross_entropy_matches_torch, P.test_cross_entropy_uniform_closed_form]),
+    ("cross-entropy gradient on rows without a target", "cross_entropy", _ce_ignored_rows_keep_gradient,
+     [P.test_cross_entropy_matches_torch, P.test_cross_entropy_uniform_closed_form]),
     ("residual scale alpha ignored", "BlockShape.of", _alpha_ignored,
      [lambda: P.test_zero_weight_block_closed_form(1), lambda: P.test_zero_weight_block_closed_form(0)]),
 ]
