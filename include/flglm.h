@@ -236,7 +236,8 @@ int fl_server_average_replicas(fl_server_t h);
 
 /* fp32 master values of tensor_id of block `block` of replica `replica` (0 <=
  * replica < cfg.n_replicas, or 0 with one replica) into host_dst[n] (n = the tensor's
- * element count); fl_server_get_param reads replica 0. */
+ * element count), synchronously; fl_server_get_param reads replica 0.  Errors:
+ * INVALID_ARG (replica, block or tensor id out of range, n not the element count, null). */
 int fl_server_get_replica_param(fl_server_t h, int32_t replica, int32_t block, int32_t tensor_id, float* host_dst,
                                 size_t n);
 
