@@ -128,11 +128,13 @@ int fl_k_gemm(const fl_gemm_args* args, int* status, void* stream);
 int fl_k_gemm_multi(const fl_gemm_args* probs, int32_t n, int* status, void* stream);
 
 /* Row LayerNorm, biased variance, fp32 statistics.  x: [T,H] of x_dtype (bf16 or fp32);
- * y: bf16 [T,H]; mean, rstd: [T].  H a power of two in [256, 4096]. */
+ * y: bf16 [T,H]; mean, rstd: [T].  H a multiple of 256 up to 2048, or a multiple of 512 up
+ * to 4096 (other H: UNSUPPORTED); T < 0: INVALID_ARG; T = 0 does nothing. */
 int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x_dtype, const float* gamma,
                        const float* beta, float eps, void* y, float* mean, float* rstd, void* stream);
 
-/* LayerNorm backward.  dy, x and resid are [T,H] of io_dtype (bf16 or fp32);
+/* LayerNorm backward.  dy, x and resid are [T,H] of io_dtype (bf16 or fp32), H a multiple
+ * of 256 up to 4096 (other H: UNSUPPORTED), T < 0: INVALID_ARG, T = 0 does nothing;
  * dx = rstd (g - mean(g) - xhat mean(g xhat)), g = gamma dy, plus resid_alpha * resid[t,:]
  * when resid != NULL; written to dx_bf16 and/or dx_f32 (either may be NULL, not both).
  * dgamma[H] += sum_t dy xhat and dbeta[H] += sum_t dy (fp32, accumulated).

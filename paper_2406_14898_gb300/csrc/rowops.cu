@@ -69,7 +69,7 @@ FL_DEV float2 block_sum2(float a, float b, float2 (*red)[32], int par) {
   return r;
 }
 
-// Forward: persistent CTAs of max(32, H/16) threads, each thread CH chunks of 8 elements
+// Forward: persistent CTAs of H/16 (CH = 2) or H/8 (CH = 1) threads, each thread CH chunks of 8 elements
 // (chunk c + k * blockDim.x) of every row.  The CTA walks rows blockIdx.x, + gridDim.x, ...
 // and keeps the next LN_STAGES of them in flight: one elected thread copies each whole row
 // into a shared-memory stage with one bulk copy (cp.async.bulk, completion on the stage's
@@ -350,11 +350,21 @@ int dispatch_ln_bwd(int nblk, int Tn, int H, const void* dy, const void* x, cons
   return FL_OK;
 }
 
+// Threads of the forward's CTA for hidden size H: H/16 (two 8-element chunks each) when that
+// is a whole number of warps, else H/8 (one chunk each); at most 8 warps (the kernel's
+// launch bound and its reduction array).
+int ln_fwd_threads(int H) { return (H / 16) % 32 == 0 ? H / 16 : H / 8; }
+bool ln_fwd_shape_ok(int H) {
+  if (H <= 0 || (H % 256) || H > 4096) return false;
+  const int t = ln_fwd_threads(H);
+  return t % 32 == 0 && t <= 256;
+}
+
 template <typename TX>
 int dispatch_ln_fwd(int Tn, int H, const void* x, const float* gamma, const float* beta, float eps, void* y,
                     float* mean, float* rstd, cudaStream_t st, int* status = nullptr) {
-  // max(32, H/16) threads of CH = H / (8 * threads) chunks (H a multiple of 256 up to 4096)
-  const int threads = H / 16 > 32 ? H / 16 : 32;
+  if (!ln_fwd_shape_ok(H)) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d", H);
+  const int threads = ln_fwd_threads(H);
   const int ch = H / (8 * threads);
   const int smem = LN_STAGES * H * (int)sizeof(TX) + LN_STAGES * 8;
   FL_CUDA_TRY(fl_func_smem((const void*)ln_fwd_bulk_kernel<TX, 1>, LN_STAGES * 4096 * (int)sizeof(TX) + LN_STAGES * 8));
@@ -590,7 +600,9 @@ int grid_for(int64_t n, int per_thread_block = 256) {
 
 extern "C" int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x_dtype, const float* gamma,
                                   const float* beta, float eps, void* y, float* mean, float* rstd, void* stream) {
-  if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d", H);
+  if (T < 0) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: negative T=%d", T);
+  if (!ln_fwd_shape_ok(H))
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d (a multiple of 256 up to 2048, or of 512 up to 4096)", H);
   if (!x || !gamma || !beta || !y || !mean || !rstd) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: null");
   if (x_dtype != FL_DT_BF16 && x_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: dtype");
   if (reinterpret_cast<uintptr_t>(x) & 15) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: x not 16-byte aligned");
@@ -608,7 +620,9 @@ extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const vo
                                   const float* mean, const float* rstd, const float* gamma, const void* resid,
                                   float resid_alpha, void* dx_bf16, float* dx_f32, float* dgamma, float* dbeta,
                                   void* workspace, void* stream) {
-  if (T < 0 || H <= 0 || (H % 256) || H > 4096) return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H=%d", H);
+  if (T < 0) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: negative T=%d", T);
+  if (H <= 0 || (H % 256) || H > 4096)
+    return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm bwd: H=%d (a multiple of 256 up to 4096)", H);
   if (!dy || !x || !mean || !rstd || !gamma || (!dx_bf16 && !dx_f32) || !dgamma || !dbeta || !workspace)
     return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: null");
   if (io_dtype != FL_DT_BF16 && io_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: dtype");

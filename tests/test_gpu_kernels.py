@@ -160,7 +160,7 @@ def test_gemm_rope_epilogue(F, hd, tile):
     assert rel_inf(f64(D), ref) < GEMM_TOL
 
 
-@pytest.mark.parametrize("H", [256, 4096])
+@pytest.mark.parametrize("H", [256, 768, 3072, 4096])  # 768: one chunk per thread; 3072: six warps
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 def test_layernorm_fwd_bwd(F, H, dtype):
     T = 77
@@ -208,6 +208,25 @@ def test_layernorm_fwd_bwd(F, H, dtype):
         assert rel_inf(f64(dxf), dxr) < 1e-4
         assert rel_inf(f64(dgam) - 0.5, dgr) < 1e-4
         assert rel_inf(f64(dbet) + 0.25, dbr) < 1e-4
+
+
+def test_layernorm_unsupported_widths(F):
+    """Hidden sizes the forward has no launch shape for (an odd multiple of 256 above 2048, a
+    width not a multiple of 256) and a negative row count are refused before any launch."""
+    H = 2304
+    x = torch.zeros((4, 4096), dtype=torch.bfloat16, device="cuda")
+    v = torch.zeros(4096, device="cuda")
+    y = torch.full((4, 4096), 1.0, dtype=torch.bfloat16, device="cuda")
+    st = torch.zeros(4, device="cuda")
+    for h, code in ((H, -7), (200, -7)):
+        with pytest.raises(F.FlError) as ei:
+            F.fl_k_layernorm_fwd(4, h, x, v, v, 1e-5, y, st, st)
+        assert ei.value.code == code
+    with pytest.raises(F.FlError) as ei:
+        F.fl_k_layernorm_fwd(-1, 256, x, v, v, 1e-5, y, st, st)
+    assert ei.value.code == -1
+    torch.cuda.synchronize()
+    assert (y == 1.0).all() and not st.any()
 
 
 @pytest.mark.parametrize("tile", ["auto", "pair"])
@@ -469,3 +488,41 @@ def test_gemm_adamw_epilogue(F, M, N, K, mn, tile):
     for got, want in ((wf, wr), (mf, mr), (vf, vr)):
         assert rel_inf(f64(got), f64(want)) < 1e-5
     np.testing.assert_array_equal(bits(wbf), bits(wf.to(torch.bfloat16)))
+
+
+def test_zero_size_calls(F):
+    """Degenerate sizes: a GEMM of M = 0 rows, LayerNorm forward and backward over T = 0
+    rows, AdamW over 0 parameters, column sums over 0 rows, and attention over one empty
+    segment are no-ops that succeed and leave every output untouched."""
+    H, N, K = 256, 256, 64
+    A = torch.zeros((8, K), dtype=torch.bfloat16, device="cuda")
+    B = torch.zeros((N, K), dtype=torch.bfloat16, device="cuda")
+    D = torch.full((8, N), 7.0, dtype=torch.bfloat16, device="cuda")
+    F.gemm(0, N, K, A, K, 0, B, K, 0, D, N)
+    x = torch.zeros((8, H), dtype=torch.bfloat16, device="cuda")
+    gam = torch.ones(H, device="cuda")
+    bet = torch.zeros(H, device="cuda")
+    y = torch.full((8, H), 3.0, dtype=torch.bfloat16, device="cuda")
+    mean = torch.full((8,), 5.0, device="cuda")
+    rstd = torch.full((8,), 5.0, device="cuda")
+    F.fl_k_layernorm_fwd(0, H, x, gam, bet, 1e-5, y, mean, rstd)
+    dgam = torch.full((H,), 2.0, device="cuda")
+    dbet = torch.full((H,), 2.0, device="cuda")
+    ws = torch.empty(max(F.fl_k_layernorm_bwd_workspace(1, H), 16), dtype=torch.uint8, device="cuda")
+    F.fl_k_layernorm_bwd(0, H, x, x, mean, rstd, gam, None, 0.0, y, dgam, dbet, ws)
+    w = torch.full((8,), 4.0, device="cuda")
+    F.fl_k_adamw(0, w, w, w, w, None, 1e-3, 0.9, 0.999, 1e-8, 0.0, 0.1, 0.001)
+    cs = torch.full((N,), 6.0, device="cuda")
+    F.fl_k_colsum(0, N, D, cs)
+    nh, hd = 2, 128
+    qkv = torch.zeros((8, 3 * nh * hd), dtype=torch.bfloat16, device="cuda")
+    cu = np.array([0, 0], np.int32)
+    tiles = torch.zeros(16, dtype=torch.int32, device="cuda")
+    o = torch.full((8, nh * hd), 9.0, dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((nh, 8), 9.0, device="cuda")
+    assert F.fl_k_attention_tiles(cu) == 0
+    F.fl_k_attention_fwd(0, nh, hd, qkv, cu, dev_i32(cu), tiles, o, lse)
+    torch.cuda.synchronize()
+    assert (D == 7.0).all() and (y == 3.0).all() and (mean == 5.0).all() and (rstd == 5.0).all()
+    assert (dgam == 2.0).all() and (dbet == 2.0).all() and (w == 4.0).all() and (cs == 6.0).all()
+    assert (o == 9.0).all() and (lse == 9.0).all() and not tiles.any()
