@@ -9,6 +9,12 @@
  * the FL_* codes of flglm.h; the message is in fl_server_last_error(NULL).
  * `status` (optional, device int) receives a nonzero code if a bounded wait inside
  * the kernel gave up; the kernel then returns without finishing its output.
+ * Alignment: a pointer must be aligned to the width its kernel accesses it with: 16 bytes
+ * for row tensors and parameter vectors read or written in 16-byte pieces (the operands
+ * and outputs of the GEMM, LayerNorm, attention, column-sum, AdamW and embedding-gather
+ * calls), 8 bytes for the GEMM's rotary table and AdamW's bf16 copy, 4 bytes for per-row
+ * scalars and index arrays; a misaligned pointer returns FL_ERR_INVALID_ARG before any
+ * work is enqueued.
  */
 #ifndef FLGLM_KERNELS_H
 #define FLGLM_KERNELS_H

@@ -137,6 +137,9 @@ extern "C" int fl_k_attention_fwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   if (cu_seqlens_host[0] != 0 || cu_seqlens_host[S] != T) return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: cu_seqlens");
   if (prefix_len < 0 || prefix_len > 128 || (prefix_len > 0 && (!prefix_k || !prefix_v)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: prefix (length 0..128)");
+  if (fl_misaligned(qkv, 16) || fl_misaligned(o, 16) || fl_misaligned(lse, 4) || fl_misaligned(cu_seqlens, 4) ||
+      fl_misaligned(tile_ws, 4) || fl_misaligned(context_lens, 4))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "attention fwd: qkv and o must be 16-byte aligned");
   int n = 0, n128 = 0;
   if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n, &n128)) return rc;
   AttnPrefix pre;
@@ -167,6 +170,12 @@ extern "C" int fl_k_attention_bwd(int32_t T, int32_t n_heads, int32_t head_dim, 
   if (prefix_len < 0 || prefix_len > 128 ||
       (prefix_len > 0 && (!prefix_k || !prefix_v || !dprefix_k || !dprefix_v)))
     return fl_internal_error(FL_ERR_INVALID_ARG, "attention bwd: prefix (length 0..128, gradients required)");
+  if (fl_misaligned(qkv, 16) || fl_misaligned(o, 16) || fl_misaligned(dout, 16) || fl_misaligned(dqkv, 16) ||
+      fl_misaligned(dprefix_k, 16) || fl_misaligned(dprefix_v, 16) || fl_misaligned(lse, 4) ||
+      fl_misaligned(delta_ws, 4) || fl_misaligned(cu_seqlens, 4) || fl_misaligned(tile_ws, 4) ||
+      fl_misaligned(context_lens, 4) || fl_misaligned(positions, 4) || fl_misaligned(block_positions, 4))
+    return fl_internal_error(FL_ERR_INVALID_ARG,
+                             "attention bwd: qkv, o, dout, dqkv and the prefix gradients must be 16-byte aligned");
   int n = 0, n128 = 0;
   if (int rc = upload_tiles(cu_seqlens_host, S, tile_ws, &n, &n128)) return rc;
   AttnPrefix pre;

@@ -173,6 +173,8 @@ extern "C" int fl_k_embedding_gather(int32_t T, int32_t H, const int32_t* tokens
                                      void* out, int* status, void* stream) {
   if (T < 0 || H <= 0 || (H % 8) || vocab < 1 || !tokens || !table || !out || !status)
     return fl_internal_error(FL_ERR_INVALID_ARG, "embedding gather: args");
+  if (fl_misaligned(table, 16) || fl_misaligned(out, 16) || fl_misaligned(tokens, 4) || fl_misaligned(status, 4))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "embedding gather: table and out must be 16-byte aligned");
   if (T == 0) return FL_OK;
   embed_gather_kernel<<<warps_grid(T), 256, 0, (cudaStream_t)stream>>>(T, H, tokens, (const bf16*)table, vocab,
                                                                        (bf16*)out, status);
@@ -184,6 +186,8 @@ extern "C" int fl_k_embedding_scatter_add(int32_t T, int32_t H, const int32_t* t
                                           float* dtable, void* stream) {
   if (T < 0 || H <= 0 || (H % 2) || vocab < 1 || !tokens || !dx || !dtable)
     return fl_internal_error(FL_ERR_INVALID_ARG, "embedding scatter: args");
+  if (fl_misaligned(dx, 4) || fl_misaligned(dtable, 4) || fl_misaligned(tokens, 4))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "embedding scatter: dx, dtable and tokens must be 4-byte aligned");
   if (T == 0) return FL_OK;
   embed_scatter_kernel<<<warps_grid(T), 256, 0, (cudaStream_t)stream>>>(T, H, tokens, vocab, (const bf16*)dx, dtable);
   FL_CUDA_TRY(cudaGetLastError());

@@ -108,3 +108,6 @@ int fl_internal_error(int code, const char* fmt, ...);
 // bytes); later calls return at once.
 int fl_sm_count();
 cudaError_t fl_func_smem(const void* func, int bytes);
+
+// True when p is not a multiple of `bytes` (a power of two); a null p counts as aligned.
+inline bool fl_misaligned(const void* p, uintptr_t bytes) { return (reinterpret_cast<uintptr_t>(p) & (bytes - 1)) != 0; }

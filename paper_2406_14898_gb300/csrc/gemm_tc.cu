@@ -110,6 +110,9 @@ int check_args(const fl_gemm_args* a) {
     return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: block positions only with the RoPE epilogue");
   }
   if (a->bias && !aligned16(a->bias)) return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: bias alignment");
+  if (fl_misaligned(a->rope_tab, 8) || fl_misaligned(a->pos, 4) || fl_misaligned(a->pos2, 4) ||
+      fl_misaligned(a->ln_mean, 4) || fl_misaligned(a->ln_rstd, 4))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "gemm: rope_tab must be 8-byte and per-row arrays 4-byte aligned");
   if (a->colsum && mode != FL_EPI_GELU_BWD)
     return fl_internal_error(FL_ERR_UNSUPPORTED, "gemm: column sums only with the GeLU-backward epilogue");
   if (a->colsum && !aligned16(a->colsum))

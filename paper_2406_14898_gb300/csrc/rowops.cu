@@ -605,7 +605,8 @@ extern "C" int fl_k_layernorm_fwd(int32_t T, int32_t H, const void* x, int32_t x
     return fl_internal_error(FL_ERR_UNSUPPORTED, "layernorm: H=%d (a multiple of 256 up to 2048, or of 512 up to 4096)", H);
   if (!x || !gamma || !beta || !y || !mean || !rstd) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: null");
   if (x_dtype != FL_DT_BF16 && x_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: dtype");
-  if (reinterpret_cast<uintptr_t>(x) & 15) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: x not 16-byte aligned");
+  if (fl_misaligned(x, 16) || fl_misaligned(gamma, 16) || fl_misaligned(beta, 16) || fl_misaligned(y, 16))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm: x, gamma, beta and y must be 16-byte aligned");
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
   return x_dtype == FL_DT_F32 ? dispatch_ln_fwd<float>(T, H, x, gamma, beta, eps, y, mean, rstd, st)
@@ -626,8 +627,10 @@ extern "C" int fl_k_layernorm_bwd(int32_t T, int32_t H, const void* dy, const vo
   if (!dy || !x || !mean || !rstd || !gamma || (!dx_bf16 && !dx_f32) || !dgamma || !dbeta || !workspace)
     return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: null");
   if (io_dtype != FL_DT_BF16 && io_dtype != FL_DT_F32) return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: dtype");
-  if ((reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(x)) & 15)
-    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd: dy / x not 16-byte aligned");
+  if (fl_misaligned(dy, 16) || fl_misaligned(x, 16) || fl_misaligned(gamma, 16) || fl_misaligned(resid, 16) ||
+      fl_misaligned(dx_bf16, 16) || fl_misaligned(dx_f32, 16) || fl_misaligned(workspace, 16))
+    return fl_internal_error(FL_ERR_INVALID_ARG,
+                             "layernorm bwd: dy, x, gamma, resid, dx and the workspace must be 16-byte aligned");
   if (T == 0) return FL_OK;
   cudaStream_t st = (cudaStream_t)stream;
   const int nblk = ln_bwd_blocks(T);
@@ -662,6 +665,8 @@ int fl_launch_layernorm_fwd_f32(int T, int H, const float* x, const float* gamma
 
 extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void* stream) {
   if (T < 0 || N <= 0 || (N % 8) || !x || !out) return fl_internal_error(FL_ERR_INVALID_ARG, "colsum: args");
+  if (fl_misaligned(x, 16) || fl_misaligned(out, 4))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "colsum: x must be 16-byte aligned");
   if (T == 0) return FL_OK;
   const int cblocks = (N + 255) / 256;
   int rblocks = (8 * sm_count() + cblocks - 1) / cblocks;  // ~8 CTAs (64 warps) per SM
@@ -677,6 +682,9 @@ extern "C" int fl_k_colsum(int32_t T, int32_t N, const void* x, float* out, void
 extern "C" int fl_k_adamw(int64_t n, float* w, float* g, float* m, float* v, void* w_bf16, float lr, float beta1,
                           float beta2, float eps, float weight_decay, float bc1, float bc2, void* stream) {
   if (n < 0 || (n % 4) || !w || !g || !m || !v) return fl_internal_error(FL_ERR_INVALID_ARG, "adamw: args (n %% 4)");
+  if (fl_misaligned(w, 16) || fl_misaligned(g, 16) || fl_misaligned(m, 16) || fl_misaligned(v, 16) ||
+      fl_misaligned(w_bf16, 8))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "adamw: w, g, m, v must be 16-byte and w_bf16 8-byte aligned");
   if (n == 0) return FL_OK;
   const int64_t n4 = n / 4;
   adamw_kernel<<<grid_for(n4), 256, 0, (cudaStream_t)stream>>>(n4, (float4*)w, (float4*)g, (float4*)m, (float4*)v,
@@ -867,8 +875,9 @@ extern "C" int fl_k_layernorm_bwd_noalloc(int32_t T, int32_t H, const void* dy, 
                              FL_LN_NOALLOC_MAX_H);
   if (!dy || !x || !mean || !rstd || !gamma || !dx || !dgamma || !dbeta)
     return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): null pointer");
-  if ((reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(x)) & 15)
-    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): dy / x not 16-byte aligned");
+  if (fl_misaligned(dy, 16) || fl_misaligned(x, 16) || fl_misaligned(gamma, 16) || fl_misaligned(resid, 16) ||
+      fl_misaligned(dx, 16))
+    return fl_internal_error(FL_ERR_INVALID_ARG, "layernorm bwd (no-alloc): dy, x, gamma, resid and dx must be 16-byte aligned");
   float* ws = nullptr;
   if (int rc = ln_scratch_address(&ws)) return rc;
   if (T == 0) return FL_OK;

@@ -75,7 +75,16 @@ def test_cfg_default_and_validation(F):
     assert F.lib().fl_client_destroy(None) == 0
 
 
+def no_gpu_here():
+    """The checks below pass made-up device addresses: they run only where no GPU exists, so
+    that a check that regressed could never launch a kernel on them."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("made-up device addresses: CPU-only check")
+
+
 def test_kernel_entry_points_validate_before_launch(F):
+    no_gpu_here()
     L = F.lib()
     a = F.fl_gemm_args()
     assert L.fl_k_gemm(ctypes.byref(a), None, None) == -1          # null operands
@@ -92,3 +101,66 @@ def test_kernel_entry_points_validate_before_launch(F):
     assert L.fl_k_gemm(ctypes.byref(a), None, None) == -7
     assert L.fl_k_layernorm_fwd(4, 300, None, 0, None, None, 1e-5, None, None, None, None) == -7
     assert L.fl_k_adamw(6, None, None, None, None, None, 1e-3, .9, .999, 1e-8, 0, .1, .001, None) == -1
+
+
+def test_kernel_entry_points_check_alignment(F):
+    """Every pointer a kernel reads or writes with vector accesses is checked for the width
+    it is accessed with; a misaligned one is refused (INVALID_ARG) before any CUDA call."""
+    no_gpu_here()
+    L = F.lib()
+    A = [0x100000 * (i + 1) for i in range(16)]          # made-up, 16-byte aligned, never dereferenced
+    odd = lambda p, b=4: p + b                           # noqa: E731
+    CUDA = -5  # aligned arguments pass the checks and fail at the first CUDA call (no device here)
+    # LayerNorm forward: x, gamma, beta, y
+    args = [4, 256, A[0], 0, A[1], A[2], 1e-5, A[3], A[4], A[5], None]
+    assert L.fl_k_layernorm_fwd(*args) == CUDA
+    for i in (2, 4, 5, 7):
+        bad = list(args)
+        bad[i] = odd(bad[i], 8)
+        assert L.fl_k_layernorm_fwd(*bad) == -1, i
+    # LayerNorm backward: dy, x, gamma, resid, dx_bf16, dx_f32, workspace
+    args = [4, 256, A[0], A[1], 0, A[2], A[3], A[4], A[5], 1.0, A[6], A[7], A[8], A[9], A[10], None]
+    assert L.fl_k_layernorm_bwd(*args) == CUDA
+    for i in (2, 3, 7, 8, 10, 11, 14):
+        bad = list(args)
+        bad[i] = odd(bad[i], 8)
+        assert L.fl_k_layernorm_bwd(*bad) == -1, i
+    args = [4, 256, A[0], A[1], A[2], A[3], A[4], A[5], 1.0, A[6], A[7], A[8], None]
+    assert L.fl_k_layernorm_bwd_noalloc(*args) == CUDA
+    for i in (2, 3, 6, 7, 9):
+        bad = list(args)
+        bad[i] = odd(bad[i], 8)
+        assert L.fl_k_layernorm_bwd_noalloc(*bad) == -1, i
+    # column sums, AdamW (w, g, m, v 16-byte, the bf16 copy 8-byte)
+    assert L.fl_k_colsum(4, 256, A[0], A[1], None) == CUDA
+    assert L.fl_k_colsum(4, 256, odd(A[0], 8), A[1], None) == -1
+    assert L.fl_k_adamw(8, A[0], A[1], A[2], A[3], A[4], 1e-3, .9, .999, 1e-8, 0., .1, .001, None) == CUDA
+    for i in (1, 2, 3, 4):
+        bad = [8, A[0], A[1], A[2], A[3], A[4], 1e-3, .9, .999, 1e-8, 0., .1, .001, None]
+        bad[i] = odd(bad[i])
+        assert L.fl_k_adamw(*bad) == -1, i
+    assert L.fl_k_adamw(8, A[0], A[1], A[2], A[3], odd(A[4]), 1e-3, .9, .999, 1e-8, 0., .1, .001, None) == -1
+    # embedding table / output rows (16-byte), scatter operands (4-byte)
+    assert L.fl_k_embedding_gather(4, 256, A[0], A[1], 10, A[2], A[3], None) == CUDA
+    assert L.fl_k_embedding_scatter_add(4, 256, A[0], 10, A[1], A[2], None) == CUDA
+    assert L.fl_k_embedding_gather(4, 256, A[0], odd(A[1], 8), 10, A[2], A[3], None) == -1
+    assert L.fl_k_embedding_gather(4, 256, A[0], A[1], 10, odd(A[2], 8), A[3], None) == -1
+    assert L.fl_k_embedding_scatter_add(4, 256, A[0], 10, odd(A[1], 2), A[2], None) == -1
+    # attention: o (forward); o, dout, dqkv and the prefix gradients (backward)
+    cu = (ctypes.c_int32 * 2)(0, 4)
+    assert L.fl_k_attention_fwd(4, 2, 128, A[0], cu, A[1], 1, A[2], A[3], A[4], None, None, 0, None, None) == CUDA
+    assert L.fl_k_attention_fwd(4, 2, 128, A[0], cu, A[1], 1, A[2], odd(A[3], 8), A[4], None, None, 0, None,
+                                None) == -1
+    bwd = [4, 2, 128, A[0], A[1], A[2], A[3], cu, A[4], 1, A[5], A[6], None, 64, A[7], A[8], A[9], 4, A[10],
+           A[11], None, None, None, None]
+    assert L.fl_k_attention_bwd(*bwd) == CUDA
+    for i in (4, 6, 14, 18, 19):
+        bad = list(bwd)
+        bad[i] = odd(bad[i], 8)
+        assert L.fl_k_attention_bwd(*bad) == -1, i
+    # GEMM: the rotary table is read as (cos, sin) pairs
+    a = F.fl_gemm_args(8, 384, 64, A[0], 64, 0, A[1], 64, 0, A[2], 384, F.FL_EPI_STORE)
+    a.rope_tab = A[3]
+    assert L.fl_k_gemm(ctypes.byref(a), None, None) == CUDA
+    a.rope_tab = odd(A[3])
+    assert L.fl_k_gemm(ctypes.byref(a), None, None) == -1
