@@ -237,6 +237,11 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
     const int row = blockIdx.x + it * gridDim.x;
     if (row >= Tn) break;
     const int st = it % LNB_STAGES;
+    // the row's statistics and the gain are requested before the stage wait, so that their
+    // latency passes while the bulk copy lands
+    float gcol[8];
+    load8<float>(gamma, c, gcol);
+    const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
     if (!__syncthreads_and(mbar_wait(full + st, (it / LNB_STAGES) & 1))) {
       if (c == 0) {
         report_status(status, FL_DEV_TIMEOUT_FULL);
@@ -244,7 +249,7 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
       }
       break;
     }
-    float d[8], xh[8], gcol[8];
+    float d[8], xh[8];
     if constexpr (sizeof(T) == 4) {
       const float4* sd = reinterpret_cast<const float4*>(lnb_smem + (2 * st) * row_bytes) + 2 * c;
       const float4* sx = reinterpret_cast<const float4*>(lnb_smem + (2 * st + 1) * row_bytes) + 2 * c;
@@ -255,8 +260,6 @@ __global__ void __launch_bounds__(512, 2) ln_bwd_kernel(int Tn, int H, const T* 
       unpack8(reinterpret_cast<const uint4*>(lnb_smem + (2 * st) * row_bytes)[c], d);
       unpack8(reinterpret_cast<const uint4*>(lnb_smem + (2 * st + 1) * row_bytes)[c], xh);
     }
-    load8<float>(gamma, c, gcol);
-    const float mu = __ldg(mean + row), rs = __ldg(rstd + row);
     float s1 = 0.f, s2 = 0.f;
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
