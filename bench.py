@@ -146,7 +146,9 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-        rows = [l.split(", ") for l in open(self.path).read().strip().splitlines() if l.strip()]
+        with open(self.path) as fh:
+            text = fh.read()
+        rows = [l.split(", ") for l in text.strip().splitlines() if l.strip()]
         os.unlink(self.path)
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
@@ -870,7 +872,8 @@ def ncu_traffic(path: str, workload_name: str):
     this workload and on the current GEMM source; else None."""
     if not os.path.exists(path) or workload_name not in os.path.basename(path):
         return None
-    txt = open(path).read()
+    with open(path) as fh:
+        txt = fh.read()
     if kernel_version() not in txt:
         return None
     for line in txt.splitlines():
@@ -891,7 +894,8 @@ def kernel_version() -> str:
     files = sorted(glob.glob(os.path.join(csrc, "gemm_*"))) + [os.path.join(csrc, "common.cuh"),
                                                                  os.path.join(csrc, "ptx.cuh")]
     for f in files:
-        h.update(open(f, "rb").read())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
     return h.hexdigest()[:16]
 
 

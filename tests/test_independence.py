@@ -26,7 +26,8 @@ def _sources(*patterns):
 def _code(path):
     """Source text without comments (# for Python, // and /* */ for C/CUDA) and strings
     that only document: what remains is what the file executes or includes."""
-    src = open(path).read()
+    with open(path) as fh:
+        src = fh.read()
     if path.endswith(".py"):
         src = re.sub(r'"""[\s\S]*?"""', "", src)
         return "\n".join(line.split("#", 1)[0] for line in src.splitlines())

@@ -13,7 +13,8 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 def declared_functions():
     names = set()
     for h in ("flglm.h", "flglm_kernels.h", "flglm_client.h"):
-        src = open(os.path.join(ROOT, "include", h)).read()
+        with open(os.path.join(ROOT, "include", h)) as fh:
+            src = fh.read()
         src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
         for m in re.finditer(r"\b(fl_[a-z0-9_]+)\s*\(", src):
             names.add(m.group(1))

@@ -64,7 +64,8 @@ def loss_and_grads(cfg, params, X, pk, dY):
 # ----------------------------------------------------------------------------- generator pins
 
 def test_splitmix64_published_vector():
-    vals = [int(l) for l in open(os.path.join(GOLDEN, "splitmix64_seed1234567.txt")) if l.strip() and not l.startswith("#")]
+    with open(os.path.join(GOLDEN, "splitmix64_seed1234567.txt")) as fh:
+        vals = [int(l) for l in fh if l.strip() and not l.startswith("#")]
     got = [int(v) for v in syn.raw_u64(1234567, 0, 5)]
     assert got == vals
 
