@@ -21,10 +21,19 @@
 //     h = alpha res1 + o Wd^T + bd,   res1 = a (residual_from_ln = 1) or x (0)
 //     m = LN2(h); y = alpha res2 + gelu(m W1^T + b1) W2^T + b2,  res2 = m or h
 //     LN: biased variance, gelu: tanh form;
+//   App. A (P-tuning v2): optional trainable prefix keys / values per block, K' =
+//     [prefix_key : key], V' = [prefix_value : value], seen by every query, not rotated;
+//     their gradients are summed over every segment;
+//   §4.1.1 (GLM blank infilling): optional per-segment context length c and mask-token
+//     position; own key u is seen by query t when u <= t or u < c (bidirectional context,
+//     causal span); positions are two-dimensional (context token t: (t, 0); span token t:
+//     (mask position, t - c + 1)), the second position rotating dims [rotary_dim,
+//     2 rotary_dim) of each head with the same frequencies;
 //   §4.1.4: Adam as AdamW with bias correction (decoupled decay, default 0).
 // The backward is the exact chain rule of the above.
 #include <omp.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -163,15 +172,15 @@ void layer_norm_bwd(const float* dy, const float* x, const float* mu, const floa
 }
 
 // Rotary encoding in place on the q or k part of a [T, 3H] row block (column offset
-// `col`): pairs (i, i + half) of dims [0, rotary_dim) of every head, position = index in
-// the own segment; inverse = rotation by the negative angle.
-void rope(float* qkv, int col, const std::vector<int>& pos, const Vec& cs, const Vec& sn, const flo_shape& sh,
-          int T, bool inverse, int ld) {
+// `col`): pairs (i, i + half) of dims [dim0, dim0 + rotary_dim) of every head, by the angle
+// of pos[t]; inverse = rotation by the negative angle.
+void rope(float* qkv, int col, int dim0, const std::vector<int>& pos, const Vec& cs, const Vec& sn,
+          const flo_shape& sh, int T, bool inverse, int ld) {
   const int half = sh.rotary_dim / 2;
 #pragma omp parallel for schedule(static)
   for (int t = 0; t < T; ++t)
     for (int h = 0; h < sh.n_heads; ++h) {
-      float* v = qkv + (size_t)t * ld + col + h * sh.head_dim;
+      float* v = qkv + (size_t)t * ld + col + h * sh.head_dim + dim0;
       for (int i = 0; i < half; ++i) {
         const float c = cs[(size_t)pos[t] * half + i];
         const float s = inverse ? -sn[(size_t)pos[t] * half + i] : sn[(size_t)pos[t] * half + i];
@@ -192,25 +201,45 @@ float gelu_grad(float u) {
   return 0.5f * (1.f + t) + 0.5f * u * (1.f - t * t) * c * (1.f + 3.f * a * u * u);
 }
 
-// Softmax probabilities of query t of one segment and head (causal: keys 0..t), into p.
-// qkv rows of the segment start at `base`; the scores are (q . k_u) / sqrt(d_h).
-void probs(const float* qkv, int ld, int H, int hd, int h, int t, float scale, float* p, float* lse) {
-  const float* q = qkv + (size_t)t * ld + h * hd;
+// The keys one segment's queries see for one head: the Lp prefix rows (pk / pv [Lp, H],
+// null when Lp = 0) then the segment's own rows (q | k | v at `seg`, row stride ld); c is
+// the segment's GLM context length (0: plainly causal).  Key j < Lp is prefix row j, key
+// Lp + u own row u.
+struct Keys {
+  const float* seg;
+  int ld, H, hd, h, L, c;
+  const float* pk;
+  const float* pv;
+  int Lp;
+  // keys 0 .. n(t) - 1 are the ones query t sees: every prefix key and the own keys u <= t,
+  // or u < c in the GLM context
+  int n(int t) const { return Lp + 1 + (c - 1 > t ? (c - 1 < L - 1 ? c - 1 : L - 1) : t); }
+  const float* k(int j) const { return j < Lp ? pk + (size_t)j * H + h * hd : seg + (size_t)(j - Lp) * ld + H + h * hd; }
+  const float* v(int j) const {
+    return j < Lp ? pv + (size_t)j * H + h * hd : seg + (size_t)(j - Lp) * ld + 2 * H + h * hd;
+  }
+  const float* q(int t) const { return seg + (size_t)t * ld + h * hd; }
+};
+
+// Softmax probabilities of query t over its visible keys 0 .. K.n(t) - 1, into p; the
+// scores are (q . k'_j) / sqrt(d_h).
+void probs(const Keys& K, int t, float scale, float* p) {
+  const float* q = K.q(t);
+  const int n = K.n(t);
   float mx = -INFINITY;
-  for (int u = 0; u <= t; ++u) {
-    const float* k = qkv + (size_t)u * ld + H + h * hd;
+  for (int j = 0; j < n; ++j) {
+    const float* k = K.k(j);
     float s = 0.f;
-    for (int d = 0; d < hd; ++d) s += q[d] * k[d];
-    p[u] = s * scale;
-    mx = std::fmax(mx, p[u]);
+    for (int d = 0; d < K.hd; ++d) s += q[d] * k[d];
+    p[j] = s * scale;
+    mx = std::fmax(mx, p[j]);
   }
   float l = 0.f;
-  for (int u = 0; u <= t; ++u) {
-    p[u] = std::exp(p[u] - mx);
-    l += p[u];
+  for (int j = 0; j < n; ++j) {
+    p[j] = std::exp(p[j] - mx);
+    l += p[j];
   }
-  for (int u = 0; u <= t; ++u) p[u] /= l;
-  if (lse) *lse = mx + std::log(l);
+  for (int j = 0; j < n; ++j) p[j] /= l;
 }
 
 struct Saved {
@@ -221,8 +250,24 @@ struct Block {
   const float *Wqkv, *bqkv, *Wd, *bd, *W1, *b1, *W2, *b2, *g1, *be1, *g2, *be2;
 };
 
+// Positions of a call: pos[t] rotates dims [0, rotary_dim) of every head; with GLM
+// segments (glm), pos2[t] rotates dims [rotary_dim, 2 rotary_dim); ctx[s] is segment s's
+// context length (all 0 without GLM).
+struct Positions {
+  std::vector<int> pos, pos2, ctx;
+  bool glm = false;
+  Vec cs, sn;  // (cos, sin) of position p, pair i at p * rotary_dim / 2 + i
+};
+
+void rope_all(float* qkv, const Positions& ps, const flo_shape& sh, int T, bool inverse) {
+  for (int col : {0, sh.hidden}) {
+    rope(qkv, col, 0, ps.pos, ps.cs, ps.sn, sh, T, inverse, 3 * sh.hidden);
+    if (ps.glm) rope(qkv, col, sh.rotary_dim, ps.pos2, ps.cs, ps.sn, sh, T, inverse, 3 * sh.hidden);
+  }
+}
+
 void block_fwd(const Block& P, const float* x, float* y, Saved& sv, const flo_shape& sh, int T, int S,
-               const int32_t* cu, const std::vector<int>& pos, const Vec& cs, const Vec& sn) {
+               const int32_t* cu, const Positions& ps, const float* pk, const float* pv, int Lp) {
   const int H = sh.hidden, F = sh.ffn_hidden, nh = sh.n_heads, hd = sh.head_dim;
   const size_t TH = (size_t)T * H;
   sv.x.assign(x, x + TH);
@@ -232,8 +277,7 @@ void block_fwd(const Block& P, const float* x, float* y, Saved& sv, const flo_sh
   layer_norm_fwd(x, P.g1, P.be1, sh.ln_eps, sv.a.data(), sv.mu1.data(), sv.rs1.data(), T, H);
   sv.qkv.resize(3 * TH);
   matmul_nt(sv.a.data(), P.Wqkv, P.bqkv, sv.qkv.data(), T, 3 * H, H);
-  rope(sv.qkv.data(), 0, pos, cs, sn, sh, T, false, 3 * H);
-  rope(sv.qkv.data(), H, pos, cs, sn, sh, T, false, 3 * H);
+  rope_all(sv.qkv.data(), ps, sh, T, false);
   sv.o.assign(TH, 0.f);
   const float scale = 1.f / std::sqrt((float)hd);
 #pragma omp parallel
@@ -243,14 +287,14 @@ void block_fwd(const Block& P, const float* x, float* y, Saved& sv, const flo_sh
     for (int sh_ = 0; sh_ < S * nh; ++sh_) {
       const int s = sh_ / nh, h = sh_ % nh;
       const int a0 = cu[s], L = cu[s + 1] - cu[s];
-      p.resize(L > 0 ? L : 1);
-      const float* seg = sv.qkv.data() + (size_t)a0 * 3 * H;
+      const Keys K{sv.qkv.data() + (size_t)a0 * 3 * H, 3 * H, H, hd, h, L, ps.ctx[s], pk, pv, Lp};
+      p.resize(Lp + (L > 0 ? L : 1));
       for (int t = 0; t < L; ++t) {
-        probs(seg, 3 * H, H, hd, h, t, scale, p.data(), nullptr);
+        probs(K, t, scale, p.data());
         float* o = sv.o.data() + (size_t)(a0 + t) * H + h * hd;
-        for (int u = 0; u <= t; ++u) {
-          const float* v = seg + (size_t)u * 3 * H + 2 * H + h * hd;
-          for (int d = 0; d < hd; ++d) o[d] += p[u] * v[d];
+        for (int j = 0; j < K.n(t); ++j) {
+          const float* v = K.v(j);
+          for (int d = 0; d < hd; ++d) o[d] += p[j] * v[d];
         }
       }
     }
@@ -273,8 +317,11 @@ void block_fwd(const Block& P, const float* x, float* y, Saved& sv, const flo_sh
   for (size_t i = 0; i < TH; ++i) y[i] = al * res2[i] + y[i];
 }
 
+// dpk / dpv (with a prefix): fp32 [Lp, H] accumulators of the prefix gradients, summed
+// over the segments in order.
 void block_bwd(const Block& P, float* const* G, const Saved& sv, const float* dy, float* dx, const flo_shape& sh,
-               int T, int S, const int32_t* cu, const std::vector<int>& pos, const Vec& cs, const Vec& sn) {
+               int T, int S, const int32_t* cu, const Positions& ps, const float* pk, const float* pv, int Lp,
+               float* dpk, float* dpv) {
   const int H = sh.hidden, F = sh.ffn_hidden, nh = sh.n_heads, hd = sh.head_dim;
   const size_t TH = (size_t)T * H;
   const float al = sh.alpha;
@@ -303,6 +350,8 @@ void block_bwd(const Block& P, float* const* G, const Saved& sv, const float* dy
   // dK = dS^T Q / sqrt(d_h); gradients w.r.t. the rotated q, k
   Vec dqkv(3 * TH, 0.f);
   const float scale = 1.f / std::sqrt((float)hd);
+  // prefix gradients of each (segment, head), added in segment order after the loop
+  std::vector<Vec> dpre(Lp > 0 ? (size_t)S * nh : 0);
 #pragma omp parallel
   {
     Vec p, dp;
@@ -310,32 +359,38 @@ void block_bwd(const Block& P, float* const* G, const Saved& sv, const float* dy
     for (int sh_ = 0; sh_ < S * nh; ++sh_) {
       const int s = sh_ / nh, h = sh_ % nh;
       const int a0 = cu[s], L = cu[s + 1] - cu[s];
-      p.resize(L > 0 ? L : 1);
-      dp.resize(L > 0 ? L : 1);
-      const float* seg = sv.qkv.data() + (size_t)a0 * 3 * H;
+      const Keys K{sv.qkv.data() + (size_t)a0 * 3 * H, 3 * H, H, hd, h, L, ps.ctx[s], pk, pv, Lp};
+      p.resize(Lp + (L > 0 ? L : 1));
+      dp.resize(Lp + (L > 0 ? L : 1));
       float* dseg = dqkv.data() + (size_t)a0 * 3 * H;
+      float* dpkv = nullptr;  // [2][Lp][hd]: this (segment, head)'s prefix key and value gradients
+      if (Lp > 0) {
+        dpre[sh_].assign((size_t)2 * Lp * hd, 0.f);
+        dpkv = dpre[sh_].data();
+      }
       for (int t = 0; t < L; ++t) {
-        probs(seg, 3 * H, H, hd, h, t, scale, p.data(), nullptr);
+        probs(K, t, scale, p.data());
+        const int n = K.n(t);
         const float* d_o = dO.data() + (size_t)(a0 + t) * H + h * hd;
         float rs = 0.f;
-        for (int u = 0; u <= t; ++u) {
-          const float* v = seg + (size_t)u * 3 * H + 2 * H + h * hd;
+        for (int j = 0; j < n; ++j) {
+          const float* v = K.v(j);
           float x = 0.f;
           for (int d = 0; d < hd; ++d) x += d_o[d] * v[d];
-          dp[u] = x;
-          rs += x * p[u];
+          dp[j] = x;
+          rs += x * p[j];
         }
-        const float* q = seg + (size_t)t * 3 * H + h * hd;
+        const float* q = K.q(t);
         float* dq = dseg + (size_t)t * 3 * H + h * hd;
-        for (int u = 0; u <= t; ++u) {
-          const float ds = p[u] * (dp[u] - rs);
-          const float* k = seg + (size_t)u * 3 * H + H + h * hd;
-          float* dk = dseg + (size_t)u * 3 * H + H + h * hd;
-          float* dv = dseg + (size_t)u * 3 * H + 2 * H + h * hd;
+        for (int j = 0; j < n; ++j) {
+          const float ds = p[j] * (dp[j] - rs);
+          const float* k = K.k(j);
+          float* dk = j < Lp ? dpkv + (size_t)j * hd : dseg + (size_t)(j - Lp) * 3 * H + H + h * hd;
+          float* dv = j < Lp ? dpkv + (size_t)(Lp + j) * hd : dseg + (size_t)(j - Lp) * 3 * H + 2 * H + h * hd;
           for (int d = 0; d < hd; ++d) {
             dq[d] += ds * k[d];
             dk[d] += ds * q[d];
-            dv[d] += p[u] * d_o[d];
+            dv[d] += p[j] * d_o[d];
           }
         }
       }
@@ -346,10 +401,18 @@ void block_bwd(const Block& P, float* const* G, const Saved& sv, const float* dy
           r[H + d] *= scale;
         }
       }
+      for (int i = 0; i < Lp * hd; ++i) dpkv[i] *= scale;
     }
   }
-  rope(dqkv.data(), 0, pos, cs, sn, sh, T, true, 3 * H);
-  rope(dqkv.data(), H, pos, cs, sn, sh, T, true, 3 * H);
+  for (int s = 0; s < S; ++s)
+    for (int h = 0; h < nh; ++h)
+      for (int j = 0; j < Lp; ++j)
+        for (int d = 0; d < hd; ++d) {
+          const float* g = dpre[(size_t)s * nh + h].data();
+          dpk[(size_t)j * H + h * hd + d] += g[(size_t)j * hd + d];
+          dpv[(size_t)j * H + h * hd + d] += g[(size_t)(Lp + j) * hd + d];
+        }
+  rope_all(dqkv.data(), ps, sh, T, true);
   matmul_tn_acc(dqkv.data(), sv.a.data(), G[0], T, 3 * H, H);
   colsum_acc(dqkv.data(), G[1], T, 3 * H);
   Vec da(TH);
@@ -372,40 +435,64 @@ int flo_threads(void) { return omp_get_max_threads(); }
 // [cu[s], cu[s+1])) through n_blocks blocks to y [T, H]; then dy [T, H] back to dx [T, H],
 // the weight gradients added into grads.  params / grads: n_blocks x 12 pointers in the
 // order Wqkv [3H,H], bqkv [3H], Wd [H,H], bd [H], W1 [F,H], b1 [F], W2 [H,F], b2 [H],
-// gamma1, beta1, gamma2, beta2 [H] (fp32, row-major).  Returns 0, or -1 on a bad argument.
-int flo_server_fwd_bwd(const flo_shape* shp, int32_t n_blocks, const float* const* params, float* const* grads,
-                       int32_t S, const int32_t* cu, const float* x, const float* dy, float* y, float* dx) {
+// gamma1, beta1, gamma2, beta2 [H] (fp32, row-major).
+// ctx / mask_pos (int32 [S] each, or null): GLM segments (§4.1.1), context length c in
+// [0, L_s] and mask-token position in [0, c) (null mask_pos: c - 1); needs rotary_dim =
+// head_dim / 2.  prefix_len in 0..: with prefix_len > 0, prefixes / prefix_grads hold
+// n_blocks x 2 pointers to the fp32 [prefix_len, H] prefix keys and values of each block
+// (App. A) and their gradient accumulators.  Returns 0, or -1 on a bad argument.
+int flo_server_fwd_bwd_ext(const flo_shape* shp, int32_t n_blocks, const float* const* params, float* const* grads,
+                           int32_t S, const int32_t* cu, const int32_t* ctx, const int32_t* mask_pos,
+                           int32_t prefix_len, const float* const* prefixes, float* const* prefix_grads,
+                           const float* x, const float* dy, float* y, float* dx) {
   if (!shp || n_blocks < 1 || !params || !grads || S < 1 || !cu || !x || !dy || !y || !dx) return -1;
+  if (prefix_len < 0 || (prefix_len > 0 && (!prefixes || !prefix_grads))) return -1;
   const flo_shape sh = *shp;
   if (sh.hidden != sh.n_heads * sh.head_dim || sh.rotary_dim < 2 || sh.rotary_dim % 2 ||
       sh.rotary_dim > sh.head_dim || cu[0] != 0)
     return -1;
+  if (ctx && 2 * sh.rotary_dim != sh.head_dim) return -1;
   for (int s = 0; s < S; ++s)
     if (cu[s + 1] < cu[s]) return -1;
   const int T = cu[S], H = sh.hidden;
   if (T < 1) return -1;
-  std::vector<int> pos(T);
+  Positions ps;
+  ps.glm = ctx != nullptr;
+  ps.pos.resize(T);
+  ps.pos2.assign(T, 0);
+  ps.ctx.assign(S, 0);
   int max_pos = 0;
-  for (int s = 0; s < S; ++s)
-    for (int t = cu[s]; t < cu[s + 1]; ++t) {
-      pos[t] = t - cu[s];
-      max_pos = pos[t] > max_pos ? pos[t] : max_pos;
+  for (int s = 0; s < S; ++s) {
+    const int L = cu[s + 1] - cu[s];
+    const int c = ctx ? ctx[s] : 0;
+    const int mp = !ctx ? 0 : mask_pos ? mask_pos[s] : c - 1;
+    if (c < 0 || c > L || (c > 0 && (mp < 0 || mp >= c))) return -1;
+    ps.ctx[s] = c;
+    for (int t = 0; t < L; ++t) {
+      const bool span = c > 0 && t >= c;
+      ps.pos[cu[s] + t] = span ? mp : t;
+      ps.pos2[cu[s] + t] = span ? t - c + 1 : 0;
+      max_pos = std::max(max_pos, std::max(ps.pos[cu[s] + t], ps.pos2[cu[s] + t]));
     }
+  }
   // rotation angles p base^(-2i/rotary_dim), evaluated in double and rounded to fp32
   const int half = sh.rotary_dim / 2;
-  Vec cs((size_t)(max_pos + 1) * half), sn((size_t)(max_pos + 1) * half);
+  ps.cs.resize((size_t)(max_pos + 1) * half);
+  ps.sn.resize((size_t)(max_pos + 1) * half);
   for (int p = 0; p <= max_pos; ++p)
     for (int i = 0; i < half; ++i) {
       const double ang = p * std::pow((double)sh.rope_base, -2.0 * i / sh.rotary_dim);
-      cs[(size_t)p * half + i] = (float)std::cos(ang);
-      sn[(size_t)p * half + i] = (float)std::sin(ang);
+      ps.cs[(size_t)p * half + i] = (float)std::cos(ang);
+      ps.sn[(size_t)p * half + i] = (float)std::sin(ang);
     }
+  const int Lp = prefix_len;
+  auto pre = [&](int b, int i) { return Lp > 0 ? prefixes[2 * b + i] : nullptr; };
   std::vector<Saved> saved(n_blocks);
   Vec cur(x, x + (size_t)T * H), nxt((size_t)T * H);
   for (int b = 0; b < n_blocks; ++b) {
     const float* const* p = params + 12 * b;
     const Block P{p[0], p[1], p[2], p[3], p[4], p[5], p[6], p[7], p[8], p[9], p[10], p[11]};
-    block_fwd(P, cur.data(), nxt.data(), saved[b], sh, T, S, cu, pos, cs, sn);
+    block_fwd(P, cur.data(), nxt.data(), saved[b], sh, T, S, cu, ps, pre(b, 0), pre(b, 1), Lp);
     cur.swap(nxt);
   }
   std::memcpy(y, cur.data(), sizeof(float) * T * H);
@@ -413,12 +500,20 @@ int flo_server_fwd_bwd(const flo_shape* shp, int32_t n_blocks, const float* cons
   for (int b = n_blocks - 1; b >= 0; --b) {
     const float* const* p = params + 12 * b;
     const Block P{p[0], p[1], p[2], p[3], p[4], p[5], p[6], p[7], p[8], p[9], p[10], p[11]};
-    block_bwd(P, grads + 12 * b, saved[b], cur.data(), nxt.data(), sh, T, S, cu, pos, cs, sn);
+    block_bwd(P, grads + 12 * b, saved[b], cur.data(), nxt.data(), sh, T, S, cu, ps, pre(b, 0), pre(b, 1), Lp,
+              Lp > 0 ? prefix_grads[2 * b] : nullptr, Lp > 0 ? prefix_grads[2 * b + 1] : nullptr);
     saved[b] = Saved();
     cur.swap(nxt);
   }
   std::memcpy(dx, cur.data(), sizeof(float) * T * H);
   return 0;
+}
+
+// The server call without GLM segments or a prefix.
+int flo_server_fwd_bwd(const flo_shape* shp, int32_t n_blocks, const float* const* params, float* const* grads,
+                       int32_t S, const int32_t* cu, const float* x, const float* dy, float* y, float* dx) {
+  return flo_server_fwd_bwd_ext(shp, n_blocks, params, grads, S, cu, nullptr, nullptr, 0, nullptr, nullptr, x, dy,
+                                y, dx);
 }
 
 // AdamW with bias correction at step t >= 1 (§4.1.4): m = b1 m + (1-b1) g,

@@ -31,6 +31,11 @@ def lib():
         L.flo_server_fwd_bwd.argtypes = [C.POINTER(_Shape), C.c_int32, C.POINTER(C.c_void_p),
                                          C.POINTER(C.c_void_p), C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                          C.c_void_p, C.c_void_p]
+        L.flo_server_fwd_bwd_ext.restype = C.c_int
+        L.flo_server_fwd_bwd_ext.argtypes = [C.POINTER(_Shape), C.c_int32, C.POINTER(C.c_void_p),
+                                             C.POINTER(C.c_void_p), C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                             C.c_int32, C.POINTER(C.c_void_p), C.POINTER(C.c_void_p), C.c_void_p,
+                                             C.c_void_p, C.c_void_p, C.c_void_p]
         L.flo_adamw.restype = C.c_int
         L.flo_adamw.argtypes = [C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
                                 C.c_float, C.c_float, C.c_float, C.c_float, C.c_float]
@@ -53,10 +58,13 @@ def shape_of(cfg) -> _Shape:
 
 
 def server_fwd_bwd(cfg, params: Sequence[Sequence[np.ndarray]], grads: List[List[np.ndarray]],
-                   cu_seqlens: Sequence[int], x: np.ndarray, dy: np.ndarray):
+                   cu_seqlens: Sequence[int], x: np.ndarray, dy: np.ndarray, context_lens=None, mask_pos=None,
+                   prefixes=None, prefix_grads=None):
     """Packed tokens x [T, H] through the blocks (params[b] = the 12 fp32 tensors of block b)
     and dy [T, H] back; returns (y, dx) [T, H] fp32 and adds the weight gradients into
-    `grads` (fp32 arrays, same shapes as params, updated in place)."""
+    `grads` (fp32 arrays, same shapes as params, updated in place).  context_lens /
+    mask_pos (one per segment): GLM segments; prefixes[b] = (prefix keys, prefix values)
+    [Lp, H] of block b, whose gradients are added into prefix_grads[b] (fp32, in place)."""
     nb = len(params)
     ps = [[_f32(p) for p in blk] for blk in params]
     for blk in grads:
@@ -71,8 +79,21 @@ def server_fwd_bwd(cfg, params: Sequence[Sequence[np.ndarray]], grads: List[List
     y = np.empty_like(x)
     dx = np.empty_like(x)
     sh = shape_of(cfg)
-    rc = lib().flo_server_fwd_bwd(C.byref(sh), nb, pp, gp, len(cu) - 1, cu.ctypes.data, x.ctypes.data, dy.ctypes.data,
-                                  y.ctypes.data, dx.ctypes.data)
+    ctx = None if context_lens is None else np.ascontiguousarray(context_lens, np.int32)
+    mp = None if mask_pos is None else np.ascontiguousarray(mask_pos, np.int32)
+    Lp, pre, pg = 0, None, None
+    if prefixes is not None:
+        pf = [[_f32(p) for p in blk] for blk in prefixes]
+        for blk in prefix_grads:
+            for g in blk:
+                if g.dtype != np.float32 or not g.flags.c_contiguous:
+                    raise ValueError("prefix_grads must be contiguous float32 arrays")
+        Lp = pf[0][0].shape[0]
+        pre = (C.c_void_p * (2 * nb))(*[p.ctypes.data for blk in pf for p in blk[:2]])
+        pg = (C.c_void_p * (2 * nb))(*[g.ctypes.data for blk in prefix_grads for g in blk[:2]])
+    rc = lib().flo_server_fwd_bwd_ext(C.byref(sh), nb, pp, gp, len(cu) - 1, cu.ctypes.data,
+                                      None if ctx is None else ctx.ctypes.data, None if mp is None else mp.ctypes.data,
+                                      Lp, pre, pg, x.ctypes.data, dy.ctypes.data, y.ctypes.data, dx.ctypes.data)
     if rc != 0:
         raise ValueError(f"flo_server_fwd_bwd: bad arguments (rc {rc})")
     return y, dx

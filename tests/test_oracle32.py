@@ -139,3 +139,83 @@ def test_bad_arguments():
     with pytest.raises(ValueError):
         O32.adamw(np.zeros(2, np.float32), np.zeros(2, np.float32), np.zeros(2, np.float32),
                   np.zeros(2, np.float32), 0, 1e-3, 0.9, 0.999, 1e-8, 0.0)
+
+
+def _fp64(cfg, params, states, grads, prefixes=None, ctx=None, mp=None):
+    ref = O.OracleServer(cfg, params, prefixes)
+    ro = ref.forward([syn.bf16_bits_to_f64(s) for s in states], ctx, mp)
+    rg = ref.backward([syn.bf16_bits_to_f64(g) for g in grads])
+    cat = lambda rs: np.concatenate([r.reshape(-1, cfg.hidden) for r in rs])  # noqa: E731
+    return cat(ro), cat(rg), ref.grads
+
+
+@pytest.mark.parametrize("rfl,Lp,glm", [(1, 0, True), (0, 0, True), (1, 3, False), (1, 3, True), (0, 2, True)],
+                         ids=["glm", "glm_pre_ln", "prefix", "prefix_glm", "prefix_glm_pre_ln"])
+def test_glm_and_prefix_match_fp64_oracle(rfl, Lp, glm):
+    """§4.1.1 GLM segments (bidirectional context, causal span, 2D positions) and App. A
+    P-tuning prefixes, two blocks over ragged segments: outputs, input gradients, the 12
+    weight gradients and the prefix key / value gradients within fp32 rounding of the fp64
+    oracle."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, client_batch=1, seq_lens=(13, 9, 5, 1), residual_from_ln=rfl,
+                                    residual_alpha=2.0 if rfl else 1.0, prefix_len=Lp)
+    params = syn.init_params(cfg)
+    rng = np.random.default_rng(40 + Lp)
+    prefixes = [[(0.5 * rng.standard_normal((Lp, cfg.hidden))) for _ in range(2)] for _ in range(cfg.n_blocks)] \
+        if Lp else None
+    ctx, mp = ([6, 0, 5, 1], [2, 0, 4, 0]) if glm else (None, None)
+    states, grads, x, dy, cu = _inputs(cfg)
+    ro, rg, rgrads = _fp64(cfg, params, states, grads, prefixes, ctx, mp)
+    g = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+    pg = [[np.zeros((Lp, cfg.hidden), np.float32) for _ in range(2)] for _ in range(cfg.n_blocks)] if Lp else None
+    y, dx = O32.server_fwd_bwd(cfg, params, g, cu, x, dy, ctx, mp, prefixes, pg)
+    assert _rel(y, ro) < 1e-5
+    assert _rel(dx, rg) < 1e-5
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            assert _rel(g[b][t], rgrads[b][t]) < 1e-5, (b, syn.TENSOR_NAMES[t])
+        for j in range(2 if Lp else 0):
+            assert _rel(pg[b][j], rgrads[b][12 + j]) < 1e-5, (b, "prefix", j)
+
+
+def test_glm_and_prefix_batching_invariant():
+    """§3.3 stacking with GLM segments and a shared prefix: packed outputs and input
+    gradients equal each segment run alone bit for bit; weight and prefix gradients are the
+    sum of the per-segment runs within fp32 rounding."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, client_batch=1, seq_lens=(11, 6, 3), prefix_len=2)
+    params = syn.init_params(cfg)
+    rng = np.random.default_rng(44)
+    prefixes = [[(0.5 * rng.standard_normal((2, cfg.hidden))) for _ in range(2)] for _ in range(cfg.n_blocks)]
+    ctx, mp = [4, 0, 3], [1, 0, 2]
+    states, grads, x, dy, cu = _inputs(cfg)
+    g = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+    pg = [[np.zeros((2, cfg.hidden), np.float32) for _ in range(2)] for _ in range(cfg.n_blocks)]
+    y, dx = O32.server_fwd_bwd(cfg, params, g, cu, x, dy, ctx, mp, prefixes, pg)
+    gs = [[np.zeros(p.shape, np.float64) for p in blk] for blk in params]
+    pgs = [[np.zeros((2, cfg.hidden), np.float64) for _ in range(2)] for _ in range(cfg.n_blocks)]
+    for s in range(len(cfg.seq_lens)):
+        a, b = cu[s], cu[s + 1]
+        g1 = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+        pg1 = [[np.zeros((2, cfg.hidden), np.float32) for _ in range(2)] for _ in range(cfg.n_blocks)]
+        y1, dx1 = O32.server_fwd_bwd(cfg, params, g1, [0, b - a], x[a:b], dy[a:b], [ctx[s]], [mp[s]], prefixes, pg1)
+        np.testing.assert_array_equal(y1, y[a:b])
+        np.testing.assert_array_equal(dx1, dx[a:b])
+        for bb in range(cfg.n_blocks):
+            for t in range(12):
+                gs[bb][t] += g1[bb][t]
+            for j in range(2):
+                pgs[bb][j] += pg1[bb][j]
+    for bb in range(cfg.n_blocks):
+        for t in range(12):
+            assert _rel(g[bb][t], gs[bb][t]) < 1e-5
+        for j in range(2):
+            assert _rel(pg[bb][j], pgs[bb][j]) < 1e-5
+
+
+def test_glm_and_prefix_bad_arguments():
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=1, client_batch=1, seq_lens=(4,))
+    params = syn.init_params(cfg)
+    x = np.zeros((4, cfg.hidden), np.float32)
+    g = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+    for ctx, mp in (([5], [0]), ([3], [3]), ([-1], [0])):   # context past the segment, [M] outside it, negative
+        with pytest.raises(ValueError):
+            O32.server_fwd_bwd(cfg, params, g, [0, 4], x, x, ctx, mp)
