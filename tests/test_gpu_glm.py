@@ -245,3 +245,46 @@ def test_glm_argument_errors(F):
     srv.backward(st, st)
     srv.sync()
     srv.close()
+
+
+def test_glm_prefix_parity_vs_fp32_oracle(F):
+    """GLM segments with P-tuning v2 prefixes, two blocks, against the fp32 C++ oracle:
+    outputs, input gradients, the 12 weight gradients and the prefix key / value gradients
+    of every block."""
+    from oracle import oracle32 as O32
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=2, client_batch=2, seq_lens=(64, 90), prefix_len=20)
+    ctx, mp = syn.glm_structure(cfg)
+    params = syn.init_params(cfg)
+    prefixes = [syn.init_prefix(cfg, b) for b in range(cfg.n_blocks)]
+    srv = F.Server(F.make_cfg(cfg, cfg.tokens), cfg.seed)
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            srv.set_param(b, t, params[b][t])
+        srv.set_param(b, F.FL_T_PREFIX_K, prefixes[b][0])
+        srv.set_param(b, F.FL_T_PREFIX_V, prefixes[b][1])
+    states, grads = syn.client_states(cfg), syn.client_grads(cfg)
+    st = [dev_bf16_from_bits(s) for s in states]
+    outs = [torch.empty_like(s) for s in st]
+    gi = [torch.empty_like(s) for s in st]
+    srv.forward(st, cfg.seq_lens, outs, context_lens=ctx, mask_pos=mp)
+    srv.backward([dev_bf16_from_bits(g) for g in grads], gi)
+    srv.sync()
+    H = cfg.hidden
+    x = np.concatenate([syn.bf16_bits_to_f64(s).reshape(-1, H) for s in states])
+    dy = np.concatenate([syn.bf16_bits_to_f64(g).reshape(-1, H) for g in grads])
+    cu = np.concatenate([[0], np.cumsum([L for L in cfg.seq_lens for _ in range(cfg.client_batch)])])
+    g32 = [[np.zeros(p.shape, np.float32) for p in blk] for blk in params]
+    pg32 = [[np.zeros(np.shape(p), np.float32) for p in pre] for pre in prefixes]
+    y, dx = O32.server_fwd_bwd(cfg, params, g32, cu, x, dy, ctx, mp, prefixes, pg32)
+    y_gpu = np.concatenate([f64(o).reshape(-1, H) for o in outs])
+    dx_gpu = np.concatenate([f64(g).reshape(-1, H) for g in gi])
+    assert rel_inf(y_gpu, y) < OUT_TOL, rel_inf(y_gpu, y)
+    assert rel_inf(dx_gpu, dx) < GRAD_TOL, rel_inf(dx_gpu, dx)
+    for b in range(cfg.n_blocks):
+        for t in range(12):
+            e = rel_inf(srv.get_grad(b, t), g32[b][t].reshape(-1))
+            assert e < GRAD_TOL, ("wgrad", b, syn.TENSOR_NAMES[t], e)
+        for j, tid in enumerate((F.FL_T_PREFIX_K, F.FL_T_PREFIX_V)):
+            e = rel_inf(srv.get_grad(b, tid), pg32[b][j].reshape(-1))
+            assert e < GRAD_TOL, ("prefix grad", b, j, e)
+    srv.close()
