@@ -182,6 +182,29 @@ def _ce_ignored_rows_keep_gradient(orig):
     return f
 
 
+def _prefix_grads_halved(orig):
+    def f(*a, **kw):
+        r = list(orig(*a, **kw))
+        if len(r) == 5:  # a prefix: dq, dk, dv, dprefix_k, dprefix_v
+            r[3], r[4] = 0.5 * r[3], 0.5 * r[4]
+        return tuple(r)
+    return f
+
+
+def _glm_context_one_short(orig):
+    return lambda ctx, s: max(orig(ctx, s) - 1, 0)
+
+
+def _rope_2d_second_half_fixed(orig):
+    def f(x, pk, rd, base, inverse=False):
+        out = orig(x, pk, rd, base, inverse)
+        if pk.pos2 is not None:
+            out = out.copy()
+            out[..., rd:] = x[..., rd:]  # block position ignored
+        return out
+    return f
+
+
 FD = lambda: P.test_finite_difference_gradients(1)  # noqa: E731
 
 # (mistake, oracle attribute, mutant factory, pins that should catch it)
@@ -222,6 +245,12 @@ CASES = [
      [P.test_cross_entropy_matches_torch, P.test_cross_entropy_uniform_closed_form]),
     ("cross-entropy gradient on rows without a target", "cross_entropy", _ce_ignored_rows_keep_gradient,
      [P.test_cross_entropy_matches_torch, P.test_cross_entropy_uniform_closed_form]),
+    ("prefix gradients halved", "attention_bwd", _prefix_grads_halved,
+     [lambda: P.test_finite_difference_prefix_gradients(1)]),
+    ("GLM context one token short", "_ctx", _glm_context_one_short,
+     [lambda: P.test_glm_attention_matches_torch_sdpa(0), P.test_glm_context_is_bidirectional_and_span_causal]),
+    ("2D rotary ignores the block position", "rope_2d", _rope_2d_second_half_fixed,
+     [P.test_rope_2d_properties]),
     ("residual scale alpha ignored", "BlockShape.of", _alpha_ignored,
      [lambda: P.test_zero_weight_block_closed_form(1), lambda: P.test_zero_weight_block_closed_form(0)]),
 ]
