@@ -29,7 +29,10 @@
 //     causal span); positions are two-dimensional (context token t: (t, 0); span token t:
 //     (mask position, t - c + 1)), the second position rotating dims [rotary_dim,
 //     2 rotary_dim) of each head with the same frequencies;
-//   §4.1.4: Adam as AdamW with bias correction (decoupled decay, default 0).
+//   §4.1.4: Adam as AdamW with bias correction (decoupled decay, default 0);
+//   §3.1 client parts (one client's round with the server's blocks left out): bottom =
+//     Embedding + Block_0, top = Block_{N-1} + final LayerNorm + bias-free LM head +
+//     cross-entropy, the mean over the tokens that carry a target (label >= 0).
 // The backward is the exact chain rule of the above.
 #include <omp.h>
 
@@ -424,6 +427,44 @@ void block_bwd(const Block& P, float* const* G, const Saved& sv, const float* dy
     for (size_t i = 0; i < TH; ++i) dx[i] = dx[i] + al * dh[i];
 }
 
+// Positions and rotary tables of a call: segment s = rows [cu[s], cu[s+1]), with GLM
+// context lengths ctx / mask positions mask_pos (null: plain segments; null mask_pos: c - 1).
+// Returns false on a bad argument.
+bool make_positions(const flo_shape& sh, int S, const int32_t* cu, const int32_t* ctx, const int32_t* mask_pos,
+                    Positions& ps) {
+  const int T = cu[S];
+  ps = Positions();
+  ps.glm = ctx != nullptr;
+  ps.pos.resize(T);
+  ps.pos2.assign(T, 0);
+  ps.ctx.assign(S, 0);
+  int max_pos = 0;
+  for (int s = 0; s < S; ++s) {
+    const int L = cu[s + 1] - cu[s];
+    const int c = ctx ? ctx[s] : 0;
+    const int mp = !ctx ? 0 : mask_pos ? mask_pos[s] : c - 1;
+    if (c < 0 || c > L || (c > 0 && (mp < 0 || mp >= c))) return false;
+    ps.ctx[s] = c;
+    for (int t = 0; t < L; ++t) {
+      const bool span = c > 0 && t >= c;
+      ps.pos[cu[s] + t] = span ? mp : t;
+      ps.pos2[cu[s] + t] = span ? t - c + 1 : 0;
+      max_pos = std::max(max_pos, std::max(ps.pos[cu[s] + t], ps.pos2[cu[s] + t]));
+    }
+  }
+  // rotation angles p base^(-2i/rotary_dim), evaluated in double and rounded to fp32
+  const int half = sh.rotary_dim / 2;
+  ps.cs.resize((size_t)(max_pos + 1) * half);
+  ps.sn.resize((size_t)(max_pos + 1) * half);
+  for (int p = 0; p <= max_pos; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double ang = p * std::pow((double)sh.rope_base, -2.0 * i / sh.rotary_dim);
+      ps.cs[(size_t)p * half + i] = (float)std::cos(ang);
+      ps.sn[(size_t)p * half + i] = (float)std::sin(ang);
+    }
+  return true;
+}
+
 }  // namespace
 
 extern "C" {
@@ -457,34 +498,7 @@ int flo_server_fwd_bwd_ext(const flo_shape* shp, int32_t n_blocks, const float* 
   const int T = cu[S], H = sh.hidden;
   if (T < 1) return -1;
   Positions ps;
-  ps.glm = ctx != nullptr;
-  ps.pos.resize(T);
-  ps.pos2.assign(T, 0);
-  ps.ctx.assign(S, 0);
-  int max_pos = 0;
-  for (int s = 0; s < S; ++s) {
-    const int L = cu[s + 1] - cu[s];
-    const int c = ctx ? ctx[s] : 0;
-    const int mp = !ctx ? 0 : mask_pos ? mask_pos[s] : c - 1;
-    if (c < 0 || c > L || (c > 0 && (mp < 0 || mp >= c))) return -1;
-    ps.ctx[s] = c;
-    for (int t = 0; t < L; ++t) {
-      const bool span = c > 0 && t >= c;
-      ps.pos[cu[s] + t] = span ? mp : t;
-      ps.pos2[cu[s] + t] = span ? t - c + 1 : 0;
-      max_pos = std::max(max_pos, std::max(ps.pos[cu[s] + t], ps.pos2[cu[s] + t]));
-    }
-  }
-  // rotation angles p base^(-2i/rotary_dim), evaluated in double and rounded to fp32
-  const int half = sh.rotary_dim / 2;
-  ps.cs.resize((size_t)(max_pos + 1) * half);
-  ps.sn.resize((size_t)(max_pos + 1) * half);
-  for (int p = 0; p <= max_pos; ++p)
-    for (int i = 0; i < half; ++i) {
-      const double ang = p * std::pow((double)sh.rope_base, -2.0 * i / sh.rotary_dim);
-      ps.cs[(size_t)p * half + i] = (float)std::cos(ang);
-      ps.sn[(size_t)p * half + i] = (float)std::sin(ang);
-    }
+  if (!make_positions(sh, S, cu, ctx, mask_pos, ps)) return -1;
   const int Lp = prefix_len;
   auto pre = [&](int b, int i) { return Lp > 0 ? prefixes[2 * b + i] : nullptr; };
   std::vector<Saved> saved(n_blocks);
@@ -514,6 +528,96 @@ int flo_server_fwd_bwd(const flo_shape* shp, int32_t n_blocks, const float* cons
                        int32_t S, const int32_t* cu, const float* x, const float* dy, float* y, float* dx) {
   return flo_server_fwd_bwd_ext(shp, n_blocks, params, grads, S, cu, nullptr, nullptr, 0, nullptr, nullptr, x, dy,
                                 y, dx);
+}
+
+// One client's round of §3.1 with the server's blocks left out (the bottom's output handed
+// straight to the top): tokens / labels int32 [b * L] (b rows of L tokens; a label < 0
+// carries no target); x = Embedding(tokens), h0 = Block_0(x), z = Block_{N-1}(h0),
+// logits = LN_f(z) head^T, loss = the mean over the tokens with a target of
+// -log softmax(logits)[label]; then the chain rule back to the embedding table.
+// Both blocks see the rows as b segments of length L (GLM: ctx / mask_pos [b] as in
+// flo_server_fwd_bwd_ext) and, with prefix_len > 0, their own prefixes (bottom[12..13],
+// top[12..13]).  Parameters: embed [V, H], bottom / top 12 (+ 2) pointers in the server
+// order, lnf_gamma / lnf_beta [H], head [V, H]; their gradients are ADDED into g_embed,
+// g_bottom, g_top (same counts), g_lnf (2 pointers) and g_head.  *loss receives the loss.
+// Returns 0, or -1 on a bad argument (a token outside [0, vocab), a label >= vocab).
+int flo_client_round(const flo_shape* shp, int32_t vocab, int32_t b, int32_t L, const int32_t* tokens,
+                     const int32_t* labels, const int32_t* ctx, const int32_t* mask_pos, int32_t prefix_len,
+                     const float* embed, const float* const* bottom, const float* const* top, const float* lnf_gamma,
+                     const float* lnf_beta, const float* head, float* g_embed, float* const* g_bottom,
+                     float* const* g_top, float* const* g_lnf, float* g_head, float* loss) {
+  if (!shp || vocab < 1 || b < 1 || L < 1 || !tokens || !labels || prefix_len < 0 || !embed || !bottom || !top ||
+      !lnf_gamma || !lnf_beta || !head || !g_embed || !g_bottom || !g_top || !g_lnf || !g_head || !loss)
+    return -1;
+  const flo_shape sh = *shp;
+  if (sh.hidden != sh.n_heads * sh.head_dim || sh.rotary_dim < 2 || sh.rotary_dim % 2 ||
+      sh.rotary_dim > sh.head_dim || (ctx && 2 * sh.rotary_dim != sh.head_dim))
+    return -1;
+  const int S = b, T = b * L, H = sh.hidden, V = vocab, Lp = prefix_len;
+  for (int t = 0; t < T; ++t)
+    if (tokens[t] < 0 || tokens[t] >= V || labels[t] >= V) return -1;
+  std::vector<int32_t> cu(S + 1);
+  for (int s = 0; s <= S; ++s) cu[s] = s * L;
+  Positions ps;
+  if (!make_positions(sh, S, cu.data(), ctx, mask_pos, ps)) return -1;
+  const Block Pb{bottom[0], bottom[1], bottom[2], bottom[3], bottom[4], bottom[5],
+                 bottom[6], bottom[7], bottom[8], bottom[9], bottom[10], bottom[11]};
+  const Block Pt{top[0], top[1], top[2], top[3], top[4], top[5], top[6], top[7], top[8], top[9], top[10], top[11]};
+  const float* bpk = Lp ? bottom[12] : nullptr;
+  const float* bpv = Lp ? bottom[13] : nullptr;
+  const float* tpk = Lp ? top[12] : nullptr;
+  const float* tpv = Lp ? top[13] : nullptr;
+  // forward: embedding rows, the two blocks, final LayerNorm, LM head
+  Vec x((size_t)T * H), h0((size_t)T * H), z((size_t)T * H), zn((size_t)T * H), mu(T), rs(T);
+  for (int t = 0; t < T; ++t)
+    std::memcpy(x.data() + (size_t)t * H, embed + (size_t)tokens[t] * H, sizeof(float) * H);
+  Saved svb, svt;
+  block_fwd(Pb, x.data(), h0.data(), svb, sh, T, S, cu.data(), ps, bpk, bpv, Lp);
+  block_fwd(Pt, h0.data(), z.data(), svt, sh, T, S, cu.data(), ps, tpk, tpv, Lp);
+  layer_norm_fwd(z.data(), lnf_gamma, lnf_beta, sh.ln_eps, zn.data(), mu.data(), rs.data(), T, H);
+  Vec logits((size_t)T * V);
+  matmul_nt(zn.data(), head, nullptr, logits.data(), T, V, H);
+  // cross-entropy over the rows with a target, and its gradient w.r.t. the logits
+  int n = 0;
+  for (int t = 0; t < T; ++t) n += labels[t] >= 0;
+  const float inv_n = 1.f / (float)(n > 0 ? n : 1);
+  Vec row_loss(T, 0.f);
+#pragma omp parallel for schedule(static)
+  for (int t = 0; t < T; ++t) {
+    float* r = logits.data() + (size_t)t * V;
+    if (labels[t] < 0) {
+      for (int v = 0; v < V; ++v) r[v] = 0.f;
+      continue;
+    }
+    float mx = -INFINITY;
+    for (int v = 0; v < V; ++v) mx = std::fmax(mx, r[v]);
+    float l = 0.f;
+    for (int v = 0; v < V; ++v) l += std::exp(r[v] - mx);
+    const float lse = mx + std::log(l);
+    row_loss[t] = lse - r[labels[t]];
+    for (int v = 0; v < V; ++v) r[v] = std::exp(r[v] - lse);
+    r[labels[t]] -= 1.f;
+    for (int v = 0; v < V; ++v) r[v] *= inv_n;
+  }
+  float sum = 0.f;
+  for (int t = 0; t < T; ++t) sum += row_loss[t];
+  *loss = sum * inv_n;
+  // backward: LM head, final LayerNorm, top block, bottom block, embedding rows
+  const float* dlog = logits.data();
+  matmul_tn_acc(dlog, zn.data(), g_head, T, V, H);
+  Vec dzn((size_t)T * H), dz((size_t)T * H), dh0((size_t)T * H), dx((size_t)T * H);
+  matmul_nn(dlog, head, dzn.data(), T, V, H);
+  layer_norm_bwd(dzn.data(), z.data(), mu.data(), rs.data(), lnf_gamma, dz.data(), g_lnf[0], g_lnf[1], T, H);
+  block_bwd(Pt, g_top, svt, dz.data(), dh0.data(), sh, T, S, cu.data(), ps, tpk, tpv, Lp, Lp ? g_top[12] : nullptr,
+            Lp ? g_top[13] : nullptr);
+  block_bwd(Pb, g_bottom, svb, dh0.data(), dx.data(), sh, T, S, cu.data(), ps, bpk, bpv, Lp,
+            Lp ? g_bottom[12] : nullptr, Lp ? g_bottom[13] : nullptr);
+  for (int t = 0; t < T; ++t) {  // rows of repeated tokens accumulate in token order
+    float* g = g_embed + (size_t)tokens[t] * H;
+    const float* d = dx.data() + (size_t)t * H;
+    for (int i = 0; i < H; ++i) g[i] += d[i];
+  }
+  return 0;
 }
 
 // AdamW with bias correction at step t >= 1 (§4.1.4): m = b1 m + (1-b1) g,

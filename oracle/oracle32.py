@@ -36,6 +36,12 @@ def lib():
                                              C.POINTER(C.c_void_p), C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                              C.c_int32, C.POINTER(C.c_void_p), C.POINTER(C.c_void_p), C.c_void_p,
                                              C.c_void_p, C.c_void_p, C.c_void_p]
+        L.flo_client_round.restype = C.c_int
+        L.flo_client_round.argtypes = [C.POINTER(_Shape), C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
+                                       C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.POINTER(C.c_void_p),
+                                       C.POINTER(C.c_void_p), C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                       C.POINTER(C.c_void_p), C.POINTER(C.c_void_p), C.POINTER(C.c_void_p),
+                                       C.c_void_p, C.c_void_p]
         L.flo_adamw.restype = C.c_int
         L.flo_adamw.argtypes = [C.c_int64, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
                                 C.c_float, C.c_float, C.c_float, C.c_float, C.c_float]
@@ -97,6 +103,32 @@ def server_fwd_bwd(cfg, params: Sequence[Sequence[np.ndarray]], grads: List[List
     if rc != 0:
         raise ValueError(f"flo_server_fwd_bwd: bad arguments (rc {rc})")
     return y, dx
+
+
+def client_round(cfg, params: dict, tokens: np.ndarray, labels: np.ndarray, context_lens=None, mask_pos=None):
+    """One client's round of §3.1 with the server's blocks left out: tokens / labels int32
+    [b, L]; params as synthetic.init_client (parts bottom, top, embed, head, final_ln).
+    Returns (loss, grads) with grads a dict of fp32 arrays shaped like params."""
+    ps = {k: [_f32(p) for p in v] for k, v in params.items()}
+    gs = {k: [np.zeros(p.shape, np.float32) for p in v] for k, v in ps.items()}
+    tok = np.ascontiguousarray(tokens, np.int32)
+    lab = np.ascontiguousarray(labels, np.int32)
+    b, L = tok.shape
+    nblk = len(ps["bottom"])
+    arr = lambda xs: (C.c_void_p * len(xs))(*[x.ctypes.data for x in xs])  # noqa: E731
+    ctx = None if context_lens is None else np.ascontiguousarray(context_lens, np.int32)
+    mp = None if mask_pos is None else np.ascontiguousarray(mask_pos, np.int32)
+    loss = np.zeros(1, np.float32)
+    sh = shape_of(cfg)
+    rc = lib().flo_client_round(C.byref(sh), cfg.vocab, b, L, tok.ctypes.data, lab.ctypes.data,
+                                None if ctx is None else ctx.ctypes.data, None if mp is None else mp.ctypes.data,
+                                cfg.prefix_len if nblk > 12 else 0, ps["embed"][0].ctypes.data, arr(ps["bottom"]),
+                                arr(ps["top"]), ps["final_ln"][0].ctypes.data, ps["final_ln"][1].ctypes.data,
+                                ps["head"][0].ctypes.data, gs["embed"][0].ctypes.data, arr(gs["bottom"]),
+                                arr(gs["top"]), arr(gs["final_ln"]), gs["head"][0].ctypes.data, loss.ctypes.data)
+    if rc != 0:
+        raise ValueError(f"flo_client_round: bad arguments (rc {rc})")
+    return float(loss[0]), gs
 
 
 def adamw(w: np.ndarray, g: np.ndarray, m: np.ndarray, v: np.ndarray, t: int, lr: float, beta1: float,

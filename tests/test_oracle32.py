@@ -219,3 +219,42 @@ def test_glm_and_prefix_bad_arguments():
     for ctx, mp in (([5], [0]), ([3], [3]), ([-1], [0])):   # context past the segment, [M] outside it, negative
         with pytest.raises(ValueError):
             O32.server_fwd_bwd(cfg, params, g, [0, 4], x, x, ctx, mp)
+
+
+@pytest.mark.parametrize("Lp,glm", [(0, False), (2, True)], ids=["plain", "prefix_glm"])
+def test_client_round_matches_fp64_oracle(Lp, glm):
+    """§3.1 client parts in fp32 (Embedding + Block_0, Block_{N-1} + final LayerNorm + LM
+    head + cross-entropy; the server's blocks left out): the loss and every client
+    parameter's gradient within fp32 rounding of the fp64 oracle client, with repeated
+    tokens, rows without a target, and optionally GLM segments with P-tuning prefixes."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=1, client_batch=2, seq_lens=(9,), vocab=37, prefix_len=Lp)
+    params = syn.init_client(cfg)
+    rng = np.random.default_rng(50 + Lp)
+    tok = rng.integers(0, cfg.vocab, size=(2, 9)).astype(np.int32)
+    lab = rng.integers(0, cfg.vocab, size=(2, 9)).astype(np.int32)
+    lab[0, :4] = -1
+    ctx, mp = ([5, 3], [2, 0]) if glm else (None, None)
+    loss32, g32 = O32.client_round(cfg, params, tok, lab, ctx, mp)
+    c = O.OracleClient(cfg, params)
+    h0 = c.bottom_forward(tok, ctx, mp)
+    loss, gh = c.top_forward_backward(h0, lab)
+    c.bottom_backward(gh)
+    assert abs(loss32 - loss) <= 1e-6 * abs(loss)
+    for k in O.CLIENT_PARTS:
+        for i, (a, b) in enumerate(zip(g32[k], c.grads[k])):
+            assert _rel(a, b) < 1e-5, (k, i)
+
+
+def test_client_round_no_target_and_bad_ids():
+    """No target at all: zero loss and zero gradients; a token id outside the vocabulary or a
+    label >= vocab is refused."""
+    cfg = syn.CONFIGS["tiny"].with_(n_blocks=1, client_batch=1, seq_lens=(4,), vocab=11)
+    params = syn.init_client(cfg)
+    tok = np.array([[1, 2, 3, 1]], np.int32)
+    loss, g = O32.client_round(cfg, params, tok, np.full((1, 4), -1, np.int32))
+    assert loss == 0.0
+    assert all(not a.any() for v in g.values() for a in v)
+    with pytest.raises(ValueError):
+        O32.client_round(cfg, params, np.array([[1, 2, 11, 0]], np.int32), np.zeros((1, 4), np.int32))
+    with pytest.raises(ValueError):
+        O32.client_round(cfg, params, tok, np.array([[0, 11, 0, 0]], np.int32))
